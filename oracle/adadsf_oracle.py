@@ -1,0 +1,306 @@
+"""AdaDSF depth-sparse forward: plain fp64 CPU oracle.
+
+TEST INFRASTRUCTURE ONLY. Only the test suite, the smoke check of the build
+entry and the benchmark's CPU-baseline leg may import this module; the product
+path never calls it and shares no code with it.
+
+Every function is the plain definition of one step of the paper's method, in
+float64 NumPy, with no blocking, fusion or reordering beyond what the definition
+states. Matrix products (``@``), ``np.lexsort`` and ``scipy.special.erf`` serve as
+library primitives.
+
+Sources (paper "Adaptive Depth Sparse Framework", AdaDSF):
+  * Sec. 3.1, Eq. 1   scaled dot-product attention softmax(QK^T/sqrt(d_k))V
+  * Sec. 3.1, Eq. 2   FFN W2 sigma(W1 x + b1) + b2
+  * Sec. 3.1, Eq. 3   a decoder layer composes attention and FFN with a
+                      residual; the concrete (pre-norm) layer forms are those of
+                      the GPT-NeoX and Qwen2.5 backbones the paper evaluates
+                      (Sec. 4.1, "Models")
+  * Sec. 3.3, Eq. 4   s_i = cosine similarity of layer input and output
+  * Sec. 3.3, Eqs. 5-8  similarity -> layer-wise retention ratio r_i
+  * Sec. 3.4          router scores, Top-K_i with K_i = floor(r_i * s), binary
+                      mask, unselected tokens bypass through the residual path
+
+Readings where the paper is silent (each one is listed in the design notes):
+  * router = Linear(d, h) -> SiLU -> Linear(h, 1) on the raw residual stream;
+  * kept tokens attend causally to kept tokens only, with rotary positions
+    taken from their original token index;
+  * Top-K ties go to the lower position; -0.0 equals +0.0; NaN ranks below -inf;
+  * Eq. 8 can give r_i > 1; the default clamps to 1 and re-spreads the excess
+    over the other layers in proportion to r'_i (``raw=True`` skips this);
+  * K_i = floor(r_i * T + 1e-9), clamped to [0, T];
+  * the similarity statistic is the mean over tokens of the per-token cosine
+    (``mode="flat"``: cosine of the flattened tensors);
+  * NeoX layer: x + Attn(LN1 x) + MLP(LN2 x); Qwen layer: h = x + Attn(RMS1 x),
+    h + MLP(RMS2 h). The layer's residual delta is written to kept rows only.
+"""
+from __future__ import annotations
+
+import numpy as np
+from scipy.special import erf
+
+NEOX = 0
+QWEN = 1
+
+
+# --------------------------------------------------------------------------
+# elementwise pieces
+# --------------------------------------------------------------------------
+def silu(x):
+    """SiLU(x) = x * sigmoid(x)."""
+    return x / (1.0 + np.exp(-x))
+
+
+def gelu(x):
+    """Exact GELU, x * Phi(x), with Phi the standard normal CDF."""
+    return 0.5 * x * (1.0 + erf(x / np.sqrt(2.0)))
+
+
+def layer_norm(x, g, b, eps):
+    """LayerNorm over the last axis: biased variance, affine gain and bias."""
+    mu = x.mean(axis=-1, keepdims=True)
+    var = ((x - mu) ** 2).mean(axis=-1, keepdims=True)
+    return (x - mu) / np.sqrt(var + eps) * g + b
+
+
+def rms_norm(x, g, eps):
+    """RMSNorm over the last axis: x / sqrt(mean(x^2) + eps) * g."""
+    return x / np.sqrt((x * x).mean(axis=-1, keepdims=True) + eps) * g
+
+
+def rope(v, pos, rotary_dim, theta):
+    """Rotary embedding ("rotate half" convention) of the first ``rotary_dim``
+    features of each row of v (n, head_dim) at integer positions pos (n,).
+    Feature i < rotary_dim/2 pairs with i + rotary_dim/2 and both turn by the
+    angle pos * theta^(-2i/rotary_dim)."""
+    half = rotary_dim // 2
+    inv = theta ** (-(np.arange(half, dtype=np.float64) * 2.0) / rotary_dim)
+    ang = np.asarray(pos, dtype=np.float64)[:, None] * inv[None, :]
+    c, s = np.cos(ang), np.sin(ang)
+    out = np.array(v, dtype=np.float64, copy=True)
+    a = v[:, :half]
+    b = v[:, half:rotary_dim]
+    out[:, :half] = a * c - b * s
+    out[:, half:rotary_dim] = b * c + a * s
+    return out
+
+
+# --------------------------------------------------------------------------
+# Eq. 1 -- attention among the given rows, causal in row order
+# --------------------------------------------------------------------------
+def causal_attention(q, k, v, n_heads, n_kv_heads, head_dim):
+    """softmax(Q K^T / sqrt(d_k)) V per head (Eq. 1); row i sees rows j <= i.
+    q (n, n_heads*hd), k and v (n, n_kv_heads*hd); query head h reads
+    key/value head h // (n_heads / n_kv_heads)."""
+    n = q.shape[0]
+    out = np.zeros((n, n_heads * head_dim), dtype=np.float64)
+    if n == 0:
+        return out
+    group = n_heads // n_kv_heads
+    allowed = np.tril(np.ones((n, n), dtype=bool))
+    for h in range(n_heads):
+        g = h // group
+        qh = q[:, h * head_dim:(h + 1) * head_dim]
+        kh = k[:, g * head_dim:(g + 1) * head_dim]
+        vh = v[:, g * head_dim:(g + 1) * head_dim]
+        s = (qh @ kh.T) / np.sqrt(head_dim)
+        s = np.where(allowed, s, -np.inf)
+        s = s - s.max(axis=1, keepdims=True)
+        p = np.exp(s)
+        p = p / p.sum(axis=1, keepdims=True)
+        out[:, h * head_dim:(h + 1) * head_dim] = p @ vh
+    return out
+
+
+# --------------------------------------------------------------------------
+# Transformer layer on a packed set of tokens (Eqs. 1-3 in the backbone forms)
+# --------------------------------------------------------------------------
+def _attention_branch(a, pos, W, p):
+    hd, H, Hkv = p["head_dim"], p["n_heads"], p["n_kv_heads"]
+    qd, kvd = H * hd, Hkv * hd
+    qkv = a @ W["w_qkv"].T + W["b_qkv"]
+    q, k, v = qkv[:, :qd], qkv[:, qd:qd + kvd], qkv[:, qd + kvd:qd + 2 * kvd]
+    q = np.concatenate([rope(q[:, h * hd:(h + 1) * hd], pos, p["rotary_dim"], p["rope_theta"])
+                        for h in range(H)], axis=1) if len(pos) else q
+    k = np.concatenate([rope(k[:, h * hd:(h + 1) * hd], pos, p["rotary_dim"], p["rope_theta"])
+                        for h in range(Hkv)], axis=1) if len(pos) else k
+    o = causal_attention(q, k, v, H, Hkv, hd)
+    out = o @ W["w_o"].T
+    if "b_o" in W:
+        out = out + W["b_o"]
+    return out
+
+
+def block_delta(xp, pos, W, p):
+    """Residual delta of one decoder layer applied to the packed rows xp (n, d)
+    at original positions pos (n,): layer(xp) - xp."""
+    eps = p["norm_eps"]
+    if p["arch"] == NEOX:
+        attn = _attention_branch(layer_norm(xp, W["ln1_w"], W["ln1_b"], eps), pos, W, p)
+        m = layer_norm(xp, W["ln2_w"], W["ln2_b"], eps)
+        mlp = gelu(m @ W["w_up"].T + W["b_up"]) @ W["w_down"].T + W["b_down"]
+        return attn + mlp
+    attn = _attention_branch(rms_norm(xp, W["ln1_w"], eps), pos, W, p)
+    h = xp + attn
+    m = rms_norm(h, W["ln2_w"], eps)
+    mlp = (silu(m @ W["w_gate"].T) * (m @ W["w_up"].T)) @ W["w_down"].T
+    return (h + mlp) - xp
+
+
+# --------------------------------------------------------------------------
+# Sec. 3.4 -- router and Top-K
+# --------------------------------------------------------------------------
+def router_scores(x, W):
+    """Per-token importance score of the lightweight MLP router (Sec. 3.4):
+    w2 . SiLU(W1 x + b1) + b2, for x (..., d)."""
+    hdn = silu(x @ W["router_w1"].T + W["router_b1"])
+    return hdn @ W["router_w2"] + W["router_b2"][0]
+
+
+def topk_keep(scores, K):
+    """Positions of the Top-K scores of one sequence (Sec. 3.4), ascending.
+    Order: higher score first, equal scores by lower position; NaN ranks below
+    every number; -0.0 and +0.0 compare equal."""
+    scores = np.asarray(scores, dtype=np.float64)
+    T = scores.shape[0]
+    K = int(K)
+    if K <= 0:
+        return np.zeros(0, dtype=np.int64)
+    nan = np.isnan(scores)
+    key = np.where(nan, 0.0, scores)
+    # lexsort: last key is primary
+    order = np.lexsort((np.arange(T), -key, nan.astype(np.int8)))
+    return np.sort(order[:K]).astype(np.int64)
+
+
+# --------------------------------------------------------------------------
+# Sec. 3.4 -- one sparse layer
+# --------------------------------------------------------------------------
+def sparse_layer_forward(x, W, p, K, idx=None):
+    """Depth-sparse layer (Sec. 3.4) on x (B, T, d).
+
+    Scores every token with the router, keeps the Top-K of each sequence
+    (or the given ``idx`` (B, K)), runs the layer on the kept tokens only and
+    adds its residual delta to those rows; every other row is copied unchanged.
+    Returns (x_out, idx (B, K), scores (B, T))."""
+    x = np.asarray(x, dtype=np.float64)
+    B, T, d = x.shape
+    scores = router_scores(x, W)
+    if idx is None:
+        idx = np.stack([topk_keep(scores[b], K) for b in range(B)]) if B else np.zeros((0, K), np.int64)
+    idx = np.asarray(idx, dtype=np.int64).reshape(B, -1)
+    out = x.copy()
+    for b in range(B):
+        sel = idx[b]
+        if sel.size == 0:
+            continue
+        xp = x[b, sel]
+        out[b, sel] = xp + block_delta(xp, sel, W, p)
+    return out, idx, scores
+
+
+# --------------------------------------------------------------------------
+# Sec. 3.3, Eq. 4 -- similarity statistic
+# --------------------------------------------------------------------------
+COS_EPS = 1e-8
+
+
+def cos_sim_stat(x_in, x_out, mode="token"):
+    """Eq. 4 accumulated over a batch. Returns the additive partial sums:
+    mode "token": (sum over rows of cos(x_in_row, x_out_row), number of rows),
+                  cos = a.b / (max(|a|, eps) * max(|b|, eps));
+    mode "flat":  (sum a.b, sum |a|^2, sum |b|^2) over all rows."""
+    a = np.asarray(x_in, dtype=np.float64).reshape(-1, np.shape(x_in)[-1])
+    b = np.asarray(x_out, dtype=np.float64).reshape(-1, np.shape(x_out)[-1])
+    dot = (a * b).sum(axis=1)
+    na2 = (a * a).sum(axis=1)
+    nb2 = (b * b).sum(axis=1)
+    if mode == "token":
+        cos = dot / (np.maximum(np.sqrt(na2), COS_EPS) * np.maximum(np.sqrt(nb2), COS_EPS))
+        return float(cos.sum()), float(a.shape[0])
+    return float(dot.sum()), float(na2.sum()), float(nb2.sum())
+
+
+def similarity(acc, mode="token"):
+    """s_i from the accumulated partial sums of ``cos_sim_stat``."""
+    if mode == "token":
+        return acc[0] / acc[1]
+    return acc[0] / (max(np.sqrt(acc[1]), COS_EPS) * max(np.sqrt(acc[2]), COS_EPS))
+
+
+# --------------------------------------------------------------------------
+# Sec. 3.3, Eqs. 5-8 -- retention allocation
+# --------------------------------------------------------------------------
+def allocate_ratios(s, t, tau=0.05, beta=10.0, raw=False):
+    """Layer-wise retention ratios from the similarity vector s (length L).
+
+    Eq. 5: w~_i = exp((s_i - max s)/tau), w = w~ / sum w~
+    Eq. 6: z_i = beta * (mean(w) - w_i)
+    Eq. 7: r'_i = 0.05 + 0.9 * sigmoid(z_i)
+    Eq. 8: r_i = t L r'_i / sum_j r'_j
+    Unless ``raw``, ratios above 1 are clamped to 1 and the remaining budget
+    t L - (#clamped) is spread over the other layers in proportion to r'_i,
+    repeated until no ratio exceeds 1 (t >= 1 gives all ones)."""
+    s = np.asarray(s, dtype=np.float64)
+    L = s.shape[0]
+    wt = np.exp((s - s.max()) / tau)
+    w = wt / wt.sum()
+    z = beta * (w.mean() - w)
+    rp = 0.05 + 0.9 / (1.0 + np.exp(-z))
+    r = t * L / rp.sum() * rp
+    if raw:
+        return r, rp
+    if t >= 1.0:
+        return np.ones(L), rp
+    fixed = np.zeros(L, dtype=bool)
+    while True:
+        over = (~fixed) & (r > 1.0)
+        if not over.any():
+            break
+        fixed |= over
+        budget = t * L - fixed.sum()
+        r = np.where(fixed, 1.0, budget / rp[~fixed].sum() * rp)
+    return r, rp
+
+
+def kept_counts(r, T, rounding="floor"):
+    """K_i = floor(r_i * T) (Sec. 3.4), with a 1e-9 guard against ratios that
+    land a hair below an integer; ``rounding="round"`` rounds to nearest."""
+    r = np.asarray(r, dtype=np.float64)
+    if rounding == "floor":
+        K = np.floor(r * T + 1e-9)
+    else:
+        K = np.floor(r * T + 0.5)
+    return np.clip(K, 0, T).astype(np.int64)
+
+
+# --------------------------------------------------------------------------
+# whole model: embedding -> L sparse layers -> final norm
+# --------------------------------------------------------------------------
+def final_norm(x, Wm, p):
+    if p["arch"] == NEOX:
+        return layer_norm(x, Wm["final_w"], Wm["final_b"], p["norm_eps"])
+    return rms_norm(x, Wm["final_w"], p["norm_eps"])
+
+
+def sparse_model_forward(ids, Wm, layers, p, K, idx_force=None, stats_mode=None):
+    """Embedding lookup, then each layer l as a sparse layer with K[l] kept
+    tokens per sequence (or the kept sets idx_force[l]), then the final norm.
+    With ``stats_mode`` the Eq. 4 partial sums of every layer's input/output
+    pair are returned too. Returns (hidden, [idx_l], [stats_l])."""
+    x = np.asarray(Wm["embed"], dtype=np.float64)[np.asarray(ids)]
+    kept, stats = [], []
+    for l, W in enumerate(layers):
+        x_new, idx, _ = sparse_layer_forward(x, W, p, K[l], None if idx_force is None else idx_force[l])
+        if stats_mode is not None:
+            stats.append(cos_sim_stat(x, x_new, stats_mode))
+        kept.append(idx)
+        x = x_new
+    return final_norm(x, Wm, p), kept, stats
+
+
+def params_of(shape):
+    """Plain dict of the backbone hyper-parameters the functions above read."""
+    return {k: getattr(shape, k) for k in
+            ("arch", "d", "n_heads", "n_kv_heads", "head_dim", "ffn", "rotary_dim",
+             "rope_theta", "norm_eps")}

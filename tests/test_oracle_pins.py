@@ -1,0 +1,412 @@
+"""Pins of the fp64 oracle against facts that do not come from the oracle itself:
+library routines it must agree with on special cases, closed forms, limits,
+invariants the paper states or the mathematics fixes, and brute force.
+
+Each group below names the passage of the paper it pins."""
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as F
+from scipy.spatial.distance import cosine as scipy_cosine_distance
+
+from oracle import adadsf_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _paper_constants():
+    vals = {}
+    with open(os.path.join(GOLDEN, "paper_constants.txt")) as f:
+        for line in f:
+            line = line.split("#")[0].strip()
+            if line:
+                k, v = line.split()
+                vals.setdefault(k, []).append(float(v))
+    return vals
+
+
+PC = _paper_constants()
+BETA = PC["beta"][0]
+TAUS = PC["tau"]
+
+
+def rng(seed=0):
+    return np.random.default_rng(seed)
+
+
+# ---------------------------------------------------------------- Eqs. 5-8
+class TestAllocation:
+    def test_budget_eq8(self):
+        """Eq. 8 rescales so that sum r = t L."""
+        g = rng(1)
+        for L in (1, 2, 5, 12, 28):
+            s = g.uniform(0.3, 1.0, L)
+            for t in (0.25, 0.5, 0.9):
+                r, _ = O.allocate_ratios(s, t, 0.05, BETA, raw=True)
+                assert r.sum() == pytest.approx(t * L, rel=1e-12)
+
+    def test_ratio_bounds_eq7(self):
+        """Eq. 7 maps into (floor, floor + span) = (0.05, 0.95)."""
+        lo, span = PC["ratio_floor"][0], PC["ratio_span"][0]
+        g = rng(2)
+        for _ in range(50):
+            s = g.uniform(-1, 1, 16)
+            _, rp = O.allocate_ratios(s, 0.5, 0.01, BETA, raw=True)
+            assert (rp > lo).all() and (rp < lo + span).all()
+
+    def test_uniform_similarity_gives_uniform_ratio(self):
+        """Equal s_i: w = 1/L, z = 0, r' = 0.05 + 0.45 = 0.5, r = t."""
+        for L in (1, 3, 12):
+            r, rp = O.allocate_ratios(np.full(L, 0.7), 0.6, 0.05, BETA)
+            assert np.allclose(rp, 0.5, rtol=0, atol=1e-15)
+            assert np.allclose(r, 0.6, rtol=1e-14)
+
+    def test_two_layer_closed_form(self):
+        """L = 2: mean(w) = 1/2 so z_2 = -z_1 and r'_1 + r'_2 = 0.1 + 0.9 = 1;
+        hence r_i = 2 t r'_i, with r'_1 = 0.05 + 0.9 sig(beta (1/2 - sig((s1 - s2)/tau)))."""
+        g = rng(3)
+        for _ in range(20):
+            s = g.uniform(0, 1, 2)
+            tau = g.choice(TAUS)
+            t = g.uniform(0.1, 0.5)
+            r, rp = O.allocate_ratios(s, t, tau, BETA, raw=True)
+            assert rp.sum() == pytest.approx(1.0, abs=1e-14)
+            sig = lambda v: 1.0 / (1.0 + math.exp(-v))
+            w1 = sig((s[0] - s[1]) / tau)
+            rp1 = 0.05 + 0.9 * sig(BETA * (0.5 - w1))
+            assert rp[0] == pytest.approx(rp1, rel=1e-13)
+            assert r == pytest.approx(2 * t * rp, rel=1e-13)
+
+    def test_worked_example(self):
+        """Values worked out by hand from Eqs. 5-8 (tau = 0.05, beta = 10, t = 0.5),
+        quoted to 4 decimals; the paper prints no numeric example."""
+        r, rp = O.allocate_ratios([0.9, 0.95, 0.99, 0.8], 0.5, 0.05, BETA, raw=True)
+        assert np.round(rp, 4) == pytest.approx([0.7845, 0.4452, 0.0737, 0.8726], abs=1e-4)
+        assert np.round(r, 4) == pytest.approx([0.7210, 0.4092, 0.0678, 0.8020], abs=1e-4)
+        r, _ = O.allocate_ratios([0.1, 0.2, 0.3, 0.99], 0.5, 0.05, BETA, raw=True)
+        assert np.round(r, 4) == pytest.approx([0.6542, 0.6542, 0.6542, 0.0375], abs=1e-4)
+        r, _ = O.allocate_ratios([0.9, 0.95, 0.99, 0.8], 1.0, 0.05, BETA, raw=True)
+        assert np.round(r, 4) == pytest.approx([1.4421, 0.8184, 0.1355, 1.6040], abs=1e-4)
+
+    def test_one_hot_limit(self):
+        """tau -> 0 with a unique maximum: w = e_max, z_max = beta (1/L - 1),
+        z_other = beta / L (closed form)."""
+        L = 4
+        _, rp = O.allocate_ratios([0.1, 0.2, 0.3, 0.99], 0.5, 1e-4, BETA, raw=True)
+        sig = lambda v: 1.0 / (1.0 + math.exp(-v))
+        assert rp[3] == pytest.approx(0.05 + 0.9 * sig(BETA * (1 / L - 1)), rel=1e-12)
+        assert rp[:3] == pytest.approx([0.05 + 0.9 * sig(BETA / L)] * 3, rel=1e-12)
+
+    def test_high_temperature_limit(self):
+        """tau -> infinity: weights become uniform, so r -> t."""
+        r, _ = O.allocate_ratios([0.1, 0.5, 0.9, 0.3], 0.4, 1e9, BETA, raw=True)
+        assert r == pytest.approx([0.4] * 4, rel=1e-7)
+
+    def test_shift_invariance(self):
+        """Eq. 5 subtracts max(s): s + c gives the same ratios."""
+        g = rng(4)
+        s = g.uniform(0.5, 1.0, 12)
+        a, _ = O.allocate_ratios(s, 0.5, 0.05, BETA, raw=True)
+        b, _ = O.allocate_ratios(s + 3.25, 0.5, 0.05, BETA, raw=True)
+        assert np.allclose(a, b, rtol=1e-12)
+
+    def test_more_similar_layer_gets_less_compute(self):
+        """Sec. 3.3: layers with larger transformation (smaller s) receive more
+        compute; so s_i > s_j implies r_i < r_j."""
+        g = rng(5)
+        s = g.permutation(np.linspace(0.6, 0.99, 10))
+        r, _ = O.allocate_ratios(s, 0.5, 0.05, BETA, raw=True)
+        order = np.argsort(s)
+        assert (np.diff(r[order]) < 0).all()
+
+    def test_smaller_tau_larger_variance(self):
+        """Sec. 4.3 (Table 3 discussion): smaller tau yields a larger variance
+        of the retention ratios."""
+        s = np.array([0.80, 0.86, 0.90, 0.93, 0.95, 0.97, 0.98, 0.99])
+        var = [np.var(O.allocate_ratios(s, 0.5, tau, BETA, raw=True)[0]) for tau in sorted(TAUS, reverse=True)]
+        assert var[0] < var[1] < var[2]
+
+    def test_clamp_redistributes(self):
+        """Reading for r_i > 1: clamp to 1 and re-spread the budget in
+        proportion to r'; the budget t L is kept and order is preserved."""
+        s = [0.9, 0.95, 0.99, 0.8]
+        r, rp = O.allocate_ratios(s, 0.75, 0.05, BETA)
+        assert r.sum() == pytest.approx(3.0, rel=1e-12)
+        assert (r <= 1.0).all()
+        assert r[0] == 1.0 and r[3] == 1.0
+        assert r[1] / r[2] == pytest.approx(rp[1] / rp[2], rel=1e-12)
+        r, _ = O.allocate_ratios(s, 1.0, 0.05, BETA)
+        assert (r == 1.0).all()
+
+    def test_kept_counts_floor(self):
+        """K_i = floor(r_i * s) (Sec. 3.4)."""
+        assert O.kept_counts([0.5, 0.25, 0.999, 1.0, 0.0], 512).tolist() == [256, 128, 511, 512, 0]
+        r = np.full(12, 0.5)
+        r = 0.5 * 12 / r.sum() * r          # ratios that may land a hair below 0.5
+        assert (O.kept_counts(r, 512) == 256).all()
+
+
+# ---------------------------------------------------------------- Sec. 3.4 Top-K
+def _brute_topk(scores, K):
+    """Kept iff fewer than K tokens rank ahead of it (O(T^2) definition)."""
+    T = len(scores)
+
+    def ahead(u, t):
+        su, st = scores[u], scores[t]
+        nu, nt = math.isnan(su), math.isnan(st)
+        if nu and nt:
+            return u < t
+        if nu != nt:
+            return nt          # a number is ahead of NaN
+        if su != st:
+            return su > st
+        return u < t
+
+    return [t for t in range(T) if sum(ahead(u, t) for u in range(T) if u != t) < K]
+
+
+class TestTopK:
+    def test_hand_built_ties(self):
+        """Ties -> lower position; -0.0 == +0.0; NaN below everything."""
+        s = [1.0, 3.0, 3.0, 2.0, 3.0, -0.0, 0.0, float("nan")]
+        expect = {0: [], 1: [1], 3: [1, 2, 4], 5: [0, 1, 2, 3, 4], 6: [0, 1, 2, 3, 4, 5],
+                  7: [0, 1, 2, 3, 4, 5, 6], 8: list(range(8))}
+        for K, e in expect.items():
+            assert O.topk_keep(s, K).tolist() == e
+
+    def test_brute_force(self):
+        g = rng(6)
+        for trial in range(60):
+            T = int(g.integers(1, 40))
+            s = g.normal(size=T)
+            if trial % 3 == 0:
+                s = np.round(s, 1)                     # many ties
+            if trial % 5 == 0:
+                s[g.integers(0, T, 3)] = np.nan
+            if trial % 7 == 0:
+                s[g.integers(0, T, 2)] = -np.inf
+            K = int(g.integers(0, T + 1))
+            assert O.topk_keep(s, K).tolist() == _brute_topk(list(s), K)
+
+
+# ---------------------------------------------------------------- Eq. 4
+class TestCosSim:
+    def test_special_cases(self):
+        g = rng(7)
+        x = g.normal(size=(5, 33))
+        assert O.similarity(O.cos_sim_stat(x, x)) == pytest.approx(1.0, abs=1e-15)
+        assert O.similarity(O.cos_sim_stat(x, -x)) == pytest.approx(-1.0, abs=1e-15)
+        assert O.similarity(O.cos_sim_stat(x, 2.5 * x)) == pytest.approx(1.0, abs=1e-15)
+        a = np.zeros((2, 4)); a[:, 0] = 1
+        b = np.zeros((2, 4)); b[:, 1] = 3
+        assert O.similarity(O.cos_sim_stat(a, b)) == 0.0
+        assert O.similarity(O.cos_sim_stat(x, x, "flat"), "flat") == pytest.approx(1.0, abs=1e-15)
+
+    def test_matches_scipy(self):
+        g = rng(8)
+        a, b = g.normal(size=(7, 20)), g.normal(size=(7, 20))
+        tot, n = O.cos_sim_stat(a, b)
+        ref = sum(1.0 - scipy_cosine_distance(a[i], b[i]) for i in range(7))
+        assert n == 7 and tot == pytest.approx(ref, rel=1e-13)
+        d, na, nb = O.cos_sim_stat(a, b, "flat")
+        assert O.similarity((d, na, nb), "flat") == pytest.approx(
+            1.0 - scipy_cosine_distance(a.ravel(), b.ravel()), rel=1e-13)
+
+
+# ---------------------------------------------------------------- Eqs. 1-3 building blocks
+T64 = torch.float64
+
+
+class TestPieces:
+    def test_gelu_silu(self):
+        x = np.linspace(-6, 6, 101)
+        assert O.gelu(x) == pytest.approx(F.gelu(torch.tensor(x, dtype=T64)).numpy(), rel=1e-13, abs=1e-15)
+        assert O.silu(x) == pytest.approx(F.silu(torch.tensor(x, dtype=T64)).numpy(), rel=1e-13, abs=1e-15)
+        assert O.gelu(np.array([1.0]))[0] == pytest.approx(0.8413447460685429, rel=1e-15)  # Phi(1)
+
+    def test_norms(self):
+        g = rng(9)
+        x, w, b = g.normal(size=(6, 40)), g.normal(size=40), g.normal(size=40)
+        ref = F.layer_norm(torch.tensor(x), (40,), torch.tensor(w), torch.tensor(b), 1e-5).numpy()
+        assert O.layer_norm(x, w, b, 1e-5) == pytest.approx(ref, rel=1e-12, abs=1e-13)
+        y = O.rms_norm(x, np.ones(40), 0.0)
+        assert np.sqrt((y * y).mean(axis=1)) == pytest.approx(np.ones(6), rel=1e-13)
+        if hasattr(F, "rms_norm"):
+            ref = F.rms_norm(torch.tensor(x), (40,), torch.tensor(w), 1e-6).numpy()
+            assert O.rms_norm(x, w, 1e-6) == pytest.approx(ref, rel=1e-12, abs=1e-13)
+
+    def test_rope_complex_form(self):
+        """Rotate-half RoPE = multiplying (a_i + i b_i) by exp(i pos theta^(-2i/r))."""
+        g = rng(10)
+        hd, rot, theta = 16, 8, 1e4
+        v = g.normal(size=(5, hd))
+        pos = np.array([0, 1, 7, 100, 4095])
+        out = O.rope(v, pos, rot, theta)
+        half = rot // 2
+        for n in range(5):
+            for i in range(half):
+                z = complex(v[n, i], v[n, i + half]) * np.exp(1j * pos[n] * theta ** (-2 * i / rot))
+                assert out[n, i] == pytest.approx(z.real, abs=1e-12)
+                assert out[n, i + half] == pytest.approx(z.imag, abs=1e-12)
+        assert out[:, rot:] == pytest.approx(v[:, rot:], abs=0)
+        assert out[0] == pytest.approx(v[0], abs=1e-15)          # position 0 is the identity
+
+    def test_rope_relative(self):
+        """q.k after RoPE depends on the position difference only."""
+        g = rng(11)
+        q, k = g.normal(size=(1, 32)), g.normal(size=(1, 32))
+        a = O.rope(q, [9], 32, 1e6) @ O.rope(k, [3], 32, 1e6).T
+        b = O.rope(q, [1009], 32, 1e6) @ O.rope(k, [1003], 32, 1e6).T
+        assert a == pytest.approx(b, rel=1e-10)
+
+    @pytest.mark.parametrize("H,Hkv", [(4, 4), (6, 2)])
+    def test_attention_vs_sdpa(self, H, Hkv):
+        g = rng(12)
+        n, hd = 9, 16
+        q, k, v = g.normal(size=(n, H * hd)), g.normal(size=(n, Hkv * hd)), g.normal(size=(n, Hkv * hd))
+        out = O.causal_attention(q, k, v, H, Hkv, hd)
+        tq = torch.tensor(q).view(n, H, hd).transpose(0, 1)
+        tk = torch.tensor(k).view(n, Hkv, hd).transpose(0, 1).repeat_interleave(H // Hkv, 0)
+        tv = torch.tensor(v).view(n, Hkv, hd).transpose(0, 1).repeat_interleave(H // Hkv, 0)
+        ref = F.scaled_dot_product_attention(tq, tk, tv, is_causal=True).transpose(0, 1).reshape(n, H * hd)
+        assert out == pytest.approx(ref.numpy(), rel=1e-12, abs=1e-13)
+
+    def test_attention_special_cases(self):
+        g = rng(13)
+        v = g.normal(size=(6, 8))
+        k = np.tile(g.normal(size=(1, 8)), (6, 1))          # identical keys
+        out = O.causal_attention(g.normal(size=(6, 8)), k, v, 1, 1, 8)
+        for i in range(6):                                   # uniform mean of the prefix
+            assert out[i] == pytest.approx(v[:i + 1].mean(axis=0), rel=1e-12)
+        one = O.causal_attention(g.normal(size=(1, 8)), g.normal(size=(1, 8)), v[:1], 1, 1, 8)
+        assert one == pytest.approx(v[:1], rel=1e-15)         # softmax of one score
+
+
+# ---------------------------------------------------------------- Sec. 3.4 layer
+def _params(arch, d=32, H=4, Hkv=4, hd=8, F_=48, rot=4, theta=1e4):
+    return {"arch": arch, "d": d, "n_heads": H, "n_kv_heads": Hkv, "head_dim": hd, "ffn": F_,
+            "rotary_dim": rot, "rope_theta": theta, "norm_eps": 1e-5}
+
+
+def _weights(p, seed, rh=8, zero=()):
+    g = rng(seed)
+    d, q, kv, F_ = p["d"], p["n_heads"] * p["head_dim"], p["n_kv_heads"] * p["head_dim"], p["ffn"]
+    W = {"router_w1": g.normal(0, 0.3, (rh, d)), "router_b1": g.normal(0, 0.3, rh),
+         "router_w2": g.normal(0, 0.3, rh), "router_b2": g.normal(0, 0.3, 1),
+         "ln1_w": 1 + g.normal(0, 0.1, d), "ln2_w": 1 + g.normal(0, 0.1, d),
+         "w_qkv": g.normal(0, 0.2, (q + 2 * kv, d)), "b_qkv": g.normal(0, 0.2, q + 2 * kv),
+         "w_o": g.normal(0, 0.2, (d, q)), "w_up": g.normal(0, 0.2, (F_, d)), "w_down": g.normal(0, 0.2, (d, F_))}
+    if p["arch"] == O.NEOX:
+        W.update({"ln1_b": g.normal(0, 0.1, d), "ln2_b": g.normal(0, 0.1, d), "b_o": g.normal(0, 0.2, d),
+                  "b_up": g.normal(0, 0.2, F_), "b_down": g.normal(0, 0.2, d)})
+    else:
+        W["w_gate"] = g.normal(0, 0.2, (F_, d))
+    for z in zero:
+        W[z] = np.zeros_like(W[z])
+    return W
+
+
+class TestLayer:
+    def test_router_closed_form(self):
+        """d=2, h=1: score = 2 * SiLU(3) + 0.5 with SiLU(3) = 3 / (1 + e^-3)."""
+        W = {"router_w1": np.array([[1.0, 0.0]]), "router_b1": np.array([0.0]),
+             "router_w2": np.array([2.0]), "router_b2": np.array([0.5])}
+        s = O.router_scores(np.array([[3.0, 7.0]]), W)
+        assert s[0] == pytest.approx(2 * 3 / (1 + math.exp(-3)) + 0.5, rel=1e-15)
+
+    @pytest.mark.parametrize("arch", [O.NEOX, O.QWEN])
+    def test_r1_is_dense_and_r0_identity(self, arch):
+        """K = T: every token kept -> the dense layer on the whole sequence;
+        K = 0: every token bypasses -> identity, byte for byte."""
+        p = _params(arch, Hkv=2 if arch == O.QWEN else 4)
+        W = _weights(p, 14)
+        x = rng(15).normal(size=(2, 11, 32))
+        out, idx, _ = O.sparse_layer_forward(x, W, p, 11)
+        for b in range(2):
+            dense = x[b] + O.block_delta(x[b], np.arange(11), W, p)
+            assert out[b] == pytest.approx(dense, rel=1e-13, abs=1e-13)
+        out0, idx0, _ = O.sparse_layer_forward(x, W, p, 0)
+        assert idx0.shape == (2, 0) and np.array_equal(out0.view(np.uint64), x.view(np.uint64))
+
+    @pytest.mark.parametrize("arch", [O.NEOX, O.QWEN])
+    def test_skipped_rows_untouched_and_kept_rows_follow_router(self, arch):
+        p = _params(arch)
+        W = _weights(p, 16)
+        x = rng(17).normal(size=(3, 13, 32))
+        out, idx, sc = O.sparse_layer_forward(x, W, p, 5)
+        for b in range(3):
+            assert idx[b].tolist() == _brute_topk(list(sc[b]), 5)
+            skip = np.setdiff1d(np.arange(13), idx[b])
+            assert np.array_equal(out[b, skip].view(np.uint64), x[b, skip].view(np.uint64))
+            assert not np.allclose(out[b, idx[b]], x[b, idx[b]])
+
+    @pytest.mark.parametrize("arch", [O.NEOX, O.QWEN])
+    def test_position_shift_invariance(self, arch):
+        """Positions enter only through RoPE, whose scores depend on position
+        differences: shifting every kept position by c leaves the delta unchanged,
+        while permuting the gaps changes it."""
+        p = _params(arch)
+        W = _weights(p, 18)
+        xp = rng(19).normal(size=(6, 32))
+        pos = np.array([0, 2, 3, 7, 8, 12])
+        a = O.block_delta(xp, pos, W, p)
+        b = O.block_delta(xp, pos + 37, W, p)
+        c = O.block_delta(xp, np.array([0, 1, 2, 3, 4, 5]), W, p)
+        assert a == pytest.approx(b, rel=1e-9, abs=1e-11)
+        assert not np.allclose(a, c)
+
+    def test_neox_closed_form_zero_projections(self):
+        """W_qkv = 0 and W_up = 0: every value row is b_v, so attention returns
+        b_v whatever the scores; delta = W_o b_v + b_o + W_down GELU(b_up) + b_down."""
+        p = _params(O.NEOX)
+        W = _weights(p, 20, zero=("w_qkv", "w_up"))
+        xp = rng(21).normal(size=(5, 32))
+        bv = W["b_qkv"][64:96]
+        expect = W["w_o"] @ bv + W["b_o"] + W["w_down"] @ O.gelu(W["b_up"]) + W["b_down"]
+        got = O.block_delta(xp, np.arange(5), W, p)
+        for i in range(5):
+            assert got[i] == pytest.approx(expect, rel=1e-12, abs=1e-13)
+
+    def test_qwen_closed_form_zero_projections(self):
+        """W_qkv = 0, W_gate = 0: query head h returns value head h // 2 (= b_v of
+        that head), h = x + W_o o and SiLU(0) = 0 kills the MLP, so delta = W_o o."""
+        p = _params(O.QWEN, Hkv=2)
+        W = _weights(p, 22, zero=("w_qkv", "w_gate"))
+        xp = rng(23).normal(size=(4, 32))
+        bv = W["b_qkv"][32 + 16:32 + 32]
+        got = O.block_delta(xp, np.arange(4), W, p)
+        for i in range(4):
+            o = np.concatenate([bv[:8], bv[:8], bv[8:], bv[8:]])
+            assert got[i] == pytest.approx(W["w_o"] @ o, rel=1e-12)
+
+    @pytest.mark.parametrize("arch", [O.NEOX, O.QWEN])
+    def test_causality(self, arch):
+        """Changing the last kept token leaves the earlier outputs unchanged."""
+        p = _params(arch)
+        W = _weights(p, 24)
+        xp = rng(25).normal(size=(7, 32))
+        a = O.block_delta(xp, np.arange(7), W, p)
+        xq = xp.copy(); xq[-1] += rng(27).normal(size=32)   # not a constant shift: LayerNorm ignores those
+        b = O.block_delta(xq, np.arange(7), W, p)
+        assert a[:-1] == pytest.approx(b[:-1], rel=1e-13, abs=1e-14)
+        assert not np.allclose(a[-1], b[-1])
+
+    def test_model_special_cases(self):
+        """All K = 0: the model is final_norm(embedding); statistics are cos = 1.
+        All K = T: the model is the dense stack."""
+        p = _params(O.NEOX)
+        g = rng(26)
+        Wm = {"embed": g.normal(size=(50, 32)), "final_w": 1 + g.normal(0, .1, 32), "final_b": g.normal(0, .1, 32)}
+        layers = [_weights(p, 30 + l) for l in range(3)]
+        ids = g.integers(0, 50, size=(2, 9))
+        h, kept, st = O.sparse_model_forward(ids, Wm, layers, p, [0, 0, 0], stats_mode="token")
+        assert h == pytest.approx(O.layer_norm(Wm["embed"][ids], Wm["final_w"], Wm["final_b"], 1e-5), rel=1e-13)
+        assert all(O.similarity(s_) == pytest.approx(1.0, abs=1e-14) for s_ in st)
+        h, kept, _ = O.sparse_model_forward(ids, Wm, layers, p, [9, 9, 9])
+        x = Wm["embed"][ids]
+        for W in layers:
+            x = np.stack([x[b] + O.block_delta(x[b], np.arange(9), W, p) for b in range(2)])
+        assert h == pytest.approx(O.layer_norm(x, Wm["final_w"], Wm["final_b"], 1e-5), rel=1e-12)
