@@ -1,0 +1,264 @@
+/*
+ * adadsf.h -- C ABI of the GB300 depth-sparse forward of AdaDSF
+ * ("Adaptive Depth Sparse Framework: Similarity-Driven Resource Allocation
+ *  for Pre-Trained LLMs").
+ *
+ * Conventions shared by every entry point
+ *  - Pointers named *_dev are device pointers (CUDA global memory of the
+ *    current device); pointers named *_host are host pointers. The caller owns
+ *    all memory. No entry point allocates or frees device memory; scratch
+ *    space comes from a caller-provided workspace (ws, ws_bytes).
+ *  - Device pointers must be 16-byte aligned; the workspace 256-byte aligned.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream). Every device entry point only enqueues work on that stream and
+ *    returns without synchronising; results are ready once the stream is.
+ *  - Tensors are dense row-major. Weights are [out_features, in_features]
+ *    (the torch.nn.Linear layout); the fused QKV weight stacks the query
+ *    rows, then the key rows, then the value rows.
+ *  - Activations and weights are stored in cfg->dtype (fp32 or bf16);
+ *    accumulation, norms, softmax and residual additions run in fp32 with one
+ *    rounding per stored tensor. Router scores are fp32. Indices are int32.
+ *  - Errors: every call returns an adadsf_status; on failure nothing was
+ *    enqueued (argument errors are detected before the first launch) unless
+ *    the status is ADADSF_ERR_CUDA. adadsf_last_error() gives a readable
+ *    message for the calling thread. No C++ exception crosses this boundary.
+ *  - Kernels that wait on barriers give up after a bounded time, record the
+ *    fact in a device error word at the start of the workspace and return;
+ *    adadsf_sync_check() reports it as ADADSF_ERR_DEVICE_TIMEOUT.
+ */
+#ifndef ADADSF_H
+#define ADADSF_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  ADADSF_OK = 0,
+  ADADSF_ERR_INVALID_ARG = 1,
+  ADADSF_ERR_UNSUPPORTED = 2,
+  ADADSF_ERR_CUDA = 3,
+  ADADSF_ERR_WORKSPACE_TOO_SMALL = 4,
+  ADADSF_ERR_DEVICE_TIMEOUT = 5
+} adadsf_status;
+
+typedef enum { ADADSF_F32 = 0, ADADSF_BF16 = 1 } adadsf_dtype;
+
+/* GPT-NeoX: out = x + Attn(LN1 x) + MLP(LN2 x), LayerNorm, exact-GELU MLP,
+ *           biases on every projection.
+ * Qwen2.5:  h = x + Attn(RMS1 x); out = h + MLP(RMS2 h), RMSNorm, SwiGLU MLP,
+ *           bias on the QKV projection only. */
+typedef enum { ADADSF_ARCH_NEOX = 0, ADADSF_ARCH_QWEN = 1 } adadsf_arch;
+
+/* Eq. 4 statistic aggregation. TOKEN: acc += {sum_rows cos(a_r, b_r), rows};
+ * FLAT: acc += {sum a.b, sum |a|^2, sum |b|^2} over all rows. */
+typedef enum { ADADSF_STATS_TOKEN = 0, ADADSF_STATS_FLAT = 1 } adadsf_stats_mode;
+
+/* adadsf_alloc_ratios flags */
+#define ADADSF_ALLOC_RAW 1u      /* return Eq. 8 unclamped (ratios may exceed 1) */
+#define ADADSF_ALLOC_ROUND 2u    /* K = round(r T) instead of floor(r T) */
+
+typedef struct {
+  int32_t d;             /* hidden size */
+  int32_t n_heads;       /* query heads */
+  int32_t n_kv_heads;    /* key/value heads; divides n_heads */
+  int32_t head_dim;      /* 64 or 128 */
+  int32_t ffn;           /* MLP width */
+  int32_t n_layers;
+  int32_t vocab;
+  int32_t router_hidden; /* width of the router's hidden layer (64) */
+  int32_t arch;          /* adadsf_arch */
+  int32_t rotary_dim;    /* leading features of each head that rotate; even */
+  float rope_theta;      /* rotary base */
+  float norm_eps;
+  int32_t dtype;         /* adadsf_dtype */
+  int32_t flags;         /* reserved, 0 */
+} adadsf_model_cfg;
+
+/* Device pointers to one layer's parameters, all in cfg->dtype.
+ * NULL marks a tensor the architecture does not have. Shapes:
+ * router_w1 [h,d] router_b1 [h] router_w2 [h] router_b2 [1]   (h = router_hidden)
+ * ln1_w, ln1_b, ln2_w, ln2_b [d]        (the *_b are NeoX only)
+ * w_qkv [q+2kv, d] b_qkv [q+2kv]        (q = n_heads*head_dim, kv = n_kv_heads*head_dim)
+ * w_o [d, q] b_o [d]                    (b_o NeoX only)
+ * w_up [ffn, d] b_up [ffn]              (b_up NeoX only)
+ * w_gate [ffn, d]                       (Qwen only)
+ * w_down [d, ffn] b_down [d]            (b_down NeoX only) */
+typedef struct {
+  const void *router_w1, *router_b1, *router_w2, *router_b2;
+  const void *ln1_w, *ln1_b, *ln2_w, *ln2_b;
+  const void *w_qkv, *b_qkv, *w_o, *b_o;
+  const void *w_up, *b_up, *w_gate, *w_down, *b_down;
+} adadsf_layer_weights;
+
+/* embed [vocab, d]; final_w, final_b [d] (final_b NeoX only);
+ * layers: HOST array of n_layers adadsf_layer_weights (pointing to device data). */
+typedef struct {
+  const void *embed, *final_w, *final_b;
+  const adadsf_layer_weights *layers;
+} adadsf_model_weights;
+
+/* Message describing the last failure on the calling thread ("" if none). */
+const char *adadsf_last_error(void);
+
+/* ------------------------------------------------------------------------
+ * Workspace sizes (bytes, multiples of 256). Return 0 when the arguments are
+ * invalid (see adadsf_last_error).
+ * ---------------------------------------------------------------------- */
+/* One sparse layer on (B,T,d) with K kept tokens per sequence. */
+size_t adadsf_layer_workspace_size(const adadsf_model_cfg *cfg, int B, int T, int K);
+/* The whole model; K_host holds n_layers kept counts. with_stats != 0 adds
+ * the room the Eq. 4 statistics pass needs. */
+size_t adadsf_model_workspace_size(const adadsf_model_cfg *cfg, int B, int T,
+                                   const int32_t *K_host, int with_stats);
+/* adadsf_layer_stats on n_rows rows. */
+size_t adadsf_stats_workspace_size(int64_t n_rows);
+
+/* ------------------------------------------------------------------------
+ * Sec. 3.3, Eq. 4: similarity of a layer's input and output hidden states.
+ * x_in_dev, x_out_dev: [n_rows, d] in `dtype`. acc_dev: device fp64 array
+ * (2 entries for TOKEN mode, 3 for FLAT, see adadsf_stats_mode) to which this
+ * call ADDS its partial sums, so calibration batches, layers' calls and ranks
+ * can be accumulated; the order of the additions inside one call is fixed
+ * (results are bit-reproducible). Per-row cosine uses
+ * a.b / (max(|a|,1e-8) max(|b|,1e-8)) with fp32 row sums.
+ * ---------------------------------------------------------------------- */
+adadsf_status adadsf_layer_stats(const void *x_in_dev, const void *x_out_dev, int64_t n_rows,
+                                 int d, int dtype, int mode, double *acc_dev,
+                                 void *ws, size_t ws_bytes, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Sec. 3.3, Eqs. 5-8: layer-wise retention ratios from the similarity vector,
+ * then K_l = floor(r_l T) (Sec. 3.4). Host only, pure, no device work.
+ * s_host[L] similarities; t target mean retention in [0,1]; tau > 0; beta > 0.
+ * Unless ADADSF_ALLOC_RAW, ratios above 1 are clamped to 1 and the leftover
+ * budget is spread over the other layers in proportion to r'_l, repeatedly,
+ * so that sum r = t L with every r_l <= 1. K_l = floor(r_l T + 1e-9) clamped
+ * to [0,T] (ADADSF_ALLOC_ROUND: nearest). Outputs: r_out_host[L] (may be
+ * NULL), K_out_host[L] (may be NULL).
+ * ---------------------------------------------------------------------- */
+adadsf_status adadsf_alloc_ratios(const double *s_host, int L, double t, double tau, double beta,
+                                  int T, unsigned flags, double *r_out_host, int32_t *K_out_host);
+
+/* ------------------------------------------------------------------------
+ * Sec. 3.4: router scores of every token, w2 . SiLU(W1 x + b1) + b2.
+ * x_dev [B*T, d] (cfg->dtype); scores_dev [B*T] fp32.
+ * ---------------------------------------------------------------------- */
+adadsf_status adadsf_router_scores(const adadsf_model_cfg *cfg, const adadsf_layer_weights *w,
+                                   const void *x_dev, int64_t n_rows, float *scores_dev,
+                                   void *ws, size_t ws_bytes, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Sec. 3.4: Top-K_i of each sequence's router scores, K_i = K for all.
+ * scores_dev [B,T] fp32. Ranking: higher score first, equal scores by lower
+ * position, -0.0 equals +0.0, NaN below every number. idx_dev [B,K] int32
+ * receives the kept positions in ascending order; rows_dev [B,K] int32 (may
+ * be NULL) receives b*T + position. 0 <= K <= T <= 16384.
+ * ---------------------------------------------------------------------- */
+adadsf_status adadsf_topk_select(const float *scores_dev, int B, int T, int K,
+                                 int32_t *idx_dev, int32_t *rows_dev, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Eq. 2 building block: out = act(x W^T + bias). x_dev [M, k_in],
+ * w_dev [n_out, k_in], bias_dev [n_out] or NULL, out_dev [M, n_out], all in
+ * `dtype`. act: 0 identity, 1 exact GELU. k_in % 64 == 0, n_out % 64 == 0 for
+ * bf16 (tcgen05 tensor-core path), multiples of 4 for fp32.
+ * ---------------------------------------------------------------------- */
+adadsf_status adadsf_linear(const void *x_dev, const void *w_dev, const void *bias_dev,
+                            int64_t M, int n_out, int k_in, int dtype, int act, void *out_dev,
+                            void *ws, size_t ws_bytes, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Eq. 1 among kept tokens: per sequence b and query head h,
+ * softmax(Q K^T / sqrt(head_dim)) V, causal in packed order (which is the
+ * original order, as kept positions ascend). qkv_dev [B*K, q+2kv] (rotary
+ * already applied), out_dev [B*K, q]; cfg->dtype. Query head h reads kv head
+ * h / (n_heads / n_kv_heads).
+ * ---------------------------------------------------------------------- */
+adadsf_status adadsf_causal_attention(const adadsf_model_cfg *cfg, const void *qkv_dev, int B,
+                                      int K, void *out_dev, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Sec. 3.4: one depth-sparse layer, in place.
+ * x_dev [B,T,d]: kept rows become x + delta (delta = the layer's residual
+ * update computed on the kept tokens only, causal among them, rotary at
+ * their original positions); every other row is left untouched (not read
+ * back nor written). K == 0 enqueues nothing; K == T runs the dense layer
+ * (router and Top-K skipped). idx_out_dev [B,K] int32 and scores_out_dev
+ * [B,T] fp32 receive the kept positions and router scores (either may be
+ * NULL; with K == T scores are not computed and scores_out_dev is ignored).
+ * ---------------------------------------------------------------------- */
+adadsf_status adadsf_sparse_layer_forward(const adadsf_model_cfg *cfg, const adadsf_layer_weights *w,
+                                          void *x_dev, int B, int T, int K, int32_t *idx_out_dev,
+                                          float *scores_out_dev, void *ws, size_t ws_bytes,
+                                          void *stream);
+
+/* ------------------------------------------------------------------------
+ * Sec. 3.2 / 3.4: the depth-sparse model. ids_dev [B,T] int32 -> embedding
+ * -> layer l as adadsf_sparse_layer_forward with K_host[l] kept tokens ->
+ * final norm -> hidden_out_dev [B,T,d] (cfg->dtype).
+ * stats_acc_dev: NULL, or device fp64 [n_layers * 2] (TOKEN mode) to which
+ *   the Eq. 4 sums of each layer's (input, output) pair are added (the
+ *   calibration pass runs this with K_l = T).
+ * idx_out_dev: NULL, or device int32 of B * sum_l K_l entries receiving each
+ *   layer's kept positions [B, K_l], layer after layer.
+ * Out-of-range token ids read as zero rows and raise the device error word.
+ * ---------------------------------------------------------------------- */
+adadsf_status adadsf_sparse_model_forward(const adadsf_model_cfg *cfg, const adadsf_model_weights *w,
+                                          const int32_t *ids_dev, int B, int T, const int32_t *K_host,
+                                          void *hidden_out_dev, double *stats_acc_dev,
+                                          int32_t *idx_out_dev, void *ws, size_t ws_bytes,
+                                          void *stream);
+
+/* ------------------------------------------------------------------------
+ * Synchronises `stream`, then reads and clears the device error word at the
+ * start of `ws`: ADADSF_ERR_DEVICE_TIMEOUT if a kernel gave up waiting,
+ * ADADSF_ERR_INVALID_ARG if a kernel met an out-of-range index,
+ * ADADSF_ERR_CUDA on a CUDA error, else ADADSF_OK.
+ * ---------------------------------------------------------------------- */
+adadsf_status adadsf_sync_check(void *ws, size_t ws_bytes, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Per-launch timing (diagnostics; no paper counterpart). Between
+ * adadsf_profile_begin and adadsf_profile_end every kernel the library
+ * launches on a stream that is not being captured is bracketed by a pair of
+ * CUDA events on that stream and recorded with its algorithmic work:
+ * flops (2 per multiply-add of the dense contractions and of attention) and
+ * bytes (each input element read once plus each output element written once,
+ * skipped rows excluded). adadsf_profile_end synchronises the device, writes
+ * up to `max` records and returns the number of records (or -1 on error).
+ * Kinds are the ADADSF_KERNEL_* values; adadsf_kernel_name names them.
+ * ---------------------------------------------------------------------- */
+typedef enum {
+  ADADSF_KERNEL_EMBED = 0, ADADSF_KERNEL_ROUTER, ADADSF_KERNEL_TOPK, ADADSF_KERNEL_POSITIONS,
+  ADADSF_KERNEL_GATHER_NORM, ADADSF_KERNEL_GEMM_QKV, ADADSF_KERNEL_ROPE_TABLE, ADADSF_KERNEL_ROPE,
+  ADADSF_KERNEL_ATTENTION, ADADSF_KERNEL_GEMM_O, ADADSF_KERNEL_NORM2, ADADSF_KERNEL_GEMM_UP,
+  ADADSF_KERNEL_GEMM_DOWN, ADADSF_KERNEL_STATS, ADADSF_KERNEL_FINAL_NORM, ADADSF_KERNEL_COPY,
+  ADADSF_KERNEL_LINEAR, ADADSF_KERNEL_SELFTEST, ADADSF_KERNEL_COUNT
+} adadsf_kernel_kind;
+
+typedef struct {
+  int32_t kind;    /* adadsf_kernel_kind */
+  int32_t dense;   /* 1 if the launch runs on tensor cores (flops-bound) */
+  double ms;       /* device time between the bracketing events */
+  double flops;    /* algorithmic floating-point operations of the launch */
+  double bytes;    /* algorithmic HBM bytes of the launch */
+} adadsf_launch_record;
+
+adadsf_status adadsf_profile_begin(int max_launches);
+int adadsf_profile_end(adadsf_launch_record *out_host, int max);
+const char *adadsf_kernel_name(int kind);
+
+/* Self-test of the bounded-wait path: launches one block that waits on a
+ * shared-memory barrier nothing arrives at, gives up after about
+ * timeout_us microseconds, records ADADSF_ERR_DEVICE_TIMEOUT in the error
+ * word of `ws` and returns, leaving the context usable. No paper counterpart. */
+adadsf_status adadsf_selftest_bounded_wait(void *ws, size_t ws_bytes, int timeout_us, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ADADSF_H */

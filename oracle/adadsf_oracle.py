@@ -85,6 +85,17 @@ def rope(v, pos, rotary_dim, theta):
     return out
 
 
+def linear(x, w, b=None, act=None):
+    """Affine map of Eq. 2, x W^T + b (W stored [out, in]), optionally followed
+    by the exact GELU."""
+    y = np.asarray(x, dtype=np.float64) @ np.asarray(w, dtype=np.float64).T
+    if b is not None:
+        y = y + b
+    if act == "gelu":
+        y = gelu(y)
+    return y
+
+
 # --------------------------------------------------------------------------
 # Eq. 1 -- attention among the given rows, causal in row order
 # --------------------------------------------------------------------------

@@ -1,0 +1,281 @@
+"""Python binding of the C ABI in include/adadsf.h (libadadsf.so).
+
+Argument marshalling only: every step of the depth-sparse forward runs in the
+library's CUDA kernels. PyTorch provides device memory and streams. The
+functions carry the C names; tensors replace (pointer, size) pairs.
+
+The library is loaded from this package directory; if it is missing every call
+raises (there is no fallback path)."""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence
+
+import numpy as np
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libadadsf.so")
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_WORKSPACE_TOO_SMALL, ERR_DEVICE_TIMEOUT = range(6)
+F32, BF16 = 0, 1
+ARCH_NEOX, ARCH_QWEN = 0, 1
+STATS_TOKEN, STATS_FLAT = 0, 1
+ALLOC_RAW, ALLOC_ROUND = 1, 2
+
+TORCH_DTYPE = {F32: torch.float32, BF16: torch.bfloat16}
+DTYPE_CODE = {torch.float32: F32, torch.bfloat16: BF16}
+
+LAYER_FIELDS = ("router_w1", "router_b1", "router_w2", "router_b2", "ln1_w", "ln1_b", "ln2_w",
+                "ln2_b", "w_qkv", "b_qkv", "w_o", "b_o", "w_up", "b_up", "w_gate", "w_down", "b_down")
+
+
+class ModelCfg(ctypes.Structure):
+    _fields_ = [("d", ctypes.c_int32), ("n_heads", ctypes.c_int32), ("n_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("ffn", ctypes.c_int32), ("n_layers", ctypes.c_int32),
+                ("vocab", ctypes.c_int32), ("router_hidden", ctypes.c_int32), ("arch", ctypes.c_int32),
+                ("rotary_dim", ctypes.c_int32), ("rope_theta", ctypes.c_float),
+                ("norm_eps", ctypes.c_float), ("dtype", ctypes.c_int32), ("flags", ctypes.c_int32)]
+
+
+class LayerWeights(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in LAYER_FIELDS]
+
+
+class ModelWeights(ctypes.Structure):
+    _fields_ = [("embed", ctypes.c_void_p), ("final_w", ctypes.c_void_p),
+                ("final_b", ctypes.c_void_p), ("layers", ctypes.POINTER(LayerWeights))]
+
+
+class AdadsfError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"adadsf status {status}: {msg}")
+        self.status = status
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded libadadsf.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with "
+                               "`python -c 'import __graft_entry__ as g; g.build()'`")
+        L = ctypes.CDLL(LIB_PATH)
+        vp, i32, i64, sz, f64, u32 = (ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_size_t,
+                                      ctypes.c_double, ctypes.c_uint)
+        pcfg, plw, pmw = ctypes.POINTER(ModelCfg), ctypes.POINTER(LayerWeights), ctypes.POINTER(ModelWeights)
+        sig = {
+            "adadsf_last_error": (ctypes.c_char_p, []),
+            "adadsf_layer_workspace_size": (sz, [pcfg, i32, i32, i32]),
+            "adadsf_model_workspace_size": (sz, [pcfg, i32, i32, vp, i32]),
+            "adadsf_stats_workspace_size": (sz, [i64]),
+            "adadsf_layer_stats": (i32, [vp, vp, i64, i32, i32, i32, vp, vp, sz, vp]),
+            "adadsf_alloc_ratios": (i32, [vp, i32, f64, f64, f64, i32, u32, vp, vp]),
+            "adadsf_router_scores": (i32, [pcfg, plw, vp, i64, vp, vp, sz, vp]),
+            "adadsf_topk_select": (i32, [vp, i32, i32, i32, vp, vp, vp]),
+            "adadsf_linear": (i32, [vp, vp, vp, i64, i32, i32, i32, i32, vp, vp, sz, vp]),
+            "adadsf_causal_attention": (i32, [pcfg, vp, i32, i32, vp, vp]),
+            "adadsf_sparse_layer_forward": (i32, [pcfg, plw, vp, i32, i32, i32, vp, vp, vp, sz, vp]),
+            "adadsf_sparse_model_forward": (i32, [pcfg, pmw, vp, i32, i32, vp, vp, vp, vp, vp, sz, vp]),
+            "adadsf_sync_check": (i32, [vp, sz, vp]),
+            "adadsf_selftest_bounded_wait": (i32, [vp, sz, i32, vp]),
+        }
+        for name, (res, args) in sig.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _check(status: int):
+    if status != OK:
+        raise AdadsfError(status, lib().adadsf_last_error().decode())
+
+
+def _p(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _s(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dev(t: torch.Tensor, name: str):
+    if not t.is_cuda or not t.is_contiguous():
+        raise ValueError(f"{name} must be a contiguous CUDA tensor")
+
+
+def workspace(nbytes: int, device=None) -> torch.Tensor:
+    """Zero-initialised device workspace (its first 256 bytes are the error word)."""
+    return torch.zeros(max(int(nbytes), 256), dtype=torch.uint8, device=device or "cuda")
+
+
+# --------------------------------------------------------------------- config
+def make_cfg(shape) -> ModelCfg:
+    """ModelCfg from any object with the backbone fields (see synth.Shape)."""
+    return ModelCfg(shape.d, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn,
+                    shape.n_layers, shape.vocab, shape.router_hidden, shape.arch, shape.rotary_dim,
+                    shape.rope_theta, shape.norm_eps, BF16 if shape.dtype == "bf16" else F32, 0)
+
+
+def layer_struct(w: dict) -> LayerWeights:
+    """LayerWeights pointing at the device tensors of dict w (missing -> NULL)."""
+    s = LayerWeights()
+    for n in LAYER_FIELDS:
+        t = w.get(n)
+        if t is not None:
+            _dev(t, n)
+        setattr(s, n, None if t is None else t.data_ptr())
+    return s
+
+
+def to_device(host: dict, dtype: torch.dtype, device="cuda") -> dict:
+    """Copies a dict of host arrays to device tensors of the storage dtype."""
+    return {k: torch.from_numpy(np.ascontiguousarray(v)).to(device=device, dtype=dtype)
+            for k, v in host.items()}
+
+
+# --------------------------------------------------------------------- C entry points
+def adadsf_last_error() -> str:
+    return lib().adadsf_last_error().decode()
+
+
+def adadsf_layer_workspace_size(cfg: ModelCfg, B: int, T: int, K: int) -> int:
+    n = lib().adadsf_layer_workspace_size(ctypes.byref(cfg), B, T, K)
+    if n == 0:
+        raise AdadsfError(ERR_INVALID_ARG, adadsf_last_error())
+    return n
+
+
+def adadsf_model_workspace_size(cfg: ModelCfg, B: int, T: int, K: Sequence[int], with_stats=False) -> int:
+    arr = (ctypes.c_int32 * len(K))(*[int(k) for k in K])
+    n = lib().adadsf_model_workspace_size(ctypes.byref(cfg), B, T, ctypes.cast(arr, ctypes.c_void_p),
+                                          1 if with_stats else 0)
+    if n == 0:
+        raise AdadsfError(ERR_INVALID_ARG, adadsf_last_error())
+    return n
+
+
+def adadsf_stats_workspace_size(n_rows: int) -> int:
+    return lib().adadsf_stats_workspace_size(int(n_rows))
+
+
+def adadsf_layer_stats(x_in: torch.Tensor, x_out: torch.Tensor, acc: torch.Tensor,
+                       mode: int = STATS_TOKEN, ws: Optional[torch.Tensor] = None, stream=None):
+    """Adds the Eq. 4 partial sums of (x_in, x_out) rows to the fp64 tensor acc."""
+    _dev(x_in, "x_in"); _dev(x_out, "x_out"); _dev(acc, "acc")
+    if acc.dtype != torch.float64:
+        raise ValueError("acc must be float64")
+    d = x_in.shape[-1]
+    n = x_in.numel() // d
+    if ws is None:
+        ws = workspace(adadsf_stats_workspace_size(n), x_in.device)
+    _check(lib().adadsf_layer_stats(_p(x_in), _p(x_out), n, d, DTYPE_CODE[x_in.dtype], mode,
+                                    _p(acc), _p(ws), ws.numel(), _s(stream)))
+
+
+def adadsf_alloc_ratios(s: Sequence[float], t: float, tau: float = 0.05, beta: float = 10.0,
+                        T: int = 0, flags: int = 0):
+    """Host-only Eqs. 5-8 (+ clamp) -> (r, K) as NumPy arrays."""
+    s = np.ascontiguousarray(s, dtype=np.float64)
+    L = s.shape[0]
+    r = np.zeros(L, dtype=np.float64)
+    K = np.zeros(L, dtype=np.int32)
+    _check(lib().adadsf_alloc_ratios(s.ctypes.data_as(ctypes.c_void_p), L, float(t), float(tau),
+                                     float(beta), int(T), int(flags), r.ctypes.data_as(ctypes.c_void_p),
+                                     K.ctypes.data_as(ctypes.c_void_p)))
+    return r, K
+
+
+def adadsf_router_scores(cfg: ModelCfg, w: dict, x: torch.Tensor, scores: torch.Tensor,
+                         ws: Optional[torch.Tensor] = None, stream=None):
+    _dev(x, "x"); _dev(scores, "scores")
+    n = x.numel() // cfg.d
+    if ws is None:
+        ws = workspace(256, x.device)
+    lw = layer_struct(w)
+    _check(lib().adadsf_router_scores(ctypes.byref(cfg), ctypes.byref(lw), _p(x), n, _p(scores),
+                                      _p(ws), ws.numel(), _s(stream)))
+
+
+def adadsf_topk_select(scores: torch.Tensor, K: int, idx: torch.Tensor,
+                       rows: Optional[torch.Tensor] = None, stream=None):
+    _dev(scores, "scores"); _dev(idx, "idx")
+    B, T = scores.shape
+    _check(lib().adadsf_topk_select(_p(scores), B, T, int(K), _p(idx), _p(rows), _s(stream)))
+
+
+def adadsf_linear(x: torch.Tensor, w: torch.Tensor, bias: Optional[torch.Tensor], out: torch.Tensor,
+                  act: int = 0, ws: Optional[torch.Tensor] = None, stream=None):
+    _dev(x, "x"); _dev(w, "w"); _dev(out, "out")
+    n_out, k_in = w.shape
+    M = x.numel() // k_in
+    if ws is None:
+        ws = workspace(256, x.device)
+    _check(lib().adadsf_linear(_p(x), _p(w), _p(bias), M, n_out, k_in, DTYPE_CODE[x.dtype], act,
+                               _p(out), _p(ws), ws.numel(), _s(stream)))
+
+
+def adadsf_causal_attention(cfg: ModelCfg, qkv: torch.Tensor, B: int, K: int, out: torch.Tensor,
+                            stream=None):
+    _dev(qkv, "qkv"); _dev(out, "out")
+    _check(lib().adadsf_causal_attention(ctypes.byref(cfg), _p(qkv), B, K, _p(out), _s(stream)))
+
+
+def adadsf_sparse_layer_forward(cfg: ModelCfg, w: dict, x: torch.Tensor, K: int,
+                                idx_out: Optional[torch.Tensor] = None,
+                                scores_out: Optional[torch.Tensor] = None,
+                                ws: Optional[torch.Tensor] = None, stream=None):
+    """In place on x (B, T, d)."""
+    _dev(x, "x")
+    B, T, _ = x.shape
+    if ws is None:
+        ws = workspace(adadsf_layer_workspace_size(cfg, B, T, K), x.device)
+    lw = layer_struct(w)
+    _check(lib().adadsf_sparse_layer_forward(ctypes.byref(cfg), ctypes.byref(lw), _p(x), B, T, int(K),
+                                             _p(idx_out), _p(scores_out), _p(ws), ws.numel(),
+                                             _s(stream)))
+
+
+class DeviceModel:
+    """Device tensors of a whole model plus the ctypes structs that point at them."""
+
+    def __init__(self, cfg: ModelCfg, layers: Sequence[dict], extra: dict):
+        self.cfg = cfg
+        self.layers = list(layers)
+        self.extra = extra
+        self._lw = (LayerWeights * len(self.layers))(*[layer_struct(w) for w in self.layers])
+        self.struct = ModelWeights(extra["embed"].data_ptr(), extra["final_w"].data_ptr(),
+                                   extra["final_b"].data_ptr() if extra.get("final_b") is not None else None,
+                                   ctypes.cast(self._lw, ctypes.POINTER(LayerWeights)))
+
+
+def adadsf_sparse_model_forward(model: DeviceModel, ids: torch.Tensor, K: Sequence[int],
+                                hidden_out: torch.Tensor, stats_acc: Optional[torch.Tensor] = None,
+                                idx_out: Optional[torch.Tensor] = None,
+                                ws: Optional[torch.Tensor] = None, stream=None):
+    _dev(ids, "ids"); _dev(hidden_out, "hidden_out")
+    B, T = ids.shape
+    Karr = (ctypes.c_int32 * len(K))(*[int(k) for k in K])
+    if ws is None:
+        ws = workspace(adadsf_model_workspace_size(model.cfg, B, T, K, stats_acc is not None), ids.device)
+    _check(lib().adadsf_sparse_model_forward(ctypes.byref(model.cfg), ctypes.byref(model.struct),
+                                             _p(ids), B, T, ctypes.cast(Karr, ctypes.c_void_p),
+                                             _p(hidden_out), _p(stats_acc), _p(idx_out), _p(ws),
+                                             ws.numel(), _s(stream)))
+
+
+def adadsf_sync_check(ws: torch.Tensor, stream=None) -> int:
+    """Synchronises and returns the status of the device error word (cleared)."""
+    return lib().adadsf_sync_check(_p(ws), ws.numel(), _s(stream))
+
+
+def adadsf_selftest_bounded_wait(ws: torch.Tensor, timeout_us: int, stream=None):
+    _check(lib().adadsf_selftest_bounded_wait(_p(ws), ws.numel(), int(timeout_us), _s(stream)))

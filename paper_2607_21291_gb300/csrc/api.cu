@@ -1,0 +1,826 @@
+// C ABI of the depth-sparse forward (declared in include/adadsf.h): argument
+// validation, workspace carving, the per-layer launch sequence and the host
+// retention allocation. No entry point allocates device memory or
+// synchronises a stream except adadsf_sync_check.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "adadsf.h"
+#include "internal.h"
+
+using namespace adadsf;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+adadsf_status fail(adadsf_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+
+adadsf_status cuda_fail(cudaError_t e, const char* what) {
+  return fail(ADADSF_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define CUDA_TRY(expr, what)                    \
+  do {                                          \
+    cudaError_t e_ = (expr);                    \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+  } while (0)
+
+#define TRY(expr)                               \
+  do {                                          \
+    adadsf_status s_ = (expr);                  \
+    if (s_ != ADADSF_OK) return s_;             \
+  } while (0)
+
+constexpr size_t kErrBytes = 256;
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int elem_size(int dtype) { return dtype == kBF16 ? 2 : 4; }
+
+adadsf_status device_info(Dev* dev, void* stream, void* ws) {
+  int device = 0;
+  CUDA_TRY(cudaGetDevice(&device), "cudaGetDevice");
+  static int sms[64] = {0};
+  if (device >= 64) return fail(ADADSF_ERR_UNSUPPORTED, "device ordinal %d >= 64", device);
+  if (!sms[device]) {
+    int n = 0;
+    CUDA_TRY(cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, device),
+             "cudaDeviceGetAttribute");
+    sms[device] = n;
+  }
+  dev->num_sms = sms[device];
+  dev->stream = static_cast<cudaStream_t>(stream);
+  dev->err = static_cast<int*>(ws);
+  return ADADSF_OK;
+}
+
+adadsf_status check_cfg(const adadsf_model_cfg* c) {
+  if (!c) return fail(ADADSF_ERR_INVALID_ARG, "cfg is NULL");
+  if (c->dtype != ADADSF_F32 && c->dtype != ADADSF_BF16)
+    return fail(ADADSF_ERR_INVALID_ARG, "dtype %d is neither ADADSF_F32 nor ADADSF_BF16", c->dtype);
+  if (c->arch != ADADSF_ARCH_NEOX && c->arch != ADADSF_ARCH_QWEN)
+    return fail(ADADSF_ERR_INVALID_ARG, "arch %d unknown", c->arch);
+  const int vec = c->dtype == ADADSF_BF16 ? 8 : 4;
+  if (c->d <= 0 || c->d % 64 != 0)
+    return fail(ADADSF_ERR_UNSUPPORTED, "d=%d must be a positive multiple of 64", c->d);
+  if (c->d > 16 * 32 * vec)
+    return fail(ADADSF_ERR_UNSUPPORTED, "d=%d exceeds %d for this dtype", c->d, 16 * 32 * vec);
+  if (c->head_dim != 64 && c->head_dim != 128)
+    return fail(ADADSF_ERR_UNSUPPORTED, "head_dim=%d must be 64 or 128", c->head_dim);
+  if (c->n_heads <= 0 || c->n_kv_heads <= 0 || c->n_heads % c->n_kv_heads != 0)
+    return fail(ADADSF_ERR_INVALID_ARG, "n_heads=%d must be a positive multiple of n_kv_heads=%d",
+                c->n_heads, c->n_kv_heads);
+  if (c->ffn <= 0 || c->ffn % 64 != 0)
+    return fail(ADADSF_ERR_UNSUPPORTED, "ffn=%d must be a positive multiple of 64", c->ffn);
+  if (c->dtype == ADADSF_BF16 && c->router_hidden != 64)
+    return fail(ADADSF_ERR_UNSUPPORTED, "bf16 router_hidden=%d must be 64", c->router_hidden);
+  if (c->router_hidden <= 0 || c->router_hidden > 1024)
+    return fail(ADADSF_ERR_INVALID_ARG, "router_hidden=%d out of range", c->router_hidden);
+  if (c->rotary_dim < 0 || c->rotary_dim > c->head_dim || c->rotary_dim % 2 != 0)
+    return fail(ADADSF_ERR_INVALID_ARG, "rotary_dim=%d must be even and <= head_dim", c->rotary_dim);
+  if (!(c->norm_eps > 0.f) || !(c->rope_theta > 0.f))
+    return fail(ADADSF_ERR_INVALID_ARG, "norm_eps and rope_theta must be positive");
+  return ADADSF_OK;
+}
+
+adadsf_status check_shape(int B, int T, int K) {
+  if (B < 0 || T <= 0 || K < 0 || K > T)
+    return fail(ADADSF_ERR_INVALID_ARG, "need B >= 0, T > 0, 0 <= K <= T (B=%d T=%d K=%d)", B, T, K);
+  if (T > 16384) return fail(ADADSF_ERR_UNSUPPORTED, "T=%d exceeds 16384", T);
+  if ((int64_t)B * T > (int64_t)1 << 30) return fail(ADADSF_ERR_UNSUPPORTED, "B*T too large");
+  return ADADSF_OK;
+}
+
+adadsf_status check_ws(void* ws, size_t ws_bytes, size_t need) {
+  if (!ws) return fail(ADADSF_ERR_INVALID_ARG, "workspace is NULL");
+  if (reinterpret_cast<uintptr_t>(ws) & 255u)
+    return fail(ADADSF_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+  if (ws_bytes < need)
+    return fail(ADADSF_ERR_WORKSPACE_TOO_SMALL, "workspace has %zu bytes, needs %zu", ws_bytes, need);
+  return ADADSF_OK;
+}
+
+// ---------------------------------------------------------------- per-launch timing
+struct Profiler {
+  std::mutex mu;
+  bool on = false;
+  int cap = 0;
+  std::vector<cudaEvent_t> ev;   // two per record
+  std::vector<adadsf_launch_record> recs;
+};
+Profiler g_prof;
+
+// Runs f() (which enqueues one kernel or copy on dev.stream); while profiling
+// is on and the stream is not being captured, brackets it with events.
+template <typename F>
+adadsf_status launch(const Dev& dev, int kind, bool dense, double flops, double bytes, F&& f) {
+  cudaEvent_t a = nullptr, b = nullptr;
+  if (g_prof.on) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(dev.stream, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusNone) {
+      std::lock_guard<std::mutex> lk(g_prof.mu);
+      const size_t i = g_prof.recs.size();
+      if ((int)i < g_prof.cap) {
+        a = g_prof.ev[2 * i];
+        b = g_prof.ev[2 * i + 1];
+        g_prof.recs.push_back({kind, dense ? 1 : 0, 0.0, flops, bytes});
+      }
+    }
+  }
+  if (a) cudaEventRecord(a, dev.stream);
+  const adadsf_status st = f();
+  if (b) cudaEventRecord(b, dev.stream);
+  return st;
+}
+
+#define NEED_PTR(p, name)                                                             \
+  do {                                                                                \
+    if (!(p)) return fail(ADADSF_ERR_INVALID_ARG, "%s is NULL", name);                \
+    if (!aligned16(p)) return fail(ADADSF_ERR_INVALID_ARG, "%s is not 16-byte aligned", name); \
+  } while (0)
+
+adadsf_status check_layer_weights(const adadsf_model_cfg* c, const adadsf_layer_weights* w,
+                                  bool need_router) {
+  if (!w) return fail(ADADSF_ERR_INVALID_ARG, "layer weights are NULL");
+  if (need_router) {
+    NEED_PTR(w->router_w1, "router_w1");
+    NEED_PTR(w->router_b1, "router_b1");
+    NEED_PTR(w->router_w2, "router_w2");
+    if (!w->router_b2) return fail(ADADSF_ERR_INVALID_ARG, "router_b2 is NULL");
+  }
+  NEED_PTR(w->ln1_w, "ln1_w");
+  NEED_PTR(w->ln2_w, "ln2_w");
+  NEED_PTR(w->w_qkv, "w_qkv");
+  NEED_PTR(w->b_qkv, "b_qkv");
+  NEED_PTR(w->w_o, "w_o");
+  NEED_PTR(w->w_up, "w_up");
+  NEED_PTR(w->w_down, "w_down");
+  if (c->arch == ADADSF_ARCH_NEOX) {
+    NEED_PTR(w->ln1_b, "ln1_b");
+    NEED_PTR(w->ln2_b, "ln2_b");
+    NEED_PTR(w->b_o, "b_o");
+    NEED_PTR(w->b_up, "b_up");
+    NEED_PTR(w->b_down, "b_down");
+  } else {
+    NEED_PTR(w->w_gate, "w_gate");
+  }
+  return ADADSF_OK;
+}
+
+// ---------------------------------------------------------------- workspace layout
+struct Carver {
+  size_t cur = 0;
+  size_t take(size_t bytes) {
+    const size_t o = cur;
+    cur = align256(cur + bytes);
+    return o;
+  }
+};
+
+struct LayerSlots {
+  size_t scores, idx, rows, n1, n2, qkv, attn, ao, act;
+};
+
+void carve_layer(const adadsf_model_cfg* c, int B, int T, int K, Carver& cv, LayerSlots& s) {
+  const size_t es = elem_size(c->dtype);
+  const size_t M = (size_t)B * K;
+  const size_t q = (size_t)c->n_heads * c->head_dim, kv = (size_t)c->n_kv_heads * c->head_dim;
+  s.scores = cv.take((size_t)B * T * 4);
+  s.idx = cv.take(M * 4);
+  s.rows = cv.take(M * 4);
+  s.n1 = cv.take(M * c->d * es);
+  s.n2 = c->arch == ADADSF_ARCH_NEOX ? cv.take(M * c->d * es) : 0;
+  s.qkv = cv.take(M * (q + 2 * kv) * es);
+  s.attn = cv.take(M * q * es);
+  s.ao = cv.take(M * c->d * es);
+  s.act = cv.take(M * c->ffn * es);
+}
+
+size_t rope_bytes(const adadsf_model_cfg* c, int T) { return (size_t)T * (c->rotary_dim / 2) * 8; }
+
+template <typename T>
+T* at(void* ws, size_t off) {
+  return reinterpret_cast<T*>(static_cast<char*>(ws) + off);
+}
+
+// ---------------------------------------------------------------- one layer
+struct LayerBufs {
+  float* scores;
+  int32_t* idx;
+  int32_t* rows;
+  const float2* rope;
+  void *n1, *n2, *qkv, *attn, *ao, *act;
+};
+
+adadsf_status run_linear(int dtype, const GemmArgs& g, const Dev& dev, const char* what) {
+  cudaError_t e = dtype == kBF16 ? gemm_bf16(g, dev) : gemm_f32(g, dev);
+  if (e != cudaSuccess) return cuda_fail(e, what);
+  return ADADSF_OK;
+}
+
+GemmArgs linear_args(const void* A, int64_t lda, const void* W, int64_t M, int N, int K) {
+  GemmArgs g;
+  g.A = A; g.lda = lda; g.W = W; g.ldw = K;
+  g.M = M; g.N = N; g.K = K;
+  return g;
+}
+
+#define CALL(expr, what)                 \
+  [&]() -> adadsf_status {               \
+    cudaError_t e_ = (expr);             \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+    return ADADSF_OK;                    \
+  }
+
+// Sec. 3.4: router -> Top-K -> gather + norm -> block on the packed rows ->
+// residual delta scattered back into x. K == T skips router and Top-K.
+adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* w, void* x, int B,
+                         int T, int K, const LayerBufs& lb, bool want_idx, const Dev& dev) {
+  if (K == 0 || B == 0) return ADADSF_OK;
+  const bool dense = K == T;
+  const int dt = c->dtype, d = c->d;
+  const double es = elem_size(dt);
+  const int64_t M = (int64_t)B * K;
+  const int64_t BT = (int64_t)B * T;
+  const int q = c->n_heads * c->head_dim, kv = c->n_kv_heads * c->head_dim;
+  const int qkv_dim = q + 2 * kv;
+  const int F = c->ffn;
+  const bool neox = c->arch == ADADSF_ARCH_NEOX;
+  const bool tc = dt == kBF16;   // dense contractions on tensor cores
+  const double Md = (double)M * d;
+  const int32_t* rows = nullptr;
+  const int32_t* pos = nullptr;
+
+  if (!dense) {
+    const double rf = 2.0 * BT * c->router_hidden * d;
+    const double rb = (double)BT * d * es + (double)c->router_hidden * d * es + BT * 4.0;
+    if (tc) {
+      GemmArgs g = linear_args(x, d, w->router_w1, BT, c->router_hidden, d);
+      g.epi.act = ACT_ROUTER;
+      g.epi.bias = w->router_b1;
+      g.epi.w2 = w->router_w2;
+      g.epi.b2 = w->router_b2;
+      g.epi.scores = lb.scores;
+      TRY(launch(dev, ADADSF_KERNEL_ROUTER, true, rf, rb, [&] { return run_linear(dt, g, dev, "router"); }));
+    } else {
+      TRY(launch(dev, ADADSF_KERNEL_ROUTER, false, rf, rb,
+                 CALL(router_f32(static_cast<const float*>(x), BT, d, c->router_hidden,
+                                 static_cast<const float*>(w->router_w1),
+                                 static_cast<const float*>(w->router_b1),
+                                 static_cast<const float*>(w->router_w2),
+                                 static_cast<const float*>(w->router_b2), lb.scores, dev),
+                      "router")));
+    }
+    TRY(launch(dev, ADADSF_KERNEL_TOPK, false, 0, BT * 4.0 + M * 8.0,
+               CALL(topk(lb.scores, B, T, K, lb.idx, lb.rows, dev), "top-k")));
+    rows = lb.rows;
+    pos = lb.idx;
+  } else if (want_idx) {
+    TRY(launch(dev, ADADSF_KERNEL_POSITIONS, false, 0, M * 4.0,
+               CALL(iota_positions(lb.idx, B, K, dev), "positions")));
+  }
+
+  // a4: gather kept rows and normalise (NeoX: LN1 and LN2 of the same row).
+  TRY(launch(dev, ADADSF_KERNEL_GATHER_NORM, false, 0, Md * es * (neox ? 3 : 2),
+             CALL(gather_norm(dt, x, rows, M, d, !neox, w->ln1_w, w->ln1_b, w->ln2_w, w->ln2_b,
+                              c->norm_eps, lb.n1, neox ? lb.n2 : nullptr, dev),
+                  "gather+norm")));
+  // a5: QKV projection (+bias), rotary at the original positions.
+  {
+    GemmArgs g = linear_args(lb.n1, d, w->w_qkv, M, qkv_dim, d);
+    g.epi.bias = w->b_qkv;
+    g.epi.out = lb.qkv;
+    g.epi.ld_out = qkv_dim;
+    TRY(launch(dev, ADADSF_KERNEL_GEMM_QKV, tc, 2.0 * M * qkv_dim * d,
+               (Md + (double)qkv_dim * d + (double)M * qkv_dim) * es,
+               [&] { return run_linear(dt, g, dev, "qkv projection"); }));
+  }
+  if (c->rotary_dim > 0)
+    TRY(launch(dev, ADADSF_KERNEL_ROPE, false, 0,
+               2.0 * M * (c->n_heads + c->n_kv_heads) * c->rotary_dim * es,
+               CALL(rope_apply(dt, lb.qkv, M, qkv_dim, c->n_heads, c->n_kv_heads, c->head_dim,
+                               c->rotary_dim, pos, T, lb.rope, dev),
+                    "rotary")));
+  // a6: causal attention among the kept tokens.
+  TRY(launch(dev, ADADSF_KERNEL_ATTENTION, tc, 2.0 * B * c->n_heads * c->head_dim * (double)K * (K + 1),
+             ((double)M * qkv_dim + (double)M * q) * es,
+             CALL(attention(dt, lb.qkv, qkv_dim, lb.attn, q, B, K, c->n_heads, c->n_kv_heads,
+                            c->head_dim, dev),
+                  "attention")));
+  if (neox) {
+    // a7: attn_out = O W_o^T + b_o (packed)
+    GemmArgs g = linear_args(lb.attn, q, w->w_o, M, d, q);
+    g.epi.bias = w->b_o;
+    g.epi.out = lb.ao;
+    g.epi.ld_out = d;
+    TRY(launch(dev, ADADSF_KERNEL_GEMM_O, tc, 2.0 * M * d * q, ((double)M * q + (double)d * q + Md) * es,
+               [&] { return run_linear(dt, g, dev, "output projection"); }));
+    // a8: act = GELU(LN2 x W_up^T + b_up)
+    GemmArgs u = linear_args(lb.n2, d, w->w_up, M, F, d);
+    u.epi.bias = w->b_up;
+    u.epi.act = ACT_GELU;
+    u.epi.out = lb.act;
+    u.epi.ld_out = F;
+    TRY(launch(dev, ADADSF_KERNEL_GEMM_UP, tc, 2.0 * M * F * d, (Md + (double)F * d + (double)M * F) * es,
+               [&] { return run_linear(dt, u, dev, "mlp up"); }));
+    // a8 + a9: x[row] = x[row] + attn_out + act W_down^T + b_down
+    GemmArgs dn = linear_args(lb.act, F, w->w_down, M, d, F);
+    dn.epi.bias = w->b_down;
+    dn.epi.add_packed = lb.ao;
+    dn.epi.ld_add_packed = d;
+    dn.epi.add_rows = x;
+    dn.epi.ld_add_rows = d;
+    dn.epi.rows = rows;
+    dn.epi.out_mapped = true;
+    dn.epi.out = x;
+    dn.epi.ld_out = d;
+    TRY(launch(dev, ADADSF_KERNEL_GEMM_DOWN, tc, 2.0 * M * d * F,
+               ((double)M * F + (double)d * F + 3.0 * Md) * es,
+               [&] { return run_linear(dt, dn, dev, "mlp down + residual scatter"); }));
+  } else {
+    // a7: h = x[row] + O W_o^T (packed)
+    GemmArgs g = linear_args(lb.attn, q, w->w_o, M, d, q);
+    g.epi.add_rows = x;
+    g.epi.ld_add_rows = d;
+    g.epi.rows = rows;
+    g.epi.out_mapped = false;
+    g.epi.out = lb.ao;
+    g.epi.ld_out = d;
+    TRY(launch(dev, ADADSF_KERNEL_GEMM_O, tc, 2.0 * M * d * q,
+               ((double)M * q + (double)d * q + 2.0 * Md) * es,
+               [&] { return run_linear(dt, g, dev, "output projection + residual"); }));
+    // a4': RMS2(h)
+    TRY(launch(dev, ADADSF_KERNEL_NORM2, false, 0, 2.0 * Md * es,
+               CALL(gather_norm(dt, lb.ao, nullptr, M, d, true, w->ln2_w, nullptr, nullptr, nullptr,
+                                c->norm_eps, lb.n1, nullptr, dev),
+                    "post-attention norm")));
+    // a8: act = SiLU(h' W_gate^T) * (h' W_up^T)
+    GemmArgs u = linear_args(lb.n1, d, w->w_gate, M, F, d);
+    u.W2 = w->w_up;
+    u.epi.act = ACT_SWIGLU;
+    u.epi.out = lb.act;
+    u.epi.ld_out = F;
+    TRY(launch(dev, ADADSF_KERNEL_GEMM_UP, tc, 4.0 * M * F * d,
+               (Md + 2.0 * F * d + (double)M * F) * es,
+               [&] { return run_linear(dt, u, dev, "mlp gate/up"); }));
+    // a8 + a9: x[row] = h + act W_down^T
+    GemmArgs dn = linear_args(lb.act, F, w->w_down, M, d, F);
+    dn.epi.add_packed = lb.ao;
+    dn.epi.ld_add_packed = d;
+    dn.epi.rows = rows;
+    dn.epi.out_mapped = true;
+    dn.epi.out = x;
+    dn.epi.ld_out = d;
+    TRY(launch(dev, ADADSF_KERNEL_GEMM_DOWN, tc, 2.0 * M * d * F,
+               ((double)M * F + (double)d * F + 2.0 * Md) * es,
+               [&] { return run_linear(dt, dn, dev, "mlp down + residual scatter"); }));
+  }
+  return ADADSF_OK;
+}
+
+size_t layer_ws_bytes(const adadsf_model_cfg* c, int B, int T, int K) {
+  Carver cv;
+  cv.take(kErrBytes);
+  cv.take(rope_bytes(c, T));
+  LayerSlots s;
+  carve_layer(c, B, T, K, cv, s);
+  return cv.cur;
+}
+
+struct ModelSlots {
+  size_t x, xin, partials, rope;
+  LayerSlots layer;
+  size_t total;
+};
+
+void carve_model(const adadsf_model_cfg* c, int B, int T, int Kmax, bool stats, ModelSlots& m) {
+  const size_t es = elem_size(c->dtype);
+  Carver cv;
+  cv.take(kErrBytes);
+  m.x = cv.take((size_t)B * T * c->d * es);
+  m.xin = stats ? cv.take((size_t)B * T * c->d * es) : 0;
+  m.partials = stats ? cv.take((size_t)stats_partials_count((int64_t)B * T) * 3 * 8) : 0;
+  m.rope = cv.take(rope_bytes(c, T));
+  carve_layer(c, B, T, Kmax, cv, m.layer);
+  m.total = cv.cur;
+}
+
+}  // namespace
+
+// ======================================================================== ABI
+extern "C" {
+
+const char* adadsf_last_error(void) { return g_last_error.c_str(); }
+
+size_t adadsf_layer_workspace_size(const adadsf_model_cfg* cfg, int B, int T, int K) {
+  if (check_cfg(cfg) != ADADSF_OK || check_shape(B, T, K) != ADADSF_OK) return 0;
+  return layer_ws_bytes(cfg, B, T, K);
+}
+
+size_t adadsf_model_workspace_size(const adadsf_model_cfg* cfg, int B, int T, const int32_t* K_host,
+                                   int with_stats) {
+  if (check_cfg(cfg) != ADADSF_OK) return 0;
+  if (!K_host || cfg->n_layers <= 0) {
+    fail(ADADSF_ERR_INVALID_ARG, "K_host is NULL or n_layers <= 0");
+    return 0;
+  }
+  int kmax = 0;
+  for (int l = 0; l < cfg->n_layers; ++l) {
+    if (check_shape(B, T, K_host[l]) != ADADSF_OK) return 0;
+    kmax = K_host[l] > kmax ? K_host[l] : kmax;
+  }
+  ModelSlots m;
+  carve_model(cfg, B, T, kmax, with_stats != 0, m);
+  return m.total;
+}
+
+size_t adadsf_stats_workspace_size(int64_t n_rows) {
+  if (n_rows < 0) return 0;
+  return kErrBytes + align256((size_t)stats_partials_count(n_rows) * 3 * 8);
+}
+
+adadsf_status adadsf_layer_stats(const void* x_in_dev, const void* x_out_dev, int64_t n_rows, int d,
+                                 int dtype, int mode, double* acc_dev, void* ws, size_t ws_bytes,
+                                 void* stream) {
+  if (dtype != ADADSF_F32 && dtype != ADADSF_BF16)
+    return fail(ADADSF_ERR_INVALID_ARG, "dtype %d unknown", dtype);
+  if (mode != ADADSF_STATS_TOKEN && mode != ADADSF_STATS_FLAT)
+    return fail(ADADSF_ERR_INVALID_ARG, "mode %d unknown", mode);
+  if (n_rows < 0 || d <= 0 || d % (dtype == ADADSF_BF16 ? 8 : 4) != 0)
+    return fail(ADADSF_ERR_INVALID_ARG, "need n_rows >= 0 and d a positive multiple of 16 bytes");
+  if (!acc_dev || (reinterpret_cast<uintptr_t>(acc_dev) & 7u))
+    return fail(ADADSF_ERR_INVALID_ARG, "acc_dev is NULL or not 8-byte aligned");
+  TRY(check_ws(ws, ws_bytes, adadsf_stats_workspace_size(n_rows)));
+  if (n_rows == 0) return ADADSF_OK;
+  NEED_PTR(x_in_dev, "x_in_dev");
+  NEED_PTR(x_out_dev, "x_out_dev");
+  Dev dev;
+  TRY(device_info(&dev, stream, ws));
+  return launch(dev, ADADSF_KERNEL_STATS, false, 0, 2.0 * n_rows * d * elem_size(dtype),
+                CALL(cos_stats(dtype, x_in_dev, x_out_dev, n_rows, d, mode, at<double>(ws, kErrBytes),
+                               acc_dev, dev),
+                     "similarity statistics"));
+}
+
+adadsf_status adadsf_alloc_ratios(const double* s_host, int L, double t, double tau, double beta,
+                                  int T, unsigned flags, double* r_out_host, int32_t* K_out_host) {
+  if (!s_host || L <= 0) return fail(ADADSF_ERR_INVALID_ARG, "s_host is NULL or L <= 0");
+  if (!(t >= 0.0 && t <= 1.0)) return fail(ADADSF_ERR_INVALID_ARG, "t=%g outside [0,1]", t);
+  if (!(tau > 0.0) || !(beta > 0.0)) return fail(ADADSF_ERR_INVALID_ARG, "tau and beta must be > 0");
+  if (T < 0) return fail(ADADSF_ERR_INVALID_ARG, "T < 0");
+  for (int i = 0; i < L; ++i)
+    if (!isfinite(s_host[i])) return fail(ADADSF_ERR_INVALID_ARG, "s[%d] is not finite", i);
+  // Eq. 5: temperature-normalised weights
+  double smax = s_host[0];
+  for (int i = 1; i < L; ++i) smax = s_host[i] > smax ? s_host[i] : smax;
+  std::vector<double> w(L), rp(L), r(L);
+  double wsum = 0.0;
+  for (int i = 0; i < L; ++i) {
+    w[i] = exp((s_host[i] - smax) / tau);
+    wsum += w[i];
+  }
+  double wmean = 0.0;
+  for (int i = 0; i < L; ++i) {
+    w[i] /= wsum;
+    wmean += w[i];
+  }
+  wmean /= L;
+  // Eqs. 6-7: deviation scaling, sigmoid into (0.05, 0.95)
+  double rpsum = 0.0;
+  for (int i = 0; i < L; ++i) {
+    const double z = beta * (wmean - w[i]);
+    rp[i] = 0.05 + 0.9 / (1.0 + exp(-z));
+    rpsum += rp[i];
+  }
+  // Eq. 8: global budget t L
+  for (int i = 0; i < L; ++i) r[i] = t * L / rpsum * rp[i];
+  if (!(flags & ADADSF_ALLOC_RAW)) {
+    if (t >= 1.0) {
+      for (int i = 0; i < L; ++i) r[i] = 1.0;
+    } else {
+      // Clamp to 1, spread the remaining budget over the unclamped layers in
+      // proportion to r', until nothing exceeds 1.
+      std::vector<char> fixed(L, 0);
+      for (;;) {
+        bool any = false;
+        for (int i = 0; i < L; ++i)
+          if (!fixed[i] && r[i] > 1.0) { fixed[i] = 1; any = true; }
+        if (!any) break;
+        int nfixed = 0;
+        double free_rp = 0.0;
+        for (int i = 0; i < L; ++i) {
+          if (fixed[i]) ++nfixed; else free_rp += rp[i];
+        }
+        const double budget = t * L - nfixed;
+        for (int i = 0; i < L; ++i) r[i] = fixed[i] ? 1.0 : budget / free_rp * rp[i];
+      }
+    }
+  }
+  for (int i = 0; i < L; ++i) {
+    if (r_out_host) r_out_host[i] = r[i];
+    if (K_out_host) {
+      double k = (flags & ADADSF_ALLOC_ROUND) ? floor(r[i] * T + 0.5) : floor(r[i] * T + 1e-9);
+      if (k < 0) k = 0;
+      if (k > T) k = T;
+      K_out_host[i] = (int32_t)k;
+    }
+  }
+  return ADADSF_OK;
+}
+
+adadsf_status adadsf_router_scores(const adadsf_model_cfg* cfg, const adadsf_layer_weights* w,
+                                   const void* x_dev, int64_t n_rows, float* scores_dev, void* ws,
+                                   size_t ws_bytes, void* stream) {
+  TRY(check_cfg(cfg));
+  if (!w) return fail(ADADSF_ERR_INVALID_ARG, "weights are NULL");
+  if (n_rows < 0 || n_rows > ((int64_t)1 << 30)) return fail(ADADSF_ERR_INVALID_ARG, "n_rows out of range");
+  TRY(check_ws(ws, ws_bytes, kErrBytes));
+  if (n_rows == 0) return ADADSF_OK;
+  NEED_PTR(x_dev, "x_dev");
+  NEED_PTR(scores_dev, "scores_dev");
+  NEED_PTR(w->router_w1, "router_w1");
+  NEED_PTR(w->router_b1, "router_b1");
+  NEED_PTR(w->router_w2, "router_w2");
+  if (!w->router_b2) return fail(ADADSF_ERR_INVALID_ARG, "router_b2 is NULL");
+  Dev dev;
+  TRY(device_info(&dev, stream, ws));
+  if (cfg->dtype == ADADSF_BF16) {
+    GemmArgs g = linear_args(x_dev, cfg->d, w->router_w1, n_rows, cfg->router_hidden, cfg->d);
+    g.epi.act = ACT_ROUTER;
+    g.epi.bias = w->router_b1;
+    g.epi.w2 = w->router_w2;
+    g.epi.b2 = w->router_b2;
+    g.epi.scores = scores_dev;
+    return run_linear(cfg->dtype, g, dev, "router");
+  }
+  CUDA_TRY(router_f32(static_cast<const float*>(x_dev), n_rows, cfg->d, cfg->router_hidden,
+                      static_cast<const float*>(w->router_w1), static_cast<const float*>(w->router_b1),
+                      static_cast<const float*>(w->router_w2), static_cast<const float*>(w->router_b2),
+                      scores_dev, dev),
+           "router");
+  return ADADSF_OK;
+}
+
+adadsf_status adadsf_topk_select(const float* scores_dev, int B, int T, int K, int32_t* idx_dev,
+                                 int32_t* rows_dev, void* stream) {
+  TRY(check_shape(B, T, K));
+  if (B == 0 || K == 0) return ADADSF_OK;
+  NEED_PTR(scores_dev, "scores_dev");
+  if (!idx_dev || (reinterpret_cast<uintptr_t>(idx_dev) & 3u))
+    return fail(ADADSF_ERR_INVALID_ARG, "idx_dev is NULL or misaligned");
+  Dev dev;
+  TRY(device_info(&dev, stream, nullptr));
+  CUDA_TRY(topk(scores_dev, B, T, K, idx_dev, rows_dev, dev), "top-k");
+  return ADADSF_OK;
+}
+
+adadsf_status adadsf_linear(const void* x_dev, const void* w_dev, const void* bias_dev, int64_t M,
+                            int n_out, int k_in, int dtype, int act, void* out_dev, void* ws,
+                            size_t ws_bytes, void* stream) {
+  if (dtype != ADADSF_F32 && dtype != ADADSF_BF16)
+    return fail(ADADSF_ERR_INVALID_ARG, "dtype %d unknown", dtype);
+  if (act != 0 && act != 1) return fail(ADADSF_ERR_INVALID_ARG, "act %d unknown", act);
+  const int mult = dtype == ADADSF_BF16 ? 64 : 4;
+  if (M < 0 || M > ((int64_t)1 << 30) || n_out <= 0 || k_in <= 0 || n_out % mult || k_in % mult)
+    return fail(ADADSF_ERR_UNSUPPORTED, "need M >= 0 and n_out, k_in positive multiples of %d", mult);
+  TRY(check_ws(ws, ws_bytes, kErrBytes));
+  if (M == 0) return ADADSF_OK;
+  NEED_PTR(x_dev, "x_dev");
+  NEED_PTR(w_dev, "w_dev");
+  NEED_PTR(out_dev, "out_dev");
+  if (bias_dev && !aligned16(bias_dev)) return fail(ADADSF_ERR_INVALID_ARG, "bias_dev misaligned");
+  Dev dev;
+  TRY(device_info(&dev, stream, ws));
+  GemmArgs g = linear_args(x_dev, k_in, w_dev, M, n_out, k_in);
+  g.epi.bias = bias_dev;
+  g.epi.act = act == 1 ? ACT_GELU : ACT_NONE;
+  g.epi.out = out_dev;
+  g.epi.ld_out = n_out;
+  const double es = elem_size(dtype);
+  return launch(dev, ADADSF_KERNEL_LINEAR, dtype == ADADSF_BF16, 2.0 * M * n_out * k_in,
+                ((double)M * k_in + (double)n_out * k_in + (double)M * n_out) * es,
+                [&] { return run_linear(dtype, g, dev, "linear"); });
+}
+
+adadsf_status adadsf_causal_attention(const adadsf_model_cfg* cfg, const void* qkv_dev, int B, int K,
+                                      void* out_dev, void* stream) {
+  TRY(check_cfg(cfg));
+  if (B < 0 || K < 0 || (int64_t)B * K > ((int64_t)1 << 30))
+    return fail(ADADSF_ERR_INVALID_ARG, "B and K must be >= 0");
+  if (B == 0 || K == 0) return ADADSF_OK;
+  NEED_PTR(qkv_dev, "qkv_dev");
+  NEED_PTR(out_dev, "out_dev");
+  Dev dev;
+  TRY(device_info(&dev, stream, nullptr));
+  const int q = cfg->n_heads * cfg->head_dim, kv = cfg->n_kv_heads * cfg->head_dim;
+  CUDA_TRY(attention(cfg->dtype, qkv_dev, q + 2 * kv, out_dev, q, B, K, cfg->n_heads,
+                     cfg->n_kv_heads, cfg->head_dim, dev),
+           "attention");
+  return ADADSF_OK;
+}
+
+adadsf_status adadsf_sparse_layer_forward(const adadsf_model_cfg* cfg, const adadsf_layer_weights* w,
+                                          void* x_dev, int B, int T, int K, int32_t* idx_out_dev,
+                                          float* scores_out_dev, void* ws, size_t ws_bytes,
+                                          void* stream) {
+  TRY(check_cfg(cfg));
+  TRY(check_shape(B, T, K));
+  if (K == 0 || B == 0) return ADADSF_OK;
+  TRY(check_layer_weights(cfg, w, K < T));
+  NEED_PTR(x_dev, "x_dev");
+  if (idx_out_dev && (reinterpret_cast<uintptr_t>(idx_out_dev) & 3u))
+    return fail(ADADSF_ERR_INVALID_ARG, "idx_out_dev misaligned");
+  if (scores_out_dev && (reinterpret_cast<uintptr_t>(scores_out_dev) & 3u))
+    return fail(ADADSF_ERR_INVALID_ARG, "scores_out_dev misaligned");
+  TRY(check_ws(ws, ws_bytes, layer_ws_bytes(cfg, B, T, K)));
+  Dev dev;
+  TRY(device_info(&dev, stream, ws));
+  Carver cv;
+  cv.take(kErrBytes);
+  const size_t rope_off = cv.take(rope_bytes(cfg, T));
+  LayerSlots s;
+  carve_layer(cfg, B, T, K, cv, s);
+  LayerBufs lb;
+  lb.scores = scores_out_dev ? scores_out_dev : at<float>(ws, s.scores);
+  lb.idx = idx_out_dev ? idx_out_dev : at<int32_t>(ws, s.idx);
+  lb.rows = at<int32_t>(ws, s.rows);
+  lb.rope = at<float2>(ws, rope_off);
+  lb.n1 = at<char>(ws, s.n1);
+  lb.n2 = at<char>(ws, s.n2);
+  lb.qkv = at<char>(ws, s.qkv);
+  lb.attn = at<char>(ws, s.attn);
+  lb.ao = at<char>(ws, s.ao);
+  lb.act = at<char>(ws, s.act);
+  if (cfg->rotary_dim > 0)
+    TRY(launch(dev, ADADSF_KERNEL_ROPE_TABLE, false, 0, rope_bytes(cfg, T),
+               CALL(rope_table(at<float2>(ws, rope_off), T, cfg->rotary_dim, cfg->rope_theta, dev),
+                    "rotary table")));
+  return layer_impl(cfg, w, x_dev, B, T, K, lb, idx_out_dev != nullptr, dev);
+}
+
+adadsf_status adadsf_sparse_model_forward(const adadsf_model_cfg* cfg, const adadsf_model_weights* w,
+                                          const int32_t* ids_dev, int B, int T, const int32_t* K_host,
+                                          void* hidden_out_dev, double* stats_acc_dev,
+                                          int32_t* idx_out_dev, void* ws, size_t ws_bytes,
+                                          void* stream) {
+  TRY(check_cfg(cfg));
+  if (!w || !w->layers) return fail(ADADSF_ERR_INVALID_ARG, "model weights or layer array is NULL");
+  if (!K_host || cfg->n_layers <= 0) return fail(ADADSF_ERR_INVALID_ARG, "K_host is NULL or n_layers <= 0");
+  TRY(check_shape(B, T, 0));
+  int kmax = 0;
+  for (int l = 0; l < cfg->n_layers; ++l) {
+    TRY(check_shape(B, T, K_host[l]));
+    if (K_host[l] > 0) TRY(check_layer_weights(cfg, &w->layers[l], K_host[l] < T));
+    kmax = K_host[l] > kmax ? K_host[l] : kmax;
+  }
+  NEED_PTR(w->embed, "embed");
+  NEED_PTR(w->final_w, "final_w");
+  if (cfg->arch == ADADSF_ARCH_NEOX) NEED_PTR(w->final_b, "final_b");
+  NEED_PTR(hidden_out_dev, "hidden_out_dev");
+  if (cfg->vocab <= 0) return fail(ADADSF_ERR_INVALID_ARG, "vocab <= 0");
+  if (B > 0) NEED_PTR(ids_dev, "ids_dev");
+  if (stats_acc_dev && (reinterpret_cast<uintptr_t>(stats_acc_dev) & 7u))
+    return fail(ADADSF_ERR_INVALID_ARG, "stats_acc_dev misaligned");
+  if (idx_out_dev && (reinterpret_cast<uintptr_t>(idx_out_dev) & 3u))
+    return fail(ADADSF_ERR_INVALID_ARG, "idx_out_dev misaligned");
+  ModelSlots m;
+  carve_model(cfg, B, T, kmax, stats_acc_dev != nullptr, m);
+  TRY(check_ws(ws, ws_bytes, m.total));
+  if (B == 0) return ADADSF_OK;
+  Dev dev;
+  TRY(device_info(&dev, stream, ws));
+  const int dt = cfg->dtype;
+  const size_t es = elem_size(dt);
+  void* x = at<char>(ws, m.x);
+  const double xbytes_d = (double)B * T * cfg->d * es;
+  TRY(launch(dev, ADADSF_KERNEL_EMBED, false, 0, 2.0 * xbytes_d + 4.0 * B * T,
+             CALL(embed(dt, ids_dev, (int64_t)B * T, w->embed, cfg->vocab, cfg->d, x, dev), "embedding")));
+  if (cfg->rotary_dim > 0)
+    TRY(launch(dev, ADADSF_KERNEL_ROPE_TABLE, false, 0, rope_bytes(cfg, T),
+               CALL(rope_table(at<float2>(ws, m.rope), T, cfg->rotary_dim, cfg->rope_theta, dev),
+                    "rotary table")));
+  LayerBufs lb;
+  lb.scores = at<float>(ws, m.layer.scores);
+  lb.rows = at<int32_t>(ws, m.layer.rows);
+  lb.rope = at<float2>(ws, m.rope);
+  lb.n1 = at<char>(ws, m.layer.n1);
+  lb.n2 = at<char>(ws, m.layer.n2);
+  lb.qkv = at<char>(ws, m.layer.qkv);
+  lb.attn = at<char>(ws, m.layer.attn);
+  lb.ao = at<char>(ws, m.layer.ao);
+  lb.act = at<char>(ws, m.layer.act);
+  const size_t xbytes = (size_t)B * T * cfg->d * es;
+  int64_t idx_off = 0;
+  for (int l = 0; l < cfg->n_layers; ++l) {
+    const int K = K_host[l];
+    lb.idx = idx_out_dev ? idx_out_dev + idx_off : at<int32_t>(ws, m.layer.idx);
+    if (stats_acc_dev)
+      TRY(launch(dev, ADADSF_KERNEL_COPY, false, 0, 2.0 * xbytes_d,
+                 CALL(cudaMemcpyAsync(at<char>(ws, m.xin), x, xbytes, cudaMemcpyDeviceToDevice, dev.stream),
+                      "copy of the layer input")));
+    TRY(layer_impl(cfg, &w->layers[l], x, B, T, K, lb, idx_out_dev != nullptr, dev));
+    if (stats_acc_dev)
+      TRY(launch(dev, ADADSF_KERNEL_STATS, false, 0, 2.0 * xbytes_d,
+                 CALL(cos_stats(dt, at<char>(ws, m.xin), x, (int64_t)B * T, cfg->d, ADADSF_STATS_TOKEN,
+                                at<double>(ws, m.partials), stats_acc_dev + 2 * l, dev),
+                      "similarity statistics")));
+    idx_off += (int64_t)B * K;
+  }
+  TRY(launch(dev, ADADSF_KERNEL_FINAL_NORM, false, 0, 2.0 * xbytes_d,
+             CALL(gather_norm(dt, x, nullptr, (int64_t)B * T, cfg->d, cfg->arch == ADADSF_ARCH_QWEN,
+                              w->final_w, w->final_b, nullptr, nullptr, cfg->norm_eps, hidden_out_dev,
+                              nullptr, dev),
+                  "final norm")));
+  return ADADSF_OK;
+}
+
+adadsf_status adadsf_sync_check(void* ws, size_t ws_bytes, void* stream) {
+  TRY(check_ws(ws, ws_bytes, kErrBytes));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int h = 0;
+  CUDA_TRY(cudaMemcpyAsync(&h, ws, sizeof(int), cudaMemcpyDeviceToHost, s), "read error word");
+  CUDA_TRY(cudaStreamSynchronize(s), "stream synchronise");
+  if (h != 0) {
+    CUDA_TRY(cudaMemsetAsync(ws, 0, sizeof(int), s), "clear error word");
+    CUDA_TRY(cudaStreamSynchronize(s), "stream synchronise");
+  }
+  if (h & DEVERR_TIMEOUT)
+    return fail(ADADSF_ERR_DEVICE_TIMEOUT, "a kernel gave up waiting on a barrier (error word %d)", h);
+  if (h & DEVERR_INDEX)
+    return fail(ADADSF_ERR_INVALID_ARG, "a kernel met an out-of-range index (error word %d)", h);
+  return ADADSF_OK;
+}
+
+adadsf_status adadsf_profile_begin(int max_launches) {
+  if (max_launches <= 0 || max_launches > (1 << 20))
+    return fail(ADADSF_ERR_INVALID_ARG, "max_launches out of range");
+  std::lock_guard<std::mutex> lk(g_prof.mu);
+  if (g_prof.on) return fail(ADADSF_ERR_INVALID_ARG, "profiling already on");
+  while ((int)g_prof.ev.size() < 2 * max_launches) {
+    cudaEvent_t e;
+    CUDA_TRY(cudaEventCreate(&e), "cudaEventCreate");
+    g_prof.ev.push_back(e);
+  }
+  g_prof.cap = max_launches;
+  g_prof.recs.clear();
+  g_prof.on = true;
+  return ADADSF_OK;
+}
+
+int adadsf_profile_end(adadsf_launch_record* out_host, int max) {
+  std::lock_guard<std::mutex> lk(g_prof.mu);
+  if (!g_prof.on) {
+    fail(ADADSF_ERR_INVALID_ARG, "profiling is not on");
+    return -1;
+  }
+  g_prof.on = false;
+  if (cudaDeviceSynchronize() != cudaSuccess) {
+    fail(ADADSF_ERR_CUDA, "cudaDeviceSynchronize failed");
+    return -1;
+  }
+  const int n = (int)g_prof.recs.size();
+  for (int i = 0; i < n && i < max && out_host; ++i) {
+    adadsf_launch_record r = g_prof.recs[i];
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, g_prof.ev[2 * i], g_prof.ev[2 * i + 1]) != cudaSuccess) ms = -1.f;
+    r.ms = ms;
+    out_host[i] = r;
+  }
+  return n;
+}
+
+const char* adadsf_kernel_name(int kind) {
+  static const char* names[ADADSF_KERNEL_COUNT] = {
+      "embed", "router", "topk", "positions", "gather_norm", "gemm_qkv", "rope_table", "rope",
+      "attention", "gemm_o", "norm2", "gemm_up", "gemm_down", "stats", "final_norm", "copy",
+      "linear", "selftest"};
+  return (kind >= 0 && kind < ADADSF_KERNEL_COUNT) ? names[kind] : "unknown";
+}
+
+adadsf_status adadsf_selftest_bounded_wait(void* ws, size_t ws_bytes, int timeout_us, void* stream) {
+  TRY(check_ws(ws, ws_bytes, kErrBytes));
+  if (timeout_us <= 0 || timeout_us > 2000000)
+    return fail(ADADSF_ERR_INVALID_ARG, "timeout_us must be in (0, 2e6]");
+  Dev dev;
+  TRY(device_info(&dev, stream, ws));
+  CUDA_TRY(bounded_wait_selftest(timeout_us, dev), "bounded-wait self-test");
+  return ADADSF_OK;
+}
+
+}  // extern "C"

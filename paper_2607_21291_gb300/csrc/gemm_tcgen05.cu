@@ -1,0 +1,400 @@
+// bf16 projections of the depth-sparse layer on the 5th-generation tensor cores.
+//
+// out = epilogue(A . W^T) with A [M, K] (packed kept tokens, row-major) and
+// W [N, K] (nn.Linear layout); both operands are K-major, which is the layout
+// tcgen05 reads natively. These are the dense contractions of Eqs. 1-2 (QKV,
+// output and MLP projections) and the router's first linear layer (Sec. 3.4).
+//
+// Kernel structure (one persistent CTA per SM, 6 warps):
+//   warp 0     TMA producer: 128x64 A tile and BNx64 W tile(s) per stage into a
+//              STAGES-deep shared-memory ring, 128-byte swizzled, signalled
+//              through mbarrier transaction counts.
+//   warp 1     allocates TMEM; one thread issues tcgen05.mma (M=128, N=BN,
+//              K=16, fp32 accumulator in TMEM) and commits stage releases and
+//              accumulator hand-offs to mbarriers.
+//   warps 2-5  epilogue: tcgen05.ld the accumulator (one row per thread),
+//              apply bias / GELU / SwiGLU / residual / row scatter / router
+//              reduction in fp32, round once and store.
+// The accumulator is double-buffered in TMEM so the epilogue of tile i runs
+// under the main loop of tile i+1. Every barrier wait is bounded in time; on
+// give-up the CTA records DEVERR_TIMEOUT, drains its in-flight copies and
+// MMAs, frees TMEM and exits.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace adadsf {
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;       // one 128-byte swizzle row of bf16
+constexpr int UK = 16;       // K of one tcgen05.mma kind::f16
+constexpr int kThreads = 192;
+constexpr int kGroupM = 16;  // tile raster: 16 M-blocks share each W column block
+
+template <int BN, bool DUAL>
+struct TileCfg {
+  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES * (DUAL ? 2 : 1);
+  static constexpr int STAGES_FIT = 196608 / STAGE_BYTES;
+  static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
+  static constexpr int ACC_COLS = BN * (DUAL ? 2 : 1);
+  static constexpr int TMEM_COLS = 2 * ACC_COLS;
+  static constexpr int BAR_BYTES = (2 * STAGES + 5) * 8 + 16;
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + BAR_BYTES;
+  static_assert(TMEM_COLS == 128 || TMEM_COLS == 256 || TMEM_COLS == 512, "TMEM columns");
+  static_assert(SMEM_BYTES <= 232448, "shared memory");
+};
+
+struct GemmDev {
+  int M, N, K;
+  int act;
+  const bf16* bias;
+  const bf16* add_packed; int64_t ld_add_packed;
+  const bf16* add_rows;   int64_t ld_add_rows;
+  const int32_t* rows;
+  int out_mapped;
+  bf16* out; int64_t ld_out;
+  const bf16* w2; const bf16* b2; float* scores;
+  int* err;
+  unsigned long long timeout_ns;
+};
+
+__device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int& mb, int& nb) {
+  const int group_tiles = kGroupM * num_n;
+  const int g = t / group_tiles;
+  const int first_m = g * kGroupM;
+  const int gsz = min(num_m - first_m, kGroupM);
+  const int r = t - g * group_tiles;
+  mb = first_m + r % gsz;
+  nb = r / gsz;
+}
+
+__device__ __forceinline__ float gelu_f(float v) { return 0.5f * v * (1.f + erff(v * 0.70710678118654752f)); }
+__device__ __forceinline__ float silu_f(float v) { return v / (1.f + expf(-v)); }
+
+// Epilogue of one 32-column chunk of one row (all values fp32 in v[]).
+__device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, int m, int64_t arow,
+                                                int64_t orow, int n0) {
+  if (p.add_packed) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float f[8];
+      load_vec(p.add_packed + (int64_t)m * p.ld_add_packed + n0 + 8 * i, f);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) v[8 * i + j] += f[j];
+    }
+  }
+  if (p.add_rows) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float f[8];
+      load_vec(p.add_rows + arow * p.ld_add_rows + n0 + 8 * i, f);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) v[8 * i + j] += f[j];
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) store_vec(p.out + orow * p.ld_out + n0 + 8 * i, v + 8 * i);
+}
+
+template <int BN, bool DUAL, bool ROUTER>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmB2, const GemmDev p) {
+  using C = TileCfg<BN, DUAL>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sA = smem_u32(smem);
+  const uint32_t sB = sA + C::STAGES * C::A_BYTES;
+  const uint32_t sB2 = sB + C::STAGES * C::B_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  const uint32_t full0 = smem_u32(bars);
+  const uint32_t empty0 = full0 + 8 * C::STAGES;
+  const uint32_t tfull0 = empty0 + 8 * C::STAGES;
+  const uint32_t tempty0 = tfull0 + 16;
+  const uint32_t drain = tempty0 + 16;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * C::STAGES + 5);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int num_m = (p.M + BM - 1) / BM;
+  const int num_n = (p.N + BN - 1) / BN;
+  const int num_tiles = num_m * num_n;
+  const int num_kb = (p.K + BK - 1) / BK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull0 + 8 * a, 1);
+      mbar_init(tempty0 + 8 * a, 4);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+    fence_proxy_async_smem();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+    if (DUAL) tma_prefetch_desc(&tmB2);
+  }
+  if (warp == 1) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int64_t issued = 0;
+      constexpr uint32_t tx = C::STAGE_BYTES;
+      for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
+        int mb, nb;
+        tile_coords(t, num_m, num_n, mb, nb);
+        bool ok = true;
+        for (int kb = 0; kb < num_kb; ++kb) {
+          if (!mbar_wait_bounded(empty0 + 8 * stage, phase ^ 1, abort_flag, p.err, p.timeout_ns)) {
+            ok = false;
+            break;
+          }
+          const uint32_t fb = full0 + 8 * stage;
+          mbar_arrive_expect_tx(fb, tx);
+          tma_load_2d(sA + stage * C::A_BYTES, &tmA, kb * BK, mb * BM, fb);
+          tma_load_2d(sB + stage * C::B_BYTES, &tmB, kb * BK, nb * BN, fb);
+          if (DUAL) tma_load_2d(sB2 + stage * C::B_BYTES, &tmB2, kb * BK, nb * BN, fb);
+          ++issued;
+          if (++stage == C::STAGES) { stage = 0; phase ^= 1; }
+        }
+        if (!ok) break;
+      }
+      // Drain: wait until the last copy issued into each stage has landed.
+      for (int s = 0; s < C::STAGES; ++s) {
+        if (issued <= s) break;
+        const int64_t last = s + ((issued - 1 - s) / C::STAGES) * C::STAGES;
+        mbar_wait_drain(full0 + 8 * s, (uint32_t)((last / C::STAGES) & 1), p.timeout_ns);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int it = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x, ++it) {
+        const int acc = it & 1;
+        if (!mbar_wait_bounded(tempty0 + 8 * acc, ((it >> 1) & 1) ^ 1, abort_flag, p.err,
+                               p.timeout_ns)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * C::ACC_COLS;
+        for (int kb = 0; kb < num_kb; ++kb) {
+          if (!mbar_wait_bounded(full0 + 8 * stage, phase, abort_flag, p.err, p.timeout_ns)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_s = sA + stage * C::A_BYTES;
+          const uint32_t b_s = sB + stage * C::B_BYTES;
+#pragma unroll
+          for (int k = 0; k < BK / UK; ++k) {
+            const uint64_t ad = smem_desc_sw128(a_s + k * UK * 2);
+            const uint64_t bd = smem_desc_sw128(b_s + k * UK * 2);
+            tc_mma_f16(d_tmem, ad, bd, idesc, (kb | k) != 0);
+            if (DUAL) {
+              const uint64_t b2d = smem_desc_sw128(sB2 + stage * C::B_BYTES + k * UK * 2);
+              tc_mma_f16(d_tmem + BN, ad, b2d, idesc, (kb | k) != 0);
+            }
+          }
+          tc_commit(empty0 + 8 * stage);   // stage free once these MMAs have read it
+          if (++stage == C::STAGES) { stage = 0; phase ^= 1; }
+        }
+        if (!ok) break;
+        tc_commit(tfull0 + 8 * acc);       // accumulator ready for the epilogue
+      }
+      // Drain: every MMA issued by this thread has completed.
+      tc_commit(drain);
+      mbar_wait_drain(drain, 0, p.timeout_ns);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue (warps 2..5)
+    const int quarter = warp & 3;   // TMEM lanes 32*quarter .. +31
+    int it = 0;
+    for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++it) {
+      int mb, nb;
+      tile_coords(t, num_m, num_n, mb, nb);
+      const int acc = it & 1;
+      int ok = 0;
+      if (lane == 0)
+        ok = mbar_wait_bounded(tfull0 + 8 * acc, (it >> 1) & 1, abort_flag, p.err, p.timeout_ns);
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      tc_fence_after();
+      const int m = mb * BM + quarter * 32 + lane;
+      const bool mvalid = m < p.M;
+      int64_t arow = m;
+      if (mvalid && p.rows) arow = p.rows[m];
+      const int64_t orow = p.out_mapped ? arow : (int64_t)m;
+      const uint32_t tacc = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C::ACC_COLS;
+      float rsum = 0.f;
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        uint32_t r[32];
+        tmem_ld32(tacc + c * 32, r);
+        uint32_t r2[DUAL ? 32 : 1];
+        if (DUAL) tmem_ld32(tacc + BN + c * 32, r2);
+        tmem_ld_wait();
+        const int n0 = nb * BN + c * 32;
+        if (!mvalid || n0 >= p.N) continue;
+        float v[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+        if (p.bias) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            float f[8];
+            load_vec(p.bias + n0 + 8 * i, f);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) v[8 * i + j] += f[j];
+          }
+        }
+        if (ROUTER) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            float f[8];
+            load_vec(p.w2 + n0 + 8 * i, f);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) rsum += f[j] * silu_f(v[8 * i + j]);
+          }
+          continue;
+        }
+        if (DUAL) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] = silu_f(v[j]) * __uint_as_float(r2[j]);
+        } else if (p.act == ACT_GELU) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v[j] = gelu_f(v[j]);
+        }
+        epi_chunk_store(p, v, m, arow, orow, n0);
+      }
+      if (ROUTER && mvalid) p.scores[m] = rsum + __bfloat162float(p.b2[0]);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------- host side
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+// Row-major bf16 [rows, cols] with leading dimension ld (elements); box of
+// 64 columns x box_rows rows, 128-byte swizzle, out-of-range reads as zero.
+bool make_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint64_t ld,
+               uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+template <int BN, bool DUAL, bool ROUTER>
+cudaError_t launch(const GemmArgs& a, const Dev& dev) {
+  using C = TileCfg<BN, DUAL>;
+  static int attr_done[64] = {0};
+  int device = 0;
+  cudaGetDevice(&device);
+  if (device < 64 && !attr_done[device]) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, DUAL, ROUTER>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    attr_done[device] = 1;
+  }
+  CUtensorMap ta, tb, tb2;
+  if (!make_tmap(&ta, a.A, (uint64_t)a.M, (uint64_t)a.K, (uint64_t)a.lda, BM) ||
+      !make_tmap(&tb, a.W, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, BN) ||
+      (DUAL && !make_tmap(&tb2, a.W2, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, BN)))
+    return cudaErrorInvalidValue;
+  if (!DUAL) tb2 = tb;
+  GemmDev p;
+  p.M = (int)a.M; p.N = a.N; p.K = a.K;
+  p.act = a.epi.act;
+  p.bias = static_cast<const bf16*>(a.epi.bias);
+  p.add_packed = static_cast<const bf16*>(a.epi.add_packed); p.ld_add_packed = a.epi.ld_add_packed;
+  p.add_rows = static_cast<const bf16*>(a.epi.add_rows); p.ld_add_rows = a.epi.ld_add_rows;
+  p.rows = a.epi.rows;
+  p.out_mapped = a.epi.out_mapped ? 1 : 0;
+  p.out = static_cast<bf16*>(a.epi.out); p.ld_out = a.epi.ld_out;
+  p.w2 = static_cast<const bf16*>(a.epi.w2); p.b2 = static_cast<const bf16*>(a.epi.b2);
+  p.scores = a.epi.scores;
+  p.err = dev.err;
+  p.timeout_ns = kWaitTimeoutNs;
+  const int64_t num_tiles = ((a.M + BM - 1) / BM) * ((a.N + BN - 1) / BN);
+  const int grid = (int)(num_tiles < dev.num_sms ? num_tiles : dev.num_sms);
+  gemm_tc_kernel<BN, DUAL, ROUTER><<<grid, kThreads, C::SMEM_BYTES, dev.stream>>>(ta, tb, tb2, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t gemm_bf16(const GemmArgs& a, const Dev& dev) {
+  if (a.M <= 0) return cudaSuccess;
+  if (a.epi.act == ACT_ROUTER) {
+    if (a.N != 64) return cudaErrorInvalidValue;
+    return launch<64, false, true>(a, dev);
+  }
+  if (a.epi.act == ACT_SWIGLU) return launch<128, true, false>(a, dev);
+  // Pick the N tile that finishes in the fewest tile-time units:
+  // ceil(tiles / SMs) waves, a 128-wide tile costing half a 256-wide one.
+  const int64_t mblocks = (a.M + BM - 1) / BM;
+  const int64_t t256 = mblocks * ((a.N + 255) / 256);
+  const int64_t t128 = mblocks * ((a.N + 127) / 128);
+  const int64_t w256 = (t256 + dev.num_sms - 1) / dev.num_sms;
+  const int64_t w128 = (t128 + dev.num_sms - 1) / dev.num_sms;
+  if (a.N % 256 == 0 && 2 * w256 <= w128) return launch<256, false, false>(a, dev);
+  return launch<128, false, false>(a, dev);
+}
+
+}  // namespace adadsf

@@ -1,0 +1,84 @@
+// Host-side declarations shared by the translation units of libadadsf.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <stddef.h>
+
+namespace adadsf {
+
+enum Dtype : int { kF32 = 0, kBF16 = 1 };
+// Bits of the device error word (first int of every workspace).
+enum : int { DEVERR_TIMEOUT = 1, DEVERR_INDEX = 2 };
+enum Act : int { ACT_NONE = 0, ACT_GELU = 1, ACT_SWIGLU = 2, ACT_ROUTER = 3 };
+
+// Epilogue of the projection kernels, applied to the fp32 accumulator
+// acc[m][n] of out = A[m,:] . W[n,:]:
+//   v = acc + bias[n]                         (bias may be null)
+//   v = gelu(v)                               (ACT_GELU)
+//   v = silu(acc) * acc2                      (ACT_SWIGLU, acc2 from the second weight)
+//   v += add_packed[m][n]                     (may be null)
+//   v += add_rows[row(m)][n]                  (may be null)
+//   out[out_mapped ? row(m) : m][n] = v       row(m) = rows ? rows[m] : m
+// ACT_ROUTER instead reduces each row to scores[m] = sum_n w2[n] silu(acc + bias[n]) + b2.
+struct Epilogue {
+  int act = ACT_NONE;
+  const void* bias = nullptr;
+  const void* add_packed = nullptr;
+  int64_t ld_add_packed = 0;
+  const void* add_rows = nullptr;
+  int64_t ld_add_rows = 0;
+  const int32_t* rows = nullptr;
+  bool out_mapped = true;
+  void* out = nullptr;
+  int64_t ld_out = 0;
+  const void* w2 = nullptr;   // router
+  const void* b2 = nullptr;   // router
+  float* scores = nullptr;    // router
+};
+
+struct GemmArgs {
+  const void* A = nullptr;  int64_t lda = 0;   // [M, K]
+  const void* W = nullptr;  int64_t ldw = 0;   // [N, K]
+  const void* W2 = nullptr;                    // [N, K] (ACT_SWIGLU: W = gate, W2 = up)
+  int64_t M = 0; int N = 0; int K = 0;
+  Epilogue epi;
+};
+
+struct Dev {
+  cudaStream_t stream;
+  int* err;          // device error word
+  int num_sms;
+};
+
+// gemm_tcgen05.cu -- bf16 tensor-core projections (tcgen05 + TMEM + TMA).
+cudaError_t gemm_bf16(const GemmArgs& a, const Dev& dev);
+// gemm_simt.cu -- fp32 projections on CUDA cores.
+cudaError_t gemm_f32(const GemmArgs& a, const Dev& dev);
+
+// attention.cu -- causal attention among kept tokens.
+cudaError_t attention(int dtype, const void* qkv, int64_t ld_qkv, void* out, int64_t ld_out, int B,
+                      int K, int n_heads, int n_kv_heads, int head_dim, const Dev& dev);
+
+// rowwise.cu
+cudaError_t embed(int dtype, const int32_t* ids, int64_t n, const void* table, int vocab, int d,
+                  void* out, const Dev& dev);
+// out1 = norm1(x[row(m)]), out2 = norm2(x[row(m)]) (out2 may be null); is_rms selects RMSNorm.
+cudaError_t gather_norm(int dtype, const void* x, const int32_t* rows, int64_t M, int d,
+                        bool is_rms, const void* g1, const void* b1, const void* g2,
+                        const void* b2, float eps, void* out1, void* out2, const Dev& dev);
+cudaError_t rope_table(float2* tab, int T, int rotary_dim, float theta, const Dev& dev);
+cudaError_t rope_apply(int dtype, void* qkv, int64_t M, int64_t ld, int n_heads, int n_kv_heads,
+                       int head_dim, int rotary_dim, const int32_t* pos, int T, const float2* tab,
+                       const Dev& dev);
+cudaError_t router_f32(const float* x, int64_t n, int d, int h, const float* w1, const float* b1,
+                       const float* w2, const float* b2, float* scores, const Dev& dev);
+cudaError_t topk(const float* scores, int B, int T, int K, int32_t* idx, int32_t* rows,
+                 const Dev& dev);
+int stats_partials_count(int64_t n_rows);
+cudaError_t iota_positions(int32_t* idx, int B, int K, const Dev& dev);
+cudaError_t cos_stats(int dtype, const void* a, const void* b, int64_t n_rows, int d, int mode,
+                      double* partials, double* acc, const Dev& dev);
+cudaError_t bounded_wait_selftest(int timeout_us, const Dev& dev);
+
+}  // namespace adadsf

@@ -1,0 +1,523 @@
+// Row-wise kernels of the depth-sparse layer: embedding, fused gather + norm,
+// rotary embedding at original positions, fp32 router, per-sequence Top-K,
+// the Eq. 4 similarity reduction, and the bounded-wait self-test.
+// All are HBM-bound: rows are moved as 16-byte vectors, one warp per row.
+#include "common.cuh"
+#include "internal.h"
+
+namespace adadsf {
+namespace {
+
+constexpr int kMaxChunks = 16;  // per-lane 16-byte vectors held in registers (d <= 16*32*vec)
+
+// ---------------------------------------------------------------- embedding
+template <typename T>
+__global__ void embed_kernel(const int32_t* ids, int64_t n, const T* table, int vocab, int d,
+                             T* out, int* err) {
+  constexpr int V = Elem<T>::kVec;
+  const int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (row >= n) return;
+  const int id = ids[row];
+  const bool ok = id >= 0 && id < vocab;
+  if (!ok && lane == 0) set_device_error(err, DEVERR_INDEX);
+  const int nv = d / V;
+  for (int c = lane; c < nv; c += 32) {
+    uint4 u = ok ? *reinterpret_cast<const uint4*>(table + (int64_t)id * d + c * V)
+                 : make_uint4(0, 0, 0, 0);
+    *reinterpret_cast<uint4*>(out + row * d + c * V) = u;
+  }
+}
+
+// ---------------------------------------------------------------- gather + norm
+// out1[m] = norm(x[row(m)]; g1, b1), out2[m] = norm(x[row(m)]; g2, b2).
+// LayerNorm: (x - mean) / sqrt(var + eps) * g + b (biased variance, two-pass
+// over the register-resident row); RMSNorm: x / sqrt(mean(x^2) + eps) * g.
+template <typename T, bool RMS>
+__global__ void gather_norm_kernel(const T* x, const int32_t* rows, int64_t M, int d, const T* g1,
+                                   const T* b1, const T* g2, const T* b2, float eps, T* out1,
+                                   T* out2) {
+  constexpr int V = Elem<T>::kVec;
+  const int64_t m = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (m >= M) return;
+  const int64_t src = rows ? (int64_t)rows[m] : m;
+  const int nv = d / V;
+  float v[kMaxChunks][V];
+  float s = 0.f;
+#pragma unroll
+  for (int c = 0; c < kMaxChunks; ++c) {
+    const int ci = c * 32 + lane;
+    if (ci < nv) {
+      load_vec(x + src * d + ci * V, v[c]);
+#pragma unroll
+      for (int j = 0; j < V; ++j) s += v[c][j];
+    }
+  }
+  float mean = 0.f, rstd;
+  if (!RMS) {
+    mean = warp_sum(s) / d;
+    float q = 0.f;
+#pragma unroll
+    for (int c = 0; c < kMaxChunks; ++c) {
+      const int ci = c * 32 + lane;
+      if (ci < nv) {
+#pragma unroll
+        for (int j = 0; j < V; ++j) {
+          const float t = v[c][j] - mean;
+          q += t * t;
+        }
+      }
+    }
+    rstd = 1.f / sqrtf(warp_sum(q) / d + eps);
+  } else {
+    float q = 0.f;
+#pragma unroll
+    for (int c = 0; c < kMaxChunks; ++c) {
+      const int ci = c * 32 + lane;
+      if (ci < nv) {
+#pragma unroll
+        for (int j = 0; j < V; ++j) q += v[c][j] * v[c][j];
+      }
+    }
+    rstd = 1.f / sqrtf(warp_sum(q) / d + eps);
+  }
+#pragma unroll
+  for (int c = 0; c < kMaxChunks; ++c) {
+    const int ci = c * 32 + lane;
+    if (ci < nv) {
+      float g[V], b[V], o[V];
+      load_vec(g1 + ci * V, g);
+      if (!RMS) load_vec(b1 + ci * V, b);
+#pragma unroll
+      for (int j = 0; j < V; ++j) o[j] = (v[c][j] - mean) * rstd * g[j] + (RMS ? 0.f : b[j]);
+      store_vec(out1 + m * d + ci * V, o);
+      if (out2) {
+        load_vec(g2 + ci * V, g);
+        if (!RMS) load_vec(b2 + ci * V, b);
+#pragma unroll
+        for (int j = 0; j < V; ++j) o[j] = (v[c][j] - mean) * rstd * g[j] + (RMS ? 0.f : b[j]);
+        store_vec(out2 + m * d + ci * V, o);
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------- rotary embedding
+// tab[p * half + i] = (cos, sin) of p * theta^(-2i / rotary_dim), evaluated in
+// fp64 and rounded once to fp32.
+__global__ void rope_table_kernel(float2* tab, int T, int half, int rotary_dim, double theta) {
+  const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= (int64_t)T * half) return;
+  const int p = (int)(k / half), i = (int)(k % half);
+  const double inv = pow(theta, -2.0 * i / rotary_dim);
+  double s, c;
+  sincos((double)p * inv, &s, &c);
+  tab[k] = make_float2((float)c, (float)s);
+}
+
+// Rotates, in place, the first rotary_dim features of every query and key
+// head of row m at position pos[m] (or m % T when pos is null): feature i pairs
+// with i + rotary_dim/2.
+template <typename T>
+__global__ void rope_apply_kernel(T* qkv, int64_t M, int64_t ld, int heads, int head_dim,
+                                  int half, const int32_t* pos, int seq_len, const float2* tab) {
+  const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t per_row = (int64_t)heads * half;
+  if (k >= M * per_row) return;
+  const int64_t m = k / per_row;
+  const int r = (int)(k % per_row);
+  const int h = r / half, i = r % half;
+  const int p = pos ? pos[m] : (int)(m % seq_len);
+  const float2 cs = tab[(int64_t)p * half + i];
+  T* base = qkv + m * ld + (int64_t)h * head_dim;
+  const float a = Elem<T>::to_f(base[i]);
+  const float b = Elem<T>::to_f(base[i + half]);
+  base[i] = Elem<T>::from_f(a * cs.x - b * cs.y);
+  base[i + half] = Elem<T>::from_f(b * cs.x + a * cs.y);
+}
+
+// ---------------------------------------------------------------- fp32 router (Sec. 3.4)
+// One warp per token: score = sum_j w2[j] * silu(w1[j] . x + b1[j]) + b2.
+__global__ void router_f32_kernel(const float* x, int64_t n, int d, int h, const float* w1,
+                                  const float* b1, const float* w2, const float* b2,
+                                  float* scores) {
+  const int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+  const int lane = threadIdx.x & 31;
+  if (row >= n) return;
+  const float* xr = x + row * d;
+  float s = 0.f;
+  for (int j = 0; j < h; ++j) {
+    const float* wr = w1 + (int64_t)j * d;
+    float dot = 0.f;
+    for (int c = lane * 4; c < d; c += 128) {
+      const float4 a = *reinterpret_cast<const float4*>(xr + c);
+      const float4 b = *reinterpret_cast<const float4*>(wr + c);
+      dot = fmaf(a.x, b.x, fmaf(a.y, b.y, fmaf(a.z, b.z, fmaf(a.w, b.w, dot))));
+    }
+    const float u = warp_sum(dot) + b1[j];
+    s += w2[j] * (u / (1.f + expf(-u)));
+  }
+  if (lane == 0) scores[row] = s + b2[0];
+}
+
+// ---------------------------------------------------------------- Top-K (Sec. 3.4)
+// Order-preserving key of an fp32 score: larger score -> larger key; -0.0 is
+// folded onto +0.0; NaN maps to 0, below every number (-inf maps to 0x007FFFFF).
+__device__ __forceinline__ uint32_t score_key(float f) {
+  if (f != f) return 0u;
+  uint32_t u = __float_as_uint(f);
+  if ((u << 1) == 0u) u = 0u;   // -0.0 -> +0.0
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// Exclusive prefix sum over the block (blockDim.x == 1024) of one int per
+// thread; also returns the block total.
+__device__ __forceinline__ int block_excl_scan(int v, int* warp_tot, int& total) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  int incl = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int t = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  if (lane == 31) warp_tot[w] = incl;
+  __syncthreads();
+  if (w == 0) {
+    int t = warp_tot[lane];
+    int ti = t;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int u = __shfl_up_sync(0xffffffffu, ti, o);
+      if (lane >= o) ti += u;
+    }
+    warp_tot[lane] = ti - t;        // exclusive prefix of warp totals
+    if (lane == 31) warp_tot[32] = ti;
+  }
+  __syncthreads();
+  const int res = warp_tot[w] + incl - v;
+  total = warp_tot[32];
+  __syncthreads();
+  return res;
+}
+
+constexpr int kTopkThreads = 1024;
+
+// One block per sequence. Radix select (4 passes of 8 bits, most significant
+// first) finds the K-th largest key kth and how many keys equal to it are
+// kept (need_eq, lowest positions first); two block scans then emit the kept
+// positions in ascending order.
+__global__ void __launch_bounds__(kTopkThreads) topk_kernel(const float* scores, int T, int K,
+                                                            int32_t* idx, int32_t* rows) {
+  extern __shared__ uint32_t keys[];
+  __shared__ int hist[256];
+  __shared__ int warp_tot[33];
+  __shared__ uint32_t s_digit;
+  __shared__ int s_remaining;
+  const int b = blockIdx.x;
+  const float* sc = scores + (int64_t)b * T;
+  for (int t = threadIdx.x; t < T; t += kTopkThreads) keys[t] = score_key(sc[t]);
+
+  uint32_t prefix = 0, pmask = 0;
+  int remaining = K;   // keys still to take at or below the current prefix
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 24 - 8 * pass;
+    if (threadIdx.x < 256) hist[threadIdx.x] = 0;
+    __syncthreads();
+    for (int t = threadIdx.x; t < T; t += kTopkThreads) {
+      const uint32_t k = keys[t];
+      if ((k & pmask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1);
+    }
+    __syncthreads();
+    if (threadIdx.x < 32) {
+      // lane l owns digits 255-8l .. 248-8l (descending)
+      const int lane = threadIdx.x;
+      int cnt[8], lsum = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        cnt[j] = hist[255 - 8 * lane - j];
+        lsum += cnt[j];
+      }
+      int incl = lsum;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += t;
+      }
+      const int excl = incl - lsum;   // keys with a larger digit than this lane's
+      const bool here = excl < remaining && incl >= remaining;
+      if (here) {
+        int above = excl;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if (above + cnt[j] >= remaining) {
+            s_digit = (uint32_t)(255 - 8 * lane - j);
+            s_remaining = remaining - above;
+            break;
+          }
+          above += cnt[j];
+        }
+      }
+    }
+    __syncthreads();
+    prefix |= s_digit << shift;
+    pmask |= 255u << shift;
+    remaining = s_remaining;
+    __syncthreads();
+  }
+  const uint32_t kth = prefix;
+  const int need_eq = remaining;
+
+  // Contiguous chunk of positions per thread keeps the output ascending.
+  const int chunk = (T + kTopkThreads - 1) / kTopkThreads;
+  const int t0 = min(T, threadIdx.x * chunk), t1 = min(T, t0 + chunk);
+  int n_eq = 0;
+  for (int t = t0; t < t1; ++t) n_eq += keys[t] == kth;
+  int total;
+  const int eq_base = block_excl_scan(n_eq, warp_tot, total);   // equal keys before my chunk
+  int n_sel = 0, er = eq_base;
+  for (int t = t0; t < t1; ++t) {
+    const uint32_t k = keys[t];
+    if (k > kth) {
+      ++n_sel;
+    } else if (k == kth) {
+      n_sel += er < need_eq;
+      ++er;
+    }
+  }
+  int out = block_excl_scan(n_sel, warp_tot, total);
+  er = eq_base;
+  for (int t = t0; t < t1; ++t) {
+    const uint32_t k = keys[t];
+    bool take = k > kth;
+    if (k == kth) {
+      take = er < need_eq;
+      ++er;
+    }
+    if (take) {
+      idx[(int64_t)b * K + out] = t;
+      if (rows) rows[(int64_t)b * K + out] = b * T + t;
+      ++out;
+    }
+  }
+}
+
+// ---------------------------------------------------------------- Eq. 4 statistics
+constexpr int kStatThreads = 256;
+
+// One warp per row: fp32 sums a.b, |a|^2, |b|^2; per block fixed-order fp64
+// sums of either the row cosines (TOKEN) or the three sums (FLAT).
+template <typename T>
+__global__ void __launch_bounds__(kStatThreads) cos_rows_kernel(const T* a, const T* b,
+                                                                int64_t n_rows, int d, int mode,
+                                                                double* partials) {
+  constexpr int V = Elem<T>::kVec;
+  __shared__ double red[kStatThreads / 32][3];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int64_t nwarps = (int64_t)gridDim.x * (kStatThreads / 32);
+  double acc0 = 0, acc1 = 0, acc2 = 0;
+  for (int64_t r = (int64_t)blockIdx.x * (kStatThreads / 32) + w; r < n_rows; r += nwarps) {
+    float dot = 0.f, na = 0.f, nb = 0.f;
+    for (int c = lane * V; c < d; c += 32 * V) {
+      float fa[V], fb[V];
+      load_vec(a + r * d + c, fa);
+      load_vec(b + r * d + c, fb);
+#pragma unroll
+      for (int j = 0; j < V; ++j) {
+        dot = fmaf(fa[j], fb[j], dot);
+        na = fmaf(fa[j], fa[j], na);
+        nb = fmaf(fb[j], fb[j], nb);
+      }
+    }
+    dot = warp_sum(dot);
+    na = warp_sum(na);
+    nb = warp_sum(nb);
+    if (mode == 0) {
+      const double den = fmax(sqrt((double)na), 1e-8) * fmax(sqrt((double)nb), 1e-8);
+      acc0 += (double)dot / den;
+    } else {
+      acc0 += dot; acc1 += na; acc2 += nb;
+    }
+  }
+  if (lane == 0) { red[w][0] = acc0; red[w][1] = acc1; red[w][2] = acc2; }
+  __syncthreads();
+  if (threadIdx.x < 3) {
+    double s = 0;
+    for (int i = 0; i < kStatThreads / 32; ++i) s += red[i][threadIdx.x];
+    partials[(int64_t)blockIdx.x * 3 + threadIdx.x] = s;
+  }
+}
+
+// Fixed-order sum of the per-block partials, added to acc.
+__global__ void cos_finish_kernel(const double* partials, int nblocks, int64_t n_rows, int mode,
+                                  double* acc) {
+  __shared__ double red[3][256];
+  double s[3] = {0, 0, 0};
+  for (int i = threadIdx.x; i < nblocks; i += 256)
+    for (int j = 0; j < 3; ++j) s[j] += partials[(int64_t)i * 3 + j];
+  for (int j = 0; j < 3; ++j) red[j][threadIdx.x] = s[j];
+  __syncthreads();
+  for (int o = 128; o > 0; o >>= 1) {
+    if (threadIdx.x < o)
+      for (int j = 0; j < 3; ++j) red[j][threadIdx.x] += red[j][threadIdx.x + o];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    if (mode == 0) {
+      acc[0] += red[0][0];
+      acc[1] += (double)n_rows;
+    } else {
+      acc[0] += red[0][0]; acc[1] += red[1][0]; acc[2] += red[2][0];
+    }
+  }
+}
+
+// idx[b * K + j] = j: the kept positions of a dense layer.
+__global__ void iota_kernel(int32_t* idx, int64_t n, int K) {
+  const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (k < n) idx[k] = (int32_t)(k % K);
+}
+
+// ---------------------------------------------------------------- bounded-wait self-test
+__global__ void bounded_wait_selftest_kernel(int* err, unsigned long long timeout_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(smem_u32(&bar), 1);
+    abort_flag = 0;
+    fence_barrier_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    // Nothing ever arrives: the wait must give up and flag the error word.
+    mbar_wait_bounded(smem_u32(&bar), 0, &abort_flag, err, timeout_ns);
+  }
+  __syncthreads();
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------- launchers
+static unsigned blocks_for(int64_t rows, int rows_per_block) {
+  return (unsigned)((rows + rows_per_block - 1) / rows_per_block);
+}
+
+cudaError_t embed(int dtype, const int32_t* ids, int64_t n, const void* table, int vocab, int d,
+                  void* out, const Dev& dev) {
+  if (n <= 0) return cudaSuccess;
+  if (dtype == kBF16)
+    embed_kernel<bf16><<<blocks_for(n, 8), 256, 0, dev.stream>>>(
+        ids, n, static_cast<const bf16*>(table), vocab, d, static_cast<bf16*>(out), dev.err);
+  else
+    embed_kernel<float><<<blocks_for(n, 8), 256, 0, dev.stream>>>(
+        ids, n, static_cast<const float*>(table), vocab, d, static_cast<float*>(out), dev.err);
+  return cudaGetLastError();
+}
+
+cudaError_t gather_norm(int dtype, const void* x, const int32_t* rows, int64_t M, int d,
+                        bool is_rms, const void* g1, const void* b1, const void* g2,
+                        const void* b2, float eps, void* out1, void* out2, const Dev& dev) {
+  if (M <= 0) return cudaSuccess;
+  const unsigned grid = blocks_for(M, 8);
+#define GN_LAUNCH(T, R)                                                                        \
+  gather_norm_kernel<T, R><<<grid, 256, 0, dev.stream>>>(                                      \
+      static_cast<const T*>(x), rows, M, d, static_cast<const T*>(g1),                         \
+      static_cast<const T*>(b1), static_cast<const T*>(g2), static_cast<const T*>(b2), eps,   \
+      static_cast<T*>(out1), static_cast<T*>(out2))
+  if (dtype == kBF16) {
+    if (is_rms) GN_LAUNCH(bf16, true); else GN_LAUNCH(bf16, false);
+  } else {
+    if (is_rms) GN_LAUNCH(float, true); else GN_LAUNCH(float, false);
+  }
+#undef GN_LAUNCH
+  return cudaGetLastError();
+}
+
+cudaError_t rope_table(float2* tab, int T, int rotary_dim, float theta, const Dev& dev) {
+  const int half = rotary_dim / 2;
+  const int64_t n = (int64_t)T * half;
+  if (n <= 0) return cudaSuccess;
+  rope_table_kernel<<<(unsigned)((n + 255) / 256), 256, 0, dev.stream>>>(tab, T, half, rotary_dim,
+                                                                          (double)theta);
+  return cudaGetLastError();
+}
+
+cudaError_t rope_apply(int dtype, void* qkv, int64_t M, int64_t ld, int n_heads, int n_kv_heads,
+                       int head_dim, int rotary_dim, const int32_t* pos, int T, const float2* tab,
+                       const Dev& dev) {
+  const int half = rotary_dim / 2;
+  const int heads = n_heads + n_kv_heads;   // query heads then key heads are contiguous
+  const int64_t n = M * heads * half;
+  if (n <= 0) return cudaSuccess;
+  const unsigned grid = (unsigned)((n + 255) / 256);
+  if (dtype == kBF16)
+    rope_apply_kernel<bf16><<<grid, 256, 0, dev.stream>>>(static_cast<bf16*>(qkv), M, ld, heads,
+                                                          head_dim, half, pos, T, tab);
+  else
+    rope_apply_kernel<float><<<grid, 256, 0, dev.stream>>>(static_cast<float*>(qkv), M, ld, heads,
+                                                           head_dim, half, pos, T, tab);
+  return cudaGetLastError();
+}
+
+cudaError_t router_f32(const float* x, int64_t n, int d, int h, const float* w1, const float* b1,
+                       const float* w2, const float* b2, float* scores, const Dev& dev) {
+  if (n <= 0) return cudaSuccess;
+  router_f32_kernel<<<blocks_for(n, 8), 256, 0, dev.stream>>>(x, n, d, h, w1, b1, w2, b2, scores);
+  return cudaGetLastError();
+}
+
+cudaError_t topk(const float* scores, int B, int T, int K, int32_t* idx, int32_t* rows,
+                 const Dev& dev) {
+  if (B <= 0 || K <= 0) return cudaSuccess;
+  const size_t smem = (size_t)T * sizeof(uint32_t);
+  static int attr_done[64] = {0};
+  int device = 0;
+  cudaGetDevice(&device);
+  if (device < 64 && !attr_done[device]) {
+    cudaError_t e = cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         16384 * (int)sizeof(uint32_t));
+    if (e != cudaSuccess) return e;
+    attr_done[device] = 1;
+  }
+  topk_kernel<<<B, kTopkThreads, smem, dev.stream>>>(scores, T, K, idx, rows);
+  return cudaGetLastError();
+}
+
+// Fixed block count for a given row count (independent of the device), so the
+// fixed-order sums are reproducible everywhere.
+int stats_partials_count(int64_t n_rows) {
+  const int64_t want = (n_rows + (kStatThreads / 32) - 1) / (kStatThreads / 32);
+  const int64_t cap = 2048;
+  return (int)(want < cap ? (want > 0 ? want : 1) : cap);
+}
+
+cudaError_t cos_stats(int dtype, const void* a, const void* b, int64_t n_rows, int d, int mode,
+                      double* partials, double* acc, const Dev& dev) {
+  if (n_rows <= 0) return cudaSuccess;
+  const int nb = stats_partials_count(n_rows);
+  if (dtype == kBF16)
+    cos_rows_kernel<bf16><<<nb, kStatThreads, 0, dev.stream>>>(
+        static_cast<const bf16*>(a), static_cast<const bf16*>(b), n_rows, d, mode, partials);
+  else
+    cos_rows_kernel<float><<<nb, kStatThreads, 0, dev.stream>>>(
+        static_cast<const float*>(a), static_cast<const float*>(b), n_rows, d, mode, partials);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  cos_finish_kernel<<<1, 256, 0, dev.stream>>>(partials, nb, n_rows, mode, acc);
+  return cudaGetLastError();
+}
+
+cudaError_t iota_positions(int32_t* idx, int B, int K, const Dev& dev) {
+  const int64_t n = (int64_t)B * K;
+  if (n <= 0) return cudaSuccess;
+  iota_kernel<<<(unsigned)((n + 255) / 256), 256, 0, dev.stream>>>(idx, n, K);
+  return cudaGetLastError();
+}
+
+cudaError_t bounded_wait_selftest(int timeout_us, const Dev& dev) {
+  bounded_wait_selftest_kernel<<<1, 32, 0, dev.stream>>>(dev.err,
+                                                         (unsigned long long)timeout_us * 1000ull);
+  return cudaGetLastError();
+}
+
+}  // namespace adadsf

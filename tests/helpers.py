@@ -1,0 +1,74 @@
+"""Shared helpers of the GPU parity tests: device copies of seeded inputs and
+error measures. Inputs come from paper_2607_21291_gb300.synth; expected values
+come from the oracle only."""
+import numpy as np
+import torch
+
+from oracle import adadsf_oracle as O
+from paper_2607_21291_gb300 import synth as S
+
+BF16_TOL = 2e-2     # max |gpu - oracle| / max |oracle| for bf16 storage
+F32_TOL = 1e-4      # same, fp32 storage
+
+
+def tdtype(shape):
+    return torch.bfloat16 if shape.dtype == "bf16" else torch.float32
+
+
+def tol(shape):
+    return BF16_TOL if shape.dtype == "bf16" else F32_TOL
+
+
+def max_rel(got, ref):
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    return float(np.max(np.abs(got - ref)) / max(float(np.max(np.abs(ref))), 1e-30))
+
+
+def rel_rms(got, ref):
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    return float(np.sqrt(np.mean((got - ref) ** 2)) / max(np.sqrt(np.mean(ref ** 2)), 1e-30))
+
+
+def host_layer(shape, seed, layer=0, gain_std=0.1):
+    """Seeded layer weights rounded to the storage dtype (float32 arrays)."""
+    return {k: S.round_to(v, shape.dtype) for k, v in S.layer_weights(shape, seed, layer, gain_std).items()}
+
+
+def host_extra(shape, seed, gain_std=0.1):
+    return {k: S.round_to(v, shape.dtype) for k, v in S.model_extra_weights(shape, seed, gain_std).items()}
+
+
+def f64(d):
+    return {k: v.astype(np.float64) for k, v in d.items()}
+
+
+def to_dev(a, dtype, device="cuda"):
+    return torch.from_numpy(np.ascontiguousarray(a)).to(device=device, dtype=dtype)
+
+
+def to_np(t):
+    return t.detach().float().cpu().numpy().astype(np.float64)
+
+
+def score_gap(scores, K):
+    """score_(K) - score_(K+1) of one sequence (inf when K is 0 or T)."""
+    s = np.sort(np.asarray(scores, dtype=np.float64))[::-1]
+    if K <= 0 or K >= len(s):
+        return np.inf
+    return s[K - 1] - s[K]
+
+
+def check_kept_sets(gpu_scores, gpu_idx, ref_scores, K):
+    """North-star kept-set rules: (1) the oracle's Top-K of the GPU scores is
+    the GPU's kept set, bit for bit; (2) from the raw (oracle) scores the kept
+    set is identical wherever the K-th/(K+1)-th gap exceeds 1e-3.
+    Returns the number of sequences checked under rule (2)."""
+    n2 = 0
+    for b in range(gpu_idx.shape[0]):
+        assert O.topk_keep(gpu_scores[b], K).tolist() == gpu_idx[b].tolist(), f"seq {b}: rule 1"
+        if score_gap(ref_scores[b], K) > 1e-3:
+            n2 += 1
+            assert O.topk_keep(ref_scores[b], K).tolist() == gpu_idx[b].tolist(), f"seq {b}: rule 2"
+    return n2
