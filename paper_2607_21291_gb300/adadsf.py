@@ -48,6 +48,11 @@ class ModelWeights(ctypes.Structure):
                 ("final_b", ctypes.c_void_p), ("layers", ctypes.POINTER(LayerWeights))]
 
 
+class LaunchRecord(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int32), ("dense", ctypes.c_int32), ("ms", ctypes.c_double),
+                ("flops", ctypes.c_double), ("bytes", ctypes.c_double)]
+
+
 class AdadsfError(RuntimeError):
     def __init__(self, status: int, msg: str):
         super().__init__(f"adadsf status {status}: {msg}")
@@ -83,6 +88,9 @@ def lib() -> ctypes.CDLL:
             "adadsf_sparse_model_forward": (i32, [pcfg, pmw, vp, i32, i32, vp, vp, vp, vp, vp, sz, vp]),
             "adadsf_sync_check": (i32, [vp, sz, vp]),
             "adadsf_selftest_bounded_wait": (i32, [vp, sz, i32, vp]),
+            "adadsf_profile_begin": (i32, [i32]),
+            "adadsf_profile_end": (i32, [ctypes.POINTER(LaunchRecord), i32]),
+            "adadsf_kernel_name": (ctypes.c_char_p, [i32]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -279,3 +287,21 @@ def adadsf_sync_check(ws: torch.Tensor, stream=None) -> int:
 
 def adadsf_selftest_bounded_wait(ws: torch.Tensor, timeout_us: int, stream=None):
     _check(lib().adadsf_selftest_bounded_wait(_p(ws), ws.numel(), int(timeout_us), _s(stream)))
+
+
+def adadsf_profile_begin(max_launches: int = 65536):
+    """Start bracketing every library launch with CUDA events."""
+    _check(lib().adadsf_profile_begin(int(max_launches)))
+
+
+def adadsf_profile_end(max_records: int = 65536) -> list:
+    """Stop profiling; returns [(kernel name, dense, ms, flops, bytes), ...] in launch order."""
+    buf = (LaunchRecord * max_records)()
+    n = lib().adadsf_profile_end(buf, max_records)
+    if n < 0:
+        raise AdadsfError(ERR_CUDA, adadsf_last_error())
+    return [(adadsf_kernel_name(r.kind), bool(r.dense), r.ms, r.flops, r.bytes) for r in buf[:min(n, max_records)]]
+
+
+def adadsf_kernel_name(kind: int) -> str:
+    return lib().adadsf_kernel_name(int(kind)).decode()
