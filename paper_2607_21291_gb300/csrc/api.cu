@@ -123,6 +123,7 @@ struct Profiler {
   int cap = 0;
   std::vector<cudaEvent_t> ev;   // two per record
   std::vector<adadsf_launch_record> recs;
+  std::vector<int> rec_err;       // cudaEventRecord status of each record
 };
 Profiler g_prof;
 
@@ -131,6 +132,7 @@ Profiler g_prof;
 template <typename F>
 adadsf_status launch(const Dev& dev, int kind, bool dense, double flops, double bytes, F&& f) {
   cudaEvent_t a = nullptr, b = nullptr;
+  size_t slot = 0;
   if (g_prof.on) {
     cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
     if (cudaStreamIsCapturing(dev.stream, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusNone) {
@@ -140,12 +142,18 @@ adadsf_status launch(const Dev& dev, int kind, bool dense, double flops, double 
         a = g_prof.ev[2 * i];
         b = g_prof.ev[2 * i + 1];
         g_prof.recs.push_back({kind, dense ? 1 : 0, 0.0, flops, bytes});
+        g_prof.rec_err.push_back(0);
+        slot = i;
       }
     }
   }
-  if (a) cudaEventRecord(a, dev.stream);
+  const cudaError_t ea = a ? cudaEventRecord(a, dev.stream) : cudaSuccess;
   const adadsf_status st = f();
-  if (b) cudaEventRecord(b, dev.stream);
+  const cudaError_t eb = b ? cudaEventRecord(b, dev.stream) : cudaSuccess;
+  if (ea != cudaSuccess || eb != cudaSuccess) {
+    std::lock_guard<std::mutex> lk(g_prof.mu);
+    g_prof.rec_err[slot] = ea != cudaSuccess ? (int)ea : (int)eb;
+  }
   return st;
 }
 
@@ -779,6 +787,7 @@ adadsf_status adadsf_profile_begin(int max_launches) {
   }
   g_prof.cap = max_launches;
   g_prof.recs.clear();
+  g_prof.rec_err.clear();
   g_prof.on = true;
   return ADADSF_OK;
 }
@@ -798,8 +807,9 @@ int adadsf_profile_end(adadsf_launch_record* out_host, int max) {
   for (int i = 0; i < n && i < max && out_host; ++i) {
     adadsf_launch_record r = g_prof.recs[i];
     float ms = 0.f;
-    if (cudaEventElapsedTime(&ms, g_prof.ev[2 * i], g_prof.ev[2 * i + 1]) != cudaSuccess) ms = -1.f;
-    r.ms = ms;
+    const cudaError_t e = cudaEventElapsedTime(&ms, g_prof.ev[2 * i], g_prof.ev[2 * i + 1]);
+    // failures are reported as negative times: -(1000 + record error) or -(2000 + query error)
+    r.ms = g_prof.rec_err[i] ? -(1000.0 + g_prof.rec_err[i]) : (e != cudaSuccess ? -(2000.0 + (int)e) : ms);
     out_host[i] = r;
   }
   return n;

@@ -1,0 +1,129 @@
+"""Micro-benchmark of single library entry points on seeded synthetic inputs.
+
+  python -m paper_2607_21291_gb300.kernel_bench linear --M 8192 --N 8192 --K 2048
+  python -m paper_2607_21291_gb300.kernel_bench layer --workload c3 --B 2
+  python -m paper_2607_21291_gb300.kernel_bench attention --workload c5 --B 1 --K 2048
+
+Each case runs `--warmup` untimed calls, then `--iters` calls each bracketed by
+CUDA events on the launching stream (L2 flushed between calls by a 256 MiB
+write), and prints one JSON line with the mean time and the algorithmic
+TFLOP/s or GB/s. This is also the command the ncu captures run.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+
+import torch
+
+from . import adadsf as A
+from . import synth as S
+
+
+def _time(fn, iters, warmup, stream):
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    for _ in range(warmup):
+        fn()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(iters)]
+    torch.cuda.synchronize()
+    for e0, e1 in ev:
+        flush.zero_()
+        e0.record(stream)
+        fn()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    return sum(e0.elapsed_time(e1) for e0, e1 in ev) / iters
+
+
+def _profile(fn, stream):
+    """One call under the library's per-launch timing."""
+    torch.cuda.synchronize()
+    A.adadsf_profile_begin(4096)
+    fn()
+    return A.adadsf_profile_end(4096)
+
+
+def case_linear(a, stream):
+    g = torch.Generator(device="cuda").manual_seed(0)
+    dt = torch.bfloat16 if a.dtype == "bf16" else torch.float32
+    x = torch.randn(a.M, a.K, generator=g, device="cuda").to(dt)
+    w = (0.02 * torch.randn(a.N, a.K, generator=g, device="cuda")).to(dt)
+    b = (0.02 * torch.randn(a.N, generator=g, device="cuda")).to(dt)
+    out = torch.empty(a.M, a.N, device="cuda", dtype=dt)
+    ws = A.workspace(256)
+    fn = lambda: A.adadsf_linear(x, w, b, out, act=a.act, ws=ws, stream=stream)
+    flops = 2.0 * a.M * a.N * a.K
+    return fn, flops, (a.M * a.K + a.N * a.K + a.M * a.N) * x.element_size(), ws
+
+
+def case_layer(a, stream):
+    wl = S.WORKLOADS[a.workload]
+    shape = wl.shape.replace(n_layers=1)
+    B = a.B or wl.B
+    T = a.T or wl.T
+    K = a.K if a.K is not None else T // 2
+    dt = torch.bfloat16 if shape.dtype == "bf16" else torch.float32
+    g = torch.Generator(device="cuda").manual_seed(0)
+    w = {n: (0.02 * torch.randn(shp, generator=g, device="cuda")).to(dt)
+         for n, shp in S.layer_weight_shapes(shape).items()}
+    for n in ("ln1_w", "ln2_w"):
+        w[n] = torch.ones_like(w[n])
+    x = torch.randn(B, T, shape.d, generator=g, device="cuda").to(dt)
+    cfg = A.make_cfg(shape)
+    ws = A.workspace(A.adadsf_layer_workspace_size(cfg, B, T, K))
+    fn = lambda: A.adadsf_sparse_layer_forward(cfg, w, x, K, ws=ws, stream=stream)
+    per_tok = 2.0 * (shape.qkv_dim * shape.d + shape.d * shape.q_dim
+                     + (3 if shape.arch == S.QWEN else 2) * shape.d * shape.ffn)
+    flops = B * K * per_tok + 2.0 * B * shape.n_heads * shape.head_dim * K * (K + 1)
+    return fn, flops, 0.0, ws
+
+
+def case_attention(a, stream):
+    wl = S.WORKLOADS[a.workload]
+    shape = wl.shape
+    B = a.B or wl.B
+    K = a.K or wl.T // 2
+    dt = torch.bfloat16 if shape.dtype == "bf16" else torch.float32
+    g = torch.Generator(device="cuda").manual_seed(0)
+    qkv = torch.randn(B * K, shape.qkv_dim, generator=g, device="cuda").to(dt)
+    out = torch.empty(B * K, shape.q_dim, device="cuda", dtype=dt)
+    cfg = A.make_cfg(shape)
+    fn = lambda: A.adadsf_causal_attention(cfg, qkv, B, K, out, stream=stream)
+    flops = 2.0 * B * shape.n_heads * shape.head_dim * K * (K + 1)
+    return fn, flops, (qkv.numel() + out.numel()) * qkv.element_size(), None
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("case", choices=("linear", "layer", "attention"))
+    ap.add_argument("--M", type=int, default=8192)
+    ap.add_argument("--N", type=int, default=8192)
+    ap.add_argument("--K", type=int, default=None)
+    ap.add_argument("--T", type=int, default=None)
+    ap.add_argument("--B", type=int, default=None)
+    ap.add_argument("--act", type=int, default=0)
+    ap.add_argument("--dtype", default="bf16")
+    ap.add_argument("--workload", default="c3")
+    ap.add_argument("--iters", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--profile", action="store_true", help="also report the library's per-launch events")
+    a = ap.parse_args()
+    if a.case == "linear" and a.K is None:
+        a.K = 2048
+    A.lib()
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        fn, flops, nbytes, ws = {"linear": case_linear, "layer": case_layer, "attention": case_attention}[a.case](a, stream)
+        ms = _time(fn, a.iters, a.warmup, stream)
+        out = {"case": a.case, "ms": ms, "tflops": flops / (ms * 1e9)}
+        if nbytes:
+            out["gbs"] = nbytes / (ms * 1e6)
+        if a.profile:
+            out["launches"] = [(n, ms_, fl / max(ms_, 1e-9) / 1e9) for n, _, ms_, fl, _ in _profile(fn, stream)]
+        if ws is not None:
+            out["device_status"] = A.adadsf_sync_check(ws, stream)
+    print(json.dumps(out))
+
+
+if __name__ == "__main__":
+    main()
