@@ -131,6 +131,34 @@ adadsf_status adadsf_layer_stats(const void *x_in_dev, const void *x_out_dev, in
                                  void *ws, size_t ws_bytes, void *stream);
 
 /* ------------------------------------------------------------------------
+ * Workspace-free variant of adadsf_layer_stats. The paper has no counterpart:
+ * it exists for callers that cannot give the library any device memory of
+ * their own -- hosts whose GPU memory is entirely owned by another allocator
+ * or a pre-reserved pool, plugins that are handed only their input and
+ * output buffers, and latency-critical paths where a cudaMalloc (and the
+ * synchronisation it may imply) is not acceptable.
+ * Same arguments, semantics and results as adadsf_layer_stats, without
+ * (ws, ws_bytes): the per-block partial sums go to a fixed 48 KiB array
+ * (2048 slots of three doubles, a file-scope static __device__ array in the
+ * library) that every GPU which loads the library holds until the process
+ * exits. Nothing is allocated: no cudaMalloc, cudaFree or allocating library
+ * call.
+ * Set-up: the first call on each device looks up the array's device address
+ * (cudaGetSymbolAddress) with that device current and caches it; make that
+ * first call before any stream capture.
+ * The array is shared by every call and keeps the last call's contents. Each
+ * call writes every slot it later reads, so nothing needs clearing, but
+ * calls whose kernels overlap on the GPU (other streams, other host threads)
+ * race on the array and return wrong sums: serialise them.
+ * Limits: n_rows <= 2^31 - 1 and d <= 65536 (the reduction uses at most 2048
+ * blocks, so the 2048 slots always suffice); larger sizes return
+ * ADADSF_ERR_UNSUPPORTED before any launch.
+ * ---------------------------------------------------------------------- */
+adadsf_status adadsf_layer_stats_noalloc(const void *x_in_dev, const void *x_out_dev,
+                                         int64_t n_rows, int d, int dtype, int mode,
+                                         double *acc_dev, void *stream);
+
+/* ------------------------------------------------------------------------
  * Sec. 3.3, Eqs. 5-8: layer-wise retention ratios from the similarity vector,
  * then K_l = floor(r_l T) (Sec. 3.4). Host only, pure, no device work.
  * s_host[L] similarities; t target mean retention in [0,1]; tau > 0; beta > 0.

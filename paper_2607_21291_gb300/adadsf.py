@@ -79,6 +79,7 @@ def lib() -> ctypes.CDLL:
             "adadsf_model_workspace_size": (sz, [pcfg, i32, i32, vp, i32]),
             "adadsf_stats_workspace_size": (sz, [i64]),
             "adadsf_layer_stats": (i32, [vp, vp, i64, i32, i32, i32, vp, vp, sz, vp]),
+            "adadsf_layer_stats_noalloc": (i32, [vp, vp, i64, i32, i32, i32, vp, vp]),
             "adadsf_alloc_ratios": (i32, [vp, i32, f64, f64, f64, i32, u32, vp, vp]),
             "adadsf_router_scores": (i32, [pcfg, plw, vp, i64, vp, vp, sz, vp]),
             "adadsf_topk_select": (i32, [vp, i32, i32, i32, vp, vp, vp]),
@@ -187,6 +188,20 @@ def adadsf_layer_stats(x_in: torch.Tensor, x_out: torch.Tensor, acc: torch.Tenso
         ws = workspace(adadsf_stats_workspace_size(n), x_in.device)
     _check(lib().adadsf_layer_stats(_p(x_in), _p(x_out), n, d, DTYPE_CODE[x_in.dtype], mode,
                                     _p(acc), _p(ws), ws.numel(), _s(stream)))
+
+
+def adadsf_layer_stats_noalloc(x_in: torch.Tensor, x_out: torch.Tensor, acc: torch.Tensor,
+                               mode: int = STATS_TOKEN, stream=None):
+    """adadsf_layer_stats without a workspace: the library keeps the partial
+    sums in a fixed device array of its own (see include/adadsf.h for the
+    set-up, sharing and size limits)."""
+    _dev(x_in, "x_in"); _dev(x_out, "x_out"); _dev(acc, "acc")
+    if acc.dtype != torch.float64:
+        raise ValueError("acc must be float64")
+    d = x_in.shape[-1]
+    n = x_in.numel() // d
+    _check(lib().adadsf_layer_stats_noalloc(_p(x_in), _p(x_out), n, d, DTYPE_CODE[x_in.dtype], mode,
+                                            _p(acc), _s(stream)))
 
 
 def adadsf_alloc_ratios(s: Sequence[float], t: float, tau: float = 0.05, beta: float = 10.0,

@@ -486,6 +486,34 @@ adadsf_status adadsf_layer_stats(const void* x_in_dev, const void* x_out_dev, in
                      "similarity statistics"));
 }
 
+adadsf_status adadsf_layer_stats_noalloc(const void* x_in_dev, const void* x_out_dev,
+                                         int64_t n_rows, int d, int dtype, int mode,
+                                         double* acc_dev, void* stream) {
+  if (dtype != ADADSF_F32 && dtype != ADADSF_BF16)
+    return fail(ADADSF_ERR_INVALID_ARG, "dtype %d unknown", dtype);
+  if (mode != ADADSF_STATS_TOKEN && mode != ADADSF_STATS_FLAT)
+    return fail(ADADSF_ERR_INVALID_ARG, "mode %d unknown", mode);
+  if (n_rows < 0 || d <= 0 || d % (dtype == ADADSF_BF16 ? 8 : 4) != 0)
+    return fail(ADADSF_ERR_INVALID_ARG, "need n_rows >= 0 and d a positive multiple of 16 bytes");
+  if (n_rows > (int64_t)INT32_MAX || d > 65536)
+    return fail(ADADSF_ERR_UNSUPPORTED,
+                "workspace-free statistics take n_rows <= %d and d <= 65536 (got n_rows=%lld, d=%d)",
+                INT32_MAX, (long long)n_rows, d);
+  if (stats_partials_count(n_rows) > stats_static_capacity())
+    return fail(ADADSF_ERR_UNSUPPORTED, "needs %d partial-sum slots, the fixed array holds %d",
+                stats_partials_count(n_rows), stats_static_capacity());
+  if (!acc_dev || (reinterpret_cast<uintptr_t>(acc_dev) & 7u))
+    return fail(ADADSF_ERR_INVALID_ARG, "acc_dev is NULL or not 8-byte aligned");
+  if (n_rows == 0) return ADADSF_OK;
+  NEED_PTR(x_in_dev, "x_in_dev");
+  NEED_PTR(x_out_dev, "x_out_dev");
+  Dev dev;
+  TRY(device_info(&dev, stream, nullptr));
+  CUDA_TRY(cos_stats_static(dtype, x_in_dev, x_out_dev, n_rows, d, mode, acc_dev, dev),
+           "workspace-free similarity statistics");
+  return ADADSF_OK;
+}
+
 adadsf_status adadsf_alloc_ratios(const double* s_host, int L, double t, double tau, double beta,
                                   int T, unsigned flags, double* r_out_host, int32_t* K_out_host) {
   if (!s_host || L <= 0) return fail(ADADSF_ERR_INVALID_ARG, "s_host is NULL or L <= 0");

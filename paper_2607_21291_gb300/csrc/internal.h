@@ -80,5 +80,9 @@ cudaError_t iota_positions(int32_t* idx, int B, int K, const Dev& dev);
 cudaError_t cos_stats(int dtype, const void* a, const void* b, int64_t n_rows, int d, int mode,
                       double* partials, double* acc, const Dev& dev);
 cudaError_t bounded_wait_selftest(int timeout_us, const Dev& dev);
+// Workspace-free variant of cos_stats: partial sums in a fixed device array.
+int stats_static_capacity();
+cudaError_t cos_stats_static(int dtype, const void* a, const void* b, int64_t n_rows, int d,
+                             int mode, double* acc, const Dev& dev);
 
 }  // namespace adadsf

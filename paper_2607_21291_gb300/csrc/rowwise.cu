@@ -2,6 +2,8 @@
 // rotary embedding at original positions, fp32 router, per-sequence Top-K,
 // the Eq. 4 similarity reduction, and the bounded-wait self-test.
 // All are HBM-bound: rows are moved as 16-byte vectors, one warp per row.
+#include <mutex>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -372,6 +374,12 @@ __global__ void cos_finish_kernel(const double* partials, int nblocks, int64_t n
   }
 }
 
+// Fixed scratch of the workspace-free statistics entry point: one slot of
+// three doubles per reduction block. The block count never exceeds
+// kStatMaxBlocks (see stats_partials_count), so 48 KiB always suffice.
+constexpr int kStatMaxBlocks = 2048;
+static __device__ __align__(256) double g_stats_scratch[kStatMaxBlocks * 3];
+
 // idx[b * K + j] = j: the kept positions of a dense layer.
 __global__ void iota_kernel(int32_t* idx, int64_t n, int K) {
   const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -487,7 +495,7 @@ cudaError_t topk(const float* scores, int B, int T, int K, int32_t* idx, int32_t
 // fixed-order sums are reproducible everywhere.
 int stats_partials_count(int64_t n_rows) {
   const int64_t want = (n_rows + (kStatThreads / 32) - 1) / (kStatThreads / 32);
-  const int64_t cap = 2048;
+  const int64_t cap = kStatMaxBlocks;
   return (int)(want < cap ? (want > 0 ? want : 1) : cap);
 }
 
@@ -505,6 +513,35 @@ cudaError_t cos_stats(int dtype, const void* a, const void* b, int64_t n_rows, i
   if (e != cudaSuccess) return e;
   cos_finish_kernel<<<1, 256, 0, dev.stream>>>(partials, nb, n_rows, mode, acc);
   return cudaGetLastError();
+}
+
+int stats_static_capacity() { return kStatMaxBlocks; }
+
+// Same reduction as cos_stats, with the partial sums in g_stats_scratch. In
+// host code g_stats_scratch names a host-side stand-in, not device memory, so
+// its device address is looked up once per device (with that device current)
+// and cached.
+cudaError_t cos_stats_static(int dtype, const void* a, const void* b, int64_t n_rows, int d,
+                             int mode, double* acc, const Dev& dev) {
+  static std::mutex mu;
+  static double* addr[64] = {nullptr};
+  int device = 0;
+  cudaError_t e = cudaGetDevice(&device);
+  if (e != cudaSuccess) return e;
+  if (device < 0 || device >= 64) return cudaErrorInvalidDevice;
+  double* scratch = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(mu);
+    if (!addr[device]) {
+      void* p = nullptr;
+      e = cudaGetSymbolAddress(&p, g_stats_scratch);
+      if (e != cudaSuccess) return e;
+      addr[device] = static_cast<double*>(p);
+    }
+    scratch = addr[device];
+  }
+  if (stats_partials_count(n_rows) > kStatMaxBlocks) return cudaErrorInvalidValue;
+  return cos_stats(dtype, a, b, n_rows, d, mode, scratch, acc, dev);
 }
 
 cudaError_t iota_positions(int32_t* idx, int B, int K, const Dev& dev) {
