@@ -7,7 +7,9 @@
  *  - Pointers named *_dev are device pointers (CUDA global memory of the
  *    current device); pointers named *_host are host pointers. The caller owns
  *    all memory. No entry point allocates or frees device memory; scratch
- *    space comes from a caller-provided workspace (ws, ws_bytes).
+ *    space comes from a caller-provided workspace (ws, ws_bytes), which must
+ *    be zero-filled before its first use (its first 256 bytes hold the device
+ *    error word, which must start at zero).
  *  - Device pointers must be 16-byte aligned; the workspace 256-byte aligned.
  *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
  *    stream). Every device entry point only enqueues work on that stream and
@@ -193,7 +195,8 @@ adadsf_status adadsf_topk_select(const float *scores_dev, int B, int T, int K,
  * Eq. 2 building block: out = act(x W^T + bias). x_dev [M, k_in],
  * w_dev [n_out, k_in], bias_dev [n_out] or NULL, out_dev [M, n_out], all in
  * `dtype`. act: 0 identity, 1 exact GELU. k_in % 64 == 0, n_out % 64 == 0 for
- * bf16 (tcgen05 tensor-core path), multiples of 4 for fp32.
+ * bf16 (tcgen05 tensor-core path), multiples of 4 for fp32. ws: at least 256
+ * bytes (the device error word).
  * ---------------------------------------------------------------------- */
 adadsf_status adadsf_linear(const void *x_dev, const void *w_dev, const void *bias_dev,
                             int64_t M, int n_out, int k_in, int dtype, int act, void *out_dev,

@@ -310,16 +310,27 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
                               c->norm_eps, lb.n1, neox ? lb.n2 : nullptr, dev),
                   "gather+norm")));
   // a5: QKV projection (+bias), rotary at the original positions.
+  // On the tensor-core path the rotation is fused into the QKV epilogue.
+  const int half = c->rotary_dim / 2;
+  const bool fuse_rope = tc && (half == 4 || half == 8 || half == 16 || (half > 0 && half % 32 == 0));
   {
     GemmArgs g = linear_args(lb.n1, d, w->w_qkv, M, qkv_dim, d);
     g.epi.bias = w->b_qkv;
     g.epi.out = lb.qkv;
     g.epi.ld_out = qkv_dim;
+    if (fuse_rope) {
+      g.epi.rope_tab = lb.rope;
+      g.epi.rope_pos = pos;
+      g.epi.rope_T = T;
+      g.epi.rope_half = half;
+      g.epi.rope_hd = c->head_dim;
+      g.epi.rope_cols = (c->n_heads + c->n_kv_heads) * c->head_dim;
+    }
     TRY(launch(dev, ADADSF_KERNEL_GEMM_QKV, tc, 2.0 * M * qkv_dim * d,
                (Md + (double)qkv_dim * d + (double)M * qkv_dim) * es,
                [&] { return run_linear(dt, g, dev, "qkv projection"); }));
   }
-  if (c->rotary_dim > 0)
+  if (c->rotary_dim > 0 && !fuse_rope)
     TRY(launch(dev, ADADSF_KERNEL_ROPE, false, 0,
                2.0 * M * (c->n_heads + c->n_kv_heads) * c->rotary_dim * es,
                CALL(rope_apply(dt, lb.qkv, M, qkv_dim, c->n_heads, c->n_kv_heads, c->head_dim,

@@ -71,6 +71,7 @@ template <int HD>
 __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* qkv, int64_t ldq, bf16* out,
                                                         int64_t ldo, int K, int n_heads, int n_kv,
                                                         float scale_log2) {
+  pdl_trigger();
   extern __shared__ __align__(128) uint8_t smem_raw[];
   bf16* sQ = reinterpret_cast<bf16*>(smem_raw);
   bf16* sK = sQ + BQ * HD;               // [2][BKV][HD]
@@ -87,6 +88,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* qkv, int64_t
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
+  pdl_wait();
   load_tile<HD>(sQ, Qg, ldq, qb * BQ, K);
   load_tile<HD>(sK, Kg, ldq, 0, K);
   load_tile<HD>(sV, Vg, ldq, 0, K);
@@ -219,6 +221,8 @@ template <int HD>
 __global__ void __launch_bounds__(128) attn_f32_kernel(const float* qkv, int64_t ldq, float* out,
                                                        int64_t ldo, int K, int n_heads, int n_kv,
                                                        float scale) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int PL = HD / 32;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int i = blockIdx.x * 4 + warp;
@@ -269,8 +273,8 @@ cudaError_t launch_bf16(const bf16* qkv, int64_t ldq, bf16* out, int64_t ldo, in
   }
   dim3 grid((K + BQ - 1) / BQ, H, B);
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)HD);
-  attn_bf16_kernel<HD><<<grid, 128, smem, dev.stream>>>(qkv, ldq, out, ldo, K, H, Hkv, scale_log2);
-  return cudaGetLastError();
+  return launch_pdl(attn_bf16_kernel<HD>, grid, dim3(128), smem, dev.stream, qkv, ldq, out, ldo, K,
+                    H, Hkv, scale_log2);
 }
 
 }  // namespace
@@ -290,12 +294,12 @@ cudaError_t attention(int dtype, const void* qkv, int64_t ld_qkv, void* out, int
   dim3 grid((K + 3) / 4, n_heads, B);
   const float scale = 1.f / sqrtf((float)head_dim);
   if (head_dim == 64)
-    attn_f32_kernel<64><<<grid, 128, 0, dev.stream>>>(q, ld_qkv, o, ld_out, K, n_heads, n_kv_heads, scale);
-  else if (head_dim == 128)
-    attn_f32_kernel<128><<<grid, 128, 0, dev.stream>>>(q, ld_qkv, o, ld_out, K, n_heads, n_kv_heads, scale);
-  else
-    return cudaErrorInvalidValue;
-  return cudaGetLastError();
+    return launch_pdl(attn_f32_kernel<64>, grid, dim3(128), 0, dev.stream, q, ld_qkv, o, ld_out, K,
+                      n_heads, n_kv_heads, scale);
+  if (head_dim == 128)
+    return launch_pdl(attn_f32_kernel<128>, grid, dim3(128), 0, dev.stream, q, ld_qkv, o, ld_out, K,
+                      n_heads, n_kv_heads, scale);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace adadsf

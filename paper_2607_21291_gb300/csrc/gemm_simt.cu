@@ -24,6 +24,8 @@ struct SimtDev {
 
 template <bool DUAL>
 __global__ void __launch_bounds__(256) gemm_f32_kernel(const SimtDev p) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ float As[TK][TM + 4];
   __shared__ float Ws[TK][TN + 4];
   __shared__ float W2s[DUAL ? TK : 1][TN + 4];
@@ -100,10 +102,8 @@ cudaError_t gemm_f32(const GemmArgs& a, const Dev& dev) {
   p.out = static_cast<float*>(a.epi.out); p.ld_out = a.epi.ld_out;
   dim3 grid((a.N + TN - 1) / TN, (unsigned)((a.M + TM - 1) / TM));
   if (a.epi.act == ACT_SWIGLU)
-    gemm_f32_kernel<true><<<grid, 256, 0, dev.stream>>>(p);
-  else
-    gemm_f32_kernel<false><<<grid, 256, 0, dev.stream>>>(p);
-  return cudaGetLastError();
+    return launch_pdl(gemm_f32_kernel<true>, grid, dim3(256), 0, dev.stream, p);
+  return launch_pdl(gemm_f32_kernel<false>, grid, dim3(256), 0, dev.stream, p);
 }
 
 }  // namespace adadsf

@@ -5,15 +5,16 @@
 // tcgen05 reads natively. These are the dense contractions of Eqs. 1-2 (QKV,
 // output and MLP projections) and the router's first linear layer (Sec. 3.4).
 //
-// Kernel structure (one persistent CTA per SM, 6 warps):
+// Kernel structure (one persistent CTA per SM, 10 warps):
 //   warp 0     TMA producer: 128x64 A tile and BNx64 W tile(s) per stage into a
 //              STAGES-deep shared-memory ring, 128-byte swizzled, signalled
 //              through mbarrier transaction counts.
 //   warp 1     allocates TMEM; one thread issues tcgen05.mma (M=128, N=BN,
 //              K=16, fp32 accumulator in TMEM) and commits stage releases and
 //              accumulator hand-offs to mbarriers.
-//   warps 2-5  epilogue: tcgen05.ld the accumulator (one row per thread),
-//              apply bias / GELU / SwiGLU / residual / row scatter / router
+//   warps 2-9  epilogue: tcgen05.ld the accumulator (one row per thread, two
+//              warps per 32-lane TMEM quarter splitting the columns), apply
+//              bias / GELU / SwiGLU / rotary / residual / row scatter / router
 //              reduction in fp32, round once and store.
 // The accumulator is double-buffered in TMEM so the epilogue of tile i runs
 // under the main loop of tile i+1. Every barrier wait is bounded in time; on
@@ -33,7 +34,8 @@ namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;       // one 128-byte swizzle row of bf16
 constexpr int UK = 16;       // K of one tcgen05.mma kind::f16
-constexpr int kThreads = 192;
+constexpr int kEpiWarps = 8;     // two per TMEM lane quarter, each on half of the columns
+constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr int kGroupM = 16;  // tile raster: 16 M-blocks share each W column block
 
 template <int BN, bool DUAL>
@@ -61,6 +63,10 @@ struct GemmDev {
   int out_mapped;
   bf16* out; int64_t ld_out;
   const bf16* w2; const bf16* b2; float* scores;
+  // rotary embedding fused into the QKV epilogue (rope_tab == nullptr: off)
+  const float2* rope_tab;    // [T][rope_half] (cos, sin)
+  const int32_t* rope_pos;   // [M] original positions, or null: m % rope_T
+  int rope_T, rope_half, rope_hd, rope_cols;
   int* err;
   unsigned long long timeout_ns;
 };
@@ -103,6 +109,42 @@ __device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, int 
   for (int i = 0; i < 4; ++i) store_vec(p.out + orow * p.ld_out + n0 + 8 * i, v + 8 * i);
 }
 
+// Rotates the pairs (a[j], b[j]) j < n by the angles of features i0 + j at
+// the row's position: a' = a cos - b sin, b' = b cos + a sin.
+__device__ __forceinline__ void rope_rotate(float* a, float* b, int n, const float2* tab_row, int i0) {
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    if (j < n) {
+      const float2 cs = tab_row[i0 + j];
+      const float x = a[j], y = b[j];
+      a[j] = x * cs.x - y * cs.y;
+      b[j] = y * cs.x + x * cs.y;
+    }
+  }
+}
+
+// Feature j < H of the chunk pairs with feature j + H (H = rotary half <= 16).
+template <int H>
+__device__ __forceinline__ void rope_in_chunk(float* v, const float2* tab_row) {
+#pragma unroll
+  for (int j = 0; j < H; ++j) {
+    const float2 cs = tab_row[j];
+    const float x = v[j], y = v[j + H];
+    v[j] = x * cs.x - y * cs.y;
+    v[j + H] = y * cs.x + x * cs.y;
+  }
+}
+
+__device__ __forceinline__ void add_bias32(const bf16* bias, int n0, float* v) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    float f[8];
+    load_vec(bias + n0 + 8 * i, f);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) v[8 * i + j] += f[j];
+  }
+}
+
 template <int BN, bool DUAL, bool ROUTER>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -127,9 +169,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int lane = threadIdx.x & 31;
   const int num_m = (p.M + BM - 1) / BM;
   const int num_n = (p.N + BN - 1) / BN;
-  const int num_tiles = num_m * num_n;
   const int num_kb = (p.K + BK - 1) / BK;
+  const int num_tiles = num_m * num_n;
 
+  pdl_trigger();
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
       mbar_init(full0 + 8 * s, 1);
@@ -137,7 +180,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull0 + 8 * a, 1);
-      mbar_init(tempty0 + 8 * a, 4);
+      mbar_init(tempty0 + 8 * a, kEpiWarps);
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -162,23 +205,44 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t phase = 0;
       int64_t issued = 0;
       constexpr uint32_t tx = C::STAGE_BYTES;
+      // The weights do not depend on the previous kernel: the first tile's
+      // weight tiles are requested before waiting for it.
+      int pre = 0;
+      if ((int)blockIdx.x < num_tiles) {
+        int mb, nb;
+        tile_coords(blockIdx.x, num_m, num_n, mb, nb);
+        pre = num_kb < C::STAGES ? num_kb : C::STAGES;
+        for (int kb = 0; kb < pre; ++kb) {
+          const uint32_t fb = full0 + 8 * kb;
+          mbar_arrive_expect_tx(fb, tx);
+          tma_load_2d(sB + kb * C::B_BYTES, &tmB, kb * BK, nb * BN, fb);
+          if (DUAL) tma_load_2d(sB2 + kb * C::B_BYTES, &tmB2, kb * BK, nb * BN, fb);
+        }
+      }
+      pdl_wait();
+      bool first = true;
       for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
         int mb, nb;
         tile_coords(t, num_m, num_n, mb, nb);
         bool ok = true;
         for (int kb = 0; kb < num_kb; ++kb) {
-          if (!mbar_wait_bounded(empty0 + 8 * stage, phase ^ 1, abort_flag, p.err, p.timeout_ns)) {
-            ok = false;
-            break;
-          }
           const uint32_t fb = full0 + 8 * stage;
-          mbar_arrive_expect_tx(fb, tx);
-          tma_load_2d(sA + stage * C::A_BYTES, &tmA, kb * BK, mb * BM, fb);
-          tma_load_2d(sB + stage * C::B_BYTES, &tmB, kb * BK, nb * BN, fb);
-          if (DUAL) tma_load_2d(sB2 + stage * C::B_BYTES, &tmB2, kb * BK, nb * BN, fb);
+          if (first && kb < pre) {
+            tma_load_2d(sA + stage * C::A_BYTES, &tmA, kb * BK, mb * BM, fb);
+          } else {
+            if (!mbar_wait_bounded(empty0 + 8 * stage, phase ^ 1, abort_flag, p.err, p.timeout_ns)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(fb, tx);
+            tma_load_2d(sA + stage * C::A_BYTES, &tmA, kb * BK, mb * BM, fb);
+            tma_load_2d(sB + stage * C::B_BYTES, &tmB, kb * BK, nb * BN, fb);
+            if (DUAL) tma_load_2d(sB2 + stage * C::B_BYTES, &tmB2, kb * BK, nb * BN, fb);
+          }
           ++issued;
           if (++stage == C::STAGES) { stage = 0; phase ^= 1; }
         }
+        first = false;
         if (!ok) break;
       }
       // Drain: wait until the last copy issued into each stage has landed.
@@ -217,10 +281,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int k = 0; k < BK / UK; ++k) {
             const uint64_t ad = smem_desc_sw128(a_s + k * UK * 2);
             const uint64_t bd = smem_desc_sw128(b_s + k * UK * 2);
-            tc_mma_f16(d_tmem, ad, bd, idesc, (kb | k) != 0);
+            const uint32_t accum = (kb > 0 || k > 0) ? 1u : 0u;
+            tc_mma_f16(d_tmem, ad, bd, idesc, accum);
             if (DUAL) {
               const uint64_t b2d = smem_desc_sw128(sB2 + stage * C::B_BYTES + k * UK * 2);
-              tc_mma_f16(d_tmem + BN, ad, b2d, idesc, (kb | k) != 0);
+              tc_mma_f16(d_tmem + BN, ad, b2d, idesc, accum);
             }
           }
           tc_commit(empty0 + 8 * stage);   // stage free once these MMAs have read it
@@ -234,8 +299,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_wait_drain(drain, 0, p.timeout_ns);
     }
   } else {
-    // ------------------------------------------------------------ epilogue (warps 2..5)
+    // ------------------------------------------------------------ epilogue (warps 2..9)
+    pdl_wait();
     const int quarter = warp & 3;   // TMEM lanes 32*quarter .. +31
+    const int half = (warp - 2) >> 2;   // columns: chunks [half*NC/2, (half+1)*NC/2)
+    const int row_in_tile = quarter * 32 + lane;
+    const bool rope = !ROUTER && !DUAL && p.rope_tab != nullptr;
     int it = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++it) {
       int mb, nb;
@@ -247,34 +316,41 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
-      const int m = mb * BM + quarter * 32 + lane;
+      const uint32_t tacc = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C::ACC_COLS;
+
+      const int m = mb * BM + row_in_tile;
       const bool mvalid = m < p.M;
       int64_t arow = m;
       if (mvalid && p.rows) arow = p.rows[m];
       const int64_t orow = p.out_mapped ? arow : (int64_t)m;
-      const uint32_t tacc = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C::ACC_COLS;
+      const float2* tab_row = nullptr;
+      if (rope && mvalid)
+        tab_row = p.rope_tab + (int64_t)(p.rope_pos ? p.rope_pos[m] : m % p.rope_T) * p.rope_half;
       float rsum = 0.f;
+      constexpr int NC = BN / 32;
 #pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
-        uint32_t r[32];
-        tmem_ld32(tacc + c * 32, r);
-        uint32_t r2[DUAL ? 32 : 1];
-        if (DUAL) tmem_ld32(tacc + BN + c * 32, r2);
-        tmem_ld_wait();
+      for (int c = 0; c < NC; ++c) {
+        // the router's row reduction stays in one warp per quarter
+        const int owner = ROUTER ? 0 : (c < NC / 2 ? 0 : 1);
+        if (owner != half) continue;
         const int n0 = nb * BN + c * 32;
+        // rotary halves of 32 or more features: chunk c pairs with chunk c2,
+        // both handled by the owner of c
+        const bool rot = rope && n0 < p.rope_cols;
+        const bool paired = rot && p.rope_half >= 32;
+        if (paired && (n0 % p.rope_hd) >= p.rope_half) continue;   // done with its partner
+        const int c2 = paired ? c + p.rope_half / 32 : c;
+        uint32_t r[32];
+        uint32_t r2[(DUAL || !ROUTER) ? 32 : 1];
+        tmem_ld32(tacc + c * 32, r);
+        if (DUAL) tmem_ld32(tacc + BN + c * 32, r2);
+        else if (!ROUTER && paired) tmem_ld32(tacc + c2 * 32, r2);
+        tmem_ld_wait();
         if (!mvalid || n0 >= p.N) continue;
         float v[32];
 #pragma unroll
         for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-        if (p.bias) {
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            float f[8];
-            load_vec(p.bias + n0 + 8 * i, f);
-#pragma unroll
-            for (int j = 0; j < 8; ++j) v[8 * i + j] += f[j];
-          }
-        }
+        if (p.bias) add_bias32(p.bias, n0, v);
         if (ROUTER) {
 #pragma unroll
           for (int i = 0; i < 4; ++i) {
@@ -292,9 +368,26 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int j = 0; j < 32; ++j) v[j] = gelu_f(v[j]);
         }
+        if (!DUAL && paired) {
+          const int n2 = nb * BN + c2 * 32;
+          float v2[32];
+#pragma unroll
+          for (int j = 0; j < 32; ++j) v2[j] = __uint_as_float(r2[j]);
+          if (p.bias) add_bias32(p.bias, n2, v2);
+          rope_rotate(v, v2, 32, tab_row, n0 % p.rope_hd);
+          epi_chunk_store(p, v2, m, arow, orow, n2);
+        } else if (rot && (n0 % p.rope_hd) == 0) {
+          // rotary half of at most 16 features: both halves inside this chunk
+          switch (p.rope_half) {
+            case 4: rope_in_chunk<4>(v, tab_row); break;
+            case 8: rope_in_chunk<8>(v, tab_row); break;
+            case 16: rope_in_chunk<16>(v, tab_row); break;
+            default: break;
+          }
+        }
         epi_chunk_store(p, v, m, arow, orow, n0);
       }
-      if (ROUTER && mvalid) p.scores[m] = rsum + __bfloat162float(p.b2[0]);
+      if (ROUTER && half == 0 && mvalid) p.scores[m] = rsum + __bfloat162float(p.b2[0]);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
@@ -369,12 +462,18 @@ cudaError_t launch(const GemmArgs& a, const Dev& dev) {
   p.out = static_cast<bf16*>(a.epi.out); p.ld_out = a.epi.ld_out;
   p.w2 = static_cast<const bf16*>(a.epi.w2); p.b2 = static_cast<const bf16*>(a.epi.b2);
   p.scores = a.epi.scores;
+  p.rope_tab = a.epi.rope_tab;
+  p.rope_pos = a.epi.rope_pos;
+  p.rope_T = a.epi.rope_T;
+  p.rope_half = a.epi.rope_half;
+  p.rope_hd = a.epi.rope_hd;
+  p.rope_cols = a.epi.rope_cols;
   p.err = dev.err;
   p.timeout_ns = kWaitTimeoutNs;
   const int64_t num_tiles = ((a.M + BM - 1) / BM) * ((a.N + BN - 1) / BN);
   const int grid = (int)(num_tiles < dev.num_sms ? num_tiles : dev.num_sms);
-  gemm_tc_kernel<BN, DUAL, ROUTER><<<grid, kThreads, C::SMEM_BYTES, dev.stream>>>(ta, tb, tb2, p);
-  return cudaGetLastError();
+  return launch_pdl(gemm_tc_kernel<BN, DUAL, ROUTER>, dim3(grid), dim3(kThreads), C::SMEM_BYTES,
+                    dev.stream, ta, tb, tb2, p);
 }
 
 }  // namespace

@@ -35,6 +35,13 @@ struct Epilogue {
   const void* w2 = nullptr;   // router
   const void* b2 = nullptr;   // router
   float* scores = nullptr;    // router
+  // Rotary embedding of the first rope_cols output columns (query and key
+  // heads), bf16 tensor-core path only: per head of rope_hd columns, feature
+  // i < rope_half pairs with i + rope_half and turns by tab[pos][i], pos =
+  // rope_pos ? rope_pos[m] : m % rope_T. Needs rope_half in {4, 8, 16} or a multiple of 32.
+  const float2* rope_tab = nullptr;
+  const int32_t* rope_pos = nullptr;
+  int rope_T = 1, rope_half = 0, rope_hd = 0, rope_cols = 0;
 };
 
 struct GemmArgs {

@@ -16,6 +16,8 @@ constexpr int kMaxChunks = 16;  // per-lane 16-byte vectors held in registers (d
 template <typename T>
 __global__ void embed_kernel(const int32_t* ids, int64_t n, const T* table, int vocab, int d,
                              T* out, int* err) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int V = Elem<T>::kVec;
   const int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
   const int lane = threadIdx.x & 31;
@@ -39,6 +41,8 @@ template <typename T, bool RMS>
 __global__ void gather_norm_kernel(const T* x, const int32_t* rows, int64_t M, int d, const T* g1,
                                    const T* b1, const T* g2, const T* b2, float eps, T* out1,
                                    T* out2) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int V = Elem<T>::kVec;
   const int64_t m = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
   const int lane = threadIdx.x & 31;
@@ -106,16 +110,23 @@ __global__ void gather_norm_kernel(const T* x, const int32_t* rows, int64_t M, i
 }
 
 // ---------------------------------------------------------------- rotary embedding
-// tab[p * half + i] = (cos, sin) of p * theta^(-2i / rotary_dim), evaluated in
-// fp64 and rounded once to fp32.
-__global__ void rope_table_kernel(float2* tab, int T, int half, int rotary_dim, double theta) {
+// tab[p * half + i] = (cos, sin) of the angle p * inv[i], inv[i] =
+// theta^(-2i / rotary_dim) given in fp64 by the host. The angle is formed and
+// reduced to [-pi, pi] in fp64, then evaluated in fp32 (error ~1e-7).
+struct InvFreq {
+  double v[64];
+};
+__global__ void rope_table_kernel(float2* tab, int T, int half, InvFreq inv) {
+  pdl_trigger();
+  pdl_wait();
   const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (k >= (int64_t)T * half) return;
   const int p = (int)(k / half), i = (int)(k % half);
-  const double inv = pow(theta, -2.0 * i / rotary_dim);
-  double s, c;
-  sincos((double)p * inv, &s, &c);
-  tab[k] = make_float2((float)c, (float)s);
+  double a = (double)p * inv.v[i];
+  a -= rint(a * 0.15915494309189535) * 6.283185307179586;
+  float s, c;
+  sincosf((float)a, &s, &c);
+  tab[k] = make_float2(c, s);
 }
 
 // Rotates, in place, the first rotary_dim features of every query and key
@@ -124,6 +135,8 @@ __global__ void rope_table_kernel(float2* tab, int T, int half, int rotary_dim, 
 template <typename T>
 __global__ void rope_apply_kernel(T* qkv, int64_t M, int64_t ld, int heads, int head_dim,
                                   int half, const int32_t* pos, int seq_len, const float2* tab) {
+  pdl_trigger();
+  pdl_wait();
   const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t per_row = (int64_t)heads * half;
   if (k >= M * per_row) return;
@@ -144,6 +157,8 @@ __global__ void rope_apply_kernel(T* qkv, int64_t M, int64_t ld, int heads, int 
 __global__ void router_f32_kernel(const float* x, int64_t n, int d, int h, const float* w1,
                                   const float* b1, const float* w2, const float* b2,
                                   float* scores) {
+  pdl_trigger();
+  pdl_wait();
   const int64_t row = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
   const int lane = threadIdx.x & 31;
   if (row >= n) return;
@@ -211,6 +226,8 @@ constexpr int kTopkThreads = 1024;
 // positions in ascending order.
 __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const float* scores, int T, int K,
                                                             int32_t* idx, int32_t* rows) {
+  pdl_trigger();
+  pdl_wait();
   extern __shared__ uint32_t keys[];
   __shared__ int hist[256];
   __shared__ int warp_tot[33];
@@ -313,6 +330,8 @@ template <typename T>
 __global__ void __launch_bounds__(kStatThreads) cos_rows_kernel(const T* a, const T* b,
                                                                 int64_t n_rows, int d, int mode,
                                                                 double* partials) {
+  pdl_trigger();
+  pdl_wait();
   constexpr int V = Elem<T>::kVec;
   __shared__ double red[kStatThreads / 32][3];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -353,6 +372,8 @@ __global__ void __launch_bounds__(kStatThreads) cos_rows_kernel(const T* a, cons
 // Fixed-order sum of the per-block partials, added to acc.
 __global__ void cos_finish_kernel(const double* partials, int nblocks, int64_t n_rows, int mode,
                                   double* acc) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ double red[3][256];
   double s[3] = {0, 0, 0};
   for (int i = threadIdx.x; i < nblocks; i += 256)
@@ -382,6 +403,8 @@ static __device__ __align__(256) double g_stats_scratch[kStatMaxBlocks * 3];
 
 // idx[b * K + j] = j: the kept positions of a dense layer.
 __global__ void iota_kernel(int32_t* idx, int64_t n, int K) {
+  pdl_trigger();
+  pdl_wait();
   const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (k < n) idx[k] = (int32_t)(k % K);
 }
@@ -414,12 +437,10 @@ cudaError_t embed(int dtype, const int32_t* ids, int64_t n, const void* table, i
                   void* out, const Dev& dev) {
   if (n <= 0) return cudaSuccess;
   if (dtype == kBF16)
-    embed_kernel<bf16><<<blocks_for(n, 8), 256, 0, dev.stream>>>(
-        ids, n, static_cast<const bf16*>(table), vocab, d, static_cast<bf16*>(out), dev.err);
-  else
-    embed_kernel<float><<<blocks_for(n, 8), 256, 0, dev.stream>>>(
-        ids, n, static_cast<const float*>(table), vocab, d, static_cast<float*>(out), dev.err);
-  return cudaGetLastError();
+    return launch_pdl(embed_kernel<bf16>, dim3(blocks_for(n, 8)), dim3(256), 0, dev.stream, ids, n,
+                      static_cast<const bf16*>(table), vocab, d, static_cast<bf16*>(out), dev.err);
+  return launch_pdl(embed_kernel<float>, dim3(blocks_for(n, 8)), dim3(256), 0, dev.stream, ids, n,
+                    static_cast<const float*>(table), vocab, d, static_cast<float*>(out), dev.err);
 }
 
 cudaError_t gather_norm(int dtype, const void* x, const int32_t* rows, int64_t M, int d,
@@ -427,27 +448,29 @@ cudaError_t gather_norm(int dtype, const void* x, const int32_t* rows, int64_t M
                         const void* b2, float eps, void* out1, void* out2, const Dev& dev) {
   if (M <= 0) return cudaSuccess;
   const unsigned grid = blocks_for(M, 8);
-#define GN_LAUNCH(T, R)                                                                        \
-  gather_norm_kernel<T, R><<<grid, 256, 0, dev.stream>>>(                                      \
-      static_cast<const T*>(x), rows, M, d, static_cast<const T*>(g1),                         \
-      static_cast<const T*>(b1), static_cast<const T*>(g2), static_cast<const T*>(b2), eps,   \
-      static_cast<T*>(out1), static_cast<T*>(out2))
+#define GN_LAUNCH(T, R)                                                                         \
+  return launch_pdl(gather_norm_kernel<T, R>, dim3(grid), dim3(256), 0, dev.stream,             \
+                    static_cast<const T*>(x), rows, M, d, static_cast<const T*>(g1),            \
+                    static_cast<const T*>(b1), static_cast<const T*>(g2),                       \
+                    static_cast<const T*>(b2), eps, static_cast<T*>(out1), static_cast<T*>(out2))
   if (dtype == kBF16) {
-    if (is_rms) GN_LAUNCH(bf16, true); else GN_LAUNCH(bf16, false);
-  } else {
-    if (is_rms) GN_LAUNCH(float, true); else GN_LAUNCH(float, false);
+    if (is_rms) GN_LAUNCH(bf16, true);
+    GN_LAUNCH(bf16, false);
   }
+  if (is_rms) GN_LAUNCH(float, true);
+  GN_LAUNCH(float, false);
 #undef GN_LAUNCH
-  return cudaGetLastError();
 }
 
 cudaError_t rope_table(float2* tab, int T, int rotary_dim, float theta, const Dev& dev) {
   const int half = rotary_dim / 2;
   const int64_t n = (int64_t)T * half;
   if (n <= 0) return cudaSuccess;
-  rope_table_kernel<<<(unsigned)((n + 255) / 256), 256, 0, dev.stream>>>(tab, T, half, rotary_dim,
-                                                                          (double)theta);
-  return cudaGetLastError();
+  if (half > 64) return cudaErrorInvalidValue;
+  InvFreq inv;
+  for (int i = 0; i < 64; ++i) inv.v[i] = i < half ? pow((double)theta, -2.0 * i / rotary_dim) : 0.0;
+  return launch_pdl(rope_table_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, dev.stream,
+                    tab, T, half, inv);
 }
 
 cudaError_t rope_apply(int dtype, void* qkv, int64_t M, int64_t ld, int n_heads, int n_kv_heads,
@@ -459,19 +482,17 @@ cudaError_t rope_apply(int dtype, void* qkv, int64_t M, int64_t ld, int n_heads,
   if (n <= 0) return cudaSuccess;
   const unsigned grid = (unsigned)((n + 255) / 256);
   if (dtype == kBF16)
-    rope_apply_kernel<bf16><<<grid, 256, 0, dev.stream>>>(static_cast<bf16*>(qkv), M, ld, heads,
-                                                          head_dim, half, pos, T, tab);
-  else
-    rope_apply_kernel<float><<<grid, 256, 0, dev.stream>>>(static_cast<float*>(qkv), M, ld, heads,
-                                                           head_dim, half, pos, T, tab);
-  return cudaGetLastError();
+    return launch_pdl(rope_apply_kernel<bf16>, dim3(grid), dim3(256), 0, dev.stream,
+                      static_cast<bf16*>(qkv), M, ld, heads, head_dim, half, pos, T, tab);
+  return launch_pdl(rope_apply_kernel<float>, dim3(grid), dim3(256), 0, dev.stream,
+                    static_cast<float*>(qkv), M, ld, heads, head_dim, half, pos, T, tab);
 }
 
 cudaError_t router_f32(const float* x, int64_t n, int d, int h, const float* w1, const float* b1,
                        const float* w2, const float* b2, float* scores, const Dev& dev) {
   if (n <= 0) return cudaSuccess;
-  router_f32_kernel<<<blocks_for(n, 8), 256, 0, dev.stream>>>(x, n, d, h, w1, b1, w2, b2, scores);
-  return cudaGetLastError();
+  return launch_pdl(router_f32_kernel, dim3(blocks_for(n, 8)), dim3(256), 0, dev.stream, x, n, d,
+                    h, w1, b1, w2, b2, scores);
 }
 
 cudaError_t topk(const float* scores, int B, int T, int K, int32_t* idx, int32_t* rows,
@@ -487,8 +508,8 @@ cudaError_t topk(const float* scores, int B, int T, int K, int32_t* idx, int32_t
     if (e != cudaSuccess) return e;
     attr_done[device] = 1;
   }
-  topk_kernel<<<B, kTopkThreads, smem, dev.stream>>>(scores, T, K, idx, rows);
-  return cudaGetLastError();
+  return launch_pdl(topk_kernel, dim3(B), dim3(kTopkThreads), smem, dev.stream, scores, T, K, idx,
+                    rows);
 }
 
 // Fixed block count for a given row count (independent of the device), so the
@@ -503,16 +524,17 @@ cudaError_t cos_stats(int dtype, const void* a, const void* b, int64_t n_rows, i
                       double* partials, double* acc, const Dev& dev) {
   if (n_rows <= 0) return cudaSuccess;
   const int nb = stats_partials_count(n_rows);
+  cudaError_t e;
   if (dtype == kBF16)
-    cos_rows_kernel<bf16><<<nb, kStatThreads, 0, dev.stream>>>(
-        static_cast<const bf16*>(a), static_cast<const bf16*>(b), n_rows, d, mode, partials);
+    e = launch_pdl(cos_rows_kernel<bf16>, dim3(nb), dim3(kStatThreads), 0, dev.stream,
+                   static_cast<const bf16*>(a), static_cast<const bf16*>(b), n_rows, d, mode, partials);
   else
-    cos_rows_kernel<float><<<nb, kStatThreads, 0, dev.stream>>>(
-        static_cast<const float*>(a), static_cast<const float*>(b), n_rows, d, mode, partials);
-  cudaError_t e = cudaGetLastError();
+    e = launch_pdl(cos_rows_kernel<float>, dim3(nb), dim3(kStatThreads), 0, dev.stream,
+                   static_cast<const float*>(a), static_cast<const float*>(b), n_rows, d, mode,
+                   partials);
   if (e != cudaSuccess) return e;
-  cos_finish_kernel<<<1, 256, 0, dev.stream>>>(partials, nb, n_rows, mode, acc);
-  return cudaGetLastError();
+  return launch_pdl(cos_finish_kernel, dim3(1), dim3(256), 0, dev.stream, partials, nb, n_rows, mode,
+                    acc);
 }
 
 int stats_static_capacity() { return kStatMaxBlocks; }
@@ -547,8 +569,8 @@ cudaError_t cos_stats_static(int dtype, const void* a, const void* b, int64_t n_
 cudaError_t iota_positions(int32_t* idx, int B, int K, const Dev& dev) {
   const int64_t n = (int64_t)B * K;
   if (n <= 0) return cudaSuccess;
-  iota_kernel<<<(unsigned)((n + 255) / 256), 256, 0, dev.stream>>>(idx, n, K);
-  return cudaGetLastError();
+  return launch_pdl(iota_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, dev.stream, idx, n,
+                    K);
 }
 
 cudaError_t bounded_wait_selftest(int timeout_us, const Dev& dev) {

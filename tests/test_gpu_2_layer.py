@@ -32,6 +32,11 @@ LAYER_CASES = [
     (NEOX_128, 2, 190, 100),
     (QWEN_SMALL, 2, 150, 70),
     (QWEN_SMALL, 1, 257, 129),
+    # rotary widths: half 32 (paired chunks, head_dim 64), half 4, and half 24
+    # (not fusable: separate rotary kernel)
+    (S.PYTHIA_160M.replace(rotary_dim=64), 2, 100, 50),
+    (S.PYTHIA_160M.replace(rotary_dim=8), 1, 90, 45),
+    (S.PYTHIA_160M.replace(rotary_dim=48), 1, 90, 45),
 ]
 
 
