@@ -38,11 +38,16 @@ constexpr int kEpiWarps = 8;     // two per TMEM lane quarter, each on half of t
 constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr int kGroupM = 16;  // tile raster: 16 M-blocks share each W column block
 
-template <int BN, bool DUAL>
+// PAIR: two-CTA variant. Plain: each CTA stages half of the BN weight rows.
+// DUAL: the even CTA stages BN rows of the first weight, the odd CTA BN rows
+// of the second, so one N = 2 BN pair MMA yields both accumulators.
+template <int BN, bool DUAL, bool PAIR = false>
 struct TileCfg {
   static constexpr int A_BYTES = BM * BK * 2;
-  static constexpr int B_BYTES = BN * BK * 2;
-  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES * (DUAL ? 2 : 1);
+  static constexpr int B_ROWS = (PAIR && !DUAL) ? BN / 2 : BN;
+  static constexpr int B_BYTES = B_ROWS * BK * 2;
+  static constexpr int NUM_B = (DUAL && !PAIR) ? 2 : 1;   // weight tiles per stage
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES * NUM_B;
   static constexpr int STAGES_FIT = 196608 / STAGE_BYTES;
   static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
   static constexpr int ACC_COLS = BN * (DUAL ? 2 : 1);
@@ -143,6 +148,84 @@ __device__ __forceinline__ void add_bias32(const bf16* bias, int n0, float* v) {
 #pragma unroll
     for (int j = 0; j < 8; ++j) v[8 * i + j] += f[j];
   }
+}
+
+// Epilogue of one accumulator tile for the calling thread's row m: chunks of
+// 32 TMEM columns (this warp's half of them) -> bias / activation / rotary /
+// residual / store, or the router's row reduction.
+template <int BN, bool DUAL, bool ROUTER>
+__device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, int m, int nb,
+                                              int half) {
+  const bool rope = !ROUTER && !DUAL && p.rope_tab != nullptr;
+  const bool mvalid = m < p.M;
+  int64_t arow = m;
+  if (mvalid && p.rows) arow = p.rows[m];
+  const int64_t orow = p.out_mapped ? arow : (int64_t)m;
+  const float2* tab_row = nullptr;
+  if (rope && mvalid)
+    tab_row = p.rope_tab + (int64_t)(p.rope_pos ? p.rope_pos[m] : m % p.rope_T) * p.rope_half;
+  float rsum = 0.f;
+  constexpr int NC = BN / 32;
+#pragma unroll 1
+  for (int c = 0; c < NC; ++c) {
+    // the router's row reduction stays in one warp per quarter
+    const int owner = ROUTER ? 0 : (c < NC / 2 ? 0 : 1);
+    if (owner != half) continue;
+    const int n0 = nb * BN + c * 32;
+    // rotary halves of 32 or more features: chunk c pairs with chunk c2,
+    // both handled by the owner of c
+    const bool rot = rope && n0 < p.rope_cols;
+    const bool paired = rot && p.rope_half >= 32;
+    if (paired && (n0 % p.rope_hd) >= p.rope_half) continue;   // done with its partner
+    const int c2 = paired ? c + p.rope_half / 32 : c;
+    uint32_t r[32];
+    uint32_t r2[(DUAL || !ROUTER) ? 32 : 1];
+    tmem_ld32(tacc + c * 32, r);
+    if (DUAL) tmem_ld32(tacc + BN + c * 32, r2);
+    else if (!ROUTER && paired) tmem_ld32(tacc + c2 * 32, r2);
+    tmem_ld_wait();
+    if (!mvalid || n0 >= p.N) continue;
+    float v[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+    if (p.bias) add_bias32(p.bias, n0, v);
+    if (ROUTER) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        float f[8];
+        load_vec(p.w2 + n0 + 8 * i, f);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) rsum += f[j] * silu_f(v[8 * i + j]);
+      }
+      continue;
+    }
+    if (DUAL) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = silu_f(v[j]) * __uint_as_float(r2[j]);
+    } else if (p.act == ACT_GELU) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = gelu_f(v[j]);
+    }
+    if (!DUAL && paired) {
+      const int n2 = nb * BN + c2 * 32;
+      float v2[32];
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v2[j] = __uint_as_float(r2[j]);
+      if (p.bias) add_bias32(p.bias, n2, v2);
+      rope_rotate(v, v2, 32, tab_row, n0 % p.rope_hd);
+      epi_chunk_store(p, v2, m, arow, orow, n2);
+    } else if (rot && (n0 % p.rope_hd) == 0) {
+      // rotary half of at most 16 features: both halves inside this chunk
+      switch (p.rope_half) {
+        case 4: rope_in_chunk<4>(v, tab_row); break;
+        case 8: rope_in_chunk<8>(v, tab_row); break;
+        case 16: rope_in_chunk<16>(v, tab_row); break;
+        default: break;
+      }
+    }
+    epi_chunk_store(p, v, m, arow, orow, n0);
+  }
+  if (ROUTER && half == 0 && mvalid) p.scores[m] = rsum + __bfloat162float(p.b2[0]);
 }
 
 template <int BN, bool DUAL, bool ROUTER>
@@ -304,7 +387,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int quarter = warp & 3;   // TMEM lanes 32*quarter .. +31
     const int half = (warp - 2) >> 2;   // columns: chunks [half*NC/2, (half+1)*NC/2)
     const int row_in_tile = quarter * 32 + lane;
-    const bool rope = !ROUTER && !DUAL && p.rope_tab != nullptr;
     int it = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++it) {
       int mb, nb;
@@ -318,76 +400,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const uint32_t tacc = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C::ACC_COLS;
 
-      const int m = mb * BM + row_in_tile;
-      const bool mvalid = m < p.M;
-      int64_t arow = m;
-      if (mvalid && p.rows) arow = p.rows[m];
-      const int64_t orow = p.out_mapped ? arow : (int64_t)m;
-      const float2* tab_row = nullptr;
-      if (rope && mvalid)
-        tab_row = p.rope_tab + (int64_t)(p.rope_pos ? p.rope_pos[m] : m % p.rope_T) * p.rope_half;
-      float rsum = 0.f;
-      constexpr int NC = BN / 32;
-#pragma unroll 1
-      for (int c = 0; c < NC; ++c) {
-        // the router's row reduction stays in one warp per quarter
-        const int owner = ROUTER ? 0 : (c < NC / 2 ? 0 : 1);
-        if (owner != half) continue;
-        const int n0 = nb * BN + c * 32;
-        // rotary halves of 32 or more features: chunk c pairs with chunk c2,
-        // both handled by the owner of c
-        const bool rot = rope && n0 < p.rope_cols;
-        const bool paired = rot && p.rope_half >= 32;
-        if (paired && (n0 % p.rope_hd) >= p.rope_half) continue;   // done with its partner
-        const int c2 = paired ? c + p.rope_half / 32 : c;
-        uint32_t r[32];
-        uint32_t r2[(DUAL || !ROUTER) ? 32 : 1];
-        tmem_ld32(tacc + c * 32, r);
-        if (DUAL) tmem_ld32(tacc + BN + c * 32, r2);
-        else if (!ROUTER && paired) tmem_ld32(tacc + c2 * 32, r2);
-        tmem_ld_wait();
-        if (!mvalid || n0 >= p.N) continue;
-        float v[32];
-#pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-        if (p.bias) add_bias32(p.bias, n0, v);
-        if (ROUTER) {
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            float f[8];
-            load_vec(p.w2 + n0 + 8 * i, f);
-#pragma unroll
-            for (int j = 0; j < 8; ++j) rsum += f[j] * silu_f(v[8 * i + j]);
-          }
-          continue;
-        }
-        if (DUAL) {
-#pragma unroll
-          for (int j = 0; j < 32; ++j) v[j] = silu_f(v[j]) * __uint_as_float(r2[j]);
-        } else if (p.act == ACT_GELU) {
-#pragma unroll
-          for (int j = 0; j < 32; ++j) v[j] = gelu_f(v[j]);
-        }
-        if (!DUAL && paired) {
-          const int n2 = nb * BN + c2 * 32;
-          float v2[32];
-#pragma unroll
-          for (int j = 0; j < 32; ++j) v2[j] = __uint_as_float(r2[j]);
-          if (p.bias) add_bias32(p.bias, n2, v2);
-          rope_rotate(v, v2, 32, tab_row, n0 % p.rope_hd);
-          epi_chunk_store(p, v2, m, arow, orow, n2);
-        } else if (rot && (n0 % p.rope_hd) == 0) {
-          // rotary half of at most 16 features: both halves inside this chunk
-          switch (p.rope_half) {
-            case 4: rope_in_chunk<4>(v, tab_row); break;
-            case 8: rope_in_chunk<8>(v, tab_row); break;
-            case 16: rope_in_chunk<16>(v, tab_row); break;
-            default: break;
-          }
-        }
-        epi_chunk_store(p, v, m, arow, orow, n0);
-      }
-      if (ROUTER && half == 0 && mvalid) p.scores[m] = rsum + __bfloat162float(p.b2[0]);
+      epilogue_tile<BN, DUAL, ROUTER>(p, tacc, mb * BM + row_in_tile, nb, half);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
@@ -399,6 +412,205 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+// Two-CTA variant for large M (plain projections): a cluster of 2 CTAs owns
+// a 256 x BN output tile. Each CTA stages its own 128 A rows and BN/2 of the
+// weight rows (32 KB per stage for BN = 256, so 6 stages fit); one thread of
+// the even CTA issues tcgen05.mma.cta_group::2 (M = 256), which reads both
+// CTAs' shared memory and writes 128 accumulator rows into each CTA's TMEM.
+// Stage completion is counted on the even CTA's full barriers (armed by the
+// even CTA with both CTAs' bytes); MMA commits are multicast to the empty / accumulator-full barriers
+// of both CTAs; both CTAs' epilogue warps release the accumulator on the even
+// CTA's empty-accumulator barrier.
+template <int BN, bool DUAL>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    const __grid_constant__ CUtensorMap tmB2, const GemmDev p) {
+  using C = TileCfg<BN, DUAL, true>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sA = smem_u32(smem);
+  const uint32_t sB = sA + C::STAGES * C::A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  const uint32_t full0 = smem_u32(bars);
+  const uint32_t empty0 = full0 + 8 * C::STAGES;
+  const uint32_t tfull0 = empty0 + 8 * C::STAGES;
+  const uint32_t tempty0 = tfull0 + 16;
+  const uint32_t drain = tempty0 + 16;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * C::STAGES + 5);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  // weight tile of this CTA: plain -> rows [nb*BN + rank*BN/2, +BN/2) of W;
+  // DUAL -> rows [nb*BN, +BN) of W (even CTA) or W2 (odd CTA)
+  const CUtensorMap* tmW = (DUAL && rank == 1) ? &tmB2 : &tmB;
+  const int brow_off = DUAL ? 0 : (int)rank * C::B_ROWS;
+  const int pair = blockIdx.x >> 1;
+  const int num_pairs = gridDim.x >> 1;
+  const int num_m = (p.M + 2 * BM - 1) / (2 * BM);
+  const int num_n = (p.N + BN - 1) / BN;
+  const int num_tiles = num_m * num_n;
+  const int num_kb = (p.K + BK - 1) / BK;
+
+  pdl_trigger();
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1);              // the even CTA's producer arms both CTAs' bytes
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull0 + 8 * a, 1);
+      mbar_init(tempty0 + 8 * a, 2 * kEpiWarps);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(tmW);
+  }
+  if (warp == 1) tmem_alloc_pair(smem_u32(tmem_slot), C::TMEM_COLS);
+  tc_fence_before();
+  cluster_sync();                 // both CTAs' barriers initialised, TMEM allocated
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const uint32_t full_lead = map_to_cta(full0, 0);
+  const uint32_t tempty_lead = map_to_cta(tempty0, 0);
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer (both CTAs)
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int64_t issued = 0;
+      // Only the even CTA arrives on (and arms) a stage's full barrier, with
+      // both CTAs' bytes; the odd CTA's copies complete transactions on it,
+      // possibly before it is armed (the transaction count may go negative).
+      constexpr uint32_t tx = 2 * C::STAGE_BYTES;
+      int pre = 0;
+      if (pair < num_tiles) {
+        int mb, nb;
+        tile_coords(pair, num_m, num_n, mb, nb);
+        pre = num_kb < C::STAGES ? num_kb : C::STAGES;
+        for (int kb = 0; kb < pre; ++kb) {
+          if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * kb, tx);
+          tma_load_2d_pair(sB + kb * C::B_BYTES, tmW, kb * BK, nb * BN + brow_off,
+                           full_lead + 8 * kb);
+        }
+      }
+      pdl_wait();
+      bool first = true;
+      for (int t = pair; t < num_tiles; t += num_pairs) {
+        int mb, nb;
+        tile_coords(t, num_m, num_n, mb, nb);
+        const int arow0 = mb * 2 * BM + (int)rank * BM;
+        const int brow0 = nb * BN + brow_off;
+        bool ok = true;
+        for (int kb = 0; kb < num_kb; ++kb) {
+          const uint32_t fb = full_lead + 8 * stage;
+          if (first && kb < pre) {
+            tma_load_2d_pair(sA + stage * C::A_BYTES, &tmA, kb * BK, arow0, fb);
+          } else {
+            if (!mbar_wait_bounded(empty0 + 8 * stage, phase ^ 1, abort_flag, p.err, p.timeout_ns)) {
+              ok = false;
+              break;
+            }
+            if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * stage, tx);
+            tma_load_2d_pair(sA + stage * C::A_BYTES, &tmA, kb * BK, arow0, fb);
+            tma_load_2d_pair(sB + stage * C::B_BYTES, tmW, kb * BK, brow0, fb);
+          }
+          ++issued;
+          if (++stage == C::STAGES) { stage = 0; phase ^= 1; }
+        }
+        first = false;
+        if (!ok) break;
+      }
+      // Drain (even CTA, whose full barriers count both CTAs' copies).
+      if (rank == 0) {
+        for (int s = 0; s < C::STAGES; ++s) {
+          if (issued <= s) break;
+          const int64_t last = s + ((issued - 1 - s) / C::STAGES) * C::STAGES;
+          mbar_wait_drain(full0 + 8 * s, (uint32_t)((last / C::STAGES) & 1), p.timeout_ns);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer (even CTA)
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(2 * BM, DUAL ? 2 * BN : BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int it = 0;
+      bool ok = true;
+      for (int t = pair; t < num_tiles && ok; t += num_pairs, ++it) {
+        const int acc = it & 1;
+        if (!mbar_wait_bounded(tempty0 + 8 * acc, ((it >> 1) & 1) ^ 1, abort_flag, p.err,
+                               p.timeout_ns)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * C::ACC_COLS;
+        for (int kb = 0; kb < num_kb; ++kb) {
+          if (!mbar_wait_bounded(full0 + 8 * stage, phase, abort_flag, p.err, p.timeout_ns)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_s = sA + stage * C::A_BYTES;
+          const uint32_t b_s = sB + stage * C::B_BYTES;
+#pragma unroll
+          for (int k = 0; k < BK / UK; ++k) {
+            const uint64_t ad = smem_desc_sw128(a_s + k * UK * 2);
+            const uint64_t bd = smem_desc_sw128(b_s + k * UK * 2);
+            tc_mma_f16_pair(d_tmem, ad, bd, idesc, (kb > 0 || k > 0) ? 1u : 0u);
+          }
+          tc_commit_pair_multicast(empty0 + 8 * stage, 0x3);   // both CTAs' stage free
+          if (++stage == C::STAGES) { stage = 0; phase ^= 1; }
+        }
+        if (!ok) break;
+        tc_commit_pair_multicast(tfull0 + 8 * acc, 0x3);       // both CTAs' accumulators ready
+      }
+      tc_commit_pair_multicast(drain, 0x1);
+      mbar_wait_drain(drain, 0, p.timeout_ns);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue (warps 2..9, both CTAs)
+    pdl_wait();
+    const int quarter = warp & 3;
+    const int half = (warp - 2) >> 2;
+    const int row_in_tile = quarter * 32 + lane;
+    int it = 0;
+    for (int t = pair; t < num_tiles; t += num_pairs, ++it) {
+      int mb, nb;
+      tile_coords(t, num_m, num_n, mb, nb);
+      const int acc = it & 1;
+      int ok = 0;
+      if (lane == 0)
+        ok = mbar_wait_bounded(tfull0 + 8 * acc, (it >> 1) & 1, abort_flag, p.err, p.timeout_ns);
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t tacc = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C::ACC_COLS;
+      epilogue_tile<BN, DUAL, false>(p, tacc, mb * 2 * BM + (int)rank * BM + row_in_tile, nb, half);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(tempty_lead + 8 * acc);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();                 // the pair's MMAs and copies are done before TMEM and smem go
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, C::TMEM_COLS);
   }
 }
 
@@ -433,24 +645,7 @@ bool make_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, ui
   return r == CUDA_SUCCESS;
 }
 
-template <int BN, bool DUAL, bool ROUTER>
-cudaError_t launch(const GemmArgs& a, const Dev& dev) {
-  using C = TileCfg<BN, DUAL>;
-  static int attr_done[64] = {0};
-  int device = 0;
-  cudaGetDevice(&device);
-  if (device < 64 && !attr_done[device]) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, DUAL, ROUTER>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    attr_done[device] = 1;
-  }
-  CUtensorMap ta, tb, tb2;
-  if (!make_tmap(&ta, a.A, (uint64_t)a.M, (uint64_t)a.K, (uint64_t)a.lda, BM) ||
-      !make_tmap(&tb, a.W, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, BN) ||
-      (DUAL && !make_tmap(&tb2, a.W2, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, BN)))
-    return cudaErrorInvalidValue;
-  if (!DUAL) tb2 = tb;
+GemmDev make_dev(const GemmArgs& a, const Dev& dev) {
   GemmDev p;
   p.M = (int)a.M; p.N = a.N; p.K = a.K;
   p.act = a.epi.act;
@@ -470,10 +665,71 @@ cudaError_t launch(const GemmArgs& a, const Dev& dev) {
   p.rope_cols = a.epi.rope_cols;
   p.err = dev.err;
   p.timeout_ns = kWaitTimeoutNs;
+  return p;
+}
+
+template <int BN, bool DUAL, bool ROUTER>
+cudaError_t launch(const GemmArgs& a, const Dev& dev) {
+  using C = TileCfg<BN, DUAL>;
+  static int attr_done[64] = {0};
+  int device = 0;
+  cudaGetDevice(&device);
+  if (device < 64 && !attr_done[device]) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, DUAL, ROUTER>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    attr_done[device] = 1;
+  }
+  CUtensorMap ta, tb, tb2;
+  if (!make_tmap(&ta, a.A, (uint64_t)a.M, (uint64_t)a.K, (uint64_t)a.lda, BM) ||
+      !make_tmap(&tb, a.W, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, BN) ||
+      (DUAL && !make_tmap(&tb2, a.W2, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, BN)))
+    return cudaErrorInvalidValue;
+  if (!DUAL) tb2 = tb;
+  GemmDev p = make_dev(a, dev);
   const int64_t num_tiles = ((a.M + BM - 1) / BM) * ((a.N + BN - 1) / BN);
   const int grid = (int)(num_tiles < dev.num_sms ? num_tiles : dev.num_sms);
   return launch_pdl(gemm_tc_kernel<BN, DUAL, ROUTER>, dim3(grid), dim3(kThreads), C::SMEM_BYTES,
                     dev.stream, ta, tb, tb2, p);
+}
+
+template <int BN, bool DUAL>
+cudaError_t launch_pair(const GemmArgs& a, const Dev& dev) {
+  using C = TileCfg<BN, DUAL, true>;
+  static int attr_done[64] = {0};
+  int device = 0;
+  cudaGetDevice(&device);
+  if (device < 64 && !attr_done[device]) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc2_kernel<BN, DUAL>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    attr_done[device] = 1;
+  }
+  // A persistent grid must not exceed the CTA pairs that can be resident at
+  // once (a TPC with one SM unavailable cannot host a pair).
+  static int max_pairs[64] = {0};
+  if (device < 64 && !max_pairs[device]) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * (dev.num_sms / 2));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = C::SMEM_BYTES;
+    int n = 0;
+    cudaError_t e = cudaOccupancyMaxActiveClusters(&n, gemm_tc2_kernel<BN, DUAL>, &cfg);
+    if (e != cudaSuccess || n <= 0) return e != cudaSuccess ? e : cudaErrorInvalidConfiguration;
+    max_pairs[device] = n;
+  }
+  const int64_t cap = device < 64 ? max_pairs[device] : dev.num_sms / 2;
+  CUtensorMap ta, tb, tb2;
+  if (!make_tmap(&ta, a.A, (uint64_t)a.M, (uint64_t)a.K, (uint64_t)a.lda, BM) ||
+      !make_tmap(&tb, a.W, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, C::B_ROWS) ||
+      (DUAL && !make_tmap(&tb2, a.W2, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, C::B_ROWS)))
+    return cudaErrorInvalidValue;
+  if (!DUAL) tb2 = tb;
+  GemmDev p = make_dev(a, dev);
+  const int64_t num_tiles = ((a.M + 2 * BM - 1) / (2 * BM)) * ((a.N + BN - 1) / BN);
+  const int64_t pairs = num_tiles < cap ? num_tiles : cap;
+  return launch_pdl(gemm_tc2_kernel<BN, DUAL>, dim3((unsigned)(2 * pairs)), dim3(kThreads),
+                    C::SMEM_BYTES, dev.stream, ta, tb, tb2, p);
 }
 
 }  // namespace
@@ -484,7 +740,16 @@ cudaError_t gemm_bf16(const GemmArgs& a, const Dev& dev) {
     if (a.N != 64) return cudaErrorInvalidValue;
     return launch<64, false, true>(a, dev);
   }
-  if (a.epi.act == ACT_SWIGLU) return launch<128, true, false>(a, dev);
+  // Large M: 256-row tiles on CTA pairs when that still gives every pair of
+  // SMs at least two tiles (256 x 128 gate/up tiles for SwiGLU, 256 x 256
+  // otherwise).
+  if (a.epi.act == ACT_SWIGLU) {
+    const int64_t pair_tiles = ((a.M + 255) / 256) * ((a.N + 127) / 128);
+    if (a.N % 128 == 0 && pair_tiles >= dev.num_sms) return launch_pair<128, true>(a, dev);
+    return launch<128, true, false>(a, dev);
+  }
+  const int64_t pair_tiles = ((a.M + 255) / 256) * ((a.N + 255) / 256);
+  if (a.N % 256 == 0 && pair_tiles >= dev.num_sms) return launch_pair<256, false>(a, dev);
   // Pick the N tile that finishes in the fewest tile-time units: ceil(tiles /
   // SMs) waves, a 128-wide tile costing 0.58 of a 256-wide one (it moves 2/3
   // of the operand bytes for 1/2 of the flops).

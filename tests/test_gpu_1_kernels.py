@@ -66,7 +66,9 @@ def test_topk_special_values(A):
 
 # ---------------------------------------------------------------- projections (Eq. 2)
 @pytest.mark.parametrize("M,N,Kd", [(1, 64, 64), (127, 128, 64), (129, 256, 128), (300, 384, 192),
-                                    (1024, 2304, 768), (2050, 512, 2048), (4099, 3072, 768)])
+                                    (1024, 2304, 768), (2050, 512, 2048), (4099, 3072, 768),
+                                    # CTA-pair 256x256 tiles (large M, N % 256 == 0)
+                                    (8192, 2048, 512), (2600, 4608, 320), (10000, 4096, 1024)])
 @pytest.mark.parametrize("act", [0, 1])
 def test_linear_bf16(A, M, N, Kd, act):
     g = np.random.default_rng(M + N + Kd + act)
