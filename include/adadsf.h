@@ -207,10 +207,13 @@ adadsf_status adadsf_linear(const void *x_dev, const void *w_dev, const void *bi
  * softmax(Q K^T / sqrt(head_dim)) V, causal in packed order (which is the
  * original order, as kept positions ascend). qkv_dev [B*K, q+2kv] (rotary
  * already applied), out_dev [B*K, q]; cfg->dtype. Query head h reads kv head
- * h / (n_heads / n_kv_heads).
+ * h / (n_heads / n_kv_heads). ws: adadsf_attention_workspace_size bytes (bf16
+ * keeps the value heads transposed there for the tensor cores).
  * ---------------------------------------------------------------------- */
+size_t adadsf_attention_workspace_size(const adadsf_model_cfg *cfg, int B, int K);
 adadsf_status adadsf_causal_attention(const adadsf_model_cfg *cfg, const void *qkv_dev, int B,
-                                      int K, void *out_dev, void *stream);
+                                      int K, void *out_dev, void *ws, size_t ws_bytes,
+                                      void *stream);
 
 /* ------------------------------------------------------------------------
  * Sec. 3.4: one depth-sparse layer, in place.

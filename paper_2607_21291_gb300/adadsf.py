@@ -84,7 +84,8 @@ def lib() -> ctypes.CDLL:
             "adadsf_router_scores": (i32, [pcfg, plw, vp, i64, vp, vp, sz, vp]),
             "adadsf_topk_select": (i32, [vp, i32, i32, i32, vp, vp, vp]),
             "adadsf_linear": (i32, [vp, vp, vp, i64, i32, i32, i32, i32, vp, vp, sz, vp]),
-            "adadsf_causal_attention": (i32, [pcfg, vp, i32, i32, vp, vp]),
+            "adadsf_attention_workspace_size": (sz, [pcfg, i32, i32]),
+            "adadsf_causal_attention": (i32, [pcfg, vp, i32, i32, vp, vp, sz, vp]),
             "adadsf_sparse_layer_forward": (i32, [pcfg, plw, vp, i32, i32, i32, vp, vp, vp, sz, vp]),
             "adadsf_sparse_model_forward": (i32, [pcfg, pmw, vp, i32, i32, vp, vp, vp, vp, vp, sz, vp]),
             "adadsf_sync_check": (i32, [vp, sz, vp]),
@@ -246,10 +247,20 @@ def adadsf_linear(x: torch.Tensor, w: torch.Tensor, bias: Optional[torch.Tensor]
                                _p(out), _p(ws), ws.numel(), _s(stream)))
 
 
+def adadsf_attention_workspace_size(cfg: ModelCfg, B: int, K: int) -> int:
+    n = lib().adadsf_attention_workspace_size(ctypes.byref(cfg), B, K)
+    if n == 0:
+        raise AdadsfError(ERR_INVALID_ARG, adadsf_last_error())
+    return n
+
+
 def adadsf_causal_attention(cfg: ModelCfg, qkv: torch.Tensor, B: int, K: int, out: torch.Tensor,
-                            stream=None):
+                            ws: Optional[torch.Tensor] = None, stream=None):
     _dev(qkv, "qkv"); _dev(out, "out")
-    _check(lib().adadsf_causal_attention(ctypes.byref(cfg), _p(qkv), B, K, _p(out), _s(stream)))
+    if ws is None:
+        ws = workspace(adadsf_attention_workspace_size(cfg, B, K), qkv.device)
+    _check(lib().adadsf_causal_attention(ctypes.byref(cfg), _p(qkv), B, K, _p(out), _p(ws), ws.numel(),
+                                         _s(stream)))
 
 
 def adadsf_sparse_layer_forward(cfg: ModelCfg, w: dict, x: torch.Tensor, K: int,

@@ -202,7 +202,7 @@ struct Carver {
 };
 
 struct LayerSlots {
-  size_t scores, idx, rows, n1, n2, qkv, attn, ao, act;
+  size_t scores, idx, rows, n1, n2, qkv, vt, attn, ao, act;
 };
 
 void carve_layer(const adadsf_model_cfg* c, int B, int T, int K, Carver& cv, LayerSlots& s) {
@@ -215,6 +215,8 @@ void carve_layer(const adadsf_model_cfg* c, int B, int T, int K, Carver& cv, Lay
   s.n1 = cv.take(M * c->d * es);
   s.n2 = c->arch == ADADSF_ARCH_NEOX ? cv.take(M * c->d * es) : 0;
   s.qkv = cv.take(M * (q + 2 * kv) * es);
+  // value heads transposed for the tensor-core attention: [B][Hkv][hd][vt_pad(K)]
+  s.vt = c->dtype == ADADSF_BF16 ? cv.take((size_t)B * kv * vt_pad(K) * es) : 0;
   s.attn = cv.take(M * q * es);
   s.ao = cv.take(M * c->d * es);
   s.act = cv.take(M * c->ffn * es);
@@ -233,7 +235,7 @@ struct LayerBufs {
   int32_t* idx;
   int32_t* rows;
   const float2* rope;
-  void *n1, *n2, *qkv, *attn, *ao, *act;
+  void *n1, *n2, *qkv, *vt, *attn, *ao, *act;
 };
 
 adadsf_status run_linear(int dtype, const GemmArgs& g, const Dev& dev, const char* what) {
@@ -326,6 +328,14 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
       g.epi.rope_hd = c->head_dim;
       g.epi.rope_cols = (c->n_heads + c->n_kv_heads) * c->head_dim;
     }
+    if (tc) {
+      g.epi.vt = lb.vt;
+      g.epi.vt_seq = K;
+      g.epi.vt_pad = vt_pad(K);
+      g.epi.vt_col0 = q + kv;
+      g.epi.vt_hd = c->head_dim;
+      g.epi.vt_hkv = c->n_kv_heads;
+    }
     TRY(launch(dev, ADADSF_KERNEL_GEMM_QKV, tc, 2.0 * M * qkv_dim * d,
                (Md + (double)qkv_dim * d + (double)M * qkv_dim) * es,
                [&] { return run_linear(dt, g, dev, "qkv projection"); }));
@@ -339,8 +349,10 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
   // a6: causal attention among the kept tokens.
   TRY(launch(dev, ADADSF_KERNEL_ATTENTION, tc, 2.0 * B * c->n_heads * c->head_dim * (double)K * (K + 1),
              ((double)M * qkv_dim + (double)M * q) * es,
-             CALL(attention(dt, lb.qkv, qkv_dim, lb.attn, q, B, K, c->n_heads, c->n_kv_heads,
-                            c->head_dim, dev),
+             CALL(tc ? attention_tc(lb.qkv, qkv_dim, lb.vt, lb.attn, q, B, K, c->n_heads,
+                                    c->n_kv_heads, c->head_dim, dev)
+                     : attention(dt, lb.qkv, qkv_dim, lb.attn, q, B, K, c->n_heads, c->n_kv_heads,
+                                 c->head_dim, dev),
                   "attention")));
   if (neox) {
     // a7: attn_out = O W_o^T + b_o (packed)
@@ -665,17 +677,33 @@ adadsf_status adadsf_linear(const void* x_dev, const void* w_dev, const void* bi
                 [&] { return run_linear(dtype, g, dev, "linear"); });
 }
 
+size_t adadsf_attention_workspace_size(const adadsf_model_cfg* cfg, int B, int K) {
+  if (check_cfg(cfg) != ADADSF_OK || B < 0 || K < 0) return 0;
+  const size_t kv = (size_t)cfg->n_kv_heads * cfg->head_dim;
+  return kErrBytes + (cfg->dtype == ADADSF_BF16 ? align256((size_t)B * kv * vt_pad(K) * 2) : 0);
+}
+
 adadsf_status adadsf_causal_attention(const adadsf_model_cfg* cfg, const void* qkv_dev, int B, int K,
-                                      void* out_dev, void* stream) {
+                                      void* out_dev, void* ws, size_t ws_bytes, void* stream) {
   TRY(check_cfg(cfg));
   if (B < 0 || K < 0 || (int64_t)B * K > ((int64_t)1 << 30))
     return fail(ADADSF_ERR_INVALID_ARG, "B and K must be >= 0");
+  TRY(check_ws(ws, ws_bytes, adadsf_attention_workspace_size(cfg, B, K)));
   if (B == 0 || K == 0) return ADADSF_OK;
   NEED_PTR(qkv_dev, "qkv_dev");
   NEED_PTR(out_dev, "out_dev");
   Dev dev;
-  TRY(device_info(&dev, stream, nullptr));
+  TRY(device_info(&dev, stream, ws));
   const int q = cfg->n_heads * cfg->head_dim, kv = cfg->n_kv_heads * cfg->head_dim;
+  if (cfg->dtype == ADADSF_BF16) {
+    void* vt = at<char>(ws, kErrBytes);
+    CUDA_TRY(vt_from_qkv(qkv_dev, q + 2 * kv, q + kv, B, K, cfg->n_kv_heads, cfg->head_dim, vt, dev),
+             "value transpose");
+    CUDA_TRY(attention_tc(qkv_dev, q + 2 * kv, vt, out_dev, q, B, K, cfg->n_heads,
+                          cfg->n_kv_heads, cfg->head_dim, dev),
+             "attention");
+    return ADADSF_OK;
+  }
   CUDA_TRY(attention(cfg->dtype, qkv_dev, q + 2 * kv, out_dev, q, B, K, cfg->n_heads,
                      cfg->n_kv_heads, cfg->head_dim, dev),
            "attention");
@@ -711,6 +739,7 @@ adadsf_status adadsf_sparse_layer_forward(const adadsf_model_cfg* cfg, const ada
   lb.n1 = at<char>(ws, s.n1);
   lb.n2 = at<char>(ws, s.n2);
   lb.qkv = at<char>(ws, s.qkv);
+  lb.vt = at<char>(ws, s.vt);
   lb.attn = at<char>(ws, s.attn);
   lb.ao = at<char>(ws, s.ao);
   lb.act = at<char>(ws, s.act);
@@ -769,6 +798,7 @@ adadsf_status adadsf_sparse_model_forward(const adadsf_model_cfg* cfg, const ada
   lb.n1 = at<char>(ws, m.layer.n1);
   lb.n2 = at<char>(ws, m.layer.n2);
   lb.qkv = at<char>(ws, m.layer.qkv);
+  lb.vt = at<char>(ws, m.layer.vt);
   lb.attn = at<char>(ws, m.layer.attn);
   lb.ao = at<char>(ws, m.layer.ao);
   lb.act = at<char>(ws, m.layer.act);

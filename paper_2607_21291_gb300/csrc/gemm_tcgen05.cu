@@ -72,6 +72,8 @@ struct GemmDev {
   const float2* rope_tab;    // [T][rope_half] (cos, sin)
   const int32_t* rope_pos;   // [M] original positions, or null: m % rope_T
   int rope_T, rope_half, rope_hd, rope_cols;
+  bf16* vt;                  // transposed value heads (see Epilogue::vt)
+  int vt_seq, vt_pad, vt_col0, vt_hd, vt_hkv;
   int* err;
   unsigned long long timeout_ns;
 };
@@ -189,6 +191,15 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
 #pragma unroll
     for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
     if (p.bias) add_bias32(p.bias, n0, v);
+    if (!ROUTER && !DUAL && p.vt && n0 >= p.vt_col0) {
+      // value columns: also store this row's 32 features transposed
+      const int vc = n0 - p.vt_col0;
+      const int bseq = m / p.vt_seq, j = m - bseq * p.vt_seq;
+      bf16* dst = p.vt + ((int64_t)(bseq * p.vt_hkv + vc / p.vt_hd) * p.vt_hd + vc % p.vt_hd) *
+                             p.vt_pad + j;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) dst[(int64_t)i * p.vt_pad] = __float2bfloat16_rn(v[i]);
+    }
     if (ROUTER) {
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
@@ -615,6 +626,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 }
 
 // ---------------------------------------------------------------- host side
+}  // namespace
+
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   static std::once_flag once;
@@ -629,20 +642,27 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// Row-major bf16 [rows, cols] with leading dimension ld (elements); box of
-// 64 columns x box_rows rows, 128-byte swizzle, out-of-range reads as zero.
-bool make_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint64_t ld,
-               uint32_t box_rows) {
+// Row-major bf16 [rows, cols] with leading dimension ld (elements): boxes of
+// box_cols x box_rows with the 128-byte swizzle; out-of-range reads as zero.
+bool make_tmap_bf16(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint64_t ld,
+                    uint32_t box_cols, uint32_t box_rows) {
   auto fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {ld * 2};
-  cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+  cuuint32_t box[2] = {box_cols, box_rows};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides,
                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+namespace {
+
+bool make_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint64_t ld,
+               uint32_t box_rows) {
+  return make_tmap_bf16(m, ptr, rows, cols, ld, (uint32_t)BK, box_rows);
 }
 
 GemmDev make_dev(const GemmArgs& a, const Dev& dev) {
@@ -663,6 +683,12 @@ GemmDev make_dev(const GemmArgs& a, const Dev& dev) {
   p.rope_half = a.epi.rope_half;
   p.rope_hd = a.epi.rope_hd;
   p.rope_cols = a.epi.rope_cols;
+  p.vt = static_cast<bf16*>(a.epi.vt);
+  p.vt_seq = a.epi.vt_seq;
+  p.vt_pad = a.epi.vt_pad;
+  p.vt_col0 = a.epi.vt_col0;
+  p.vt_hd = a.epi.vt_hd;
+  p.vt_hkv = a.epi.vt_hkv;
   p.err = dev.err;
   p.timeout_ns = kWaitTimeoutNs;
   return p;

@@ -1,6 +1,7 @@
 // Host-side declarations shared by the translation units of libadadsf.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 #include <stddef.h>
@@ -42,6 +43,12 @@ struct Epilogue {
   const float2* rope_tab = nullptr;
   const int32_t* rope_pos = nullptr;
   int rope_T = 1, rope_half = 0, rope_hd = 0, rope_cols = 0;
+  // Value heads also stored transposed (bf16 tensor-core path): output
+  // column n >= vt_col0 of row m = b * vt_seq + j goes to
+  // vt[((b * vt_hkv + g) * vt_hd + e) * vt_pad + j], g = (n - vt_col0) / vt_hd,
+  // e = (n - vt_col0) % vt_hd.
+  void* vt = nullptr;
+  int vt_seq = 1, vt_pad = 0, vt_col0 = 0, vt_hd = 0, vt_hkv = 0;
 };
 
 struct GemmArgs {
@@ -58,14 +65,27 @@ struct Dev {
   int num_sms;
 };
 
+// Tensor map of a row-major bf16 [rows, cols] matrix (leading dimension ld
+// elements), box_cols x box_rows boxes, 128-byte swizzle, zero fill.
+bool make_tmap_bf16(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint64_t ld,
+                    uint32_t box_cols, uint32_t box_rows);
+
 // gemm_tcgen05.cu -- bf16 tensor-core projections (tcgen05 + TMEM + TMA).
 cudaError_t gemm_bf16(const GemmArgs& a, const Dev& dev);
 // gemm_simt.cu -- fp32 projections on CUDA cores.
 cudaError_t gemm_f32(const GemmArgs& a, const Dev& dev);
 
-// attention.cu -- causal attention among kept tokens.
+// attention.cu -- causal attention among kept tokens, fp32 storage.
 cudaError_t attention(int dtype, const void* qkv, int64_t ld_qkv, void* out, int64_t ld_out, int B,
                       int K, int n_heads, int n_kv_heads, int head_dim, const Dev& dev);
+
+// attention_tc.cu -- bf16 attention on tcgen05; V enters transposed:
+// vt[((b * Hkv + g) * hd + e) * vt_pad(K) + j].
+int vt_pad(int K);
+cudaError_t vt_from_qkv(const void* qkv, int64_t ld_qkv, int col0, int B, int K, int Hkv, int hd,
+                        void* vt, const Dev& dev);
+cudaError_t attention_tc(const void* qkv, int64_t ld_qkv, const void* vt, void* out, int64_t ld_out,
+                         int B, int K, int n_heads, int n_kv_heads, int head_dim, const Dev& dev);
 
 // rowwise.cu
 cudaError_t embed(int dtype, const int32_t* ids, int64_t n, const void* table, int vocab, int d,

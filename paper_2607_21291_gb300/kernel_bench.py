@@ -88,9 +88,10 @@ def case_attention(a, stream):
     qkv = torch.randn(B * K, shape.qkv_dim, generator=g, device="cuda").to(dt)
     out = torch.empty(B * K, shape.q_dim, device="cuda", dtype=dt)
     cfg = A.make_cfg(shape)
-    fn = lambda: A.adadsf_causal_attention(cfg, qkv, B, K, out, stream=stream)
+    ws = A.workspace(A.adadsf_attention_workspace_size(cfg, B, K))
+    fn = lambda: A.adadsf_causal_attention(cfg, qkv, B, K, out, ws=ws, stream=stream)
     flops = 2.0 * B * shape.n_heads * shape.head_dim * K * (K + 1)
-    return fn, flops, (qkv.numel() + out.numel()) * qkv.element_size(), None
+    return fn, flops, (qkv.numel() + out.numel()) * qkv.element_size(), ws
 
 
 def main():
