@@ -695,14 +695,19 @@ adadsf_status adadsf_causal_attention(const adadsf_model_cfg* cfg, const void* q
   Dev dev;
   TRY(device_info(&dev, stream, ws));
   const int q = cfg->n_heads * cfg->head_dim, kv = cfg->n_kv_heads * cfg->head_dim;
+  const double flops = 2.0 * B * cfg->n_heads * cfg->head_dim * (double)K * (K + 1);
+  const double es = elem_size(cfg->dtype);
+  const double bytes = (double)B * K * (q + 2.0 * kv + q) * es;
   if (cfg->dtype == ADADSF_BF16) {
     void* vt = at<char>(ws, kErrBytes);
-    CUDA_TRY(vt_from_qkv(qkv_dev, q + 2 * kv, q + kv, B, K, cfg->n_kv_heads, cfg->head_dim, vt, dev),
-             "value transpose");
-    CUDA_TRY(attention_tc(qkv_dev, q + 2 * kv, vt, out_dev, q, B, K, cfg->n_heads,
-                          cfg->n_kv_heads, cfg->head_dim, dev),
-             "attention");
-    return ADADSF_OK;
+    TRY(launch(dev, ADADSF_KERNEL_COPY, false, 0, 2.0 * B * K * kv * es,
+               CALL(vt_from_qkv(qkv_dev, q + 2 * kv, q + kv, B, K, cfg->n_kv_heads, cfg->head_dim, vt,
+                                dev),
+                    "value transpose")));
+    return launch(dev, ADADSF_KERNEL_ATTENTION, true, flops, bytes,
+                  CALL(attention_tc(qkv_dev, q + 2 * kv, vt, out_dev, q, B, K, cfg->n_heads,
+                                    cfg->n_kv_heads, cfg->head_dim, dev),
+                       "attention"));
   }
   CUDA_TRY(attention(cfg->dtype, qkv_dev, q + 2 * kv, out_dev, q, B, K, cfg->n_heads,
                      cfg->n_kv_heads, cfg->head_dim, dev),

@@ -3,16 +3,21 @@
 // One CTA per (128-query block, query head, sequence). Keys arrive in blocks
 // of 128; attention is causal in packed order (kept positions ascend, so this
 // is the original causal mask restricted to the kept set, Sec. 3.4).
-//   warp 0     TMA: the Q tile once, then K and V^T tiles of each key block
-//              into a 2-stage ring (128-byte swizzled, K-major operands).
+//   warp 0     TMA: the Q tile once, then the K tile of each key block into a
+//              2-stage ring released as soon as S of that block is done;
+//   warp 10    TMA: the V^T tile of each key block into a 2-stage ring
+//              released after P V (128-byte swizzled, K-major operands).
 //   warp 1     allocates TMEM; one thread issues S = Q K^T into a double-
 //              buffered TMEM S (tcgen05.mma, M = 128, N = 128) and, once the
 //              softmax warps have written P, O += P V into TMEM O (N = hd).
-//   warps 2-5  one query row per thread: read S from TMEM, mask, online
+//   warps 2-9  one query row and half of the key columns per thread (two
+//              warps per TMEM lane quarter, exchanging row maxima and sums
+//              through shared memory): read S from TMEM, mask, online
 //              softmax in fp32 (exp2 with a row maximum held at most 2^8
 //              below the true one, so O is rescaled only when the maximum
-//              grows by more than that), write P as bf16 into the swizzled
-//              operand tile, and at the end O / l -> bf16 -> global.
+//              grows by more than that), write P as bf16 into one of two
+//              swizzled operand tiles (so P of block j is written while
+//              P V of block j-1 runs), and at the end O / l -> global.
 // V enters as V^T (features x keys per key-value head), written by the QKV
 // projection's epilogue, so both MMAs read K-major operands.
 // Every barrier wait is bounded in time (device error word on give-up).
@@ -26,7 +31,9 @@ namespace {
 
 constexpr int kQB = 128;            // queries per CTA = TMEM lanes
 constexpr int kKB = 128;            // keys per block
-constexpr int kAttnThreads = 192;   // producer, MMA, 4 softmax warps
+constexpr int kSoftWarps = 8;       // two per TMEM lane quarter, each on 64 key columns
+constexpr int kVWarp = 2 + kSoftWarps;   // warp loading the V^T tiles
+constexpr int kAttnThreads = 32 * (kVWarp + 1);
 constexpr float kRescaleLog2 = 8.f; // O rescaled only when the row max grows by > 2^8
 
 template <int HD>
@@ -38,10 +45,24 @@ struct AttnCfg {
   static constexpr int V_SLAB = HD * 128;          // HD feature rows x 64 keys
   static constexpr int V_BYTES = 2 * V_SLAB;       // 128 keys
   static constexpr int P_BYTES = 2 * SLAB;         // 128 queries x 128 keys
-  static constexpr int DATA = Q_BYTES + 2 * K_BYTES + 2 * V_BYTES + P_BYTES;
-  // pad so that one CTA holds an SM (TMEM is allocated in full)
-  static constexpr int SMEM = (DATA + 2048 > 120 * 1024 ? DATA + 2048 : 120 * 1024);
+  static constexpr int DATA = Q_BYTES + 2 * K_BYTES + 2 * V_BYTES + 2 * P_BYTES;   // P double-buffered
+  static constexpr int TAIL = 256 + 2048;         // barriers, then the softmax exchange area
+  // Room left for aligning the dynamic base to 1024 bytes (the kernel checks
+  // its actual misalignment); padded so that one CTA holds an SM (TMEM is
+  // allocated in full).
+  static constexpr int SLACK = (232448 - DATA - TAIL) < 1024 ? (232448 - DATA - TAIL) : 1024;
+  static constexpr int SMEM_RAW = DATA + TAIL + SLACK;
+  static constexpr int SMEM = SMEM_RAW > 120 * 1024 ? SMEM_RAW : 120 * 1024;
+  static_assert(SLACK >= 256, "shared memory");
 };
+
+// 2^x on the SFU (ex2.approx.ftz.f32: relative error ~2^-22, flushes
+// denormal results; P is rounded to bf16 afterwards).
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
 
 struct AttnDev {
   int K;                 // kept tokens per sequence
@@ -61,23 +82,32 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
+  if (smem - smem_raw > C::SLACK) {   // the layout would not fit: report and touch nothing
+    if (threadIdx.x == 0) set_device_error(p.err, DEVERR_TIMEOUT);
+    return;
+  }
   const uint32_t sQ = smem_u32(smem);
   const uint32_t sK0 = sQ + C::Q_BYTES;
   const uint32_t sV0 = sK0 + 2 * C::K_BYTES;
-  const uint32_t sP = sV0 + 2 * C::V_BYTES;
-  uint8_t* sP_ptr = smem + (sP - sQ);
+  const uint32_t sP0 = sV0 + 2 * C::V_BYTES;       // [2]
+  uint8_t* sP_ptr = smem + (sP0 - sQ);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::DATA);
   const uint32_t b0 = smem_u32(bars);
   const uint32_t q_full = b0;
-  const uint32_t kv_full0 = b0 + 8;      // [2]
-  const uint32_t kv_empty0 = b0 + 24;    // [2]
+  const uint32_t k_full0 = b0 + 8;       // [2] K ring: free once S of the block is done
+  const uint32_t k_empty0 = b0 + 24;     // [2]
   const uint32_t s_full0 = b0 + 40;      // [2]
   const uint32_t s_free0 = b0 + 56;      // [2]
-  const uint32_t p_full = b0 + 72;
-  const uint32_t pv_done = b0 + 80;
-  const uint32_t drain = b0 + 88;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
+  const uint32_t p_full0 = b0 + 72;      // [2] per P buffer
+  const uint32_t pv_done0 = b0 + 88;     // [2] per P buffer
+  const uint32_t drain = b0 + 104;
+  const uint32_t pair0 = b0 + 112;       // [4] the two softmax warps of a lane quarter
+  const uint32_t v_full0 = b0 + 144;     // [2] V^T ring: free once P V of the block is done
+  const uint32_t v_empty0 = b0 + 160;    // [2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 22);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  // per quarter, per exchange slot (2), per half: one float per lane
+  float* xchg = reinterpret_cast<float*>(smem + C::DATA + 256);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -92,13 +122,16 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(kv_full0 + 8 * i, 1);
-      mbar_init(kv_empty0 + 8 * i, 1);
+      mbar_init(k_full0 + 8 * i, 1);
+      mbar_init(k_empty0 + 8 * i, 1);
+      mbar_init(v_full0 + 8 * i, 1);
+      mbar_init(v_empty0 + 8 * i, 1);
       mbar_init(s_full0 + 8 * i, 1);
-      mbar_init(s_free0 + 8 * i, 4);
+      mbar_init(s_free0 + 8 * i, kSoftWarps);
+      mbar_init(p_full0 + 8 * i, kSoftWarps);
+      mbar_init(pv_done0 + 8 * i, 1);
     }
-    mbar_init(p_full, 4);
-    mbar_init(pv_done, 1);
+    for (int i = 0; i < 4; ++i) mbar_init(pair0 + 8 * i, 2);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -116,34 +149,43 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const uint32_t tS = tmem_base;          // S buffers at columns 0 and 128
   const uint32_t tO = tmem_base + 256;    // O at columns 256 .. 256 + HD
 
-  if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
+  if (warp == 0 || warp == kVWarp) {
+    // ------------------------------------------------------------ TMA producers
+    // warp 0: Q once, then the K ring; warp kVWarp: the V^T ring
     if (lane == 0) {
+      const bool kprod = warp == 0;
       pdl_wait();
-      mbar_arrive_expect_tx(q_full, C::Q_BYTES);
-      for (int s = 0; s < C::HS; ++s)
-        tma_load_2d(sQ + s * C::SLAB, &tmQK, h * HD + s * 64, row0 + qb * kQB, q_full);
+      if (kprod) {
+        mbar_arrive_expect_tx(q_full, C::Q_BYTES);
+        for (int s = 0; s < C::HS; ++s)
+          tma_load_2d(sQ + s * C::SLAB, &tmQK, h * HD + s * 64, row0 + qb * kQB, q_full);
+      }
+      const uint32_t full0 = kprod ? k_full0 : v_full0;
+      const uint32_t empty0 = kprod ? k_empty0 : v_empty0;
       int issued = 0;
       for (int j = 0; j < n_kv; ++j) {
         const int st = j & 1;
-        if (!mbar_wait_bounded(kv_empty0 + 8 * st, ((j >> 1) & 1) ^ 1, abort_flag, p.err,
-                               p.timeout_ns))
+        if (!mbar_wait_bounded(empty0 + 8 * st, ((j >> 1) & 1) ^ 1, abort_flag, p.err, p.timeout_ns))
           break;
-        const uint32_t fb = kv_full0 + 8 * st;
-        mbar_arrive_expect_tx(fb, C::K_BYTES + C::V_BYTES);
-        for (int s = 0; s < C::HS; ++s)
-          tma_load_2d(sK0 + st * C::K_BYTES + s * C::SLAB, &tmQK, p.q_dim + g * HD + s * 64,
-                      row0 + j * kKB, fb);
-        for (int ks = 0; ks < 2; ++ks)
-          tma_load_2d(sV0 + st * C::V_BYTES + ks * C::V_SLAB, &tmVt, j * kKB + ks * 64,
-                      (b * p.Hkv + g) * HD, fb);
+        const uint32_t fb = full0 + 8 * st;
+        if (kprod) {
+          mbar_arrive_expect_tx(fb, C::K_BYTES);
+          for (int s = 0; s < C::HS; ++s)
+            tma_load_2d(sK0 + st * C::K_BYTES + s * C::SLAB, &tmQK, p.q_dim + g * HD + s * 64,
+                        row0 + j * kKB, fb);
+        } else {
+          mbar_arrive_expect_tx(fb, C::V_BYTES);
+          for (int ks = 0; ks < 2; ++ks)
+            tma_load_2d(sV0 + st * C::V_BYTES + ks * C::V_SLAB, &tmVt, j * kKB + ks * 64,
+                        (b * p.Hkv + g) * HD, fb);
+        }
         ++issued;
       }
       // drain: the copies issued last into each stage have landed
-      mbar_wait_drain(q_full, 0, p.timeout_ns);
+      if (kprod) mbar_wait_drain(q_full, 0, p.timeout_ns);
       for (int st = 0; st < 2 && st < issued; ++st) {
         const int last = st + ((issued - 1 - st) / 2) * 2;
-        mbar_wait_drain(kv_full0 + 8 * st, (uint32_t)((last >> 1) & 1), p.timeout_ns);
+        mbar_wait_drain(full0 + 8 * st, (uint32_t)((last >> 1) & 1), p.timeout_ns);
       }
     }
   } else if (warp == 1) {
@@ -155,7 +197,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       for (int j = 0; ok && j <= n_kv; ++j) {
         if (j < n_kv) {
           const int st = j & 1;
-          if (!mbar_wait_bounded(kv_full0 + 8 * st, (j >> 1) & 1, abort_flag, p.err, p.timeout_ns) ||
+          if (!mbar_wait_bounded(k_full0 + 8 * st, (j >> 1) & 1, abort_flag, p.err, p.timeout_ns) ||
               (j >= 2 && !mbar_wait_bounded(s_free0 + 8 * st, ((j >> 1) - 1) & 1, abort_flag, p.err,
                                             p.timeout_ns))) {
             ok = false;
@@ -170,35 +212,56 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
                        kk > 0 ? 1u : 0u);
           }
           tc_commit(s_full0 + 8 * st);
+          tc_commit(k_empty0 + 8 * st);   // K tile consumed
         }
         if (j >= 1) {
-          const int jj = j - 1, stv = jj & 1;
-          if (!mbar_wait_bounded(p_full, jj & 1, abort_flag, p.err, p.timeout_ns)) {
+          const int jj = j - 1, pb = jj & 1;   // V^T stage and P buffer of block jj
+          if (!mbar_wait_bounded(p_full0 + 8 * pb, (jj >> 1) & 1, abort_flag, p.err, p.timeout_ns) ||
+              !mbar_wait_bounded(v_full0 + 8 * pb, (jj >> 1) & 1, abort_flag, p.err, p.timeout_ns)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t vst = sV0 + stv * C::V_BYTES;
+          const uint32_t vst = sV0 + pb * C::V_BYTES;
+          const uint32_t pst = sP0 + pb * C::P_BYTES;
 #pragma unroll
           for (int kk = 0; kk < kKB / 16; ++kk) {
-            tc_mma_f16(tO, smem_desc_sw128(sP + (kk >> 2) * C::SLAB + (kk & 3) * 32),
+            tc_mma_f16(tO, smem_desc_sw128(pst + (kk >> 2) * C::SLAB + (kk & 3) * 32),
                        smem_desc_sw128(vst + (kk >> 2) * C::V_SLAB + (kk & 3) * 32), idesc_o,
                        (jj > 0 || kk > 0) ? 1u : 0u);
           }
-          tc_commit(pv_done);
-          tc_commit(kv_empty0 + 8 * stv);
+          tc_commit(pv_done0 + 8 * pb);
+          tc_commit(v_empty0 + 8 * pb);
         }
       }
       tc_commit(drain);
       mbar_wait_drain(drain, 0, p.timeout_ns);
     }
   } else {
-    // ------------------------------------------------------------ softmax (warps 2..5)
+    // ------------------------------------------------------------ softmax (warps 2..9)
     pdl_wait();
     const int quarter = warp & 3;
+    const int half = (warp - 2) >> 2;              // key columns [64 half, 64 half + 64)
     const int r = quarter * 32 + lane;             // query row in the block = TMEM lane
     const int qi = qb * kQB + r;                   // query index in the sequence
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
+    const uint32_t pairbar = pair0 + 8 * quarter;
+    uint32_t xk = 0;                               // exchanges done with the partner warp
+    // value of the partner warp (same rows, other half) for this exchange
+    auto exchange = [&](float mine, float* theirs) -> bool {
+      float* slot = xchg + ((quarter * 2 + (xk & 1)) * 2) * 32;
+      slot[half * 32 + lane] = mine;
+      __syncwarp();
+      int w = 1;
+      if (lane == 0) {
+        mbar_arrive(pairbar);
+        w = mbar_wait_bounded(pairbar, xk & 1, abort_flag, p.err, p.timeout_ns);
+      }
+      ++xk;
+      if (!__shfl_sync(0xffffffffu, w, 0)) return false;
+      *theirs = slot[(half ^ 1) * 32 + lane];
+      return true;
+    };
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < n_kv && ok; ++j) {
@@ -207,92 +270,114 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       if (lane == 0) w = mbar_wait_bounded(s_full0 + 8 * st, (j >> 1) & 1, abort_flag, p.err, p.timeout_ns);
       if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
       tc_fence_after();
-      float x[kKB];
-#pragma unroll
-      for (int c = 0; c < kKB / 32; ++c) {
+      const uint32_t s_row = tS + lane_off + st * kKB + half * 64;
+      // keys above lim (relative to this half) are masked: diagonal block only
+      const int lim = (j == qb) ? qi - j * kKB - half * 64 : kKB;
+      // pass 1: row maximum of the raw scores (scale > 0) over both halves
+      float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll 1
+      for (int c = 0; c < 2; ++c) {
         uint32_t u[32];
-        tmem_ld32(tS + lane_off + st * kKB + c * 32, u);
+        tmem_ld32(s_row + c * 32, u);
         tmem_ld_wait();
 #pragma unroll
-        for (int i = 0; i < 32; ++i) x[c * 32 + i] = __uint_as_float(u[i]);
+        for (int i = 0; i < 32; ++i) {
+          const float v = (c * 32 + i <= lim) ? __uint_as_float(u[i]) : -INFINITY;
+          mx[i & 3] = fmaxf(mx[i & 3], v);
+        }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(s_free0 + 8 * st);   // S buffer may be overwritten
-      float bmax = -INFINITY;
-      const bool diag = j == qb;
-#pragma unroll
-      for (int c = 0; c < kKB; ++c) {
-        float v = x[c] * p.scale_log2;
-        if (diag && j * kKB + c > qi) v = -INFINITY;
-        x[c] = v;
-        bmax = fmaxf(bmax, v);
-      }
+      float part = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), other;
+      if (!exchange(part, &other)) { ok = false; break; }
+      const float bmax = fmaxf(part, other) * p.scale_log2;
       bool need = false;
       if (j == 0) m_used = bmax;
       else need = bmax > m_used + kRescaleLog2;
-      // P buffer and O are free once the previous block's P V has completed
-      if (j >= 1) {
+      const int pb = j & 1;
+      // P buffer pb is free once P V of block j - 2 has completed
+      if (j >= 2) {
         int w2 = 0;
-        if (lane == 0) w2 = mbar_wait_bounded(pv_done, (j - 1) & 1, abort_flag, p.err, p.timeout_ns);
+        if (lane == 0)
+          w2 = mbar_wait_bounded(pv_done0 + 8 * pb, ((j >> 1) - 1) & 1, abort_flag, p.err, p.timeout_ns);
         if (!__shfl_sync(0xffffffffu, w2, 0)) { ok = false; break; }
       }
       if (__any_sync(0xffffffffu, need)) {
-        const float alpha = need ? exp2f(m_used - bmax) : 1.f;
+        // O is stable once P V of block j - 1 has completed; each half
+        // rescales its half of the O columns
+        int w3 = 0;
+        if (lane == 0)
+          w3 = mbar_wait_bounded(pv_done0 + 8 * (pb ^ 1), ((j - 1) >> 1) & 1, abort_flag, p.err,
+                                 p.timeout_ns);
+        if (!__shfl_sync(0xffffffffu, w3, 0)) { ok = false; break; }
+        const float alpha = need ? ex2_approx(m_used - bmax) : 1.f;
         if (need) {
           l *= alpha;
           m_used = bmax;
         }
         tc_fence_after();
 #pragma unroll 1
-        for (int c = 0; c < HD / 32; ++c) {
+        for (int c = 0; c < HD / 64; ++c) {
+          const uint32_t ta = tO + lane_off + half * (HD / 2) + c * 32;
           uint32_t u[32];
-          tmem_ld32(tO + lane_off + c * 32, u);
+          tmem_ld32(ta, u);
           tmem_ld_wait();
 #pragma unroll
           for (int i = 0; i < 32; ++i) u[i] = __float_as_uint(__uint_as_float(u[i]) * alpha);
-          tmem_st32(tO + lane_off + c * 32, u);
+          tmem_st32(ta, u);
         }
         tmem_st_wait();
       }
-      float sum = 0.f;
+      // pass 2: p = 2^(s * scale - m_used), partial row sum, this half's 64
+      // keys of P row r as bf16 into slab `half` (16-byte chunks XOR-swizzled)
+      uint8_t* prow = sP_ptr + pb * C::P_BYTES + half * C::SLAB + r * 128;
+      float sm[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 1
+      for (int c = 0; c < 2; ++c) {
+        uint32_t u[32];
+        tmem_ld32(s_row + c * 32, u);
+        tmem_ld_wait();
+        float e[32];
 #pragma unroll
-      for (int c = 0; c < kKB; ++c) {
-        const float e = exp2f(x[c] - m_used);
-        x[c] = e;
-        sum += e;
-      }
-      l += sum;
-      // P row r -> two 64-key slabs, 16-byte chunks XOR-swizzled by r % 8
+        for (int i = 0; i < 32; ++i) {
+          const float t = ex2_approx(fmaf(__uint_as_float(u[i]), p.scale_log2, -m_used));
+          e[i] = (c * 32 + i <= lim) ? t : 0.f;
+          sm[i & 3] += e[i];
+        }
 #pragma unroll
-      for (int s = 0; s < 2; ++s) {
-#pragma unroll
-        for (int ch = 0; ch < 8; ++ch) {
-          const float* e = x + s * 64 + ch * 8;
-          const uint4 q4 = make_uint4(pack_bf16x2(e[0], e[1]), pack_bf16x2(e[2], e[3]),
-                                      pack_bf16x2(e[4], e[5]), pack_bf16x2(e[6], e[7]));
-          *reinterpret_cast<uint4*>(sP_ptr + s * C::SLAB + r * 128 + ((ch ^ (r & 7)) << 4)) = q4;
+        for (int k = 0; k < 4; ++k) {
+          const int ch = c * 4 + k;
+          const float* q = e + 8 * k;
+          *reinterpret_cast<uint4*>(prow + ((ch ^ (r & 7)) << 4)) =
+              make_uint4(pack_bf16x2(q[0], q[1]), pack_bf16x2(q[2], q[3]), pack_bf16x2(q[4], q[5]),
+                         pack_bf16x2(q[6], q[7]));
         }
       }
+      l += (sm[0] + sm[1]) + (sm[2] + sm[3]);
       fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(p_full);
+      if (lane == 0) {
+        mbar_arrive(s_free0 + 8 * st);   // S buffer may be overwritten
+        mbar_arrive(p_full0 + 8 * pb);
+      }
     }
-    // epilogue: O / l
+    // epilogue: O / (l of both halves); each half stores its HD/2 columns
+    float l_other = 0.f;
+    if (ok) ok = exchange(l, &l_other);
     if (ok) {
       int w = 0;
-      if (lane == 0) w = mbar_wait_bounded(pv_done, (n_kv - 1) & 1, abort_flag, p.err, p.timeout_ns);
+      if (lane == 0)
+        w = mbar_wait_bounded(pv_done0 + 8 * ((n_kv - 1) & 1), ((n_kv - 1) >> 1) & 1, abort_flag, p.err,
+                              p.timeout_ns);
       ok = __shfl_sync(0xffffffffu, w, 0) != 0;
     }
     if (ok) {
       tc_fence_after();
-      const float inv = 1.f / l;
-      bf16* dst = p.out + (int64_t)(row0 + qi) * p.ld_out + (int64_t)h * HD;
+      const float inv = 1.f / (l + l_other);
+      bf16* dst = p.out + (int64_t)(row0 + qi) * p.ld_out + (int64_t)h * HD + half * (HD / 2);
 #pragma unroll 1
-      for (int c = 0; c < HD / 32; ++c) {
+      for (int c = 0; c < HD / 64; ++c) {
         uint32_t u[32];
-        tmem_ld32(tO + lane_off + c * 32, u);
+        tmem_ld32(tO + lane_off + half * (HD / 2) + c * 32, u);
         tmem_ld_wait();
         if (qi < p.K) {
           float v[32];
