@@ -196,8 +196,13 @@ adadsf_status adadsf_topk_select(const float *scores_dev, int B, int T, int K,
  * w_dev [n_out, k_in], bias_dev [n_out] or NULL, out_dev [M, n_out], all in
  * `dtype`. act: 0 identity, 1 exact GELU. k_in % 64 == 0, n_out % 64 == 0 for
  * bf16 (tcgen05 tensor-core path), multiples of 4 for fp32. ws: at least 256
- * bytes (the device error word).
+ * bytes (the device error word); on the bf16 path any bytes beyond the first
+ * 256 may serve as fp32 scratch for splitting a small-M product along K over
+ * clusters of CTAs (ADADSF_LINEAR_SPLIT_WS_BYTES allows every such split;
+ * with less the split is used only where it fits). ws is owned by the caller
+ * and must not be in use by another call in flight.
  * ---------------------------------------------------------------------- */
+#define ADADSF_LINEAR_SPLIT_WS_BYTES (256u + 160u * 128u * 256u * 4u)
 adadsf_status adadsf_linear(const void *x_dev, const void *w_dev, const void *bias_dev,
                             int64_t M, int n_out, int k_in, int dtype, int act, void *out_dev,
                             void *ws, size_t ws_bytes, void *stream);
@@ -271,7 +276,10 @@ typedef enum {
   ADADSF_KERNEL_GATHER_NORM, ADADSF_KERNEL_GEMM_QKV, ADADSF_KERNEL_ROPE_TABLE, ADADSF_KERNEL_ROPE,
   ADADSF_KERNEL_ATTENTION, ADADSF_KERNEL_GEMM_O, ADADSF_KERNEL_NORM2, ADADSF_KERNEL_GEMM_UP,
   ADADSF_KERNEL_GEMM_DOWN, ADADSF_KERNEL_STATS, ADADSF_KERNEL_FINAL_NORM, ADADSF_KERNEL_COPY,
-  ADADSF_KERNEL_LINEAR, ADADSF_KERNEL_SELFTEST, ADADSF_KERNEL_COUNT
+  ADADSF_KERNEL_LINEAR, ADADSF_KERNEL_SELFTEST,
+  ADADSF_KERNEL_GEMM_QKV_UP,   /* GPT-NeoX, bf16: QKV and MLP-up projections in one launch */
+  ADADSF_KERNEL_GEMM_O_DOWN,   /* GPT-NeoX, bf16: output + MLP-down projections, one accumulator */
+  ADADSF_KERNEL_COUNT
 } adadsf_kernel_kind;
 
 typedef struct {

@@ -22,6 +22,7 @@ OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_WORKSPACE_TOO_SMALL, ERR_DEV
 F32, BF16 = 0, 1
 ARCH_NEOX, ARCH_QWEN = 0, 1
 STATS_TOKEN, STATS_FLAT = 0, 1
+LINEAR_SPLIT_WS_BYTES = 256 + 160 * 128 * 256 * 4   # ADADSF_LINEAR_SPLIT_WS_BYTES
 ALLOC_RAW, ALLOC_ROUND = 1, 2
 
 TORCH_DTYPE = {F32: torch.float32, BF16: torch.bfloat16}

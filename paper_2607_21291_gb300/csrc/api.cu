@@ -202,7 +202,7 @@ struct Carver {
 };
 
 struct LayerSlots {
-  size_t scores, idx, rows, n1, n2, qkv, vt, attn, ao, act;
+  size_t scores, idx, rows, n1, n2, qkv, vt, attn, ao, act, split;
 };
 
 void carve_layer(const adadsf_model_cfg* c, int B, int T, int K, Carver& cv, LayerSlots& s) {
@@ -220,6 +220,8 @@ void carve_layer(const adadsf_model_cfg* c, int B, int T, int K, Carver& cv, Lay
   s.attn = cv.take(M * q * es);
   s.ao = cv.take(M * c->d * es);
   s.act = cv.take(M * c->ffn * es);
+  // fp32 partial tiles of projections split along K (tensor-core path)
+  s.split = c->dtype == ADADSF_BF16 ? cv.take(gemm_split_scratch_bytes()) : 0;
 }
 
 size_t rope_bytes(const adadsf_model_cfg* c, int T) { return (size_t)T * (c->rotary_dim / 2) * 8; }
@@ -236,6 +238,7 @@ struct LayerBufs {
   int32_t* rows;
   const float2* rope;
   void *n1, *n2, *qkv, *vt, *attn, *ao, *act;
+  float* split;   // null on the fp32 path
 };
 
 adadsf_status run_linear(int dtype, const GemmArgs& g, const Dev& dev, const char* what) {
@@ -312,11 +315,16 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
                               c->norm_eps, lb.n1, neox ? lb.n2 : nullptr, dev),
                   "gather+norm")));
   // a5: QKV projection (+bias), rotary at the original positions.
-  // On the tensor-core path the rotation is fused into the QKV epilogue.
+  // On the tensor-core path the rotation is fused into the QKV epilogue, and
+  // for GPT-NeoX (parallel residual) the MLP up projection of the second
+  // norm shares the launch (a8).
   const int half = c->rotary_dim / 2;
   const bool fuse_rope = tc && (half == 4 || half == 8 || half == 16 || (half > 0 && half % 32 == 0));
+  const bool neox_tc = neox && tc;
   {
     GemmArgs g = linear_args(lb.n1, d, w->w_qkv, M, qkv_dim, d);
+    g.scratch = lb.split;
+    g.scratch_bytes = lb.split ? gemm_split_scratch_bytes() : 0;
     g.epi.bias = w->b_qkv;
     g.epi.out = lb.qkv;
     g.epi.ld_out = qkv_dim;
@@ -336,9 +344,21 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
       g.epi.vt_hd = c->head_dim;
       g.epi.vt_hkv = c->n_kv_heads;
     }
-    TRY(launch(dev, ADADSF_KERNEL_GEMM_QKV, tc, 2.0 * M * qkv_dim * d,
-               (Md + (double)qkv_dim * d + (double)M * qkv_dim) * es,
-               [&] { return run_linear(dt, g, dev, "qkv projection"); }));
+    if (neox_tc) {
+      // act = GELU(LN2 x W_up^T + b_up), grouped with the QKV tiles
+      GemmArgs u = linear_args(lb.n2, d, w->w_up, M, F, d);
+      u.epi.bias = w->b_up;
+      u.epi.act = ACT_GELU;
+      u.epi.out = lb.act;
+      u.epi.ld_out = F;
+      TRY(launch(dev, ADADSF_KERNEL_GEMM_QKV_UP, true, 2.0 * M * ((double)qkv_dim + F) * d,
+                 (2.0 * Md + ((double)qkv_dim + F) * d + (double)M * (qkv_dim + F)) * es,
+                 CALL(gemm_bf16_grouped(g, u, dev), "qkv + mlp up projections")));
+    } else {
+      TRY(launch(dev, ADADSF_KERNEL_GEMM_QKV, tc, 2.0 * M * qkv_dim * d,
+                 (Md + (double)qkv_dim * d + (double)M * qkv_dim) * es,
+                 [&] { return run_linear(dt, g, dev, "qkv projection"); }));
+    }
   }
   if (c->rotary_dim > 0 && !fuse_rope)
     TRY(launch(dev, ADADSF_KERNEL_ROPE, false, 0,
@@ -354,9 +374,33 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
                      : attention(dt, lb.qkv, qkv_dim, lb.attn, q, B, K, c->n_heads, c->n_kv_heads,
                                  c->head_dim, dev),
                   "attention")));
-  if (neox) {
+  if (neox_tc) {
+    // a7 + a8 + a9 as one GEMM with two K sources (parallel residual, Eq. 2):
+    // x[row] = x[row] + O W_o^T + act W_down^T + b_o + b_down
+    GemmArgs g = linear_args(lb.attn, q, w->w_o, M, d, q);
+    g.scratch = lb.split;
+    g.scratch_bytes = lb.split ? gemm_split_scratch_bytes() : 0;
+    g.A2 = lb.act;
+    g.lda2 = F;
+    g.Wk2 = w->w_down;
+    g.ldwk2 = F;
+    g.K2 = F;
+    g.epi.bias = w->b_o;
+    g.epi.bias2 = w->b_down;
+    g.epi.add_rows = x;
+    g.epi.ld_add_rows = d;
+    g.epi.rows = rows;
+    g.epi.out_mapped = true;
+    g.epi.out = x;
+    g.epi.ld_out = d;
+    TRY(launch(dev, ADADSF_KERNEL_GEMM_O_DOWN, true, 2.0 * M * d * ((double)q + F),
+               ((double)M * (q + F) + (double)d * (q + F) + 2.0 * Md) * es,
+               [&] { return run_linear(dt, g, dev, "output + mlp down projections + residual scatter"); }));
+  } else if (neox) {
     // a7: attn_out = O W_o^T + b_o (packed)
     GemmArgs g = linear_args(lb.attn, q, w->w_o, M, d, q);
+    g.scratch = lb.split;
+    g.scratch_bytes = lb.split ? gemm_split_scratch_bytes() : 0;
     g.epi.bias = w->b_o;
     g.epi.out = lb.ao;
     g.epi.ld_out = d;
@@ -372,6 +416,8 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
                [&] { return run_linear(dt, u, dev, "mlp up"); }));
     // a8 + a9: x[row] = x[row] + attn_out + act W_down^T + b_down
     GemmArgs dn = linear_args(lb.act, F, w->w_down, M, d, F);
+    dn.scratch = lb.split;
+    dn.scratch_bytes = lb.split ? gemm_split_scratch_bytes() : 0;
     dn.epi.bias = w->b_down;
     dn.epi.add_packed = lb.ao;
     dn.epi.ld_add_packed = d;
@@ -387,6 +433,8 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
   } else {
     // a7: h = x[row] + O W_o^T (packed)
     GemmArgs g = linear_args(lb.attn, q, w->w_o, M, d, q);
+    g.scratch = lb.split;
+    g.scratch_bytes = lb.split ? gemm_split_scratch_bytes() : 0;
     g.epi.add_rows = x;
     g.epi.ld_add_rows = d;
     g.epi.rows = rows;
@@ -412,6 +460,8 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
                [&] { return run_linear(dt, u, dev, "mlp gate/up"); }));
     // a8 + a9: x[row] = h + act W_down^T
     GemmArgs dn = linear_args(lb.act, F, w->w_down, M, d, F);
+    dn.scratch = lb.split;
+    dn.scratch_bytes = lb.split ? gemm_split_scratch_bytes() : 0;
     dn.epi.add_packed = lb.ao;
     dn.epi.ld_add_packed = d;
     dn.epi.rows = rows;
@@ -667,6 +717,10 @@ adadsf_status adadsf_linear(const void* x_dev, const void* w_dev, const void* bi
   Dev dev;
   TRY(device_info(&dev, stream, ws));
   GemmArgs g = linear_args(x_dev, k_in, w_dev, M, n_out, k_in);
+  if (dtype == ADADSF_BF16 && ws_bytes > kErrBytes) {   // the rest of ws: split-K scratch
+    g.scratch = at<float>(ws, kErrBytes);
+    g.scratch_bytes = ws_bytes - kErrBytes;
+  }
   g.epi.bias = bias_dev;
   g.epi.act = act == 1 ? ACT_GELU : ACT_NONE;
   g.epi.out = out_dev;
@@ -748,6 +802,7 @@ adadsf_status adadsf_sparse_layer_forward(const adadsf_model_cfg* cfg, const ada
   lb.attn = at<char>(ws, s.attn);
   lb.ao = at<char>(ws, s.ao);
   lb.act = at<char>(ws, s.act);
+  lb.split = s.split ? at<float>(ws, s.split) : nullptr;
   if (cfg->rotary_dim > 0)
     TRY(launch(dev, ADADSF_KERNEL_ROPE_TABLE, false, 0, rope_bytes(cfg, T),
                CALL(rope_table(at<float2>(ws, rope_off), T, cfg->rotary_dim, cfg->rope_theta, dev),
@@ -807,6 +862,7 @@ adadsf_status adadsf_sparse_model_forward(const adadsf_model_cfg* cfg, const ada
   lb.attn = at<char>(ws, m.layer.attn);
   lb.ao = at<char>(ws, m.layer.ao);
   lb.act = at<char>(ws, m.layer.act);
+  lb.split = m.layer.split ? at<float>(ws, m.layer.split) : nullptr;
   const size_t xbytes = (size_t)B * T * cfg->d * es;
   int64_t idx_off = 0;
   for (int l = 0; l < cfg->n_layers; ++l) {
@@ -893,7 +949,7 @@ const char* adadsf_kernel_name(int kind) {
   static const char* names[ADADSF_KERNEL_COUNT] = {
       "embed", "router", "topk", "positions", "gather_norm", "gemm_qkv", "rope_table", "rope",
       "attention", "gemm_o", "norm2", "gemm_up", "gemm_down", "stats", "final_norm", "copy",
-      "linear", "selftest"};
+      "linear", "selftest", "gemm_qkv_up", "gemm_o_down"};
   return (kind >= 0 && kind < ADADSF_KERNEL_COUNT) ? names[kind] : "unknown";
 }
 

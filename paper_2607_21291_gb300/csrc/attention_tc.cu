@@ -142,6 +142,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     tma_prefetch_desc(&tmVt);
   }
   if (warp == 1) tmem_alloc(smem_u32(tmem_slot), 512);
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -390,6 +391,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     }
   }
 
+  // Reconverge each warp first: in the producer and MMA warps only lane 0
+  // ran the role loop, and the block barrier counts whole warps.
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {

@@ -5,7 +5,7 @@
 // tcgen05 reads natively. These are the dense contractions of Eqs. 1-2 (QKV,
 // output and MLP projections) and the router's first linear layer (Sec. 3.4).
 //
-// Kernel structure (one persistent CTA per SM, 10 warps):
+// Kernel structure (one CTA per SM, 10 warps):
 //   warp 0     TMA producer: 128x64 A tile and BNx64 W tile(s) per stage into a
 //              STAGES-deep shared-memory ring, 128-byte swizzled, signalled
 //              through mbarrier transaction counts.
@@ -15,14 +15,30 @@
 //   warps 2-9  epilogue: tcgen05.ld the accumulator (one row per thread, two
 //              warps per 32-lane TMEM quarter splitting the columns), apply
 //              bias / GELU / SwiGLU / rotary / residual / row scatter / router
-//              reduction in fp32, round once and store.
-// The accumulator is double-buffered in TMEM so the epilogue of tile i runs
-// under the main loop of tile i+1. Every barrier wait is bounded in time; on
-// give-up the CTA records DEVERR_TIMEOUT, drains its in-flight copies and
-// MMAs, frees TMEM and exits.
+//              reduction in fp32, round once and store. Per-column constants
+//              (biases, the router's second layer) are staged in shared memory
+//              and the first residual chunks loaded into registers before the
+//              accumulator is ready, so their latency hides under the K loop.
+// Three kernels share this structure:
+//   gemm_tc_kernel     persistent, 128-row tiles; double-buffered TMEM so the
+//                      epilogue of tile i runs under the main loop of tile i+1.
+//   gemm_tc2_kernel    CTA pairs (cta_group::2), 256-row tiles, for large M.
+//   gemm_tc_sk_kernel  small M: K split over the 2 or 4 CTAs of a cluster,
+//                      partial tiles exchanged through a global scratch buffer.
+// Two problem shapes beyond a single A . W^T:
+//   two K sources      out = epi(A . W^T + A2 . W2^T): the K loop reads its
+//                      first kb_split blocks through (A, W), the rest through
+//                      (A2, W2) (the GPT-NeoX output and MLP-down projections
+//                      of the parallel residual, Eq. 2, in one accumulator).
+//   grouped            two independent problems (own A, W, epilogue) share one
+//                      persistent launch (the GPT-NeoX QKV and MLP-up
+//                      projections, which read the two norms of the same rows).
+// Every barrier wait is bounded in time; on give-up the CTA records
+// DEVERR_TIMEOUT, drains its in-flight copies and MMAs, frees TMEM and exits.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <cstdlib>
 #include <mutex>
 
 #include "common.cuh"
@@ -37,6 +53,7 @@ constexpr int UK = 16;       // K of one tcgen05.mma kind::f16
 constexpr int kEpiWarps = 8;     // two per TMEM lane quarter, each on half of the columns
 constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr int kGroupM = 16;  // tile raster: 16 M-blocks share each W column block
+constexpr int kConstFloats = 256;   // staged per-column constants per epilogue warp and slot
 
 // PAIR: two-CTA variant. Plain: each CTA stages half of the BN weight rows.
 // DUAL: the even CTA stages BN rows of the first weight, the odd CTA BN rows
@@ -50,20 +67,25 @@ struct TileCfg {
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES * NUM_B;
   static constexpr int STAGES_FIT = 196608 / STAGE_BYTES;
   static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
+  static constexpr int RING_BYTES = STAGES * STAGE_BYTES;
   static constexpr int ACC_COLS = BN * (DUAL ? 2 : 1);
   static constexpr int TMEM_COLS = 2 * ACC_COLS;
-  static constexpr int BAR_BYTES = (2 * STAGES + 5) * 8 + 16;
-  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + BAR_BYTES;
+  static constexpr int BAR_BYTES = (2 * STAGES + 6) * 8 + 16;
+  static constexpr int CONST_BYTES = kEpiWarps * 2 * kConstFloats * 4;
+  static constexpr int SMEM_BYTES = RING_BYTES + 1024 + BAR_BYTES + CONST_BYTES;
   static_assert(TMEM_COLS == 128 || TMEM_COLS == 256 || TMEM_COLS == 512, "TMEM columns");
+  static_assert(BAR_BYTES % 16 == 0, "constants stay 16-byte aligned");
   static_assert(SMEM_BYTES <= 232448, "shared memory");
 };
 
 struct GemmDev {
-  int M, N, K;
+  int M, N, K;               // K: both sources together
+  int kb_split;              // k-blocks read through (tmA, tmB); the rest through (tmA2, tmB2)
   int act;
   const bf16* bias;
-  const bf16* add_packed; int64_t ld_add_packed;
-  const bf16* add_rows;   int64_t ld_add_rows;
+  const bf16* bias2;         // second bias (two K sources), or null
+  const bf16* add; int64_t ld_add;   // residual: row m, or rows[m] when add_gathered
+  int add_gathered;
   const int32_t* rows;
   int out_mapped;
   bf16* out; int64_t ld_out;
@@ -74,6 +96,7 @@ struct GemmDev {
   int rope_T, rope_half, rope_hd, rope_cols;
   bf16* vt;                  // transposed value heads (see Epilogue::vt)
   int vt_seq, vt_pad, vt_col0, vt_hd, vt_hkv;
+  float* scratch;            // split-K partial tiles (gemm_tc_sk_kernel)
   int* err;
   unsigned long long timeout_ns;
 };
@@ -88,26 +111,138 @@ __device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int& mb
   nb = r / gsz;
 }
 
-__device__ __forceinline__ float gelu_f(float v) { return 0.5f * v * (1.f + erff(v * 0.70710678118654752f)); }
-__device__ __forceinline__ float silu_f(float v) { return v / (1.f + expf(-v)); }
+__device__ __forceinline__ int tiles_of(const GemmDev& p, int bm, int bn) {
+  return p.M > 0 ? ((p.M + bm - 1) / bm) * ((p.N + bn - 1) / bn) : 0;
+}
 
-// Epilogue of one 32-column chunk of one row (all values fp32 in v[]).
-__device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, int m, int64_t arow,
-                                                int64_t orow, int n0) {
-  if (p.add_packed) {
+// Tile t of a (possibly grouped) launch: problem, block coordinates, k-blocks.
+struct TileInfo {
+  int prob, mb, nb, nkb, kb_split;
+};
+__device__ __forceinline__ TileInfo tile_info(int t, const GemmDev& p, const GemmDev& p2,
+                                              int tiles0, int bm, int bn) {
+  TileInfo ti;
+  ti.prob = t < tiles0 ? 0 : 1;
+  const GemmDev& P = ti.prob ? p2 : p;
+  const int tt = ti.prob ? t - tiles0 : t;
+  tile_coords(tt, (P.M + bm - 1) / bm, (P.N + bn - 1) / bn, ti.mb, ti.nb);
+  ti.nkb = (P.K + BK - 1) / BK;
+  ti.kb_split = ti.prob ? 0 : P.kb_split;   // the second problem reads through (tmA2, tmB2)
+  return ti;
+}
+
+// Tensor maps and K coordinate of k-block kb of a tile.
+struct KbSrc {
+  const CUtensorMap* a;
+  const CUtensorMap* b;
+  int kc;
+};
+__device__ __forceinline__ KbSrc kb_source(const TileInfo& ti, int kb, const CUtensorMap* tmA,
+                                           const CUtensorMap* tmB, const CUtensorMap* tmA2,
+                                           const CUtensorMap* tmB2) {
+  const bool second = kb >= ti.kb_split;
+  KbSrc s;
+  s.a = second ? tmA2 : tmA;
+  s.b = second ? tmB2 : tmB;
+  s.kc = (second && ti.prob == 0 ? kb - ti.kb_split : kb) * BK;
+  return s;
+}
+
+// erf by formula 7.1.26 of Abramowitz & Stegun, Handbook of Mathematical
+// Functions (|error| <= 1.5e-7): for x >= 0, erf(x) = 1 - t (a1 + t (a2 + t
+// (a3 + t (a4 + t a5)))) exp(-x^2) with t = 1 / (1 + p x); erf is odd.
+__device__ __forceinline__ float erf_as(float x) {
+  const float ax = fabsf(x);
+  const float t = __fdividef(1.f, fmaf(0.3275911f, ax, 1.f));
+  float y = fmaf(t, 1.061405429f, -1.453152027f);
+  y = fmaf(t, y, 1.421413741f);
+  y = fmaf(t, y, -0.284496736f);
+  y = fmaf(t, y, 0.254829592f);
+  y = 1.f - t * y * __expf(-ax * ax);
+  return copysignf(y, x);
+}
+__device__ __forceinline__ float gelu_f(float v) { return 0.5f * v * (1.f + erf_as(v * 0.70710678118654752f)); }
+// v sigmoid(v); the exponent is capped so the fast division stays in range.
+__device__ __forceinline__ float silu_f(float v) {
+  return v * __fdividef(1.f, 1.f + __expf(fminf(-v, 80.f)));
+}
+
+__device__ __forceinline__ void st_shared_f4(uint32_t addr, const float* f) {
+  asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(f[0]), "f"(f[1]),
+               "f"(f[2]), "f"(f[3])
+               : "memory");
+}
+__device__ __forceinline__ void ld_shared_f4(uint32_t addr, float* f) {
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(f[0]), "=f"(f[1]), "=f"(f[2]), "=f"(f[3])
+               : "r"(addr)
+               : "memory");
+}
+
+// Per-column constants of a tile, staged by each epilogue warp in its own
+// shared-memory slot (no cross-warp barrier): sc[j] = bias[n] + bias2[n] for
+// the tile's columns n = nb BN + j; the router stages sc[j] = bias[j] and
+// sc[64 + j] = w2[j]. Each lane moves 16 bytes at a time.
+template <int BN, bool ROUTER>
+__device__ __forceinline__ void stage_consts(const GemmDev& p, int nb, uint32_t sc, int lane) {
+  if (ROUTER) {
+    static_assert(!ROUTER || BN == 64, "router tile");
+    if (lane < 16) {
+      const bf16* src = lane < 8 ? p.bias : p.w2;
+      const int j = 8 * (lane & 7);
+      float f[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      if (src) load_vec(src + j, f);
+      st_shared_f4(sc + 4u * (8 * lane), f);
+      st_shared_f4(sc + 4u * (8 * lane + 4), f + 4);
+    }
+  } else {
+    for (int j8 = lane; j8 < BN / 8; j8 += 32) {
+      const int n = nb * BN + 8 * j8;
+      float f[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      if (n < p.N) {
+        if (p.bias) load_vec(p.bias + n, f);
+        if (p.bias2) {
+          float g[8];
+          load_vec(p.bias2 + n, g);
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      float f[8];
-      load_vec(p.add_packed + (int64_t)m * p.ld_add_packed + n0 + 8 * i, f);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) v[8 * i + j] += f[j];
+          for (int i = 0; i < 8; ++i) f[i] += g[i];
+        }
+      }
+      st_shared_f4(sc + 4u * (8 * j8), f);
+      st_shared_f4(sc + 4u * (8 * j8 + 4), f + 4);
     }
   }
-  if (p.add_rows) {
+  __syncwarp();
+}
+
+// v[0..31] += staged constants of columns [col, col + 32) of the tile.
+__device__ __forceinline__ void add_consts32(uint32_t sc, int col, float* v) {
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    float f[4];
+    ld_shared_f4(sc + 4u * (col + 4 * q), f);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) v[4 * q + j] += f[j];
+  }
+}
+
+// Residual chunk: 32 bf16 of row rrow at column n0, as four 16-byte words.
+__device__ __forceinline__ void load_res32(const GemmDev& p, int64_t rrow, int n0, uint4* u) {
+  const uint4* src = reinterpret_cast<const uint4*>(p.add + rrow * p.ld_add + n0);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) u[i] = src[i];
+}
+
+// Store one 32-column chunk of output row orow (adding the residual `res`
+// if RES and the problem has one).
+template <bool RES>
+__device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, const uint4* res,
+                                                int64_t orow, int n0) {
+  if (RES && p.add) {
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       float f[8];
-      load_vec(p.add_rows + arow * p.ld_add_rows + n0 + 8 * i, f);
+      unpack16(res[i], f, bf16());
 #pragma unroll
       for (int j = 0; j < 8; ++j) v[8 * i + j] += f[j];
     }
@@ -116,17 +251,49 @@ __device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, int 
   for (int i = 0; i < 4; ++i) store_vec(p.out + orow * p.ld_out + n0 + 8 * i, v + 8 * i);
 }
 
-// Rotates the pairs (a[j], b[j]) j < n by the angles of features i0 + j at
-// the row's position: a' = a cos - b sin, b' = b cos + a sin.
-__device__ __forceinline__ void rope_rotate(float* a, float* b, int n, const float2* tab_row, int i0) {
+// Rotary halves of 32 or more features: chunk c (first half of a head's
+// rotated features) and chunk c2 (second half) of row m, 8 features at a time
+// to keep few registers live: a' = a cos - b sin, b' = b cos + a sin.
+// These are query / key columns: no activation, residual or transposed copy.
+__device__ __forceinline__ void rope_pair(const GemmDev& p, uint32_t tacc, int c, int c2, int bn,
+                                          int nb, uint32_t sc, bool has_consts,
+                                          const float2* tab_row, bool mvalid, int64_t orow) {
+  const int n0 = nb * bn + c * 32, n2 = nb * bn + c2 * 32;
+  const int i0 = n0 % p.rope_hd;
+#pragma unroll 1
+  for (int g = 0; g < 4; ++g) {
+    uint32_t ra[8], rb[8];
+    tmem_ld8(tacc + c * 32 + 8 * g, ra);
+    tmem_ld8(tacc + c2 * 32 + 8 * g, rb);
+    tmem_ld_wait();
+    if (!mvalid) continue;
+    float a[8], b[8];
 #pragma unroll
-  for (int j = 0; j < 32; ++j) {
-    if (j < n) {
-      const float2 cs = tab_row[i0 + j];
+    for (int j = 0; j < 8; ++j) {
+      a[j] = __uint_as_float(ra[j]);
+      b[j] = __uint_as_float(rb[j]);
+    }
+    if (has_consts) {
+      float f[4];
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        ld_shared_f4(sc + 4u * (c * 32 + 8 * g + 4 * h), f);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) a[4 * h + j] += f[j];
+        ld_shared_f4(sc + 4u * (c2 * 32 + 8 * g + 4 * h), f);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) b[4 * h + j] += f[j];
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float2 cs = tab_row[i0 + 8 * g + j];
       const float x = a[j], y = b[j];
       a[j] = x * cs.x - y * cs.y;
       b[j] = y * cs.x + x * cs.y;
     }
+    store_vec(p.out + orow * p.ld_out + n0 + 8 * g, a);
+    store_vec(p.out + orow * p.ld_out + n2 + 8 * g, b);
   }
 }
 
@@ -142,23 +309,37 @@ __device__ __forceinline__ void rope_in_chunk(float* v, const float2* tab_row) {
   }
 }
 
-__device__ __forceinline__ void add_bias32(const bf16* bias, int n0, float* v) {
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    float f[8];
-    load_vec(bias + n0 + 8 * i, f);
-#pragma unroll
-    for (int j = 0; j < 8; ++j) v[8 * i + j] += f[j];
-  }
+// Split-K partial tile of one CTA in global scratch: fp32, column groups of
+// four outermost, [BN / 4][BM][4], so that a warp (32 consecutive rows) moves
+// 512 contiguous bytes per 16-byte access.
+__device__ __forceinline__ size_t partial_idx(int row, int col) {
+  return (size_t)(col >> 2) * BM + row;   // in float4 units
 }
 
-// Epilogue of one accumulator tile for the calling thread's row m: chunks of
-// 32 TMEM columns (this warp's half of them) -> bias / activation / rotary /
-// residual / store, or the router's row reduction.
-template <int BN, bool DUAL, bool ROUTER>
+// The partial tiles the epilogue adds (S == 0: none): those of the cluster's
+// CTAs other than `rank`, in rank order, at base + q BM bn floats.
+struct EpiRed {
+  const float* base;
+  int S, rank, bn;
+};
+
+// Values the epilogue fetched before the accumulator was ready.
+struct EpiPre {
+  uint4 res[2][4];   // residual of the first two chunks this warp finalises
+  int n;             // how many of them are valid
+};
+
+// Epilogue of one accumulator tile for the calling thread's row m over the
+// chunks [c_lo, c_hi) of 32 TMEM columns -> constants / activation / rotary /
+// residual / store, or the router's row reduction. `sc` holds the staged
+// per-column constants (has_consts), `pre` the prefetched residual chunks,
+// `red` the split-K partial to add first. ROPE: the instance for rotary
+// tiles (query / key / value projections, which have no residual).
+template <int BN, bool DUAL, bool ROUTER, bool ROPE>
 __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, int m, int nb,
-                                              int half) {
-  const bool rope = !ROUTER && !DUAL && p.rope_tab != nullptr;
+                                              int c_lo, int c_hi, uint32_t sc, bool has_consts,
+                                              const EpiPre& pre, const EpiRed& red) {
+  constexpr bool rope = ROPE && !ROUTER && !DUAL;
   const bool mvalid = m < p.M;
   int64_t arow = m;
   if (mvalid && p.rows) arow = p.rows[m];
@@ -166,32 +347,53 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
   const float2* tab_row = nullptr;
   if (rope && mvalid)
     tab_row = p.rope_tab + (int64_t)(p.rope_pos ? p.rope_pos[m] : m % p.rope_T) * p.rope_half;
+  const int row = m & (BM - 1);
   float rsum = 0.f;
-  constexpr int NC = BN / 32;
 #pragma unroll 1
-  for (int c = 0; c < NC; ++c) {
-    // the router's row reduction stays in one warp per quarter
-    const int owner = ROUTER ? 0 : (c < NC / 2 ? 0 : 1);
-    if (owner != half) continue;
+  for (int c = c_lo; c < c_hi; ++c) {
     const int n0 = nb * BN + c * 32;
-    // rotary halves of 32 or more features: chunk c pairs with chunk c2,
-    // both handled by the owner of c
+    // rotary halves of 32 or more features: chunk c pairs with chunk
+    // c + half / 32, both handled by the owner of c
     const bool rot = rope && n0 < p.rope_cols;
-    const bool paired = rot && p.rope_half >= 32;
-    if (paired && (n0 % p.rope_hd) >= p.rope_half) continue;   // done with its partner
-    const int c2 = paired ? c + p.rope_half / 32 : c;
+    if (rot && p.rope_half >= 32) {
+      if ((n0 % p.rope_hd) < p.rope_half && n0 < p.N)   // else done with its partner
+        rope_pair(p, tacc, c, c + p.rope_half / 32, BN, nb, sc, has_consts, tab_row, mvalid, orow);
+      continue;
+    }
     uint32_t r[32];
-    uint32_t r2[(DUAL || !ROUTER) ? 32 : 1];
+    uint32_t r2[DUAL ? 32 : 1];
     tmem_ld32(tacc + c * 32, r);
     if (DUAL) tmem_ld32(tacc + BN + c * 32, r2);
-    else if (!ROUTER && paired) tmem_ld32(tacc + c2 * 32, r2);
     tmem_ld_wait();
     if (!mvalid || n0 >= p.N) continue;
     float v[32];
 #pragma unroll
     for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-    if (p.bias) add_bias32(p.bias, n0, v);
-    if (!ROUTER && !DUAL && p.vt && n0 >= p.vt_col0) {
+    for (int q = 0; q < red.S; ++q) {
+      if (q == red.rank) continue;
+      const float4* src = reinterpret_cast<const float4*>(red.base + (size_t)q * BM * red.bn);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float4 f = __ldcg(src + partial_idx(row, c * 32 + 4 * j));
+        v[4 * j] += f.x;
+        v[4 * j + 1] += f.y;
+        v[4 * j + 2] += f.z;
+        v[4 * j + 3] += f.w;
+      }
+    }
+    if (ROUTER) {
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        float b[4], w[4];
+        ld_shared_f4(sc + 4u * (c * 32 + 4 * q), b);
+        ld_shared_f4(sc + 4u * (64 + c * 32 + 4 * q), w);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) rsum += w[j] * silu_f(v[4 * q + j] + b[j]);
+      }
+      continue;
+    }
+    if (has_consts) add_consts32(sc, c * 32, v);
+    if (!DUAL && p.vt && n0 >= p.vt_col0) {
       // value columns: also store this row's 32 features transposed
       const int vc = n0 - p.vt_col0;
       const int bseq = m / p.vt_seq, j = m - bseq * p.vt_seq;
@@ -200,16 +402,6 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
 #pragma unroll
       for (int i = 0; i < 32; ++i) dst[(int64_t)i * p.vt_pad] = __float2bfloat16_rn(v[i]);
     }
-    if (ROUTER) {
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        float f[8];
-        load_vec(p.w2 + n0 + 8 * i, f);
-#pragma unroll
-        for (int j = 0; j < 8; ++j) rsum += f[j] * silu_f(v[8 * i + j]);
-      }
-      continue;
-    }
     if (DUAL) {
 #pragma unroll
       for (int j = 0; j < 32; ++j) v[j] = silu_f(v[j]) * __uint_as_float(r2[j]);
@@ -217,15 +409,18 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
 #pragma unroll
       for (int j = 0; j < 32; ++j) v[j] = gelu_f(v[j]);
     }
-    if (!DUAL && paired) {
-      const int n2 = nb * BN + c2 * 32;
-      float v2[32];
+    // residual of this chunk: prefetched for the first two, else loaded now
+    uint4 res[4];
+    if (!ROPE && p.add) {
+      const int k = c - c_lo;
+      if (k < pre.n) {
 #pragma unroll
-      for (int j = 0; j < 32; ++j) v2[j] = __uint_as_float(r2[j]);
-      if (p.bias) add_bias32(p.bias, n2, v2);
-      rope_rotate(v, v2, 32, tab_row, n0 % p.rope_hd);
-      epi_chunk_store(p, v2, m, arow, orow, n2);
-    } else if (rot && (n0 % p.rope_hd) == 0) {
+        for (int i = 0; i < 4; ++i) res[i] = k == 0 ? pre.res[0][i] : pre.res[1][i];
+      } else {
+        load_res32(p, p.add_gathered ? arow : (int64_t)m, n0, res);
+      }
+    }
+    if (rot && (n0 % p.rope_hd) == 0) {
       // rotary half of at most 16 features: both halves inside this chunk
       switch (p.rope_half) {
         case 4: rope_in_chunk<4>(v, tab_row); break;
@@ -234,15 +429,64 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
         default: break;
       }
     }
-    epi_chunk_store(p, v, m, arow, orow, n0);
+    epi_chunk_store<!ROPE>(p, v, res, orow, n0);
   }
-  if (ROUTER && half == 0 && mvalid) p.scores[m] = rsum + __bfloat162float(p.b2[0]);
+  if (ROUTER && c_hi > c_lo && mvalid) p.scores[m] = rsum + __bfloat162float(p.b2[0]);
+}
+
+// Prefetch of the residual of chunks c_lo, c_lo + 1 for row m (before the
+// accumulator is ready; the residual is an input of the kernel).
+template <int BN>
+__device__ __forceinline__ void prefetch_res(const GemmDev& p, int m, int nb, int c_lo, int c_hi,
+                                             EpiPre& pre) {
+  pre.n = 0;
+  if (!p.add || m >= p.M) return;
+  const int64_t rrow = p.add_gathered ? (int64_t)p.rows[m] : (int64_t)m;
+  const int n = min(2, c_hi - c_lo);
+  for (int k = 0; k < n; ++k) {
+    const int n0 = nb * BN + (c_lo + k) * 32;
+    if (n0 >= p.N) break;
+    if (k == 0) load_res32(p, rrow, n0, pre.res[0]);
+    else load_res32(p, rrow, n0, pre.res[1]);
+    pre.n = k + 1;
+  }
+}
+
+// The epilogue warps' part of a tile once its coordinates are known: stage
+// constants, prefetch residuals, wait for the accumulator (bounded), run the
+// epilogue. Returns false if the wait gave up.
+template <int BN, bool DUAL, bool ROUTER>
+__device__ __forceinline__ bool epilogue_role(const GemmDev& P, int m, int nb, int half,
+                                              uint32_t tacc, uint32_t sc, uint32_t tfull,
+                                              uint32_t parity, volatile int* abort_flag,
+                                              int lane) {
+  constexpr int NC = BN / 32;
+  // the router's row reduction stays in one warp per quarter
+  const int c_lo = ROUTER ? (half == 0 ? 0 : NC) : half * (NC / 2);
+  const int c_hi = ROUTER ? NC : (half + 1) * (NC / 2);
+  const bool has_consts = ROUTER || P.bias || P.bias2;
+  if (has_consts) stage_consts<BN, ROUTER>(P, nb, sc, lane);
+  EpiPre pre;
+  pre.n = 0;
+  if (!P.rope_tab) prefetch_res<BN>(P, m, nb, c_lo, c_hi, pre);
+  int ok = 0;
+  if (lane == 0) ok = mbar_wait_bounded(tfull, parity, abort_flag, P.err, P.timeout_ns);
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  if (!ok) return false;
+  tc_fence_after();
+  const EpiRed none = {nullptr, 0, 0, 0};
+  if (!ROUTER && !DUAL && P.rope_tab)
+    epilogue_tile<BN, DUAL, ROUTER, true>(P, tacc, m, nb, c_lo, c_hi, sc, has_consts, pre, none);
+  else
+    epilogue_tile<BN, DUAL, ROUTER, false>(P, tacc, m, nb, c_lo, c_hi, sc, has_consts, pre, none);
+  return true;
 }
 
 template <int BN, bool DUAL, bool ROUTER>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const __grid_constant__ CUtensorMap tmB2, const GemmDev p) {
+                   const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmB2,
+                   const __grid_constant__ GemmDev p, const __grid_constant__ GemmDev p2) {
   using C = TileCfg<BN, DUAL>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -250,21 +494,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t sA = smem_u32(smem);
   const uint32_t sB = sA + C::STAGES * C::A_BYTES;
   const uint32_t sB2 = sB + C::STAGES * C::B_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::RING_BYTES);
   const uint32_t full0 = smem_u32(bars);
   const uint32_t empty0 = full0 + 8 * C::STAGES;
   const uint32_t tfull0 = empty0 + 8 * C::STAGES;
   const uint32_t tempty0 = tfull0 + 16;
   const uint32_t drain = tempty0 + 16;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * C::STAGES + 5);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * C::STAGES + 6);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const uint32_t sconst = sA + C::RING_BYTES + C::BAR_BYTES;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int num_m = (p.M + BM - 1) / BM;
-  const int num_n = (p.N + BN - 1) / BN;
-  const int num_kb = (p.K + BK - 1) / BK;
-  const int num_tiles = num_m * num_n;
+  const int tiles0 = tiles_of(p, BM, BN);
+  const int num_tiles = tiles0 + tiles_of(p2, BM, BN);
 
   pdl_trigger();
   if (threadIdx.x == 0) {
@@ -284,9 +527,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
-    if (DUAL) tma_prefetch_desc(&tmB2);
+    if (DUAL || p.kb_split * BK < p.K || p2.M > 0) {
+      if (!DUAL) tma_prefetch_desc(&tmA2);
+      tma_prefetch_desc(&tmB2);
+    }
   }
   if (warp == 1) tmem_alloc(smem_u32(tmem_slot), C::TMEM_COLS);
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -303,35 +550,35 @@ __global__ void __launch_bounds__(kThreads, 1)
       // weight tiles are requested before waiting for it.
       int pre = 0;
       if ((int)blockIdx.x < num_tiles) {
-        int mb, nb;
-        tile_coords(blockIdx.x, num_m, num_n, mb, nb);
-        pre = num_kb < C::STAGES ? num_kb : C::STAGES;
+        const TileInfo ti = tile_info(blockIdx.x, p, p2, tiles0, BM, BN);
+        pre = ti.nkb < C::STAGES ? ti.nkb : C::STAGES;
         for (int kb = 0; kb < pre; ++kb) {
+          const KbSrc src = kb_source(ti, kb, &tmA, &tmB, &tmA2, &tmB2);
           const uint32_t fb = full0 + 8 * kb;
           mbar_arrive_expect_tx(fb, tx);
-          tma_load_2d(sB + kb * C::B_BYTES, &tmB, kb * BK, nb * BN, fb);
-          if (DUAL) tma_load_2d(sB2 + kb * C::B_BYTES, &tmB2, kb * BK, nb * BN, fb);
+          tma_load_2d(sB + kb * C::B_BYTES, src.b, src.kc, ti.nb * BN, fb);
+          if (DUAL) tma_load_2d(sB2 + kb * C::B_BYTES, &tmB2, src.kc, ti.nb * BN, fb);
         }
       }
       pdl_wait();
       bool first = true;
       for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
-        int mb, nb;
-        tile_coords(t, num_m, num_n, mb, nb);
+        const TileInfo ti = tile_info(t, p, p2, tiles0, BM, BN);
         bool ok = true;
-        for (int kb = 0; kb < num_kb; ++kb) {
+        for (int kb = 0; kb < ti.nkb; ++kb) {
+          const KbSrc src = kb_source(ti, kb, &tmA, &tmB, &tmA2, &tmB2);
           const uint32_t fb = full0 + 8 * stage;
           if (first && kb < pre) {
-            tma_load_2d(sA + stage * C::A_BYTES, &tmA, kb * BK, mb * BM, fb);
+            tma_load_2d(sA + stage * C::A_BYTES, src.a, src.kc, ti.mb * BM, fb);
           } else {
             if (!mbar_wait_bounded(empty0 + 8 * stage, phase ^ 1, abort_flag, p.err, p.timeout_ns)) {
               ok = false;
               break;
             }
             mbar_arrive_expect_tx(fb, tx);
-            tma_load_2d(sA + stage * C::A_BYTES, &tmA, kb * BK, mb * BM, fb);
-            tma_load_2d(sB + stage * C::B_BYTES, &tmB, kb * BK, nb * BN, fb);
-            if (DUAL) tma_load_2d(sB2 + stage * C::B_BYTES, &tmB2, kb * BK, nb * BN, fb);
+            tma_load_2d(sA + stage * C::A_BYTES, src.a, src.kc, ti.mb * BM, fb);
+            tma_load_2d(sB + stage * C::B_BYTES, src.b, src.kc, ti.nb * BN, fb);
+            if (DUAL) tma_load_2d(sB2 + stage * C::B_BYTES, &tmB2, src.kc, ti.nb * BN, fb);
           }
           ++issued;
           if (++stage == C::STAGES) { stage = 0; phase ^= 1; }
@@ -355,6 +602,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int it = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x, ++it) {
+        const TileInfo ti = tile_info(t, p, p2, tiles0, BM, BN);
         const int acc = it & 1;
         if (!mbar_wait_bounded(tempty0 + 8 * acc, ((it >> 1) & 1) ^ 1, abort_flag, p.err,
                                p.timeout_ns)) {
@@ -363,7 +611,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * C::ACC_COLS;
-        for (int kb = 0; kb < num_kb; ++kb) {
+        for (int kb = 0; kb < ti.nkb; ++kb) {
           if (!mbar_wait_bounded(full0 + 8 * stage, phase, abort_flag, p.err, p.timeout_ns)) {
             ok = false;
             break;
@@ -400,29 +648,224 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int row_in_tile = quarter * 32 + lane;
     int it = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++it) {
-      int mb, nb;
-      tile_coords(t, num_m, num_n, mb, nb);
+      const TileInfo ti = tile_info(t, p, p2, tiles0, BM, BN);
+      const GemmDev& P = ti.prob ? p2 : p;
       const int acc = it & 1;
-      int ok = 0;
-      if (lane == 0)
-        ok = mbar_wait_bounded(tfull0 + 8 * acc, (it >> 1) & 1, abort_flag, p.err, p.timeout_ns);
-      ok = __shfl_sync(0xffffffffu, ok, 0);
-      if (!ok) break;
-      tc_fence_after();
+      const uint32_t sc = sconst + 4u * kConstFloats * ((warp - 2) * 2 + acc);
       const uint32_t tacc = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C::ACC_COLS;
-
-      epilogue_tile<BN, DUAL, ROUTER>(p, tacc, mb * BM + row_in_tile, nb, half);
+      if (!epilogue_role<BN, DUAL, ROUTER>(P, ti.mb * BM + row_in_tile, ti.nb, half, tacc, sc,
+                                           tfull0 + 8 * acc, (it >> 1) & 1, abort_flag, lane))
+        break;
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
     }
   }
 
+  // Reconverge each warp first: in the producer and MMA warps only lane 0
+  // ran the role loop, and the block barrier counts whole warps.
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+// Split-K variant for GEMMs with too few output tiles to fill the GPU (small
+// M): a cluster of S CTAs (S = 2 or 4, consecutive along x) owns one 128 x BN
+// output tile; CTA r accumulates k-blocks [r KB/S, (r+1) KB/S) in its own
+// TMEM and finalises the columns [r W, (r+1) W), W = BN / S. Reduce-scatter
+// through the L2: each CTA writes its partial of the other CTAs' columns to
+// its slot of a global scratch buffer, a cluster barrier (release / acquire)
+// orders the writes before the reads, and each CTA adds the other CTAs'
+// slots in rank order (a fixed order: the sum does not depend on timing) to
+// its own columns before the usual epilogue.
+template <int BN>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_tc_sk_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                      const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmB2,
+                      const __grid_constant__ GemmDev p) {
+  using C = TileCfg<BN, false>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const uint32_t sA = smem_u32(smem);
+  const uint32_t sB = sA + C::STAGES * C::A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::RING_BYTES);
+  const uint32_t full0 = smem_u32(bars);
+  const uint32_t empty0 = full0 + 8 * C::STAGES;
+  const uint32_t tfull = empty0 + 8 * C::STAGES;
+  const uint32_t drain = tfull + 8;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * C::STAGES + 6);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const uint32_t sconst = sA + C::RING_BYTES + C::BAR_BYTES;
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int S = (int)cluster_nctarank();
+  const int rank = (int)cluster_ctarank();
+  const int NCO = BN / S / 32;                // chunks finalised by each CTA
+  const int tile = blockIdx.x / S;
+  const TileInfo ti = tile_info(tile, p, p, 1 << 30, BM, BN);
+  const int kb0 = rank * ti.nkb / S;
+  const int kb1 = (rank + 1) * ti.nkb / S;
+  const int nkb = kb1 - kb0;
+
+  pdl_trigger();
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    mbar_init(tfull, 1);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+    fence_proxy_async_smem();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+    if (p.kb_split < ti.nkb) {
+      tma_prefetch_desc(&tmA2);
+      tma_prefetch_desc(&tmB2);
+    }
+  }
+  if (warp == 1) tmem_alloc(smem_u32(tmem_slot), BN);
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  // epilogue warps: this warp's TMEM lane quarter, its chunks of a CTA's
+  // columns (both halves when there are two or more chunks, else half 0)
+  const int quarter = warp & 3;
+  const int half = (warp - 2) >> 2;
+  const int row = quarter * 32 + lane;
+  const int m = ti.mb * BM + row;
+  const uint32_t tacc = tmem_base + ((uint32_t)(quarter * 32) << 16);
+  const uint32_t sc = sconst + 4u * kConstFloats * ((warp - 2) * 2);
+  const int h_lo = NCO >= 2 ? half * (NCO / 2) : half;
+  const int h_hi = NCO >= 2 ? (half + 1) * (NCO / 2) : 1;
+  const int c_lo = rank * NCO + h_lo, c_hi = rank * NCO + h_hi;
+  const bool has_consts = p.bias || p.bias2;
+  EpiPre pre;
+  pre.n = 0;
+  int ok = 0;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      constexpr uint32_t tx = C::STAGE_BYTES;
+      const int npre = nkb < C::STAGES ? nkb : C::STAGES;
+      for (int i = 0; i < npre; ++i) {   // weights first: independent of the previous kernel
+        const KbSrc src = kb_source(ti, kb0 + i, &tmA, &tmB, &tmA2, &tmB2);
+        mbar_arrive_expect_tx(full0 + 8 * i, tx);
+        tma_load_2d(sB + i * C::B_BYTES, src.b, src.kc, ti.nb * BN, full0 + 8 * i);
+      }
+      pdl_wait();
+      int stage = 0;
+      uint32_t phase = 0;
+      int issued = 0;
+      for (int i = 0; i < nkb; ++i) {
+        const KbSrc src = kb_source(ti, kb0 + i, &tmA, &tmB, &tmA2, &tmB2);
+        const uint32_t fb = full0 + 8 * stage;
+        if (i < npre) {
+          tma_load_2d(sA + stage * C::A_BYTES, src.a, src.kc, ti.mb * BM, fb);
+        } else {
+          if (!mbar_wait_bounded(empty0 + 8 * stage, phase ^ 1, abort_flag, p.err, p.timeout_ns))
+            break;
+          mbar_arrive_expect_tx(fb, tx);
+          tma_load_2d(sA + stage * C::A_BYTES, src.a, src.kc, ti.mb * BM, fb);
+          tma_load_2d(sB + stage * C::B_BYTES, src.b, src.kc, ti.nb * BN, fb);
+        }
+        ++issued;
+        if (++stage == C::STAGES) { stage = 0; phase ^= 1; }
+      }
+      for (int s = 0; s < C::STAGES; ++s) {
+        if (issued <= s) break;
+        const int last = s + ((issued - 1 - s) / C::STAGES) * C::STAGES;
+        mbar_wait_drain(full0 + 8 * s, (uint32_t)((last / C::STAGES) & 1), p.timeout_ns);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      bool mok = true;
+      for (int i = 0; i < nkb; ++i) {
+        if (!mbar_wait_bounded(full0 + 8 * stage, phase, abort_flag, p.err, p.timeout_ns)) {
+          mok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a_s = sA + stage * C::A_BYTES;
+        const uint32_t b_s = sB + stage * C::B_BYTES;
+#pragma unroll
+        for (int k = 0; k < BK / UK; ++k) {
+          const uint64_t ad = smem_desc_sw128(a_s + k * UK * 2);
+          const uint64_t bd = smem_desc_sw128(b_s + k * UK * 2);
+          tc_mma_f16(tmem_base, ad, bd, idesc, (i > 0 || k > 0) ? 1u : 0u);
+        }
+        tc_commit(empty0 + 8 * stage);
+        if (++stage == C::STAGES) { stage = 0; phase ^= 1; }
+      }
+      if (mok) tc_commit(tfull);
+      tc_commit(drain);
+      mbar_wait_drain(drain, 0, p.timeout_ns);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue, part 1
+    pdl_wait();
+    if (has_consts) stage_consts<BN, false>(p, ti.nb, sc, lane);
+    if (lane == 0) ok = mbar_wait_bounded(tfull, 0, abort_flag, p.err, p.timeout_ns);
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    tc_fence_after();
+    if (ok) {
+      // this CTA's partial of the other CTAs' columns -> its scratch slot
+      float4* dst = reinterpret_cast<float4*>(p.scratch + (size_t)blockIdx.x * BM * BN);
+      for (int q = 0; q < S; ++q) {
+        if (q == rank) continue;
+        for (int c = q * NCO + h_lo; c < q * NCO + h_hi; ++c) {
+          uint32_t r[32];
+          tmem_ld32(tacc + c * 32, r);
+          tmem_ld_wait();
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            __stcg(dst + partial_idx(row, c * 32 + 4 * j),
+                   make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
+                               __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3])));
+        }
+      }
+      if (h_lo < h_hi) prefetch_res<BN>(p, m, ti.nb, c_lo, c_hi, pre);
+    }
+  }
+
+  // Every CTA's partials are in the scratch buffer (release / acquire at
+  // cluster scope); a CTA that gave up still arrives.
+  __syncwarp();
+  cluster_sync();
+
+  if (warp >= 2 && ok && h_lo < h_hi) {
+    // ------------------------------------------------------------ epilogue, part 2
+    const EpiRed red = {p.scratch + (size_t)tile * S * BM * BN, S, rank, BN};
+    if (p.rope_tab)   // rotary halves of at most 16 features (one chunk)
+      epilogue_tile<BN, false, false, true>(p, tacc, m, ti.nb, c_lo, c_hi, sc, has_consts, pre, red);
+    else
+      epilogue_tile<BN, false, false, false>(p, tacc, m, ti.nb, c_lo, c_hi, sc, has_consts, pre, red);
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, BN);
   }
 }
 
@@ -434,39 +877,43 @@ __global__ void __launch_bounds__(kThreads, 1)
 // Stage completion is counted on the even CTA's full barriers (armed by the
 // even CTA with both CTAs' bytes); MMA commits are multicast to the empty / accumulator-full barriers
 // of both CTAs; both CTAs' epilogue warps release the accumulator on the even
-// CTA's empty-accumulator barrier.
+// CTA's empty-accumulator barrier. Two K sources and grouped problems work
+// as in the one-CTA kernel (not with DUAL).
 template <int BN, bool DUAL>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                    const __grid_constant__ CUtensorMap tmB2, const GemmDev p) {
+                    const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmB2,
+                    const __grid_constant__ GemmDev p, const __grid_constant__ GemmDev p2) {
   using C = TileCfg<BN, DUAL, true>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   const uint32_t sA = smem_u32(smem);
   const uint32_t sB = sA + C::STAGES * C::A_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::RING_BYTES);
   const uint32_t full0 = smem_u32(bars);
   const uint32_t empty0 = full0 + 8 * C::STAGES;
   const uint32_t tfull0 = empty0 + 8 * C::STAGES;
   const uint32_t tempty0 = tfull0 + 16;
   const uint32_t drain = tempty0 + 16;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * C::STAGES + 5);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * C::STAGES + 6);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  const uint32_t sconst = sA + C::RING_BYTES + C::BAR_BYTES;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();
   // weight tile of this CTA: plain -> rows [nb*BN + rank*BN/2, +BN/2) of W;
   // DUAL -> rows [nb*BN, +BN) of W (even CTA) or W2 (odd CTA)
-  const CUtensorMap* tmW = (DUAL && rank == 1) ? &tmB2 : &tmB;
   const int brow_off = DUAL ? 0 : (int)rank * C::B_ROWS;
   const int pair = blockIdx.x >> 1;
   const int num_pairs = gridDim.x >> 1;
-  const int num_m = (p.M + 2 * BM - 1) / (2 * BM);
-  const int num_n = (p.N + BN - 1) / BN;
-  const int num_tiles = num_m * num_n;
-  const int num_kb = (p.K + BK - 1) / BK;
+  const int tiles0 = tiles_of(p, 2 * BM, BN);
+  const int num_tiles = tiles0 + tiles_of(p2, 2 * BM, BN);
+  // DUAL: the odd CTA reads the second weight for every k-block
+  auto wmap = [&](const KbSrc& s) -> const CUtensorMap* {
+    return DUAL ? (rank == 1 ? &tmB2 : &tmB) : s.b;
+  };
 
   pdl_trigger();
   if (threadIdx.x == 0) {
@@ -484,9 +931,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   }
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmA);
-    tma_prefetch_desc(tmW);
+    tma_prefetch_desc(&tmB);
+    if (DUAL || p.kb_split * BK < p.K || p2.M > 0) {
+      if (!DUAL) tma_prefetch_desc(&tmA2);
+      tma_prefetch_desc(&tmB2);
+    }
   }
   if (warp == 1) tmem_alloc_pair(smem_u32(tmem_slot), C::TMEM_COLS);
+  __syncwarp();
   tc_fence_before();
   cluster_sync();                 // both CTAs' barriers initialised, TMEM allocated
   tc_fence_after();
@@ -506,35 +958,35 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       constexpr uint32_t tx = 2 * C::STAGE_BYTES;
       int pre = 0;
       if (pair < num_tiles) {
-        int mb, nb;
-        tile_coords(pair, num_m, num_n, mb, nb);
-        pre = num_kb < C::STAGES ? num_kb : C::STAGES;
+        const TileInfo ti = tile_info(pair, p, p2, tiles0, 2 * BM, BN);
+        pre = ti.nkb < C::STAGES ? ti.nkb : C::STAGES;
         for (int kb = 0; kb < pre; ++kb) {
+          const KbSrc src = kb_source(ti, kb, &tmA, &tmB, &tmA2, &tmB2);
           if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * kb, tx);
-          tma_load_2d_pair(sB + kb * C::B_BYTES, tmW, kb * BK, nb * BN + brow_off,
+          tma_load_2d_pair(sB + kb * C::B_BYTES, wmap(src), src.kc, ti.nb * BN + brow_off,
                            full_lead + 8 * kb);
         }
       }
       pdl_wait();
       bool first = true;
       for (int t = pair; t < num_tiles; t += num_pairs) {
-        int mb, nb;
-        tile_coords(t, num_m, num_n, mb, nb);
-        const int arow0 = mb * 2 * BM + (int)rank * BM;
-        const int brow0 = nb * BN + brow_off;
+        const TileInfo ti = tile_info(t, p, p2, tiles0, 2 * BM, BN);
+        const int arow0 = ti.mb * 2 * BM + (int)rank * BM;
+        const int brow0 = ti.nb * BN + brow_off;
         bool ok = true;
-        for (int kb = 0; kb < num_kb; ++kb) {
+        for (int kb = 0; kb < ti.nkb; ++kb) {
+          const KbSrc src = kb_source(ti, kb, &tmA, &tmB, &tmA2, &tmB2);
           const uint32_t fb = full_lead + 8 * stage;
           if (first && kb < pre) {
-            tma_load_2d_pair(sA + stage * C::A_BYTES, &tmA, kb * BK, arow0, fb);
+            tma_load_2d_pair(sA + stage * C::A_BYTES, src.a, src.kc, arow0, fb);
           } else {
             if (!mbar_wait_bounded(empty0 + 8 * stage, phase ^ 1, abort_flag, p.err, p.timeout_ns)) {
               ok = false;
               break;
             }
             if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * stage, tx);
-            tma_load_2d_pair(sA + stage * C::A_BYTES, &tmA, kb * BK, arow0, fb);
-            tma_load_2d_pair(sB + stage * C::B_BYTES, tmW, kb * BK, brow0, fb);
+            tma_load_2d_pair(sA + stage * C::A_BYTES, src.a, src.kc, arow0, fb);
+            tma_load_2d_pair(sB + stage * C::B_BYTES, wmap(src), src.kc, brow0, fb);
           }
           ++issued;
           if (++stage == C::STAGES) { stage = 0; phase ^= 1; }
@@ -560,6 +1012,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       int it = 0;
       bool ok = true;
       for (int t = pair; t < num_tiles && ok; t += num_pairs, ++it) {
+        const TileInfo ti = tile_info(t, p, p2, tiles0, 2 * BM, BN);
         const int acc = it & 1;
         if (!mbar_wait_bounded(tempty0 + 8 * acc, ((it >> 1) & 1) ^ 1, abort_flag, p.err,
                                p.timeout_ns)) {
@@ -568,7 +1021,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * C::ACC_COLS;
-        for (int kb = 0; kb < num_kb; ++kb) {
+        for (int kb = 0; kb < ti.nkb; ++kb) {
           if (!mbar_wait_bounded(full0 + 8 * stage, phase, abort_flag, p.err, p.timeout_ns)) {
             ok = false;
             break;
@@ -599,23 +1052,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const int row_in_tile = quarter * 32 + lane;
     int it = 0;
     for (int t = pair; t < num_tiles; t += num_pairs, ++it) {
-      int mb, nb;
-      tile_coords(t, num_m, num_n, mb, nb);
+      const TileInfo ti = tile_info(t, p, p2, tiles0, 2 * BM, BN);
+      const GemmDev& P = ti.prob ? p2 : p;
       const int acc = it & 1;
-      int ok = 0;
-      if (lane == 0)
-        ok = mbar_wait_bounded(tfull0 + 8 * acc, (it >> 1) & 1, abort_flag, p.err, p.timeout_ns);
-      ok = __shfl_sync(0xffffffffu, ok, 0);
-      if (!ok) break;
-      tc_fence_after();
+      const uint32_t sc = sconst + 4u * kConstFloats * ((warp - 2) * 2 + acc);
       const uint32_t tacc = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C::ACC_COLS;
-      epilogue_tile<BN, DUAL, false>(p, tacc, mb * 2 * BM + (int)rank * BM + row_in_tile, nb, half);
+      if (!epilogue_role<BN, DUAL, false>(P, ti.mb * 2 * BM + (int)rank * BM + row_in_tile, ti.nb,
+                                          half, tacc, sc, tfull0 + 8 * acc, (it >> 1) & 1,
+                                          abort_flag, lane))
+        break;
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(tempty_lead + 8 * acc);
     }
   }
 
+  // Reconverge each warp first: in the producer and MMA warps only lane 0
+  // ran the role loop, and the block barrier counts whole warps.
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   cluster_sync();                 // the pair's MMAs and copies are done before TMEM and smem go
@@ -665,13 +1119,25 @@ bool make_tmap(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, ui
   return make_tmap_bf16(m, ptr, rows, cols, ld, (uint32_t)BK, box_rows);
 }
 
-GemmDev make_dev(const GemmArgs& a, const Dev& dev) {
-  GemmDev p;
-  p.M = (int)a.M; p.N = a.N; p.K = a.K;
+bool make_dev(const GemmArgs& a, const Dev& dev, GemmDev& p) {
+  p = GemmDev{};
+  if (a.epi.add_packed && a.epi.add_rows) return false;   // one residual source per launch
+  if (a.epi.rope_tab && (a.epi.add_packed || a.epi.add_rows)) return false;   // rotary tiles: none
+  if (a.K2 > 0 && a.K % BK != 0) return false;            // the K sources meet on a k-block
+  p.M = (int)a.M; p.N = a.N; p.K = a.K + (a.K2 > 0 ? a.K2 : 0);
+  p.kb_split = a.K2 > 0 ? a.K / BK : (p.K + BK - 1) / BK;
   p.act = a.epi.act;
   p.bias = static_cast<const bf16*>(a.epi.bias);
-  p.add_packed = static_cast<const bf16*>(a.epi.add_packed); p.ld_add_packed = a.epi.ld_add_packed;
-  p.add_rows = static_cast<const bf16*>(a.epi.add_rows); p.ld_add_rows = a.epi.ld_add_rows;
+  p.bias2 = static_cast<const bf16*>(a.epi.bias2);
+  if (a.epi.add_packed) {
+    p.add = static_cast<const bf16*>(a.epi.add_packed);
+    p.ld_add = a.epi.ld_add_packed;
+    p.add_gathered = 0;
+  } else if (a.epi.add_rows) {
+    p.add = static_cast<const bf16*>(a.epi.add_rows);
+    p.ld_add = a.epi.ld_add_rows;
+    p.add_gathered = a.epi.rows ? 1 : 0;
+  }
   p.rows = a.epi.rows;
   p.out_mapped = a.epi.out_mapped ? 1 : 0;
   p.out = static_cast<bf16*>(a.epi.out); p.ld_out = a.epi.ld_out;
@@ -689,13 +1155,52 @@ GemmDev make_dev(const GemmArgs& a, const Dev& dev) {
   p.vt_col0 = a.epi.vt_col0;
   p.vt_hd = a.epi.vt_hd;
   p.vt_hkv = a.epi.vt_hkv;
+  p.scratch = a.scratch;
   p.err = dev.err;
   p.timeout_ns = kWaitTimeoutNs;
-  return p;
+  return true;
+}
+
+// Tensor maps of one problem: (A, W) and, for two K sources, (A2, W2).
+bool problem_maps(const GemmArgs& a, uint32_t a_rows, uint32_t b_rows, CUtensorMap& ta,
+                  CUtensorMap& tb, CUtensorMap* ta2, CUtensorMap* tb2) {
+  if (!make_tmap(&ta, a.A, (uint64_t)a.M, (uint64_t)a.K, (uint64_t)a.lda, a_rows) ||
+      !make_tmap(&tb, a.W, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, b_rows))
+    return false;
+  if (a.K2 > 0) {
+    if (!ta2 || !tb2 ||
+        !make_tmap(ta2, a.A2, (uint64_t)a.M, (uint64_t)a.K2, (uint64_t)a.lda2, a_rows) ||
+        !make_tmap(tb2, a.Wk2, (uint64_t)a.N, (uint64_t)a.K2, (uint64_t)a.ldwk2, b_rows))
+      return false;
+  }
+  return true;
+}
+
+// Maps and device descriptors for a launch of problem `a` (plus the grouped
+// problem `b`, or the DUAL second weight).
+template <bool DUAL>
+cudaError_t prepare(const GemmArgs& a, const GemmArgs* b, uint32_t a_rows, uint32_t b_rows,
+                    const Dev& dev, CUtensorMap (&tm)[4], GemmDev& p, GemmDev& p2) {
+  if (!make_dev(a, dev, p)) return cudaErrorInvalidValue;
+  p2 = GemmDev{};
+  if (!problem_maps(a, a_rows, b_rows, tm[0], tm[1], &tm[2], &tm[3])) return cudaErrorInvalidValue;
+  if (DUAL) {
+    if (!make_tmap(&tm[3], a.W2, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, b_rows))
+      return cudaErrorInvalidValue;
+    tm[2] = tm[0];
+  } else if (b) {
+    if (a.K2 > 0 || b->K2 > 0 || !make_dev(*b, dev, p2)) return cudaErrorInvalidValue;
+    if (!problem_maps(*b, a_rows, b_rows, tm[2], tm[3], nullptr, nullptr))
+      return cudaErrorInvalidValue;
+  } else if (a.K2 == 0) {
+    tm[2] = tm[0];
+    tm[3] = tm[1];
+  }
+  return cudaSuccess;
 }
 
 template <int BN, bool DUAL, bool ROUTER>
-cudaError_t launch(const GemmArgs& a, const Dev& dev) {
+cudaError_t launch(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
   using C = TileCfg<BN, DUAL>;
   static int attr_done[64] = {0};
   int device = 0;
@@ -706,21 +1211,19 @@ cudaError_t launch(const GemmArgs& a, const Dev& dev) {
     if (e != cudaSuccess) return e;
     attr_done[device] = 1;
   }
-  CUtensorMap ta, tb, tb2;
-  if (!make_tmap(&ta, a.A, (uint64_t)a.M, (uint64_t)a.K, (uint64_t)a.lda, BM) ||
-      !make_tmap(&tb, a.W, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, BN) ||
-      (DUAL && !make_tmap(&tb2, a.W2, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, BN)))
-    return cudaErrorInvalidValue;
-  if (!DUAL) tb2 = tb;
-  GemmDev p = make_dev(a, dev);
-  const int64_t num_tiles = ((a.M + BM - 1) / BM) * ((a.N + BN - 1) / BN);
+  CUtensorMap tm[4];
+  GemmDev p, p2;
+  cudaError_t e = prepare<DUAL>(a, b, BM, BN, dev, tm, p, p2);
+  if (e != cudaSuccess) return e;
+  int64_t num_tiles = ((a.M + BM - 1) / BM) * ((a.N + BN - 1) / BN);
+  if (b) num_tiles += ((b->M + BM - 1) / BM) * ((b->N + BN - 1) / BN);
   const int grid = (int)(num_tiles < dev.num_sms ? num_tiles : dev.num_sms);
   return launch_pdl(gemm_tc_kernel<BN, DUAL, ROUTER>, dim3(grid), dim3(kThreads), C::SMEM_BYTES,
-                    dev.stream, ta, tb, tb2, p);
+                    dev.stream, tm[0], tm[1], tm[2], tm[3], p, p2);
 }
 
 template <int BN, bool DUAL>
-cudaError_t launch_pair(const GemmArgs& a, const Dev& dev) {
+cudaError_t launch_pair(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
   using C = TileCfg<BN, DUAL, true>;
   static int attr_done[64] = {0};
   int device = 0;
@@ -745,47 +1248,169 @@ cudaError_t launch_pair(const GemmArgs& a, const Dev& dev) {
     max_pairs[device] = n;
   }
   const int64_t cap = device < 64 ? max_pairs[device] : dev.num_sms / 2;
-  CUtensorMap ta, tb, tb2;
-  if (!make_tmap(&ta, a.A, (uint64_t)a.M, (uint64_t)a.K, (uint64_t)a.lda, BM) ||
-      !make_tmap(&tb, a.W, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, C::B_ROWS) ||
-      (DUAL && !make_tmap(&tb2, a.W2, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, C::B_ROWS)))
-    return cudaErrorInvalidValue;
-  if (!DUAL) tb2 = tb;
-  GemmDev p = make_dev(a, dev);
-  const int64_t num_tiles = ((a.M + 2 * BM - 1) / (2 * BM)) * ((a.N + BN - 1) / BN);
+  CUtensorMap tm[4];
+  GemmDev p, p2;
+  cudaError_t e = prepare<DUAL>(a, b, BM, C::B_ROWS, dev, tm, p, p2);
+  if (e != cudaSuccess) return e;
+  int64_t num_tiles = ((a.M + 2 * BM - 1) / (2 * BM)) * ((a.N + BN - 1) / BN);
+  if (b) num_tiles += ((b->M + 2 * BM - 1) / (2 * BM)) * ((b->N + BN - 1) / BN);
   const int64_t pairs = num_tiles < cap ? num_tiles : cap;
   return launch_pdl(gemm_tc2_kernel<BN, DUAL>, dim3((unsigned)(2 * pairs)), dim3(kThreads),
-                    C::SMEM_BYTES, dev.stream, ta, tb, tb2, p);
+                    C::SMEM_BYTES, dev.stream, tm[0], tm[1], tm[2], tm[3], p, p2);
+}
+
+// Clusters of S CTAs of the split-K kernel that can be resident at once
+// (cached per device and size; 0 if none).
+template <int BN>
+int sk_max_clusters(int S, const Dev& dev) {
+  using C = TileCfg<BN, false>;
+  static int cache[64][5] = {};
+  static int attr_done[64] = {0};
+  int device = 0;
+  cudaGetDevice(&device);
+  if (device >= 64 || S < 2 || S > 4) return 0;
+  if (!attr_done[device]) {
+    if (cudaFuncSetAttribute(gemm_tc_sk_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             C::SMEM_BYTES) != cudaSuccess)
+      return 0;
+    attr_done[device] = 1;
+  }
+  if (!cache[device][S]) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(S * (dev.num_sms / S)));
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = C::SMEM_BYTES;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)S;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_sk_kernel<BN>, &cfg) != cudaSuccess) n = 0;
+    cache[device][S] = n > 0 ? n : -1;
+  }
+  return cache[device][S] > 0 ? cache[device][S] : 0;
+}
+
+// Tuning override: ADADSF_GEMM_SPLIT=1 disables the split-K kernel, 2 or 4
+// forces that cluster size where it applies; unset or 0 chooses by the cost
+// model.
+int split_override() {
+  static int v = -1;
+  if (v < 0) {
+    const char* e = getenv("ADADSF_GEMM_SPLIT");
+    v = e ? atoi(e) : 0;
+    if (v != 1 && v != 2 && v != 4) v = 0;
+  }
+  return v;
+}
+
+template <int BN>
+cudaError_t launch_sk(const GemmArgs& a, const Dev& dev, int S) {
+  using C = TileCfg<BN, false>;
+  CUtensorMap tm[4];
+  GemmDev p, p2;
+  cudaError_t e = prepare<false>(a, nullptr, BM, BN, dev, tm, p, p2);
+  if (e != cudaSuccess) return e;
+  const int64_t num_tiles = ((a.M + BM - 1) / BM) * ((a.N + BN - 1) / BN);
+  return launch_pdl_cluster(gemm_tc_sk_kernel<BN>, dim3((unsigned)(num_tiles * S)), dim3(kThreads),
+                            C::SMEM_BYTES, dev.stream, S, tm[0], tm[1], tm[2], tm[3], p);
+}
+
+// Plain and two-source projections (no SwiGLU, no router). Cost model in
+// units of one k-block of one CTA: a tcgen05.mma with M = 128 takes about
+// the same time for N = 128 as for N = 256, so a k-block costs the same for
+// every tile width and a launch costs (tile rounds) x (k-blocks per CTA),
+// plus its epilogue (per 32-column chunk of a thread) and, split along K,
+// the exchange of partial tiles through the L2 (needs a.scratch). CTA pairs (256-row tiles) move half of the
+// weight bytes per SM, the tie-breaker for large M.
+cudaError_t gemm_plain(const GemmArgs& a, const Dev& dev) {
+  const int num_kb = (a.K + (a.K2 > 0 ? a.K2 : 0) + BK - 1) / BK;
+  const int64_t mb128 = (a.M + BM - 1) / BM, mb256 = (a.M + 2 * BM - 1) / (2 * BM);
+  const int64_t t128 = mb128 * ((a.N + 127) / 128), t256 = mb128 * ((a.N + 255) / 256);
+  const int64_t tpair = mb256 * ((a.N + 255) / 256);
+  const int64_t sms = dev.num_sms;
+  constexpr int64_t kChunk = 2;      // 2 x (k-block cost) per epilogue chunk of 32 columns
+  constexpr int64_t kExchange = 4;   // partial-tile exchange through distributed shared memory
+  auto rounds = [](int64_t tiles, int64_t slots) { return (tiles + slots - 1) / slots; };
+  const int64_t cost_pair = rounds(tpair, sms / 2) * num_kb + 4 * kChunk;
+  const int64_t cost256 = rounds(t256, sms) * num_kb + 4 * kChunk;
+  const int64_t cost128 = rounds(t128, sms) * num_kb + 2 * kChunk;
+  int64_t best = cost_pair;
+  int pick = 0;   // 0 pair, 1 one-CTA 256, 2 one-CTA 128, 3 split 256, 4 split 128
+  if (cost256 < best) { best = cost256; pick = 1; }
+  if (cost128 < best) { best = cost128; pick = 2; }
+  // Split along K (rotary tiles only with halves of at most 16 features,
+  // which stay inside one 32-column chunk).
+  const int force = split_override();
+  int split_s = 0;
+  const bool can_split = force != 1 && num_kb >= 2 && a.scratch != nullptr &&
+                         (a.epi.rope_tab == nullptr || a.epi.rope_half <= 16);
+  auto fits = [&](int64_t tiles, int S, int bn) {
+    return (size_t)(tiles * S) * BM * bn * 4 <= a.scratch_bytes;
+  };
+  if (can_split) {
+    for (int S = 2; S <= 4; S += 2) {
+      if (S > num_kb || (force && force != S)) continue;
+      const int64_t k = (num_kb + S - 1) / S + kExchange;
+      if (fits(t256, S, 256) && t256 <= sk_max_clusters<256>(S, dev)) {
+        const int64_t c = k + kChunk * ((256 / S / 32 + 1) / 2);
+        if (c < best || force) { best = c; pick = 3; split_s = S; }
+      }
+      if (fits(t128, S, 128) && t128 <= sk_max_clusters<128>(S, dev)) {
+        const int64_t c = k + kChunk * ((128 / S / 32 + 1) / 2);
+        if (c < best || (force && pick != 3)) { best = c; pick = 4; split_s = S; }
+      }
+    }
+  }
+  switch (pick) {
+    case 0: return launch_pair<256, false>(a, nullptr, dev);
+    case 1: return launch<256, false, false>(a, nullptr, dev);
+    case 2: return launch<128, false, false>(a, nullptr, dev);
+    case 3: return launch_sk<256>(a, dev, split_s);
+    default: return launch_sk<128>(a, dev, split_s);
+  }
 }
 
 }  // namespace
 
+// Room for the partial tiles of up to 160 CTAs of 128 x 256 fp32 (every
+// split the cost model can choose on a GPU with up to 160 SMs).
+size_t gemm_split_scratch_bytes() { return (size_t)160 * BM * 256 * 4; }
+
 cudaError_t gemm_bf16(const GemmArgs& a, const Dev& dev) {
   if (a.M <= 0) return cudaSuccess;
   if (a.epi.act == ACT_ROUTER) {
-    if (a.N != 64) return cudaErrorInvalidValue;
-    return launch<64, false, true>(a, dev);
+    if (a.N != 64 || a.K2 > 0) return cudaErrorInvalidValue;
+    return launch<64, false, true>(a, nullptr, dev);
   }
-  // Large M: 256-row tiles on CTA pairs when that still gives every pair of
-  // SMs at least two tiles (256 x 128 gate/up tiles for SwiGLU, 256 x 256
-  // otherwise).
+  // SwiGLU: 256 x 128 gate/up tiles on CTA pairs when that still gives every
+  // pair of SMs at least two tiles.
   if (a.epi.act == ACT_SWIGLU) {
+    if (a.K2 > 0) return cudaErrorInvalidValue;
     const int64_t pair_tiles = ((a.M + 255) / 256) * ((a.N + 127) / 128);
-    if (a.N % 128 == 0 && pair_tiles >= dev.num_sms) return launch_pair<128, true>(a, dev);
-    return launch<128, true, false>(a, dev);
+    if (a.N % 128 == 0 && pair_tiles >= dev.num_sms) return launch_pair<128, true>(a, nullptr, dev);
+    return launch<128, true, false>(a, nullptr, dev);
   }
-  const int64_t pair_tiles = ((a.M + 255) / 256) * ((a.N + 255) / 256);
-  if (a.N % 256 == 0 && pair_tiles >= dev.num_sms) return launch_pair<256, false>(a, dev);
-  // Pick the N tile that finishes in the fewest tile-time units: ceil(tiles /
-  // SMs) waves, a 128-wide tile costing 0.58 of a 256-wide one (it moves 2/3
-  // of the operand bytes for 1/2 of the flops).
-  const int64_t mblocks = (a.M + BM - 1) / BM;
-  const int64_t t256 = mblocks * ((a.N + 255) / 256);
-  const int64_t t128 = mblocks * ((a.N + 127) / 128);
-  const int64_t w256 = (t256 + dev.num_sms - 1) / dev.num_sms;
-  const int64_t w128 = (t128 + dev.num_sms - 1) / dev.num_sms;
-  if (a.N % 256 == 0 && 100 * w256 <= 58 * w128) return launch<256, false, false>(a, dev);
-  return launch<128, false, false>(a, dev);
+  return gemm_plain(a, dev);
+}
+
+cudaError_t gemm_bf16_grouped(const GemmArgs& a, const GemmArgs& b, const Dev& dev) {
+  if (a.M <= 0 && b.M <= 0) return cudaSuccess;
+  if (a.M <= 0) return gemm_bf16(b, dev);
+  if (b.M <= 0) return gemm_bf16(a, dev);
+  auto plain = [](const GemmArgs& g) {
+    return g.epi.act != ACT_ROUTER && g.epi.act != ACT_SWIGLU && g.K2 == 0;
+  };
+  if (!plain(a) || !plain(b)) return cudaErrorInvalidValue;
+  // CTA pairs when both problems have 256-wide N tiles and enough of them.
+  const int64_t pair_tiles = ((a.M + 255) / 256) * ((a.N + 255) / 256) +
+                             ((b.M + 255) / 256) * ((b.N + 255) / 256);
+  if (a.N % 256 == 0 && b.N % 256 == 0 && pair_tiles >= dev.num_sms)
+    return launch_pair<256, false>(a, &b, dev);
+  return launch<128, false, false>(a, &b, dev);
 }
 
 }  // namespace adadsf

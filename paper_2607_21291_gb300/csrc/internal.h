@@ -15,7 +15,7 @@ enum Act : int { ACT_NONE = 0, ACT_GELU = 1, ACT_SWIGLU = 2, ACT_ROUTER = 3 };
 
 // Epilogue of the projection kernels, applied to the fp32 accumulator
 // acc[m][n] of out = A[m,:] . W[n,:]:
-//   v = acc + bias[n]                         (bias may be null)
+//   v = acc + bias[n] + bias2[n]              (either may be null)
 //   v = gelu(v)                               (ACT_GELU)
 //   v = silu(acc) * acc2                      (ACT_SWIGLU, acc2 from the second weight)
 //   v += add_packed[m][n]                     (may be null)
@@ -25,6 +25,7 @@ enum Act : int { ACT_NONE = 0, ACT_GELU = 1, ACT_SWIGLU = 2, ACT_ROUTER = 3 };
 struct Epilogue {
   int act = ACT_NONE;
   const void* bias = nullptr;
+  const void* bias2 = nullptr;   // bf16 tensor-core path only
   const void* add_packed = nullptr;
   int64_t ld_add_packed = 0;
   const void* add_rows = nullptr;
@@ -51,13 +52,23 @@ struct Epilogue {
   int vt_seq = 1, vt_pad = 0, vt_col0 = 0, vt_hd = 0, vt_hkv = 0;
 };
 
+// acc = A . W^T (+ A2 . Wk2^T when K2 > 0: a second K source, bf16
+// tensor-core path only, K a multiple of 64).
 struct GemmArgs {
   const void* A = nullptr;  int64_t lda = 0;   // [M, K]
   const void* W = nullptr;  int64_t ldw = 0;   // [N, K]
   const void* W2 = nullptr;                    // [N, K] (ACT_SWIGLU: W = gate, W2 = up)
-  int64_t M = 0; int N = 0; int K = 0;
+  const void* A2 = nullptr;  int64_t lda2 = 0;    // [M, K2]
+  const void* Wk2 = nullptr; int64_t ldwk2 = 0;   // [N, K2]
+  int64_t M = 0; int N = 0; int K = 0; int K2 = 0;
   Epilogue epi;
+  // fp32 scratch for splitting small-M products along K (bf16 path); the
+  // split is used only when it fits (gemm_split_scratch_bytes covers every case)
+  float* scratch = nullptr;
+  size_t scratch_bytes = 0;
 };
+// Scratch that lets gemm_bf16 split any small-M product along K.
+size_t gemm_split_scratch_bytes();
 
 struct Dev {
   cudaStream_t stream;
@@ -72,6 +83,9 @@ bool make_tmap_bf16(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t col
 
 // gemm_tcgen05.cu -- bf16 tensor-core projections (tcgen05 + TMEM + TMA).
 cudaError_t gemm_bf16(const GemmArgs& a, const Dev& dev);
+// Two independent plain projections (no SwiGLU, router or second K source)
+// in one launch.
+cudaError_t gemm_bf16_grouped(const GemmArgs& a, const GemmArgs& b, const Dev& dev);
 // gemm_simt.cu -- fp32 projections on CUDA cores.
 cudaError_t gemm_f32(const GemmArgs& a, const Dev& dev);
 

@@ -8,6 +8,12 @@ Each case runs `--warmup` untimed calls, then `--iters` calls each bracketed by
 CUDA events on the launching stream (L2 flushed between calls by a 256 MiB
 write), and prints one JSON line with the mean time and the algorithmic
 TFLOP/s or GB/s. This is also the command the ncu captures run.
+
+`--graph R` also captures R back-to-back calls in one CUDA graph and reports the
+replay time divided by R ("graph_ms"): the per-call cost without host work
+(tensor-map encoding, launch calls), with consecutive launches overlapped by
+programmatic dependent launch as in the model forward. L2 is flushed before
+each replay, not between the R calls.
 """
 from __future__ import annotations
 
@@ -35,6 +41,27 @@ def _time(fn, iters, warmup, stream):
     return sum(e0.elapsed_time(e1) for e0, e1 in ev) / iters
 
 
+def _time_graph(fn, reps, iters, stream):
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    fn()                                    # first call outside capture (lazy set-up)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for _ in range(reps):
+            fn()
+    for _ in range(3):
+        g.replay()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(iters)]
+    torch.cuda.synchronize()
+    for e0, e1 in ev:
+        flush.zero_()
+        e0.record(stream)
+        g.replay()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    return sum(e0.elapsed_time(e1) for e0, e1 in ev) / (iters * reps)
+
+
 def _profile(fn, stream):
     """One call under the library's per-launch timing."""
     torch.cuda.synchronize()
@@ -50,7 +77,7 @@ def case_linear(a, stream):
     w = (0.02 * torch.randn(a.N, a.K, generator=g, device="cuda")).to(dt)
     b = (0.02 * torch.randn(a.N, generator=g, device="cuda")).to(dt)
     out = torch.empty(a.M, a.N, device="cuda", dtype=dt)
-    ws = A.workspace(256)
+    ws = A.workspace(A.LINEAR_SPLIT_WS_BYTES)
     fn = lambda: A.adadsf_linear(x, w, b, out, act=a.act, ws=ws, stream=stream)
     flops = 2.0 * a.M * a.N * a.K
     return fn, flops, (a.M * a.K + a.N * a.K + a.M * a.N) * x.element_size(), ws
@@ -94,9 +121,40 @@ def case_attention(a, stream):
     return fn, flops, (qkv.numel() + out.numel()) * qkv.element_size(), ws
 
 
+def case_router(a, stream):
+    wl = S.WORKLOADS[a.workload]
+    shape = wl.shape.replace(n_layers=1)
+    B = a.B or wl.B
+    T = a.T or wl.T
+    dt = torch.bfloat16 if shape.dtype == "bf16" else torch.float32
+    g = torch.Generator(device="cuda").manual_seed(0)
+    w = {n: (0.02 * torch.randn(shp, generator=g, device="cuda")).to(dt)
+         for n, shp in S.layer_weight_shapes(shape).items()}
+    x = torch.randn(B * T, shape.d, generator=g, device="cuda").to(dt)
+    scores = torch.empty(B * T, device="cuda", dtype=torch.float32)
+    cfg = A.make_cfg(shape)
+    ws = A.workspace(256)
+    fn = lambda: A.adadsf_router_scores(cfg, w, x, scores, ws=ws, stream=stream)
+    flops = 2.0 * B * T * shape.d * shape.router_hidden
+    return fn, flops, x.numel() * x.element_size(), ws
+
+
+def case_topk(a, stream):
+    wl = S.WORKLOADS[a.workload]
+    B = a.B or wl.B
+    T = a.T or wl.T
+    K = a.K if a.K is not None else T // 2
+    g = torch.Generator(device="cuda").manual_seed(0)
+    scores = torch.randn(B, T, generator=g, device="cuda")
+    idx = torch.empty(B, K, device="cuda", dtype=torch.int32)
+    rows = torch.empty(B, K, device="cuda", dtype=torch.int32)
+    fn = lambda: A.adadsf_topk_select(scores, K, idx, rows, stream=stream)
+    return fn, 0.0, scores.numel() * 4 + 2 * idx.numel() * 4, None
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
-    ap.add_argument("case", choices=("linear", "layer", "attention"))
+    ap.add_argument("case", choices=("linear", "layer", "attention", "router", "topk"))
     ap.add_argument("--M", type=int, default=8192)
     ap.add_argument("--N", type=int, default=8192)
     ap.add_argument("--K", type=int, default=None)
@@ -108,17 +166,26 @@ def main():
     ap.add_argument("--iters", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--profile", action="store_true", help="also report the library's per-launch events")
+    ap.add_argument("--graph", type=int, default=0, help="also time R calls replayed from one CUDA graph")
     a = ap.parse_args()
     if a.case == "linear" and a.K is None:
         a.K = 2048
     A.lib()
     stream = torch.cuda.Stream()
     with torch.cuda.stream(stream):
-        fn, flops, nbytes, ws = {"linear": case_linear, "layer": case_layer, "attention": case_attention}[a.case](a, stream)
+        fn, flops, nbytes, ws = {"linear": case_linear, "layer": case_layer, "attention": case_attention,
+                            "router": case_router, "topk": case_topk}[a.case](a, stream)
         ms = _time(fn, a.iters, a.warmup, stream)
-        out = {"case": a.case, "ms": ms, "tflops": flops / (ms * 1e9)}
+        out = {"case": a.case, "ms": ms}
+        if flops:
+            out["tflops"] = flops / (ms * 1e9)
         if nbytes:
             out["gbs"] = nbytes / (ms * 1e6)
+        if a.graph:
+            gms = _time_graph(fn, a.graph, a.iters, stream)
+            out["graph_ms"] = gms
+            if flops:
+                out["graph_tflops"] = flops / (gms * 1e9)
         if a.profile:
             out["launches"] = [(n, ms_, fl / max(ms_, 1e-9) / 1e9) for n, _, ms_, fl, _ in _profile(fn, stream)]
         if ws is not None:

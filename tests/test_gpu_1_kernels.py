@@ -83,25 +83,31 @@ def test_linear_bf16(A, M, N, Kd, act):
 
 
 @pytest.mark.parametrize("M,N,Kd,act", [(1, 64, 3072, 0), (300, 768, 3072, 1), (1384, 768, 3072, 0),
-                                        (128, 256, 2048, 0), (777, 2304, 768, 1), (1000, 384, 1024, 0)])
+                                        (128, 256, 2048, 0), (777, 2304, 768, 1), (1000, 384, 1024, 0),
+                                        (1024, 768, 768, 1), (1024, 768, 3072, 0), (333, 640, 960, 1),
+                                        (129, 128, 192, 0)])
 def test_linear_bf16_small_m(A, M, N, Kd, act):
-    """Small-M projections of the sparse layers: one wave of tiles, long K;
-    two launches in a row agree bit for bit."""
+    """Small-M projections of the sparse layers: one wave of tiles, long K
+    (with room for scratch most of these run split along K over clusters of 2
+    or 4 CTAs, with ragged M, N and K tails and uneven K ranges per CTA; with
+    the minimum workspace they do not); two launches in a row agree bit for
+    bit (the partial tiles are summed in a fixed order)."""
     g = np.random.default_rng(M * 7 + N + Kd)
     x = S.round_to(g.standard_normal((M, Kd)).astype(np.float32), "bf16")
     w = S.round_to((0.05 * g.standard_normal((N, Kd))).astype(np.float32), "bf16")
     b = S.round_to((0.1 * g.standard_normal(N)).astype(np.float32), "bf16")
-    ws = A.workspace(256)
     ref = O.linear(x, w, b, "gelu" if act else None)
-    outs = []
-    for _ in range(2):
-        out = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
-        A.adadsf_linear(H.to_dev(x, torch.bfloat16), H.to_dev(w, torch.bfloat16),
-                        H.to_dev(b, torch.bfloat16), out, act=act, ws=ws)
-        assert A.adadsf_sync_check(ws) == A.OK
-        assert H.max_rel(H.to_np(out), ref) < 8e-3
-        outs.append(out)
-    assert torch.equal(outs[0], outs[1])
+    for ws_bytes in (A.LINEAR_SPLIT_WS_BYTES, 256):
+        ws = A.workspace(ws_bytes)
+        outs = []
+        for _ in range(2):
+            out = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+            A.adadsf_linear(H.to_dev(x, torch.bfloat16), H.to_dev(w, torch.bfloat16),
+                            H.to_dev(b, torch.bfloat16), out, act=act, ws=ws)
+            assert A.adadsf_sync_check(ws) == A.OK
+            assert H.max_rel(H.to_np(out), ref) < 8e-3
+            outs.append(out)
+        assert torch.equal(outs[0], outs[1])
 
 
 @pytest.mark.parametrize("M,N,Kd", [(1, 4, 4), (65, 132, 68), (200, 2048, 512)])
@@ -116,7 +122,7 @@ def test_linear_f32(A, M, N, Kd):
 
 # ---------------------------------------------------------------- router (Sec. 3.4)
 @pytest.mark.parametrize("shape,n", [(S.PYTHIA_160M, 1), (S.PYTHIA_160M, 2048), (S.QWEN25_1_5B, 333),
-                                     (S.PYTHIA_70M, 128)])
+                                     (S.PYTHIA_70M, 128), (S.PYTHIA_160M, 777), (S.PYTHIA_1_4B, 16384)])
 def test_router(A, shape, n):
     W = H.host_layer(shape, 3)
     x = S.round_to(np.random.default_rng(n).standard_normal((n, shape.d)).astype(np.float32), shape.dtype)
