@@ -279,6 +279,7 @@ typedef enum {
   ADADSF_KERNEL_LINEAR, ADADSF_KERNEL_SELFTEST,
   ADADSF_KERNEL_GEMM_QKV_UP,   /* GPT-NeoX, bf16: QKV and MLP-up projections in one launch */
   ADADSF_KERNEL_GEMM_O_DOWN,   /* GPT-NeoX, bf16: output + MLP-down projections, one accumulator */
+  ADADSF_KERNEL_TOPK_GATHER_NORM, /* Top-K fused with the gather and norms of the kept rows */
   ADADSF_KERNEL_COUNT
 } adadsf_kernel_kind;
 

@@ -300,20 +300,38 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
                                  static_cast<const float*>(w->router_b2), lb.scores, dev),
                       "router")));
     }
-    TRY(launch(dev, ADADSF_KERNEL_TOPK, false, 0, BT * 4.0 + M * 8.0,
-               CALL(topk(lb.scores, B, T, K, lb.idx, lb.rows, dev), "top-k")));
+    if (M <= 32LL * dev.num_sms) {
+      // a3 + a4: Top-K of each sequence fused with the gather of the kept rows
+      // and their norms (NeoX: LN1 and LN2 of the same row). Every block
+      // repeats its sequence's selection: worth it while a launch less
+      // outweighs that (up to about one row per warp on four blocks per SM).
+      TRY(launch(dev, ADADSF_KERNEL_TOPK_GATHER_NORM, false, 0,
+                 BT * 4.0 + M * 8.0 + Md * es * (neox ? 3 : 2),
+                 CALL(select_gather_norm(dt, lb.scores, B, T, K, x, d, !neox, w->ln1_w, w->ln1_b,
+                                         w->ln2_w, w->ln2_b, c->norm_eps, lb.n1,
+                                         neox ? lb.n2 : nullptr, lb.idx, lb.rows, dev),
+                      "top-k + gather + norm")));
+    } else {
+      TRY(launch(dev, ADADSF_KERNEL_TOPK, false, 0, BT * 4.0 + M * 8.0,
+                 CALL(topk(lb.scores, B, T, K, lb.idx, lb.rows, dev), "top-k")));
+      // a4: gather the kept rows and normalise them (NeoX: LN1 and LN2)
+      TRY(launch(dev, ADADSF_KERNEL_GATHER_NORM, false, 0, Md * es * (neox ? 3 : 2),
+                 CALL(gather_norm(dt, x, lb.rows, M, d, !neox, w->ln1_w, w->ln1_b, w->ln2_w,
+                                  w->ln2_b, c->norm_eps, lb.n1, neox ? lb.n2 : nullptr, dev),
+                      "gather+norm")));
+    }
     rows = lb.rows;
     pos = lb.idx;
-  } else if (want_idx) {
-    TRY(launch(dev, ADADSF_KERNEL_POSITIONS, false, 0, M * 4.0,
-               CALL(iota_positions(lb.idx, B, K, dev), "positions")));
+  } else {
+    if (want_idx)
+      TRY(launch(dev, ADADSF_KERNEL_POSITIONS, false, 0, M * 4.0,
+                 CALL(iota_positions(lb.idx, B, K, dev), "positions")));
+    // a4: normalise every row (NeoX: LN1 and LN2 of the same row).
+    TRY(launch(dev, ADADSF_KERNEL_GATHER_NORM, false, 0, Md * es * (neox ? 3 : 2),
+               CALL(gather_norm(dt, x, nullptr, M, d, !neox, w->ln1_w, w->ln1_b, w->ln2_w,
+                                w->ln2_b, c->norm_eps, lb.n1, neox ? lb.n2 : nullptr, dev),
+                    "norm")));
   }
-
-  // a4: gather kept rows and normalise (NeoX: LN1 and LN2 of the same row).
-  TRY(launch(dev, ADADSF_KERNEL_GATHER_NORM, false, 0, Md * es * (neox ? 3 : 2),
-             CALL(gather_norm(dt, x, rows, M, d, !neox, w->ln1_w, w->ln1_b, w->ln2_w, w->ln2_b,
-                              c->norm_eps, lb.n1, neox ? lb.n2 : nullptr, dev),
-                  "gather+norm")));
   // a5: QKV projection (+bias), rotary at the original positions.
   // On the tensor-core path the rotation is fused into the QKV epilogue, and
   // for GPT-NeoX (parallel residual) the MLP up projection of the second
@@ -345,7 +363,8 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
       g.epi.vt_hkv = c->n_kv_heads;
     }
     if (neox_tc) {
-      // act = GELU(LN2 x W_up^T + b_up), grouped with the QKV tiles
+      // act = GELU(LN2 x W_up^T + b_up), grouped with the QKV tiles (first:
+      // its GELU epilogue is the costlier)
       GemmArgs u = linear_args(lb.n2, d, w->w_up, M, F, d);
       u.epi.bias = w->b_up;
       u.epi.act = ACT_GELU;
@@ -353,7 +372,7 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
       u.epi.ld_out = F;
       TRY(launch(dev, ADADSF_KERNEL_GEMM_QKV_UP, true, 2.0 * M * ((double)qkv_dim + F) * d,
                  (2.0 * Md + ((double)qkv_dim + F) * d + (double)M * (qkv_dim + F)) * es,
-                 CALL(gemm_bf16_grouped(g, u, dev), "qkv + mlp up projections")));
+                 CALL(gemm_bf16_grouped(u, g, dev), "qkv + mlp up projections")));
     } else {
       TRY(launch(dev, ADADSF_KERNEL_GEMM_QKV, tc, 2.0 * M * qkv_dim * d,
                  (Md + (double)qkv_dim * d + (double)M * qkv_dim) * es,
@@ -949,7 +968,7 @@ const char* adadsf_kernel_name(int kind) {
   static const char* names[ADADSF_KERNEL_COUNT] = {
       "embed", "router", "topk", "positions", "gather_norm", "gemm_qkv", "rope_table", "rope",
       "attention", "gemm_o", "norm2", "gemm_up", "gemm_down", "stats", "final_norm", "copy",
-      "linear", "selftest", "gemm_qkv_up", "gemm_o_down"};
+      "linear", "selftest", "gemm_qkv_up", "gemm_o_down", "topk_gather_norm"};
   return (kind >= 0 && kind < ADADSF_KERNEL_COUNT) ? names[kind] : "unknown";
 }
 

@@ -19,6 +19,8 @@
 //              (biases, the router's second layer) are staged in shared memory
 //              and the first residual chunks loaded into registers before the
 //              accumulator is ready, so their latency hides under the K loop.
+//              GELU uses an erf with one exponential and no division (the
+//              special-function unit bounds this epilogue).
 // Three kernels share this structure:
 //   gemm_tc_kernel     persistent, 128-row tiles; double-buffered TMEM so the
 //                      epilogue of tile i runs under the main loop of tile i+1.
@@ -148,20 +150,27 @@ __device__ __forceinline__ KbSrc kb_source(const TileInfo& ti, int kb, const CUt
   return s;
 }
 
-// erf by formula 7.1.26 of Abramowitz & Stegun, Handbook of Mathematical
-// Functions (|error| <= 1.5e-7): for x >= 0, erf(x) = 1 - t (a1 + t (a2 + t
-// (a3 + t (a4 + t a5)))) exp(-x^2) with t = 1 / (1 + p x); erf is odd.
-__device__ __forceinline__ float erf_as(float x) {
-  const float ax = fabsf(x);
-  const float t = __fdividef(1.f, fmaf(0.3275911f, ax, 1.f));
-  float y = fmaf(t, 1.061405429f, -1.453152027f);
-  y = fmaf(t, y, 1.421413741f);
-  y = fmaf(t, y, -0.284496736f);
-  y = fmaf(t, y, 0.254829592f);
-  y = 1.f - t * y * __expf(-ax * ax);
-  return copysignf(y, x);
+// erf(z) = 1 - exp(-z^2) R(z) for z >= 0 (erf is odd), R(z) = erfc(z) exp(z^2)
+// approximated on [0, 4] by a degree-10 polynomial in z / 4 (coefficients
+// and error bound from csrc/erf_poly.py: |error| <= 3.3e-7 in fp32); erf = 1
+// beyond z = 4 (to 1.6e-8). One exponential, no division.
+__device__ __forceinline__ float erf_fit(float x) {
+  const float z = fminf(fabsf(x), 4.f);
+  const float u = z * 0.25f;
+  float r = 1.019359436e+02f;
+  r = fmaf(r, u, -3.950886841e+02f);
+  r = fmaf(r, u, 6.843880615e+02f);
+  r = fmaf(r, u, -7.131018066e+02f);
+  r = fmaf(r, u, 5.127547607e+02f);
+  r = fmaf(r, u, -2.798540955e+02f);
+  r = fmaf(r, u, 1.249815445e+02f);
+  r = fmaf(r, u, -4.795371628e+01f);
+  r = fmaf(r, u, 1.599380779e+01f);
+  r = fmaf(r, u, -4.513438225e+00f);
+  r = fmaf(r, u, 9.999998212e-01f);
+  return copysignf(fmaf(-__expf(-z * z), r, 1.f), x);
 }
-__device__ __forceinline__ float gelu_f(float v) { return 0.5f * v * (1.f + erf_as(v * 0.70710678118654752f)); }
+__device__ __forceinline__ float gelu_f(float v) { return 0.5f * v * (1.f + erf_fit(v * 0.70710678118654752f)); }
 // v sigmoid(v); the exponent is capped so the fast division stays in range.
 __device__ __forceinline__ float silu_f(float v) {
   return v * __fdividef(1.f, 1.f + __expf(fminf(-v, 80.f)));
@@ -1405,11 +1414,17 @@ cudaError_t gemm_bf16_grouped(const GemmArgs& a, const GemmArgs& b, const Dev& d
     return g.epi.act != ACT_ROUTER && g.epi.act != ACT_SWIGLU && g.K2 == 0;
   };
   if (!plain(a) || !plain(b)) return cudaErrorInvalidValue;
-  // CTA pairs when both problems have 256-wide N tiles and enough of them.
-  const int64_t pair_tiles = ((a.M + 255) / 256) * ((a.N + 255) / 256) +
-                             ((b.M + 255) / 256) * ((b.N + 255) / 256);
-  if (a.N % 256 == 0 && b.N % 256 == 0 && pair_tiles >= dev.num_sms)
-    return launch_pair<256, false>(a, &b, dev);
+  // Fewest rounds of tiles (a k-block costs the same for any tile width);
+  // ties go to CTA pairs (half the weight bytes per SM), then to 256-wide
+  // tiles. Problem `a` comes first in the tile order: pass the one with the
+  // costlier epilogue as `a` so that it runs in the first round.
+  auto tiles = [](const GemmArgs& g, int bm, int bn) { return ((g.M + bm - 1) / bm) * ((g.N + bn - 1) / bn); };
+  const int64_t sms = dev.num_sms;
+  const int64_t r_pair = (tiles(a, 256, 256) + tiles(b, 256, 256) + sms / 2 - 1) / (sms / 2);
+  const int64_t r256 = (tiles(a, 128, 256) + tiles(b, 128, 256) + sms - 1) / sms;
+  const int64_t r128 = (tiles(a, 128, 128) + tiles(b, 128, 128) + sms - 1) / sms;
+  if (r_pair <= r256 && r_pair <= r128) return launch_pair<256, false>(a, &b, dev);
+  if (r256 <= r128) return launch<256, false, false>(a, &b, dev);
   return launch<128, false, false>(a, &b, dev);
 }
 

@@ -116,6 +116,12 @@ cudaError_t router_f32(const float* x, int64_t n, int d, int h, const float* w1,
                        const float* w2, const float* b2, float* scores, const Dev& dev);
 cudaError_t topk(const float* scores, int B, int T, int K, int32_t* idx, int32_t* rows,
                  const Dev& dev);
+// Top-K of each sequence's scores fused with gather_norm of the kept rows
+// (out rows b K + i, i-th kept position ascending); also writes idx / rows.
+cudaError_t select_gather_norm(int dtype, const float* scores, int B, int T, int K, const void* x,
+                               int d, bool is_rms, const void* g1, const void* b1, const void* g2,
+                               const void* b2, float eps, void* out1, void* out2, int32_t* idx,
+                               int32_t* rows, const Dev& dev);
 int stats_partials_count(int64_t n_rows);
 cudaError_t iota_positions(int32_t* idx, int B, int K, const Dev& dev);
 cudaError_t cos_stats(int dtype, const void* a, const void* b, int64_t n_rows, int d, int mode,

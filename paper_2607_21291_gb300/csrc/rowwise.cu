@@ -2,7 +2,9 @@
 // rotary embedding at original positions, fp32 router, per-sequence Top-K,
 // the Eq. 4 similarity reduction, and the bounded-wait self-test.
 // All are HBM-bound: rows are moved as 16-byte vectors, one warp per row.
+#include <algorithm>
 #include <mutex>
+#include <type_traits>
 
 #include "common.cuh"
 #include "internal.h"
@@ -34,79 +36,162 @@ __global__ void embed_kernel(const int32_t* ids, int64_t n, const T* table, int 
 }
 
 // ---------------------------------------------------------------- gather + norm
-// out1[m] = norm(x[row(m)]; g1, b1), out2[m] = norm(x[row(m)]; g2, b2).
-// LayerNorm: (x - mean) / sqrt(var + eps) * g + b (biased variance, two-pass
-// over the register-resident row); RMSNorm: x / sqrt(mean(x^2) + eps) * g.
-template <typename T, bool RMS>
-__global__ void gather_norm_kernel(const T* x, const int32_t* rows, int64_t M, int d, const T* g1,
-                                   const T* b1, const T* g2, const T* b2, float eps, T* out1,
-                                   T* out2) {
-  pdl_trigger();
-  pdl_wait();
+// Norm parameters (g1, b1, g2, b2; biases absent for RMSNorm, second pair
+// absent without out2) staged once per block in shared memory, so that the
+// per-row loop reads them without waiting behind its own global stores.
+template <typename T>
+__device__ __forceinline__ void stage_norm_params(const T* g1, const T* b1, const T* g2, const T* b2,
+                                                  int d, T* sp) {
   constexpr int V = Elem<T>::kVec;
-  const int64_t m = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
-  const int lane = threadIdx.x & 31;
-  if (m >= M) return;
-  const int64_t src = rows ? (int64_t)rows[m] : m;
   const int nv = d / V;
-  float v[kMaxChunks][V];
-  float s = 0.f;
+  const T* src[4] = {g1, b1, g2, b2};
+  for (int k = 0; k < 4; ++k) {
+    if (!src[k]) continue;
+    for (int i = threadIdx.x; i < nv; i += blockDim.x)
+      reinterpret_cast<uint4*>(sp + k * d)[i] = reinterpret_cast<const uint4*>(src[k])[i];
+  }
+  __syncthreads();
+}
+
+// o1 = norm(xr; g1, b1), o2 = norm(xr; g2, b2) for R rows at once (their
+// loads overlap), by one warp; row r is skipped when xr[r] is null. NCH: the
+// 16-byte vectors per lane a row needs, ceil(d / (32 V)), fixed at compile
+// time so that no dead chunk is issued. sp holds the staged parameters
+// ([4][d]: g1, b1, g2, b2). LayerNorm: (x - mean) / sqrt(var + eps) * g + b
+// (biased variance, two-pass over the register-resident row); RMSNorm:
+// x / sqrt(mean(x^2) + eps) * g.
+template <typename T, bool RMS, int NCH, int R>
+__device__ __forceinline__ void norm_rows(const T* const (&xr)[R], int d, const T* sp, float eps,
+                                          T* const (&o1)[R], T* const (&o2)[R], int lane) {
+  constexpr int V = Elem<T>::kVec;
+  const int nv = d / V;
+  float v[R][NCH][V];
+  float s[R], mean[R], rstd[R];
 #pragma unroll
-  for (int c = 0; c < kMaxChunks; ++c) {
-    const int ci = c * 32 + lane;
-    if (ci < nv) {
-      load_vec(x + src * d + ci * V, v[c]);
+  for (int r = 0; r < R; ++r) {
+    s[r] = 0.f;
+    if (!xr[r]) continue;
 #pragma unroll
-      for (int j = 0; j < V; ++j) s += v[c][j];
+    for (int c = 0; c < NCH; ++c) {
+      const int ci = c * 32 + lane;
+      if (ci < nv) load_vec(xr[r] + ci * V, v[r][c]);
     }
   }
-  float mean = 0.f, rstd;
-  if (!RMS) {
-    mean = warp_sum(s) / d;
-    float q = 0.f;
 #pragma unroll
-    for (int c = 0; c < kMaxChunks; ++c) {
+  for (int r = 0; r < R; ++r) {
+#pragma unroll
+    for (int c = 0; c < NCH; ++c) {
       const int ci = c * 32 + lane;
-      if (ci < nv) {
+      if (xr[r] && ci < nv) {
 #pragma unroll
-        for (int j = 0; j < V; ++j) {
-          const float t = v[c][j] - mean;
-          q += t * t;
+        for (int j = 0; j < V; ++j) s[r] += RMS ? v[r][c][j] * v[r][c][j] : v[r][c][j];
+      }
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    if (RMS) {
+      mean[r] = 0.f;
+      rstd[r] = 1.f / sqrtf(warp_sum(s[r]) / d + eps);
+    } else {
+      mean[r] = warp_sum(s[r]) / d;
+    }
+  }
+  if (!RMS) {
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+      float q = 0.f;
+#pragma unroll
+      for (int c = 0; c < NCH; ++c) {
+        const int ci = c * 32 + lane;
+        if (xr[r] && ci < nv) {
+#pragma unroll
+          for (int j = 0; j < V; ++j) {
+            const float t = v[r][c][j] - mean[r];
+            q += t * t;
+          }
+        }
+      }
+      rstd[r] = 1.f / sqrtf(warp_sum(q) / d + eps);
+    }
+  }
+#pragma unroll
+  for (int c = 0; c < NCH; ++c) {
+    const int ci = c * 32 + lane;
+    if (ci < nv) {
+      float g[V], bb[V], o[V];
+      load_vec(sp + ci * V, g);
+      if (!RMS) load_vec(sp + d + ci * V, bb);
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        if (!xr[r]) continue;
+#pragma unroll
+        for (int j = 0; j < V; ++j)
+          o[j] = (v[r][c][j] - mean[r]) * rstd[r] * g[j] + (RMS ? 0.f : bb[j]);
+        store_vec(o1[r] + ci * V, o);
+      }
+      if (o2[0]) {
+        load_vec(sp + 2 * d + ci * V, g);
+        if (!RMS) load_vec(sp + 3 * d + ci * V, bb);
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+          if (!xr[r]) continue;
+#pragma unroll
+          for (int j = 0; j < V; ++j)
+            o[j] = (v[r][c][j] - mean[r]) * rstd[r] * g[j] + (RMS ? 0.f : bb[j]);
+          store_vec(o2[r] + ci * V, o);
         }
       }
     }
-    rstd = 1.f / sqrtf(warp_sum(q) / d + eps);
-  } else {
-    float q = 0.f;
-#pragma unroll
-    for (int c = 0; c < kMaxChunks; ++c) {
-      const int ci = c * 32 + lane;
-      if (ci < nv) {
-#pragma unroll
-        for (int j = 0; j < V; ++j) q += v[c][j] * v[c][j];
-      }
-    }
-    rstd = 1.f / sqrtf(warp_sum(q) / d + eps);
   }
+}
+
+// Rows per step of one warp: two while a row needs at most 8 vectors per lane.
+template <int NCH>
+constexpr int rows_per_step() { return NCH <= 8 ? 2 : 1; }
+
+// Rows [lo, hi) of the block's share, warp w taking w, w + nw, ... in steps
+// of R rows; src(i) / dst(i) give the source row and the output row.
+template <typename T, bool RMS, int NCH, typename Src, typename Dst>
+__device__ __forceinline__ void norm_share(int64_t lo, int64_t hi, const T* x, int d, const T* sp,
+                                           float eps, T* out1, T* out2, Src src, Dst dst) {
+  constexpr int R = rows_per_step<NCH>();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  for (int64_t i = lo + warp; i < hi; i += (int64_t)R * nw) {
+    const T* xr[R];
+    T* o1[R];
+    T* o2[R];
 #pragma unroll
-  for (int c = 0; c < kMaxChunks; ++c) {
-    const int ci = c * 32 + lane;
-    if (ci < nv) {
-      float g[V], b[V], o[V];
-      load_vec(g1 + ci * V, g);
-      if (!RMS) load_vec(b1 + ci * V, b);
-#pragma unroll
-      for (int j = 0; j < V; ++j) o[j] = (v[c][j] - mean) * rstd * g[j] + (RMS ? 0.f : b[j]);
-      store_vec(out1 + m * d + ci * V, o);
-      if (out2) {
-        load_vec(g2 + ci * V, g);
-        if (!RMS) load_vec(b2 + ci * V, b);
-#pragma unroll
-        for (int j = 0; j < V; ++j) o[j] = (v[c][j] - mean) * rstd * g[j] + (RMS ? 0.f : b[j]);
-        store_vec(out2 + m * d + ci * V, o);
-      }
+    for (int r = 0; r < R; ++r) {
+      const int64_t ii = i + (int64_t)r * nw;
+      const bool ok = ii < hi;
+      const int64_t m = ok ? dst(ii) : 0;
+      xr[r] = ok ? x + src(ii) * d : nullptr;
+      o1[r] = out1 + m * d;
+      o2[r] = out2 ? out2 + m * d : nullptr;
     }
+    norm_rows<T, RMS, NCH, R>(xr, d, sp, eps, o1, o2, lane);
   }
+}
+
+constexpr int kNormThreads = 256;
+constexpr int kNormRowsPerBlock = 32;   // four rows per warp
+
+// out1[m] = norm(x[row(m)]; g1, b1), out2[m] = norm(x[row(m)]; g2, b2), one warp per row.
+template <typename T, bool RMS, int NCH>
+__global__ void __launch_bounds__(kNormThreads)
+    gather_norm_kernel(const T* x, const int32_t* rows, int64_t M, int d, const T* g1, const T* b1,
+                       const T* g2, const T* b2, float eps, T* out1, T* out2) {
+  pdl_trigger();
+  extern __shared__ __align__(16) uint8_t smem_norm[];
+  T* sp = reinterpret_cast<T*>(smem_norm);
+  stage_norm_params(g1, RMS ? nullptr : b1, out2 ? g2 : nullptr, (RMS || !out2) ? nullptr : b2, d,
+                    sp);   // weights: independent of the previous kernel
+  pdl_wait();
+  const int64_t m0 = (int64_t)blockIdx.x * kNormRowsPerBlock;
+  norm_share<T, RMS, NCH>(
+      m0, min(M, m0 + kNormRowsPerBlock), x, d, sp, eps, out1, out2,
+      [&](int64_t m) { return rows ? (int64_t)rows[m] : m; }, [](int64_t m) { return m; });
 }
 
 // ---------------------------------------------------------------- rotary embedding
@@ -188,9 +273,11 @@ __device__ __forceinline__ uint32_t score_key(float f) {
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-// Exclusive prefix sum over the block (blockDim.x == 1024) of one int per
-// thread; also returns the block total.
+// Exclusive prefix sum over a block of NT threads of one int per thread;
+// also returns the block total. warp_tot: NT / 32 + 1 ints of shared memory.
+template <int NT>
 __device__ __forceinline__ int block_excl_scan(int v, int* warp_tot, int& total) {
+  constexpr int NW = NT / 32;
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   int incl = v;
 #pragma unroll
@@ -201,51 +288,46 @@ __device__ __forceinline__ int block_excl_scan(int v, int* warp_tot, int& total)
   if (lane == 31) warp_tot[w] = incl;
   __syncthreads();
   if (w == 0) {
-    int t = warp_tot[lane];
+    int t = lane < NW ? warp_tot[lane] : 0;
     int ti = t;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const int u = __shfl_up_sync(0xffffffffu, ti, o);
       if (lane >= o) ti += u;
     }
-    warp_tot[lane] = ti - t;        // exclusive prefix of warp totals
-    if (lane == 31) warp_tot[32] = ti;
+    if (lane < NW) warp_tot[lane] = ti - t;   // exclusive prefix of warp totals
+    if (lane == 31) warp_tot[NW] = ti;
   }
   __syncthreads();
   const int res = warp_tot[w] + incl - v;
-  total = warp_tot[32];
+  total = warp_tot[NW];
   __syncthreads();
   return res;
 }
 
-constexpr int kTopkThreads = 1024;
+// Shared state of the block-wide Top-K.
+struct TopkShared {
+  int hist[256];
+  int warp_tot[33];
+  uint32_t digit;
+  int remaining;
+};
 
-// One block per sequence. Radix select (4 passes of 8 bits, most significant
-// first) finds the K-th largest key kth and how many keys equal to it are
-// kept (need_eq, lowest positions first); two block scans then emit the kept
-// positions in ascending order.
-__global__ void __launch_bounds__(kTopkThreads) topk_kernel(const float* scores, int T, int K,
-                                                            int32_t* idx, int32_t* rows) {
-  pdl_trigger();
-  pdl_wait();
-  extern __shared__ uint32_t keys[];
-  __shared__ int hist[256];
-  __shared__ int warp_tot[33];
-  __shared__ uint32_t s_digit;
-  __shared__ int s_remaining;
-  const int b = blockIdx.x;
-  const float* sc = scores + (int64_t)b * T;
-  for (int t = threadIdx.x; t < T; t += kTopkThreads) keys[t] = score_key(sc[t]);
-
+// Radix select over the T order-preserving keys in shared memory (4 passes
+// of 8 bits, most significant first): the K-th largest key `kth` and how many
+// keys equal to it are kept (need_eq, lowest positions first). K >= 1.
+template <int NT>
+__device__ __forceinline__ void radix_select(const uint32_t* keys, int T, int K, TopkShared& sh,
+                                             uint32_t& kth, int& need_eq) {
   uint32_t prefix = 0, pmask = 0;
   int remaining = K;   // keys still to take at or below the current prefix
   for (int pass = 0; pass < 4; ++pass) {
     const int shift = 24 - 8 * pass;
-    if (threadIdx.x < 256) hist[threadIdx.x] = 0;
+    for (int i = threadIdx.x; i < 256; i += NT) sh.hist[i] = 0;
     __syncthreads();
-    for (int t = threadIdx.x; t < T; t += kTopkThreads) {
+    for (int t = threadIdx.x; t < T; t += NT) {
       const uint32_t k = keys[t];
-      if ((k & pmask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1);
+      if ((k & pmask) == prefix) atomicAdd(&sh.hist[(k >> shift) & 255u], 1);
     }
     __syncthreads();
     if (threadIdx.x < 32) {
@@ -254,7 +336,7 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const float* scores,
       int cnt[8], lsum = 0;
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
-        cnt[j] = hist[255 - 8 * lane - j];
+        cnt[j] = sh.hist[255 - 8 * lane - j];
         lsum += cnt[j];
       }
       int incl = lsum;
@@ -270,8 +352,8 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const float* scores,
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
           if (above + cnt[j] >= remaining) {
-            s_digit = (uint32_t)(255 - 8 * lane - j);
-            s_remaining = remaining - above;
+            sh.digit = (uint32_t)(255 - 8 * lane - j);
+            sh.remaining = remaining - above;
             break;
           }
           above += cnt[j];
@@ -279,21 +361,27 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const float* scores,
       }
     }
     __syncthreads();
-    prefix |= s_digit << shift;
+    prefix |= sh.digit << shift;
     pmask |= 255u << shift;
-    remaining = s_remaining;
+    remaining = sh.remaining;
     __syncthreads();
   }
-  const uint32_t kth = prefix;
-  const int need_eq = remaining;
+  kth = prefix;
+  need_eq = remaining;
+}
 
-  // Contiguous chunk of positions per thread keeps the output ascending.
-  const int chunk = (T + kTopkThreads - 1) / kTopkThreads;
-  const int t0 = min(T, threadIdx.x * chunk), t1 = min(T, t0 + chunk);
+// Calls emit(i, t) for the kept positions t in ascending order, i = 0..K-1:
+// keys above kth, and the first need_eq keys equal to it. Contiguous chunks
+// of positions per thread and two block scans keep the output ascending.
+template <int NT, typename Emit>
+__device__ __forceinline__ void emit_kept(const uint32_t* keys, int T, uint32_t kth, int need_eq,
+                                          TopkShared& sh, Emit emit) {
+  const int chunk = (T + NT - 1) / NT;
+  const int t0 = min(T, (int)threadIdx.x * chunk), t1 = min(T, t0 + chunk);
   int n_eq = 0;
   for (int t = t0; t < t1; ++t) n_eq += keys[t] == kth;
   int total;
-  const int eq_base = block_excl_scan(n_eq, warp_tot, total);   // equal keys before my chunk
+  const int eq_base = block_excl_scan<NT>(n_eq, sh.warp_tot, total);   // equal keys before my chunk
   int n_sel = 0, er = eq_base;
   for (int t = t0; t < t1; ++t) {
     const uint32_t k = keys[t];
@@ -304,7 +392,7 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const float* scores,
       ++er;
     }
   }
-  int out = block_excl_scan(n_sel, warp_tot, total);
+  int out = block_excl_scan<NT>(n_sel, sh.warp_tot, total);
   er = eq_base;
   for (int t = t0; t < t1; ++t) {
     const uint32_t k = keys[t];
@@ -313,12 +401,68 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const float* scores,
       take = er < need_eq;
       ++er;
     }
-    if (take) {
-      idx[(int64_t)b * K + out] = t;
-      if (rows) rows[(int64_t)b * K + out] = b * T + t;
-      ++out;
-    }
+    if (take) emit(out++, t);
   }
+}
+
+constexpr int kTopkThreads = 1024;
+constexpr int kMaxTopkT = 16384;   // sequence length limit of the Top-K kernels
+
+// One block per sequence: idx[b][i] = i-th kept position (ascending), rows[b][i] = b T + position.
+__global__ void __launch_bounds__(kTopkThreads) topk_kernel(const float* scores, int T, int K,
+                                                            int32_t* idx, int32_t* rows) {
+  pdl_trigger();
+  pdl_wait();
+  extern __shared__ uint32_t keys[];
+  __shared__ TopkShared sh;
+  const int b = blockIdx.x;
+  const float* sc = scores + (int64_t)b * T;
+  for (int t = threadIdx.x; t < T; t += kTopkThreads) keys[t] = score_key(sc[t]);
+  uint32_t kth;
+  int need_eq;
+  radix_select<kTopkThreads>(keys, T, K, sh, kth, need_eq);
+  emit_kept<kTopkThreads>(keys, T, kth, need_eq, sh, [&](int i, int t) {
+    idx[(int64_t)b * K + i] = t;
+    if (rows) rows[(int64_t)b * K + i] = b * T + t;
+  });
+}
+
+constexpr int kSelThreads = 256;
+
+// Top-K of sequence b fused with the gather and norm of its kept rows: every
+// block of the sequence selects the same kept set (deterministic) into shared
+// memory, then normalises its share [g K / G, (g+1) K / G) of the packed rows
+// (one warp per row) and writes that share of idx / rows.
+template <typename T, bool RMS, int NCH>
+__global__ void __launch_bounds__(kSelThreads)
+    select_gather_norm_kernel(const float* scores, int Tlen, int K, const T* x, int d, const T* g1,
+                              const T* b1, const T* g2, const T* b2, float eps, T* out1, T* out2,
+                              int32_t* idx, int32_t* rows) {
+  pdl_trigger();
+  extern __shared__ __align__(16) uint32_t smem_sel[];
+  T* sp = reinterpret_cast<T*>(smem_sel);                               // [4][d] norm parameters
+  uint32_t* keys = smem_sel + (4 * d * sizeof(T)) / 4;                  // [Tlen]
+  int32_t* kept = reinterpret_cast<int32_t*>(keys + Tlen);              // [K]
+  __shared__ TopkShared sh;
+  stage_norm_params(g1, RMS ? nullptr : b1, out2 ? g2 : nullptr, (RMS || !out2) ? nullptr : b2, d,
+                    sp);   // weights: independent of the previous kernel
+  pdl_wait();
+  const int b = blockIdx.y, g = blockIdx.x, G = gridDim.x;
+  const float* sc = scores + (int64_t)b * Tlen;
+  for (int t = threadIdx.x; t < Tlen; t += kSelThreads) keys[t] = score_key(sc[t]);
+  uint32_t kth;
+  int need_eq;
+  radix_select<kSelThreads>(keys, Tlen, K, sh, kth, need_eq);
+  emit_kept<kSelThreads>(keys, Tlen, kth, need_eq, sh, [&](int i, int t) { kept[i] = t; });
+  __syncthreads();
+  const int lo = (int)((int64_t)g * K / G), hi = (int)((int64_t)(g + 1) * K / G);
+  for (int i = lo + (int)threadIdx.x; i < hi; i += kSelThreads) {
+    idx[(int64_t)b * K + i] = kept[i];
+    rows[(int64_t)b * K + i] = b * Tlen + kept[i];
+  }
+  norm_share<T, RMS, NCH>(
+      lo, hi, x, d, sp, eps, out1, out2, [&](int64_t i) { return (int64_t)b * Tlen + kept[i]; },
+      [&](int64_t i) { return (int64_t)b * K + i; });
 }
 
 // ---------------------------------------------------------------- Eq. 4 statistics
@@ -443,23 +587,67 @@ cudaError_t embed(int dtype, const int32_t* ids, int64_t n, const void* table, i
                     static_cast<const float*>(table), vocab, d, static_cast<float*>(out), dev.err);
 }
 
+// Chunk-count bucket (vectors per lane) of a row of d elements.
+template <typename T>
+int nch_bucket(int d) {
+  const int n = (d / Elem<T>::kVec + 31) / 32;
+  if (n <= 2) return 2;
+  if (n <= 4) return n;
+  if (n <= 6) return 6;
+  if (n <= 8) return 8;
+  if (n <= 12) return 12;
+  if (n <= 14) return 14;
+  return 16;
+}
+
+// Calls f(std::integral_constant<int, NCH>) for the bucket of d.
+template <typename T, typename F>
+cudaError_t with_nch(int d, F f) {
+  switch (nch_bucket<T>(d)) {
+    case 2: return f(std::integral_constant<int, 2>());
+    case 3: return f(std::integral_constant<int, 3>());
+    case 4: return f(std::integral_constant<int, 4>());
+    case 6: return f(std::integral_constant<int, 6>());
+    case 8: return f(std::integral_constant<int, 8>());
+    case 12: return f(std::integral_constant<int, 12>());
+    case 14: return f(std::integral_constant<int, 14>());
+    default: return f(std::integral_constant<int, 16>());
+  }
+}
+
+template <typename T, bool RMS>
+cudaError_t gather_norm_t(const void* x, const int32_t* rows, int64_t M, int d, const void* g1,
+                          const void* b1, const void* g2, const void* b2, float eps, void* out1,
+                          void* out2, const Dev& dev) {
+  const unsigned grid = (unsigned)((M + kNormRowsPerBlock - 1) / kNormRowsPerBlock);
+  const size_t smem = 4 * (size_t)d * sizeof(T);
+  return with_nch<T>(d, [&](auto nch) -> cudaError_t {
+    constexpr int NCH = decltype(nch)::value;
+    static int attr_done[64] = {0};
+    int device = 0;
+    cudaGetDevice(&device);
+    if (device < 64 && !attr_done[device]) {
+      cudaError_t e = cudaFuncSetAttribute(gather_norm_kernel<T, RMS, NCH>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, 4 * 4096 * 4);
+      if (e != cudaSuccess) return e;
+      attr_done[device] = 1;
+    }
+    return launch_pdl(gather_norm_kernel<T, RMS, NCH>, dim3(grid), dim3(kNormThreads), smem,
+                      dev.stream, static_cast<const T*>(x), rows, M, d, static_cast<const T*>(g1),
+                      static_cast<const T*>(b1), static_cast<const T*>(g2),
+                      static_cast<const T*>(b2), eps, static_cast<T*>(out1), static_cast<T*>(out2));
+  });
+}
+
 cudaError_t gather_norm(int dtype, const void* x, const int32_t* rows, int64_t M, int d,
                         bool is_rms, const void* g1, const void* b1, const void* g2,
                         const void* b2, float eps, void* out1, void* out2, const Dev& dev) {
   if (M <= 0) return cudaSuccess;
-  const unsigned grid = blocks_for(M, 8);
-#define GN_LAUNCH(T, R)                                                                         \
-  return launch_pdl(gather_norm_kernel<T, R>, dim3(grid), dim3(256), 0, dev.stream,             \
-                    static_cast<const T*>(x), rows, M, d, static_cast<const T*>(g1),            \
-                    static_cast<const T*>(b1), static_cast<const T*>(g2),                       \
-                    static_cast<const T*>(b2), eps, static_cast<T*>(out1), static_cast<T*>(out2))
-  if (dtype == kBF16) {
-    if (is_rms) GN_LAUNCH(bf16, true);
-    GN_LAUNCH(bf16, false);
-  }
-  if (is_rms) GN_LAUNCH(float, true);
-  GN_LAUNCH(float, false);
-#undef GN_LAUNCH
+  if (dtype == kBF16)
+    return is_rms ? gather_norm_t<bf16, true>(x, rows, M, d, g1, b1, g2, b2, eps, out1, out2, dev)
+                  : gather_norm_t<bf16, false>(x, rows, M, d, g1, b1, g2, b2, eps, out1, out2, dev);
+  return is_rms ? gather_norm_t<float, true>(x, rows, M, d, g1, b1, g2, b2, eps, out1, out2, dev)
+                : gather_norm_t<float, false>(x, rows, M, d, g1, b1, g2, b2, eps, out1, out2, dev);
 }
 
 cudaError_t rope_table(float2* tab, int T, int rotary_dim, float theta, const Dev& dev) {
@@ -504,12 +692,62 @@ cudaError_t topk(const float* scores, int B, int T, int K, int32_t* idx, int32_t
   cudaGetDevice(&device);
   if (device < 64 && !attr_done[device]) {
     cudaError_t e = cudaFuncSetAttribute(topk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         16384 * (int)sizeof(uint32_t));
+                                         kMaxTopkT * (int)sizeof(uint32_t));
     if (e != cudaSuccess) return e;
     attr_done[device] = 1;
   }
   return launch_pdl(topk_kernel, dim3(B), dim3(kTopkThreads), smem, dev.stream, scores, T, K, idx,
                     rows);
+}
+
+constexpr int kSelSmemMax = 2 * kMaxTopkT * 4 + 4 * 4096 * 4;   // keys, kept, fp32 params (d <= 4096)
+
+template <typename T, bool RMS>
+cudaError_t select_gather_norm_t(const float* scores, int B, int seq_len, int K, const void* x, int d,
+                                 const void* g1, const void* b1, const void* g2, const void* b2,
+                                 float eps, void* out1, void* out2, int32_t* idx, int32_t* rows,
+                                 const Dev& dev) {
+  const size_t smem = 4 * (size_t)d * sizeof(T) + (size_t)(seq_len + K) * 4;
+  // Blocks per sequence: one row per warp when that keeps the grid within
+  // about four blocks per SM (every block repeats the selection, so with
+  // more rows each block takes several per warp).
+  const int64_t per_block = std::max<int64_t>(kSelThreads / 32,
+                                              ((int64_t)B * K + 4 * dev.num_sms - 1) / (4 * dev.num_sms));
+  const int G = (int)std::max<int64_t>(1, (K + per_block - 1) / per_block);
+  return with_nch<T>(d, [&](auto nch) -> cudaError_t {
+    constexpr int NCH = decltype(nch)::value;
+    static int attr_done[64] = {0};
+    int device = 0;
+    cudaGetDevice(&device);
+    if (device < 64 && !attr_done[device]) {
+      cudaError_t e = cudaFuncSetAttribute(select_gather_norm_kernel<T, RMS, NCH>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, kSelSmemMax);
+      if (e != cudaSuccess) return e;
+      attr_done[device] = 1;
+    }
+    return launch_pdl(select_gather_norm_kernel<T, RMS, NCH>, dim3(G, B), dim3(kSelThreads), smem,
+                      dev.stream, scores, seq_len, K, static_cast<const T*>(x), d,
+                      static_cast<const T*>(g1), static_cast<const T*>(b1),
+                      static_cast<const T*>(g2), static_cast<const T*>(b2), eps,
+                      static_cast<T*>(out1), static_cast<T*>(out2), idx, rows);
+  });
+}
+
+cudaError_t select_gather_norm(int dtype, const float* scores, int B, int T, int K, const void* x,
+                               int d, bool is_rms, const void* g1, const void* b1, const void* g2,
+                               const void* b2, float eps, void* out1, void* out2, int32_t* idx,
+                               int32_t* rows, const Dev& dev) {
+  if (B <= 0 || K <= 0) return cudaSuccess;
+  if (T > kMaxTopkT) return cudaErrorInvalidValue;
+  if (dtype == kBF16)
+    return is_rms ? select_gather_norm_t<bf16, true>(scores, B, T, K, x, d, g1, b1, g2, b2, eps,
+                                                     out1, out2, idx, rows, dev)
+                  : select_gather_norm_t<bf16, false>(scores, B, T, K, x, d, g1, b1, g2, b2, eps,
+                                                      out1, out2, idx, rows, dev);
+  return is_rms ? select_gather_norm_t<float, true>(scores, B, T, K, x, d, g1, b1, g2, b2, eps,
+                                                    out1, out2, idx, rows, dev)
+                : select_gather_norm_t<float, false>(scores, B, T, K, x, d, g1, b1, g2, b2, eps,
+                                                     out1, out2, idx, rows, dev);
 }
 
 // Fixed block count for a given row count (independent of the device), so the
