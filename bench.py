@@ -120,10 +120,17 @@ def gpu_id_for_smi(dev_index: int) -> str:
         return str(dev_index)
 
 
-def kernel_source_hash() -> str:
+# Sources that decide a kernel family's launches (tile choice, fusion) and code.
+KIND_SOURCES = {
+    "gemm": ("gemm_tcgen05.cu", "common.cuh", "internal.h", "api.cu"),
+}
+
+
+def kernel_source_hash(kind: str = "") -> str:
     h = hashlib.sha1()
     csrc = os.path.join(ROOT, "paper_2607_21291_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
+    files = KIND_SOURCES.get(kind) or sorted(os.listdir(csrc))
+    for f in files:
         with open(os.path.join(csrc, f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:12]
@@ -135,7 +142,7 @@ def recorded_traffic(kind: str, workload: str):
     pdir = os.path.join(ROOT, "profiles")
     if not os.path.isdir(pdir):
         return None
-    want = kernel_source_hash()
+    want = kernel_source_hash(kind)
     for f in sorted(os.listdir(pdir)):
         if not f.endswith((".md", ".txt")):
             continue
