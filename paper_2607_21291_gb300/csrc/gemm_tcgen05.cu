@@ -40,6 +40,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cstdlib>
 #include <mutex>
 
@@ -82,6 +83,7 @@ struct TileCfg {
 
 struct GemmDev {
   int M, N, K;               // K: both sources together
+  int bn;                    // tile width (N) of this problem's tiles
   int kb_split;              // k-blocks read through (tmA, tmB); the rest through (tmA2, tmB2)
   int act;
   const bf16* bias;
@@ -113,21 +115,22 @@ __device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int& mb
   nb = r / gsz;
 }
 
-__device__ __forceinline__ int tiles_of(const GemmDev& p, int bm, int bn) {
-  return p.M > 0 ? ((p.M + bm - 1) / bm) * ((p.N + bn - 1) / bn) : 0;
+__device__ __forceinline__ int tiles_of(const GemmDev& p, int bm) {
+  return p.M > 0 ? ((p.M + bm - 1) / bm) * ((p.N + p.bn - 1) / p.bn) : 0;
 }
 
 // Tile t of a (possibly grouped) launch: problem, block coordinates, k-blocks.
 struct TileInfo {
-  int prob, mb, nb, nkb, kb_split;
+  int prob, mb, nb, nkb, kb_split, bn;
 };
 __device__ __forceinline__ TileInfo tile_info(int t, const GemmDev& p, const GemmDev& p2,
-                                              int tiles0, int bm, int bn) {
+                                              int tiles0, int bm) {
   TileInfo ti;
   ti.prob = t < tiles0 ? 0 : 1;
   const GemmDev& P = ti.prob ? p2 : p;
   const int tt = ti.prob ? t - tiles0 : t;
-  tile_coords(tt, (P.M + bm - 1) / bm, (P.N + bn - 1) / bn, ti.mb, ti.nb);
+  ti.bn = P.bn;
+  tile_coords(tt, (P.M + bm - 1) / bm, (P.N + P.bn - 1) / P.bn, ti.mb, ti.nb);
   ti.nkb = (P.K + BK - 1) / BK;
   ti.kb_split = ti.prob ? 0 : P.kb_split;   // the second problem reads through (tmA2, tmB2)
   return ti;
@@ -192,10 +195,9 @@ __device__ __forceinline__ void ld_shared_f4(uint32_t addr, float* f) {
 // shared-memory slot (no cross-warp barrier): sc[j] = bias[n] + bias2[n] for
 // the tile's columns n = nb BN + j; the router stages sc[j] = bias[j] and
 // sc[64 + j] = w2[j]. Each lane moves 16 bytes at a time.
-template <int BN, bool ROUTER>
-__device__ __forceinline__ void stage_consts(const GemmDev& p, int nb, uint32_t sc, int lane) {
-  if (ROUTER) {
-    static_assert(!ROUTER || BN == 64, "router tile");
+template <bool ROUTER>
+__device__ __forceinline__ void stage_consts(const GemmDev& p, int nb, int bn, uint32_t sc, int lane) {
+  if (ROUTER) {   // bn == 64
     if (lane < 16) {
       const bf16* src = lane < 8 ? p.bias : p.w2;
       const int j = 8 * (lane & 7);
@@ -205,8 +207,8 @@ __device__ __forceinline__ void stage_consts(const GemmDev& p, int nb, uint32_t 
       st_shared_f4(sc + 4u * (8 * lane + 4), f + 4);
     }
   } else {
-    for (int j8 = lane; j8 < BN / 8; j8 += 32) {
-      const int n = nb * BN + 8 * j8;
+    for (int j8 = lane; j8 < bn / 8; j8 += 32) {
+      const int n = nb * bn + 8 * j8;
       float f[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
       if (n < p.N) {
         if (p.bias) load_vec(p.bias + n, f);
@@ -345,7 +347,7 @@ struct EpiPre {
 // `red` the split-K partial to add first. ROPE: the instance for rotary
 // tiles (query / key / value projections, which have no residual).
 template <int BN, bool DUAL, bool ROUTER, bool ROPE>
-__device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, int m, int nb,
+__device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, int m, int nb, int bn,
                                               int c_lo, int c_hi, uint32_t sc, bool has_consts,
                                               const EpiPre& pre, const EpiRed& red) {
   constexpr bool rope = ROPE && !ROUTER && !DUAL;
@@ -360,13 +362,13 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
   float rsum = 0.f;
 #pragma unroll 1
   for (int c = c_lo; c < c_hi; ++c) {
-    const int n0 = nb * BN + c * 32;
+    const int n0 = nb * bn + c * 32;
     // rotary halves of 32 or more features: chunk c pairs with chunk
     // c + half / 32, both handled by the owner of c
     const bool rot = rope && n0 < p.rope_cols;
     if (rot && p.rope_half >= 32) {
       if ((n0 % p.rope_hd) < p.rope_half && n0 < p.N)   // else done with its partner
-        rope_pair(p, tacc, c, c + p.rope_half / 32, BN, nb, sc, has_consts, tab_row, mvalid, orow);
+        rope_pair(p, tacc, c, c + p.rope_half / 32, bn, nb, sc, has_consts, tab_row, mvalid, orow);
       continue;
     }
     uint32_t r[32];
@@ -445,15 +447,14 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
 
 // Prefetch of the residual of chunks c_lo, c_lo + 1 for row m (before the
 // accumulator is ready; the residual is an input of the kernel).
-template <int BN>
-__device__ __forceinline__ void prefetch_res(const GemmDev& p, int m, int nb, int c_lo, int c_hi,
-                                             EpiPre& pre) {
+__device__ __forceinline__ void prefetch_res(const GemmDev& p, int m, int nb, int bn, int c_lo,
+                                             int c_hi, EpiPre& pre) {
   pre.n = 0;
   if (!p.add || m >= p.M) return;
   const int64_t rrow = p.add_gathered ? (int64_t)p.rows[m] : (int64_t)m;
   const int n = min(2, c_hi - c_lo);
   for (int k = 0; k < n; ++k) {
-    const int n0 = nb * BN + (c_lo + k) * 32;
+    const int n0 = nb * bn + (c_lo + k) * 32;
     if (n0 >= p.N) break;
     if (k == 0) load_res32(p, rrow, n0, pre.res[0]);
     else load_res32(p, rrow, n0, pre.res[1]);
@@ -469,15 +470,16 @@ __device__ __forceinline__ bool epilogue_role(const GemmDev& P, int m, int nb, i
                                               uint32_t tacc, uint32_t sc, uint32_t tfull,
                                               uint32_t parity, volatile int* abort_flag,
                                               int lane) {
-  constexpr int NC = BN / 32;
+  const int bn = P.bn;
+  const int NC = bn / 32;
   // the router's row reduction stays in one warp per quarter
   const int c_lo = ROUTER ? (half == 0 ? 0 : NC) : half * (NC / 2);
   const int c_hi = ROUTER ? NC : (half + 1) * (NC / 2);
   const bool has_consts = ROUTER || P.bias || P.bias2;
-  if (has_consts) stage_consts<BN, ROUTER>(P, nb, sc, lane);
+  if (has_consts) stage_consts<ROUTER>(P, nb, bn, sc, lane);
   EpiPre pre;
   pre.n = 0;
-  if (!P.rope_tab) prefetch_res<BN>(P, m, nb, c_lo, c_hi, pre);
+  if (!P.rope_tab) prefetch_res(P, m, nb, bn, c_lo, c_hi, pre);
   int ok = 0;
   if (lane == 0) ok = mbar_wait_bounded(tfull, parity, abort_flag, P.err, P.timeout_ns);
   ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -485,9 +487,9 @@ __device__ __forceinline__ bool epilogue_role(const GemmDev& P, int m, int nb, i
   tc_fence_after();
   const EpiRed none = {nullptr, 0, 0, 0};
   if (!ROUTER && !DUAL && P.rope_tab)
-    epilogue_tile<BN, DUAL, ROUTER, true>(P, tacc, m, nb, c_lo, c_hi, sc, has_consts, pre, none);
+    epilogue_tile<BN, DUAL, ROUTER, true>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none);
   else
-    epilogue_tile<BN, DUAL, ROUTER, false>(P, tacc, m, nb, c_lo, c_hi, sc, has_consts, pre, none);
+    epilogue_tile<BN, DUAL, ROUTER, false>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none);
   return true;
 }
 
@@ -515,8 +517,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int tiles0 = tiles_of(p, BM, BN);
-  const int num_tiles = tiles0 + tiles_of(p2, BM, BN);
+  const int tiles0 = tiles_of(p, BM);
+  const int num_tiles = tiles0 + tiles_of(p2, BM);
 
   pdl_trigger();
   if (threadIdx.x == 0) {
@@ -554,25 +556,27 @@ __global__ void __launch_bounds__(kThreads, 1)
       int stage = 0;
       uint32_t phase = 0;
       int64_t issued = 0;
-      constexpr uint32_t tx = C::STAGE_BYTES;
+      // bytes per stage: the A tile and this problem's weight tile(s)
+      auto stage_tx = [](int bn) { return (uint32_t)(C::A_BYTES + bn * BK * 2 * C::NUM_B); };
       // The weights do not depend on the previous kernel: the first tile's
       // weight tiles are requested before waiting for it.
       int pre = 0;
       if ((int)blockIdx.x < num_tiles) {
-        const TileInfo ti = tile_info(blockIdx.x, p, p2, tiles0, BM, BN);
+        const TileInfo ti = tile_info(blockIdx.x, p, p2, tiles0, BM);
         pre = ti.nkb < C::STAGES ? ti.nkb : C::STAGES;
         for (int kb = 0; kb < pre; ++kb) {
           const KbSrc src = kb_source(ti, kb, &tmA, &tmB, &tmA2, &tmB2);
           const uint32_t fb = full0 + 8 * kb;
-          mbar_arrive_expect_tx(fb, tx);
-          tma_load_2d(sB + kb * C::B_BYTES, src.b, src.kc, ti.nb * BN, fb);
-          if (DUAL) tma_load_2d(sB2 + kb * C::B_BYTES, &tmB2, src.kc, ti.nb * BN, fb);
+          mbar_arrive_expect_tx(fb, stage_tx(ti.bn));
+          tma_load_2d(sB + kb * C::B_BYTES, src.b, src.kc, ti.nb * ti.bn, fb);
+          if (DUAL) tma_load_2d(sB2 + kb * C::B_BYTES, &tmB2, src.kc, ti.nb * ti.bn, fb);
         }
       }
       pdl_wait();
       bool first = true;
       for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
-        const TileInfo ti = tile_info(t, p, p2, tiles0, BM, BN);
+        const TileInfo ti = tile_info(t, p, p2, tiles0, BM);
+        const uint32_t tx = stage_tx(ti.bn);
         bool ok = true;
         for (int kb = 0; kb < ti.nkb; ++kb) {
           const KbSrc src = kb_source(ti, kb, &tmA, &tmB, &tmA2, &tmB2);
@@ -586,8 +590,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             mbar_arrive_expect_tx(fb, tx);
             tma_load_2d(sA + stage * C::A_BYTES, src.a, src.kc, ti.mb * BM, fb);
-            tma_load_2d(sB + stage * C::B_BYTES, src.b, src.kc, ti.nb * BN, fb);
-            if (DUAL) tma_load_2d(sB2 + stage * C::B_BYTES, &tmB2, src.kc, ti.nb * BN, fb);
+            tma_load_2d(sB + stage * C::B_BYTES, src.b, src.kc, ti.nb * ti.bn, fb);
+            if (DUAL) tma_load_2d(sB2 + stage * C::B_BYTES, &tmB2, src.kc, ti.nb * ti.bn, fb);
           }
           ++issued;
           if (++stage == C::STAGES) { stage = 0; phase ^= 1; }
@@ -605,13 +609,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+      constexpr uint32_t idesc_full = idesc_bf16_f32(BM, BN);
+      constexpr uint32_t idesc_half = idesc_bf16_f32(BM, BN / 2 < 64 ? 64 : BN / 2);
       int stage = 0;
       uint32_t phase = 0;
       int it = 0;
       bool ok = true;
       for (int t = blockIdx.x; t < num_tiles && ok; t += gridDim.x, ++it) {
-        const TileInfo ti = tile_info(t, p, p2, tiles0, BM, BN);
+        const TileInfo ti = tile_info(t, p, p2, tiles0, BM);
+        const uint32_t idesc = ti.bn == BN ? idesc_full : idesc_half;
         const int acc = it & 1;
         if (!mbar_wait_bounded(tempty0 + 8 * acc, ((it >> 1) & 1) ^ 1, abort_flag, p.err,
                                p.timeout_ns)) {
@@ -657,7 +663,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int row_in_tile = quarter * 32 + lane;
     int it = 0;
     for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++it) {
-      const TileInfo ti = tile_info(t, p, p2, tiles0, BM, BN);
+      const TileInfo ti = tile_info(t, p, p2, tiles0, BM);
       const GemmDev& P = ti.prob ? p2 : p;
       const int acc = it & 1;
       const uint32_t sc = sconst + 4u * kConstFloats * ((warp - 2) * 2 + acc);
@@ -717,7 +723,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int rank = (int)cluster_ctarank();
   const int NCO = BN / S / 32;                // chunks finalised by each CTA
   const int tile = blockIdx.x / S;
-  const TileInfo ti = tile_info(tile, p, p, 1 << 30, BM, BN);
+  const TileInfo ti = tile_info(tile, p, p, 1 << 30, BM);
   const int kb0 = rank * ti.nkb / S;
   const int kb1 = (rank + 1) * ti.nkb / S;
   const int nkb = kb1 - kb0;
@@ -831,7 +837,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     // ------------------------------------------------------------ epilogue, part 1
     pdl_wait();
-    if (has_consts) stage_consts<BN, false>(p, ti.nb, sc, lane);
+    if (has_consts) stage_consts<false>(p, ti.nb, BN, sc, lane);
     if (lane == 0) ok = mbar_wait_bounded(tfull, 0, abort_flag, p.err, p.timeout_ns);
     ok = __shfl_sync(0xffffffffu, ok, 0);
     tc_fence_after();
@@ -851,7 +857,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3])));
         }
       }
-      if (h_lo < h_hi) prefetch_res<BN>(p, m, ti.nb, c_lo, c_hi, pre);
+      if (h_lo < h_hi) prefetch_res(p, m, ti.nb, BN, c_lo, c_hi, pre);
     }
   }
 
@@ -864,9 +870,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ epilogue, part 2
     const EpiRed red = {p.scratch + (size_t)tile * S * BM * BN, S, rank, BN};
     if (p.rope_tab)   // rotary halves of at most 16 features (one chunk)
-      epilogue_tile<BN, false, false, true>(p, tacc, m, ti.nb, c_lo, c_hi, sc, has_consts, pre, red);
+      epilogue_tile<BN, false, false, true>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre, red);
     else
-      epilogue_tile<BN, false, false, false>(p, tacc, m, ti.nb, c_lo, c_hi, sc, has_consts, pre, red);
+      epilogue_tile<BN, false, false, false>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre,
+                                             red);
   }
 
   __syncwarp();
@@ -917,8 +924,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int brow_off = DUAL ? 0 : (int)rank * C::B_ROWS;
   const int pair = blockIdx.x >> 1;
   const int num_pairs = gridDim.x >> 1;
-  const int tiles0 = tiles_of(p, 2 * BM, BN);
-  const int num_tiles = tiles0 + tiles_of(p2, 2 * BM, BN);
+  const int tiles0 = tiles_of(p, 2 * BM);
+  const int num_tiles = tiles0 + tiles_of(p2, 2 * BM);
   // DUAL: the odd CTA reads the second weight for every k-block
   auto wmap = [&](const KbSrc& s) -> const CUtensorMap* {
     return DUAL ? (rank == 1 ? &tmB2 : &tmB) : s.b;
@@ -967,7 +974,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       constexpr uint32_t tx = 2 * C::STAGE_BYTES;
       int pre = 0;
       if (pair < num_tiles) {
-        const TileInfo ti = tile_info(pair, p, p2, tiles0, 2 * BM, BN);
+        const TileInfo ti = tile_info(pair, p, p2, tiles0, 2 * BM);
         pre = ti.nkb < C::STAGES ? ti.nkb : C::STAGES;
         for (int kb = 0; kb < pre; ++kb) {
           const KbSrc src = kb_source(ti, kb, &tmA, &tmB, &tmA2, &tmB2);
@@ -979,7 +986,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       pdl_wait();
       bool first = true;
       for (int t = pair; t < num_tiles; t += num_pairs) {
-        const TileInfo ti = tile_info(t, p, p2, tiles0, 2 * BM, BN);
+        const TileInfo ti = tile_info(t, p, p2, tiles0, 2 * BM);
         const int arow0 = ti.mb * 2 * BM + (int)rank * BM;
         const int brow0 = ti.nb * BN + brow_off;
         bool ok = true;
@@ -1021,7 +1028,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       int it = 0;
       bool ok = true;
       for (int t = pair; t < num_tiles && ok; t += num_pairs, ++it) {
-        const TileInfo ti = tile_info(t, p, p2, tiles0, 2 * BM, BN);
+        const TileInfo ti = tile_info(t, p, p2, tiles0, 2 * BM);
         const int acc = it & 1;
         if (!mbar_wait_bounded(tempty0 + 8 * acc, ((it >> 1) & 1) ^ 1, abort_flag, p.err,
                                p.timeout_ns)) {
@@ -1061,7 +1068,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const int row_in_tile = quarter * 32 + lane;
     int it = 0;
     for (int t = pair; t < num_tiles; t += num_pairs, ++it) {
-      const TileInfo ti = tile_info(t, p, p2, tiles0, 2 * BM, BN);
+      const TileInfo ti = tile_info(t, p, p2, tiles0, 2 * BM);
       const GemmDev& P = ti.prob ? p2 : p;
       const int acc = it & 1;
       const uint32_t sc = sconst + 4u * kConstFloats * ((warp - 2) * 2 + acc);
@@ -1186,20 +1193,29 @@ bool problem_maps(const GemmArgs& a, uint32_t a_rows, uint32_t b_rows, CUtensorM
 }
 
 // Maps and device descriptors for a launch of problem `a` (plus the grouped
-// problem `b`, or the DUAL second weight).
+// problem `b`, or the DUAL second weight). bn: the kernel's tile width; a
+// problem may ask for half of it (tile_n); b_rows: weight rows a CTA stages
+// per full-width tile (half of bn on CTA pairs).
 template <bool DUAL>
-cudaError_t prepare(const GemmArgs& a, const GemmArgs* b, uint32_t a_rows, uint32_t b_rows,
+cudaError_t prepare(const GemmArgs& a, const GemmArgs* b, uint32_t a_rows, int bn, uint32_t b_rows,
                     const Dev& dev, CUtensorMap (&tm)[4], GemmDev& p, GemmDev& p2) {
+  auto width = [&](const GemmArgs& g) { return g.tile_n > 0 && g.tile_n < bn ? g.tile_n : bn; };
+  auto rows = [&](const GemmArgs& g) { return (uint32_t)((uint64_t)b_rows * width(g) / bn); };
+  if ((a.tile_n && width(a) * 2 != bn && width(a) != bn) || (b && b->tile_n && width(*b) * 2 != bn && width(*b) != bn))
+    return cudaErrorInvalidValue;
   if (!make_dev(a, dev, p)) return cudaErrorInvalidValue;
+  p.bn = width(a);
   p2 = GemmDev{};
-  if (!problem_maps(a, a_rows, b_rows, tm[0], tm[1], &tm[2], &tm[3])) return cudaErrorInvalidValue;
+  p2.bn = bn;
+  if (!problem_maps(a, a_rows, rows(a), tm[0], tm[1], &tm[2], &tm[3])) return cudaErrorInvalidValue;
   if (DUAL) {
-    if (!make_tmap(&tm[3], a.W2, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, b_rows))
+    if (p.bn != bn || !make_tmap(&tm[3], a.W2, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, b_rows))
       return cudaErrorInvalidValue;
     tm[2] = tm[0];
   } else if (b) {
     if (a.K2 > 0 || b->K2 > 0 || !make_dev(*b, dev, p2)) return cudaErrorInvalidValue;
-    if (!problem_maps(*b, a_rows, b_rows, tm[2], tm[3], nullptr, nullptr))
+    p2.bn = width(*b);
+    if (!problem_maps(*b, a_rows, rows(*b), tm[2], tm[3], nullptr, nullptr))
       return cudaErrorInvalidValue;
   } else if (a.K2 == 0) {
     tm[2] = tm[0];
@@ -1222,10 +1238,10 @@ cudaError_t launch(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
   }
   CUtensorMap tm[4];
   GemmDev p, p2;
-  cudaError_t e = prepare<DUAL>(a, b, BM, BN, dev, tm, p, p2);
+  cudaError_t e = prepare<DUAL>(a, b, BM, BN, BN, dev, tm, p, p2);
   if (e != cudaSuccess) return e;
-  int64_t num_tiles = ((a.M + BM - 1) / BM) * ((a.N + BN - 1) / BN);
-  if (b) num_tiles += ((b->M + BM - 1) / BM) * ((b->N + BN - 1) / BN);
+  int64_t num_tiles = ((a.M + BM - 1) / BM) * ((a.N + p.bn - 1) / p.bn);
+  if (b) num_tiles += ((b->M + BM - 1) / BM) * ((b->N + p2.bn - 1) / p2.bn);
   const int grid = (int)(num_tiles < dev.num_sms ? num_tiles : dev.num_sms);
   return launch_pdl(gemm_tc_kernel<BN, DUAL, ROUTER>, dim3(grid), dim3(kThreads), C::SMEM_BYTES,
                     dev.stream, tm[0], tm[1], tm[2], tm[3], p, p2);
@@ -1259,7 +1275,14 @@ cudaError_t launch_pair(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
   const int64_t cap = device < 64 ? max_pairs[device] : dev.num_sms / 2;
   CUtensorMap tm[4];
   GemmDev p, p2;
-  cudaError_t e = prepare<DUAL>(a, b, BM, C::B_ROWS, dev, tm, p, p2);
+  GemmArgs a_full = a;
+  a_full.tile_n = 0;   // CTA pairs: full-width tiles only
+  GemmArgs b_full;
+  if (b) {
+    b_full = *b;
+    b_full.tile_n = 0;
+  }
+  cudaError_t e = prepare<DUAL>(a_full, b ? &b_full : nullptr, BM, BN, C::B_ROWS, dev, tm, p, p2);
   if (e != cudaSuccess) return e;
   int64_t num_tiles = ((a.M + 2 * BM - 1) / (2 * BM)) * ((a.N + BN - 1) / BN);
   if (b) num_tiles += ((b->M + 2 * BM - 1) / (2 * BM)) * ((b->N + BN - 1) / BN);
@@ -1321,7 +1344,9 @@ cudaError_t launch_sk(const GemmArgs& a, const Dev& dev, int S) {
   using C = TileCfg<BN, false>;
   CUtensorMap tm[4];
   GemmDev p, p2;
-  cudaError_t e = prepare<false>(a, nullptr, BM, BN, dev, tm, p, p2);
+  GemmArgs a_full = a;
+  a_full.tile_n = 0;
+  cudaError_t e = prepare<false>(a_full, nullptr, BM, BN, BN, dev, tm, p, p2);
   if (e != cudaSuccess) return e;
   const int64_t num_tiles = ((a.M + BM - 1) / BM) * ((a.N + BN - 1) / BN);
   return launch_pdl_cluster(gemm_tc_sk_kernel<BN>, dim3((unsigned)(num_tiles * S)), dim3(kThreads),
@@ -1418,13 +1443,29 @@ cudaError_t gemm_bf16_grouped(const GemmArgs& a, const GemmArgs& b, const Dev& d
   // ties go to CTA pairs (half the weight bytes per SM), then to 256-wide
   // tiles. Problem `a` comes first in the tile order: pass the one with the
   // costlier epilogue as `a` so that it runs in the first round.
+  // Cost in k-block units: rounds of tiles x k-blocks, plus the epilogue of
+  // a last-round tile (per 32-column chunk of a thread: ~1.5 units, ~3 with
+  // GELU). Giving the first problem half-width (128-column) tiles doubles
+  // its tiles but halves their epilogue.
   auto tiles = [](const GemmArgs& g, int bm, int bn) { return ((g.M + bm - 1) / bm) * ((g.N + bn - 1) / bn); };
+  auto chunk = [](const GemmArgs& g) -> int64_t { return g.epi.act == ACT_GELU ? 3 : 2; };
   const int64_t sms = dev.num_sms;
-  const int64_t r_pair = (tiles(a, 256, 256) + tiles(b, 256, 256) + sms / 2 - 1) / (sms / 2);
-  const int64_t r256 = (tiles(a, 128, 256) + tiles(b, 128, 256) + sms - 1) / sms;
-  const int64_t r128 = (tiles(a, 128, 128) + tiles(b, 128, 128) + sms - 1) / sms;
-  if (r_pair <= r256 && r_pair <= r128) return launch_pair<256, false>(a, &b, dev);
-  if (r256 <= r128) return launch<256, false, false>(a, &b, dev);
+  const int64_t kb = (std::max(a.K, b.K) + BK - 1) / BK;
+  const int64_t epi_w = 4 * std::max(chunk(a), chunk(b));
+  const int64_t c_pair = (tiles(a, 256, 256) + tiles(b, 256, 256) + sms / 2 - 1) / (sms / 2) * kb + epi_w;
+  const int64_t c256 = (tiles(a, 128, 256) + tiles(b, 128, 256) + sms - 1) / sms * kb + epi_w;
+  const int64_t c_half = (tiles(a, 128, 128) + tiles(b, 128, 256) + sms - 1) / sms * kb +
+                         std::max(2 * chunk(a), 4 * chunk(b));
+  const int64_t c128 = (tiles(a, 128, 128) + tiles(b, 128, 128) + sms - 1) / sms * kb +
+                       2 * std::max(chunk(a), chunk(b));
+  const int64_t best = std::min(std::min(c_pair, c256), std::min(c_half, c128));
+  if (c_pair == best) return launch_pair<256, false>(a, &b, dev);
+  if (c256 == best) return launch<256, false, false>(a, &b, dev);
+  if (c_half == best) {
+    GemmArgs a_half = a;
+    a_half.tile_n = 128;
+    return launch<256, false, false>(a_half, &b, dev);
+  }
   return launch<128, false, false>(a, &b, dev);
 }
 

@@ -66,6 +66,9 @@ struct GemmArgs {
   // split is used only when it fits (gemm_split_scratch_bytes covers every case)
   float* scratch = nullptr;
   size_t scratch_bytes = 0;
+  // tile width (N) for this problem when the kernel's is 256: 0 = full, or
+  // 128 (half-width tiles; one-CTA kernel)
+  int tile_n = 0;
 };
 // Scratch that lets gemm_bf16 split any small-M product along K.
 size_t gemm_split_scratch_bytes();
