@@ -135,33 +135,17 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Same, acquiring at cluster scope: for phases completed by arrivals (with
-// release at cluster scope) from other CTAs of the cluster.
-__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
 // Wait for the phase of parity `parity` of barrier `bar` to complete, giving
 // up after `timeout_ns` or as soon as another role of the block raised
 // *abort. On give-up the block's abort flag and the device error word are
 // set and false is returned.
-template <bool CLUSTER = false>
 __device__ __forceinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity,
                                                   volatile int* abort_flag, int* err,
                                                   unsigned long long timeout_ns) {
-  auto try_wait = [&] { return CLUSTER ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity); };
-  if (try_wait()) return true;
+  if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = globaltimer_ns();
   for (uint32_t it = 1;; ++it) {
-    if (try_wait()) return true;
+    if (mbar_try_wait(bar, parity)) return true;
     if ((it & 15u) == 0) {
       if (abort_flag && *abort_flag) return false;
       if (globaltimer_ns() - t0 > timeout_ns) {
@@ -314,22 +298,14 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const void* tmap,
       "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(cluster_bar)
       : "memory");
 }
-// Bulk copy of `bytes` (multiple of 16) from this CTA's shared memory to
-// shared memory of another CTA of the cluster; completion is counted as
-// transaction bytes on `cluster_bar`, an mbarrier of the destination CTA.
-__device__ __forceinline__ void bulk_copy_to_cta(uint32_t dst_cluster, uint32_t src, uint32_t bytes,
-                                                 uint32_t cluster_bar) {
+// Bulk copy of `bytes` (multiple of 16, both addresses 16-byte aligned) from
+// global memory into this CTA's shared memory; completion is counted as
+// transaction bytes on `bar`.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
   asm volatile(
-      "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-          dst_cluster),
-      "r"(src), "r"(bytes), "r"(cluster_bar)
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar)
       : "memory");
-}
-// 16-byte store to shared memory of any CTA of the cluster (address from mapa).
-__device__ __forceinline__ void st_cluster_f4(uint32_t addr, const float* f) {
-  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(f[0]),
-               "f"(f[1]), "f"(f[2]), "f"(f[3])
-               : "memory");
 }
 // Barrier among `nthreads` threads (whole warps) on named barrier `id` (1..15).
 __device__ __forceinline__ void named_bar_sync(int id, int nthreads) {

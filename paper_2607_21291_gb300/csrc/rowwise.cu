@@ -174,24 +174,141 @@ __device__ __forceinline__ void norm_share(int64_t lo, int64_t hi, const T* x, i
   }
 }
 
-constexpr int kNormThreads = 256;
-constexpr int kNormRowsPerBlock = 32;   // four rows per warp
+// ---------------------------------------------------------------- TMA-staged gather + norm
+// For large row counts (HBM bound): one warp streams whole source rows into a
+// shared-memory ring with one bulk copy each (cp.async.bulk, completion on the
+// slot's mbarrier), eight warps normalise them from shared memory, one warp
+// per row, and release the slot. Many rows are in flight per SM with few
+// registers, and each 16-byte global store of a warp covers 512 contiguous
+// bytes of an output row.
+constexpr int kRowWarps = 8;                       // consumer warps
+constexpr int kRowThreads = 32 * (kRowWarps + 1);  // + the producer warp
+constexpr int kRowSlots = 16;                      // ring slots (two rows per consumer warp)
+static_assert(kRowSlots % kRowWarps == 0, "a slot is always consumed by the same warp");
+constexpr int kMaxRowBytes = 8192;   // d <= 4096 (bf16) or 2048 (fp32)
 
-// out1[m] = norm(x[row(m)]; g1, b1), out2[m] = norm(x[row(m)]; g2, b2), one warp per row.
-template <typename T, bool RMS, int NCH>
-__global__ void __launch_bounds__(kNormThreads)
-    gather_norm_kernel(const T* x, const int32_t* rows, int64_t M, int d, const T* g1, const T* b1,
-                       const T* g2, const T* b2, float eps, T* out1, T* out2) {
+// out1[m] = norm(x[row(m)]; g1, b1), out2[m] = norm(x[row(m)]; g2, b2) for the
+// block's contiguous share of m. Shared memory: the staged parameters
+// ([4][d]), then the ring (kRowSlots rows of d), then 2 kRowSlots mbarriers.
+template <typename T, bool RMS>
+__global__ void __launch_bounds__(kRowThreads)
+    gather_norm_tma_kernel(const T* x, const int32_t* rows, int64_t M, int d, const T* g1,
+                           const T* b1, const T* g2, const T* b2, float eps, T* out1, T* out2,
+                           int* err, unsigned long long timeout_ns) {
   pdl_trigger();
-  extern __shared__ __align__(16) uint8_t smem_norm[];
-  T* sp = reinterpret_cast<T*>(smem_norm);
+  extern __shared__ __align__(16) uint8_t smem_rows[];
+  constexpr int V = Elem<T>::kVec;
+  const uint32_t row_bytes = (uint32_t)d * sizeof(T);
+  T* sp = reinterpret_cast<T*>(smem_rows);
+  uint8_t* ring = smem_rows + 4 * (size_t)row_bytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ring + (size_t)kRowSlots * row_bytes);
+  const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * kRowSlots;
+  __shared__ int abort_flag;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kRowSlots; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    abort_flag = 0;
+    fence_barrier_init();
+  }
   stage_norm_params(g1, RMS ? nullptr : b1, out2 ? g2 : nullptr, (RMS || !out2) ? nullptr : b2, d,
-                    sp);   // weights: independent of the previous kernel
+                    sp);   // weights: independent of the previous kernel (also syncs the block)
   pdl_wait();
-  const int64_t m0 = (int64_t)blockIdx.x * kNormRowsPerBlock;
-  norm_share<T, RMS, NCH>(
-      m0, min(M, m0 + kNormRowsPerBlock), x, d, sp, eps, out1, out2,
-      [&](int64_t m) { return rows ? (int64_t)rows[m] : m; }, [](int64_t m) { return m; });
+  const int64_t lo = (int64_t)blockIdx.x * M / gridDim.x, hi = (int64_t)(blockIdx.x + 1) * M / gridDim.x;
+  const int64_t n = hi - lo;
+  volatile int* abort_v = &abort_flag;
+
+  if (warp == kRowWarps) {
+    // ------------------------------------------------------------ producer
+    // The warp reads the source row indices 32 at a time; lane 0 issues the copies.
+    int64_t issued = 0;
+    bool ok = true;
+    for (int64_t j0 = 0; j0 < n && ok; j0 += 32) {
+      int64_t src_l = 0;
+      if (j0 + lane < n) src_l = rows ? (int64_t)rows[lo + j0 + lane] : lo + j0 + lane;
+      const int cnt = (int)(n - j0 < 32 ? n - j0 : 32);
+      for (int k = 0; k < cnt; ++k) {
+        const int64_t src = __shfl_sync(0xffffffffu, src_l, k);
+        const int64_t j = j0 + k;
+        const int s = (int)(j % kRowSlots);
+        const uint32_t round = (uint32_t)(j / kRowSlots);
+        int w = 1;
+        if (lane == 0) {
+          if (round > 0)
+            w = mbar_wait_bounded(empty0 + 8 * s, (round - 1) & 1, abort_v, err, timeout_ns);
+          if (w) {
+            mbar_arrive_expect_tx(full0 + 8 * s, row_bytes);
+            bulk_load(smem_u32(ring + (size_t)s * row_bytes), x + src * d, row_bytes, full0 + 8 * s);
+          }
+        }
+        if (!__shfl_sync(0xffffffffu, w, 0)) {
+          ok = false;
+          break;
+        }
+        ++issued;
+      }
+    }
+    // every copy issued has landed before the block may exit
+    if (lane == 0)
+      for (int s = 0; s < kRowSlots && s < issued; ++s) {
+        const int64_t last = s + ((issued - 1 - s) / kRowSlots) * kRowSlots;
+        mbar_wait_drain(full0 + 8 * s, (uint32_t)((last / kRowSlots) & 1), timeout_ns);
+      }
+  } else {
+    // ------------------------------------------------------------ consumers
+    const int nv = d / V;
+    for (int64_t j = warp; j < n; j += kRowWarps) {
+      const int s = (int)(j % kRowSlots);
+      int ok = 0;
+      if (lane == 0)
+        ok = mbar_wait_bounded(full0 + 8 * s, (uint32_t)((j / kRowSlots) & 1), abort_v, err, timeout_ns);
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      const T* xr = reinterpret_cast<const T*>(ring + (size_t)s * row_bytes);
+      float sum = 0.f;
+      for (int ci = lane; ci < nv; ci += 32) {
+        float f[V];
+        load_vec(xr + ci * V, f);
+#pragma unroll
+        for (int k = 0; k < V; ++k) sum += RMS ? f[k] * f[k] : f[k];
+      }
+      float mean = 0.f, rstd;
+      if (RMS) {
+        rstd = 1.f / sqrtf(warp_sum(sum) / d + eps);
+      } else {
+        mean = warp_sum(sum) / d;
+        float q = 0.f;
+        for (int ci = lane; ci < nv; ci += 32) {
+          float f[V];
+          load_vec(xr + ci * V, f);
+#pragma unroll
+          for (int k = 0; k < V; ++k) q += (f[k] - mean) * (f[k] - mean);
+        }
+        rstd = 1.f / sqrtf(warp_sum(q) / d + eps);
+      }
+      const int64_t m = lo + j;
+      for (int ci = lane; ci < nv; ci += 32) {
+        float f[V], g[V], bb[V], o[V];
+        load_vec(xr + ci * V, f);
+        load_vec(sp + ci * V, g);
+        if (!RMS) load_vec(sp + d + ci * V, bb);
+#pragma unroll
+        for (int k = 0; k < V; ++k) o[k] = (f[k] - mean) * rstd * g[k] + (RMS ? 0.f : bb[k]);
+        store_vec(out1 + m * d + ci * V, o);
+        if (out2) {
+          load_vec(sp + 2 * d + ci * V, g);
+          if (!RMS) load_vec(sp + 3 * d + ci * V, bb);
+#pragma unroll
+          for (int k = 0; k < V; ++k) o[k] = (f[k] - mean) * rstd * g[k] + (RMS ? 0.f : bb[k]);
+          store_vec(out2 + m * d + ci * V, o);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(empty0 + 8 * s);   // the slot may be refilled
+    }
+  }
 }
 
 // ---------------------------------------------------------------- rotary embedding
@@ -619,24 +736,28 @@ template <typename T, bool RMS>
 cudaError_t gather_norm_t(const void* x, const int32_t* rows, int64_t M, int d, const void* g1,
                           const void* b1, const void* g2, const void* b2, float eps, void* out1,
                           void* out2, const Dev& dev) {
-  const unsigned grid = (unsigned)((M + kNormRowsPerBlock - 1) / kNormRowsPerBlock);
-  const size_t smem = 4 * (size_t)d * sizeof(T);
-  return with_nch<T>(d, [&](auto nch) -> cudaError_t {
-    constexpr int NCH = decltype(nch)::value;
-    static int attr_done[64] = {0};
-    int device = 0;
-    cudaGetDevice(&device);
-    if (device < 64 && !attr_done[device]) {
-      cudaError_t e = cudaFuncSetAttribute(gather_norm_kernel<T, RMS, NCH>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize, 4 * 4096 * 4);
-      if (e != cudaSuccess) return e;
-      attr_done[device] = 1;
-    }
-    return launch_pdl(gather_norm_kernel<T, RMS, NCH>, dim3(grid), dim3(kNormThreads), smem,
-                      dev.stream, static_cast<const T*>(x), rows, M, d, static_cast<const T*>(g1),
-                      static_cast<const T*>(b1), static_cast<const T*>(g2),
-                      static_cast<const T*>(b2), eps, static_cast<T*>(out1), static_cast<T*>(out2));
-  });
+  const size_t row_bytes = (size_t)d * sizeof(T);
+  const size_t smem = 4 * row_bytes + kRowSlots * row_bytes + 2 * kRowSlots * 8;
+  static int attr_done[64] = {0};
+  int device = 0;
+  cudaGetDevice(&device);
+  if (device < 64 && !attr_done[device]) {
+    cudaError_t e = cudaFuncSetAttribute(gather_norm_tma_kernel<T, RMS>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (4 + kRowSlots) * kMaxRowBytes + 2 * kRowSlots * 8);
+    if (e != cudaSuccess) return e;
+    attr_done[device] = 1;
+  }
+  // one wave: as many blocks per SM as fit (at most two), at least one row
+  // per consumer warp
+  const int64_t fit = std::max<int64_t>(1, std::min<int64_t>(2, 232448 / (int64_t)(smem + 1024)));
+  const int64_t grid = std::max<int64_t>(1, std::min<int64_t>((M + kRowWarps - 1) / kRowWarps,
+                                                             fit * dev.num_sms));
+  return launch_pdl(gather_norm_tma_kernel<T, RMS>, dim3((unsigned)grid), dim3(kRowThreads), smem,
+                    dev.stream, static_cast<const T*>(x), rows, M, d, static_cast<const T*>(g1),
+                    static_cast<const T*>(b1), static_cast<const T*>(g2),
+                    static_cast<const T*>(b2), eps, static_cast<T*>(out1), static_cast<T*>(out2),
+                    dev.err, kWaitTimeoutNs);
 }
 
 cudaError_t gather_norm(int dtype, const void* x, const int32_t* rows, int64_t M, int d,
