@@ -263,8 +263,9 @@ __device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, cons
 }
 
 // Rotary halves of 32 or more features: chunk c (first half of a head's
-// rotated features) and chunk c2 (second half) of row m, 8 features at a time
-// to keep few registers live: a' = a cos - b sin, b' = b cos + a sin.
+// rotated features) and chunk c2 (second half) of row m: a' = a cos - b sin,
+// b' = b cos + a sin. The row's (cos, sin) pairs are loaded 16 at a time
+// (their latency paid twice per chunk pair), the accumulator 8 columns at a time.
 // These are query / key columns: no activation, residual or transposed copy.
 __device__ __forceinline__ void rope_pair(const GemmDev& p, uint32_t tacc, int c, int c2, int bn,
                                           int nb, uint32_t sc, bool has_consts,
@@ -272,39 +273,50 @@ __device__ __forceinline__ void rope_pair(const GemmDev& p, uint32_t tacc, int c
   const int n0 = nb * bn + c * 32, n2 = nb * bn + c2 * 32;
   const int i0 = n0 % p.rope_hd;
 #pragma unroll 1
-  for (int g = 0; g < 4; ++g) {
-    uint32_t ra[8], rb[8];
-    tmem_ld8(tacc + c * 32 + 8 * g, ra);
-    tmem_ld8(tacc + c2 * 32 + 8 * g, rb);
-    tmem_ld_wait();
-    if (!mvalid) continue;
-    float a[8], b[8];
+  for (int gh = 0; gh < 2; ++gh) {
+    float4 t[8];   // t[k] = (cos, sin) of features i0 + 16 gh + 2k and the next one
+    if (mvalid) {
+      const float4* t4 = reinterpret_cast<const float4*>(tab_row + i0 + 16 * gh);
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      a[j] = __uint_as_float(ra[j]);
-      b[j] = __uint_as_float(rb[j]);
+      for (int k = 0; k < 8; ++k) t[k] = t4[k];
     }
-    if (has_consts) {
-      float f[4];
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        ld_shared_f4(sc + 4u * (c * 32 + 8 * g + 4 * h), f);
+    for (int gg = 0; gg < 2; ++gg) {
+      const int g = 2 * gh + gg;
+      uint32_t ra[8], rb[8];
+      tmem_ld8(tacc + c * 32 + 8 * g, ra);
+      tmem_ld8(tacc + c2 * 32 + 8 * g, rb);
+      tmem_ld_wait();
+      if (!mvalid) continue;
+      float a[8], b[8];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) a[4 * h + j] += f[j];
-        ld_shared_f4(sc + 4u * (c2 * 32 + 8 * g + 4 * h), f);
-#pragma unroll
-        for (int j = 0; j < 4; ++j) b[4 * h + j] += f[j];
+      for (int j = 0; j < 8; ++j) {
+        a[j] = __uint_as_float(ra[j]);
+        b[j] = __uint_as_float(rb[j]);
       }
-    }
+      if (has_consts) {
+        float f[4];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const float2 cs = tab_row[i0 + 8 * g + j];
-      const float x = a[j], y = b[j];
-      a[j] = x * cs.x - y * cs.y;
-      b[j] = y * cs.x + x * cs.y;
+        for (int h = 0; h < 2; ++h) {
+          ld_shared_f4(sc + 4u * (c * 32 + 8 * g + 4 * h), f);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) a[4 * h + j] += f[j];
+          ld_shared_f4(sc + 4u * (c2 * 32 + 8 * g + 4 * h), f);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) b[4 * h + j] += f[j];
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float4 q = t[4 * gg + j / 2];
+        const float cs = (j & 1) ? q.z : q.x, sn = (j & 1) ? q.w : q.y;
+        const float x = a[j], y = b[j];
+        a[j] = x * cs - y * sn;
+        b[j] = y * cs + x * sn;
+      }
+      store_vec(p.out + orow * p.ld_out + n0 + 8 * g, a);
+      store_vec(p.out + orow * p.ld_out + n2 + 8 * g, b);
     }
-    store_vec(p.out + orow * p.ld_out + n0 + 8 * g, a);
-    store_vec(p.out + orow * p.ld_out + n2 + 8 * g, b);
   }
 }
 
