@@ -424,27 +424,31 @@ __device__ __forceinline__ int block_excl_scan(int v, int* warp_tot, int& total)
 
 // Shared state of the block-wide Top-K.
 struct TopkShared {
-  int hist[256];
+  int hist[2][256];     // alternate passes use alternate histograms
   int warp_tot[33];
-  uint32_t digit;
-  int remaining;
+  uint32_t digit[4];    // per pass, so no pass overwrites what another still reads
+  int remaining[4];
 };
 
 // Radix select over the T order-preserving keys in shared memory (4 passes
 // of 8 bits, most significant first): the K-th largest key `kth` and how many
-// keys equal to it are kept (need_eq, lowest positions first). K >= 1.
+// keys equal to it are kept (need_eq, lowest positions first). K >= 1. Two
+// block barriers per pass: the next pass's histogram is cleared while this
+// pass's is filled.
 template <int NT>
 __device__ __forceinline__ void radix_select(const uint32_t* keys, int T, int K, TopkShared& sh,
                                              uint32_t& kth, int& need_eq) {
   uint32_t prefix = 0, pmask = 0;
   int remaining = K;   // keys still to take at or below the current prefix
+  for (int i = threadIdx.x; i < 256; i += NT) sh.hist[0][i] = 0;
+  __syncthreads();
   for (int pass = 0; pass < 4; ++pass) {
     const int shift = 24 - 8 * pass;
-    for (int i = threadIdx.x; i < 256; i += NT) sh.hist[i] = 0;
-    __syncthreads();
+    int* hist = sh.hist[pass & 1];
+    for (int i = threadIdx.x; i < 256; i += NT) sh.hist[(pass + 1) & 1][i] = 0;
     for (int t = threadIdx.x; t < T; t += NT) {
       const uint32_t k = keys[t];
-      if ((k & pmask) == prefix) atomicAdd(&sh.hist[(k >> shift) & 255u], 1);
+      if ((k & pmask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1);
     }
     __syncthreads();
     if (threadIdx.x < 32) {
@@ -453,7 +457,7 @@ __device__ __forceinline__ void radix_select(const uint32_t* keys, int T, int K,
       int cnt[8], lsum = 0;
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
-        cnt[j] = sh.hist[255 - 8 * lane - j];
+        cnt[j] = hist[255 - 8 * lane - j];
         lsum += cnt[j];
       }
       int incl = lsum;
@@ -469,8 +473,8 @@ __device__ __forceinline__ void radix_select(const uint32_t* keys, int T, int K,
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
           if (above + cnt[j] >= remaining) {
-            sh.digit = (uint32_t)(255 - 8 * lane - j);
-            sh.remaining = remaining - above;
+            sh.digit[pass] = (uint32_t)(255 - 8 * lane - j);
+            sh.remaining[pass] = remaining - above;
             break;
           }
           above += cnt[j];
@@ -478,39 +482,33 @@ __device__ __forceinline__ void radix_select(const uint32_t* keys, int T, int K,
       }
     }
     __syncthreads();
-    prefix |= sh.digit << shift;
+    prefix |= sh.digit[pass] << shift;
     pmask |= 255u << shift;
-    remaining = sh.remaining;
-    __syncthreads();
+    remaining = sh.remaining[pass];
   }
   kth = prefix;
   need_eq = remaining;
 }
 
 // Calls emit(i, t) for the kept positions t in ascending order, i = 0..K-1:
-// keys above kth, and the first need_eq keys equal to it. Contiguous chunks
-// of positions per thread and two block scans keep the output ascending.
+// keys above kth, and the first need_eq keys equal to it. Each thread owns a
+// contiguous chunk of positions; one block scan of the packed counts
+// (above << 16 | equal; T <= 16384) places every chunk's output.
 template <int NT, typename Emit>
 __device__ __forceinline__ void emit_kept(const uint32_t* keys, int T, uint32_t kth, int need_eq,
                                           TopkShared& sh, Emit emit) {
   const int chunk = (T + NT - 1) / NT;
   const int t0 = min(T, (int)threadIdx.x * chunk), t1 = min(T, t0 + chunk);
-  int n_eq = 0;
-  for (int t = t0; t < t1; ++t) n_eq += keys[t] == kth;
-  int total;
-  const int eq_base = block_excl_scan<NT>(n_eq, sh.warp_tot, total);   // equal keys before my chunk
-  int n_sel = 0, er = eq_base;
+  int n_gt = 0, n_eq = 0;
   for (int t = t0; t < t1; ++t) {
-    const uint32_t k = keys[t];
-    if (k > kth) {
-      ++n_sel;
-    } else if (k == kth) {
-      n_sel += er < need_eq;
-      ++er;
-    }
+    n_gt += keys[t] > kth;
+    n_eq += keys[t] == kth;
   }
-  int out = block_excl_scan<NT>(n_sel, sh.warp_tot, total);
-  er = eq_base;
+  int total;
+  const int base = block_excl_scan<NT>((n_gt << 16) | n_eq, sh.warp_tot, total);
+  const int eq_base = base & 0xffff;   // equal keys before my chunk
+  int out = (base >> 16) + min(eq_base, need_eq);
+  int er = eq_base;
   for (int t = t0; t < t1; ++t) {
     const uint32_t k = keys[t];
     bool take = k > kth;
