@@ -175,7 +175,11 @@ adadsf_status adadsf_alloc_ratios(const double *s_host, int L, double t, double 
 
 /* ------------------------------------------------------------------------
  * Sec. 3.4: router scores of every token, w2 . SiLU(W1 x + b1) + b2.
- * x_dev [B*T, d] (cfg->dtype); scores_dev [B*T] fp32.
+ * x_dev [B*T, d] (cfg->dtype); scores_dev [B*T] fp32. ws: at least 256
+ * bytes (the device error word); on the bf16 path, with
+ * adadsf_router_select_workspace_size(cfg, 1, 1) bytes or more (zero-filled
+ * before first use), tiles of 128 tokens may also be split along d over
+ * several CTAs.
  * ---------------------------------------------------------------------- */
 adadsf_status adadsf_router_scores(const adadsf_model_cfg *cfg, const adadsf_layer_weights *w,
                                    const void *x_dev, int64_t n_rows, float *scores_dev,
@@ -190,6 +194,27 @@ adadsf_status adadsf_router_scores(const adadsf_model_cfg *cfg, const adadsf_lay
  * ---------------------------------------------------------------------- */
 adadsf_status adadsf_topk_select(const float *scores_dev, int B, int T, int K,
                                  int32_t *idx_dev, int32_t *rows_dev, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Sec. 3.4: router scores of every token and the Top-K of each sequence in
+ * one call (the router kernel, then the Top-K kernel). x_dev [B*T, d]
+ * (cfg->dtype); scores_dev [B*T] fp32 receives the scores; idx_dev [B,K]
+ * int32 the kept positions of each sequence in ascending order; rows_dev
+ * [B,K] int32 (may be NULL) b*T + position. Same ranking as
+ * adadsf_topk_select; 1 <= K <= T <= 16384.
+ * ws: adadsf_router_select_workspace_size(cfg, B, T) bytes (the same for
+ * every B, T), zero-filled before first use. On the bf16 path the router
+ * splits 128-token tiles along d over several CTAs when there are few
+ * tiles: arrival counters sit in a fixed area right after the device error
+ * word (every completed call leaves them at zero, so one workspace serves
+ * calls of any shape, here and in the layer and model forwards), fp32
+ * partial tiles after it.
+ * ---------------------------------------------------------------------- */
+size_t adadsf_router_select_workspace_size(const adadsf_model_cfg *cfg, int B, int T);
+adadsf_status adadsf_router_select(const adadsf_model_cfg *cfg, const adadsf_layer_weights *w,
+                                   const void *x_dev, int B, int T, int K, float *scores_dev,
+                                   int32_t *idx_dev, int32_t *rows_dev, void *ws, size_t ws_bytes,
+                                   void *stream);
 
 /* ------------------------------------------------------------------------
  * Eq. 2 building block: out = act(x W^T + bias). x_dev [M, k_in],

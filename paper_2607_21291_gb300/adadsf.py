@@ -84,6 +84,8 @@ def lib() -> ctypes.CDLL:
             "adadsf_alloc_ratios": (i32, [vp, i32, f64, f64, f64, i32, u32, vp, vp]),
             "adadsf_router_scores": (i32, [pcfg, plw, vp, i64, vp, vp, sz, vp]),
             "adadsf_topk_select": (i32, [vp, i32, i32, i32, vp, vp, vp]),
+            "adadsf_router_select_workspace_size": (sz, [pcfg, i32, i32]),
+            "adadsf_router_select": (i32, [pcfg, plw, vp, i32, i32, i32, vp, vp, vp, vp, sz, vp]),
             "adadsf_linear": (i32, [vp, vp, vp, i64, i32, i32, i32, i32, vp, vp, sz, vp]),
             "adadsf_attention_workspace_size": (sz, [pcfg, i32, i32]),
             "adadsf_causal_attention": (i32, [pcfg, vp, i32, i32, vp, vp, sz, vp]),
@@ -235,6 +237,21 @@ def adadsf_topk_select(scores: torch.Tensor, K: int, idx: torch.Tensor,
     _dev(scores, "scores"); _dev(idx, "idx")
     B, T = scores.shape
     _check(lib().adadsf_topk_select(_p(scores), B, T, int(K), _p(idx), _p(rows), _s(stream)))
+
+
+def adadsf_router_select_workspace_size(cfg: ModelCfg, B: int, T: int) -> int:
+    return int(lib().adadsf_router_select_workspace_size(ctypes.byref(cfg), int(B), int(T)))
+
+
+def adadsf_router_select(cfg: ModelCfg, w: dict, x: torch.Tensor, B: int, T: int, K: int,
+                         scores: torch.Tensor, idx: torch.Tensor, rows: Optional[torch.Tensor] = None,
+                         ws: Optional[torch.Tensor] = None, stream=None):
+    _dev(x, "x"); _dev(scores, "scores"); _dev(idx, "idx")
+    if ws is None:
+        ws = workspace(adadsf_router_select_workspace_size(cfg, B, T), x.device)
+    lw = layer_struct(w)
+    _check(lib().adadsf_router_select(ctypes.byref(cfg), ctypes.byref(lw), _p(x), int(B), int(T), int(K),
+                                      _p(scores), _p(idx), _p(rows), _p(ws), ws.numel(), _s(stream)))
 
 
 def adadsf_linear(x: torch.Tensor, w: torch.Tensor, bias: Optional[torch.Tensor], out: torch.Tensor,

@@ -202,7 +202,7 @@ struct Carver {
 };
 
 struct LayerSlots {
-  size_t scores, idx, rows, n1, n2, qkv, vt, attn, ao, act, split;
+  size_t scores, idx, rows, n1, n2, qkv, vt, attn, ao, act, split, rsel;
 };
 
 void carve_layer(const adadsf_model_cfg* c, int B, int T, int K, Carver& cv, LayerSlots& s) {
@@ -222,6 +222,9 @@ void carve_layer(const adadsf_model_cfg* c, int B, int T, int K, Carver& cv, Lay
   s.act = cv.take(M * c->ffn * es);
   // fp32 partial tiles of projections split along K (tensor-core path)
   s.split = c->dtype == ADADSF_BF16 ? cv.take(gemm_split_scratch_bytes()) : 0;
+  // router partial tiles (tensor-core path; its counters sit in the
+  // workspace's synchronisation area)
+  s.rsel = c->dtype == ADADSF_BF16 ? cv.take(router_partial_bytes()) : 0;
 }
 
 size_t rope_bytes(const adadsf_model_cfg* c, int T) { return (size_t)T * (c->rotary_dim / 2) * 8; }
@@ -239,6 +242,8 @@ struct LayerBufs {
   const float2* rope;
   void *n1, *n2, *qkv, *vt, *attn, *ao, *act;
   float* split;   // null on the fp32 path
+  int* sync;       // the workspace's synchronisation area
+  float* rpart;    // router partial tiles, null on the fp32 path
 };
 
 adadsf_status run_linear(int dtype, const GemmArgs& g, const Dev& dev, const char* what) {
@@ -283,23 +288,17 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
   if (!dense) {
     const double rf = 2.0 * BT * c->router_hidden * d;
     const double rb = (double)BT * d * es + (double)c->router_hidden * d * es + BT * 4.0;
-    if (tc) {
-      GemmArgs g = linear_args(x, d, w->router_w1, BT, c->router_hidden, d);
-      g.epi.act = ACT_ROUTER;
-      g.epi.bias = w->router_b1;
-      g.epi.w2 = w->router_w2;
-      g.epi.b2 = w->router_b2;
-      g.epi.scores = lb.scores;
-      TRY(launch(dev, ADADSF_KERNEL_ROUTER, true, rf, rb, [&] { return run_linear(dt, g, dev, "router"); }));
-    } else {
-      TRY(launch(dev, ADADSF_KERNEL_ROUTER, false, rf, rb,
-                 CALL(router_f32(static_cast<const float*>(x), BT, d, c->router_hidden,
-                                 static_cast<const float*>(w->router_w1),
-                                 static_cast<const float*>(w->router_b1),
-                                 static_cast<const float*>(w->router_w2),
-                                 static_cast<const float*>(w->router_b2), lb.scores, dev),
-                      "router")));
-    }
+    // a2: router scores of every token (bf16: tensor cores, tiles split
+    // along d when there are few of them)
+    TRY(launch(dev, ADADSF_KERNEL_ROUTER, false, rf, rb,
+               CALL(tc ? router_tc(x, BT, d, w->router_w1, w->router_b1, w->router_w2, w->router_b2,
+                                   lb.scores, lb.sync, lb.rpart, dev)
+                       : router_f32(static_cast<const float*>(x), BT, d, c->router_hidden,
+                                    static_cast<const float*>(w->router_w1),
+                                    static_cast<const float*>(w->router_b1),
+                                    static_cast<const float*>(w->router_w2),
+                                    static_cast<const float*>(w->router_b2), lb.scores, dev),
+                    "router")));
     if (M <= 32LL * dev.num_sms) {
       // a3 + a4: Top-K of each sequence fused with the gather of the kept rows
       // and their norms (NeoX: LN1 and LN2 of the same row). Every block
@@ -497,6 +496,7 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
 size_t layer_ws_bytes(const adadsf_model_cfg* c, int B, int T, int K) {
   Carver cv;
   cv.take(kErrBytes);
+  cv.take(kSyncBytes);   // self-resetting counters (fixed place)
   cv.take(rope_bytes(c, T));
   LayerSlots s;
   carve_layer(c, B, T, K, cv, s);
@@ -513,6 +513,7 @@ void carve_model(const adadsf_model_cfg* c, int B, int T, int Kmax, bool stats, 
   const size_t es = elem_size(c->dtype);
   Carver cv;
   cv.take(kErrBytes);
+  cv.take(kSyncBytes);   // self-resetting counters (fixed place)
   m.x = cv.take((size_t)B * T * c->d * es);
   m.xin = stats ? cv.take((size_t)B * T * c->d * es) : 0;
   m.partials = stats ? cv.take((size_t)stats_partials_count((int64_t)B * T) * 3 * 8) : 0;
@@ -689,13 +690,14 @@ adadsf_status adadsf_router_scores(const adadsf_model_cfg* cfg, const adadsf_lay
   Dev dev;
   TRY(device_info(&dev, stream, ws));
   if (cfg->dtype == ADADSF_BF16) {
-    GemmArgs g = linear_args(x_dev, cfg->d, w->router_w1, n_rows, cfg->router_hidden, cfg->d);
-    g.epi.act = ACT_ROUTER;
-    g.epi.bias = w->router_b1;
-    g.epi.w2 = w->router_w2;
-    g.epi.b2 = w->router_b2;
-    g.epi.scores = scores_dev;
-    return run_linear(cfg->dtype, g, dev, "router");
+    // with room for them: counters (synchronisation area) and partial tiles
+    // for 128-token tiles split along d
+    const bool split = ws_bytes >= kErrBytes + kSyncBytes + router_partial_bytes();
+    CUDA_TRY(router_tc(x_dev, n_rows, cfg->d, w->router_w1, w->router_b1, w->router_w2, w->router_b2,
+                       scores_dev, split ? at<int>(ws, kErrBytes) : nullptr,
+                       split ? at<float>(ws, kErrBytes + kSyncBytes) : nullptr, dev),
+             "router");
+    return ADADSF_OK;
   }
   CUDA_TRY(router_f32(static_cast<const float*>(x_dev), n_rows, cfg->d, cfg->router_hidden,
                       static_cast<const float*>(w->router_w1), static_cast<const float*>(w->router_b1),
@@ -714,6 +716,48 @@ adadsf_status adadsf_topk_select(const float* scores_dev, int B, int T, int K, i
     return fail(ADADSF_ERR_INVALID_ARG, "idx_dev is NULL or misaligned");
   Dev dev;
   TRY(device_info(&dev, stream, nullptr));
+  CUDA_TRY(topk(scores_dev, B, T, K, idx_dev, rows_dev, dev), "top-k");
+  return ADADSF_OK;
+}
+
+size_t adadsf_router_select_workspace_size(const adadsf_model_cfg* cfg, int B, int T) {
+  if (check_cfg(cfg) != ADADSF_OK || check_shape(B, T, 0) != ADADSF_OK) return 0;
+  return kErrBytes + kSyncBytes + (cfg->dtype == ADADSF_BF16 ? align256(router_partial_bytes()) : 0);
+}
+
+adadsf_status adadsf_router_select(const adadsf_model_cfg* cfg, const adadsf_layer_weights* w,
+                                   const void* x_dev, int B, int T, int K, float* scores_dev,
+                                   int32_t* idx_dev, int32_t* rows_dev, void* ws, size_t ws_bytes,
+                                   void* stream) {
+  TRY(check_cfg(cfg));
+  if (!w) return fail(ADADSF_ERR_INVALID_ARG, "weights are NULL");
+  TRY(check_shape(B, T, K));
+  if (B == 0) return ADADSF_OK;
+  if (K < 1) return fail(ADADSF_ERR_INVALID_ARG, "K must be at least 1");
+  TRY(check_ws(ws, ws_bytes, adadsf_router_select_workspace_size(cfg, B, T)));
+  NEED_PTR(x_dev, "x_dev");
+  NEED_PTR(scores_dev, "scores_dev");
+  if (!idx_dev || (reinterpret_cast<uintptr_t>(idx_dev) & 3u))
+    return fail(ADADSF_ERR_INVALID_ARG, "idx_dev is NULL or misaligned");
+  if (rows_dev && (reinterpret_cast<uintptr_t>(rows_dev) & 3u))
+    return fail(ADADSF_ERR_INVALID_ARG, "rows_dev misaligned");
+  NEED_PTR(w->router_w1, "router_w1");
+  NEED_PTR(w->router_b1, "router_b1");
+  NEED_PTR(w->router_w2, "router_w2");
+  if (!w->router_b2) return fail(ADADSF_ERR_INVALID_ARG, "router_b2 is NULL");
+  Dev dev;
+  TRY(device_info(&dev, stream, ws));
+  const int64_t BT = (int64_t)B * T;
+  if (cfg->dtype == ADADSF_BF16)
+    CUDA_TRY(router_tc(x_dev, BT, cfg->d, w->router_w1, w->router_b1, w->router_w2, w->router_b2,
+                       scores_dev, at<int>(ws, kErrBytes), at<float>(ws, kErrBytes + kSyncBytes), dev),
+             "router");
+  else
+    CUDA_TRY(router_f32(static_cast<const float*>(x_dev), BT, cfg->d, cfg->router_hidden,
+                      static_cast<const float*>(w->router_w1), static_cast<const float*>(w->router_b1),
+                      static_cast<const float*>(w->router_w2), static_cast<const float*>(w->router_b2),
+                      scores_dev, dev),
+           "router");
   CUDA_TRY(topk(scores_dev, B, T, K, idx_dev, rows_dev, dev), "top-k");
   return ADADSF_OK;
 }
@@ -806,6 +850,7 @@ adadsf_status adadsf_sparse_layer_forward(const adadsf_model_cfg* cfg, const ada
   TRY(device_info(&dev, stream, ws));
   Carver cv;
   cv.take(kErrBytes);
+  cv.take(kSyncBytes);   // self-resetting counters (fixed place)
   const size_t rope_off = cv.take(rope_bytes(cfg, T));
   LayerSlots s;
   carve_layer(cfg, B, T, K, cv, s);
@@ -822,6 +867,8 @@ adadsf_status adadsf_sparse_layer_forward(const adadsf_model_cfg* cfg, const ada
   lb.ao = at<char>(ws, s.ao);
   lb.act = at<char>(ws, s.act);
   lb.split = s.split ? at<float>(ws, s.split) : nullptr;
+  lb.sync = at<int>(ws, kErrBytes);
+  lb.rpart = s.rsel ? at<float>(ws, s.rsel) : nullptr;
   if (cfg->rotary_dim > 0)
     TRY(launch(dev, ADADSF_KERNEL_ROPE_TABLE, false, 0, rope_bytes(cfg, T),
                CALL(rope_table(at<float2>(ws, rope_off), T, cfg->rotary_dim, cfg->rope_theta, dev),
@@ -882,6 +929,8 @@ adadsf_status adadsf_sparse_model_forward(const adadsf_model_cfg* cfg, const ada
   lb.ao = at<char>(ws, m.layer.ao);
   lb.act = at<char>(ws, m.layer.act);
   lb.split = m.layer.split ? at<float>(ws, m.layer.split) : nullptr;
+  lb.sync = at<int>(ws, kErrBytes);
+  lb.rpart = m.layer.rsel ? at<float>(ws, m.layer.rsel) : nullptr;
   const size_t xbytes = (size_t)B * T * cfg->d * es;
   int64_t idx_off = 0;
   for (int l = 0; l < cfg->n_layers; ++l) {

@@ -73,6 +73,12 @@ struct GemmArgs {
 // Scratch that lets gemm_bf16 split any small-M product along K.
 size_t gemm_split_scratch_bytes();
 
+// Every workspace that carries cross-CTA counters holds them in one area of
+// this size right after the device error word (offset 256), whatever the
+// shapes of the call: the kernels that count there leave the counters at
+// zero, so a workspace zero-filled once stays valid for calls of any shape.
+constexpr size_t kSyncBytes = 16384;
+
 struct Dev {
   cudaStream_t stream;
   int* err;          // device error word
@@ -119,6 +125,14 @@ cudaError_t router_f32(const float* x, int64_t n, int d, int h, const float* w1,
                        const float* w2, const float* b2, float* scores, const Dev& dev);
 cudaError_t topk(const float* scores, int B, int T, int K, int32_t* idx, int32_t* rows,
                  const Dev& dev);
+// router_tc.cu -- bf16 router on tcgen05: scores[r] = w2 . SiLU(W1 x[r] + b1) + b2
+// for r < rows. sync: the workspace's synchronisation area (kSyncBytes, zero
+// before the call and left at zero) and partials: router_partial_bytes() of
+// fp32 scratch, both needed to split 128-token tiles along d (either null:
+// no split).
+size_t router_partial_bytes();
+cudaError_t router_tc(const void* x, int64_t rows, int d, const void* w1, const void* b1, const void* w2,
+                      const void* b2, float* scores, int* sync, float* partials, const Dev& dev);
 // Top-K of each sequence's scores fused with gather_norm of the kept rows
 // (out rows b K + i, i-th kept position ascending); also writes idx / rows.
 cudaError_t select_gather_norm(int dtype, const float* scores, int B, int T, int K, const void* x,

@@ -8,6 +8,7 @@
 
 #include "common.cuh"
 #include "internal.h"
+#include "topk.cuh"
 
 namespace adadsf {
 namespace {
@@ -381,147 +382,8 @@ __global__ void router_f32_kernel(const float* x, int64_t n, int d, int h, const
 }
 
 // ---------------------------------------------------------------- Top-K (Sec. 3.4)
-// Order-preserving key of an fp32 score: larger score -> larger key; -0.0 is
-// folded onto +0.0; NaN maps to 0, below every number (-inf maps to 0x007FFFFF).
-__device__ __forceinline__ uint32_t score_key(float f) {
-  if (f != f) return 0u;
-  uint32_t u = __float_as_uint(f);
-  if ((u << 1) == 0u) u = 0u;   // -0.0 -> +0.0
-  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-}
-
-// Exclusive prefix sum over a block of NT threads of one int per thread;
-// also returns the block total. warp_tot: NT / 32 + 1 ints of shared memory.
-template <int NT>
-__device__ __forceinline__ int block_excl_scan(int v, int* warp_tot, int& total) {
-  constexpr int NW = NT / 32;
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  int incl = v;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int t = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += t;
-  }
-  if (lane == 31) warp_tot[w] = incl;
-  __syncthreads();
-  if (w == 0) {
-    int t = lane < NW ? warp_tot[lane] : 0;
-    int ti = t;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int u = __shfl_up_sync(0xffffffffu, ti, o);
-      if (lane >= o) ti += u;
-    }
-    if (lane < NW) warp_tot[lane] = ti - t;   // exclusive prefix of warp totals
-    if (lane == 31) warp_tot[NW] = ti;
-  }
-  __syncthreads();
-  const int res = warp_tot[w] + incl - v;
-  total = warp_tot[NW];
-  __syncthreads();
-  return res;
-}
-
-// Shared state of the block-wide Top-K.
-struct TopkShared {
-  int hist[2][256];     // alternate passes use alternate histograms
-  int warp_tot[33];
-  uint32_t digit[4];    // per pass, so no pass overwrites what another still reads
-  int remaining[4];
-};
-
-// Radix select over the T order-preserving keys in shared memory (4 passes
-// of 8 bits, most significant first): the K-th largest key `kth` and how many
-// keys equal to it are kept (need_eq, lowest positions first). K >= 1. Two
-// block barriers per pass: the next pass's histogram is cleared while this
-// pass's is filled.
-template <int NT>
-__device__ __forceinline__ void radix_select(const uint32_t* keys, int T, int K, TopkShared& sh,
-                                             uint32_t& kth, int& need_eq) {
-  uint32_t prefix = 0, pmask = 0;
-  int remaining = K;   // keys still to take at or below the current prefix
-  for (int i = threadIdx.x; i < 256; i += NT) sh.hist[0][i] = 0;
-  __syncthreads();
-  for (int pass = 0; pass < 4; ++pass) {
-    const int shift = 24 - 8 * pass;
-    int* hist = sh.hist[pass & 1];
-    for (int i = threadIdx.x; i < 256; i += NT) sh.hist[(pass + 1) & 1][i] = 0;
-    for (int t = threadIdx.x; t < T; t += NT) {
-      const uint32_t k = keys[t];
-      if ((k & pmask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1);
-    }
-    __syncthreads();
-    if (threadIdx.x < 32) {
-      // lane l owns digits 255-8l .. 248-8l (descending)
-      const int lane = threadIdx.x;
-      int cnt[8], lsum = 0;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        cnt[j] = hist[255 - 8 * lane - j];
-        lsum += cnt[j];
-      }
-      int incl = lsum;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int t = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += t;
-      }
-      const int excl = incl - lsum;   // keys with a larger digit than this lane's
-      const bool here = excl < remaining && incl >= remaining;
-      if (here) {
-        int above = excl;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          if (above + cnt[j] >= remaining) {
-            sh.digit[pass] = (uint32_t)(255 - 8 * lane - j);
-            sh.remaining[pass] = remaining - above;
-            break;
-          }
-          above += cnt[j];
-        }
-      }
-    }
-    __syncthreads();
-    prefix |= sh.digit[pass] << shift;
-    pmask |= 255u << shift;
-    remaining = sh.remaining[pass];
-  }
-  kth = prefix;
-  need_eq = remaining;
-}
-
-// Calls emit(i, t) for the kept positions t in ascending order, i = 0..K-1:
-// keys above kth, and the first need_eq keys equal to it. Each thread owns a
-// contiguous chunk of positions; one block scan of the packed counts
-// (above << 16 | equal; T <= 16384) places every chunk's output.
-template <int NT, typename Emit>
-__device__ __forceinline__ void emit_kept(const uint32_t* keys, int T, uint32_t kth, int need_eq,
-                                          TopkShared& sh, Emit emit) {
-  const int chunk = (T + NT - 1) / NT;
-  const int t0 = min(T, (int)threadIdx.x * chunk), t1 = min(T, t0 + chunk);
-  int n_gt = 0, n_eq = 0;
-  for (int t = t0; t < t1; ++t) {
-    n_gt += keys[t] > kth;
-    n_eq += keys[t] == kth;
-  }
-  int total;
-  const int base = block_excl_scan<NT>((n_gt << 16) | n_eq, sh.warp_tot, total);
-  const int eq_base = base & 0xffff;   // equal keys before my chunk
-  int out = (base >> 16) + min(eq_base, need_eq);
-  int er = eq_base;
-  for (int t = t0; t < t1; ++t) {
-    const uint32_t k = keys[t];
-    bool take = k > kth;
-    if (k == kth) {
-      take = er < need_eq;
-      ++er;
-    }
-    if (take) emit(out++, t);
-  }
-}
-
+// (radix select and emission: topk.cuh)
 constexpr int kTopkThreads = 1024;
-constexpr int kMaxTopkT = 16384;   // sequence length limit of the Top-K kernels
 
 // One block per sequence: idx[b][i] = i-th kept position (ascending), rows[b][i] = b T + position.
 __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const float* scores, int T, int K,
@@ -535,8 +397,9 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const float* scores,
   for (int t = threadIdx.x; t < T; t += kTopkThreads) keys[t] = score_key(sc[t]);
   uint32_t kth;
   int need_eq;
-  radix_select<kTopkThreads>(keys, T, K, sh, kth, need_eq);
-  emit_kept<kTopkThreads>(keys, T, kth, need_eq, sh, [&](int i, int t) {
+  const auto sync = [] { __syncthreads(); };
+  radix_select<kTopkThreads>(keys, T, K, sh, kth, need_eq, (int)threadIdx.x, sync);
+  emit_kept<kTopkThreads>(keys, T, kth, need_eq, sh, (int)threadIdx.x, sync, [&](int i, int t) {
     idx[(int64_t)b * K + i] = t;
     if (rows) rows[(int64_t)b * K + i] = b * T + t;
   });
@@ -567,8 +430,10 @@ __global__ void __launch_bounds__(kSelThreads)
   for (int t = threadIdx.x; t < Tlen; t += kSelThreads) keys[t] = score_key(sc[t]);
   uint32_t kth;
   int need_eq;
-  radix_select<kSelThreads>(keys, Tlen, K, sh, kth, need_eq);
-  emit_kept<kSelThreads>(keys, Tlen, kth, need_eq, sh, [&](int i, int t) { kept[i] = t; });
+  const auto sync = [] { __syncthreads(); };
+  radix_select<kSelThreads>(keys, Tlen, K, sh, kth, need_eq, (int)threadIdx.x, sync);
+  emit_kept<kSelThreads>(keys, Tlen, kth, need_eq, sh, (int)threadIdx.x, sync,
+                         [&](int i, int t) { kept[i] = t; });
   __syncthreads();
   const int lo = (int)((int64_t)g * K / G), hi = (int)((int64_t)(g + 1) * K / G);
   for (int i = lo + (int)threadIdx.x; i < hi; i += kSelThreads) {

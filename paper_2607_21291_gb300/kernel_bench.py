@@ -133,8 +133,15 @@ def case_router(a, stream):
     x = torch.randn(B * T, shape.d, generator=g, device="cuda").to(dt)
     scores = torch.empty(B * T, device="cuda", dtype=torch.float32)
     cfg = A.make_cfg(shape)
-    ws = A.workspace(256)
-    fn = lambda: A.adadsf_router_scores(cfg, w, x, scores, ws=ws, stream=stream)
+    if a.case == "router_select":
+        K = a.K if a.K is not None else T // 2
+        idx = torch.empty(B, K, device="cuda", dtype=torch.int32)
+        rows = torch.empty(B, K, device="cuda", dtype=torch.int32)
+        ws = A.workspace(A.adadsf_router_select_workspace_size(cfg, B, T))
+        fn = lambda: A.adadsf_router_select(cfg, w, x, B, T, K, scores, idx, rows, ws=ws, stream=stream)
+    else:
+        ws = A.workspace(A.adadsf_router_select_workspace_size(cfg, 1, 1))
+        fn = lambda: A.adadsf_router_scores(cfg, w, x, scores, ws=ws, stream=stream)
     flops = 2.0 * B * T * shape.d * shape.router_hidden
     return fn, flops, x.numel() * x.element_size(), ws
 
@@ -154,7 +161,7 @@ def case_topk(a, stream):
 
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
-    ap.add_argument("case", choices=("linear", "layer", "attention", "router", "topk"))
+    ap.add_argument("case", choices=("linear", "layer", "attention", "router", "router_select", "topk"))
     ap.add_argument("--M", type=int, default=8192)
     ap.add_argument("--N", type=int, default=8192)
     ap.add_argument("--K", type=int, default=None)
@@ -174,7 +181,8 @@ def main():
     stream = torch.cuda.Stream()
     with torch.cuda.stream(stream):
         fn, flops, nbytes, ws = {"linear": case_linear, "layer": case_layer, "attention": case_attention,
-                            "router": case_router, "topk": case_topk}[a.case](a, stream)
+                            "router": case_router, "router_select": case_router,
+                            "topk": case_topk}[a.case](a, stream)
         ms = _time(fn, a.iters, a.warmup, stream)
         out = {"case": a.case, "ms": ms}
         if flops:

@@ -96,4 +96,7 @@ def test_argument_errors_precede_launch(A):
     assert lib.adadsf_sparse_layer_forward(ctypes.byref(cfg), None, None, 2, 16, 8, None, None,
                                            None, 0, None) == A.ERR_INVALID_ARG
     assert lib.adadsf_linear(None, None, None, 4, 100, 64, A.BF16, 0, None, None, 0, None) == A.ERR_UNSUPPORTED
+    assert lib.adadsf_router_select(ctypes.byref(cfg), None, None, 2, 16, 4, None, None, None, None, 0,
+                                    None) == A.ERR_INVALID_ARG
+    assert lib.adadsf_router_select_workspace_size(ctypes.byref(cfg), 4, 512) > 256 + 4 * (16 + 4)
     assert lib.adadsf_layer_stats(None, None, 4, 64, A.BF16, 0, None, None, 0, None) == A.ERR_INVALID_ARG

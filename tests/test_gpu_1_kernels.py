@@ -10,6 +10,7 @@ from paper_2607_21291_gb300 import synth as S
 from tests import helpers as H
 
 pytestmark = pytest.mark.gpu
+SYNC_BYTES = 16384   # arrival counters right after the device error word
 
 
 @pytest.fixture(scope="module")
@@ -132,6 +133,68 @@ def test_router(A, shape, n):
     ref = O.router_scores(x.astype(np.float64), H.f64(W))
     err = np.max(np.abs(sc.cpu().numpy() - ref)) / np.max(np.abs(ref))
     assert err < (5e-3 if shape.dtype == "bf16" else 1e-5)
+
+
+@pytest.mark.parametrize("shape,n", [(S.PYTHIA_160M, 2048), (S.PYTHIA_1_4B, 16384), (S.QWEN25_1_5B, 999),
+                                     (S.QWEN25_7B.replace(ffn=256), 4096)])
+def test_router_split(A, shape, n):
+    """Router with room for scratch: 128-token tiles split along d over
+    several CTAs (partial tiles summed by the last CTA in a fixed order), so
+    two calls agree bit for bit and the tile counters end at zero."""
+    W = H.host_layer(shape, 3)
+    x = S.round_to(np.random.default_rng(n + 1).standard_normal((n, shape.d)).astype(np.float32), shape.dtype)
+    w = A.to_device(W, H.tdtype(shape))
+    cfg = A.make_cfg(shape)
+    ws = A.workspace(A.adadsf_router_select_workspace_size(cfg, 1, 1))
+    ref = O.router_scores(x.astype(np.float64), H.f64(W))
+    outs = []
+    for _ in range(2):
+        sc = torch.empty(n, dtype=torch.float32, device="cuda")
+        A.adadsf_router_scores(cfg, w, H.to_dev(x, H.tdtype(shape)), sc, ws=ws)
+        assert A.adadsf_sync_check(ws) == A.OK
+        err = np.max(np.abs(sc.cpu().numpy() - ref)) / np.max(np.abs(ref))
+        assert err < 5e-3
+        outs.append(sc)
+    assert torch.equal(outs[0], outs[1])
+    assert int(ws[256:256 + SYNC_BYTES].view(torch.int32).abs().sum()) == 0
+
+
+@pytest.mark.parametrize("shape,B,T,K", [(S.PYTHIA_160M, 4, 512, 256), (S.PYTHIA_1_4B, 8, 2048, 1024),
+                                         (S.QWEN25_1_5B, 3, 333, 100), (S.PYTHIA_160M, 2, 100, 1),
+                                         (S.PYTHIA_160M, 5, 64, 64), (S.PYTHIA_160M, 300, 1, 1),
+                                         (S.QWEN25_7B.replace(ffn=256), 2, 4096, 2000), (S.PYTHIA_160M, 1, 16384, 777)])
+def test_router_select(A, shape, B, T, K):
+    """Router scores and the per-sequence Top-K in one launch (Sec. 3.4):
+    scores within the router tolerance of the oracle, and the kept positions
+    bit-exact against the oracle's Top-K of the GPU's own scores; the
+    counters in the workspace end at zero, so a second call selects the same."""
+    W = H.host_layer(shape, 5)
+    g = np.random.default_rng(B * 1000 + T + K)
+    x = S.round_to(g.standard_normal((B * T, shape.d)).astype(np.float32), shape.dtype)
+    w = A.to_device(W, H.tdtype(shape))
+    cfg = A.make_cfg(shape)
+    ws = A.workspace(A.adadsf_router_select_workspace_size(cfg, B, T))
+    ref = O.router_scores(x.astype(np.float64), H.f64(W))
+    xd = H.to_dev(x, H.tdtype(shape))
+    first = None
+    for rep in range(2):
+        sc = torch.empty(B * T, dtype=torch.float32, device="cuda")
+        idx = torch.full((B, K), -1, dtype=torch.int32, device="cuda")
+        rows = torch.full((B, K), -1, dtype=torch.int32, device="cuda")
+        A.adadsf_router_select(cfg, w, xd, B, T, K, sc, idx, rows, ws=ws)
+        assert A.adadsf_sync_check(ws) == A.OK
+        s = sc.cpu().numpy()
+        assert np.max(np.abs(s - ref)) / np.max(np.abs(ref)) < 5e-3
+        gi, gr = idx.cpu().numpy(), rows.cpu().numpy()
+        for b in range(B):
+            kept = O.topk_keep(s[b * T:(b + 1) * T], K)
+            assert gi[b].tolist() == kept.tolist(), b
+            assert gr[b].tolist() == (b * T + kept).tolist(), b
+        if first is None:
+            first = (sc, idx)
+        else:
+            assert torch.equal(first[0], sc) and torch.equal(first[1], idx)
+    assert int(ws[256:256 + SYNC_BYTES].view(torch.int32).abs().sum()) == 0
 
 
 # ---------------------------------------------------------------- attention (Eq. 1)

@@ -135,6 +135,19 @@ def test_model_c2_end_to_end(A):
         off += B * k
     ref, _, _ = O.sparse_model_forward(ids, extra, hostL, p, K.tolist(), idx_force=kept)
     assert H.max_rel(H.to_np(hidden), ref) <= H.BF16_TOL
+    # one workspace for calls of different shapes (dense with statistics,
+    # then sparse, twice): the same results bit for bit as fresh workspaces
+    ws = A.workspace(A.adadsf_model_workspace_size(model.cfg, B, T, [T] * L, True))
+    acc = torch.zeros(2 * L, dtype=torch.float64, device="cuda")
+    h_cal = torch.empty((B, T, shape.d), dtype=torch.bfloat16, device="cuda")
+    for _ in range(2):
+        A.adadsf_sparse_model_forward(model, torch.from_numpy(ids_cal).cuda(), [T] * L, h_cal,
+                                      stats_acc=acc, ws=ws)
+        h2 = torch.empty_like(hidden)
+        idx2 = torch.empty_like(idx)
+        A.adadsf_sparse_model_forward(model, torch.from_numpy(ids).cuda(), K.tolist(), h2, idx_out=idx2, ws=ws)
+        assert A.adadsf_sync_check(ws) == A.OK
+        assert torch.equal(h2, hidden) and torch.equal(idx2, idx)
     # kept sets of every layer: rule 1 (oracle Top-K of the GPU scores) needs the
     # GPU scores, so re-run each layer on its oracle input teacher-forced.
     x = extra["embed"][ids]
