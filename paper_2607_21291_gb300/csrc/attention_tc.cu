@@ -1,25 +1,39 @@
 // Eq. 1 among the kept tokens on the 5th-generation tensor cores (bf16).
 //
-// One CTA per (128-query block, query head, sequence). Keys arrive in blocks
-// of 128; attention is causal in packed order (kept positions ascend, so this
-// is the original causal mask restricted to the kept set, Sec. 3.4).
-//   warp 0     TMA: the Q tile once, then the K tile of each key block into a
-//              2-stage ring released as soon as S of that block is done;
-//   warp 10    TMA: the V^T tile of each key block into a 2-stage ring
-//              released after P V (128-byte swizzled, K-major operands).
-//   warp 1     allocates TMEM; one thread issues S = Q K^T into a double-
-//              buffered TMEM S (tcgen05.mma, M = 128, N = 128) and, once the
-//              softmax warps have written P, O += P V into TMEM O (N = hd).
-//   warps 2-9  one query row and half of the key columns per thread (two
-//              warps per TMEM lane quarter, exchanging row maxima and sums
-//              through shared memory): read S from TMEM, mask, online
-//              softmax in fp32 (exp2 with a row maximum held at most 2^8
-//              below the true one, so O is rescaled only when the maximum
-//              grows by more than that), write P as bf16 into one of two
-//              swizzled operand tiles (so P of block j is written while
-//              P V of block j-1 runs), and at the end O / l -> global.
+// One CTA per (pair of 128-query blocks, query head, sequence): the two
+// query tiles share every K / V tile the CTA loads, which halves the K / V
+// traffic per flop, and their softmax work alternates with the other tile's
+// matrix products. Keys arrive in blocks of 128; attention is causal in
+// packed order (kept positions ascend, so this is the original causal mask
+// restricted to the kept set, Sec. 3.4).
+//   warp 0     TMA, lane 0: both Q tiles once, then the K tile of each key
+//              block into a ring released once both tiles' S of that block
+//              are done; lane 1: the V^T tile of each key block into a ring
+//              released after both tiles' P V (128-byte swizzled, K-major
+//              operands). The two lanes run their loops independently.
+//   warp 1     allocates TMEM; one thread issues, per tile t, S_t = Q_t K^T
+//              (tcgen05.mma, M = 128, N = 128) into TMEM S_t and, once the
+//              tile's softmax warps have written P_t over S_t (bf16 pairs),
+//              O_t += P_t V with P_t read from TMEM as the A operand. The
+//              order S_0(j) S_1(j) P_0V(j) S_0(j+1) P_1V(j) S_1(j+1) ... keeps
+//              the tensor pipe busy with one tile while the other's softmax
+//              runs; a tile's next S is issued after its P V, and the
+//              tensor-core pipe runs one thread's operations in order.
+//   warps 2-9  softmax of tile 0, warps 10-17 of tile 1: two warps per TMEM
+//              lane quarter, one query row and 64 of the 128 key columns per
+//              thread (the pair exchanges row maxima and sums through shared
+//              memory on a named barrier): read S once, mask (diagonal block
+//              only), online softmax in fp32 (exp2 with a row maximum held at
+//              most 2^8 below the true one, so O is rescaled only when the
+//              maximum grows by more than that), write P as bf16 pairs over
+//              the first 32 of its own 64 S columns (so neither warp of the
+//              pair overwrites scores the other has yet to read), and at the
+//              end O / l -> global.
+//              When S_t(j) is complete, P_t V of block j-1 is too (same pipe,
+//              issued earlier), so the rescale of O_t and the overwrite of
+//              P_t need no other wait.
 // V enters as V^T (features x keys per key-value head), written by the QKV
-// projection's epilogue, so both MMAs read K-major operands.
+// projection's epilogue.
 // Every barrier wait is bounded in time (device error word on give-up).
 #include <cuda.h>
 
@@ -29,24 +43,28 @@
 namespace adadsf {
 namespace {
 
-constexpr int kQB = 128;            // queries per CTA = TMEM lanes
+constexpr int kQB = 128;            // queries per tile = TMEM lanes
 constexpr int kKB = 128;            // keys per block
-constexpr int kSoftWarps = 8;       // two per TMEM lane quarter, each on 64 key columns
-constexpr int kVWarp = 2 + kSoftWarps;   // warp loading the V^T tiles
-constexpr int kAttnThreads = 32 * (kVWarp + 1);
+constexpr int kSoftWarps = 16;      // eight per tile, two per TMEM lane quarter
+constexpr int kAttnThreads = 32 * (2 + kSoftWarps);
 constexpr float kRescaleLog2 = 8.f; // O rescaled only when the row max grows by > 2^8
 
 template <int HD>
 struct AttnCfg {
+  static constexpr int KST = HD == 64 ? 4 : 3;     // K ring stages
+  static constexpr int VST = HD == 64 ? 4 : 2;     // V^T ring stages
   static constexpr int HS = HD / 64;               // 64-feature slabs of a head row
   static constexpr int SLAB = kQB * 128;           // one 128-row x 128-byte slab
-  static constexpr int Q_BYTES = HS * SLAB;
+  static constexpr int Q_BYTES = HS * SLAB;        // one query tile
   static constexpr int K_BYTES = HS * SLAB;
   static constexpr int V_SLAB = HD * 128;          // HD feature rows x 64 keys
   static constexpr int V_BYTES = 2 * V_SLAB;       // 128 keys
-  static constexpr int P_BYTES = 2 * SLAB;         // 128 queries x 128 keys
-  static constexpr int DATA = Q_BYTES + 2 * K_BYTES + 2 * V_BYTES + 2 * P_BYTES;   // P double-buffered
-  static constexpr int TAIL = 256 + 2048;         // barriers, then the softmax exchange area
+  static constexpr int DATA = 2 * Q_BYTES + KST * K_BYTES + VST * V_BYTES;
+  static constexpr int NBARS = 1 + 2 * KST + 2 * VST + 7;
+  // barriers, TMEM address, abort flag; then the softmax pairs' exchange
+  // area: [tile][quarter][half][lane] floats
+  static constexpr int XCHG = 2 * 4 * 2 * 32 * 4;
+  static constexpr int TAIL = 256 + XCHG;
   // Room left for aligning the dynamic base to 1024 bytes (the kernel checks
   // its actual misalignment); padded so that one CTA holds an SM (TMEM is
   // allocated in full).
@@ -54,6 +72,11 @@ struct AttnCfg {
   static constexpr int SMEM_RAW = DATA + TAIL + SLACK;
   static constexpr int SMEM = SMEM_RAW > 120 * 1024 ? SMEM_RAW : 120 * 1024;
   static_assert(SLACK >= 256, "shared memory");
+  static_assert(NBARS * 8 + 8 <= TAIL, "barrier area");
+  // TMEM: S_0 (P_0 over its first 64 columns) at 0, S_1 at 128, O_0 at 256,
+  // O_1 at 256 + HD
+  static constexpr uint32_t TS = 0, TO = 256;
+  static_assert(TO + 2 * HD <= 512, "TMEM columns");
 };
 
 // 2^x on the SFU (ex2.approx.ftz.f32: relative error ~2^-22, flushes
@@ -79,6 +102,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQK, const __grid_constant__ CUtensorMap tmVt,
                    const AttnDev p) {
   using C = AttnCfg<HD>;
+  constexpr int KST = C::KST, VST = C::VST;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -86,52 +110,53 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     if (threadIdx.x == 0) set_device_error(p.err, DEVERR_TIMEOUT);
     return;
   }
-  const uint32_t sQ = smem_u32(smem);
-  const uint32_t sK0 = sQ + C::Q_BYTES;
-  const uint32_t sV0 = sK0 + 2 * C::K_BYTES;
-  const uint32_t sP0 = sV0 + 2 * C::V_BYTES;       // [2]
-  uint8_t* sP_ptr = smem + (sP0 - sQ);
+  const uint32_t sQ = smem_u32(smem);                  // [2] query tiles
+  const uint32_t sK0 = sQ + 2 * C::Q_BYTES;
+  const uint32_t sV0 = sK0 + KST * C::K_BYTES;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::DATA);
   const uint32_t b0 = smem_u32(bars);
   const uint32_t q_full = b0;
-  const uint32_t k_full0 = b0 + 8;       // [2] K ring: free once S of the block is done
-  const uint32_t k_empty0 = b0 + 24;     // [2]
-  const uint32_t s_full0 = b0 + 40;      // [2]
-  const uint32_t s_free0 = b0 + 56;      // [2]
-  const uint32_t p_full0 = b0 + 72;      // [2] per P buffer
-  const uint32_t pv_done0 = b0 + 88;     // [2] per P buffer
-  const uint32_t drain = b0 + 104;
-  const uint32_t pair0 = b0 + 112;       // [4] the two softmax warps of a lane quarter
-  const uint32_t v_full0 = b0 + 144;     // [2] V^T ring: free once P V of the block is done
-  const uint32_t v_empty0 = b0 + 160;    // [2]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 22);
+  const uint32_t k_full0 = b0 + 8;                 // [KST]
+  const uint32_t k_empty0 = k_full0 + 8 * KST;     // [KST]
+  const uint32_t v_full0 = k_empty0 + 8 * KST;     // [VST]
+  const uint32_t v_empty0 = v_full0 + 8 * VST;     // [VST]
+  const uint32_t s_full0 = v_empty0 + 8 * VST;     // [2] per tile: S_t of the block done
+  const uint32_t p_full0 = s_full0 + 16;           // [2] per tile: P_t written (8 warps)
+  const uint32_t o_done0 = p_full0 + 16;           // [2] per tile: P_t V of the block done
+  const uint32_t drain = o_done0 + 16;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::NBARS);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  // per quarter, per exchange slot (2), per half: one float per lane
-  float* xchg = reinterpret_cast<float*>(smem + C::DATA + 256);
+  // softmax pairs' exchange: [tile][quarter][half][lane]
+  volatile float* xchg = reinterpret_cast<volatile float*>(smem + C::DATA + 256);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int nqb = (p.K + kQB - 1) / kQB;
-  const int qb = nqb - 1 - (int)blockIdx.x;   // longest rows first
+  const int npair = (nqb + 1) / 2;
+  const int pr = npair - 1 - (int)blockIdx.x;   // longest rows first
+  const int qb0 = 2 * pr;
+  const bool two = qb0 + 1 < nqb;               // tile 1 holds query block qb0 + 1
+  const int n_kv = two ? qb0 + 2 : qb0 + 1;     // tile 0 takes blocks 0..qb0, tile 1 all
   const int h = blockIdx.y, b = blockIdx.z;
   const int g = h / (p.Hq / p.Hkv);
-  const int n_kv = qb + 1;
   const int row0 = b * p.K;
 
   pdl_trigger();
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < KST; ++i) {
       mbar_init(k_full0 + 8 * i, 1);
       mbar_init(k_empty0 + 8 * i, 1);
+    }
+    for (int i = 0; i < VST; ++i) {
       mbar_init(v_full0 + 8 * i, 1);
       mbar_init(v_empty0 + 8 * i, 1);
-      mbar_init(s_full0 + 8 * i, 1);
-      mbar_init(s_free0 + 8 * i, kSoftWarps);
-      mbar_init(p_full0 + 8 * i, kSoftWarps);
-      mbar_init(pv_done0 + 8 * i, 1);
     }
-    for (int i = 0; i < 4; ++i) mbar_init(pair0 + 8 * i, 2);
+    for (int t = 0; t < 2; ++t) {
+      mbar_init(s_full0 + 8 * t, 1);
+      mbar_init(p_full0 + 8 * t, 8);
+      mbar_init(o_done0 + 8 * t, 1);
+    }
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -147,26 +172,27 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const uint32_t tS = tmem_base;          // S buffers at columns 0 and 128
-  const uint32_t tO = tmem_base + 256;    // O at columns 256 .. 256 + HD
 
-  if (warp == 0 || warp == kVWarp) {
+  if (warp == 0) {
     // ------------------------------------------------------------ TMA producers
-    // warp 0: Q once, then the K ring; warp kVWarp: the V^T ring
-    if (lane == 0) {
-      const bool kprod = warp == 0;
+    // lane 0: both Q tiles once, then the K ring; lane 1: the V^T ring
+    if (lane < 2) {
+      const bool kprod = lane == 0;
+      const int NST = kprod ? KST : VST;
       pdl_wait();
       if (kprod) {
-        mbar_arrive_expect_tx(q_full, C::Q_BYTES);
-        for (int s = 0; s < C::HS; ++s)
-          tma_load_2d(sQ + s * C::SLAB, &tmQK, h * HD + s * 64, row0 + qb * kQB, q_full);
+        mbar_arrive_expect_tx(q_full, (two ? 2 : 1) * C::Q_BYTES);
+        for (int t = 0; t < (two ? 2 : 1); ++t)
+          for (int s = 0; s < C::HS; ++s)
+            tma_load_2d(sQ + t * C::Q_BYTES + s * C::SLAB, &tmQK, h * HD + s * 64,
+                        row0 + (qb0 + t) * kQB, q_full);
       }
       const uint32_t full0 = kprod ? k_full0 : v_full0;
       const uint32_t empty0 = kprod ? k_empty0 : v_empty0;
       int issued = 0;
       for (int j = 0; j < n_kv; ++j) {
-        const int st = j & 1;
-        if (!mbar_wait_bounded(empty0 + 8 * st, ((j >> 1) & 1) ^ 1, abort_flag, p.err, p.timeout_ns))
+        const int st = j % NST;
+        if (!mbar_wait_bounded(empty0 + 8 * st, ((j / NST) & 1) ^ 1, abort_flag, p.err, p.timeout_ns))
           break;
         const uint32_t fb = full0 + 8 * st;
         if (kprod) {
@@ -184,9 +210,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       }
       // drain: the copies issued last into each stage have landed
       if (kprod) mbar_wait_drain(q_full, 0, p.timeout_ns);
-      for (int st = 0; st < 2 && st < issued; ++st) {
-        const int last = st + ((issued - 1 - st) / 2) * 2;
-        mbar_wait_drain(full0 + 8 * st, (uint32_t)((last >> 1) & 1), p.timeout_ns);
+      for (int st = 0; st < NST && st < issued; ++st) {
+        const int last = st + ((issued - 1 - st) / NST) * NST;
+        mbar_wait_drain(full0 + 8 * st, (uint32_t)((last / NST) & 1), p.timeout_ns);
       }
     }
   } else if (warp == 1) {
@@ -194,198 +220,193 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     if (lane == 0) {
       constexpr uint32_t idesc_s = idesc_bf16_f32(kQB, kKB);
       constexpr uint32_t idesc_o = idesc_bf16_f32(kQB, HD);
-      bool ok = mbar_wait_bounded(q_full, 0, abort_flag, p.err, p.timeout_ns);
-      for (int j = 0; ok && j <= n_kv; ++j) {
-        if (j < n_kv) {
-          const int st = j & 1;
-          if (!mbar_wait_bounded(k_full0 + 8 * st, (j >> 1) & 1, abort_flag, p.err, p.timeout_ns) ||
-              (j >= 2 && !mbar_wait_bounded(s_free0 + 8 * st, ((j >> 1) - 1) & 1, abort_flag, p.err,
-                                            p.timeout_ns))) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t kst = sK0 + st * C::K_BYTES;
+      // S_t(j) = Q_t K(j)^T into TMEM S_t
+      auto issue_s = [&](int t, int j) {
+        const uint32_t kst = sK0 + (j % KST) * C::K_BYTES;
+        const uint32_t qt = sQ + t * C::Q_BYTES;
 #pragma unroll
-          for (int kk = 0; kk < HD / 16; ++kk) {
-            const uint32_t off = (kk >> 2) * C::SLAB + (kk & 3) * 32;
-            tc_mma_f16(tS + st * kKB, smem_desc_sw128(sQ + off), smem_desc_sw128(kst + off), idesc_s,
-                       kk > 0 ? 1u : 0u);
-          }
-          tc_commit(s_full0 + 8 * st);
-          tc_commit(k_empty0 + 8 * st);   // K tile consumed
+        for (int kk = 0; kk < HD / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * C::SLAB + (kk & 3) * 32;
+          tc_mma_f16(tmem_base + C::TS + t * kKB, smem_desc_sw128(qt + off), smem_desc_sw128(kst + off),
+                     idesc_s, kk > 0 ? 1u : 0u);
         }
-        if (j >= 1) {
-          const int jj = j - 1, pb = jj & 1;   // V^T stage and P buffer of block jj
-          if (!mbar_wait_bounded(p_full0 + 8 * pb, (jj >> 1) & 1, abort_flag, p.err, p.timeout_ns) ||
-              !mbar_wait_bounded(v_full0 + 8 * pb, (jj >> 1) & 1, abort_flag, p.err, p.timeout_ns)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t vst = sV0 + pb * C::V_BYTES;
-          const uint32_t pst = sP0 + pb * C::P_BYTES;
+        tc_commit(s_full0 + 8 * t);
+      };
+      // O_t += P_t(j) V(j), P_t read from TMEM
+      auto issue_pv = [&](int t, int j) {
+        const uint32_t vst = sV0 + (j % VST) * C::V_BYTES;
 #pragma unroll
-          for (int kk = 0; kk < kKB / 16; ++kk) {
-            tc_mma_f16(tO, smem_desc_sw128(pst + (kk >> 2) * C::SLAB + (kk & 3) * 32),
-                       smem_desc_sw128(vst + (kk >> 2) * C::V_SLAB + (kk & 3) * 32), idesc_o,
-                       (jj > 0 || kk > 0) ? 1u : 0u);
-          }
-          tc_commit(pv_done0 + 8 * pb);
-          tc_commit(v_empty0 + 8 * pb);
+        for (int kk = 0; kk < kKB / 16; ++kk)   // keys 16 kk.. of P_t: columns 64 (kk / 4) + 8 (kk % 4)
+          tc_mma_f16_ta(tmem_base + C::TO + t * HD, tmem_base + C::TS + t * kKB + (kk >> 2) * 64 + (kk & 3) * 8,
+                        smem_desc_sw128(vst + (kk >> 2) * C::V_SLAB + (kk & 3) * 32), idesc_o,
+                        (j > 0 || kk > 0) ? 1u : 0u);
+        tc_commit(o_done0 + 8 * t);
+      };
+      auto wait = [&](uint32_t bar, uint32_t parity) {
+        return mbar_wait_bounded(bar, parity, abort_flag, p.err, p.timeout_ns);
+      };
+      const int last0 = qb0;   // tile 0's last key block
+      bool ok = wait(q_full, 0) && wait(k_full0, 0);
+      if (ok) {
+        tc_fence_after();
+        issue_s(0, 0);
+        if (two) issue_s(1, 0);
+        tc_commit(k_empty0);
+      }
+      for (int j = 0; ok && j < n_kv; ++j) {
+        const bool has0 = j <= last0;
+        const bool next = j + 1 < n_kv;
+        if (!wait(v_full0 + 8 * (j % VST), (j / VST) & 1)) { ok = false; break; }
+        if (has0) {
+          if (!wait(p_full0, j & 1)) { ok = false; break; }
+          tc_fence_after();
+          issue_pv(0, j);
         }
+        if (next && !wait(k_full0 + 8 * ((j + 1) % KST), ((j + 1) / KST) & 1)) { ok = false; break; }
+        tc_fence_after();
+        if (next && j + 1 <= last0) issue_s(0, j + 1);
+        if (two) {
+          if (!wait(p_full0 + 8, j & 1)) { ok = false; break; }
+          tc_fence_after();
+          issue_pv(1, j);
+          if (next) issue_s(1, j + 1);
+        }
+        tc_commit(v_empty0 + 8 * (j % VST));            // V(j) read by both tiles
+        if (next) tc_commit(k_empty0 + 8 * ((j + 1) % KST));   // K(j+1) read by both tiles
       }
       tc_commit(drain);
       mbar_wait_drain(drain, 0, p.timeout_ns);
     }
   } else {
-    // ------------------------------------------------------------ softmax (warps 2..9)
+    // ------------------------------------------------------------ softmax (warps 2..17)
     pdl_wait();
+    const int t = (warp - 2) >> 3;                 // tile
+    const int half = ((warp - 2) >> 2) & 1;        // key columns [64 half, 64 half + 64)
     const int quarter = warp & 3;
-    const int half = (warp - 2) >> 2;              // key columns [64 half, 64 half + 64)
-    const int r = quarter * 32 + lane;             // query row in the block = TMEM lane
-    const int qi = qb * kQB + r;                   // query index in the sequence
+    const int r = quarter * 32 + lane;             // query row in the tile = TMEM lane
+    const int qbt = qb0 + t;
+    const int qi = qbt * kQB + r;                  // query index in the sequence
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
-    const uint32_t pairbar = pair0 + 8 * quarter;
-    uint32_t xk = 0;                               // exchanges done with the partner warp
-    // value of the partner warp (same rows, other half) for this exchange
-    auto exchange = [&](float mine, float* theirs) -> bool {
-      float* slot = xchg + ((quarter * 2 + (xk & 1)) * 2) * 32;
-      slot[half * 32 + lane] = mine;
-      __syncwarp();
-      int w = 1;
-      if (lane == 0) {
-        mbar_arrive(pairbar);
-        w = mbar_wait_bounded(pairbar, xk & 1, abort_flag, p.err, p.timeout_ns);
-      }
-      ++xk;
-      if (!__shfl_sync(0xffffffffu, w, 0)) return false;
-      *theirs = slot[(half ^ 1) * 32 + lane];
-      return true;
+    const uint32_t tS = tmem_base + C::TS + t * kKB + lane_off;
+    const uint32_t tO = tmem_base + C::TO + t * HD + lane_off + half * (HD / 2);
+    const bool active = t == 0 || two;
+    const int bar_id = 1 + t * 4 + quarter;        // named barrier of the warp pair
+    volatile float* xq = xchg + (t * 4 + quarter) * 64;
+    // partner's value (same rows, other half of the columns); the second
+    // barrier lets the next exchange reuse the slots
+    auto exchange = [&](float mine) {
+      xq[half * 32 + lane] = mine;
+      named_bar_sync(bar_id, 64);
+      const float theirs = xq[(half ^ 1) * 32 + lane];
+      named_bar_sync(bar_id, 64);
+      return theirs;
     };
     float m_used = -INFINITY, l = 0.f;
-    bool ok = true;
-    for (int j = 0; j < n_kv && ok; ++j) {
-      const int st = j & 1;
+    bool ok = active;
+    for (int j = 0; ok && j <= qbt; ++j) {
       int w = 0;
-      if (lane == 0) w = mbar_wait_bounded(s_full0 + 8 * st, (j >> 1) & 1, abort_flag, p.err, p.timeout_ns);
-      if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
+      if (lane == 0) w = mbar_wait_bounded(s_full0 + 8 * t, j & 1, abort_flag, p.err, p.timeout_ns);
+      w = __shfl_sync(0xffffffffu, w, 0);
       tc_fence_after();
-      const uint32_t s_row = tS + lane_off + st * kKB + half * 64;
+      const uint32_t tSh = tS + half * 64;         // this half's 64 score columns
       // keys above lim (relative to this half) are masked: diagonal block only
-      const int lim = (j == qb) ? qi - j * kKB - half * 64 : kKB;
-      // pass 1: row maximum of the raw scores (scale > 0) over both halves
+      const bool diag = j == qbt;
+      const int lim = diag ? qi - j * kKB - half * 64 : kKB;
       float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll 1
-      for (int c = 0; c < 2; ++c) {
-        uint32_t u[32];
-        tmem_ld32(s_row + c * 32, u);
+      if (w) {
+        uint32_t u[64];
+        tmem_ld32(tSh, u);
+        tmem_ld32(tSh + 32, u + 32);
         tmem_ld_wait();
+        if (diag) {
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const float v = (c * 32 + i <= lim) ? __uint_as_float(u[i]) : -INFINITY;
-          mx[i & 3] = fmaxf(mx[i & 3], v);
+          for (int i = 0; i < 64; ++i) mx[i & 3] = fmaxf(mx[i & 3], (i <= lim) ? __uint_as_float(u[i]) : -INFINITY);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 64; ++i) mx[i & 3] = fmaxf(mx[i & 3], __uint_as_float(u[i]));
         }
       }
-      float part = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])), other;
-      if (!exchange(part, &other)) { ok = false; break; }
+      // a wait that gave up travels as NaN, so the pair leaves together (the
+      // exchange is a barrier of both warps)
+      const float part = w ? fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) : NAN;
+      const float other = exchange(part);
+      if (part != part || other != other) { ok = false; break; }
       const float bmax = fmaxf(part, other) * p.scale_log2;
       bool need = false;
       if (j == 0) m_used = bmax;
       else need = bmax > m_used + kRescaleLog2;
-      const int pb = j & 1;
-      // P buffer pb is free once P V of block j - 2 has completed
-      if (j >= 2) {
-        int w2 = 0;
-        if (lane == 0)
-          w2 = mbar_wait_bounded(pv_done0 + 8 * pb, ((j >> 1) - 1) & 1, abort_flag, p.err, p.timeout_ns);
-        if (!__shfl_sync(0xffffffffu, w2, 0)) { ok = false; break; }
-      }
       if (__any_sync(0xffffffffu, need)) {
-        // O is stable once P V of block j - 1 has completed; each half
-        // rescales its half of the O columns
-        int w3 = 0;
-        if (lane == 0)
-          w3 = mbar_wait_bounded(pv_done0 + 8 * (pb ^ 1), ((j - 1) >> 1) & 1, abort_flag, p.err,
-                                 p.timeout_ns);
-        if (!__shfl_sync(0xffffffffu, w3, 0)) { ok = false; break; }
+        // O_t is stable: P_t V of block j - 1 completed before S_t(j)
         const float alpha = need ? ex2_approx(m_used - bmax) : 1.f;
         if (need) {
           l *= alpha;
           m_used = bmax;
         }
-        tc_fence_after();
 #pragma unroll 1
         for (int c = 0; c < HD / 64; ++c) {
-          const uint32_t ta = tO + lane_off + half * (HD / 2) + c * 32;
-          uint32_t u[32];
-          tmem_ld32(ta, u);
+          uint32_t o[32];
+          tmem_ld32(tO + c * 32, o);
           tmem_ld_wait();
 #pragma unroll
-          for (int i = 0; i < 32; ++i) u[i] = __float_as_uint(__uint_as_float(u[i]) * alpha);
-          tmem_st32(ta, u);
+          for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+          tmem_st32(tO + c * 32, o);
         }
-        tmem_st_wait();
       }
-      // pass 2: p = 2^(s * scale - m_used), partial row sum, this half's 64
-      // keys of P row r as bf16 into slab `half` (16-byte chunks XOR-swizzled)
-      uint8_t* prow = sP_ptr + pb * C::P_BYTES + half * C::SLAB + r * 128;
+      // p = 2^(s * scale - m_used) as bf16 pairs over the first 32 of this
+      // half's columns (chunk c's 32 scores are read before P of chunk c
+      // covers columns 16 c .. 16 c + 15, whose scores are already used);
+      // row sum in fp32
       float sm[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll 1
+#pragma unroll
       for (int c = 0; c < 2; ++c) {
-        uint32_t u[32];
-        tmem_ld32(s_row + c * 32, u);
+        uint32_t u[32], pk[16];
+        tmem_ld32(tSh + 32 * c, u);
         tmem_ld_wait();
-        float e[32];
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const float t = ex2_approx(fmaf(__uint_as_float(u[i]), p.scale_log2, -m_used));
-          e[i] = (c * 32 + i <= lim) ? t : 0.f;
-          sm[i & 3] += e[i];
+        for (int i = 0; i < 16; ++i) {
+          const int k0 = 32 * c + 2 * i;
+          float e0 = ex2_approx(fmaf(__uint_as_float(u[2 * i]), p.scale_log2, -m_used));
+          float e1 = ex2_approx(fmaf(__uint_as_float(u[2 * i + 1]), p.scale_log2, -m_used));
+          if (diag) {
+            e0 = (k0 <= lim) ? e0 : 0.f;
+            e1 = (k0 + 1 <= lim) ? e1 : 0.f;
+          }
+          sm[k0 & 3] += e0;
+          sm[(k0 + 1) & 3] += e1;
+          pk[i] = pack_bf16x2(e0, e1);
         }
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const int ch = c * 4 + k;
-          const float* q = e + 8 * k;
-          *reinterpret_cast<uint4*>(prow + ((ch ^ (r & 7)) << 4)) =
-              make_uint4(pack_bf16x2(q[0], q[1]), pack_bf16x2(q[2], q[3]), pack_bf16x2(q[4], q[5]),
-                         pack_bf16x2(q[6], q[7]));
-        }
+        tmem_st16(tSh + 16 * c, pk);
       }
+      tmem_st_wait();
       l += (sm[0] + sm[1]) + (sm[2] + sm[3]);
-      fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(s_free0 + 8 * st);   // S buffer may be overwritten
-        mbar_arrive(p_full0 + 8 * pb);
+      if (lane == 0) mbar_arrive(p_full0 + 8 * t);
+    }
+    // epilogue: O_t / l (both halves' sums) once the tile's last P V is done
+    if (active) {
+      const float l_all = l + exchange(l);
+      if (ok) {
+        int w = 0;
+        if (lane == 0) w = mbar_wait_bounded(o_done0 + 8 * t, qbt & 1, abort_flag, p.err, p.timeout_ns);
+        ok = __shfl_sync(0xffffffffu, w, 0) != 0;
       }
-    }
-    // epilogue: O / (l of both halves); each half stores its HD/2 columns
-    float l_other = 0.f;
-    if (ok) ok = exchange(l, &l_other);
-    if (ok) {
-      int w = 0;
-      if (lane == 0)
-        w = mbar_wait_bounded(pv_done0 + 8 * ((n_kv - 1) & 1), ((n_kv - 1) >> 1) & 1, abort_flag, p.err,
-                              p.timeout_ns);
-      ok = __shfl_sync(0xffffffffu, w, 0) != 0;
-    }
-    if (ok) {
-      tc_fence_after();
-      const float inv = 1.f / (l + l_other);
-      bf16* dst = p.out + (int64_t)(row0 + qi) * p.ld_out + (int64_t)h * HD + half * (HD / 2);
+      if (ok) {
+        tc_fence_after();
+        const float inv = 1.f / l_all;
+        bf16* dst = p.out + (int64_t)(row0 + qi) * p.ld_out + (int64_t)h * HD + half * (HD / 2);
 #pragma unroll 1
-      for (int c = 0; c < HD / 64; ++c) {
-        uint32_t u[32];
-        tmem_ld32(tO + lane_off + half * (HD / 2) + c * 32, u);
-        tmem_ld_wait();
-        if (qi < p.K) {
-          float v[32];
+        for (int c = 0; c < HD / 64; ++c) {
+          uint32_t o[32];
+          tmem_ld32(tO + c * 32, o);
+          tmem_ld_wait();
+          if (qi < p.K) {
+            float v[32];
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(u[i]) * inv;
+            for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(o[i]) * inv;
 #pragma unroll
-          for (int i = 0; i < 4; ++i) store_vec(dst + c * 32 + 8 * i, v + 8 * i);
+            for (int i = 0; i < 4; ++i) store_vec(dst + c * 32 + 8 * i, v + 8 * i);
+          }
         }
       }
     }
@@ -448,7 +469,7 @@ cudaError_t launch_attn(const void* qkv, int64_t ld_qkv, const void* vt, int pad
   p.ld_out = ld_out;
   p.err = dev.err;
   p.timeout_ns = kWaitTimeoutNs;
-  dim3 grid((K + kQB - 1) / kQB, Hq, B);
+  dim3 grid(((K + kQB - 1) / kQB + 1) / 2, Hq, B);
   return launch_pdl(attn_tc_kernel<HD>, grid, dim3(kAttnThreads), C::SMEM, dev.stream, tq, tv, p);
 }
 

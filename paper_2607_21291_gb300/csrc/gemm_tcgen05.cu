@@ -3,7 +3,7 @@
 // out = epilogue(A . W^T) with A [M, K] (packed kept tokens, row-major) and
 // W [N, K] (nn.Linear layout); both operands are K-major, which is the layout
 // tcgen05 reads natively. These are the dense contractions of Eqs. 1-2 (QKV,
-// output and MLP projections) and the router's first linear layer (Sec. 3.4).
+// output and MLP projections).
 //
 // Kernel structure (one CTA per SM, 10 warps):
 //   warp 0     TMA producer: 128x64 A tile and BNx64 W tile(s) per stage into a
@@ -14,9 +14,9 @@
 //              accumulator hand-offs to mbarriers.
 //   warps 2-9  epilogue: tcgen05.ld the accumulator (one row per thread, two
 //              warps per 32-lane TMEM quarter splitting the columns), apply
-//              bias / GELU / SwiGLU / rotary / residual / row scatter / router
-//              reduction in fp32, round once and store. Per-column constants
-//              (biases, the router's second layer) are staged in shared memory
+//              bias / GELU / SwiGLU / rotary / residual / row scatter in
+//              fp32, round once and store. Per-column constants (biases) are
+//              staged in shared memory
 //              and the first residual chunks loaded into registers before the
 //              accumulator is ready, so their latency hides under the K loop.
 //              GELU uses an erf with one exponential and no division (the
@@ -93,7 +93,6 @@ struct GemmDev {
   const int32_t* rows;
   int out_mapped;
   bf16* out; int64_t ld_out;
-  const bf16* w2; const bf16* b2; float* scores;
   // rotary embedding fused into the QKV epilogue (rope_tab == nullptr: off)
   const float2* rope_tab;    // [T][rope_half] (cos, sin)
   const int32_t* rope_pos;   // [M] original positions, or null: m % rope_T
@@ -193,35 +192,22 @@ __device__ __forceinline__ void ld_shared_f4(uint32_t addr, float* f) {
 
 // Per-column constants of a tile, staged by each epilogue warp in its own
 // shared-memory slot (no cross-warp barrier): sc[j] = bias[n] + bias2[n] for
-// the tile's columns n = nb BN + j; the router stages sc[j] = bias[j] and
-// sc[64 + j] = w2[j]. Each lane moves 16 bytes at a time.
-template <bool ROUTER>
+// the tile's columns n = nb BN + j. Each lane moves 16 bytes at a time.
 __device__ __forceinline__ void stage_consts(const GemmDev& p, int nb, int bn, uint32_t sc, int lane) {
-  if (ROUTER) {   // bn == 64
-    if (lane < 16) {
-      const bf16* src = lane < 8 ? p.bias : p.w2;
-      const int j = 8 * (lane & 7);
-      float f[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      if (src) load_vec(src + j, f);
-      st_shared_f4(sc + 4u * (8 * lane), f);
-      st_shared_f4(sc + 4u * (8 * lane + 4), f + 4);
-    }
-  } else {
-    for (int j8 = lane; j8 < bn / 8; j8 += 32) {
-      const int n = nb * bn + 8 * j8;
-      float f[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      if (n < p.N) {
-        if (p.bias) load_vec(p.bias + n, f);
-        if (p.bias2) {
-          float g[8];
-          load_vec(p.bias2 + n, g);
+  for (int j8 = lane; j8 < bn / 8; j8 += 32) {
+    const int n = nb * bn + 8 * j8;
+    float f[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    if (n < p.N) {
+      if (p.bias) load_vec(p.bias + n, f);
+      if (p.bias2) {
+        float g[8];
+        load_vec(p.bias2 + n, g);
 #pragma unroll
-          for (int i = 0; i < 8; ++i) f[i] += g[i];
-        }
+        for (int i = 0; i < 8; ++i) f[i] += g[i];
       }
-      st_shared_f4(sc + 4u * (8 * j8), f);
-      st_shared_f4(sc + 4u * (8 * j8 + 4), f + 4);
     }
+    st_shared_f4(sc + 4u * (8 * j8), f);
+    st_shared_f4(sc + 4u * (8 * j8 + 4), f + 4);
   }
   __syncwarp();
 }
@@ -354,15 +340,15 @@ struct EpiPre {
 
 // Epilogue of one accumulator tile for the calling thread's row m over the
 // chunks [c_lo, c_hi) of 32 TMEM columns -> constants / activation / rotary /
-// residual / store, or the router's row reduction. `sc` holds the staged
+// residual / store. `sc` holds the staged
 // per-column constants (has_consts), `pre` the prefetched residual chunks,
 // `red` the split-K partial to add first. ROPE: the instance for rotary
 // tiles (query / key / value projections, which have no residual).
-template <int BN, bool DUAL, bool ROUTER, bool ROPE>
+template <int BN, bool DUAL, bool ROPE>
 __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, int m, int nb, int bn,
                                               int c_lo, int c_hi, uint32_t sc, bool has_consts,
                                               const EpiPre& pre, const EpiRed& red) {
-  constexpr bool rope = ROPE && !ROUTER && !DUAL;
+  constexpr bool rope = ROPE && !DUAL;
   const bool mvalid = m < p.M;
   int64_t arow = m;
   if (mvalid && p.rows) arow = p.rows[m];
@@ -371,7 +357,6 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
   if (rope && mvalid)
     tab_row = p.rope_tab + (int64_t)(p.rope_pos ? p.rope_pos[m] : m % p.rope_T) * p.rope_half;
   const int row = m & (BM - 1);
-  float rsum = 0.f;
 #pragma unroll 1
   for (int c = c_lo; c < c_hi; ++c) {
     const int n0 = nb * bn + c * 32;
@@ -403,17 +388,6 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
         v[4 * j + 2] += f.z;
         v[4 * j + 3] += f.w;
       }
-    }
-    if (ROUTER) {
-#pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        float b[4], w[4];
-        ld_shared_f4(sc + 4u * (c * 32 + 4 * q), b);
-        ld_shared_f4(sc + 4u * (64 + c * 32 + 4 * q), w);
-#pragma unroll
-        for (int j = 0; j < 4; ++j) rsum += w[j] * silu_f(v[4 * q + j] + b[j]);
-      }
-      continue;
     }
     if (has_consts) add_consts32(sc, c * 32, v);
     if (!DUAL && p.vt && n0 >= p.vt_col0) {
@@ -454,7 +428,6 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
     }
     epi_chunk_store<!ROPE>(p, v, res, orow, n0);
   }
-  if (ROUTER && c_hi > c_lo && mvalid) p.scores[m] = rsum + __bfloat162float(p.b2[0]);
 }
 
 // Prefetch of the residual of chunks c_lo, c_lo + 1 for row m (before the
@@ -477,18 +450,17 @@ __device__ __forceinline__ void prefetch_res(const GemmDev& p, int m, int nb, in
 // The epilogue warps' part of a tile once its coordinates are known: stage
 // constants, prefetch residuals, wait for the accumulator (bounded), run the
 // epilogue. Returns false if the wait gave up.
-template <int BN, bool DUAL, bool ROUTER>
+template <int BN, bool DUAL>
 __device__ __forceinline__ bool epilogue_role(const GemmDev& P, int m, int nb, int half,
                                               uint32_t tacc, uint32_t sc, uint32_t tfull,
                                               uint32_t parity, volatile int* abort_flag,
                                               int lane) {
   const int bn = P.bn;
   const int NC = bn / 32;
-  // the router's row reduction stays in one warp per quarter
-  const int c_lo = ROUTER ? (half == 0 ? 0 : NC) : half * (NC / 2);
-  const int c_hi = ROUTER ? NC : (half + 1) * (NC / 2);
-  const bool has_consts = ROUTER || P.bias || P.bias2;
-  if (has_consts) stage_consts<ROUTER>(P, nb, bn, sc, lane);
+  const int c_lo = half * (NC / 2);
+  const int c_hi = (half + 1) * (NC / 2);
+  const bool has_consts = P.bias || P.bias2;
+  if (has_consts) stage_consts(P, nb, bn, sc, lane);
   EpiPre pre;
   pre.n = 0;
   if (!P.rope_tab) prefetch_res(P, m, nb, bn, c_lo, c_hi, pre);
@@ -498,14 +470,14 @@ __device__ __forceinline__ bool epilogue_role(const GemmDev& P, int m, int nb, i
   if (!ok) return false;
   tc_fence_after();
   const EpiRed none = {nullptr, 0, 0, 0};
-  if (!ROUTER && !DUAL && P.rope_tab)
-    epilogue_tile<BN, DUAL, ROUTER, true>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none);
+  if (!DUAL && P.rope_tab)
+    epilogue_tile<BN, DUAL, true>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none);
   else
-    epilogue_tile<BN, DUAL, ROUTER, false>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none);
+    epilogue_tile<BN, DUAL, false>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none);
   return true;
 }
 
-template <int BN, bool DUAL, bool ROUTER>
+template <int BN, bool DUAL>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmB2,
@@ -680,7 +652,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int acc = it & 1;
       const uint32_t sc = sconst + 4u * kConstFloats * ((warp - 2) * 2 + acc);
       const uint32_t tacc = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C::ACC_COLS;
-      if (!epilogue_role<BN, DUAL, ROUTER>(P, ti.mb * BM + row_in_tile, ti.nb, half, tacc, sc,
+      if (!epilogue_role<BN, DUAL>(P, ti.mb * BM + row_in_tile, ti.nb, half, tacc, sc,
                                            tfull0 + 8 * acc, (it >> 1) & 1, abort_flag, lane))
         break;
       tc_fence_before();
@@ -849,7 +821,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else {
     // ------------------------------------------------------------ epilogue, part 1
     pdl_wait();
-    if (has_consts) stage_consts<false>(p, ti.nb, BN, sc, lane);
+    if (has_consts) stage_consts(p, ti.nb, BN, sc, lane);
     if (lane == 0) ok = mbar_wait_bounded(tfull, 0, abort_flag, p.err, p.timeout_ns);
     ok = __shfl_sync(0xffffffffu, ok, 0);
     tc_fence_after();
@@ -882,9 +854,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ epilogue, part 2
     const EpiRed red = {p.scratch + (size_t)tile * S * BM * BN, S, rank, BN};
     if (p.rope_tab)   // rotary halves of at most 16 features (one chunk)
-      epilogue_tile<BN, false, false, true>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre, red);
+      epilogue_tile<BN, false, true>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre, red);
     else
-      epilogue_tile<BN, false, false, false>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre,
+      epilogue_tile<BN, false, false>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre,
                                              red);
   }
 
@@ -1085,7 +1057,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int acc = it & 1;
       const uint32_t sc = sconst + 4u * kConstFloats * ((warp - 2) * 2 + acc);
       const uint32_t tacc = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C::ACC_COLS;
-      if (!epilogue_role<BN, DUAL, false>(P, ti.mb * 2 * BM + (int)rank * BM + row_in_tile, ti.nb,
+      if (!epilogue_role<BN, DUAL>(P, ti.mb * 2 * BM + (int)rank * BM + row_in_tile, ti.nb,
                                           half, tacc, sc, tfull0 + 8 * acc, (it >> 1) & 1,
                                           abort_flag, lane))
         break;
@@ -1169,8 +1141,6 @@ bool make_dev(const GemmArgs& a, const Dev& dev, GemmDev& p) {
   p.rows = a.epi.rows;
   p.out_mapped = a.epi.out_mapped ? 1 : 0;
   p.out = static_cast<bf16*>(a.epi.out); p.ld_out = a.epi.ld_out;
-  p.w2 = static_cast<const bf16*>(a.epi.w2); p.b2 = static_cast<const bf16*>(a.epi.b2);
-  p.scores = a.epi.scores;
   p.rope_tab = a.epi.rope_tab;
   p.rope_pos = a.epi.rope_pos;
   p.rope_T = a.epi.rope_T;
@@ -1236,14 +1206,14 @@ cudaError_t prepare(const GemmArgs& a, const GemmArgs* b, uint32_t a_rows, int b
   return cudaSuccess;
 }
 
-template <int BN, bool DUAL, bool ROUTER>
+template <int BN, bool DUAL>
 cudaError_t launch(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
   using C = TileCfg<BN, DUAL>;
   static int attr_done[64] = {0};
   int device = 0;
   cudaGetDevice(&device);
   if (device < 64 && !attr_done[device]) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, DUAL, ROUTER>,
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, DUAL>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
     if (e != cudaSuccess) return e;
     attr_done[device] = 1;
@@ -1255,7 +1225,7 @@ cudaError_t launch(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
   int64_t num_tiles = ((a.M + BM - 1) / BM) * ((a.N + p.bn - 1) / p.bn);
   if (b) num_tiles += ((b->M + BM - 1) / BM) * ((b->N + p2.bn - 1) / p2.bn);
   const int grid = (int)(num_tiles < dev.num_sms ? num_tiles : dev.num_sms);
-  return launch_pdl(gemm_tc_kernel<BN, DUAL, ROUTER>, dim3(grid), dim3(kThreads), C::SMEM_BYTES,
+  return launch_pdl(gemm_tc_kernel<BN, DUAL>, dim3(grid), dim3(kThreads), C::SMEM_BYTES,
                     dev.stream, tm[0], tm[1], tm[2], tm[3], p, p2);
 }
 
@@ -1413,8 +1383,8 @@ cudaError_t gemm_plain(const GemmArgs& a, const Dev& dev) {
   }
   switch (pick) {
     case 0: return launch_pair<256, false>(a, nullptr, dev);
-    case 1: return launch<256, false, false>(a, nullptr, dev);
-    case 2: return launch<128, false, false>(a, nullptr, dev);
+    case 1: return launch<256, false>(a, nullptr, dev);
+    case 2: return launch<128, false>(a, nullptr, dev);
     case 3: return launch_sk<256>(a, dev, split_s);
     default: return launch_sk<128>(a, dev, split_s);
   }
@@ -1428,17 +1398,13 @@ size_t gemm_split_scratch_bytes() { return (size_t)160 * BM * 256 * 4; }
 
 cudaError_t gemm_bf16(const GemmArgs& a, const Dev& dev) {
   if (a.M <= 0) return cudaSuccess;
-  if (a.epi.act == ACT_ROUTER) {
-    if (a.N != 64 || a.K2 > 0) return cudaErrorInvalidValue;
-    return launch<64, false, true>(a, nullptr, dev);
-  }
   // SwiGLU: 256 x 128 gate/up tiles on CTA pairs when that still gives every
   // pair of SMs at least two tiles.
   if (a.epi.act == ACT_SWIGLU) {
     if (a.K2 > 0) return cudaErrorInvalidValue;
     const int64_t pair_tiles = ((a.M + 255) / 256) * ((a.N + 127) / 128);
     if (a.N % 128 == 0 && pair_tiles >= dev.num_sms) return launch_pair<128, true>(a, nullptr, dev);
-    return launch<128, true, false>(a, nullptr, dev);
+    return launch<128, true>(a, nullptr, dev);
   }
   return gemm_plain(a, dev);
 }
@@ -1448,7 +1414,7 @@ cudaError_t gemm_bf16_grouped(const GemmArgs& a, const GemmArgs& b, const Dev& d
   if (a.M <= 0) return gemm_bf16(b, dev);
   if (b.M <= 0) return gemm_bf16(a, dev);
   auto plain = [](const GemmArgs& g) {
-    return g.epi.act != ACT_ROUTER && g.epi.act != ACT_SWIGLU && g.K2 == 0;
+    return g.epi.act != ACT_SWIGLU && g.K2 == 0;
   };
   if (!plain(a) || !plain(b)) return cudaErrorInvalidValue;
   // Fewest rounds of tiles (a k-block costs the same for any tile width);
@@ -1472,13 +1438,13 @@ cudaError_t gemm_bf16_grouped(const GemmArgs& a, const GemmArgs& b, const Dev& d
                        2 * std::max(chunk(a), chunk(b));
   const int64_t best = std::min(std::min(c_pair, c256), std::min(c_half, c128));
   if (c_pair == best) return launch_pair<256, false>(a, &b, dev);
-  if (c256 == best) return launch<256, false, false>(a, &b, dev);
+  if (c256 == best) return launch<256, false>(a, &b, dev);
   if (c_half == best) {
     GemmArgs a_half = a;
     a_half.tile_n = 128;
-    return launch<256, false, false>(a_half, &b, dev);
+    return launch<256, false>(a_half, &b, dev);
   }
-  return launch<128, false, false>(a, &b, dev);
+  return launch<128, false>(a, &b, dev);
 }
 
 }  // namespace adadsf

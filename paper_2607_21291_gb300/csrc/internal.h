@@ -11,7 +11,7 @@ namespace adadsf {
 enum Dtype : int { kF32 = 0, kBF16 = 1 };
 // Bits of the device error word (first int of every workspace).
 enum : int { DEVERR_TIMEOUT = 1, DEVERR_INDEX = 2 };
-enum Act : int { ACT_NONE = 0, ACT_GELU = 1, ACT_SWIGLU = 2, ACT_ROUTER = 3 };
+enum Act : int { ACT_NONE = 0, ACT_GELU = 1, ACT_SWIGLU = 2 };
 
 // Epilogue of the projection kernels, applied to the fp32 accumulator
 // acc[m][n] of out = A[m,:] . W[n,:]:
@@ -21,7 +21,6 @@ enum Act : int { ACT_NONE = 0, ACT_GELU = 1, ACT_SWIGLU = 2, ACT_ROUTER = 3 };
 //   v += add_packed[m][n]                     (may be null)
 //   v += add_rows[row(m)][n]                  (may be null)
 //   out[out_mapped ? row(m) : m][n] = v       row(m) = rows ? rows[m] : m
-// ACT_ROUTER instead reduces each row to scores[m] = sum_n w2[n] silu(acc + bias[n]) + b2.
 struct Epilogue {
   int act = ACT_NONE;
   const void* bias = nullptr;
@@ -34,9 +33,6 @@ struct Epilogue {
   bool out_mapped = true;
   void* out = nullptr;
   int64_t ld_out = 0;
-  const void* w2 = nullptr;   // router
-  const void* b2 = nullptr;   // router
-  float* scores = nullptr;    // router
   // Rotary embedding of the first rope_cols output columns (query and key
   // heads), bf16 tensor-core path only: per head of rope_hd columns, feature
   // i < rope_half pairs with i + rope_half and turns by tab[pos][i], pos =
