@@ -25,7 +25,9 @@
 //              memory on a named barrier): read S once, mask (diagonal block
 //              only), online softmax in fp32 (exp2 with a row maximum held at
 //              most 2^8 below the true one, so O is rescaled only when the
-//              maximum grows by more than that), write P as bf16 pairs over
+//              maximum grows by more than that; paired fp32 arithmetic and
+//              three-input maxima keep the instruction count down), write P
+//              as bf16 pairs over
 //              the first 32 of its own 64 S columns (so neither warp of the
 //              pair overwrites scores the other has yet to read), and at the
 //              end O / l -> global.
@@ -85,6 +87,13 @@ __device__ __forceinline__ float ex2_approx(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+// max(a, b, c) in one instruction.
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
 }
 
 struct AttnDev {
@@ -323,7 +332,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
           for (int i = 0; i < 64; ++i) mx[i & 3] = fmaxf(mx[i & 3], (i <= lim) ? __uint_as_float(u[i]) : -INFINITY);
         } else {
 #pragma unroll
-          for (int i = 0; i < 64; ++i) mx[i & 3] = fmaxf(mx[i & 3], __uint_as_float(u[i]));
+          for (int i = 0; i < 64; i += 2)
+            mx[(i >> 1) & 3] = fmax3(mx[(i >> 1) & 3], __uint_as_float(u[i]), __uint_as_float(u[i + 1]));
         }
       }
       // a wait that gave up travels as NaN, so the pair leaves together (the
@@ -356,7 +366,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       // half's columns (chunk c's 32 scores are read before P of chunk c
       // covers columns 16 c .. 16 c + 15, whose scores are already used);
       // row sum in fp32
-      float sm[4] = {0.f, 0.f, 0.f, 0.f};
+      const float2 scale2 = make_float2(p.scale_log2, p.scale_log2);
+      const float2 negm2 = make_float2(-m_used, -m_used);
+      float2 sm[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
         uint32_t u[32], pk[16];
@@ -365,20 +377,20 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const int k0 = 32 * c + 2 * i;
-          float e0 = ex2_approx(fmaf(__uint_as_float(u[2 * i]), p.scale_log2, -m_used));
-          float e1 = ex2_approx(fmaf(__uint_as_float(u[2 * i + 1]), p.scale_log2, -m_used));
+          const float2 x = __ffma2_rn(make_float2(__uint_as_float(u[2 * i]), __uint_as_float(u[2 * i + 1])),
+                                      scale2, negm2);
+          float2 e = make_float2(ex2_approx(x.x), ex2_approx(x.y));
           if (diag) {
-            e0 = (k0 <= lim) ? e0 : 0.f;
-            e1 = (k0 + 1 <= lim) ? e1 : 0.f;
+            e.x = (k0 <= lim) ? e.x : 0.f;
+            e.y = (k0 + 1 <= lim) ? e.y : 0.f;
           }
-          sm[k0 & 3] += e0;
-          sm[(k0 + 1) & 3] += e1;
-          pk[i] = pack_bf16x2(e0, e1);
+          sm[i & 1] = __fadd2_rn(sm[i & 1], e);
+          pk[i] = pack_bf16x2(e.x, e.y);
         }
         tmem_st16(tSh + 16 * c, pk);
       }
       tmem_st_wait();
-      l += (sm[0] + sm[1]) + (sm[2] + sm[3]);
+      l += (sm[0].x + sm[1].x) + (sm[0].y + sm[1].y);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(p_full0 + 8 * t);
