@@ -3,7 +3,8 @@
 // One CTA per (pair of 128-query blocks, query head, sequence): the two
 // query tiles share every K / V tile the CTA loads, which halves the K / V
 // traffic per flop, and their softmax work alternates with the other tile's
-// matrix products. Keys arrive in blocks of 128; attention is causal in
+// matrix products. When pairs would leave SMs idle (few, short sequences),
+// one CTA per query block instead. Keys arrive in blocks of 128; attention is causal in
 // packed order (kept positions ascend, so this is the original causal mask
 // restricted to the kept set, Sec. 3.4).
 //   warp 0     TMA, lane 0: both Q tiles once, then the K tile of each key
@@ -98,6 +99,7 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
 
 struct AttnDev {
   int K;                 // kept tokens per sequence
+  int pair;              // 1: two query blocks per CTA, 0: one
   int Hq, Hkv, q_dim;
   float scale_log2;      // log2(e) / sqrt(hd)
   bf16* out;
@@ -141,10 +143,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int nqb = (p.K + kQB - 1) / kQB;
-  const int npair = (nqb + 1) / 2;
-  const int pr = npair - 1 - (int)blockIdx.x;   // longest rows first
-  const int qb0 = 2 * pr;
-  const bool two = qb0 + 1 < nqb;               // tile 1 holds query block qb0 + 1
+  // longest rows first
+  const int qb0 = p.pair ? 2 * ((nqb + 1) / 2 - 1 - (int)blockIdx.x) : nqb - 1 - (int)blockIdx.x;
+  const bool two = p.pair && qb0 + 1 < nqb;     // tile 1 holds query block qb0 + 1
   const int n_kv = two ? qb0 + 2 : qb0 + 1;     // tile 0 takes blocks 0..qb0, tile 1 all
   const int h = blockIdx.y, b = blockIdx.z;
   const int g = h / (p.Hq / p.Hkv);
@@ -481,7 +482,9 @@ cudaError_t launch_attn(const void* qkv, int64_t ld_qkv, const void* vt, int pad
   p.ld_out = ld_out;
   p.err = dev.err;
   p.timeout_ns = kWaitTimeoutNs;
-  dim3 grid(((K + kQB - 1) / kQB + 1) / 2, Hq, B);
+  const int nqb = (K + kQB - 1) / kQB;
+  p.pair = (int64_t)((nqb + 1) / 2) * Hq * B >= dev.num_sms ? 1 : 0;
+  dim3 grid(p.pair ? (nqb + 1) / 2 : nqb, Hq, B);
   return launch_pdl(attn_tc_kernel<HD>, grid, dim3(kAttnThreads), C::SMEM, dev.stream, tq, tv, p);
 }
 

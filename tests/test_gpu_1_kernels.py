@@ -218,6 +218,27 @@ def test_attention(A, hq, hkv, hd, B, K, dtype):
         assert H.max_rel(got[b * K:(b + 1) * K], ref) < (2e-2 if dtype == "bf16" else 1e-5)
 
 
+@pytest.mark.parametrize("hq,hkv,hd,B,K", [(12, 12, 64, 7, 520), (12, 12, 64, 7, 300), (12, 2, 128, 5, 520),
+                                          (4, 4, 128, 20, 300), (28, 4, 128, 2, 1100)])
+def test_attention_paired_tiles(A, hq, hkv, hd, B, K):
+    """Enough (query-block pair, head, sequence) work units to fill the GPU:
+    the kernel runs two query tiles per CTA (with an odd number of query
+    blocks the last pair has one tile), bf16 against the oracle."""
+    shape = S.PYTHIA_160M.replace(n_heads=hq, n_kv_heads=hkv, head_dim=hd, d=hq * hd, dtype="bf16")
+    width = (hq + 2 * hkv) * hd
+    g = np.random.default_rng(B * K + hq + hd + 7)
+    qkv = S.round_to(g.standard_normal((B * K, width)).astype(np.float32), "bf16")
+    out = torch.empty((B * K, hq * hd), dtype=torch.bfloat16, device="cuda")
+    A.adadsf_causal_attention(A.make_cfg(shape), H.to_dev(qkv, torch.bfloat16), B, K, out)
+    got = H.to_np(out)
+    q64 = qkv.astype(np.float64)
+    for b in range(B):
+        blk = q64[b * K:(b + 1) * K]
+        ref = O.causal_attention(blk[:, :hq * hd], blk[:, hq * hd:(hq + hkv) * hd], blk[:, (hq + hkv) * hd:],
+                                 hq, hkv, hd)
+        assert H.max_rel(got[b * K:(b + 1) * K], ref) < 2e-2
+
+
 # ---------------------------------------------------------------- Eq. 4 statistics
 @pytest.mark.parametrize("n,d,dtype", [(1, 64, "f32"), (37, 768, "bf16"), (5000, 1536, "bf16"),
                                        (3000, 512, "f32")])
