@@ -152,27 +152,36 @@ __device__ __forceinline__ KbSrc kb_source(const TileInfo& ti, int kb, const CUt
   return s;
 }
 
+__device__ __forceinline__ float2 splat2(float a) { return make_float2(a, a); }
+
 // erf(z) = 1 - exp(-z^2) R(z) for z >= 0 (erf is odd), R(z) = erfc(z) exp(z^2)
 // approximated on [0, 4] by a degree-10 polynomial in z / 4 (coefficients
 // and error bound from csrc/erf_poly.py: |error| <= 3.3e-7 in fp32); erf = 1
-// beyond z = 4 (to 1.6e-8). One exponential, no division.
-__device__ __forceinline__ float erf_fit(float x) {
-  const float z = fminf(fabsf(x), 4.f);
-  const float u = z * 0.25f;
-  float r = 1.019359436e+02f;
-  r = fmaf(r, u, -3.950886841e+02f);
-  r = fmaf(r, u, 6.843880615e+02f);
-  r = fmaf(r, u, -7.131018066e+02f);
-  r = fmaf(r, u, 5.127547607e+02f);
-  r = fmaf(r, u, -2.798540955e+02f);
-  r = fmaf(r, u, 1.249815445e+02f);
-  r = fmaf(r, u, -4.795371628e+01f);
-  r = fmaf(r, u, 1.599380779e+01f);
-  r = fmaf(r, u, -4.513438225e+00f);
-  r = fmaf(r, u, 9.999998212e-01f);
-  return copysignf(fmaf(-__expf(-z * z), r, 1.f), x);
+// beyond z = 4 (to 1.6e-8). One exponential, no division; two values at a
+// time on the paired fp32 pipe (the epilogue is issue bound).
+__device__ __forceinline__ float2 erf_fit2(float2 x) {
+  const float zx = fminf(fabsf(x.x), 4.f), zy = fminf(fabsf(x.y), 4.f);
+  const float2 u = make_float2(zx * 0.25f, zy * 0.25f);
+  float2 r = splat2(1.019359436e+02f);
+  r = __ffma2_rn(r, u, splat2(-3.950886841e+02f));
+  r = __ffma2_rn(r, u, splat2(6.843880615e+02f));
+  r = __ffma2_rn(r, u, splat2(-7.131018066e+02f));
+  r = __ffma2_rn(r, u, splat2(5.127547607e+02f));
+  r = __ffma2_rn(r, u, splat2(-2.798540955e+02f));
+  r = __ffma2_rn(r, u, splat2(1.249815445e+02f));
+  r = __ffma2_rn(r, u, splat2(-4.795371628e+01f));
+  r = __ffma2_rn(r, u, splat2(1.599380779e+01f));
+  r = __ffma2_rn(r, u, splat2(-4.513438225e+00f));
+  r = __ffma2_rn(r, u, splat2(9.999998212e-01f));
+  const float2 e = __ffma2_rn(make_float2(-__expf(-zx * zx), -__expf(-zy * zy)), r, splat2(1.f));
+  return make_float2(copysignf(e.x, x.x), copysignf(e.y, x.y));
 }
-__device__ __forceinline__ float gelu_f(float v) { return 0.5f * v * (1.f + erf_fit(v * 0.70710678118654752f)); }
+// exact GELU, 0.5 v (1 + erf(v / sqrt 2)), of two values
+__device__ __forceinline__ float2 gelu2(float2 v) {
+  const float2 e = erf_fit2(__fmul2_rn(v, splat2(0.70710678118654752f)));
+  const float2 h = __fmul2_rn(v, splat2(0.5f));
+  return __ffma2_rn(h, e, h);
+}
 // v sigmoid(v); the exponent is capped so the fast division stays in range.
 __device__ __forceinline__ float silu_f(float v) {
   return v * __fdividef(1.f, 1.f + __expf(fminf(-v, 80.f)));
@@ -404,7 +413,11 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
       for (int j = 0; j < 32; ++j) v[j] = silu_f(v[j]) * __uint_as_float(r2[j]);
     } else if (p.act == ACT_GELU) {
 #pragma unroll
-      for (int j = 0; j < 32; ++j) v[j] = gelu_f(v[j]);
+      for (int j = 0; j < 32; j += 2) {
+        const float2 g = gelu2(make_float2(v[j], v[j + 1]));
+        v[j] = g.x;
+        v[j + 1] = g.y;
+      }
     }
     // residual of this chunk: prefetched for the first two, else loaded now
     uint4 res[4];

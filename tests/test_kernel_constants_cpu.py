@@ -30,7 +30,7 @@ def test_erf_fit_matches_kernel_and_bound():
     m = _load("erf_poly")
     c = m.fit()
     src = open(os.path.join(CSRC, "gemm_tcgen05.cu")).read()
-    body = src[src.index("float erf_fit("):src.index("float gelu_f(")]
+    body = src[src.index("float2 erf_fit2("):src.index("float2 gelu2(")]
     kern = _floats(body)[::-1]             # Horner order: highest degree first
     assert len(kern) == len(c)
     assert np.allclose(kern, c, rtol=1e-6, atol=0)
