@@ -57,6 +57,7 @@ constexpr int kEpiWarps = 8;     // two per TMEM lane quarter, each on half of t
 constexpr int kThreads = 64 + 32 * kEpiWarps;
 constexpr int kGroupM = 16;  // tile raster: 16 M-blocks share each W column block
 constexpr int kConstFloats = 256;   // staged per-column constants per epilogue warp and slot
+constexpr int kStgBytes = 32 * 64;  // one 32-row x 32-column bf16 chunk per epilogue warp
 
 // PAIR: two-CTA variant. Plain: each CTA stages half of the BN weight rows.
 // DUAL: the even CTA stages BN rows of the first weight, the odd CTA BN rows
@@ -75,7 +76,8 @@ struct TileCfg {
   static constexpr int TMEM_COLS = 2 * ACC_COLS;
   static constexpr int BAR_BYTES = (2 * STAGES + 6) * 8 + 16;
   static constexpr int CONST_BYTES = kEpiWarps * 2 * kConstFloats * 4;
-  static constexpr int SMEM_BYTES = RING_BYTES + 1024 + BAR_BYTES + CONST_BYTES;
+  static constexpr int STG_BYTES = kEpiWarps * kStgBytes;   // store staging, per epilogue warp
+  static constexpr int SMEM_BYTES = RING_BYTES + 1024 + BAR_BYTES + CONST_BYTES + STG_BYTES;
   static_assert(TMEM_COLS == 128 || TMEM_COLS == 256 || TMEM_COLS == 512, "TMEM columns");
   static_assert(BAR_BYTES % 16 == 0, "constants stay 16-byte aligned");
   static_assert(SMEM_BYTES <= 232448, "shared memory");
@@ -239,41 +241,93 @@ __device__ __forceinline__ void load_res32(const GemmDev& p, int64_t rrow, int n
   for (int i = 0; i < 4; ++i) u[i] = src[i];
 }
 
+__device__ __forceinline__ void st_shared_u4(uint32_t addr, uint4 v) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
+__device__ __forceinline__ uint4 ld_shared_u4(uint32_t addr) {
+  uint4 v;
+  asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr)
+               : "memory");
+  return v;
+}
+
+// One 32-column bf16 chunk (4 x 16 bytes, pk) for each of the warp's 32
+// rows (one per lane; dst = the lane's row at the chunk's first column, or
+// null for no row), passed through the warp's staging area so that each
+// global store instruction writes 8 rows x 64 contiguous bytes instead of
+// 32 rows x 16 bytes (the rows are scattered or a full row apart). The 16-byte
+// pieces are XOR-swizzled so neither phase has bank conflicts. Whole warp.
+__device__ __forceinline__ void store_chunk_rows(uint32_t stg, int lane, const uint4* pk, bf16* dst) {
+#pragma unroll
+  for (int q = 0; q < 4; ++q) st_shared_u4(stg + lane * 64 + ((q ^ ((lane >> 1) & 3)) << 4), pk[q]);
+  __syncwarp();
+  const int q = lane & 3;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int r = 8 * k + (lane >> 2);
+    const uint4 v = ld_shared_u4(stg + r * 64 + ((q ^ ((r >> 1) & 3)) << 4));
+    bf16* d = reinterpret_cast<bf16*>(
+        __shfl_sync(0xffffffffu, (unsigned long long)reinterpret_cast<uintptr_t>(dst), r));
+    if (d) *reinterpret_cast<uint4*>(d + 8 * q) = v;
+  }
+  __syncwarp();
+}
+
 // Store one 32-column chunk of output row orow (adding the residual `res`
-// if RES and the problem has one).
+// if RES and the problem has one); rows with !valid store nothing. Whole warp.
 template <bool RES>
 __device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, const uint4* res,
-                                                int64_t orow, int n0) {
+                                                int64_t orow, int n0, bool valid, uint32_t stg,
+                                                int lane) {
   if (RES && p.add) {
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       float f[8];
       unpack16(res[i], f, bf16());
 #pragma unroll
-      for (int j = 0; j < 8; ++j) v[8 * i + j] += f[j];
+      for (int j = 0; j < 8; j += 2) {
+        const float2 s2 = __fadd2_rn(make_float2(v[8 * i + j], v[8 * i + j + 1]), make_float2(f[j], f[j + 1]));
+        v[8 * i + j] = s2.x;
+        v[8 * i + j + 1] = s2.y;
+      }
     }
   }
+  uint4 pk[4];
 #pragma unroll
-  for (int i = 0; i < 4; ++i) store_vec(p.out + orow * p.ld_out + n0 + 8 * i, v + 8 * i);
+  for (int i = 0; i < 4; ++i) pk[i] = pack16(v + 8 * i, bf16());
+  store_chunk_rows(stg, lane, pk, valid ? p.out + orow * p.ld_out + n0 : nullptr);
 }
 
 // Rotary halves of 32 or more features: chunk c (first half of a head's
 // rotated features) and chunk c2 (second half) of row m: a' = a cos - b sin,
-// b' = b cos + a sin. The row's (cos, sin) pairs are loaded 16 at a time
-// (their latency paid twice per chunk pair), the accumulator 8 columns at a time.
-// These are query / key columns: no activation, residual or transposed copy.
+// b' = b cos + a sin. The row's (cos, sin) pairs are loaded 16 at a time (the
+// first 16 of the tile may have been prefetched before the accumulator was
+// ready: tpre), the accumulator 8 columns at a time. These are query / key
+// columns: no activation, residual or transposed copy.
 __device__ __forceinline__ void rope_pair(const GemmDev& p, uint32_t tacc, int c, int c2, int bn,
                                           int nb, uint32_t sc, bool has_consts,
-                                          const float2* tab_row, bool mvalid, int64_t orow) {
+                                          const float2* tab_row, bool mvalid, int64_t orow,
+                                          const uint4 (&tpre)[2][4], bool use_pre, uint32_t stg,
+                                          int lane) {
   const int n0 = nb * bn + c * 32, n2 = nb * bn + c2 * 32;
   const int i0 = n0 % p.rope_hd;
-#pragma unroll 1
+  uint4 pa[4], pb[4];   // the two chunks, bf16
+#pragma unroll
   for (int gh = 0; gh < 2; ++gh) {
     float4 t[8];   // t[k] = (cos, sin) of features i0 + 16 gh + 2k and the next one
     if (mvalid) {
       const float4* t4 = reinterpret_cast<const float4*>(tab_row + i0 + 16 * gh);
 #pragma unroll
-      for (int k = 0; k < 8; ++k) t[k] = t4[k];
+      for (int k = 0; k < 8; ++k) {
+        if (gh == 0 && use_pre) {
+          const uint4 q = tpre[k >> 2][k & 3];
+          t[k] = make_float4(__uint_as_float(q.x), __uint_as_float(q.y), __uint_as_float(q.z),
+                             __uint_as_float(q.w));
+        } else {
+          t[k] = t4[k];
+        }
+      }
     }
 #pragma unroll
     for (int gg = 0; gg < 2; ++gg) {
@@ -282,7 +336,6 @@ __device__ __forceinline__ void rope_pair(const GemmDev& p, uint32_t tacc, int c
       tmem_ld8(tacc + c * 32 + 8 * g, ra);
       tmem_ld8(tacc + c2 * 32 + 8 * g, rb);
       tmem_ld_wait();
-      if (!mvalid) continue;
       float a[8], b[8];
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
@@ -309,10 +362,12 @@ __device__ __forceinline__ void rope_pair(const GemmDev& p, uint32_t tacc, int c
         a[j] = x * cs - y * sn;
         b[j] = y * cs + x * sn;
       }
-      store_vec(p.out + orow * p.ld_out + n0 + 8 * g, a);
-      store_vec(p.out + orow * p.ld_out + n2 + 8 * g, b);
+      pa[g] = pack16(a, bf16());
+      pb[g] = pack16(b, bf16());
     }
   }
+  store_chunk_rows(stg, lane, pa, mvalid ? p.out + orow * p.ld_out + n0 : nullptr);
+  store_chunk_rows(stg, lane, pb, mvalid ? p.out + orow * p.ld_out + n2 : nullptr);
 }
 
 // Feature j < H of the chunk pairs with feature j + H (H = rotary half <= 16).
@@ -342,9 +397,12 @@ struct EpiRed {
 };
 
 // Values the epilogue fetched before the accumulator was ready.
+// Rotary tiles (no residual) reuse the registers for the (cos, sin) pairs
+// of their first chunk's first 16 features (res read as 8 float4).
 struct EpiPre {
   uint4 res[2][4];   // residual of the first two chunks this warp finalises
   int n;             // how many of them are valid
+  bool nt;           // res holds rotary pairs instead
 };
 
 // Epilogue of one accumulator tile for the calling thread's row m over the
@@ -356,7 +414,8 @@ struct EpiPre {
 template <int BN, bool DUAL, bool ROPE>
 __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, int m, int nb, int bn,
                                               int c_lo, int c_hi, uint32_t sc, bool has_consts,
-                                              const EpiPre& pre, const EpiRed& red) {
+                                              const EpiPre& pre, const EpiRed& red, uint32_t stg,
+                                              int lane) {
   constexpr bool rope = ROPE && !DUAL;
   const bool mvalid = m < p.M;
   int64_t arow = m;
@@ -374,7 +433,8 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
     const bool rot = rope && n0 < p.rope_cols;
     if (rot && p.rope_half >= 32) {
       if ((n0 % p.rope_hd) < p.rope_half && n0 < p.N)   // else done with its partner
-        rope_pair(p, tacc, c, c + p.rope_half / 32, bn, nb, sc, has_consts, tab_row, mvalid, orow);
+        rope_pair(p, tacc, c, c + p.rope_half / 32, bn, nb, sc, has_consts, tab_row, mvalid, orow,
+                  pre.res, c == c_lo && pre.nt, stg, lane);
       continue;
     }
     uint32_t r[32];
@@ -382,7 +442,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
     tmem_ld32(tacc + c * 32, r);
     if (DUAL) tmem_ld32(tacc + BN + c * 32, r2);
     tmem_ld_wait();
-    if (!mvalid || n0 >= p.N) continue;
+    if (n0 >= p.N) continue;   // (the same for the whole warp: the store below is warp-wide)
     float v[32];
 #pragma unroll
     for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
@@ -399,7 +459,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
       }
     }
     if (has_consts) add_consts32(sc, c * 32, v);
-    if (!DUAL && p.vt && n0 >= p.vt_col0) {
+    if (!DUAL && p.vt && n0 >= p.vt_col0 && mvalid) {
       // value columns: also store this row's 32 features transposed
       const int vc = n0 - p.vt_col0;
       const int bseq = m / p.vt_seq, j = m - bseq * p.vt_seq;
@@ -420,8 +480,9 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
       }
     }
     // residual of this chunk: prefetched for the first two, else loaded now
-    uint4 res[4];
-    if (!ROPE && p.add) {
+    uint4 res[4] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0),
+                    make_uint4(0, 0, 0, 0)};
+    if (!ROPE && p.add && mvalid) {
       const int k = c - c_lo;
       if (k < pre.n) {
 #pragma unroll
@@ -430,7 +491,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
         load_res32(p, p.add_gathered ? arow : (int64_t)m, n0, res);
       }
     }
-    if (rot && (n0 % p.rope_hd) == 0) {
+    if (rot && (n0 % p.rope_hd) == 0 && mvalid) {
       // rotary half of at most 16 features: both halves inside this chunk
       switch (p.rope_half) {
         case 4: rope_in_chunk<4>(v, tab_row); break;
@@ -439,7 +500,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
         default: break;
       }
     }
-    epi_chunk_store<!ROPE>(p, v, res, orow, n0);
+    epi_chunk_store<!ROPE>(p, v, res, orow, n0, mvalid, stg, lane);
   }
 }
 
@@ -467,7 +528,7 @@ template <int BN, bool DUAL>
 __device__ __forceinline__ bool epilogue_role(const GemmDev& P, int m, int nb, int half,
                                               uint32_t tacc, uint32_t sc, uint32_t tfull,
                                               uint32_t parity, volatile int* abort_flag,
-                                              int lane) {
+                                              int lane, uint32_t stg) {
   const int bn = P.bn;
   const int NC = bn / 32;
   const int c_lo = half * (NC / 2);
@@ -476,7 +537,21 @@ __device__ __forceinline__ bool epilogue_role(const GemmDev& P, int m, int nb, i
   if (has_consts) stage_consts(P, nb, bn, sc, lane);
   EpiPre pre;
   pre.n = 0;
-  if (!P.rope_tab) prefetch_res(P, m, nb, bn, c_lo, c_hi, pre);
+  pre.nt = false;
+  if (!P.rope_tab) {
+    prefetch_res(P, m, nb, bn, c_lo, c_hi, pre);
+  } else if (!DUAL && P.rope_half >= 32 && m < P.M) {
+    // the first rotary chunk's (cos, sin) pairs (inputs of the kernel)
+    const int n0 = nb * bn + c_lo * 32;
+    if (n0 < P.rope_cols && n0 < P.N && (n0 % P.rope_hd) < P.rope_half) {
+      const float4* t4 = reinterpret_cast<const float4*>(
+          P.rope_tab + (int64_t)(P.rope_pos ? P.rope_pos[m] : m % P.rope_T) * P.rope_half + n0 % P.rope_hd);
+      const uint4* q4 = reinterpret_cast<const uint4*>(t4);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) pre.res[k >> 2][k & 3] = q4[k];
+      pre.nt = true;
+    }
+  }
   int ok = 0;
   if (lane == 0) ok = mbar_wait_bounded(tfull, parity, abort_flag, P.err, P.timeout_ns);
   ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -484,9 +559,9 @@ __device__ __forceinline__ bool epilogue_role(const GemmDev& P, int m, int nb, i
   tc_fence_after();
   const EpiRed none = {nullptr, 0, 0, 0};
   if (!DUAL && P.rope_tab)
-    epilogue_tile<BN, DUAL, true>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none);
+    epilogue_tile<BN, DUAL, true>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none, stg, lane);
   else
-    epilogue_tile<BN, DUAL, false>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none);
+    epilogue_tile<BN, DUAL, false>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none, stg, lane);
   return true;
 }
 
@@ -666,7 +741,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t sc = sconst + 4u * kConstFloats * ((warp - 2) * 2 + acc);
       const uint32_t tacc = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C::ACC_COLS;
       if (!epilogue_role<BN, DUAL>(P, ti.mb * BM + row_in_tile, ti.nb, half, tacc, sc,
-                                           tfull0 + 8 * acc, (it >> 1) & 1, abort_flag, lane))
+                                           tfull0 + 8 * acc, (it >> 1) & 1, abort_flag, lane,
+                                           sconst + C::CONST_BYTES + kStgBytes * (warp - 2)))
         break;
       tc_fence_before();
       __syncwarp();
@@ -867,10 +943,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ epilogue, part 2
     const EpiRed red = {p.scratch + (size_t)tile * S * BM * BN, S, rank, BN};
     if (p.rope_tab)   // rotary halves of at most 16 features (one chunk)
-      epilogue_tile<BN, false, true>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre, red);
+      epilogue_tile<BN, false, true>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre, red,
+                                     sconst + C::CONST_BYTES + kStgBytes * (warp - 2), lane);
     else
       epilogue_tile<BN, false, false>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre,
-                                             red);
+                                      red, sconst + C::CONST_BYTES + kStgBytes * (warp - 2), lane);
   }
 
   __syncwarp();
@@ -1072,7 +1149,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const uint32_t tacc = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C::ACC_COLS;
       if (!epilogue_role<BN, DUAL>(P, ti.mb * 2 * BM + (int)rank * BM + row_in_tile, ti.nb,
                                           half, tacc, sc, tfull0 + 8 * acc, (it >> 1) & 1,
-                                          abort_flag, lane))
+                                          abort_flag, lane, sconst + C::CONST_BYTES + kStgBytes * (warp - 2)))
         break;
       tc_fence_before();
       __syncwarp();
