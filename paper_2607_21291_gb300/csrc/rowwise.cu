@@ -3,7 +3,6 @@
 // the Eq. 4 similarity reduction, and the bounded-wait self-test.
 // All are HBM-bound: rows are moved as 16-byte vectors, one warp per row.
 #include <algorithm>
-#include <cstdlib>
 #include <mutex>
 #include <type_traits>
 
@@ -185,30 +184,30 @@ __device__ __forceinline__ void norm_share(int64_t lo, int64_t hi, const T* x, i
 // bytes of an output row.
 constexpr int kRowWarps = 8;                       // consumer warps
 constexpr int kRowThreads = 32 * (kRowWarps + 1);  // + the producer warp
-constexpr int kRowSlotsMax = 64;                   // ring slots: a multiple of kRowWarps
-                                                   // (a slot is always consumed by the same warp)
+constexpr int kRowSlots = 16;                      // ring slots (two rows per consumer warp)
+static_assert(kRowSlots % kRowWarps == 0, "a slot is always consumed by the same warp");
 constexpr int kMaxRowBytes = 8192;   // d <= 4096 (bf16) or 2048 (fp32)
 
 // out1[m] = norm(x[row(m)]; g1, b1), out2[m] = norm(x[row(m)]; g2, b2) for the
 // block's contiguous share of m. Shared memory: the staged parameters
-// ([4][d]), then the ring (`slots` rows of d), then 2 `slots` mbarriers.
-template <typename T, bool RMS, int NCH>
-__global__ void __launch_bounds__(kRowThreads, 2)
+// ([4][d]), then the ring (kRowSlots rows of d), then 2 kRowSlots mbarriers.
+template <typename T, bool RMS>
+__global__ void __launch_bounds__(kRowThreads)
     gather_norm_tma_kernel(const T* x, const int32_t* rows, int64_t M, int d, const T* g1,
                            const T* b1, const T* g2, const T* b2, float eps, T* out1, T* out2,
-                           int slots, int* err, unsigned long long timeout_ns) {
+                           int* err, unsigned long long timeout_ns) {
   pdl_trigger();
   extern __shared__ __align__(16) uint8_t smem_rows[];
   constexpr int V = Elem<T>::kVec;
   const uint32_t row_bytes = (uint32_t)d * sizeof(T);
   T* sp = reinterpret_cast<T*>(smem_rows);
   uint8_t* ring = smem_rows + 4 * (size_t)row_bytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(ring + (size_t)slots * row_bytes);
-  const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * slots;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ring + (size_t)kRowSlots * row_bytes);
+  const uint32_t full0 = smem_u32(bars), empty0 = full0 + 8 * kRowSlots;
   __shared__ int abort_flag;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < slots; ++s) {
+    for (int s = 0; s < kRowSlots; ++s) {
       mbar_init(full0 + 8 * s, 1);
       mbar_init(empty0 + 8 * s, 1);
     }
@@ -234,8 +233,8 @@ __global__ void __launch_bounds__(kRowThreads, 2)
       for (int k = 0; k < cnt; ++k) {
         const int64_t src = __shfl_sync(0xffffffffu, src_l, k);
         const int64_t j = j0 + k;
-        const int s = (int)(j % slots);
-        const uint32_t round = (uint32_t)(j / slots);
+        const int s = (int)(j % kRowSlots);
+        const uint32_t round = (uint32_t)(j / kRowSlots);
         int w = 1;
         if (lane == 0) {
           if (round > 0)
@@ -254,40 +253,27 @@ __global__ void __launch_bounds__(kRowThreads, 2)
     }
     // every copy issued has landed before the block may exit
     if (lane == 0)
-      for (int s = 0; s < slots && s < issued; ++s) {
-        const int64_t last = s + ((issued - 1 - s) / slots) * slots;
-        mbar_wait_drain(full0 + 8 * s, (uint32_t)((last / slots) & 1), timeout_ns);
+      for (int s = 0; s < kRowSlots && s < issued; ++s) {
+        const int64_t last = s + ((issued - 1 - s) / kRowSlots) * kRowSlots;
+        mbar_wait_drain(full0 + 8 * s, (uint32_t)((last / kRowSlots) & 1), timeout_ns);
       }
   } else {
     // ------------------------------------------------------------ consumers
     const int nv = d / V;
     for (int64_t j = warp; j < n; j += kRowWarps) {
-      const int s = (int)(j % slots);
+      const int s = (int)(j % kRowSlots);
       int ok = 0;
       if (lane == 0)
-        ok = mbar_wait_bounded(full0 + 8 * s, (uint32_t)((j / slots) & 1), abort_v, err, timeout_ns);
+        ok = mbar_wait_bounded(full0 + 8 * s, (uint32_t)((j / kRowSlots) & 1), abort_v, err, timeout_ns);
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
-      // the row into registers (NCH 16-byte vectors per lane, kept packed so
-      // that two blocks fit an SM), then the slot is free
-      const uint4* xr = reinterpret_cast<const uint4*>(ring + (size_t)s * row_bytes);
-      uint4 raw[NCH];
-#pragma unroll
-      for (int c = 0; c < NCH; ++c) {
-        const int ci = c * 32 + lane;
-        if (ci < nv) raw[c] = xr[ci];
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(empty0 + 8 * s);   // the slot may be refilled
+      const T* xr = reinterpret_cast<const T*>(ring + (size_t)s * row_bytes);
       float sum = 0.f;
+      for (int ci = lane; ci < nv; ci += 32) {
+        float f[V];
+        load_vec(xr + ci * V, f);
 #pragma unroll
-      for (int c = 0; c < NCH; ++c) {
-        if (c * 32 + lane < nv) {
-          float f[V];
-          unpack16(raw[c], f, T());
-#pragma unroll
-          for (int k = 0; k < V; ++k) sum += RMS ? f[k] * f[k] : f[k];
-        }
+        for (int k = 0; k < V; ++k) sum += RMS ? f[k] * f[k] : f[k];
       }
       float mean = 0.f, rstd;
       if (RMS) {
@@ -295,24 +281,18 @@ __global__ void __launch_bounds__(kRowThreads, 2)
       } else {
         mean = warp_sum(sum) / d;
         float q = 0.f;
+        for (int ci = lane; ci < nv; ci += 32) {
+          float f[V];
+          load_vec(xr + ci * V, f);
 #pragma unroll
-        for (int c = 0; c < NCH; ++c) {
-          if (c * 32 + lane < nv) {
-            float f[V];
-            unpack16(raw[c], f, T());
-#pragma unroll
-            for (int k = 0; k < V; ++k) q += (f[k] - mean) * (f[k] - mean);
-          }
+          for (int k = 0; k < V; ++k) q += (f[k] - mean) * (f[k] - mean);
         }
         rstd = 1.f / sqrtf(warp_sum(q) / d + eps);
       }
       const int64_t m = lo + j;
-#pragma unroll
-      for (int c = 0; c < NCH; ++c) {
-        const int ci = c * 32 + lane;
-        if (ci >= nv) continue;
+      for (int ci = lane; ci < nv; ci += 32) {
         float f[V], g[V], bb[V], o[V];
-        unpack16(raw[c], f, T());
+        load_vec(xr + ci * V, f);
         load_vec(sp + ci * V, g);
         if (!RMS) load_vec(sp + d + ci * V, bb);
 #pragma unroll
@@ -326,6 +306,8 @@ __global__ void __launch_bounds__(kRowThreads, 2)
           store_vec(out2 + m * d + ci * V, o);
         }
       }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(empty0 + 8 * s);   // the slot may be refilled
     }
   }
 }
@@ -613,50 +595,32 @@ cudaError_t with_nch(int d, F f) {
   }
 }
 
-// Ring slots of the gather + norm kernel. Tuning override: ADADSF_ROW_SLOTS
-// (a multiple of 8 up to 64); default 16.
-int row_slots() {
-  static int v = -1;
-  if (v < 0) {
-    const char* e = getenv("ADADSF_ROW_SLOTS");
-    const int r = e ? atoi(e) : 0;
-    v = (r >= kRowWarps && r <= kRowSlotsMax && r % kRowWarps == 0) ? r : 16;
-  }
-  return v;
-}
-
 template <typename T, bool RMS>
 cudaError_t gather_norm_t(const void* x, const int32_t* rows, int64_t M, int d, const void* g1,
                           const void* b1, const void* g2, const void* b2, float eps, void* out1,
                           void* out2, const Dev& dev) {
   const size_t row_bytes = (size_t)d * sizeof(T);
-  const int slots = row_slots();
-  const size_t smem = 4 * row_bytes + slots * row_bytes + 2 * slots * 8;
-  if (smem > 232448 - 1024) return cudaErrorInvalidValue;
+  const size_t smem = 4 * row_bytes + kRowSlots * row_bytes + 2 * kRowSlots * 8;
+  static int attr_done[64] = {0};
+  int device = 0;
+  cudaGetDevice(&device);
+  if (device < 64 && !attr_done[device]) {
+    cudaError_t e = cudaFuncSetAttribute(gather_norm_tma_kernel<T, RMS>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (4 + kRowSlots) * kMaxRowBytes + 2 * kRowSlots * 8);
+    if (e != cudaSuccess) return e;
+    attr_done[device] = 1;
+  }
   // one wave: as many blocks per SM as fit (at most two), at least one row
   // per consumer warp
   const int64_t fit = std::max<int64_t>(1, std::min<int64_t>(2, 232448 / (int64_t)(smem + 1024)));
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>((M + kRowWarps - 1) / kRowWarps,
                                                              fit * dev.num_sms));
-  return with_nch<T>(d, [&](auto nch) -> cudaError_t {
-    constexpr int NCH = decltype(nch)::value;
-    // opt in to the dynamic shared memory this call needs (per device,
-    // grown as needed)
-    static size_t attr_bytes[64] = {0};
-    int device = 0;
-    cudaGetDevice(&device);
-    if (device >= 64 || attr_bytes[device] < smem) {
-      cudaError_t e = cudaFuncSetAttribute(gather_norm_tma_kernel<T, RMS, NCH>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-      if (e != cudaSuccess) return e;
-      if (device < 64) attr_bytes[device] = smem;
-    }
-    return launch_pdl(gather_norm_tma_kernel<T, RMS, NCH>, dim3((unsigned)grid), dim3(kRowThreads),
-                      smem, dev.stream, static_cast<const T*>(x), rows, M, d,
-                      static_cast<const T*>(g1), static_cast<const T*>(b1),
-                      static_cast<const T*>(g2), static_cast<const T*>(b2), eps,
-                      static_cast<T*>(out1), static_cast<T*>(out2), slots, dev.err, kWaitTimeoutNs);
-  });
+  return launch_pdl(gather_norm_tma_kernel<T, RMS>, dim3((unsigned)grid), dim3(kRowThreads), smem,
+                    dev.stream, static_cast<const T*>(x), rows, M, d, static_cast<const T*>(g1),
+                    static_cast<const T*>(b1), static_cast<const T*>(g2),
+                    static_cast<const T*>(b2), eps, static_cast<T*>(out1), static_cast<T*>(out2),
+                    dev.err, kWaitTimeoutNs);
 }
 
 cudaError_t gather_norm(int dtype, const void* x, const int32_t* rows, int64_t M, int d,
