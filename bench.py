@@ -225,6 +225,12 @@ def run_ours(args, rank, world, local_rank):
         c1.record(stream)
         torch.cuda.synchronize()
         calib_ms = c0.elapsed_time(c1)
+        # event profile of one calibration forward (the Eq. 4 statistics kernel)
+        acc.zero_()
+        A.adadsf_profile_begin(4 + 12 * L)
+        A.adadsf_sparse_model_forward(model, ids_cal, Kd, hid_cal, stats_acc=acc, ws=ws, stream=stream)
+        cal_recs = A.adadsf_profile_end(4 + 12 * L)
+        torch.cuda.synchronize()
         from paper_2607_21291_gb300 import calibrate as C
         acc = C.allreduce_stats(acc)          # the one exchange: 2L doubles over replicas
         s, r, K = C.retention_plan(acc, T, t_target, TAU, BETA)
@@ -343,6 +349,21 @@ def run_ours(args, rank, world, local_rank):
         a_["bytes"] += by
     tot_ms = sum(v["ms"] for v in agg.values())
     peaks, peak_src = load_peaks()
+    # the HBM-bound steps before the projections (router, Top-K, gather +
+    # norms) as one figure: their bytes over their time
+    hbm_names = [n for n in agg if n in ("router", "topk", "gather_norm", "topk_gather_norm")]
+    hbm_ms = sum(agg[n]["ms"] for n in hbm_names)
+    hbm_path = None
+    if hbm_ms > 0:
+        gbs = sum(agg[n]["bytes"] for n in hbm_names) / (hbm_ms * 1e6)
+        hbm_path = {"kernels": sorted(hbm_names), "gbs": gbs, "frac_of_hbm_peak": gbs / peaks["hbm_gbs"],
+                    "ms_per_step": hbm_ms / n_prof}
+    st = [r for r in cal_recs if r[0] == "stats" and r[2] > 0]
+    stats_kernel = None
+    if st:
+        st_ms, st_bytes = sum(r[2] for r in st), sum(r[4] for r in st)
+        stats_kernel = {"launches": len(st), "ms_per_launch": st_ms / len(st),
+                        "gbs": st_bytes / (st_ms * 1e6), "frac_of_hbm_peak": st_bytes / (st_ms * 1e6) / peaks["hbm_gbs"]}
     long_step = ms * args.steps > 1000.0
     tc_peak = peaks["bf16_tflops_sustained" if long_step else "bf16_tflops"]
     kernels = {}
@@ -413,7 +434,8 @@ def run_ours(args, rank, world, local_rank):
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clocks,
         "dense_same_kernels": {"ms_per_step": dense, "value": tokens / (dense * 1e-3), "unit": "tokens/s"},
-        "calibration": {"ms": calib_ms, "batch": list(wl.calib), "similarity": [float(x) for x in s],
+        "hbm_path": hbm_path,
+        "calibration": {"ms": calib_ms, "stats_kernel": stats_kernel, "batch": list(wl.calib), "similarity": [float(x) for x in s],
                         "ratios": [float(x) for x in r]},
         "normalized_flops": sparse_flops / max(1.0, sum(
             (2.0 * B * T * (shape.qkv_dim * shape.d + shape.d * shape.q_dim +
