@@ -3,9 +3,11 @@
 //
 // H = X W1^T is a [B T, d] x [64, d]^T product (tcgen05, M = 128 tokens,
 // N = 64 hidden units), cut into units of one 128-token tile x one 64-deep
-// k-block. The G CTAs take equal contiguous ranges of units, tile-major, so
-// every SM streams the same share of X whatever the number of tiles (for
-// few tokens, every tile is split along d over several CTAs). A tile whose
+// k-block. With at most one wave of tiles every CTA takes whole tiles (an
+// exchange of partial tiles costs more than it saves); with more tiles than
+// SMs the G CTAs take equal contiguous ranges of units, tile-major, so that
+// no partial last wave leaves SMs idle, and a range may end inside a tile
+// (the tile is then split along d). A tile whose
 // units span several CTAs is finished by the last of them to get there: the
 // others leave fp32 partial tiles in scratch (L2), and the finisher adds all
 // partials in CTA order, so the sum does not depend on timing. No CTA ever
