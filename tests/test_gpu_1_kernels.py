@@ -136,11 +136,15 @@ def test_router(A, shape, n):
 
 
 @pytest.mark.parametrize("shape,n", [(S.PYTHIA_160M, 2048), (S.PYTHIA_1_4B, 16384), (S.QWEN25_1_5B, 999),
-                                     (S.QWEN25_7B.replace(ffn=256), 4096)])
+                                     (S.QWEN25_7B.replace(ffn=256), 4096),
+                                     (S.QWEN25_7B.replace(ffn=256), 25600 - 77)])
 def test_router_split(A, shape, n):
-    """Router with room for scratch: 128-token tiles split along d over
-    several CTAs (partial tiles summed by the last CTA in a fixed order), so
-    two calls agree bit for bit and the tile counters end at zero."""
+    """Router with room for scratch. Up to one wave of 128-token tiles every
+    CTA takes whole tiles; past it (the last case: 200 tiles of d = 3584 on
+    the GPU's ~150 SMs) the CTAs take equal ranges of k-blocks, tiles are
+    split along d and the last CTA of a tile sums the partials in a fixed
+    order. Either way two calls agree bit for bit and the counters end at
+    zero."""
     W = H.host_layer(shape, 3)
     x = S.round_to(np.random.default_rng(n + 1).standard_normal((n, shape.d)).astype(np.float32), shape.dtype)
     w = A.to_device(W, H.tdtype(shape))
@@ -159,7 +163,8 @@ def test_router_split(A, shape, n):
     assert int(ws[256:256 + SYNC_BYTES].view(torch.int32).abs().sum()) == 0
 
 
-@pytest.mark.parametrize("shape,B,T,K", [(S.PYTHIA_160M, 4, 512, 256), (S.PYTHIA_1_4B, 8, 2048, 1024),
+@pytest.mark.parametrize("shape,B,T,K", [(S.PYTHIA_70M, 2, 128, 64),
+                                         (S.PYTHIA_160M, 4, 512, 256), (S.PYTHIA_1_4B, 8, 2048, 1024),
                                          (S.QWEN25_1_5B, 3, 333, 100), (S.PYTHIA_160M, 2, 100, 1),
                                          (S.PYTHIA_160M, 5, 64, 64), (S.PYTHIA_160M, 300, 1, 1),
                                          (S.QWEN25_7B.replace(ffn=256), 2, 4096, 2000), (S.PYTHIA_160M, 1, 16384, 777)])
