@@ -143,11 +143,13 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int nqb = (p.K + kQB - 1) / kQB;
-  // longest rows first
-  const int qb0 = p.pair ? 2 * ((nqb + 1) / 2 - 1 - (int)blockIdx.x) : nqb - 1 - (int)blockIdx.x;
+  // Block (h, b, z): blocks are dispatched in linear order (x fastest), so
+  // every head and sequence starts its longest rows (z = 0) before any
+  // shorter ones and the last wave holds the short ones.
+  const int qb0 = p.pair ? 2 * ((nqb + 1) / 2 - 1 - (int)blockIdx.z) : nqb - 1 - (int)blockIdx.z;
   const bool two = p.pair && qb0 + 1 < nqb;     // tile 1 holds query block qb0 + 1
   const int n_kv = two ? qb0 + 2 : qb0 + 1;     // tile 0 takes blocks 0..qb0, tile 1 all
-  const int h = blockIdx.y, b = blockIdx.z;
+  const int h = blockIdx.x, b = blockIdx.y;
   const int g = h / (p.Hq / p.Hkv);
   const int row0 = b * p.K;
 
@@ -484,7 +486,7 @@ cudaError_t launch_attn(const void* qkv, int64_t ld_qkv, const void* vt, int pad
   p.timeout_ns = kWaitTimeoutNs;
   const int nqb = (K + kQB - 1) / kQB;
   p.pair = (int64_t)((nqb + 1) / 2) * Hq * B >= dev.num_sms ? 1 : 0;
-  dim3 grid(p.pair ? (nqb + 1) / 2 : nqb, Hq, B);
+  dim3 grid(Hq, B, p.pair ? (nqb + 1) / 2 : nqb);
   return launch_pdl(attn_tc_kernel<HD>, grid, dim3(kAttnThreads), C::SMEM, dev.stream, tq, tv, p);
 }
 
