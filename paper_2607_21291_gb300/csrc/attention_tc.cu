@@ -440,20 +440,39 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 
 // V^T of every key-value head: vt[((b * Hkv + g) * hd + e) * pad + j] =
 // qkv[(b * K + j) * ld + col0 + g * hd + e]. Used when V^T is not produced by
-// the QKV projection itself.
-__global__ void vt_transpose_kernel(const bf16* qkv, int64_t ld, int col0, int B, int K, int Hkv,
-                                    int hd, int pad, bf16* vt) {
+// the QKV projection itself. Each block moves 32 x 32 tiles through shared
+// memory so that a warp reads 32 consecutive e of one row and writes 32
+// consecutive j of one output row; the blocks stride over all tiles.
+constexpr int kVtTile = 32;
+constexpr int kVtThreads = 256;
+
+__global__ void __launch_bounds__(kVtThreads)
+    vt_transpose_kernel(const bf16* qkv, int64_t ld, int col0, int B, int K, int Hkv, int hd,
+                        int pad, bf16* vt) {
+  __shared__ bf16 tile[kVtTile][kVtTile + 2];
   pdl_trigger();
   pdl_wait();
-  const int64_t n = (int64_t)B * Hkv * hd * K;
-  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
-       i += (int64_t)gridDim.x * blockDim.x) {
-    const int j = (int)(i % K);
-    const int64_t re = i / K;                       // (b * Hkv + g) * hd + e
-    const int e = (int)(re % hd);
-    const int64_t bg = re / hd;
-    const int g = (int)(bg % Hkv), b = (int)(bg / Hkv);
-    vt[re * pad + j] = qkv[((int64_t)b * K + j) * ld + col0 + g * hd + e];
+  constexpr int kRows = kVtThreads / kVtTile;
+  const int tx = threadIdx.x % kVtTile, ty = threadIdx.x / kVtTile;
+  const int ntj = (K + kVtTile - 1) / kVtTile, nte = (hd + kVtTile - 1) / kVtTile;
+  const int64_t ntiles = (int64_t)ntj * nte * B * Hkv;
+  for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x) {
+    const int j0 = (int)(t % ntj) * kVtTile;
+    const int64_t r = t / ntj;
+    const int e0 = (int)(r % nte) * kVtTile;
+    const int64_t bg = r / nte;                     // b * Hkv + g
+    const int g = (int)(bg % Hkv);
+    const int64_t b = bg / Hkv;
+    for (int jj = ty; jj < kVtTile; jj += kRows) {
+      const int j = j0 + jj, e = e0 + tx;
+      if (j < K && e < hd) tile[jj][tx] = qkv[(b * K + j) * ld + col0 + g * hd + e];
+    }
+    __syncthreads();
+    for (int ee = ty; ee < kVtTile; ee += kRows) {
+      const int e = e0 + ee, j = j0 + tx;
+      if (j < K && e < hd) vt[(bg * hd + e) * pad + j] = tile[tx][ee];
+    }
+    __syncthreads();
   }
 }
 
@@ -496,11 +515,11 @@ int vt_pad(int K) { return (K + 7) & ~7; }
 
 cudaError_t vt_from_qkv(const void* qkv, int64_t ld_qkv, int col0, int B, int K, int Hkv, int hd,
                         void* vt, const Dev& dev) {
-  const int64_t n = (int64_t)B * Hkv * hd * K;
-  if (n <= 0) return cudaSuccess;
-  const int64_t blocks = (n + 255) / 256;
-  return launch_pdl(vt_transpose_kernel, dim3((unsigned)(blocks < 65535 * 8 ? blocks : 65535 * 8)),
-                    dim3(256), 0, dev.stream, static_cast<const bf16*>(qkv), ld_qkv, col0, B, K, Hkv,
+  if ((int64_t)B * Hkv * hd * K <= 0) return cudaSuccess;
+  const int64_t tiles = (int64_t)((K + kVtTile - 1) / kVtTile) * ((hd + kVtTile - 1) / kVtTile) * B * Hkv;
+  const int64_t cap = 8 * (int64_t)dev.num_sms;   // 8 blocks of 256 threads per SM
+  return launch_pdl(vt_transpose_kernel, dim3((unsigned)std::min(tiles, cap)), dim3(kVtThreads), 0,
+                    dev.stream, static_cast<const bf16*>(qkv), ld_qkv, col0, B, K, Hkv,
                     hd, vt_pad(K), static_cast<bf16*>(vt));
 }
 
