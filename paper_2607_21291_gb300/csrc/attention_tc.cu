@@ -439,21 +439,23 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 }
 
 // V^T of every key-value head: vt[((b * Hkv + g) * hd + e) * pad + j] =
-// qkv[(b * K + j) * ld + col0 + g * hd + e]. Used when V^T is not produced by
-// the QKV projection itself. Each block moves 32 x 32 tiles through shared
-// memory so that a warp reads 32 consecutive e of one row and writes 32
-// consecutive j of one output row; the blocks stride over all tiles.
-constexpr int kVtTile = 32;
+// qkv[(b * K + j) * ld + col0 + g * hd + e]; the pad - K columns past the last
+// key get zeros where a 16-byte store reaches them. Used when V^T is not
+// produced by the QKV projection itself. Blocks stride over 64 x 64 tiles:
+// 16-byte loads along e (eight threads per 128-byte row piece) into shared
+// memory, then 16-byte stores along j. Needs hd, ld and col0 multiples of 8
+// and 16-byte aligned pointers (checked by the caller).
+constexpr int kVtTile = 64;
 constexpr int kVtThreads = 256;
+constexpr int kVtLd = kVtTile / 2 + 1;   // 32-bit words per shared row: odd, so column reads spread over banks
 
 __global__ void __launch_bounds__(kVtThreads)
     vt_transpose_kernel(const bf16* qkv, int64_t ld, int col0, int B, int K, int Hkv, int hd,
                         int pad, bf16* vt) {
-  __shared__ bf16 tile[kVtTile][kVtTile + 2];
+  __shared__ uint32_t tile[kVtTile * kVtLd];   // [j][e], two bf16 per word
   pdl_trigger();
   pdl_wait();
-  constexpr int kRows = kVtThreads / kVtTile;
-  const int tx = threadIdx.x % kVtTile, ty = threadIdx.x / kVtTile;
+  const uint16_t* tile16 = reinterpret_cast<const uint16_t*>(tile);
   const int ntj = (K + kVtTile - 1) / kVtTile, nte = (hd + kVtTile - 1) / kVtTile;
   const int64_t ntiles = (int64_t)ntj * nte * B * Hkv;
   for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x) {
@@ -463,14 +465,33 @@ __global__ void __launch_bounds__(kVtThreads)
     const int64_t bg = r / nte;                     // b * Hkv + g
     const int g = (int)(bg % Hkv);
     const int64_t b = bg / Hkv;
-    for (int jj = ty; jj < kVtTile; jj += kRows) {
-      const int j = j0 + jj, e = e0 + tx;
-      if (j < K && e < hd) tile[jj][tx] = qkv[(b * K + j) * ld + col0 + g * hd + e];
+    for (int c = threadIdx.x; c < kVtTile * 8; c += kVtThreads) {
+      const int jj = c >> 3, ec = (c & 7) * 8;
+      const int j = j0 + jj, e = e0 + ec;
+      if (j < K && e + 8 <= hd) {
+        const uint4 v = *reinterpret_cast<const uint4*>(qkv + (b * K + j) * ld + col0 + g * hd + e);
+        uint32_t* w = tile + jj * kVtLd + ec / 2;
+        w[0] = v.x;
+        w[1] = v.y;
+        w[2] = v.z;
+        w[3] = v.w;
+      }
     }
     __syncthreads();
-    for (int ee = ty; ee < kVtTile; ee += kRows) {
-      const int e = e0 + ee, j = j0 + tx;
-      if (j < K && e < hd) vt[(bg * hd + e) * pad + j] = tile[tx][ee];
+    for (int c = threadIdx.x; c < kVtTile * 8; c += kVtThreads) {
+      const int ee = c >> 3, jc = (c & 7) * 8;
+      const int e = e0 + ee, j = j0 + jc;
+      if (e < hd && j < K) {
+        uint32_t o[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int ja = jc + 2 * i;
+          const uint32_t lo = j0 + ja < K ? tile16[ja * 2 * kVtLd + ee] : 0u;
+          const uint32_t hi = j0 + ja + 1 < K ? tile16[(ja + 1) * 2 * kVtLd + ee] : 0u;
+          o[i] = lo | (hi << 16);
+        }
+        *reinterpret_cast<uint4*>(vt + (bg * hd + e) * pad + j) = make_uint4(o[0], o[1], o[2], o[3]);
+      }
     }
     __syncthreads();
   }
@@ -516,6 +537,9 @@ int vt_pad(int K) { return (K + 7) & ~7; }
 cudaError_t vt_from_qkv(const void* qkv, int64_t ld_qkv, int col0, int B, int K, int Hkv, int hd,
                         void* vt, const Dev& dev) {
   if ((int64_t)B * Hkv * hd * K <= 0) return cudaSuccess;
+  if (hd % 8 || ld_qkv % 8 || col0 % 8 || (reinterpret_cast<uintptr_t>(qkv) & 15) ||
+      (reinterpret_cast<uintptr_t>(vt) & 15))
+    return cudaErrorInvalidValue;
   const int64_t tiles = (int64_t)((K + kVtTile - 1) / kVtTile) * ((hd + kVtTile - 1) / kVtTile) * B * Hkv;
   const int64_t cap = 8 * (int64_t)dev.num_sms;   // 8 blocks of 256 threads per SM
   return launch_pdl(vt_transpose_kernel, dim3((unsigned)std::min(tiles, cap)), dim3(kVtThreads), 0,
