@@ -156,9 +156,16 @@ def round_to(a: np.ndarray, dtype: str) -> np.ndarray:
     a = np.ascontiguousarray(a, dtype=np.float32)
     if dtype == "f32":
         return a.copy()
-    u = a.view(np.uint32).astype(np.uint64)
+    u = a.view(np.uint32)
+    # In place on one uint32 array: u + 0x7FFF + (bit 16 of u), low half
+    # cleared. Finite inputs cannot wrap (largest 0xFF7FFFFF + 0x8000); NaNs
+    # may, and are replaced below.
+    r = (u >> 16) & np.uint32(1)
+    r += np.uint32(0x7FFF)
+    r += u
+    r &= np.uint32(0xFFFF0000)
+    out = r.view(np.float32)
     nan = np.isnan(a)
-    r = ((u + 0x7FFF + ((u >> 16) & 1)) >> 16) << 16
-    r = r.astype(np.uint32).view(np.float32)
-    r = np.where(nan, np.float32(np.nan), r)
-    return r.astype(np.float32)
+    if nan.any():
+        out[nan] = np.float32(np.nan)
+    return out
