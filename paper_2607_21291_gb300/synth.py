@@ -160,7 +160,7 @@ def round_to(a: np.ndarray, dtype: str) -> np.ndarray:
     # In place on one uint32 array: u + 0x7FFF + (bit 16 of u), low half
     # cleared. Finite inputs cannot wrap (largest 0xFF7FFFFF + 0x8000); NaNs
     # may, and are replaced below.
-    r = (u >> 16) & np.uint32(1)
+    r = np.asarray((u >> 16) & np.uint32(1))   # an array also for 0-d input
     r += np.uint32(0x7FFF)
     r += u
     r &= np.uint32(0xFFFF0000)
