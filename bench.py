@@ -448,6 +448,23 @@ def run_ours(args, rank, world, local_rank):
     print(json.dumps(out), flush=True)
 
 
+def host_threads() -> int:
+    """Threads the oracle's NumPy BLAS runs with: threadpoolctl's report where
+    it is installed, else the CPUs this process may run on (OpenBLAS's
+    default)."""
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i["num_threads"] for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return max(n)
+    except ImportError:
+        pass
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
 def cpu_baseline(model, shape, K, ids, budget_s=20.0):
     """The fp64 oracle as it stands on the host cores, on a bounded sample of the
     same workload: sequence after sequence, layer after layer (each layer's
@@ -477,7 +494,7 @@ def cpu_baseline(model, shape, K, ids, budget_s=20.0):
         if spent > budget_s:
             break
     per_layer_seq = spent / n_evals
-    return {"value": T / (per_layer_seq * L), "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+    return {"value": T / (per_layer_seq * L), "unit": "tokens/s", "cores": host_threads(), "kind": "oracle",
             "sample": f"{n_evals} (sequence, layer) evaluations over {seqs} of {B} sequences x {T} tokens, "
                       f"fp64 NumPy (BLAS threads = host cores), {spent:.1f} s; rate extrapolated to all "
                       f"{L} layers"}
@@ -520,7 +537,7 @@ def run_reference(args, rank, world):
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": wl.name, "model": shape.name, "B": 1, "T": T, "layers": L,
                    "retention_target": t_target, "K_per_layer": K},
-        "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+        "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": host_threads(), "kind": "oracle",
                          "sample": f"1 sequence x {T} tokens per step through all {L} layers"},
         "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
