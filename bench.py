@@ -9,8 +9,9 @@ assigns from a dense calibration pass. The calibration pass and the
 allocation run once before timing (the retention is fixed across steps) and
 are reported separately.
 
-Prints ONE JSON line on rank 0. Default workload: the 12-layer Pythia-160M
-shape, B=4, T=512, bf16, mean retention 0.5.
+Prints ONE JSON line on rank 0. Default workload: the 28-layer Qwen2.5-7B
+shape, B=16, T=4096, bf16, mean retention 0.5 (calibration over 16 x 4096
+tokens), with the retention sweep 1.0 / 0.75 / 0.25 in the same line.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c2|c3|c4|c5]
   python bench.py --impl reference ...   (the fp64 CPU oracle, same metric)
@@ -22,6 +23,7 @@ from __future__ import annotations
 import argparse
 import hashlib
 import json
+import math
 import os
 import re
 import statistics
@@ -160,43 +162,51 @@ def retention_of(args, wl):
 
 
 # ----------------------------------------------------------------------------- model set-up
+WEIGHT_SEED, CALIB_SEED, EVAL_SEED = 2, 1, 2
+RECIPE = ("counter-based draws (synth.bench_*): linear weights and biases N(0, 0.02), norm gains 1, "
+          "norm biases 0, weight seed 2; token ids uniform over the vocabulary, calibration seed 1, "
+          "evaluation seed 2")
+L2_NOTE = ("GPU arm: L2 flushed between timed steps (256 MiB write outside the step events); "
+           "CPU oracle arm: each step's fp64 layer weights exceed every host cache")
+
+
+def rank_seed(seed, rank):
+    return seed + 7919 * rank
+
+
 def device_model(A, shape, seed, device):
-    """Random-init weights of the backbone shape, drawn on the device (recipe of
-    synth: linear weights and biases N(0, 0.02), norm gains 1, norm biases 0)."""
+    """Random-init weights of the backbone shape in the benchmark recipe,
+    drawn on the device (the reference arm draws the same tensors)."""
     td = torch.bfloat16 if shape.dtype == "bf16" else torch.float32
-    gen = torch.Generator(device=device)
-
-    def draw(tag, shp, std):
-        gen.manual_seed(seed * 1000003 + tag)
-        return (torch.randn(shp, generator=gen, device=device, dtype=torch.float32) * std).to(td)
-
-    layers = []
-    for l in range(shape.n_layers):
-        w = {}
-        for j, (name, shp) in enumerate(S.layer_weight_shapes(shape).items()):
-            if name in ("ln1_w", "ln2_w"):
-                w[name] = torch.ones(shp, device=device, dtype=td)
-            elif name in ("ln1_b", "ln2_b"):
-                w[name] = torch.zeros(shp, device=device, dtype=td)
-            else:
-                w[name] = draw(l * 64 + j, shp, 0.02)
-        layers.append(w)
-    extra = {"embed": draw(10 ** 6, (shape.vocab, shape.d), 0.02),
+    layers = [{k: v.to(td) for k, v in S.bench_layer_weights(shape, seed, l, device).items()}
+              for l in range(shape.n_layers)]
+    extra = {"embed": S.bench_embed(shape, seed, device).to(td),
              "final_w": torch.ones(shape.d, device=device, dtype=td)}
     if shape.arch == S.NEOX:
         extra["final_b"] = torch.zeros(shape.d, device=device, dtype=td)
     return A.DeviceModel(A.make_cfg(shape), layers, extra)
 
 
-def device_ids(seed, B, T, vocab, device):
-    gen = torch.Generator(device=device)
-    gen.manual_seed(seed)
-    return torch.randint(0, vocab, (B, T), generator=gen, device=device, dtype=torch.int32)
+def shared_config(wl, t_target, world):
+    """The workload's definition: identical in both arms' JSON lines."""
+    shape = wl.shape
+    return {"workload": wl.name, "model": shape.name, "B": wl.B, "T": wl.T, "layers": shape.n_layers,
+            "global_batch": wl.B * world, "seq_len": wl.T, "retention_target": t_target,
+            "tau": TAU, "beta": BETA, "calibration_batch": list(wl.calib), "inputs": RECIPE,
+            "parallelism": f"replicas x{world} (batch-sharded, no collective)", "l2": L2_NOTE}
+
+
+def dense_flops_per_layer(shape, B, T):
+    """GEMM + causal-attention flops of one dense layer over B sequences of T."""
+    per_tok = 2.0 * (shape.qkv_dim * shape.d + shape.d * shape.q_dim
+                     + (3 if shape.arch == S.QWEN else 2) * shape.d * shape.ffn)
+    return B * T * per_tok + 2.0 * B * shape.n_heads * shape.head_dim * T * (T + 1)
 
 
 # ----------------------------------------------------------------------------- our arm
 def run_ours(args, rank, world, local_rank):
     from paper_2607_21291_gb300 import adadsf as A
+    from paper_2607_21291_gb300 import calibrate as C
     A.lib()
     device = torch.device("cuda", local_rank)
     torch.cuda.set_device(device)
@@ -205,12 +215,13 @@ def run_ours(args, rank, world, local_rank):
     L = shape.n_layers
     t_target = retention_of(args, wl)
     stream = torch.cuda.Stream(device)
-    model = device_model(A, shape, 2, device)
+    model = device_model(A, shape, WEIGHT_SEED, device)
     sampler = ClockSampler(gpu_id_for_smi(local_rank))
+    n_rec = 4 + 12 * L
 
     with torch.cuda.stream(stream):
         # ---- calibration (Eq. 4, dense forward) + allocation (Eqs. 5-8), once
-        ids_cal = device_ids(1 + 7919 * rank, *wl.calib, shape.vocab, device)
+        ids_cal = S.counter_ids(rank_seed(CALIB_SEED, rank), *wl.calib, shape.vocab, device)
         Kd = [T] * L
         ws = A.workspace(max(A.adadsf_model_workspace_size(model.cfg, max(B, wl.calib[0]), T, Kd, True), 256), device)
         acc = torch.zeros(2 * L, dtype=torch.float64, device=device)
@@ -227,27 +238,29 @@ def run_ours(args, rank, world, local_rank):
         calib_ms = c0.elapsed_time(c1)
         # event profile of one calibration forward (the Eq. 4 statistics kernel)
         acc.zero_()
-        A.adadsf_profile_begin(4 + 12 * L)
+        A.adadsf_profile_begin(n_rec)
         A.adadsf_sparse_model_forward(model, ids_cal, Kd, hid_cal, stats_acc=acc, ws=ws, stream=stream)
-        cal_recs = A.adadsf_profile_end(4 + 12 * L)
-        torch.cuda.synchronize()
-        from paper_2607_21291_gb300 import calibrate as C
+        cal_recs = A.adadsf_profile_end(n_rec)
         acc = C.allreduce_stats(acc)          # the one exchange: 2L doubles over replicas
-        s, r, K = C.retention_plan(acc, T, t_target, TAU, BETA)
-        K = [int(k) for k in K]
+        plans = {}
+        for t in sorted(set((t_target,) + tuple(wl.retention))):
+            s_, r_, K_ = C.retention_plan(acc, T, t, TAU, BETA)
+            plans[t] = (s_, r_, [int(k) for k in K_])
+        s, r, K = plans[t_target]
+        del hid_cal
 
-        # spin-up: keep the GPU busy ~1.5 s so its clocks leave the idle state
-        # before anything is measured (the calibration forward, repeated)
+        # spin-up: keep the GPU busy before anything is measured, so its
+        # clocks leave the idle state (the calibration forward, repeated)
         spin_t0 = time.time()
         spin_n = 0
+        spin_out = torch.empty((wl.calib[0], T, shape.d), dtype=torch.bfloat16, device=device)
         while time.time() - spin_t0 < args.spin_up:
-            A.adadsf_sparse_model_forward(model, ids_cal, Kd, hid_cal, ws=ws, stream=stream)
+            A.adadsf_sparse_model_forward(model, ids_cal, Kd, spin_out, ws=ws, stream=stream)
             spin_n += 1
-            if spin_n % 8 == 0:
-                torch.cuda.synchronize()
-        torch.cuda.synchronize()
+            torch.cuda.synchronize()
+        del spin_out
 
-        ids = device_ids(2 + 7919 * rank, B, T, shape.vocab, device)
+        ids = S.counter_ids(rank_seed(EVAL_SEED, rank), B, T, shape.vocab, device)
         hidden = torch.empty((B, T, shape.d), dtype=torch.bfloat16, device=device)
         flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
 
@@ -259,36 +272,34 @@ def run_ours(args, rank, world, local_rank):
             fwd(K)
         torch.cuda.synchronize()
         n_prof = max(3, min(10, args.steps))
-        A.adadsf_profile_begin((4 + 12 * L) * n_prof)
+        A.adadsf_profile_begin(n_rec * n_prof)
         for _ in range(n_prof):
             flush.zero_()
             torch.cuda.nvtx.range_push("adadsf_sparse_step")
             fwd(K)
             torch.cuda.nvtx.range_pop()
-        recs = A.adadsf_profile_end((4 + 12 * L) * n_prof)
-        bad = [r for r in recs if r[2] < 0]
+        recs = A.adadsf_profile_end(n_rec * n_prof)
+        bad = [x for x in recs if x[2] < 0]
         assert not bad, f"launch timing failed: {bad[:3]}"
         assert A.adadsf_sync_check(ws, stream) == A.OK, A.adadsf_last_error()
         launches_per_step = len(recs) // n_prof
 
-        # ---- CUDA graphs of the sparse and the dense forward
-        graphs = {}
-        for name, Ks in (("sparse", K), ("dense", Kd)):
+        def capture(Ks):
             for _ in range(max(3, args.warmup)):
                 fwd(Ks)
             torch.cuda.synchronize()
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g, stream=stream):
                 fwd(Ks)
-            graphs[name] = g
-        torch.cuda.synchronize()
+            torch.cuda.synchronize()
+            return g
 
-        def time_graph(g, steps, warmup):
+        def time_graph(g, steps, warmup, barrier=False):
             for _ in range(warmup):
                 flush.zero_()
                 g.replay()
             ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
-            if world > 1:
+            if barrier and world > 1:
                 torch.distributed.barrier()
             torch.cuda.synchronize()
             t0 = time.time()
@@ -299,12 +310,36 @@ def run_ours(args, rank, world, local_rank):
                 e1.record(stream)
             torch.cuda.synchronize()
             t1 = time.time()
-            if world > 1:
+            if barrier and world > 1:
                 torch.distributed.barrier()
             return [e0.elapsed_time(e1) for e0, e1 in ev], t0, t1
 
-        dense_ms, _, _ = time_graph(graphs["dense"], max(3, args.steps // 4), args.warmup)
-        step_ms, t0, t1 = time_graph(graphs["sparse"], args.steps, args.warmup)
+        # ---- the timed region: the sparse forward at the target retention
+        g_sparse = capture(K)
+        step_ms, t0, t1 = time_graph(g_sparse, args.steps, args.warmup, barrier=True)
+        clocks = sampler.stop(t0, t1)
+        assert A.adadsf_sync_check(ws, stream) == A.OK, A.adadsf_last_error()
+        del g_sparse
+
+        # ---- the dense forward on the same kernels, and the retention sweep
+        n_side = max(3, args.steps // 4)
+        g_dense = capture(Kd)
+        dense_ms, _, _ = time_graph(g_dense, n_side, 2)
+        del g_dense
+        sweep = {}
+        for t, (_, _, Kt) in sorted(plans.items()):
+            if t == t_target:
+                continue
+            if all(k == T for k in Kt):
+                ms_t = dense_ms
+            else:
+                g_t = capture(Kt)
+                ms_t, _, _ = time_graph(g_t, n_side, 2)
+                del g_t
+            mt = float(np.mean(ms_t))
+            sweep[f"{t:g}"] = {"ms_per_step": mt, "value": B * T * world / (mt * 1e-3), "unit": "tokens/s",
+                               "K_per_layer": Kt, "retention_mean": float(np.mean(Kt)) / T, "steps": len(ms_t),
+                               "dense": all(k == T for k in Kt)}
         assert A.adadsf_sync_check(ws, stream) == A.OK, A.adadsf_last_error()
 
         # ---- end to end through the public call, host buffers in and out
@@ -327,14 +362,13 @@ def run_ours(args, rank, world, local_rank):
         torch.cuda.synchronize()
         e2e_ms = [e0.elapsed_time(e1) for e0, e1 in e2e_ev]
 
-    clocks = sampler.stop(t0, t1)
     ms = float(np.mean(step_ms))
     e2e = float(np.mean(e2e_ms))
     dense = float(np.mean(dense_ms))
     if world > 1:
-        t = torch.tensor([ms, e2e, dense], device=device, dtype=torch.float64)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms, e2e, dense = t.tolist()
+        tt = torch.tensor([ms, e2e, dense], device=device, dtype=torch.float64)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        ms, e2e, dense = tt.tolist()
     if rank != 0:
         return
 
@@ -358,14 +392,15 @@ def run_ours(args, rank, world, local_rank):
         gbs = sum(agg[n]["bytes"] for n in hbm_names) / (hbm_ms * 1e6)
         hbm_path = {"kernels": sorted(hbm_names), "gbs": gbs, "frac_of_hbm_peak": gbs / peaks["hbm_gbs"],
                     "ms_per_step": hbm_ms / n_prof}
-    st = [r for r in cal_recs if r[0] == "stats" and r[2] > 0]
+    st = [x for x in cal_recs if x[0] == "stats" and x[2] > 0]
     stats_kernel = None
     if st:
-        st_ms, st_bytes = sum(r[2] for r in st), sum(r[4] for r in st)
+        st_ms, st_bytes = sum(x[2] for x in st), sum(x[4] for x in st)
         stats_kernel = {"launches": len(st), "ms_per_launch": st_ms / len(st),
                         "gbs": st_bytes / (st_ms * 1e6), "frac_of_hbm_peak": st_bytes / (st_ms * 1e6) / peaks["hbm_gbs"]}
     long_step = ms * args.steps > 1000.0
-    tc_peak = peaks["bf16_tflops_sustained" if long_step else "bf16_tflops"]
+    tc_key = "bf16_tflops_sustained" if long_step else "bf16_tflops"
+    tc_peak = peaks[tc_key]
     kernels = {}
     for name, v in sorted(agg.items(), key=lambda kv: -kv[1]["ms"]):
         per = v["launches"] / n_prof
@@ -377,7 +412,7 @@ def run_ours(args, rank, world, local_rank):
             k["gbs"] = v["bytes"] / (v["ms"] * 1e6)
             k["frac_of_hbm_peak"] = k["gbs"] / peaks["hbm_gbs"]
         kernels[name] = k
-    # the dominant kernel binary is the tcgen05 GEMM (qkv/o/up/down/router share it)
+    # the dominant kernel binary is the tcgen05 GEMM (QKV / output / MLP projections)
     gemm_names = [n for n in agg if n.startswith("gemm_")]
     gemm_ms = sum(agg[n]["ms"] for n in gemm_names)
     top = max(agg, key=lambda n: agg[n]["ms"])
@@ -385,10 +420,9 @@ def run_ours(args, rank, world, local_rank):
         launches = sum(agg[n]["launches"] for n in gemm_names)
         flops = sum(agg[n]["flops"] for n in gemm_names)
         achieved = flops / (gemm_ms * 1e9)
-        roof = {"kernel": "gemm_tc_kernel (tcgen05 projections: " + ",".join(sorted(gemm_names)) + ")",
+        roof = {"kernel": "tcgen05 projection GEMMs (" + ",".join(sorted(gemm_names)) + ")",
                 "bound": "tensor", "achieved": achieved, "peak": tc_peak, "unit": "TFLOP/s",
-                "frac": achieved / tc_peak,
-                "peak_source": f"{peak_src} {'bf16_tflops_sustained' if long_step else 'bf16_tflops'}",
+                "frac": achieved / tc_peak, "peak_source": f"{peak_src} {tc_key}",
                 "avg_launch_ms": gemm_ms / launches,
                 "traffic": recorded_traffic("gemm", wl.name)}
     else:
@@ -419,13 +453,14 @@ def run_ours(args, rank, world, local_rank):
         "vs_baseline": None,
         "dtype": "bf16" if shape.dtype == "bf16" else "f32",
         "data": "synthetic (seeded token ids, random-init weights of the backbone shape)",
-        "config": {"workload": wl.name, "model": shape.name, "B": B, "T": T, "layers": L,
-                   "global_batch": B * world, "seq_len": T, "retention_target": t_target,
-                   "K_per_layer": K, "retention_mean": float(np.mean(K)) / T,
-                   "tau": TAU, "beta": BETA, "parallelism": f"replicas x{world} (batch-sharded, no collective)",
-                   "l2": "flushed between timed steps (256 MiB write outside the step events)",
-                   "spin_up": f"{spin_n} dense forwards over {args.spin_up:.1f} s before any measurement",
-                   "timing": "CUDA graph replay of adadsf_sparse_model_forward, CUDA events per step"},
+        "config": shared_config(wl, t_target, world),
+        "timing": {"how": "CUDA graph replay of adadsf_sparse_model_forward, CUDA events per step on the "
+                          "launching stream",
+                   "spin_up": f"{spin_n} dense forwards over {args.spin_up:.1f} s before any measurement"},
+        "retention_plan": {"K_per_layer": K, "retention_mean": float(np.mean(K)) / T,
+                           "similarity": [float(x) for x in s], "ratios": [float(x) for x in r],
+                           "calibration": f"dense forward with Eq. 4 statistics over {wl.calib[0]} x {wl.calib[1]} "
+                                          f"tokens per replica on this GPU, summed over {world} replica(s)"},
         "roofline": roof,
         "e2e": {"value": tokens / (e2e * 1e-3), "unit": "tokens/s",
                 "h2d_bytes_per_step": int(ids.numel() * ids.element_size()),
@@ -433,15 +468,18 @@ def run_ours(args, rank, world, local_rank):
                 "how": "eager adadsf_sparse_model_forward per step with pinned-host ids in and hidden states out"},
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clocks,
-        "dense_same_kernels": {"ms_per_step": dense, "value": tokens / (dense * 1e-3), "unit": "tokens/s"},
+        "dense_same_kernels": {"ms_per_step": dense, "value": tokens / (dense * 1e-3), "unit": "tokens/s",
+                               "steps": n_side},
+        "retention_sweep": sweep,
         "hbm_path": hbm_path,
-        "calibration": {"ms": calib_ms, "stats_kernel": stats_kernel, "batch": list(wl.calib), "similarity": [float(x) for x in s],
-                        "ratios": [float(x) for x in r]},
-        "normalized_flops": sparse_flops / max(1.0, sum(
-            (2.0 * B * T * (shape.qkv_dim * shape.d + shape.d * shape.q_dim +
-                            (3 if shape.arch == S.QWEN else 2) * shape.d * shape.ffn) +
-             2.0 * B * shape.n_heads * shape.head_dim * T * (T + 1)) for _ in range(L))),
+        "calibration": {"ms": calib_ms, "stats_kernel": stats_kernel, "batch": list(wl.calib)},
+        "normalized_flops": sparse_flops / max(1.0, L * dense_flops_per_layer(shape, B, T)),
         "kernels": kernels,
+        "kernels_vs_step": {"sum_ms_per_step": tot_ms / n_prof, "graph_ms_per_step": ms,
+                            "ratio": tot_ms / n_prof / ms,
+                            "how": "kernels: an eager pass with CUDA events around every launch (no overlap "
+                                   "between launches); graph: the timed replay, where each launch's prologue "
+                                   "overlaps the previous one (programmatic dependent launch)"},
     }
     if world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(model, shape, K, ids, budget_s=args.cpu_budget)
@@ -465,80 +503,153 @@ def host_threads() -> int:
         return os.cpu_count() or 1
 
 
+# ----------------------------------------------------------------------------- the oracle on the host
+def _f64(t):
+    return t.float().cpu().numpy().astype(np.float64)
+
+
+def layer_order(L: int):
+    """Layers in an order that spreads any prefix over the depth (a stride
+    coprime with L)."""
+    stride = max(1, round(L * 0.618))
+    while math.gcd(stride, L) != 1:
+        stride += 1
+    return [(j * stride) % L for j in range(L)]
+
+
+def oracle_sample(shape, K, ids_host, layer_weights, budget_s, max_evals=None):
+    """Times the oracle's sparse layer (Sec. 3.4) on (sequence, layer) pairs of
+    the workload: sequences in turn, layers spread over the depth, until
+    budget_s seconds of oracle time (or max_evals pairs). layer_weights(l)
+    returns layer l's weights as fp64 NumPy arrays (drawn outside the timing);
+    the layer input is the sequence's embedding. Returns (seconds per pair,
+    pairs, sequences touched)."""
+    from oracle import adadsf_oracle as O
+    p = O.params_of(shape)
+    B = ids_host.shape[0]
+    order = layer_order(shape.n_layers)
+    spent, times, seqs = 0.0, [], set()
+    j = 0
+    while spent < budget_s and (max_evals is None or j < max_evals):
+        b = j % B
+        l = order[j % len(order)]
+        W = layer_weights(l)
+        x = _f64(S.round_to_torch(S.bench_embed_rows(shape, WEIGHT_SEED, ids_host[b:b + 1]), shape.dtype))
+        t0 = time.time()
+        O.sparse_layer_forward(x, W, p, K[l])
+        dt = time.time() - t0
+        times.append(dt)
+        spent += dt
+        seqs.add(b)
+        j += 1
+    return float(np.mean(times)), len(times), len(seqs)
+
+
 def cpu_baseline(model, shape, K, ids, budget_s=20.0):
     """The fp64 oracle as it stands on the host cores, on a bounded sample of the
-    same workload: sequence after sequence, layer after layer (each layer's
-    weights copied to the host when first used), until about budget_s; the
-    rate is extrapolated to all layers from the mean time of one layer on one
-    sequence."""
-    from oracle import adadsf_oracle as O
-    to = lambda t: t.float().cpu().numpy().astype(np.float64)
-    p = O.params_of(shape)
-    ids_h = ids.cpu().numpy()
-    B, T = ids_h.shape
+    same workload (the GPU arm's weights and kept counts), extrapolated to all
+    layers."""
+    T = ids.shape[1]
     L = shape.n_layers
-    host = {}
-    spent, n_evals, seqs = 0.0, 0, 0
-    for b in range(B):
-        x = to(model.extra["embed"][ids[b:b + 1].long()])
-        for l in range(L):
-            if l not in host:
-                host[l] = {k: to(v) for k, v in model.layers[l].items()}
-            t0 = time.time()
-            x, _, _ = O.sparse_layer_forward(x, host[l], p, K[l])
-            spent += time.time() - t0
-            n_evals += 1
-            if spent > budget_s:
-                break
-        seqs += 1
-        if spent > budget_s:
-            break
-    per_layer_seq = spent / n_evals
-    return {"value": T / (per_layer_seq * L), "unit": "tokens/s", "cores": host_threads(), "kind": "oracle",
-            "sample": f"{n_evals} (sequence, layer) evaluations over {seqs} of {B} sequences x {T} tokens, "
-                      f"fp64 NumPy (BLAS threads = host cores), {spent:.1f} s; rate extrapolated to all "
-                      f"{L} layers"}
+    cache = {}
+
+    def weights(l):
+        if l not in cache:
+            cache.clear()
+            cache[l] = {k: _f64(v) for k, v in model.layers[l].items()}
+        return cache[l]
+
+    per, n, seqs = oracle_sample(shape, K, ids.cpu(), weights, budget_s)
+    return {"value": T / (per * L), "unit": "tokens/s", "cores": host_threads(), "kind": "oracle",
+            "sample": f"{n} (sequence, layer) evaluations of the oracle's sparse layer over {seqs} of "
+                      f"{ids.shape[0]} sequences x {T} tokens at this line's K_l, layers spread over the depth, "
+                      f"{per:.2f} s each on average; rate extrapolated to all {L} layers (fp64 NumPy, BLAS threads = "
+                      f"host cores)"}
 
 
 # ----------------------------------------------------------------------------- reference arm
+def reference_calibration(shape, wl, layer_weights, flop_budget=2e12):
+    """Eq. 4 statistics of the dense model with the oracle on a bounded prefix
+    of the calibration batch (the first n tokens of its first sequences, n
+    sized to about flop_budget fp64 flops), then Eqs. 5-8 at the workload's
+    full T. Returns (s, n_sequences, n_tokens)."""
+    from oracle import adadsf_oracle as O
+    p = O.params_of(shape)
+    L = shape.n_layers
+    per_tok = dense_flops_per_layer(shape, 1, 1) - 4.0 * shape.n_heads * shape.head_dim
+    n_tok = int(max(128, min(wl.calib[0] * wl.calib[1], flop_budget / (L * per_tok))))
+    n_seq = max(1, min(wl.calib[0], n_tok // wl.calib[1]))
+    n_len = min(wl.calib[1], n_tok)
+    ids = S.counter_ids(CALIB_SEED, *wl.calib, shape.vocab)[:n_seq, :n_len]
+    x = _f64(S.round_to_torch(S.bench_embed_rows(shape, WEIGHT_SEED, ids), shape.dtype))
+    s = []
+    for l in range(L):
+        W = layer_weights(l)
+        x_new, _, _ = O.sparse_layer_forward(x, W, p, n_len)
+        s.append(O.similarity(O.cos_sim_stat(x, x_new)))
+        x = x_new
+    return np.array(s), n_seq, n_len
+
+
 def run_reference(args, rank, world):
-    """The fp64 CPU oracle timed on the host cores: each step pushes one
-    sequence of the workload through every sparse layer."""
+    """The fp64 CPU oracle timed on the host cores: each step is one bounded
+    sample of the workload -- the oracle's sparse layer on one sequence of the
+    batch, layers spread over the depth -- and the rate is extrapolated to the
+    whole model. The kept counts come from the oracle's own Eq. 4 statistics
+    on a bounded prefix of the calibration batch."""
     if rank != 0:
         return
     from oracle import adadsf_oracle as O
     wl = S.WORKLOADS[args.workload]
-    shape, T = wl.shape, wl.T
+    shape, B, T = wl.shape, wl.B, wl.T
     L = shape.n_layers
     t_target = retention_of(args, wl)
-    layers = [{k: S.round_to(v, shape.dtype).astype(np.float64)
-               for k, v in S.layer_weights(shape, 2, l, gain_std=0.0).items()} for l in range(L)]
-    extra = {k: S.round_to(v, shape.dtype).astype(np.float64)
-             for k, v in S.model_extra_weights(shape, 2, gain_std=0.0).items()}
-    p = O.params_of(shape)
-    ids_cal = S.token_ids(1, 1, T, shape.vocab)
-    _, _, st = O.sparse_model_forward(ids_cal, extra, layers, p, [T] * L, stats_mode="token")
-    s = np.array([O.similarity(a) for a in st])
+    # inputs: the same counter-based draws as the GPU arm; drawn with PyTorch
+    # on the GPU when one is present (seconds instead of minutes), the
+    # oracle's arithmetic always on the host
+    gen = "cuda" if torch.cuda.is_available() else "cpu"
+    td = torch.bfloat16 if shape.dtype == "bf16" else torch.float32
+
+    def layer_weights(l):
+        return {k: _f64(v.to(td)) for k, v in S.bench_layer_weights(shape, WEIGHT_SEED, l, gen).items()}
+
+    c0 = time.time()
+    s, n_seq, n_len = reference_calibration(shape, wl, layer_weights)
     r, _ = O.allocate_ratios(s, t_target, TAU, BETA)
     K = O.kept_counts(r, T).tolist()
-    ids = S.token_ids(2, args.warmup + args.steps, T, shape.vocab)
-    for i in range(args.warmup):
-        O.sparse_model_forward(ids[i:i + 1], extra, layers, p, K)
+    calib_s = time.time() - c0
+    ids = S.counter_ids(rank_seed(EVAL_SEED, 0), B, T, shape.vocab)
+    p = O.params_of(shape)
+    order = layer_order(L)
     t = []
-    for i in range(args.steps):
+    for i in range(args.warmup + args.steps):
+        j = i - args.warmup if i >= args.warmup else args.steps + i     # warm-up pairs after the timed ones
+        b, l = j % B, order[j % L]
+        W = layer_weights(l)
+        x = _f64(S.round_to_torch(S.bench_embed_rows(shape, WEIGHT_SEED, ids[b:b + 1]), shape.dtype))
         t0 = time.time()
-        O.sparse_model_forward(ids[args.warmup + i:args.warmup + i + 1], extra, layers, p, K)
-        t.append(time.time() - t0)
+        O.sparse_layer_forward(x, W, p, K[l])
+        if i >= args.warmup:
+            t.append(time.time() - t0)
     sec = float(np.mean(t))
-    v = T / sec
+    v = T / (sec * L)
+    sample = (f"each step: the oracle's sparse layer on one sequence x {T} tokens (layer input = the sequence's "
+              f"embedding), layers spread over the depth ({len(set(order[j % L] for j in range(args.steps)))} "
+              f"distinct layers over {args.steps} steps); rate extrapolated to all {L} layers "
+              f"(tokens/s = T / (L x mean step time)); K_l from the oracle's Eq. 4 statistics on "
+              f"{n_seq} x {n_len} calibration tokens ({calib_s:.0f} s)")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": v, "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": wl.name, "model": shape.name, "B": 1, "T": T, "layers": L,
-                   "retention_target": t_target, "K_per_layer": K},
+        "extrapolated": True,
+        "config": shared_config(wl, t_target, world),
+        "retention_plan": {"K_per_layer": K, "retention_mean": float(np.mean(K)) / T,
+                           "similarity": [float(x) for x in s],
+                           "calibration": f"oracle dense forward with Eq. 4 statistics over {n_seq} x {n_len} "
+                                          f"tokens of the calibration batch"},
         "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": host_threads(), "kind": "oracle",
-                         "sample": f"1 sequence x {T} tokens per step through all {L} layers"},
+                         "sample": sample},
         "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
 
@@ -547,10 +658,10 @@ def run_reference(args, rank, world):
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
-    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
-    ap.add_argument("--workload", choices=("c2", "c3", "c4", "c5"), default="c2")
+    ap.add_argument("--workload", choices=("c2", "c3", "c4", "c5"), default="c5")
     ap.add_argument("--retention", type=float, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=20.0)

@@ -146,19 +146,35 @@ adadsf_status adadsf_layer_stats(const void *x_in_dev, const void *x_out_dev, in
  * exits. Nothing is allocated: no cudaMalloc, cudaFree or allocating library
  * call.
  * Set-up: the first call on each device looks up the array's device address
- * (cudaGetSymbolAddress) with that device current and caches it; make that
- * first call before any stream capture.
+ * (cudaGetSymbolAddress) with that device current and caches it per device
+ * ordinal; make that first call before any stream capture. The cached address
+ * belongs to the context that was current then: the entry point is not valid
+ * after cudaDeviceReset, nor from a second context on the same device.
  * The array is shared by every call and keeps the last call's contents. Each
  * call writes every slot it later reads, so nothing needs clearing, but
  * calls whose kernels overlap on the GPU (other streams, other host threads)
  * race on the array and return wrong sums: serialise them.
- * Limits: n_rows <= 2^31 - 1 and d <= 65536 (the reduction uses at most 2048
- * blocks, so the 2048 slots always suffice); larger sizes return
- * ADADSF_ERR_UNSUPPORTED before any launch.
+ * Limit: n_rows <= 2^31 - 1 (larger returns ADADSF_ERR_UNSUPPORTED before any
+ * launch). The reduction's launch rule caps its block count at 2048 for every
+ * n_rows, one slot per block, so the 2048 slots always suffice; d has no
+ * limit beyond that of adadsf_layer_stats.
  * ---------------------------------------------------------------------- */
 adadsf_status adadsf_layer_stats_noalloc(const void *x_in_dev, const void *x_out_dev,
                                          int64_t n_rows, int d, int dtype, int mode,
                                          double *acc_dev, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Sec. 3.3, Eq. 4: the similarity s_l of each layer from the partial sums
+ * that adadsf_layer_stats / adadsf_sparse_model_forward accumulated (summed
+ * over calibration batches and replicas). Host only, pure.
+ * acc_host: L blocks laid out as the stats accumulator of `mode` --
+ *   TOKEN: {sum of cosines, token count} per layer, s_l = sum / count;
+ *   FLAT:  {sum a.b, sum |a|^2, sum |b|^2} per layer,
+ *          s_l = a.b / (max(|a|,1e-8) max(|b|,1e-8)).
+ * s_out_host[L] receives s_l. A non-positive token count or a non-finite
+ * result returns ADADSF_ERR_INVALID_ARG.
+ * ---------------------------------------------------------------------- */
+adadsf_status adadsf_similarity(const double *acc_host, int L, int mode, double *s_out_host);
 
 /* ------------------------------------------------------------------------
  * Sec. 3.3, Eqs. 5-8: layer-wise retention ratios from the similarity vector,
@@ -207,8 +223,9 @@ adadsf_status adadsf_topk_select(const float *scores_dev, int B, int T, int K,
  * splits 128-token tiles along d over several CTAs when there are few
  * tiles: arrival counters sit in a fixed area right after the device error
  * word (every completed call leaves them at zero, so one workspace serves
- * calls of any shape, here and in the layer and model forwards), fp32
- * partial tiles after it.
+ * calls of any shape, here and in the layer and model forwards; after a
+ * device timeout, adadsf_sync_check zeroes them), fp32 partial tiles after
+ * it.
  * ---------------------------------------------------------------------- */
 size_t adadsf_router_select_workspace_size(const adadsf_model_cfg *cfg, int B, int T);
 adadsf_status adadsf_router_select(const adadsf_model_cfg *cfg, const adadsf_layer_weights *w,
@@ -282,6 +299,11 @@ adadsf_status adadsf_sparse_model_forward(const adadsf_model_cfg *cfg, const ada
  * start of `ws`: ADADSF_ERR_DEVICE_TIMEOUT if a kernel gave up waiting,
  * ADADSF_ERR_INVALID_ARG if a kernel met an out-of-range index,
  * ADADSF_ERR_CUDA on a CUDA error, else ADADSF_OK.
+ * After a timeout it also zero-fills the synchronisation area that follows
+ * the error word (16 KiB of cross-CTA arrival counters, when ws_bytes covers
+ * it): a kernel that gave up may have left a counter part-way. A workspace
+ * that saw a timeout must pass through this call (or be zero-filled again)
+ * before its next use.
  * ---------------------------------------------------------------------- */
 adadsf_status adadsf_sync_check(void *ws, size_t ws_bytes, void *stream);
 

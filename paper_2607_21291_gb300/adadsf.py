@@ -81,6 +81,7 @@ def lib() -> ctypes.CDLL:
             "adadsf_stats_workspace_size": (sz, [i64]),
             "adadsf_layer_stats": (i32, [vp, vp, i64, i32, i32, i32, vp, vp, sz, vp]),
             "adadsf_layer_stats_noalloc": (i32, [vp, vp, i64, i32, i32, i32, vp, vp]),
+            "adadsf_similarity": (i32, [vp, i32, i32, vp]),
             "adadsf_alloc_ratios": (i32, [vp, i32, f64, f64, f64, i32, u32, vp, vp]),
             "adadsf_router_scores": (i32, [pcfg, plw, vp, i64, vp, vp, sz, vp]),
             "adadsf_topk_select": (i32, [vp, i32, i32, i32, vp, vp, vp]),
@@ -206,6 +207,22 @@ def adadsf_layer_stats_noalloc(x_in: torch.Tensor, x_out: torch.Tensor, acc: tor
     n = x_in.numel() // d
     _check(lib().adadsf_layer_stats_noalloc(_p(x_in), _p(x_out), n, d, DTYPE_CODE[x_in.dtype], mode,
                                             _p(acc), _s(stream)))
+
+
+def adadsf_similarity(acc, mode: int = STATS_TOKEN) -> np.ndarray:
+    """Host-only Eq. 4: s_l from the accumulated partial sums (any array-like,
+    [L, 2] for TOKEN mode or [L, 3] for FLAT)."""
+    if isinstance(acc, torch.Tensor):
+        acc = acc.detach().cpu()
+    a = np.ascontiguousarray(np.asarray(acc, dtype=np.float64).reshape(-1))
+    width = 2 if mode == STATS_TOKEN else 3
+    if a.size == 0 or a.size % width:
+        raise ValueError(f"accumulator of {a.size} values is not a multiple of {width}")
+    L = a.size // width
+    s = np.zeros(L, dtype=np.float64)
+    _check(lib().adadsf_similarity(a.ctypes.data_as(ctypes.c_void_p), L, int(mode),
+                                   s.ctypes.data_as(ctypes.c_void_p)))
+    return s
 
 
 def adadsf_alloc_ratios(s: Sequence[float], t: float, tau: float = 0.05, beta: float = 10.0,

@@ -33,9 +33,9 @@ def allreduce_stats(acc: torch.Tensor, group: Optional[dist.ProcessGroup] = None
 
 
 def similarity_of(acc) -> np.ndarray:
-    """s_l = (sum of cosines) / (token count) for acc laid out [L, 2]."""
-    a = np.asarray(acc.detach().cpu() if isinstance(acc, torch.Tensor) else acc, dtype=np.float64).reshape(-1, 2)
-    return a[:, 0] / a[:, 1]
+    """s_l = (sum of cosines) / (token count) for acc laid out [L, 2]
+    (Eq. 4, evaluated by the library's adadsf_similarity)."""
+    return A.adadsf_similarity(acc, A.STATS_TOKEN)
 
 
 def retention_plan(acc, T: int, t: float, tau: float = 0.05, beta: float = 10.0, flags: int = 0):

@@ -588,10 +588,10 @@ adadsf_status adadsf_layer_stats_noalloc(const void* x_in_dev, const void* x_out
     return fail(ADADSF_ERR_INVALID_ARG, "mode %d unknown", mode);
   if (n_rows < 0 || d <= 0 || d % (dtype == ADADSF_BF16 ? 8 : 4) != 0)
     return fail(ADADSF_ERR_INVALID_ARG, "need n_rows >= 0 and d a positive multiple of 16 bytes");
-  if (n_rows > (int64_t)INT32_MAX || d > 65536)
+  if (n_rows > (int64_t)INT32_MAX)
     return fail(ADADSF_ERR_UNSUPPORTED,
-                "workspace-free statistics take n_rows <= %d and d <= 65536 (got n_rows=%lld, d=%d)",
-                INT32_MAX, (long long)n_rows, d);
+                "workspace-free statistics take n_rows <= %d (got n_rows=%lld)", INT32_MAX,
+                (long long)n_rows);
   if (stats_partials_count(n_rows) > stats_static_capacity())
     return fail(ADADSF_ERR_UNSUPPORTED, "needs %d partial-sum slots, the fixed array holds %d",
                 stats_partials_count(n_rows), stats_static_capacity());
@@ -669,6 +669,27 @@ adadsf_status adadsf_alloc_ratios(const double* s_host, int L, double t, double 
       if (k > T) k = T;
       K_out_host[i] = (int32_t)k;
     }
+  }
+  return ADADSF_OK;
+}
+
+adadsf_status adadsf_similarity(const double* acc_host, int L, int mode, double* s_out_host) {
+  if (!acc_host || !s_out_host || L <= 0)
+    return fail(ADADSF_ERR_INVALID_ARG, "acc_host / s_out_host is NULL or L <= 0");
+  if (mode != ADADSF_STATS_TOKEN && mode != ADADSF_STATS_FLAT)
+    return fail(ADADSF_ERR_INVALID_ARG, "mode %d unknown", mode);
+  for (int l = 0; l < L; ++l) {
+    if (mode == ADADSF_STATS_TOKEN) {
+      // Eq. 4, token mode: mean of the per-token cosines
+      const double sum = acc_host[2 * l], n = acc_host[2 * l + 1];
+      if (!(n > 0.0)) return fail(ADADSF_ERR_INVALID_ARG, "layer %d: token count %g is not positive", l, n);
+      s_out_host[l] = sum / n;
+    } else {
+      // Eq. 4, flat mode: cosine of the flattened tensors, zero norms guarded
+      const double dot = acc_host[3 * l], na = sqrt(acc_host[3 * l + 1]), nb = sqrt(acc_host[3 * l + 2]);
+      s_out_host[l] = dot / ((na > 1e-8 ? na : 1e-8) * (nb > 1e-8 ? nb : 1e-8));
+    }
+    if (!isfinite(s_out_host[l])) return fail(ADADSF_ERR_INVALID_ARG, "layer %d: similarity is not finite", l);
   }
   return ADADSF_OK;
 }
@@ -964,6 +985,12 @@ adadsf_status adadsf_sync_check(void* ws, size_t ws_bytes, void* stream) {
   CUDA_TRY(cudaStreamSynchronize(s), "stream synchronise");
   if (h != 0) {
     CUDA_TRY(cudaMemsetAsync(ws, 0, sizeof(int), s), "clear error word");
+    // A kernel that gave up may have left arrival counters of the
+    // synchronisation area part-way (other CTAs of the same tile had already
+    // counted): zero them so the workspace is valid for the next call.
+    if ((h & DEVERR_TIMEOUT) && ws_bytes >= kErrBytes + kSyncBytes)
+      CUDA_TRY(cudaMemsetAsync(static_cast<char*>(ws) + kErrBytes, 0, kSyncBytes, s),
+               "clear synchronisation area");
     CUDA_TRY(cudaStreamSynchronize(s), "stream synchronise");
   }
   if (h & DEVERR_TIMEOUT)

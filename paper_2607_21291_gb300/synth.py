@@ -11,11 +11,14 @@ Recipe (the same for every workload):
   * norm biases            N(0, gain_std)
   * token ids              uniform over [0, vocab)
 All draws use NumPy's PCG64 stream keyed by (seed, layer, tensor name), so every
-tensor is reproducible on its own and independent of draw order.
+tensor is reproducible on its own and independent of draw order. The
+benchmark-size models use the counter-based draws at the end of this module
+(same recipe, norm gains 1 and biases 0).
 """
 from __future__ import annotations
 
 import dataclasses
+import math
 import zlib
 
 import numpy as np
@@ -169,3 +172,128 @@ def round_to(a: np.ndarray, dtype: str) -> np.ndarray:
     if nan.any():
         out[nan] = np.float32(np.nan)
     return out
+
+
+# ----------------------------------------------------------------------------
+# Counter-based draws (benchmark-size models)
+#
+# The full-size benchmark models hold billions of parameters: drawing them with
+# the NumPy streams above on the host would take minutes. These draws use a
+# counter-based generator instead -- element i of the tensor named by
+# (seed, key) is a pure function of (seed, key, i) -- written with PyTorch
+# integer and float64 operations, so the same tensor comes out on the GPU (in
+# milliseconds) and on the host (for any subset of its elements, such as the
+# embedding rows of a few token ids), apart from float64 ulps of log / cos that
+# vanish in the final float32 / bf16 rounding.
+#
+# Generator: SplitMix64 (G. Steele, D. Lea, C. Flood, "Fast splittable
+# pseudorandom number generators", OOPSLA 2014), the 64-bit finaliser applied
+# to stream_base + (i + 1) * 0x9E3779B97F4A7C15. Normal draws take two 24-bit
+# uniforms from one 64-bit output and apply the Box-Muller transform in
+# float64; token ids take the output modulo the vocabulary size.
+# ----------------------------------------------------------------------------
+_SM_GAMMA = 0x9E3779B97F4A7C15
+_SM_MUL1 = 0xBF58476D1CE4E5B9
+_SM_MUL2 = 0x94D049BB133111EB
+_CHUNK = 1 << 24
+
+
+def _i64(u: int) -> int:
+    """Two's-complement int64 value of a 64-bit unsigned constant."""
+    return u - (1 << 64) if u >= (1 << 63) else u
+
+
+def _lsr(z, s: int):
+    """Logical right shift of int64 tensor z by s bits."""
+    import torch
+    return torch.bitwise_and(torch.bitwise_right_shift(z, s), (1 << (64 - s)) - 1)
+
+
+def _splitmix64(ctr, base: int):
+    """SplitMix64 outputs for int64 counters ctr (wrapping int64 arithmetic)."""
+    z = ctr * _i64(_SM_GAMMA) + _i64(base)
+    z = _xor(z, _lsr(z, 30)) * _i64(_SM_MUL1)
+    z = _xor(z, _lsr(z, 27)) * _i64(_SM_MUL2)
+    return _xor(z, _lsr(z, 31))
+
+
+def _xor(a, b):
+    import torch
+    return torch.bitwise_xor(a, b)
+
+
+def _stream_base(seed: int, key: tuple) -> int:
+    h = zlib.crc32(repr((int(seed),) + tuple(key)).encode())
+    return ((int(seed) & 0xFFFFFFFF) << 32 | h) & 0xFFFFFFFFFFFFFFFF
+
+
+def counter_normal_at(seed: int, key: tuple, index, std: float = 1.0, mean: float = 0.0):
+    """float32 tensor of N(mean, std^2) draws at the flat element positions
+    `index` (int64 tensor, on the device the result should live on) of the
+    tensor named by (seed, key)."""
+    import torch
+    base = _stream_base(seed, key)
+    out = torch.empty(index.shape, dtype=torch.float32, device=index.device)
+    flat_i, flat_o = index.reshape(-1), out.view(-1)
+    for s in range(0, flat_i.numel(), _CHUNK):
+        z = _splitmix64(flat_i[s:s + _CHUNK] + 1, base)
+        u1 = (_lsr(z, 40).double() + 0.5) * (1.0 / (1 << 24))
+        u2 = (torch.bitwise_and(_lsr(z, 16), 0xFFFFFF).double() + 0.5) * (1.0 / (1 << 24))
+        n = torch.sqrt(-2.0 * torch.log(u1)) * torch.cos((2.0 * math.pi) * u2)
+        flat_o[s:s + _CHUNK] = (n * std + mean).float()
+    return out
+
+
+def counter_normal(seed: int, key: tuple, shape, std: float = 1.0, mean: float = 0.0, device="cpu"):
+    """The whole tensor of counter_normal_at, shaped `shape`."""
+    import torch
+    n = int(np.prod(shape)) if len(shape) else 1
+    out = torch.empty(n, dtype=torch.float32, device=device)
+    for s in range(0, n, _CHUNK):
+        e = min(n, s + _CHUNK)
+        out[s:e] = counter_normal_at(seed, key, torch.arange(s, e, dtype=torch.int64, device=device), std, mean)
+    return out.view(*shape)
+
+
+def counter_ids(seed: int, B: int, T: int, vocab: int, device="cpu"):
+    """int32 token ids (B, T), uniform over [0, vocab) (modulo bias < vocab / 2^63)."""
+    import torch
+    z = _splitmix64(torch.arange(B * T, dtype=torch.int64, device=device) + 1, _stream_base(seed, ("ids",)))
+    return torch.remainder(_lsr(z, 1), vocab).to(torch.int32).view(B, T)
+
+
+def bench_layer_weights(s: Shape, seed: int, layer: int, device="cpu") -> dict:
+    """float32 torch tensors of one layer in the benchmark recipe (counter-based
+    N(0, std 0.02) weights and biases, norm gains 1, norm biases 0)."""
+    import torch
+    out = {}
+    for name, shp in layer_weight_shapes(s).items():
+        if name in ("ln1_w", "ln2_w"):
+            out[name] = torch.ones(shp, dtype=torch.float32, device=device)
+        elif name in ("ln1_b", "ln2_b"):
+            out[name] = torch.zeros(shp, dtype=torch.float32, device=device)
+        else:
+            out[name] = counter_normal(seed, ("layer", layer, name), shp, 0.02, device=device)
+    return out
+
+
+def bench_embed(s: Shape, seed: int, device="cpu"):
+    """The whole embedding table [vocab, d] of the benchmark recipe (float32)."""
+    return counter_normal(seed, ("embed",), (s.vocab, s.d), 0.02, device=device)
+
+
+def bench_embed_rows(s: Shape, seed: int, ids):
+    """Rows ids (int tensor, any shape) of bench_embed, shape ids.shape + (d,),
+    drawn without building the table."""
+    import torch
+    flat = ids.reshape(-1).to(torch.int64)
+    cols = torch.arange(s.d, dtype=torch.int64, device=flat.device)
+    return counter_normal_at(seed, ("embed",), flat[:, None] * s.d + cols[None, :], 0.02).view(
+        *ids.shape, s.d)
+
+
+def round_to_torch(t, dtype: str):
+    """float32 copy of tensor t rounded to the storage dtype (bf16: round to
+    nearest even, as round_to)."""
+    import torch
+    return t.to(torch.bfloat16).float() if dtype == "bf16" else t.float().clone()

@@ -31,6 +31,25 @@ def rel_rms(got, ref):
     return float(np.sqrt(np.mean((got - ref) ** 2)) / max(np.sqrt(np.mean(ref ** 2)), 1e-30))
 
 
+def elem_rel(got, ref):
+    """Largest element-wise error, each element's |g - r| over max(|r|, rms(r)):
+    an error is judged against its own element unless that element is smaller
+    than the tensor's rms (the floor keeps near-zero elements from dividing
+    by ~0)."""
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    floor = max(float(np.sqrt(np.mean(ref ** 2))), 1e-30)
+    return float(np.max(np.abs(got - ref) / np.maximum(np.abs(ref), floor)))
+
+
+def assert_close(got, ref, tol, what=""):
+    """Both acceptance measures within tol: the per-tensor max|g - r| / max|r|
+    and the element-wise error with the rms floor."""
+    m, e = max_rel(got, ref), elem_rel(got, ref)
+    assert m <= tol and e <= tol, f"{what}: max_rel {m:.3g}, elem_rel {e:.3g} (rel_rms {rel_rms(got, ref):.3g}), tol {tol}"
+    return m, e
+
+
 def host_layer(shape, seed, layer=0, gain_std=0.1):
     """Seeded layer weights rounded to the storage dtype (float32 arrays)."""
     return {k: S.round_to(v, shape.dtype) for k, v in S.layer_weights(shape, seed, layer, gain_std).items()}

@@ -59,6 +59,25 @@ def test_alloc_matches_oracle(A):
                     assert Kr.tolist() == O.kept_counts(ro, T, "round").tolist()
 
 
+def test_similarity_matches_oracle(A):
+    """Eq. 4's final step on the host: s_l from accumulated partial sums, in
+    both aggregation modes, against the oracle's cos_sim_stat / similarity."""
+    g = np.random.default_rng(3)
+    tok, flat = [], []
+    for l in range(5):
+        a = g.standard_normal((40, 16))
+        b = a + (0.2 + 0.3 * l) * g.standard_normal((40, 16))
+        tok.append(O.cos_sim_stat(a, b))
+        flat.append(O.cos_sim_stat(a, b, "flat"))
+    assert A.adadsf_similarity(np.array(tok)) == pytest.approx([O.similarity(t) for t in tok], rel=1e-15)
+    assert A.adadsf_similarity(np.array(flat), A.STATS_FLAT) == pytest.approx(
+        [O.similarity(f, "flat") for f in flat], rel=1e-15)
+    with pytest.raises(A.AdadsfError):
+        A.adadsf_similarity(np.array([[1.0, 0.0]]))                # no tokens counted
+    with pytest.raises(ValueError):
+        A.adadsf_similarity(np.zeros(3))                           # not [L, 2]
+
+
 def test_alloc_rejects_bad_args(A):
     with pytest.raises(A.AdadsfError):
         A.adadsf_alloc_ratios([0.5, 0.6], 1.5)

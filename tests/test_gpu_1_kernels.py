@@ -31,6 +31,28 @@ def test_bounded_wait_gives_up_cleanly(A):
     assert float((x * 2).sum()) == 32.0                 # context still usable
 
 
+
+def test_timeout_clears_sync_area(A):
+    """A kernel that gives up waiting may leave cross-CTA arrival counters
+    part-way. After a timeout, adadsf_sync_check zeroes the synchronisation
+    area, so the same workspace then gives correct router scores on a shape
+    whose tiles are split along d (counters in use)."""
+    shape = S.QWEN25_7B.replace(ffn=256)
+    n = 25600 - 77                                          # 200 tiles: split past one wave
+    cfg = A.make_cfg(shape)
+    ws = A.workspace(A.adadsf_router_select_workspace_size(cfg, 1, 1))
+    ws[256:256 + SYNC_BYTES].view(torch.int32)[::7] = 3     # counters left part-way
+    A.adadsf_selftest_bounded_wait(ws, 2000)
+    assert A.adadsf_sync_check(ws) == A.ERR_DEVICE_TIMEOUT
+    assert int(ws[256:256 + SYNC_BYTES].view(torch.int32).abs().sum()) == 0
+    W = H.host_layer(shape, 3)
+    x = S.round_to(np.random.default_rng(n + 1).standard_normal((n, shape.d)).astype(np.float32), shape.dtype)
+    sc = torch.empty(n, dtype=torch.float32, device="cuda")
+    A.adadsf_router_scores(cfg, A.to_device(W, H.tdtype(shape)), H.to_dev(x, H.tdtype(shape)), sc, ws=ws)
+    assert A.adadsf_sync_check(ws) == A.OK
+    ref = O.router_scores(x.astype(np.float64), H.f64(W))
+    assert np.max(np.abs(sc.cpu().numpy() - ref)) / np.max(np.abs(ref)) < 5e-3
+
 # ---------------------------------------------------------------- Top-K (Sec. 3.4)
 @pytest.mark.parametrize("B,T,K", [(1, 1, 1), (3, 7, 3), (2, 128, 64), (4, 512, 256), (2, 1000, 1),
                                    (2, 1000, 999), (2, 1000, 1000), (5, 2048, 1024), (16, 4096, 2048),

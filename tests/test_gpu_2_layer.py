@@ -65,7 +65,7 @@ def test_sparse_layer(A, shape, B, T, K):
     H.check_kept_sets(gs, gi, ref_scores, K)
     ref, _, _ = O.sparse_layer_forward(x64, W64, p, K, idx=gi)
     got = H.to_np(xd)
-    assert H.max_rel(got, ref) <= H.tol(shape)
+    H.assert_close(got, ref, H.tol(shape), "layer")
     # skipped rows are untouched, bit for bit
     gx = xd.cpu()
     hx = H.to_dev(x, H.tdtype(shape), "cpu")
@@ -83,7 +83,7 @@ def test_r1_is_dense_and_r0_identity(A, shape):
     W64 = H.f64(W)
     ref = np.stack([x[b].astype(np.float64) + O.block_delta(x[b].astype(np.float64), np.arange(T), W64,
                                                           O.params_of(shape)) for b in range(B)])
-    assert H.max_rel(H.to_np(xd), ref) <= H.tol(shape)
+    H.assert_close(H.to_np(xd), ref, H.tol(shape), "dense layer")
     _, x0, xd0, _, _ = run_layer(A, shape, B, T, 0)
     assert torch.equal(xd0.cpu(), H.to_dev(x0, H.tdtype(shape), "cpu"))
 
@@ -95,8 +95,7 @@ def calibrate(A, model, ids, L, T, t):
     out = torch.empty((B, T, model.cfg.d), device="cuda",
                       dtype=torch.bfloat16 if model.cfg.dtype == A.BF16 else torch.float32)
     A.adadsf_sparse_model_forward(model, ids, [T] * L, out, stats_acc=acc)
-    a = acc.cpu().numpy().reshape(L, 2)
-    s = a[:, 0] / a[:, 1]
+    s = A.adadsf_similarity(acc)
     r, K = A.adadsf_alloc_ratios(s, t, 0.05, 10.0, T)
     return s, r, K
 
@@ -134,7 +133,7 @@ def test_model_c2_end_to_end(A):
         kept.append(gi[off:off + B * k].reshape(B, k))
         off += B * k
     ref, _, _ = O.sparse_model_forward(ids, extra, hostL, p, K.tolist(), idx_force=kept)
-    assert H.max_rel(H.to_np(hidden), ref) <= H.BF16_TOL
+    H.assert_close(H.to_np(hidden), ref, H.BF16_TOL, "model")
     # one workspace for calls of different shapes (dense with statistics,
     # then sparse, twice): the same results bit for bit as fresh workspaces
     ws = A.workspace(A.adadsf_model_workspace_size(model.cfg, B, T, [T] * L, True))
@@ -157,3 +156,27 @@ def test_model_c2_end_to_end(A):
             if H.score_gap(sc_ref[b], K[l]) > 1e-3:
                 assert O.topk_keep(sc_ref[b], K[l]).tolist() == kept[l][b].tolist()
         x, _, _ = O.sparse_layer_forward(x, hostL[l], p, K[l], idx=kept[l])
+
+
+def test_model_qwen_end_to_end(A):
+    """A 3-layer Qwen2.5-style model (RMSNorm, GQA, SwiGLU, final RMSNorm)
+    through adadsf_sparse_model_forward with a dense, a sparse and a very
+    sparse layer, against the oracle on the GPU's kept sets."""
+    shape = QWEN_SMALL.replace(n_layers=3, vocab=1000)
+    B, T = 2, 256
+    K = [T, 100, 7]
+    model = build_model(A, shape, 8)
+    ids = S.token_ids(9, B, T, shape.vocab)
+    hidden = torch.empty((B, T, shape.d), dtype=torch.bfloat16, device="cuda")
+    idx = torch.empty(B * sum(K), dtype=torch.int32, device="cuda")
+    A.adadsf_sparse_model_forward(model, torch.from_numpy(ids).cuda(), K, hidden, idx_out=idx)
+    gi = idx.cpu().numpy()
+    kept, off = [], 0
+    for k in K:
+        kept.append(gi[off:off + B * k].reshape(B, k))
+        off += B * k
+    assert (kept[0] == np.arange(T)[None, :]).all()
+    hostL = [H.f64(H.host_layer(shape, 8, l)) for l in range(3)]
+    extra = H.f64(H.host_extra(shape, 8))
+    ref, _, _ = O.sparse_model_forward(ids, extra, hostL, O.params_of(shape), K, idx_force=kept)
+    H.assert_close(H.to_np(hidden), ref, H.BF16_TOL, "qwen model")

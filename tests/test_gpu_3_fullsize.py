@@ -1,9 +1,14 @@
 """Full-size parity in the benchmark's launch configuration: one layer of each
-bf16 workload shape at its full (B, T) with r = 0.5, checked against the fp64
-oracle on sampled sequences (sequences are independent, so one sequence is a
-complete check of itself), plus whole-batch properties that hold at any size:
-skipped rows bit-identical and kept sets identical to the oracle's Top-K of
-the GPU scores."""
+bf16 workload shape at its full (B, T), with the first, a middle and the last
+layer's weights, and kept counts from the retention sweep (r = 0.25 / 0.5 /
+0.75, and r = 1 from the t = 1 allocation, which clamps every layer to dense).
+Each layer gets the same input on both sides (teacher forcing: the GPU's
+earlier layers do not feed it). The oracle checks sampled sequences (sequences
+are independent, so one sequence is a complete check of itself); properties
+that hold at any size are checked on the whole batch: skipped rows
+bit-identical and kept sets identical to the oracle's Top-K of the GPU scores."""
+import functools
+
 import numpy as np
 import pytest
 import torch
@@ -22,37 +27,71 @@ def A():
     return adadsf
 
 
-@pytest.mark.parametrize("key,samples", [("c2", (0, 3)), ("c3", (0, 7)), ("c4", (0, 7)), ("c5", (15,))])
-def test_fullsize_layer(A, key, samples):
+@functools.lru_cache(maxsize=2)
+def _weights(key, layer):
+    return H.host_layer(S.WORKLOADS[key].shape, 11, layer, gain_std=0.1)
+
+
+def _mid(key):
+    return S.WORKLOADS[key].shape.n_layers // 2
+
+
+def _last(key):
+    return S.WORKLOADS[key].shape.n_layers - 1
+
+
+CASES = [("c2", 0, 0.5), ("c2", _mid("c2"), 0.5), ("c2", _last("c2"), 0.5),
+         ("c3", 0, 0.5), ("c3", _mid("c3"), 0.5), ("c3", _mid("c3"), 0.25), ("c3", _mid("c3"), 0.75),
+         ("c3", _last("c3"), 0.5),
+         ("c4", 0, 0.5), ("c4", _mid("c4"), 0.5), ("c4", _last("c4"), 0.5),
+         ("c5", 0, 0.5), ("c5", _mid("c5"), 0.5), ("c5", _mid("c5"), 0.75), ("c5", _last("c5"), 0.5),
+         ("c5", _last("c5"), 0.25), ("c5", _last("c5"), 1.0)]
+
+
+@pytest.mark.parametrize("key,layer,r", CASES)
+def test_fullsize_layer(A, key, layer, r):
     wl = S.WORKLOADS[key]
     shape, B, T = wl.shape, wl.B, wl.T
-    K = T // 2
+    if r == 1.0:
+        # t = 1: Eq. 8 gives some r_l > 1 on an uneven similarity vector; the
+        # clamp makes every layer dense
+        s = np.linspace(0.80, 0.99, shape.n_layers)
+        r_raw, _ = A.adadsf_alloc_ratios(s, 1.0, 0.05, 10.0, T, A.ALLOC_RAW)
+        assert r_raw.max() > 1.0
+        _, Ks = A.adadsf_alloc_ratios(s, 1.0, 0.05, 10.0, T)
+        assert Ks.tolist() == [T] * shape.n_layers
+        K = int(Ks[layer])
+    else:
+        K = int(np.floor(r * T))
     td = H.tdtype(shape)
-    W = H.host_layer(shape, 11, 0, gain_std=0.1)
-    x = S.round_to(S.hidden(11, B, T, shape.d), shape.dtype)
+    W = _weights(key, layer)
+    x = S.round_to(S.hidden(11 + layer, B, T, shape.d), shape.dtype)
     xd = H.to_dev(x, td)
     x0 = xd.clone()
     idx = torch.empty((B, K), dtype=torch.int32, device="cuda")
-    sc = torch.empty((B, T), dtype=torch.float32, device="cuda")
+    sc = torch.full((B, T), float("nan"), dtype=torch.float32, device="cuda")
     cfg = A.make_cfg(shape)
     ws = A.workspace(A.adadsf_layer_workspace_size(cfg, B, T, K))
     A.adadsf_sparse_layer_forward(cfg, A.to_device(W, td), xd, K, idx, sc, ws)
     assert A.adadsf_sync_check(ws) == A.OK
     gi = idx.cpu().numpy()
     gs = sc.cpu().numpy()
-    # whole batch: kept sets are the Top-K of the GPU scores; skipped rows untouched
-    keep = torch.zeros((B, T), dtype=torch.bool, device="cuda")
-    keep.scatter_(1, idx.long(), True)
-    assert torch.equal(xd[~keep], x0[~keep])
-    for b in range(B):
-        assert O.topk_keep(gs[b], K).tolist() == gi[b].tolist()
-    # sampled sequences against the oracle
+    if K < T:
+        # whole batch: kept sets are the Top-K of the GPU scores; skipped rows untouched
+        keep = torch.zeros((B, T), dtype=torch.bool, device="cuda")
+        keep.scatter_(1, idx.long(), True)
+        assert torch.equal(xd[~keep], x0[~keep])
+        for b in range(B):
+            assert O.topk_keep(gs[b], K).tolist() == gi[b].tolist()
+    else:
+        assert (gi == np.arange(T)[None, :]).all()
+    # two sampled sequences (the first and the last) against the oracle
     W64 = H.f64(W)
     p = O.params_of(shape)
     got = xd.float().cpu().numpy()
-    for b in samples:
+    for b in (0, B - 1):
         xb = x[b:b + 1].astype(np.float64)
-        ref_sc = O.router_scores(xb, W64)
-        H.check_kept_sets(gs[b:b + 1], gi[b:b + 1], ref_sc, K)
+        if K < T:
+            H.check_kept_sets(gs[b:b + 1], gi[b:b + 1], O.router_scores(xb, W64), K)
         ref, _, _ = O.sparse_layer_forward(xb, W64, p, K, idx=gi[b:b + 1])
-        assert H.max_rel(got[b:b + 1], ref) <= H.BF16_TOL
+        H.assert_close(got[b:b + 1], ref, H.BF16_TOL, f"{key} layer {layer} K {K} seq {b}")

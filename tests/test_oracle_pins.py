@@ -410,3 +410,109 @@ class TestLayer:
         for W in layers:
             x = np.stack([x[b] + O.block_delta(x[b], np.arange(9), W, p) for b in range(2)])
         assert h == pytest.approx(O.layer_norm(x, Wm["final_w"], Wm["final_b"], 1e-5), rel=1e-12)
+
+
+# ---------------------------------------------------------------- Eqs. 1-3: how the layer composes
+def _tiny(arch):
+    """One head of width 2 on d = 2, FFN width 2, norm eps 0, full rotary."""
+    return {"arch": arch, "d": 2, "n_heads": 1, "n_kv_heads": 1, "head_dim": 2, "ffn": 2,
+            "rotary_dim": 2, "rope_theta": 1e4, "norm_eps": 0.0}
+
+
+_ROUTER_ONLY = {"router_w1": np.ones((1, 2)), "router_b1": np.zeros(1), "router_w2": np.ones(1),
+                "router_b2": np.zeros(1)}   # K = 0: the layer only scores its tokens
+
+
+class TestComposition:
+    """Hand-worked single-token layers. One token attends only to itself, so
+    attention returns its value row exactly (softmax of one score) and rotary
+    angles do not matter; every other step is worked out below with distinct
+    norm gains and non-symmetric weights, so that swapping the two norms of
+    GPT-NeoX, the gate and up roles of SwiGLU, or the input of Qwen's second
+    RMSNorm changes the result."""
+
+    def test_neox_parallel_branches(self):
+        """x = (3, 1): mean 2, variance 1, so LayerNorm gives (1, -1) before the
+        affine step.
+        LN1: gain (2, 3), bias (0.5, -1)  -> n1 = (2.5, -4)
+        LN2: gain (1, 0.5), bias (-1, 2)  -> n2 = (0, 1.5)
+        attention: V = I n1 + 0 = (2.5, -4); W_o = [[1, 1], [0, 2]], b_o = (0.25, 0)
+                   -> attn = (2.5 - 4 + 0.25, -8) = (-1.25, -8)
+        MLP: up = I n2 + 0 = (0, 1.5); GELU -> (0, 1.5 Phi(1.5)) = (0, 1.3997891980967129)
+             W_down = I, b_down = (0, 0.5) -> mlp = (0, 1.8997891980967129)
+        delta = attn + mlp = (-1.25, -6.1002108019032871).
+        With LN1 and LN2 swapped the result would be (4.2345, 3.4999)."""
+        p = _tiny(O.NEOX)
+        W = {"ln1_w": np.array([2.0, 3.0]), "ln1_b": np.array([0.5, -1.0]),
+             "ln2_w": np.array([1.0, 0.5]), "ln2_b": np.array([-1.0, 2.0]),
+             "w_qkv": np.vstack([np.array([[0.3, -0.7], [1.1, 0.2]]),       # q
+                                 np.array([[-0.4, 0.9], [0.6, 0.5]]),       # k
+                                 np.eye(2)]),                               # v
+             "b_qkv": np.array([0.1, -0.2, 0.3, 0.05, 0.0, 0.0]),
+             "w_o": np.array([[1.0, 1.0], [0.0, 2.0]]), "b_o": np.array([0.25, 0.0]),
+             "w_up": np.eye(2), "b_up": np.zeros(2),
+             "w_down": np.eye(2), "b_down": np.array([0.0, 0.5])}
+        got = O.block_delta(np.array([[3.0, 1.0]]), np.array([5]), W, p)
+        assert got[0] == pytest.approx([-1.25, -6.1002108019032871], rel=1e-14)
+
+    def test_qwen_sequential_residual(self):
+        """x = (1, -1): RMS 1.
+        RMS1 gain (2, 3) -> n1 = (2, -3)
+        attention: V = I n1 + (0.5, 0) = (2.5, -3); W_o = [[1, 0], [1, 1]]
+                   -> attn = (2.5, -0.5); h = x + attn = (3.5, -1.5), RMS(h) = sqrt(7.25)
+        RMS2 of h, gain (1, 2) -> n2 = (a, b), a = 3.5/sqrt(7.25) = 1.2998673672393630,
+                                  b = 2 (-1.5)/sqrt(7.25) = -1.1141720290623112
+        gate = W_gate n2, W_gate = [[1, 0], [0, 0.5]] -> (a, b/2)
+        up   = W_up n2,   W_up   = [[0, 1], [2, 0]]   -> (b, 2a)
+        act = SiLU(gate) * up = (SiLU(a) b, SiLU(b/2) 2a)
+            = (-1.1380735080494927, -0.52749388389216593)
+        W_down = I: delta = attn + act = (1.3619264919505073, -1.0274938838921659).
+        Swapping gate and up gives act = (-0.3579, -1.3481); RMS2 of x instead
+        of h gives n2 = (1, -2)."""
+        p = _tiny(O.QWEN)
+        W = {"ln1_w": np.array([2.0, 3.0]), "ln2_w": np.array([1.0, 2.0]),
+             "w_qkv": np.vstack([np.array([[0.3, -0.7], [1.1, 0.2]]),
+                                 np.array([[-0.4, 0.9], [0.6, 0.5]]),
+                                 np.eye(2)]),
+             "b_qkv": np.array([0.1, -0.2, 0.3, 0.05, 0.5, 0.0]),
+             "w_o": np.array([[1.0, 0.0], [1.0, 1.0]]),
+             "w_gate": np.array([[1.0, 0.0], [0.0, 0.5]]), "w_up": np.array([[0.0, 1.0], [2.0, 0.0]]),
+             "w_down": np.eye(2)}
+        got = O.block_delta(np.array([[1.0, -1.0]]), np.array([9]), W, p)
+        assert got[0] == pytest.approx([1.3619264919505073, -1.0274938838921659], rel=1e-14)
+
+    def test_qwen_final_norm(self):
+        """All K = 0: the Qwen model returns RMSNorm(embedding) with the final
+        gain. Row (3, 4): RMS = sqrt(12.5), normalised (0.84852813742385703,
+        1.1313708498984760), gain (2, 0.5) -> (1.6970562748477141,
+        0.56568542494923802)."""
+        p = _tiny(O.QWEN)
+        Wm = {"embed": np.array([[3.0, 4.0], [0.0, 0.0]]), "final_w": np.array([2.0, 0.5])}
+        h, _, _ = O.sparse_model_forward(np.array([[0]]), Wm, [_ROUTER_ONLY], p, [0])
+        assert h[0, 0] == pytest.approx([1.6970562748477141, 0.56568542494923802], rel=1e-14)
+        ref = F.rms_norm(torch.tensor([[3.0, 4.0]], dtype=torch.float64), (2,),
+                         torch.tensor([2.0, 0.5], dtype=torch.float64), eps=0.0)
+        assert h[0] == pytest.approx(ref.numpy(), rel=1e-14)
+
+    def test_neox_final_norm_matches_torch(self):
+        p = _tiny(O.NEOX)
+        p["norm_eps"] = 1e-5
+        g = rng(40)
+        Wm = {"embed": g.normal(size=(7, 2)), "final_w": 1 + g.normal(0, 0.3, 2), "final_b": g.normal(0, 0.3, 2)}
+        ids = np.array([[3, 0, 6, 6]])
+        h, _, _ = O.sparse_model_forward(ids, Wm, [_ROUTER_ONLY], p, [0])
+        ref = F.layer_norm(torch.from_numpy(Wm["embed"][ids]), (2,), torch.from_numpy(Wm["final_w"]),
+                           torch.from_numpy(Wm["final_b"]), eps=1e-5)
+        assert h == pytest.approx(ref.numpy(), rel=1e-13)
+
+    def test_linear_orientation_bias_and_gelu(self):
+        """W stored [out, in]: x = (1, -1), W = [[1, 2], [0, 3]], b = (0, 0)
+        -> x W^T = (-1, -3) (the transposed product would give (1, -1));
+        GELU: (-Phi(-1), -3 Phi(-3)) = (-0.15865525393145705, -0.0040496940948902836).
+        With bias (0.5, -1): (11.5, 16) for x = (1, 2), W = [[3, 4], [5, 6]]."""
+        y = O.linear(np.array([[1.0, -1.0]]), np.array([[1.0, 2.0], [0.0, 3.0]]))
+        assert y[0].tolist() == [-1.0, -3.0]
+        g_ = O.linear(np.array([[1.0, -1.0]]), np.array([[1.0, 2.0], [0.0, 3.0]]), act="gelu")
+        assert g_[0] == pytest.approx([-0.15865525393145705, -0.0040496940948902836], rel=1e-14)
+        b = O.linear(np.array([[1.0, 2.0]]), np.array([[3.0, 4.0], [5.0, 6.0]]), np.array([0.5, -1.0]))
+        assert b[0].tolist() == [11.5, 16.0]

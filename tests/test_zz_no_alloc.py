@@ -4,13 +4,16 @@ Some callers cannot hand the library scratch memory: their GPU memory belongs
 to another allocator or a pre-reserved pool, or they only receive their input
 and output buffers. For them the library keeps the reduction's partial sums in
 a fixed device array of its own. This file checks, through the C ABI, that two
-calls in a row give the same sums as the workspace entry point
-adadsf_layer_stats, and that sizes beyond the array's limits are refused.
+calls in a row give the same sums, bit for bit, as the workspace entry point
+adadsf_layer_stats, that both agree with the oracle's Eq. 4 sums, and that
+sizes beyond the array's limit are refused.
 It is collected last and needs nothing from the other test files, so it can run
 alone in a fresh process or after the rest of the suite."""
 import numpy as np
 import pytest
 import torch
+
+from oracle import adadsf_oracle as O
 
 pytestmark = pytest.mark.gpu
 
@@ -39,7 +42,13 @@ def test_noalloc_matches_workspace_entry_point(n, d, dtype, mode):
         torch.cuda.synchronize()
         r, g_ = ref.cpu().numpy(), got.cpu().numpy()
         assert np.all(np.isfinite(g_)), (call, g_)
-        assert g_ == pytest.approx(r, rel=REL_TOL), (call, g_, r)
+        # same kernels, same block count, same fixed summation order: the two
+        # entry points agree bit for bit (a stale slot would show here)
+        assert np.array_equal(g_, r), (call, g_, r)
+        # and both follow the oracle's Eq. 4 sums on the same rounded inputs
+        o = O.cos_sim_stat(a.double().cpu().numpy(), b.double().cpu().numpy(),
+                           "token" if mode == A.STATS_TOKEN else "flat")
+        assert g_ == pytest.approx(np.array(o), rel=REL_TOL), (call, g_, o)
 
 
 def test_noalloc_refuses_oversized_calls():
@@ -47,7 +56,7 @@ def test_noalloc_refuses_oversized_calls():
     lib = A.lib()
     acc = torch.zeros(2, dtype=torch.float64, device="cuda")
     x = torch.zeros(8, 8, dtype=torch.float32, device="cuda")
-    for n_rows, d in ((2 ** 31, 8), (1, 65540)):
+    for n_rows, d in ((2 ** 31, 8), (2 ** 40, 512)):
         st = lib.adadsf_layer_stats_noalloc(x.data_ptr(), x.data_ptr(), n_rows, d, A.F32, A.STATS_TOKEN,
                                             acc.data_ptr(), None)
         assert st == A.ERR_UNSUPPORTED
