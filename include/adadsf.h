@@ -59,6 +59,16 @@ typedef enum { ADADSF_ARCH_NEOX = 0, ADADSF_ARCH_QWEN = 1 } adadsf_arch;
  * FLAT: acc += {sum a.b, sum |a|^2, sum |b|^2} over all rows. */
 typedef enum { ADADSF_STATS_TOKEN = 0, ADADSF_STATS_FLAT = 1 } adadsf_stats_mode;
 
+/* adadsf_model_cfg.flags.
+ * ADADSF_FLAG_GATE_SIGMOID: the score-gated variant of Sec. 3.4 ("the
+ * router-score pathway is kept differentiable"), in the Mixture-of-Depths
+ * form: a kept row becomes x + sigmoid(s) * delta, s its router score, delta
+ * the layer's whole residual update (inside the layer nothing changes).
+ * Without it (default) scores only select and kept rows get x + delta, so
+ * K == T is exactly the dense layer. With it the router runs even when
+ * K == T. */
+#define ADADSF_FLAG_GATE_SIGMOID 1u
+
 /* adadsf_alloc_ratios flags */
 #define ADADSF_ALLOC_RAW 1u      /* return Eq. 8 unclamped (ratios may exceed 1) */
 #define ADADSF_ALLOC_ROUND 2u    /* K = round(r T) instead of floor(r T) */
@@ -77,7 +87,7 @@ typedef struct {
   float rope_theta;      /* rotary base */
   float norm_eps;
   int32_t dtype;         /* adadsf_dtype */
-  int32_t flags;         /* reserved, 0 */
+  int32_t flags;         /* ADADSF_FLAG_* (other bits: ADADSF_ERR_UNSUPPORTED) */
 } adadsf_model_cfg;
 
 /* Device pointers to one layer's parameters, all in cfg->dtype.
@@ -266,11 +276,13 @@ adadsf_status adadsf_causal_attention(const adadsf_model_cfg *cfg, const void *q
  * Sec. 3.4: one depth-sparse layer, in place.
  * x_dev [B,T,d]: kept rows become x + delta (delta = the layer's residual
  * update computed on the kept tokens only, causal among them, rotary at
- * their original positions); every other row is left untouched (not read
+ * their original positions; x + sigmoid(score) delta with
+ * ADADSF_FLAG_GATE_SIGMOID); every other row is left untouched (not read
  * back nor written). K == 0 enqueues nothing; K == T runs the dense layer
- * (router and Top-K skipped). idx_out_dev [B,K] int32 and scores_out_dev
- * [B,T] fp32 receive the kept positions and router scores (either may be
- * NULL; with K == T scores are not computed and scores_out_dev is ignored).
+ * (Top-K skipped; the router too unless the gate is on). idx_out_dev [B,K]
+ * int32 and scores_out_dev [B,T] fp32 receive the kept positions and router
+ * scores (either may be NULL; with K == T and no gate, scores are not
+ * computed and scores_out_dev is ignored).
  * ---------------------------------------------------------------------- */
 adadsf_status adadsf_sparse_layer_forward(const adadsf_model_cfg *cfg, const adadsf_layer_weights *w,
                                           void *x_dev, int B, int T, int K, int32_t *idx_out_dev,

@@ -33,6 +33,12 @@ Readings where the paper is silent (each one is listed in the design notes):
     (``mode="flat"``: cosine of the flattened tensors);
   * NeoX layer: x + Attn(LN1 x) + MLP(LN2 x); Qwen layer: h = x + Attn(RMS1 x),
     h + MLP(RMS2 h). The layer's residual delta is written to kept rows only.
+  * router scores only select by default (kept rows get x + delta, so r = 1 is
+    the dense layer); the score-gated variant (``p["gate"] == "sigmoid"``)
+    scales each kept row's delta by sigmoid(score), which keeps the score
+    pathway differentiable as Sec. 3.4 asks of training (Mixture-of-Depths
+    style). The gate applies to the layer's whole delta; inside the layer
+    (Qwen's h, the norms) nothing changes.
 """
 from __future__ import annotations
 
@@ -49,6 +55,11 @@ QWEN = 1
 def silu(x):
     """SiLU(x) = x * sigmoid(x)."""
     return x / (1.0 + np.exp(-x))
+
+
+def sigmoid(x):
+    """Logistic function 1 / (1 + e^-x)."""
+    return 1.0 / (1.0 + np.exp(-np.asarray(x, dtype=np.float64)))
 
 
 def gelu(x):
@@ -192,7 +203,8 @@ def sparse_layer_forward(x, W, p, K, idx=None):
 
     Scores every token with the router, keeps the Top-K of each sequence
     (or the given ``idx`` (B, K)), runs the layer on the kept tokens only and
-    adds its residual delta to those rows; every other row is copied unchanged.
+    adds its residual delta to those rows (scaled by sigmoid(score) when
+    ``p["gate"] == "sigmoid"``); every other row is copied unchanged.
     Returns (x_out, idx (B, K), scores (B, T))."""
     x = np.asarray(x, dtype=np.float64)
     B, T, d = x.shape
@@ -200,13 +212,17 @@ def sparse_layer_forward(x, W, p, K, idx=None):
     if idx is None:
         idx = np.stack([topk_keep(scores[b], K) for b in range(B)]) if B else np.zeros((0, K), np.int64)
     idx = np.asarray(idx, dtype=np.int64).reshape(B, -1)
+    gated = p.get("gate", "none") == "sigmoid"
     out = x.copy()
     for b in range(B):
         sel = idx[b]
         if sel.size == 0:
             continue
         xp = x[b, sel]
-        out[b, sel] = xp + block_delta(xp, sel, W, p)
+        delta = block_delta(xp, sel, W, p)
+        if gated:
+            delta = sigmoid(scores[b, sel])[:, None] * delta
+        out[b, sel] = xp + delta
     return out, idx, scores
 
 

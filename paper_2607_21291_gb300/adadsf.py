@@ -24,6 +24,7 @@ ARCH_NEOX, ARCH_QWEN = 0, 1
 STATS_TOKEN, STATS_FLAT = 0, 1
 LINEAR_SPLIT_WS_BYTES = 256 + 160 * 128 * 256 * 4   # ADADSF_LINEAR_SPLIT_WS_BYTES
 ALLOC_RAW, ALLOC_ROUND = 1, 2
+FLAG_GATE_SIGMOID = 1
 
 TORCH_DTYPE = {F32: torch.float32, BF16: torch.bfloat16}
 DTYPE_CODE = {torch.float32: F32, torch.bfloat16: BF16}
@@ -132,11 +133,12 @@ def workspace(nbytes: int, device=None) -> torch.Tensor:
 
 
 # --------------------------------------------------------------------- config
-def make_cfg(shape) -> ModelCfg:
-    """ModelCfg from any object with the backbone fields (see synth.Shape)."""
+def make_cfg(shape, flags: int = 0) -> ModelCfg:
+    """ModelCfg from any object with the backbone fields (see synth.Shape);
+    flags: FLAG_* bits (FLAG_GATE_SIGMOID: the score-gated variant)."""
     return ModelCfg(shape.d, shape.n_heads, shape.n_kv_heads, shape.head_dim, shape.ffn,
                     shape.n_layers, shape.vocab, shape.router_hidden, shape.arch, shape.rotary_dim,
-                    shape.rope_theta, shape.norm_eps, BF16 if shape.dtype == "bf16" else F32, 0)
+                    shape.rope_theta, shape.norm_eps, BF16 if shape.dtype == "bf16" else F32, int(flags))
 
 
 def layer_struct(w: dict) -> LayerWeights:

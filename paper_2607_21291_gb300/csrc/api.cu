@@ -96,8 +96,12 @@ adadsf_status check_cfg(const adadsf_model_cfg* c) {
     return fail(ADADSF_ERR_INVALID_ARG, "rotary_dim=%d must be even and <= head_dim", c->rotary_dim);
   if (!(c->norm_eps > 0.f) || !(c->rope_theta > 0.f))
     return fail(ADADSF_ERR_INVALID_ARG, "norm_eps and rope_theta must be positive");
+  if ((unsigned)c->flags & ~(unsigned)ADADSF_FLAG_GATE_SIGMOID)
+    return fail(ADADSF_ERR_UNSUPPORTED, "flags 0x%x has unknown bits", (unsigned)c->flags);
   return ADADSF_OK;
 }
+
+bool gated(const adadsf_model_cfg* c) { return ((unsigned)c->flags & ADADSF_FLAG_GATE_SIGMOID) != 0; }
 
 adadsf_status check_shape(int B, int T, int K) {
   if (B < 0 || T <= 0 || K < 0 || K > T)
@@ -272,6 +276,7 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
                          int T, int K, const LayerBufs& lb, bool want_idx, const Dev& dev) {
   if (K == 0 || B == 0) return ADADSF_OK;
   const bool dense = K == T;
+  const bool gate = gated(c);
   const int dt = c->dtype, d = c->d;
   const double es = elem_size(dt);
   const int64_t M = (int64_t)B * K;
@@ -285,11 +290,12 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
   const int32_t* rows = nullptr;
   const int32_t* pos = nullptr;
 
-  if (!dense) {
+  if (!dense || gate) {
     const double rf = 2.0 * BT * c->router_hidden * d;
     const double rb = (double)BT * d * es + (double)c->router_hidden * d * es + BT * 4.0;
     // a2: router scores of every token (bf16: tensor cores, tiles split
-    // along d when there are few of them)
+    // along d when there are few of them); the gated variant also needs
+    // them when every token is kept
     TRY(launch(dev, ADADSF_KERNEL_ROUTER, false, rf, rb,
                CALL(tc ? router_tc(x, BT, d, w->router_w1, w->router_b1, w->router_w2, w->router_b2,
                                    lb.scores, lb.sync, lb.rpart, dev)
@@ -299,6 +305,8 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
                                     static_cast<const float*>(w->router_w2),
                                     static_cast<const float*>(w->router_b2), lb.scores, dev),
                     "router")));
+  }
+  if (!dense) {
     if (M <= 32LL * dev.num_sms) {
       // a3 + a4: Top-K of each sequence fused with the gather of the kept rows
       // and their norms (NeoX: LN1 and LN2 of the same row). Every block
@@ -411,6 +419,7 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
     g.epi.out_mapped = true;
     g.epi.out = x;
     g.epi.ld_out = d;
+    if (gate) g.epi.gate_scores = lb.scores;   // x[row] + sigmoid(s) delta
     TRY(launch(dev, ADADSF_KERNEL_GEMM_O_DOWN, true, 2.0 * M * d * ((double)q + F),
                ((double)M * (q + F) + (double)d * (q + F) + 2.0 * Md) * es,
                [&] { return run_linear(dt, g, dev, "output + mlp down projections + residual scatter"); }));
@@ -445,6 +454,7 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
     dn.epi.out_mapped = true;
     dn.epi.out = x;
     dn.epi.ld_out = d;
+    if (gate) dn.epi.gate_scores = lb.scores;   // x[row] + sigmoid(s) delta
     TRY(launch(dev, ADADSF_KERNEL_GEMM_DOWN, tc, 2.0 * M * d * F,
                ((double)M * F + (double)d * F + 3.0 * Md) * es,
                [&] { return run_linear(dt, dn, dev, "mlp down + residual scatter"); }));
@@ -486,8 +496,14 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
     dn.epi.out_mapped = true;
     dn.epi.out = x;
     dn.epi.ld_out = d;
+    if (gate) {
+      // x[row] + sigmoid(s) (h + mlp - x[row]): the gate scales the whole delta
+      dn.epi.gate_scores = lb.scores;
+      dn.epi.gate_base = x;
+      dn.epi.ld_gate_base = d;
+    }
     TRY(launch(dev, ADADSF_KERNEL_GEMM_DOWN, tc, 2.0 * M * d * F,
-               ((double)M * F + (double)d * F + 2.0 * Md) * es,
+               ((double)M * F + (double)d * F + (gate ? 3.0 : 2.0) * Md) * es,
                [&] { return run_linear(dt, dn, dev, "mlp down + residual scatter"); }));
   }
   return ADADSF_OK;
@@ -860,7 +876,7 @@ adadsf_status adadsf_sparse_layer_forward(const adadsf_model_cfg* cfg, const ada
   TRY(check_cfg(cfg));
   TRY(check_shape(B, T, K));
   if (K == 0 || B == 0) return ADADSF_OK;
-  TRY(check_layer_weights(cfg, w, K < T));
+  TRY(check_layer_weights(cfg, w, K < T || gated(cfg)));
   NEED_PTR(x_dev, "x_dev");
   if (idx_out_dev && (reinterpret_cast<uintptr_t>(idx_out_dev) & 3u))
     return fail(ADADSF_ERR_INVALID_ARG, "idx_out_dev misaligned");
@@ -909,7 +925,7 @@ adadsf_status adadsf_sparse_model_forward(const adadsf_model_cfg* cfg, const ada
   int kmax = 0;
   for (int l = 0; l < cfg->n_layers; ++l) {
     TRY(check_shape(B, T, K_host[l]));
-    if (K_host[l] > 0) TRY(check_layer_weights(cfg, &w->layers[l], K_host[l] < T));
+    if (K_host[l] > 0) TRY(check_layer_weights(cfg, &w->layers[l], K_host[l] < T || gated(cfg)));
     kmax = K_host[l] > kmax ? K_host[l] : kmax;
   }
   NEED_PTR(w->embed, "embed");

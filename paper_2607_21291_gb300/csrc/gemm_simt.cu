@@ -20,6 +20,8 @@ struct SimtDev {
   const int32_t* rows;
   int out_mapped;
   float* out; int64_t ld_out;
+  const float* gate;                        // score gate (see internal.h), or null
+  const float* gbase; int64_t ld_gbase;
 };
 
 template <bool DUAL>
@@ -66,6 +68,7 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(const SimtDev p) {
     if (m >= p.M) continue;
     const int64_t arow = p.rows ? (int64_t)p.rows[m] : (int64_t)m;
     const int64_t orow = p.out_mapped ? arow : (int64_t)m;
+    const float g = p.gate ? 1.f / (1.f + expf(-p.gate[arow])) : 1.f;
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const int n = col0 + tx * 4 + j;
@@ -78,7 +81,14 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(const SimtDev p) {
         v = 0.5f * v * (1.f + erff(v * 0.70710678118654752f));
       }
       if (p.add_packed) v += p.add_packed[(int64_t)m * p.ld_add_packed + n];
-      if (p.add_rows) v += p.add_rows[arow * p.ld_add_rows + n];
+      if (p.gate && p.gbase) {
+        const float b = p.gbase[arow * p.ld_gbase + n];
+        v = fmaf(g, v - b, b);
+      } else if (p.gate) {
+        v = fmaf(g, v, p.add_rows[arow * p.ld_add_rows + n]);
+      } else if (p.add_rows) {
+        v += p.add_rows[arow * p.ld_add_rows + n];
+      }
       p.out[orow * p.ld_out + n] = v;
     }
   }
@@ -100,6 +110,9 @@ cudaError_t gemm_f32(const GemmArgs& a, const Dev& dev) {
   p.rows = a.epi.rows;
   p.out_mapped = a.epi.out_mapped ? 1 : 0;
   p.out = static_cast<float*>(a.epi.out); p.ld_out = a.epi.ld_out;
+  p.gate = a.epi.gate_scores;
+  p.gbase = static_cast<const float*>(a.epi.gate_base); p.ld_gbase = a.epi.ld_gate_base;
+  if (p.gate && (p.gbase ? p.add_rows != nullptr : p.add_rows == nullptr)) return cudaErrorInvalidValue;
   dim3 grid((a.N + TN - 1) / TN, (unsigned)((a.M + TM - 1) / TM));
   if (a.epi.act == ACT_SWIGLU)
     return launch_pdl(gemm_f32_kernel<true>, grid, dim3(256), 0, dev.stream, p);

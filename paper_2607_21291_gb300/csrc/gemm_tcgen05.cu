@@ -102,6 +102,10 @@ struct GemmDev {
   bf16* vt;                  // transposed value heads (see Epilogue::vt)
   int vt_seq, vt_pad, vt_col0, vt_hd, vt_hkv;
   float* scratch;            // split-K partial tiles (gemm_tc_sk_kernel)
+  // score gate: g = sigmoid(gate[rows[m]]); out = add + g v (add gathered) or
+  // gbase + g (v + add - gbase) (add packed, gbase gathered)
+  const float* gate;
+  const bf16* gbase; int64_t ld_gbase;
   int* err;
   unsigned long long timeout_ns;
 };
@@ -278,18 +282,39 @@ __device__ __forceinline__ void store_chunk_rows(uint32_t stg, int lane, const u
 // if RES and the problem has one); rows with !valid store nothing. Whole warp.
 template <bool RES>
 __device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, const uint4* res,
-                                                int64_t orow, int n0, bool valid, uint32_t stg,
-                                                int lane) {
+                                                float g, const uint4* gb, int64_t orow, int n0,
+                                                bool valid, uint32_t stg, int lane) {
   if (RES && p.add) {
+    if (!p.gate) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      float f[8];
-      unpack16(res[i], f, bf16());
+      for (int i = 0; i < 4; ++i) {
+        float f[8];
+        unpack16(res[i], f, bf16());
 #pragma unroll
-      for (int j = 0; j < 8; j += 2) {
-        const float2 s2 = __fadd2_rn(make_float2(v[8 * i + j], v[8 * i + j + 1]), make_float2(f[j], f[j + 1]));
-        v[8 * i + j] = s2.x;
-        v[8 * i + j + 1] = s2.y;
+        for (int j = 0; j < 8; j += 2) {
+          const float2 s2 = __fadd2_rn(make_float2(v[8 * i + j], v[8 * i + j + 1]), make_float2(f[j], f[j + 1]));
+          v[8 * i + j] = s2.x;
+          v[8 * i + j + 1] = s2.y;
+        }
+      }
+    } else if (!p.gbase) {
+      // gated, residual = the layer input x: out = x + g v
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        float f[8];
+        unpack16(res[i], f, bf16());
+#pragma unroll
+        for (int j = 0; j < 8; ++j) v[8 * i + j] = fmaf(g, v[8 * i + j], f[j]);
+      }
+    } else {
+      // gated, residual = h (packed), base = x: out = x + g (v + h - x)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        float f[8], b[8];
+        unpack16(res[i], f, bf16());
+        unpack16(gb[i], b, bf16());
+#pragma unroll
+        for (int j = 0; j < 8; ++j) v[8 * i + j] = fmaf(g, (v[8 * i + j] + f[j]) - b[j], b[j]);
       }
     }
   }
@@ -421,6 +446,8 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
   int64_t arow = m;
   if (mvalid && p.rows) arow = p.rows[m];
   const int64_t orow = p.out_mapped ? arow : (int64_t)m;
+  float gate = 1.f;
+  if (!ROPE && p.gate && mvalid) gate = 1.f / (1.f + expf(-p.gate[arow]));
   const float2* tab_row = nullptr;
   if (rope && mvalid)
     tab_row = p.rope_tab + (int64_t)(p.rope_pos ? p.rope_pos[m] : m % p.rope_T) * p.rope_half;
@@ -500,7 +527,14 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
         default: break;
       }
     }
-    epi_chunk_store<!ROPE>(p, v, res, orow, n0, mvalid, stg, lane);
+    uint4 gb[4] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0),
+                   make_uint4(0, 0, 0, 0)};
+    if (!ROPE && p.gbase && mvalid) {
+      const uint4* src = reinterpret_cast<const uint4*>(p.gbase + arow * p.ld_gbase + n0);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) gb[i] = src[i];
+    }
+    epi_chunk_store<!ROPE>(p, v, res, gate, gb, orow, n0, mvalid, stg, lane);
   }
 }
 
@@ -1231,6 +1265,14 @@ bool make_dev(const GemmArgs& a, const Dev& dev, GemmDev& p) {
   p.rows = a.epi.rows;
   p.out_mapped = a.epi.out_mapped ? 1 : 0;
   p.out = static_cast<bf16*>(a.epi.out); p.ld_out = a.epi.ld_out;
+  if (a.epi.gate_scores) {
+    // gated residual: x gathered (out = x + g v), or h packed with x as the base
+    if (a.epi.rope_tab) return false;
+    if (a.epi.gate_base ? !a.epi.add_packed : !a.epi.add_rows) return false;
+    p.gate = a.epi.gate_scores;
+    p.gbase = static_cast<const bf16*>(a.epi.gate_base);
+    p.ld_gbase = a.epi.ld_gate_base;
+  }
   p.rope_tab = a.epi.rope_tab;
   p.rope_pos = a.epi.rope_pos;
   p.rope_T = a.epi.rope_T;

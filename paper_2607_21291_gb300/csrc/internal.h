@@ -21,6 +21,10 @@ enum Act : int { ACT_NONE = 0, ACT_GELU = 1, ACT_SWIGLU = 2 };
 //   v += add_packed[m][n]                     (may be null)
 //   v += add_rows[row(m)][n]                  (may be null)
 //   out[out_mapped ? row(m) : m][n] = v       row(m) = rows ? rows[m] : m
+// Score gate (gate_scores set; the gated variant of Sec. 3.4): with
+// g = sigmoid(gate_scores[row(m)]) and t = v + add_packed[m][n],
+//   out = add_rows[row(m)][n] + g t                                (no gate_base)
+//   out = gate_base[row(m)][n] + g (t - gate_base[row(m)][n])      (gate_base; no add_rows)
 struct Epilogue {
   int act = ACT_NONE;
   const void* bias = nullptr;
@@ -46,6 +50,9 @@ struct Epilogue {
   // e = (n - vt_col0) % vt_hd.
   void* vt = nullptr;
   int vt_seq = 1, vt_pad = 0, vt_col0 = 0, vt_hd = 0, vt_hkv = 0;
+  const float* gate_scores = nullptr;
+  const void* gate_base = nullptr;
+  int64_t ld_gate_base = 0;
 };
 
 // acc = A . W^T (+ A2 . Wk2^T when K2 > 0: a second K source, bf16

@@ -40,7 +40,7 @@ LAYER_CASES = [
 ]
 
 
-def run_layer(A, shape, B, T, K, seed=5, x=None):
+def run_layer(A, shape, B, T, K, seed=5, x=None, flags=0):
     W = H.host_layer(shape, seed)
     if x is None:
         x = S.round_to(S.hidden(seed, B, T, shape.d), shape.dtype)
@@ -48,7 +48,7 @@ def run_layer(A, shape, B, T, K, seed=5, x=None):
     xd = H.to_dev(x, td)
     idx = torch.full((B, max(K, 1)), -1, dtype=torch.int32, device="cuda")
     sc = torch.full((B, T), float("nan"), dtype=torch.float32, device="cuda")
-    cfg = A.make_cfg(shape.replace(n_layers=1))
+    cfg = A.make_cfg(shape.replace(n_layers=1), flags)
     ws = A.workspace(A.adadsf_layer_workspace_size(cfg, B, T, K))
     A.adadsf_sparse_layer_forward(cfg, A.to_device(W, td), xd, K, idx, sc, ws)
     assert A.adadsf_sync_check(ws) == A.OK
@@ -86,6 +86,46 @@ def test_r1_is_dense_and_r0_identity(A, shape):
     H.assert_close(H.to_np(xd), ref, H.tol(shape), "dense layer")
     _, x0, xd0, _, _ = run_layer(A, shape, B, T, 0)
     assert torch.equal(xd0.cpu(), H.to_dev(x0, H.tdtype(shape), "cpu"))
+
+
+GATE_CASES = [
+    # (shape, B, T, K): fp32 and bf16, both architectures, split-K (small M),
+    # CTA-pair (large M) and one-CTA tiles, and the dense case (K = T)
+    (S.PYTHIA_70M, 1, 128, 64),
+    (S.PYTHIA_160M, 2, 200, 77),
+    (S.PYTHIA_160M, 2, 96, 96),
+    (QWEN_SMALL, 2, 150, 70),
+    (QWEN_SMALL, 1, 96, 96),
+    (QWEN_SMALL, 4, 2048, 1024),
+    (NEOX_128, 3, 1500, 1200),
+]
+
+
+@pytest.mark.parametrize("shape,B,T,K", GATE_CASES)
+def test_gated_layer(A, shape, B, T, K):
+    """Score-gated variant (Sec. 3.4, differentiable score pathway): kept rows
+    get x + sigmoid(s) delta; checked against the oracle's gated layer on the
+    GPU's kept sets, skipped rows bit-identical, scores returned also when
+    every token is kept."""
+    W, x, xd, gi, gs = run_layer(A, shape, B, T, K, seed=6, flags=A.FLAG_GATE_SIGMOID)
+    p = dict(O.params_of(shape), gate="sigmoid")
+    W64 = H.f64(W)
+    x64 = x.astype(np.float64)
+    ref_scores = O.router_scores(x64, W64)
+    assert np.max(np.abs(gs - ref_scores)) / np.max(np.abs(ref_scores)) < (5e-3 if shape.dtype == "bf16" else 1e-5)
+    if K < T:
+        H.check_kept_sets(gs, gi, ref_scores, K)
+    else:
+        assert (gi == np.arange(T)[None, :]).all()
+    ref, _, _ = O.sparse_layer_forward(x64, W64, p, K, idx=gi)
+    H.assert_close(H.to_np(xd), ref, H.tol(shape), "gated layer")
+    # the gate matters here: these scores are near 0, sigmoid near 1/2
+    plain, _, _ = O.sparse_layer_forward(x64, W64, O.params_of(shape), K, idx=gi)
+    assert H.max_rel(ref - x64, plain - x64) > 0.2
+    gx, hx = xd.cpu(), H.to_dev(x, H.tdtype(shape), "cpu")
+    for b in range(B):
+        skip = np.setdiff1d(np.arange(T), gi[b])
+        assert torch.equal(gx[b, skip], hx[b, skip])
 
 
 def calibrate(A, model, ids, L, T, t):

@@ -516,3 +516,56 @@ class TestComposition:
         assert g_[0] == pytest.approx([-0.15865525393145705, -0.0040496940948902836], rel=1e-14)
         b = O.linear(np.array([[1.0, 2.0]]), np.array([[3.0, 4.0], [5.0, 6.0]]), np.array([0.5, -1.0]))
         assert b[0].tolist() == [11.5, 16.0]
+
+
+# ---------------------------------------------------------------- Sec. 3.4: score-gated variant
+class TestGate:
+    """Kept rows get x + sigmoid(score) delta in the gated variant."""
+
+    def test_hand_worked_single_token(self):
+        """The NeoX single-token layer of TestComposition (delta =
+        (-1.25, -6.1002108019032871)) with a router whose hidden unit is
+        SiLU(0 . x + 1) = SiLU(1) = 0.73105857863000488 and score
+        2 SiLU(1) - 0.5 = 0.96211715726000976; sigmoid of it is
+        0.72354549497730215, so the gated delta is
+        (-0.90443186872162769, -4.4137800441289991)."""
+        p = _tiny(O.NEOX)
+        p["gate"] = "sigmoid"
+        W = {"router_w1": np.zeros((1, 2)), "router_b1": np.array([1.0]), "router_w2": np.array([2.0]),
+             "router_b2": np.array([-0.5]),
+             "ln1_w": np.array([2.0, 3.0]), "ln1_b": np.array([0.5, -1.0]),
+             "ln2_w": np.array([1.0, 0.5]), "ln2_b": np.array([-1.0, 2.0]),
+             "w_qkv": np.vstack([np.array([[0.3, -0.7], [1.1, 0.2]]), np.array([[-0.4, 0.9], [0.6, 0.5]]),
+                                 np.eye(2)]),
+             "b_qkv": np.array([0.1, -0.2, 0.3, 0.05, 0.0, 0.0]),
+             "w_o": np.array([[1.0, 1.0], [0.0, 2.0]]), "b_o": np.array([0.25, 0.0]),
+             "w_up": np.eye(2), "b_up": np.zeros(2),
+             "w_down": np.eye(2), "b_down": np.array([0.0, 0.5])}
+        x = np.array([[[3.0, 1.0]]])
+        out, idx, sc = O.sparse_layer_forward(x, W, p, 1)
+        assert sc[0, 0] == pytest.approx(0.96211715726000976, rel=1e-15)
+        assert out[0, 0] - x[0, 0] == pytest.approx([-0.90443186872162769, -4.4137800441289991], rel=1e-14)
+
+    @pytest.mark.parametrize("arch", [O.NEOX, O.QWEN])
+    def test_constant_score_scales_every_delta(self, arch):
+        """A router with w2 = 0 gives every token the score b2: score 0 halves
+        every kept row's delta (sigmoid(0) = 1/2); a large score recovers the
+        ungated layer; skipped rows stay untouched either way."""
+        p = _params(arch, Hkv=2 if arch == O.QWEN else 4)
+        W = _weights(p, 41)
+        x = rng(42).normal(size=(2, 9, 32))
+        idx = np.array([[0, 2, 3, 7], [1, 4, 5, 8]])
+        plain, _, _ = O.sparse_layer_forward(x, W, p, 4, idx=idx)
+        pg = dict(p, gate="sigmoid")
+        for b2, factor in ((0.0, 0.5), (60.0, 1.0)):
+            Wc = dict(W, router_w2=np.zeros_like(W["router_w2"]), router_b2=np.array([b2]))
+            got, _, _ = O.sparse_layer_forward(x, Wc, pg, 4, idx=idx)
+            assert got - x == pytest.approx(factor * (plain - x), rel=1e-12, abs=1e-14)
+            for b in range(2):
+                skip = np.setdiff1d(np.arange(9), idx[b])
+                assert np.array_equal(got[b, skip].view(np.uint64), x[b, skip].view(np.uint64))
+
+    def test_sigmoid(self):
+        assert O.sigmoid(0.0) == 0.5
+        assert O.sigmoid(np.log(3.0)) == pytest.approx(0.75, rel=1e-15)
+        assert O.sigmoid(-np.log(3.0)) == pytest.approx(0.25, rel=1e-15)
