@@ -42,11 +42,17 @@ def elem_rel(got, ref):
     return float(np.max(np.abs(got - ref) / np.maximum(np.abs(ref), floor)))
 
 
-def assert_close(got, ref, tol, what=""):
-    """Both acceptance measures within tol: the per-tensor max|g - r| / max|r|
-    and the element-wise error with the rms floor."""
+def assert_close(got, ref, tol, what="", elem_tol=None):
+    """Both acceptance measures: the per-tensor max|g - r| / max|r| within tol
+    and the element-wise error with the rms floor within elem_tol (default
+    tol). Through L stacked bf16 layers each layer's stored residual stream
+    adds its own rounding (up to 2^-9 relative per element), so the
+    element-wise error of a model output grows like sqrt(L): model-level
+    checks pass elem_tol = tol * sqrt(L)."""
+    elem_tol = tol if elem_tol is None else elem_tol
     m, e = max_rel(got, ref), elem_rel(got, ref)
-    assert m <= tol and e <= tol, f"{what}: max_rel {m:.3g}, elem_rel {e:.3g} (rel_rms {rel_rms(got, ref):.3g}), tol {tol}"
+    assert m <= tol and e <= elem_tol, (f"{what}: max_rel {m:.3g} (tol {tol}), elem_rel {e:.3g} "
+                                        f"(tol {elem_tol:.3g}), rel_rms {rel_rms(got, ref):.3g}")
     return m, e
 
 
