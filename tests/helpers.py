@@ -9,6 +9,15 @@ from paper_2607_21291_gb300 import synth as S
 
 BF16_TOL = 2e-2     # max |gpu - oracle| / max |oracle| for bf16 storage
 F32_TOL = 1e-4      # same, fp32 storage
+# Element-wise bound (|gpu - oracle| / max(|oracle|, rms(oracle))) for bf16
+# storage. Every bf16 tensor the layer stores between kernels (normed rows,
+# q/k/v, attention output, h, the MLP hidden, the output rows) rounds each
+# element by up to 2^-9 relative; emulating exactly these roundings in fp64
+# gives a per-element error of rms ~0.4% of the output's rms and, over the
+# ~10^7 elements of a Qwen2.5-7B-shape layer, a largest element error of
+# 3-4% of rms (tests/test_precision_cpu.py). 5e-2 bounds that with margin;
+# fp32 storage keeps F32_TOL element-wise.
+BF16_ELEM_TOL = 5e-2
 
 
 def tdtype(shape):
@@ -44,12 +53,10 @@ def elem_rel(got, ref):
 
 def assert_close(got, ref, tol, what="", elem_tol=None):
     """Both acceptance measures: the per-tensor max|g - r| / max|r| within tol
-    and the element-wise error with the rms floor within elem_tol (default
-    tol). Through L stacked bf16 layers each layer's stored residual stream
-    adds its own rounding (up to 2^-9 relative per element), so the
-    element-wise error of a model output grows like sqrt(L): model-level
-    checks pass elem_tol = tol * sqrt(L)."""
-    elem_tol = tol if elem_tol is None else elem_tol
+    and the element-wise error with the rms floor within elem_tol (default:
+    BF16_ELEM_TOL for the bf16 tolerance, else tol)."""
+    if elem_tol is None:
+        elem_tol = BF16_ELEM_TOL if tol == BF16_TOL else tol
     m, e = max_rel(got, ref), elem_rel(got, ref)
     assert m <= tol and e <= elem_tol, (f"{what}: max_rel {m:.3g} (tol {tol}), elem_rel {e:.3g} "
                                         f"(tol {elem_tol:.3g}), rel_rms {rel_rms(got, ref):.3g}")

@@ -173,7 +173,7 @@ def test_model_c2_end_to_end(A):
         kept.append(gi[off:off + B * k].reshape(B, k))
         off += B * k
     ref, _, _ = O.sparse_model_forward(ids, extra, hostL, p, K.tolist(), idx_force=kept)
-    H.assert_close(H.to_np(hidden), ref, H.BF16_TOL, "model", elem_tol=H.BF16_TOL * np.sqrt(L))
+    H.assert_close(H.to_np(hidden), ref, H.BF16_TOL, "model")
     # one workspace for calls of different shapes (dense with statistics,
     # then sparse, twice): the same results bit for bit as fresh workspaces
     ws = A.workspace(A.adadsf_model_workspace_size(model.cfg, B, T, [T] * L, True))
@@ -219,4 +219,4 @@ def test_model_qwen_end_to_end(A):
     hostL = [H.f64(H.host_layer(shape, 8, l)) for l in range(3)]
     extra = H.f64(H.host_extra(shape, 8))
     ref, _, _ = O.sparse_model_forward(ids, extra, hostL, O.params_of(shape), K, idx_force=kept)
-    H.assert_close(H.to_np(hidden), ref, H.BF16_TOL, "qwen model", elem_tol=H.BF16_TOL * np.sqrt(3))
+    H.assert_close(H.to_np(hidden), ref, H.BF16_TOL, "qwen model")
