@@ -339,6 +339,7 @@ def run_ours(args, rank, world, local_rank):
             mt = float(np.mean(ms_t))
             sweep[f"{t:g}"] = {"ms_per_step": mt, "value": B * T * world / (mt * 1e-3), "unit": "tokens/s",
                                "K_per_layer": Kt, "retention_mean": float(np.mean(Kt)) / T, "steps": len(ms_t),
+                               "normalized_flops": A.adadsf_normalized_flops(model.cfg, T, Kt),
                                "dense": all(k == T for k in Kt)}
         assert A.adadsf_sync_check(ws, stream) == A.OK, A.adadsf_last_error()
 
@@ -439,7 +440,6 @@ def run_ours(args, rank, world, local_rank):
         roof["avg_launch_ms"] = v["ms"] / v["launches"]
         roof["traffic"] = recorded_traffic(top, wl.name)
 
-    sparse_flops = sum(v["flops"] for v in agg.values()) / n_prof
     out = {
         "metric": METRIC,
         "value": tokens / (ms * 1e-3),
@@ -473,7 +473,7 @@ def run_ours(args, rank, world, local_rank):
         "retention_sweep": sweep,
         "hbm_path": hbm_path,
         "calibration": {"ms": calib_ms, "stats_kernel": stats_kernel, "batch": list(wl.calib)},
-        "normalized_flops": sparse_flops / max(1.0, L * dense_flops_per_layer(shape, B, T)),
+        "normalized_flops": A.adadsf_normalized_flops(model.cfg, T, K),
         "kernels": kernels,
         "kernels_vs_step": {"sum_ms_per_step": tot_ms / n_prof, "graph_ms_per_step": ms,
                             "ratio": tot_ms / n_prof / ms,

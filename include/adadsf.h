@@ -200,6 +200,21 @@ adadsf_status adadsf_alloc_ratios(const double *s_host, int L, double t, double 
                                   int T, unsigned flags, double *r_out_host, int32_t *K_out_host);
 
 /* ------------------------------------------------------------------------
+ * Sec. 4.1 (the normalized FLOPs of Tables 1-2): FLOPs of the depth-sparse
+ * forward over those of the dense model, per sequence of T tokens. Host
+ * only, pure. Counted per layer l: the router on all T tokens when
+ * K_host[l] < T (2 flops per multiply-add of W1 and w2), plus the layer on its
+ * K_host[l] kept tokens -- the QKV, output and MLP projections (three MLP
+ * matrices for Qwen's SwiGLU, two for GPT-NeoX) and causal attention among
+ * the kept tokens (2 n_heads head_dim K (K + 1)); divided by n_layers dense
+ * layers on T tokens. Embedding, final norm and LM head are the same in both
+ * and left out. The paper does not state its counting rules; this is the
+ * reading used here. K = T everywhere gives 1. *out_host receives the ratio.
+ * ---------------------------------------------------------------------- */
+adadsf_status adadsf_normalized_flops(const adadsf_model_cfg *cfg, int T, const int32_t *K_host,
+                                      double *out_host);
+
+/* ------------------------------------------------------------------------
  * Sec. 3.4: router scores of every token, w2 . SiLU(W1 x + b1) + b2.
  * x_dev [B*T, d] (cfg->dtype); scores_dev [B*T] fp32. ws: at least 256
  * bytes (the device error word); on the bf16 path, with

@@ -331,3 +331,36 @@ def params_of(shape):
     return {k: getattr(shape, k) for k in
             ("arch", "d", "n_heads", "n_kv_heads", "head_dim", "ffn", "rotary_dim",
              "rope_theta", "norm_eps")}
+
+
+# --------------------------------------------------------------------------
+# Sec. 4.1 (Tables 1-2) -- normalized FLOPs of the depth-sparse forward
+# --------------------------------------------------------------------------
+def block_flops(p, K):
+    """Floating-point operations (2 per multiply-add) of one decoder layer on
+    the K kept tokens of one sequence: the QKV, output and MLP projections
+    (3 MLP matrices for SwiGLU, 2 for GELU) plus causal attention among the
+    kept tokens (query i meets i + 1 keys in Q K^T and in P V)."""
+    d, H, Hkv, hd, F_ = p["d"], p["n_heads"], p["n_kv_heads"], p["head_dim"], p["ffn"]
+    q, kv = H * hd, Hkv * hd
+    n_mlp = 3 if p["arch"] == QWEN else 2
+    proj = 2.0 * K * ((q + 2 * kv) * d + d * q + n_mlp * d * F_)
+    attn = 2.0 * H * hd * K * (K + 1)
+    return proj + attn
+
+
+def router_flops(p, T, h=64):
+    """The router's multiply-adds on all T tokens of one sequence: W1 (h x d)
+    and w2 (h)."""
+    return 2.0 * T * h * (p["d"] + 1)
+
+
+def normalized_flops(p, T, K, h=64):
+    """Sparse-forward FLOPs over the dense model's, per sequence of T tokens:
+    sum over layers of (router on all T tokens when the layer drops any,
+    plus the layer on its K_l kept tokens) divided by the sum of the dense
+    layers on T tokens. Embedding, final norm and LM head are left out (the
+    same in both). K = T everywhere gives 1; K = 0 everywhere gives the
+    routers' cost alone."""
+    num = sum((router_flops(p, T, h) if k < T else 0.0) + block_flops(p, k) for k in K)
+    return num / (len(K) * block_flops(p, T))

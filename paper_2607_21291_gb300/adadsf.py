@@ -83,6 +83,7 @@ def lib() -> ctypes.CDLL:
             "adadsf_layer_stats": (i32, [vp, vp, i64, i32, i32, i32, vp, vp, sz, vp]),
             "adadsf_layer_stats_noalloc": (i32, [vp, vp, i64, i32, i32, i32, vp, vp]),
             "adadsf_similarity": (i32, [vp, i32, i32, vp]),
+            "adadsf_normalized_flops": (i32, [pcfg, i32, vp, vp]),
             "adadsf_alloc_ratios": (i32, [vp, i32, f64, f64, f64, i32, u32, vp, vp]),
             "adadsf_router_scores": (i32, [pcfg, plw, vp, i64, vp, vp, sz, vp]),
             "adadsf_topk_select": (i32, [vp, i32, i32, i32, vp, vp, vp]),
@@ -225,6 +226,15 @@ def adadsf_similarity(acc, mode: int = STATS_TOKEN) -> np.ndarray:
     _check(lib().adadsf_similarity(a.ctypes.data_as(ctypes.c_void_p), L, int(mode),
                                    s.ctypes.data_as(ctypes.c_void_p)))
     return s
+
+
+def adadsf_normalized_flops(cfg: ModelCfg, T: int, K: Sequence[int]) -> float:
+    """Host-only: sparse-forward FLOPs over the dense model's (Sec. 4.1)."""
+    arr = (ctypes.c_int32 * len(K))(*[int(k) for k in K])
+    out = ctypes.c_double(0.0)
+    _check(lib().adadsf_normalized_flops(ctypes.byref(cfg), int(T), ctypes.cast(arr, ctypes.c_void_p),
+                                         ctypes.byref(out)))
+    return out.value
 
 
 def adadsf_alloc_ratios(s: Sequence[float], t: float, tau: float = 0.05, beta: float = 10.0,

@@ -710,6 +710,30 @@ adadsf_status adadsf_similarity(const double* acc_host, int L, int mode, double*
   return ADADSF_OK;
 }
 
+adadsf_status adadsf_normalized_flops(const adadsf_model_cfg* cfg, int T, const int32_t* K_host,
+                                      double* out_host) {
+  TRY(check_cfg(cfg));
+  if (!K_host || !out_host || cfg->n_layers <= 0)
+    return fail(ADADSF_ERR_INVALID_ARG, "K_host / out_host is NULL or n_layers <= 0");
+  if (T <= 0) return fail(ADADSF_ERR_INVALID_ARG, "T=%d must be positive", T);
+  const double d = cfg->d, hd = cfg->head_dim, F = cfg->ffn;
+  const double q = (double)cfg->n_heads * hd, kv = (double)cfg->n_kv_heads * hd;
+  const double n_mlp = cfg->arch == ADADSF_ARCH_QWEN ? 3.0 : 2.0;
+  // one layer on K tokens of a sequence: projections + causal attention
+  auto block = [&](double K) {
+    return 2.0 * K * ((q + 2.0 * kv) * d + d * q + n_mlp * d * F) + 2.0 * q * K * (K + 1.0);
+  };
+  const double router = 2.0 * T * cfg->router_hidden * (d + 1.0);
+  double num = 0.0;
+  for (int l = 0; l < cfg->n_layers; ++l) {
+    const int K = K_host[l];
+    if (K < 0 || K > T) return fail(ADADSF_ERR_INVALID_ARG, "K[%d]=%d outside [0, T=%d]", l, K, T);
+    num += (K < T ? router : 0.0) + block(K);
+  }
+  *out_host = num / (cfg->n_layers * block(T));
+  return ADADSF_OK;
+}
+
 adadsf_status adadsf_router_scores(const adadsf_model_cfg* cfg, const adadsf_layer_weights* w,
                                    const void* x_dev, int64_t n_rows, float* scores_dev, void* ws,
                                    size_t ws_bytes, void* stream) {

@@ -78,6 +78,20 @@ def test_similarity_matches_oracle(A):
         A.adadsf_similarity(np.zeros(3))                           # not [L, 2]
 
 
+def test_normalized_flops_matches_oracle(A):
+    g = np.random.default_rng(4)
+    for key in ("c1", "c2", "c3", "c4", "c5"):
+        wl = S.WORKLOADS[key]
+        shape = wl.shape
+        for K in ([wl.T] * shape.n_layers, [0] * shape.n_layers,
+                  g.integers(0, wl.T + 1, shape.n_layers).tolist()):
+            got = A.adadsf_normalized_flops(A.make_cfg(shape), wl.T, K)
+            assert got == pytest.approx(O.normalized_flops(O.params_of(shape), wl.T, K, shape.router_hidden),
+                                        rel=1e-13)
+    with pytest.raises(A.AdadsfError):
+        A.adadsf_normalized_flops(A.make_cfg(S.PYTHIA_160M), 100, [101] * 12)
+
+
 def test_alloc_rejects_bad_args(A):
     with pytest.raises(A.AdadsfError):
         A.adadsf_alloc_ratios([0.5, 0.6], 1.5)

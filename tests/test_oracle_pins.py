@@ -569,3 +569,32 @@ class TestGate:
         assert O.sigmoid(0.0) == 0.5
         assert O.sigmoid(np.log(3.0)) == pytest.approx(0.75, rel=1e-15)
         assert O.sigmoid(-np.log(3.0)) == pytest.approx(0.25, rel=1e-15)
+
+
+# ---------------------------------------------------------------- Sec. 4.1: normalized FLOPs
+class TestNormalizedFlops:
+    P = {"arch": O.NEOX, "d": 4, "n_heads": 1, "n_kv_heads": 1, "head_dim": 4, "ffn": 8,
+         "rotary_dim": 4, "rope_theta": 1e4, "norm_eps": 1e-5}
+
+    def test_hand_counted(self):
+        """d = 4, one head of 4, FFN 8, GELU MLP, T = 4, router width 2.
+        Per token the projections take 12*4 (QKV) + 4*4 (output) + 2*4*8 (MLP)
+        = 128 multiply-adds = 256 flops; causal attention on K tokens takes
+        2 * 4 * K (K + 1) flops. K = 4: 1024 + 160 = 1184; K = 2: 512 + 48 = 560.
+        The router on 4 tokens: 2 * 4 * 2 * (4 + 1) = 80.
+        Layers K = (2, 4): (80 + 560 + 1184) / (2 * 1184) = 1824 / 2368."""
+        assert O.block_flops(self.P, 4) == 1184
+        assert O.block_flops(self.P, 2) == 560
+        assert O.router_flops(self.P, 4, h=2) == 80
+        assert O.normalized_flops(self.P, 4, [2, 4], h=2) == pytest.approx(1824 / 2368, rel=1e-15)
+
+    def test_limits(self):
+        """Every token kept: exactly 1 (no router counted, nothing dropped);
+        none kept: the routers' share alone."""
+        assert O.normalized_flops(self.P, 4, [4, 4, 4], h=2) == 1.0
+        assert O.normalized_flops(self.P, 4, [0, 0], h=2) == pytest.approx(80 / 1184, rel=1e-15)
+
+    def test_swiglu_counts_three_mlp_matrices(self):
+        """The Qwen form adds the gate matrix: 2 * 4 * 8 more multiply-adds a token."""
+        q = dict(self.P, arch=O.QWEN)
+        assert O.block_flops(q, 4) - O.block_flops(self.P, 4) == 2 * 4 * 4 * 8
