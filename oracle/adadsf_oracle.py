@@ -364,3 +364,79 @@ def normalized_flops(p, T, K, h=64):
     routers' cost alone."""
     num = sum((router_flops(p, T, h) if k < T else 0.0) + block_flops(p, k) for k in K)
     return num / (len(K) * block_flops(p, T))
+
+
+# --------------------------------------------------------------------------
+# Autoregressive decode with a cache of kept tokens only (the paper is silent
+# on generation; this is a Mixture-of-Depths style reading)
+# --------------------------------------------------------------------------
+def kept_threshold(scores, idx):
+    """The lowest router score among a sequence's kept tokens (the K-th
+    largest of Sec. 3.4's Top-K); +inf when nothing is kept (a layer that
+    keeps no prompt token keeps no generated token either)."""
+    s = np.asarray(scores, dtype=np.float64)[np.asarray(idx, dtype=np.int64)]
+    return float(s.min()) if s.size else np.inf
+
+
+def decode_keep(score, threshold):
+    """Causal keep decision of a new token: kept iff its score beats the
+    threshold strictly (a tie loses, as the later position loses ties in
+    Top-K; NaN never wins)."""
+    return bool(score > threshold)
+
+
+def sparse_prefill(ids, Wm, layers, p, K):
+    """The sparse model on the prompt (sparse_model_forward) plus the state a
+    decode needs per layer l and sequence b: the kept positions, the kept
+    tokens' layer-l INPUT rows (their keys and values are functions of
+    these), and the threshold of Sec. 3.4's Top-K. Returns
+    (hidden, state) with state = {"pos": [l][b] list, "rows": [l][b] list,
+    "thr": [l][b], "T": prompt length}."""
+    ids = np.asarray(ids)
+    x = np.asarray(Wm["embed"], dtype=np.float64)[ids]
+    B, T = ids.shape
+    st = {"pos": [], "rows": [], "thr": [], "T": T}
+    for l, W in enumerate(layers):
+        x_new, idx, sc = sparse_layer_forward(x, W, p, K[l])
+        st["pos"].append([list(idx[b]) for b in range(B)])
+        st["rows"].append([[x[b, t].copy() for t in idx[b]] for b in range(B)])
+        st["thr"].append([kept_threshold(sc[b], idx[b]) for b in range(B)])
+        x = x_new
+    return final_norm(x, Wm, p), st
+
+
+def decode_step(ids_new, Wm, layers, p, st):
+    """One generated token per sequence at position st["T"] (then st["T"] +=
+    1). Layer by layer: the router scores the token's current hidden state;
+    if it beats the layer's threshold the token is kept -- it attends
+    causally to the layer's kept tokens (rotary at original positions), its
+    residual delta is added, and it joins the layer's kept set (its input
+    row is cached); otherwise it bypasses the layer unchanged. Computed from
+    the definition: the layer is re-run on the kept rows plus the new one
+    and the last row's delta is taken (attention is causal, so earlier kept
+    rows are unaffected). Returns (hidden (B, d) after the final norm,
+    kept (L, B) bool)."""
+    ids_new = np.asarray(ids_new).reshape(-1)
+    B = ids_new.shape[0]
+    t = st["T"]
+    x = np.asarray(Wm["embed"], dtype=np.float64)[ids_new]
+    kept = np.zeros((len(layers), B), dtype=bool)
+    gated = p.get("gate", "none") == "sigmoid"
+    for l, W in enumerate(layers):
+        sc = router_scores(x, W)
+        x_next = x.copy()
+        for b in range(B):
+            if not decode_keep(sc[b], st["thr"][l][b]):
+                continue
+            kept[l, b] = True
+            rows = np.array(st["rows"][l][b] + [x[b]])
+            pos = np.array(st["pos"][l][b] + [t])
+            delta = block_delta(rows, pos, W, p)[-1]
+            if gated:
+                delta = sigmoid(sc[b]) * delta
+            x_next[b] = x[b] + delta
+            st["rows"][l][b].append(x[b].copy())
+            st["pos"][l][b].append(t)
+        x = x_next
+    st["T"] = t + 1
+    return final_norm(x, Wm, p), kept

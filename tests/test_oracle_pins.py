@@ -598,3 +598,81 @@ class TestNormalizedFlops:
         """The Qwen form adds the gate matrix: 2 * 4 * 8 more multiply-adds a token."""
         q = dict(self.P, arch=O.QWEN)
         assert O.block_flops(q, 4) - O.block_flops(self.P, 4) == 2 * 4 * 4 * 8
+
+
+# ---------------------------------------------------------------- decode with a kept-token cache
+class TestDecode:
+    """Generation reading: a new token is kept at layer l iff its router score
+    beats the lowest kept prompt score of that layer; kept tokens attend to
+    the layer's kept tokens and join them."""
+
+    def _model(self, arch, seed):
+        p = _params(arch, Hkv=2 if arch == O.QWEN else 4)
+        g = rng(seed)
+        Wm = {"embed": g.normal(size=(30, 32)), "final_w": 1 + g.normal(0, .1, 32)}
+        if arch == O.NEOX:
+            Wm["final_b"] = g.normal(0, .1, 32)
+        layers = [_weights(p, seed + 1 + l) for l in range(3)]
+        return p, Wm, layers
+
+    @pytest.mark.parametrize("arch", [O.NEOX, O.QWEN])
+    def test_matches_sparse_forward_on_the_extended_sequence(self, arch):
+        """Prompt of 10, two decoded tokens; per sequence, the decoded token's
+        output equals the last row of the sparse model on the extended
+        sequence with each layer's kept set = the prompt's kept set plus the
+        new token where it was kept (causality makes the two the same)."""
+        p, Wm, layers = self._model(arch, 50)
+        ids = rng(51).integers(0, 30, size=(3, 12))
+        K = [6, 3, 8]
+        _, st = O.sparse_prefill(ids[:, :10], Wm, layers, p, K)
+        decided = [[list(st["pos"][l][b]) for b in range(3)] for l in range(3)]
+        n_kept = 0
+        for t in (10, 11):
+            h, kept = O.decode_step(ids[:, t], Wm, layers, p, st)
+            n_kept += kept.sum()
+            for l in range(3):
+                for b in range(3):
+                    if kept[l, b]:
+                        decided[l][b].append(t)
+            for b in range(3):
+                force = [np.array([decided[l][b]]) for l in range(3)]
+                ref, _, _ = O.sparse_model_forward(ids[b:b + 1, :t + 1], Wm, layers, p,
+                                                   [len(f[0]) for f in force], idx_force=force)
+                assert h[b] == pytest.approx(ref[0, -1], rel=1e-12, abs=1e-12)
+        assert 0 < n_kept < 2 * 3 * 3          # some kept, some skipped
+
+    def test_always_kept_is_the_dense_model(self):
+        """Thresholds -inf (every token kept) and a dense prompt: the decoded
+        token's output is the dense model's last row on the extended sequence."""
+        p, Wm, layers = self._model(O.NEOX, 60)
+        ids = rng(61).integers(0, 30, size=(2, 8))
+        _, st = O.sparse_prefill(ids[:, :7], Wm, layers, p, [7, 7, 7])
+        st["thr"] = [[-np.inf] * 2 for _ in range(3)]
+        h, kept = O.decode_step(ids[:, 7], Wm, layers, p, st)
+        assert kept.all()
+        x = np.asarray(Wm["embed"])[ids]
+        for W in layers:
+            x = np.stack([x[b] + O.block_delta(x[b], np.arange(8), W, p) for b in range(2)])
+        dense = O.layer_norm(x, Wm["final_w"], Wm["final_b"], p["norm_eps"])
+        assert h == pytest.approx(dense[:, -1], rel=1e-12, abs=1e-12)
+
+    def test_never_kept_bypasses_every_layer(self):
+        p, Wm, layers = self._model(O.QWEN, 70)
+        ids = rng(71).integers(0, 30, size=(2, 6))
+        _, st = O.sparse_prefill(ids[:, :5], Wm, layers, p, [2, 2, 2])
+        st["thr"] = [[np.inf] * 2 for _ in range(3)]
+        h, kept = O.decode_step(ids[:, 5], Wm, layers, p, st)
+        assert not kept.any()
+        assert h == pytest.approx(O.rms_norm(np.asarray(Wm["embed"])[ids[:, 5]], Wm["final_w"], p["norm_eps"]),
+                                  rel=1e-14)
+        assert [len(r) for r in st["rows"][0]] == [2, 2]          # nothing joined the cache
+
+    def test_threshold_and_keep_rule(self):
+        """The threshold is the K-th largest score; a tie loses (the later
+        position loses Top-K ties); NaN never wins."""
+        sc = np.array([0.5, 2.0, -1.0, 2.0, 0.7])
+        idx = O.topk_keep(sc, 3)
+        assert O.kept_threshold(sc, idx) == 0.7
+        assert O.decode_keep(0.71, 0.7) and not O.decode_keep(0.7, 0.7)
+        assert not O.decode_keep(float("nan"), 0.7) and not O.decode_keep(float("nan"), -np.inf)
+        assert O.kept_threshold(sc, []) == np.inf              # nothing kept: nothing will be
