@@ -322,6 +322,50 @@ adadsf_status adadsf_sparse_model_forward(const adadsf_model_cfg *cfg, const ada
                                           void *stream);
 
 /* ------------------------------------------------------------------------
+ * Autoregressive decode with a cache of kept tokens only. The paper defines
+ * the sparse forward over whole sequences (Sec. 3.4) and says nothing about
+ * generation; this is a Mixture-of-Depths style reading:
+ *  - adadsf_prefill runs adadsf_sparse_model_forward on the prompt (B
+ *    sequences of T tokens, K_host[l] kept per layer) and also stores, per
+ *    layer l and sequence b, the kept tokens' keys (rotated) and values, their
+ *    count, and the keep threshold: the lowest router score the layer kept
+ *    (the K-th largest; +inf when K_host[l] == 0). It runs the router on
+ *    every layer, dense ones included. idx_out_dev as in
+ *    adadsf_sparse_model_forward (NULL or B * sum_l K_l int32).
+ *  - adadsf_decode_step takes one new token per sequence (ids_dev [B], at
+ *    the position after the last one) through every layer: the router
+ *    scores the token's hidden state; if the score is strictly above the
+ *    layer's threshold (a tie loses, as the later position loses Top-K ties;
+ *    NaN never wins), the token attends to the layer's cached kept tokens and
+ *    itself, gets the layer's residual delta (x sigmoid(score) with
+ *    ADADSF_FLAG_GATE_SIGMOID) and its key and value join the cache;
+ *    otherwise it bypasses the layer unchanged. hidden_out_dev [B, d]
+ *    receives the final-normed hidden states; kept_out_dev (NULL or int32
+ *    [n_layers][B]) the decisions (1 kept, 0 bypassed).
+ * The cache is one caller buffer of adadsf_kv_cache_size bytes (256-byte
+ * aligned; C_max = positions it can hold, prompt included): a header with
+ * the current position, per-layer counts and thresholds, the rotary table
+ * of every position and, per layer, K and V as [B][n_kv_heads][C_max]
+ * [head_dim] in cfg->dtype. Decode steps read the position and counts from
+ * the cache, so their launch arguments never change (one CUDA graph can
+ * replay them). A step whose position reaches C_max, or whose layer's
+ * cache is full, sets the device error word (adadsf_sync_check reports
+ * ADADSF_ERR_INVALID_ARG) and appends nothing. Prefill needs T < C_max and
+ * the workspace of adadsf_model_workspace_size(cfg, B, T, K_host, 0); a
+ * decode step adadsf_decode_workspace_size(cfg, B, C_max).
+ * ---------------------------------------------------------------------- */
+size_t adadsf_kv_cache_size(const adadsf_model_cfg *cfg, int B, int C_max);
+adadsf_status adadsf_prefill(const adadsf_model_cfg *cfg, const adadsf_model_weights *w,
+                             const int32_t *ids_dev, int B, int T, const int32_t *K_host,
+                             void *hidden_out_dev, int32_t *idx_out_dev, void *cache_dev,
+                             size_t cache_bytes, int C_max, void *ws, size_t ws_bytes, void *stream);
+size_t adadsf_decode_workspace_size(const adadsf_model_cfg *cfg, int B, int C_max);
+adadsf_status adadsf_decode_step(const adadsf_model_cfg *cfg, const adadsf_model_weights *w,
+                                 const int32_t *ids_dev, int B, void *hidden_out_dev,
+                                 int32_t *kept_out_dev, void *cache_dev, size_t cache_bytes,
+                                 int C_max, void *ws, size_t ws_bytes, void *stream);
+
+/* ------------------------------------------------------------------------
  * Synchronises `stream`, then reads and clears the device error word at the
  * start of `ws`: ADADSF_ERR_DEVICE_TIMEOUT if a kernel gave up waiting,
  * ADADSF_ERR_INVALID_ARG if a kernel met an out-of-range index,
@@ -354,6 +398,8 @@ typedef enum {
   ADADSF_KERNEL_GEMM_QKV_UP,   /* GPT-NeoX, bf16: QKV and MLP-up projections in one launch */
   ADADSF_KERNEL_GEMM_O_DOWN,   /* GPT-NeoX, bf16: output + MLP-down projections, one accumulator */
   ADADSF_KERNEL_TOPK_GATHER_NORM, /* Top-K fused with the gather and norms of the kept rows */
+  ADADSF_KERNEL_DECIDE,        /* decode: keep decision of each new token */
+  ADADSF_KERNEL_KV_CACHE,      /* decode cache: fill (prefill), thresholds, append */
   ADADSF_KERNEL_COUNT
 } adadsf_kernel_kind;
 

@@ -385,19 +385,20 @@ def decode_keep(score, threshold):
     return bool(score > threshold)
 
 
-def sparse_prefill(ids, Wm, layers, p, K):
+def sparse_prefill(ids, Wm, layers, p, K, idx_force=None):
     """The sparse model on the prompt (sparse_model_forward) plus the state a
     decode needs per layer l and sequence b: the kept positions, the kept
     tokens' layer-l INPUT rows (their keys and values are functions of
-    these), and the threshold of Sec. 3.4's Top-K. Returns
-    (hidden, state) with state = {"pos": [l][b] list, "rows": [l][b] list,
-    "thr": [l][b], "T": prompt length}."""
+    these), and the threshold of Sec. 3.4's Top-K. ``idx_force[l]`` (B, K_l)
+    replaces layer l's Top-K (the threshold is then taken over the forced
+    set). Returns (hidden, state) with state = {"pos": [l][b] list, "rows":
+    [l][b] list, "thr": [l][b], "T": prompt length}."""
     ids = np.asarray(ids)
     x = np.asarray(Wm["embed"], dtype=np.float64)[ids]
     B, T = ids.shape
     st = {"pos": [], "rows": [], "thr": [], "T": T}
     for l, W in enumerate(layers):
-        x_new, idx, sc = sparse_layer_forward(x, W, p, K[l])
+        x_new, idx, sc = sparse_layer_forward(x, W, p, K[l], None if idx_force is None else idx_force[l])
         st["pos"].append([list(idx[b]) for b in range(B)])
         st["rows"].append([[x[b, t].copy() for t in idx[b]] for b in range(B)])
         st["thr"].append([kept_threshold(sc[b], idx[b]) for b in range(B)])
@@ -405,7 +406,7 @@ def sparse_prefill(ids, Wm, layers, p, K):
     return final_norm(x, Wm, p), st
 
 
-def decode_step(ids_new, Wm, layers, p, st):
+def decode_step(ids_new, Wm, layers, p, st, kept_force=None):
     """One generated token per sequence at position st["T"] (then st["T"] +=
     1). Layer by layer: the router scores the token's current hidden state;
     if it beats the layer's threshold the token is kept -- it attends
@@ -414,21 +415,25 @@ def decode_step(ids_new, Wm, layers, p, st):
     row is cached); otherwise it bypasses the layer unchanged. Computed from
     the definition: the layer is re-run on the kept rows plus the new one
     and the last row's delta is taken (attention is causal, so earlier kept
-    rows are unaffected). Returns (hidden (B, d) after the final norm,
-    kept (L, B) bool)."""
+    rows are unaffected). ``kept_force`` (L, B) bool replaces the decisions
+    (the scores and own decisions are still returned). Returns (hidden (B, d)
+    after the final norm, kept (L, B) bool -- this function's own decisions
+    --, scores (L, B) of the router at each layer)."""
     ids_new = np.asarray(ids_new).reshape(-1)
     B = ids_new.shape[0]
     t = st["T"]
     x = np.asarray(Wm["embed"], dtype=np.float64)[ids_new]
     kept = np.zeros((len(layers), B), dtype=bool)
+    scores = np.zeros((len(layers), B))
     gated = p.get("gate", "none") == "sigmoid"
     for l, W in enumerate(layers):
         sc = router_scores(x, W)
+        scores[l] = sc
         x_next = x.copy()
         for b in range(B):
-            if not decode_keep(sc[b], st["thr"][l][b]):
+            kept[l, b] = decode_keep(sc[b], st["thr"][l][b])
+            if not (kept[l, b] if kept_force is None else kept_force[l][b]):
                 continue
-            kept[l, b] = True
             rows = np.array(st["rows"][l][b] + [x[b]])
             pos = np.array(st["pos"][l][b] + [t])
             delta = block_delta(rows, pos, W, p)[-1]
@@ -439,4 +444,4 @@ def decode_step(ids_new, Wm, layers, p, st):
             st["pos"][l][b].append(t)
         x = x_next
     st["T"] = t + 1
-    return final_norm(x, Wm, p), kept
+    return final_norm(x, Wm, p), kept, scores

@@ -94,6 +94,10 @@ def lib() -> ctypes.CDLL:
             "adadsf_causal_attention": (i32, [pcfg, vp, i32, i32, vp, vp, sz, vp]),
             "adadsf_sparse_layer_forward": (i32, [pcfg, plw, vp, i32, i32, i32, vp, vp, vp, sz, vp]),
             "adadsf_sparse_model_forward": (i32, [pcfg, pmw, vp, i32, i32, vp, vp, vp, vp, vp, sz, vp]),
+            "adadsf_kv_cache_size": (sz, [pcfg, i32, i32]),
+            "adadsf_prefill": (i32, [pcfg, pmw, vp, i32, i32, vp, vp, vp, vp, sz, i32, vp, sz, vp]),
+            "adadsf_decode_workspace_size": (sz, [pcfg, i32, i32]),
+            "adadsf_decode_step": (i32, [pcfg, pmw, vp, i32, vp, vp, vp, sz, i32, vp, sz, vp]),
             "adadsf_sync_check": (i32, [vp, sz, vp]),
             "adadsf_selftest_bounded_wait": (i32, [vp, sz, i32, vp]),
             "adadsf_profile_begin": (i32, [i32]),
@@ -351,6 +355,53 @@ def adadsf_sparse_model_forward(model: DeviceModel, ids: torch.Tensor, K: Sequen
                                              _p(ids), B, T, ctypes.cast(Karr, ctypes.c_void_p),
                                              _p(hidden_out), _p(stats_acc), _p(idx_out), _p(ws),
                                              ws.numel(), _s(stream)))
+
+
+def adadsf_kv_cache_size(cfg: ModelCfg, B: int, C_max: int) -> int:
+    n = lib().adadsf_kv_cache_size(ctypes.byref(cfg), int(B), int(C_max))
+    if n == 0:
+        raise AdadsfError(ERR_INVALID_ARG, adadsf_last_error())
+    return n
+
+
+def adadsf_decode_workspace_size(cfg: ModelCfg, B: int, C_max: int) -> int:
+    n = lib().adadsf_decode_workspace_size(ctypes.byref(cfg), int(B), int(C_max))
+    if n == 0:
+        raise AdadsfError(ERR_INVALID_ARG, adadsf_last_error())
+    return n
+
+
+def kv_cache(cfg: ModelCfg, B: int, C_max: int, device=None) -> torch.Tensor:
+    """A zeroed decode cache for B sequences of up to C_max positions."""
+    return torch.zeros(adadsf_kv_cache_size(cfg, B, C_max), dtype=torch.uint8, device=device or "cuda")
+
+
+def adadsf_prefill(model: DeviceModel, ids: torch.Tensor, K: Sequence[int], hidden_out: torch.Tensor,
+                   cache: torch.Tensor, C_max: int, idx_out: Optional[torch.Tensor] = None,
+                   ws: Optional[torch.Tensor] = None, stream=None):
+    """The sparse forward on the prompt ids (B, T), filling the decode cache."""
+    _dev(ids, "ids"); _dev(hidden_out, "hidden_out"); _dev(cache, "cache")
+    B, T = ids.shape
+    Karr = (ctypes.c_int32 * len(K))(*[int(k) for k in K])
+    if ws is None:
+        ws = workspace(adadsf_model_workspace_size(model.cfg, B, T, K, False), ids.device)
+    _check(lib().adadsf_prefill(ctypes.byref(model.cfg), ctypes.byref(model.struct), _p(ids), B, T,
+                                ctypes.cast(Karr, ctypes.c_void_p), _p(hidden_out), _p(idx_out), _p(cache),
+                                cache.numel(),
+                                int(C_max), _p(ws), ws.numel(), _s(stream)))
+
+
+def adadsf_decode_step(model: DeviceModel, ids: torch.Tensor, hidden_out: torch.Tensor, cache: torch.Tensor,
+                       C_max: int, kept_out: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None,
+                       stream=None):
+    """One generated token per sequence (ids (B,)) through every layer."""
+    _dev(ids, "ids"); _dev(hidden_out, "hidden_out"); _dev(cache, "cache")
+    B = ids.numel()
+    if ws is None:
+        ws = workspace(adadsf_decode_workspace_size(model.cfg, B, C_max), ids.device)
+    _check(lib().adadsf_decode_step(ctypes.byref(model.cfg), ctypes.byref(model.struct), _p(ids), B,
+                                    _p(hidden_out), _p(kept_out), _p(cache), cache.numel(), int(C_max), _p(ws),
+                                    ws.numel(), _s(stream)))
 
 
 def adadsf_sync_check(ws: torch.Tensor, stream=None) -> int:

@@ -270,12 +270,43 @@ GemmArgs linear_args(const void* A, int64_t lda, const void* W, int64_t M, int N
     return ADADSF_OK;                    \
   }
 
+// Prefill into a decode cache: the layer's kept keys / values, kept counts
+// and keep thresholds (see decode.cu).
+struct CacheSink {
+  void *kc, *vc;
+  int32_t* lens;   // [B]
+  float* thr;      // [B]
+  int C_max;
+};
+
+// One decode step of a layer: B new tokens (one per sequence, T = K = 1).
+struct DecodeCtx {
+  const float* thr;      // [B] this layer's thresholds
+  const int32_t* hdr;    // cache header (current position)
+  int32_t* lens;         // [B] this layer's cached counts
+  void *kc, *vc;         // this layer's cache
+  int C_max;
+  int32_t* rows;         // [B] b if kept, -1 if the token bypasses the layer
+  int32_t* pos;          // [B] the token's position
+  float* part_o;         // split-attention partials
+  float2* part_ml;
+  int32_t* kept_out;     // [B] or null
+};
+
 // Sec. 3.4: router -> Top-K -> gather + norm -> block on the packed rows ->
 // residual delta scattered back into x. K == T skips router and Top-K.
+// sink: also fill a decode cache (prefill). dec: a decode step instead.
 adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* w, void* x, int B,
-                         int T, int K, const LayerBufs& lb, bool want_idx, const Dev& dev) {
-  if (K == 0 || B == 0) return ADADSF_OK;
-  const bool dense = K == T;
+                         int T, int K, const LayerBufs& lb, bool want_idx, const Dev& dev,
+                         const CacheSink* sink = nullptr, const DecodeCtx* dec = nullptr) {
+  if (K == 0 || B == 0) {
+    // a layer that keeps nothing: an empty cache that keeps nothing either
+    if (sink && B > 0)
+      TRY(launch(dev, ADADSF_KERNEL_KV_CACHE, false, 0, 8.0 * B,
+                 CALL(kv_threshold(lb.scores, lb.idx, B, T, 0, sink->lens, sink->thr, dev), "cache thresholds")));
+    return ADADSF_OK;
+  }
+  const bool dense = K == T && !dec;
   const bool gate = gated(c);
   const int dt = c->dtype, d = c->d;
   const double es = elem_size(dt);
@@ -290,7 +321,7 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
   const int32_t* rows = nullptr;
   const int32_t* pos = nullptr;
 
-  if (!dense || gate) {
+  if (!dense || gate || sink) {
     const double rf = 2.0 * BT * c->router_hidden * d;
     const double rb = (double)BT * d * es + (double)c->router_hidden * d * es + BT * 4.0;
     // a2: router scores of every token (bf16: tensor cores, tiles split
@@ -306,7 +337,21 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
                                     static_cast<const float*>(w->router_b2), lb.scores, dev),
                     "router")));
   }
-  if (!dense) {
+  if (dec) {
+    // decode: keep decision of each new token, then the norms of all B rows
+    // (a bypassing token's block output is computed and dropped: the
+    // projections stream their weights once either way)
+    TRY(launch(dev, ADADSF_KERNEL_DECIDE, false, 0, 16.0 * B,
+               CALL(decode_decide(lb.scores, dec->thr, dec->hdr, B, dec->C_max, dec->rows, dec->pos,
+                                  dec->kept_out, dev),
+                    "keep decision")));
+    TRY(launch(dev, ADADSF_KERNEL_GATHER_NORM, false, 0, Md * es * (neox ? 3 : 2),
+               CALL(gather_norm(dt, x, nullptr, M, d, !neox, w->ln1_w, w->ln1_b, w->ln2_w,
+                                w->ln2_b, c->norm_eps, lb.n1, neox ? lb.n2 : nullptr, dev),
+                    "norm")));
+    rows = dec->rows;
+    pos = dec->pos;
+  } else if (!dense) {
     if (M <= 32LL * dev.num_sms) {
       // a3 + a4: Top-K of each sequence fused with the gather of the kept rows
       // and their norms (NeoX: LN1 and LN2 of the same row). Every block
@@ -330,7 +375,7 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
     rows = lb.rows;
     pos = lb.idx;
   } else {
-    if (want_idx)
+    if (want_idx || sink)
       TRY(launch(dev, ADADSF_KERNEL_POSITIONS, false, 0, M * 4.0,
                  CALL(iota_positions(lb.idx, B, K, dev), "positions")));
     // a4: normalise every row (NeoX: LN1 and LN2 of the same row).
@@ -361,7 +406,7 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
       g.epi.rope_hd = c->head_dim;
       g.epi.rope_cols = (c->n_heads + c->n_kv_heads) * c->head_dim;
     }
-    if (tc) {
+    if (tc && !dec) {
       g.epi.vt = lb.vt;
       g.epi.vt_seq = K;
       g.epi.vt_pad = vt_pad(K);
@@ -392,14 +437,37 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
                CALL(rope_apply(dt, lb.qkv, M, qkv_dim, c->n_heads, c->n_kv_heads, c->head_dim,
                                c->rotary_dim, pos, T, lb.rope, dev),
                     "rotary")));
-  // a6: causal attention among the kept tokens.
-  TRY(launch(dev, ADADSF_KERNEL_ATTENTION, tc, 2.0 * B * c->n_heads * c->head_dim * (double)K * (K + 1),
-             ((double)M * qkv_dim + (double)M * q) * es,
-             CALL(tc ? attention_tc(lb.qkv, qkv_dim, lb.vt, lb.attn, q, B, K, c->n_heads,
-                                    c->n_kv_heads, c->head_dim, dev)
-                     : attention(dt, lb.qkv, qkv_dim, lb.attn, q, B, K, c->n_heads, c->n_kv_heads,
-                                 c->head_dim, dev),
-                  "attention")));
+  if (dec) {
+    // a6 (decode): the new token against the layer's cached kept tokens and
+    // itself; then the kept tokens' keys and values join the cache
+    TRY(launch(dev, ADADSF_KERNEL_ATTENTION, false, 0,
+               (double)B * (q + 2.0 * kv) * es + 2.0 * B * kv * es * dec->C_max,
+               CALL(decode_attention(dt, lb.qkv, qkv_dim, c->n_heads, c->n_kv_heads, c->head_dim, dec->kc,
+                                     dec->vc, dec->lens, dec->C_max, B, dec->part_o, dec->part_ml, lb.attn, q,
+                                     dev),
+                    "decode attention")));
+    TRY(launch(dev, ADADSF_KERNEL_KV_CACHE, false, 0, 4.0 * B * kv * es,
+               CALL(kv_append(dt, lb.qkv, qkv_dim, q, kv, c->head_dim, B, dec->rows, dec->lens, dec->C_max,
+                              dec->kc, dec->vc, dev),
+                    "cache append")));
+  } else {
+    // a6: causal attention among the kept tokens.
+    TRY(launch(dev, ADADSF_KERNEL_ATTENTION, tc, 2.0 * B * c->n_heads * c->head_dim * (double)K * (K + 1),
+               ((double)M * qkv_dim + (double)M * q) * es,
+               CALL(tc ? attention_tc(lb.qkv, qkv_dim, lb.vt, lb.attn, q, B, K, c->n_heads,
+                                      c->n_kv_heads, c->head_dim, dev)
+                       : attention(dt, lb.qkv, qkv_dim, lb.attn, q, B, K, c->n_heads, c->n_kv_heads,
+                                   c->head_dim, dev),
+                    "attention")));
+  }
+  if (sink) {
+    // prefill: the kept tokens' keys (rotated) and values, counts and thresholds into the cache
+    TRY(launch(dev, ADADSF_KERNEL_KV_CACHE, false, 0, 4.0 * M * kv * es,
+               CALL(kv_fill(dt, lb.qkv, qkv_dim, q, kv, B, K, c->head_dim, sink->C_max, sink->kc, sink->vc, dev),
+                    "cache fill")));
+    TRY(launch(dev, ADADSF_KERNEL_KV_CACHE, false, 0, 8.0 * M,
+               CALL(kv_threshold(lb.scores, lb.idx, B, T, K, sink->lens, sink->thr, dev), "cache thresholds")));
+  }
   if (neox_tc) {
     // a7 + a8 + a9 as one GEMM with two K sources (parallel residual, Eq. 2):
     // x[row] = x[row] + O W_o^T + act W_down^T + b_o + b_down
@@ -536,6 +604,164 @@ void carve_model(const adadsf_model_cfg* c, int B, int T, int Kmax, bool stats, 
   m.rope = cv.take(rope_bytes(c, T));
   carve_layer(c, B, T, Kmax, cv, m.layer);
   m.total = cv.cur;
+}
+
+// ---------------------------------------------------------------- decode cache (see decode.cu)
+struct CacheView {
+  int32_t* hdr;
+  int32_t* lens;   // [L][B]
+  float* thr;      // [L][B]
+  float2* rope;    // [C_max][rot/2]
+  char* kv;        // per layer: K then V, each [B][Hkv][C_max][hd]
+  size_t kv_layer_bytes;
+  int C_max;
+  void* kc(int l) const { return kv + (size_t)l * 2 * kv_layer_bytes; }
+  void* vc(int l) const { return kv + (size_t)l * 2 * kv_layer_bytes + kv_layer_bytes; }
+};
+
+struct CacheLayout {
+  size_t hdr, lens, thr, rope, kv, kv_layer_bytes, total;
+};
+
+CacheLayout cache_layout(const adadsf_model_cfg* c, int B, int C_max) {
+  CacheLayout cl;
+  Carver cv;
+  const size_t L = c->n_layers;
+  cl.hdr = cv.take(256);
+  cl.lens = cv.take(L * B * 4);
+  cl.thr = cv.take(L * B * 4);
+  cl.rope = cv.take(rope_bytes(c, C_max));
+  cl.kv_layer_bytes = align256((size_t)B * c->n_kv_heads * C_max * c->head_dim * elem_size(c->dtype));
+  cl.kv = cv.take(2 * L * cl.kv_layer_bytes);
+  cl.total = cv.cur;
+  return cl;
+}
+
+CacheView cache_view(const adadsf_model_cfg* c, int B, int C_max, void* base) {
+  const CacheLayout cl = cache_layout(c, B, C_max);
+  CacheView v;
+  v.hdr = at<int32_t>(base, cl.hdr);
+  v.lens = at<int32_t>(base, cl.lens);
+  v.thr = at<float>(base, cl.thr);
+  v.rope = at<float2>(base, cl.rope);
+  v.kv = at<char>(base, cl.kv);
+  v.kv_layer_bytes = cl.kv_layer_bytes;
+  v.C_max = C_max;
+  return v;
+}
+
+struct DecodeSlots {
+  size_t x, rows, pos, part_o, part_ml;
+  LayerSlots layer;
+  size_t total;
+};
+
+DecodeSlots decode_layout(const adadsf_model_cfg* c, int B) {
+  DecodeSlots d;
+  Carver cv;
+  cv.take(kErrBytes);
+  cv.take(kSyncBytes);
+  d.x = cv.take((size_t)B * c->d * elem_size(c->dtype));
+  d.rows = cv.take((size_t)B * 4);
+  d.pos = cv.take((size_t)B * 4);
+  // split-attention partials: at most 64 splits per (sequence, query head)
+  d.part_o = cv.take((size_t)B * c->n_heads * 64 * c->head_dim * 4);
+  d.part_ml = cv.take((size_t)B * c->n_heads * 64 * 8);
+  carve_layer(c, B, 1, 1, cv, d.layer);
+  d.total = cv.cur;
+  return d;
+}
+
+adadsf_status model_forward_impl(const adadsf_model_cfg* cfg, const adadsf_model_weights* w,
+                                 const int32_t* ids_dev, int B, int T, const int32_t* K_host,
+                                 void* hidden_out_dev, double* stats_acc_dev, int32_t* idx_out_dev, void* ws,
+                                 size_t ws_bytes, void* stream, const CacheView* cache) {
+  TRY(check_cfg(cfg));
+  if (!w || !w->layers) return fail(ADADSF_ERR_INVALID_ARG, "model weights or layer array is NULL");
+  if (!K_host || cfg->n_layers <= 0) return fail(ADADSF_ERR_INVALID_ARG, "K_host is NULL or n_layers <= 0");
+  TRY(check_shape(B, T, 0));
+  int kmax = 0;
+  for (int l = 0; l < cfg->n_layers; ++l) {
+    TRY(check_shape(B, T, K_host[l]));
+    if (K_host[l] > 0) TRY(check_layer_weights(cfg, &w->layers[l], K_host[l] < T || gated(cfg)));
+    kmax = K_host[l] > kmax ? K_host[l] : kmax;
+  }
+  NEED_PTR(w->embed, "embed");
+  NEED_PTR(w->final_w, "final_w");
+  if (cfg->arch == ADADSF_ARCH_NEOX) NEED_PTR(w->final_b, "final_b");
+  NEED_PTR(hidden_out_dev, "hidden_out_dev");
+  if (cfg->vocab <= 0) return fail(ADADSF_ERR_INVALID_ARG, "vocab <= 0");
+  if (B > 0) NEED_PTR(ids_dev, "ids_dev");
+  if (stats_acc_dev && (reinterpret_cast<uintptr_t>(stats_acc_dev) & 7u))
+    return fail(ADADSF_ERR_INVALID_ARG, "stats_acc_dev misaligned");
+  if (idx_out_dev && (reinterpret_cast<uintptr_t>(idx_out_dev) & 3u))
+    return fail(ADADSF_ERR_INVALID_ARG, "idx_out_dev misaligned");
+  ModelSlots m;
+  carve_model(cfg, B, T, kmax, stats_acc_dev != nullptr, m);
+  TRY(check_ws(ws, ws_bytes, m.total));
+  if (B == 0) return ADADSF_OK;
+  Dev dev;
+  TRY(device_info(&dev, stream, ws));
+  const int dt = cfg->dtype;
+  const size_t es = elem_size(dt);
+  void* x = at<char>(ws, m.x);
+  const double xbytes_d = (double)B * T * cfg->d * es;
+  TRY(launch(dev, ADADSF_KERNEL_EMBED, false, 0, 2.0 * xbytes_d + 4.0 * B * T,
+             CALL(embed(dt, ids_dev, (int64_t)B * T, w->embed, cfg->vocab, cfg->d, x, dev), "embedding")));
+  // the rotary table: T rows in the workspace, or every cache position
+  float2* rope_tab = cache ? cache->rope : at<float2>(ws, m.rope);
+  const int rope_rows = cache ? cache->C_max : T;
+  if (cfg->rotary_dim > 0)
+    TRY(launch(dev, ADADSF_KERNEL_ROPE_TABLE, false, 0, rope_bytes(cfg, rope_rows),
+               CALL(rope_table(rope_tab, rope_rows, cfg->rotary_dim, cfg->rope_theta, dev), "rotary table")));
+  if (cache)
+    TRY(launch(dev, ADADSF_KERNEL_KV_CACHE, false, 0, 16.0,
+               CALL(cache_header(cache->hdr, T, cache->C_max, cfg->n_layers, B, dev), "cache header")));
+  LayerBufs lb;
+  lb.scores = at<float>(ws, m.layer.scores);
+  lb.rows = at<int32_t>(ws, m.layer.rows);
+  lb.rope = rope_tab;
+  lb.n1 = at<char>(ws, m.layer.n1);
+  lb.n2 = at<char>(ws, m.layer.n2);
+  lb.qkv = at<char>(ws, m.layer.qkv);
+  lb.vt = at<char>(ws, m.layer.vt);
+  lb.attn = at<char>(ws, m.layer.attn);
+  lb.ao = at<char>(ws, m.layer.ao);
+  lb.act = at<char>(ws, m.layer.act);
+  lb.split = m.layer.split ? at<float>(ws, m.layer.split) : nullptr;
+  lb.sync = at<int>(ws, kErrBytes);
+  lb.rpart = m.layer.rsel ? at<float>(ws, m.layer.rsel) : nullptr;
+  const size_t xbytes = (size_t)B * T * cfg->d * es;
+  int64_t idx_off = 0;
+  for (int l = 0; l < cfg->n_layers; ++l) {
+    const int K = K_host[l];
+    lb.idx = idx_out_dev ? idx_out_dev + idx_off : at<int32_t>(ws, m.layer.idx);
+    if (stats_acc_dev)
+      TRY(launch(dev, ADADSF_KERNEL_COPY, false, 0, 2.0 * xbytes_d,
+                 CALL(cudaMemcpyAsync(at<char>(ws, m.xin), x, xbytes, cudaMemcpyDeviceToDevice, dev.stream),
+                      "copy of the layer input")));
+    CacheSink sink;
+    if (cache) {
+      sink.kc = cache->kc(l);
+      sink.vc = cache->vc(l);
+      sink.lens = cache->lens + (int64_t)l * B;
+      sink.thr = cache->thr + (int64_t)l * B;
+      sink.C_max = cache->C_max;
+    }
+    TRY(layer_impl(cfg, &w->layers[l], x, B, T, K, lb, idx_out_dev != nullptr, dev, cache ? &sink : nullptr));
+    if (stats_acc_dev)
+      TRY(launch(dev, ADADSF_KERNEL_STATS, false, 0, 2.0 * xbytes_d,
+                 CALL(cos_stats(dt, at<char>(ws, m.xin), x, (int64_t)B * T, cfg->d, ADADSF_STATS_TOKEN,
+                                at<double>(ws, m.partials), stats_acc_dev + 2 * l, dev),
+                      "similarity statistics")));
+    idx_off += (int64_t)B * K;
+  }
+  TRY(launch(dev, ADADSF_KERNEL_FINAL_NORM, false, 0, 2.0 * xbytes_d,
+             CALL(gather_norm(dt, x, nullptr, (int64_t)B * T, cfg->d, cfg->arch == ADADSF_ARCH_QWEN,
+                              w->final_w, w->final_b, nullptr, nullptr, cfg->norm_eps, hidden_out_dev,
+                              nullptr, dev),
+                  "final norm")));
+  return ADADSF_OK;
 }
 
 }  // namespace
@@ -942,78 +1168,112 @@ adadsf_status adadsf_sparse_model_forward(const adadsf_model_cfg* cfg, const ada
                                           void* hidden_out_dev, double* stats_acc_dev,
                                           int32_t* idx_out_dev, void* ws, size_t ws_bytes,
                                           void* stream) {
+  return model_forward_impl(cfg, w, ids_dev, B, T, K_host, hidden_out_dev, stats_acc_dev, idx_out_dev, ws,
+                            ws_bytes, stream, nullptr);
+}
+
+size_t adadsf_kv_cache_size(const adadsf_model_cfg* cfg, int B, int C_max) {
+  if (check_cfg(cfg) != ADADSF_OK) return 0;
+  if (B <= 0 || C_max <= 0 || C_max > 65536 || cfg->n_layers <= 0) {
+    fail(ADADSF_ERR_INVALID_ARG, "need B > 0, 0 < C_max <= 65536 and n_layers > 0");
+    return 0;
+  }
+  return cache_layout(cfg, B, C_max).total;
+}
+
+adadsf_status adadsf_prefill(const adadsf_model_cfg* cfg, const adadsf_model_weights* w, const int32_t* ids_dev,
+                             int B, int T, const int32_t* K_host, void* hidden_out_dev, int32_t* idx_out_dev,
+                             void* cache_dev, size_t cache_bytes, int C_max, void* ws, size_t ws_bytes,
+                             void* stream) {
+  TRY(check_cfg(cfg));
+  if (B <= 0) return fail(ADADSF_ERR_INVALID_ARG, "B=%d must be positive", B);
+  if (T <= 0 || T >= C_max)
+    return fail(ADADSF_ERR_INVALID_ARG, "need 0 < T < C_max (T=%d, C_max=%d): room for generated tokens", T, C_max);
+  const size_t need = adadsf_kv_cache_size(cfg, B, C_max);
+  if (need == 0) return ADADSF_ERR_INVALID_ARG;
+  if (!cache_dev || (reinterpret_cast<uintptr_t>(cache_dev) & 255u))
+    return fail(ADADSF_ERR_INVALID_ARG, "cache_dev is NULL or not 256-byte aligned");
+  if (cache_bytes < need)
+    return fail(ADADSF_ERR_WORKSPACE_TOO_SMALL, "cache has %zu bytes, needs %zu", cache_bytes, need);
+  const CacheView cv = cache_view(cfg, B, C_max, cache_dev);
+  return model_forward_impl(cfg, w, ids_dev, B, T, K_host, hidden_out_dev, nullptr, idx_out_dev, ws, ws_bytes,
+                            stream, &cv);
+}
+
+size_t adadsf_decode_workspace_size(const adadsf_model_cfg* cfg, int B, int C_max) {
+  if (check_cfg(cfg) != ADADSF_OK) return 0;
+  if (B <= 0 || C_max <= 0) {
+    fail(ADADSF_ERR_INVALID_ARG, "need B > 0 and C_max > 0");
+    return 0;
+  }
+  return decode_layout(cfg, B).total;
+}
+
+adadsf_status adadsf_decode_step(const adadsf_model_cfg* cfg, const adadsf_model_weights* w, const int32_t* ids_dev,
+                                 int B, void* hidden_out_dev, int32_t* kept_out_dev, void* cache_dev,
+                                 size_t cache_bytes, int C_max, void* ws, size_t ws_bytes, void* stream) {
   TRY(check_cfg(cfg));
   if (!w || !w->layers) return fail(ADADSF_ERR_INVALID_ARG, "model weights or layer array is NULL");
-  if (!K_host || cfg->n_layers <= 0) return fail(ADADSF_ERR_INVALID_ARG, "K_host is NULL or n_layers <= 0");
-  TRY(check_shape(B, T, 0));
-  int kmax = 0;
-  for (int l = 0; l < cfg->n_layers; ++l) {
-    TRY(check_shape(B, T, K_host[l]));
-    if (K_host[l] > 0) TRY(check_layer_weights(cfg, &w->layers[l], K_host[l] < T || gated(cfg)));
-    kmax = K_host[l] > kmax ? K_host[l] : kmax;
-  }
+  if (B <= 0) return fail(ADADSF_ERR_INVALID_ARG, "B=%d must be positive", B);
+  for (int l = 0; l < cfg->n_layers; ++l) TRY(check_layer_weights(cfg, &w->layers[l], true));
   NEED_PTR(w->embed, "embed");
   NEED_PTR(w->final_w, "final_w");
   if (cfg->arch == ADADSF_ARCH_NEOX) NEED_PTR(w->final_b, "final_b");
+  NEED_PTR(ids_dev, "ids_dev");
   NEED_PTR(hidden_out_dev, "hidden_out_dev");
-  if (cfg->vocab <= 0) return fail(ADADSF_ERR_INVALID_ARG, "vocab <= 0");
-  if (B > 0) NEED_PTR(ids_dev, "ids_dev");
-  if (stats_acc_dev && (reinterpret_cast<uintptr_t>(stats_acc_dev) & 7u))
-    return fail(ADADSF_ERR_INVALID_ARG, "stats_acc_dev misaligned");
-  if (idx_out_dev && (reinterpret_cast<uintptr_t>(idx_out_dev) & 3u))
-    return fail(ADADSF_ERR_INVALID_ARG, "idx_out_dev misaligned");
-  ModelSlots m;
-  carve_model(cfg, B, T, kmax, stats_acc_dev != nullptr, m);
-  TRY(check_ws(ws, ws_bytes, m.total));
-  if (B == 0) return ADADSF_OK;
+  if (kept_out_dev && (reinterpret_cast<uintptr_t>(kept_out_dev) & 3u))
+    return fail(ADADSF_ERR_INVALID_ARG, "kept_out_dev misaligned");
+  const size_t need = adadsf_kv_cache_size(cfg, B, C_max);
+  if (need == 0) return ADADSF_ERR_INVALID_ARG;
+  if (!cache_dev || (reinterpret_cast<uintptr_t>(cache_dev) & 255u))
+    return fail(ADADSF_ERR_INVALID_ARG, "cache_dev is NULL or not 256-byte aligned");
+  if (cache_bytes < need)
+    return fail(ADADSF_ERR_WORKSPACE_TOO_SMALL, "cache has %zu bytes, needs %zu", cache_bytes, need);
+  const DecodeSlots ds = decode_layout(cfg, B);
+  TRY(check_ws(ws, ws_bytes, ds.total));
   Dev dev;
   TRY(device_info(&dev, stream, ws));
+  const CacheView cv = cache_view(cfg, B, C_max, cache_dev);
   const int dt = cfg->dtype;
-  const size_t es = elem_size(dt);
-  void* x = at<char>(ws, m.x);
-  const double xbytes_d = (double)B * T * cfg->d * es;
-  TRY(launch(dev, ADADSF_KERNEL_EMBED, false, 0, 2.0 * xbytes_d + 4.0 * B * T,
-             CALL(embed(dt, ids_dev, (int64_t)B * T, w->embed, cfg->vocab, cfg->d, x, dev), "embedding")));
-  if (cfg->rotary_dim > 0)
-    TRY(launch(dev, ADADSF_KERNEL_ROPE_TABLE, false, 0, rope_bytes(cfg, T),
-               CALL(rope_table(at<float2>(ws, m.rope), T, cfg->rotary_dim, cfg->rope_theta, dev),
-                    "rotary table")));
+  const double es = elem_size(dt);
+  void* x = at<char>(ws, ds.x);
+  TRY(launch(dev, ADADSF_KERNEL_EMBED, false, 0, 2.0 * B * cfg->d * es + 4.0 * B,
+             CALL(embed(dt, ids_dev, B, w->embed, cfg->vocab, cfg->d, x, dev), "embedding")));
   LayerBufs lb;
-  lb.scores = at<float>(ws, m.layer.scores);
-  lb.rows = at<int32_t>(ws, m.layer.rows);
-  lb.rope = at<float2>(ws, m.rope);
-  lb.n1 = at<char>(ws, m.layer.n1);
-  lb.n2 = at<char>(ws, m.layer.n2);
-  lb.qkv = at<char>(ws, m.layer.qkv);
-  lb.vt = at<char>(ws, m.layer.vt);
-  lb.attn = at<char>(ws, m.layer.attn);
-  lb.ao = at<char>(ws, m.layer.ao);
-  lb.act = at<char>(ws, m.layer.act);
-  lb.split = m.layer.split ? at<float>(ws, m.layer.split) : nullptr;
+  lb.scores = at<float>(ws, ds.layer.scores);
+  lb.idx = at<int32_t>(ws, ds.layer.idx);
+  lb.rows = at<int32_t>(ws, ds.layer.rows);
+  lb.rope = cv.rope;
+  lb.n1 = at<char>(ws, ds.layer.n1);
+  lb.n2 = at<char>(ws, ds.layer.n2);
+  lb.qkv = at<char>(ws, ds.layer.qkv);
+  lb.vt = at<char>(ws, ds.layer.vt);
+  lb.attn = at<char>(ws, ds.layer.attn);
+  lb.ao = at<char>(ws, ds.layer.ao);
+  lb.act = at<char>(ws, ds.layer.act);
+  lb.split = ds.layer.split ? at<float>(ws, ds.layer.split) : nullptr;
   lb.sync = at<int>(ws, kErrBytes);
-  lb.rpart = m.layer.rsel ? at<float>(ws, m.layer.rsel) : nullptr;
-  const size_t xbytes = (size_t)B * T * cfg->d * es;
-  int64_t idx_off = 0;
+  lb.rpart = ds.layer.rsel ? at<float>(ws, ds.layer.rsel) : nullptr;
   for (int l = 0; l < cfg->n_layers; ++l) {
-    const int K = K_host[l];
-    lb.idx = idx_out_dev ? idx_out_dev + idx_off : at<int32_t>(ws, m.layer.idx);
-    if (stats_acc_dev)
-      TRY(launch(dev, ADADSF_KERNEL_COPY, false, 0, 2.0 * xbytes_d,
-                 CALL(cudaMemcpyAsync(at<char>(ws, m.xin), x, xbytes, cudaMemcpyDeviceToDevice, dev.stream),
-                      "copy of the layer input")));
-    TRY(layer_impl(cfg, &w->layers[l], x, B, T, K, lb, idx_out_dev != nullptr, dev));
-    if (stats_acc_dev)
-      TRY(launch(dev, ADADSF_KERNEL_STATS, false, 0, 2.0 * xbytes_d,
-                 CALL(cos_stats(dt, at<char>(ws, m.xin), x, (int64_t)B * T, cfg->d, ADADSF_STATS_TOKEN,
-                                at<double>(ws, m.partials), stats_acc_dev + 2 * l, dev),
-                      "similarity statistics")));
-    idx_off += (int64_t)B * K;
+    DecodeCtx dc;
+    dc.thr = cv.thr + (int64_t)l * B;
+    dc.hdr = cv.hdr;
+    dc.lens = cv.lens + (int64_t)l * B;
+    dc.kc = cv.kc(l);
+    dc.vc = cv.vc(l);
+    dc.C_max = C_max;
+    dc.rows = at<int32_t>(ws, ds.rows);
+    dc.pos = at<int32_t>(ws, ds.pos);
+    dc.part_o = at<float>(ws, ds.part_o);
+    dc.part_ml = at<float2>(ws, ds.part_ml);
+    dc.kept_out = kept_out_dev ? kept_out_dev + (int64_t)l * B : nullptr;
+    TRY(layer_impl(cfg, &w->layers[l], x, B, 1, 1, lb, false, dev, nullptr, &dc));
   }
-  TRY(launch(dev, ADADSF_KERNEL_FINAL_NORM, false, 0, 2.0 * xbytes_d,
-             CALL(gather_norm(dt, x, nullptr, (int64_t)B * T, cfg->d, cfg->arch == ADADSF_ARCH_QWEN,
-                              w->final_w, w->final_b, nullptr, nullptr, cfg->norm_eps, hidden_out_dev,
-                              nullptr, dev),
+  TRY(launch(dev, ADADSF_KERNEL_FINAL_NORM, false, 0, 2.0 * B * cfg->d * es,
+             CALL(gather_norm(dt, x, nullptr, B, cfg->d, cfg->arch == ADADSF_ARCH_QWEN, w->final_w, w->final_b,
+                              nullptr, nullptr, cfg->norm_eps, hidden_out_dev, nullptr, dev),
                   "final norm")));
+  TRY(launch(dev, ADADSF_KERNEL_KV_CACHE, false, 0, 8.0, CALL(decode_advance(cv.hdr, dev), "advance position")));
   return ADADSF_OK;
 }
 
@@ -1084,7 +1344,7 @@ const char* adadsf_kernel_name(int kind) {
   static const char* names[ADADSF_KERNEL_COUNT] = {
       "embed", "router", "topk", "positions", "gather_norm", "gemm_qkv", "rope_table", "rope",
       "attention", "gemm_o", "norm2", "gemm_up", "gemm_down", "stats", "final_norm", "copy",
-      "linear", "selftest", "gemm_qkv_up", "gemm_o_down", "topk_gather_norm"};
+      "linear", "selftest", "gemm_qkv_up", "gemm_o_down", "topk_gather_norm", "decide", "kv_cache"};
   return (kind >= 0 && kind < ADADSF_KERNEL_COUNT) ? names[kind] : "unknown";
 }
 

@@ -67,6 +67,7 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(const SimtDev p) {
     const int m = row0 + ty * 4 + i;
     if (m >= p.M) continue;
     const int64_t arow = p.rows ? (int64_t)p.rows[m] : (int64_t)m;
+    if (arow < 0) continue;   // a row that bypasses the layer: nothing read or written
     const int64_t orow = p.out_mapped ? arow : (int64_t)m;
     const float g = p.gate ? 1.f / (1.f + expf(-p.gate[arow])) : 1.f;
 #pragma unroll

@@ -442,9 +442,12 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
                                               const EpiPre& pre, const EpiRed& red, uint32_t stg,
                                               int lane) {
   constexpr bool rope = ROPE && !DUAL;
-  const bool mvalid = m < p.M;
+  bool mvalid = m < p.M;
   int64_t arow = m;
-  if (mvalid && p.rows) arow = p.rows[m];
+  if (mvalid && p.rows) {
+    arow = p.rows[m];
+    if (arow < 0) mvalid = false;   // a row that bypasses the layer: nothing read or written
+  }
   const int64_t orow = p.out_mapped ? arow : (int64_t)m;
   float gate = 1.f;
   if (!ROPE && p.gate && mvalid) gate = 1.f / (1.f + expf(-p.gate[arow]));
@@ -545,6 +548,7 @@ __device__ __forceinline__ void prefetch_res(const GemmDev& p, int m, int nb, in
   pre.n = 0;
   if (!p.add || m >= p.M) return;
   const int64_t rrow = p.add_gathered ? (int64_t)p.rows[m] : (int64_t)m;
+  if (rrow < 0) return;
   const int n = min(2, c_hi - c_lo);
   for (int k = 0; k < n; ++k) {
     const int n0 = nb * bn + (c_lo + k) * 32;

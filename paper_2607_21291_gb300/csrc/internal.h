@@ -21,6 +21,7 @@ enum Act : int { ACT_NONE = 0, ACT_GELU = 1, ACT_SWIGLU = 2 };
 //   v += add_packed[m][n]                     (may be null)
 //   v += add_rows[row(m)][n]                  (may be null)
 //   out[out_mapped ? row(m) : m][n] = v       row(m) = rows ? rows[m] : m
+// A packed row with rows[m] < 0 is skipped: no residual read, no store.
 // Score gate (gate_scores set; the gated variant of Sec. 3.4): with
 // g = sigmoid(gate_scores[row(m)]) and t = v + add_packed[m][n],
 //   out = add_rows[row(m)][n] + g t                                (no gate_base)
@@ -151,5 +152,21 @@ cudaError_t bounded_wait_selftest(int timeout_us, const Dev& dev);
 int stats_static_capacity();
 cudaError_t cos_stats_static(int dtype, const void* a, const void* b, int64_t n_rows, int d,
                              int mode, double* acc, const Dev& dev);
+
+// decode.cu -- generation with a cache of kept tokens only (see decode.cu).
+int decode_splits(int B, int Hkv, int C_max, int num_sms);
+cudaError_t kv_fill(int dtype, const void* qkv, int64_t ld, int q, int kvw, int B, int K, int hd,
+                    int C_max, void* kc, void* vc, const Dev& dev);
+cudaError_t kv_threshold(const float* scores, const int32_t* idx, int B, int T, int K, int32_t* lens,
+                         float* thr, const Dev& dev);
+cudaError_t cache_header(int32_t* hdr, int T, int C_max, int L, int B, const Dev& dev);
+cudaError_t decode_decide(const float* scores, const float* thr, const int32_t* hdr, int B, int C_max,
+                          int32_t* rows, int32_t* pos, int32_t* kept_out, const Dev& dev);
+cudaError_t decode_attention(int dtype, const void* qkv, int64_t ld, int Hq, int Hkv, int hd, const void* kc,
+                             const void* vc, const int32_t* lens, int C_max, int B, float* part_o,
+                             float2* part_ml, void* out, int64_t ld_out, const Dev& dev);
+cudaError_t kv_append(int dtype, const void* qkv, int64_t ld, int q, int kvw, int hd, int B, const int32_t* rows,
+                      int32_t* lens, int C_max, void* kc, void* vc, const Dev& dev);
+cudaError_t decode_advance(int32_t* hdr, const Dev& dev);
 
 }  // namespace adadsf

@@ -133,3 +133,23 @@ def test_argument_errors_precede_launch(A):
                                     None) == A.ERR_INVALID_ARG
     assert lib.adadsf_router_select_workspace_size(ctypes.byref(cfg), 4, 512) > 256 + 4 * (16 + 4)
     assert lib.adadsf_layer_stats(None, None, 4, 64, A.BF16, 0, None, None, 0, None) == A.ERR_INVALID_ARG
+
+
+def test_decode_argument_errors_precede_launch(A):
+    lib = A.lib()
+    cfg = A.make_cfg(S.PYTHIA_160M)
+    n = lib.adadsf_kv_cache_size(ctypes.byref(cfg), 2, 100)
+    # header + counts + thresholds + rotary table + K and V of 12 layers
+    assert n >= 12 * 2 * (2 * 12 * 100 * 64 * 2)
+    assert lib.adadsf_kv_cache_size(ctypes.byref(cfg), 0, 100) == 0
+    # the prompt must leave room in the cache
+    assert lib.adadsf_prefill(ctypes.byref(cfg), None, None, 2, 100, None, None, None, None, n, 100, None, 0,
+                              None) == A.ERR_INVALID_ARG
+    assert "C_max" in A.adadsf_last_error()
+    buf = ctypes.create_string_buffer(1024)
+    base = (ctypes.addressof(buf) + 255) & ~255
+    assert lib.adadsf_prefill(ctypes.byref(cfg), None, None, 2, 50, None, None, None, base, 256, 100, None, 0,
+                              None) == A.ERR_WORKSPACE_TOO_SMALL
+    assert lib.adadsf_decode_step(ctypes.byref(cfg), None, None, 2, None, None, None, n, 100, None, 0,
+                                  None) == A.ERR_INVALID_ARG
+    assert lib.adadsf_decode_workspace_size(ctypes.byref(cfg), 2, 100) > 0

@@ -1,0 +1,147 @@
+"""GPU parity of generation with a kept-token cache (adadsf_prefill, then
+adadsf_decode_step) against the oracle's sparse_prefill / decode_step,
+through the C ABI.
+
+The GPU's prompt kept sets are given to the oracle (kept-set rules as for the
+sparse forward), and so are its per-step keep decisions; each decision must
+equal the oracle's own wherever the oracle's score is more than 1e-3 away
+from its threshold. Hidden states within the parity tolerance; cached counts
+follow the decisions; the cache's thresholds match the oracle's."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import adadsf_oracle as O
+from paper_2607_21291_gb300 import synth as S
+from tests import helpers as H
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def A():
+    from paper_2607_21291_gb300 import adadsf
+    adadsf.lib()
+    return adadsf
+
+
+QWEN_SMALL = S.QWEN25_1_5B.replace(d=1024, n_heads=8, n_kv_heads=2, ffn=1536, n_layers=3, vocab=500)
+NEOX_SMALL = S.PYTHIA_160M.replace(n_layers=3, vocab=500)
+NEOX_F32 = S.PYTHIA_70M.replace(n_layers=2, vocab=500)
+
+CASES = [
+    # (shape, B, T0, K per layer, steps, C_max, gated)
+    (NEOX_SMALL, 3, 64, [64, 20, 40], 5, 80, False),
+    (QWEN_SMALL, 2, 100, [50, 100, 0], 4, 128, False),
+    (QWEN_SMALL, 2, 96, [48, 30, 96], 3, 100, True),
+    (NEOX_F32, 2, 40, [20, 40], 4, 48, False),
+]
+
+
+def _cache_counts(A, cache, L, B):
+    """Per-layer kept counts and thresholds from the cache header area
+    ([L][B] int32 at byte 256, then [L][B] fp32 256-aligned)."""
+    lens = cache[256:256 + 4 * L * B].view(torch.int32).view(L, B).cpu().numpy()
+    off = 256 + ((4 * L * B + 255) // 256) * 256
+    thr = cache[off:off + 4 * L * B].view(torch.float32).view(L, B).cpu().numpy()
+    return lens, thr
+
+
+@pytest.mark.parametrize("shape,B,T0,K,steps,C_max,gated", CASES)
+def test_prefill_then_decode(A, shape, B, T0, K, steps, C_max, gated):
+    L = shape.n_layers
+    td = H.tdtype(shape)
+    flags = A.FLAG_GATE_SIGMOID if gated else 0
+    hostL = [H.host_layer(shape, 13, l) for l in range(L)]
+    extra = H.host_extra(shape, 13)
+    model = A.DeviceModel(A.make_cfg(shape, flags), [A.to_device(w, td) for w in hostL], A.to_device(extra, td))
+    ids = S.token_ids(14, B, T0 + steps, shape.vocab)
+    ids_d = torch.from_numpy(ids).cuda()
+    cache = A.kv_cache(model.cfg, B, C_max)
+    hidden = torch.empty((B, T0, shape.d), dtype=td, device="cuda")
+    idx = torch.full((B * sum(K),), -1, dtype=torch.int32, device="cuda")
+    ws = A.workspace(A.adadsf_model_workspace_size(model.cfg, B, T0, K, False))
+    A.adadsf_prefill(model, ids_d[:, :T0].contiguous(), K, hidden, cache, C_max, idx_out=idx, ws=ws)
+    assert A.adadsf_sync_check(ws) == A.OK
+    gi, off, kept_sets = idx.cpu().numpy(), 0, []
+    for k in K:
+        kept_sets.append(gi[off:off + B * k].reshape(B, k))
+        off += B * k
+    p = dict(O.params_of(shape), gate="sigmoid") if gated else O.params_of(shape)
+    W64 = [H.f64(w) for w in hostL]
+    E64 = H.f64(extra)
+    ref, st = O.sparse_prefill(ids[:, :T0], E64, W64, p, K, idx_force=kept_sets)
+    H.assert_close(H.to_np(hidden), ref, H.tol(shape), "prefill")
+    lens, thr = _cache_counts(A, cache, L, B)
+    assert lens.tolist() == [[k] * B for k in K]
+    thr_ref = np.array(st["thr"])
+    finite = np.isfinite(thr_ref)
+    assert (np.isinf(thr) == ~finite).all() and (thr[~finite] > 0).all()   # K = 0: +inf
+    sc_tol = 5e-3 if shape.dtype == "bf16" else 1e-5
+    assert np.abs(thr[finite] - thr_ref[finite]).max(initial=0) <= sc_tol * max(1.0, np.abs(thr_ref[finite]).max(initial=0))
+
+    dws = A.workspace(A.adadsf_decode_workspace_size(model.cfg, B, C_max))
+    counts = np.array(lens, dtype=np.int64)
+    n_checked = 0
+    for step in range(steps):
+        h = torch.empty((B, shape.d), dtype=td, device="cuda")
+        kept = torch.full((L, B), -1, dtype=torch.int32, device="cuda")
+        A.adadsf_decode_step(model, ids_d[:, T0 + step].contiguous(), h, cache, C_max, kept_out=kept, ws=dws)
+        assert A.adadsf_sync_check(dws) == A.OK
+        kg = kept.cpu().numpy().astype(bool)
+        href, kown, sref = O.decode_step(ids[:, T0 + step], E64, W64, p, st, kept_force=kg)
+        margin = np.abs(sref - thr_ref) > 1e-3 * np.maximum(1.0, np.abs(thr_ref))
+        assert (kg[margin] == kown[margin]).all(), (step, kg, kown)
+        n_checked += int(margin.sum())
+        H.assert_close(H.to_np(h), href, H.tol(shape), f"decode step {step}")
+        counts += kg
+        lens, _ = _cache_counts(A, cache, L, B)
+        assert (lens == counts).all()
+    assert n_checked > 0
+    # a layer that kept no prompt token keeps no generated token
+    for l, k in enumerate(K):
+        if k == 0:
+            assert (counts[l] == 0).all()
+
+
+def test_decode_step_in_a_cuda_graph(A):
+    """A decode step reads its position and counts from the cache, so one
+    captured graph replays step after step: the same outputs as eager steps."""
+    shape = NEOX_SMALL
+    B, T0, C_max, K = 2, 48, 64, [24, 48, 12]
+    td = H.tdtype(shape)
+    hostL = [H.host_layer(shape, 21, l) for l in range(shape.n_layers)]
+    model = A.DeviceModel(A.make_cfg(shape), [A.to_device(w, td) for w in hostL],
+                          A.to_device(H.host_extra(shape, 21), td))
+    ids = torch.from_numpy(S.token_ids(22, B, T0 + 4, shape.vocab)).cuda()
+    outs = []
+    for use_graph in (False, True):
+        cache = A.kv_cache(model.cfg, B, C_max)
+        A.adadsf_prefill(model, ids[:, :T0].contiguous(), K,
+                         torch.empty((B, T0, shape.d), dtype=td, device="cuda"), cache, C_max)
+        dws = A.workspace(A.adadsf_decode_workspace_size(model.cfg, B, C_max))
+        tok = torch.empty(B, dtype=torch.int32, device="cuda")
+        h = torch.empty((B, shape.d), dtype=td, device="cuda")
+        stream = torch.cuda.Stream()
+        res = []
+        with torch.cuda.stream(stream):
+            if use_graph:
+                tok.copy_(ids[:, T0])
+                A.adadsf_decode_step(model, tok, h, cache, C_max, ws=dws, stream=stream)   # warm-up step
+                res.append(h.clone())
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=stream):
+                    A.adadsf_decode_step(model, tok, h, cache, C_max, ws=dws, stream=stream)
+                for t in range(1, 4):
+                    tok.copy_(ids[:, T0 + t])
+                    g.replay()
+                    res.append(h.clone())
+            else:
+                for t in range(4):
+                    tok.copy_(ids[:, T0 + t])
+                    A.adadsf_decode_step(model, tok, h, cache, C_max, ws=dws, stream=stream)
+                    res.append(h.clone())
+        torch.cuda.synchronize()
+        assert A.adadsf_sync_check(dws) == A.OK
+        outs.append(torch.stack(res))
+    assert torch.equal(outs[0], outs[1])

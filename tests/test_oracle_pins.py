@@ -628,7 +628,7 @@ class TestDecode:
         decided = [[list(st["pos"][l][b]) for b in range(3)] for l in range(3)]
         n_kept = 0
         for t in (10, 11):
-            h, kept = O.decode_step(ids[:, t], Wm, layers, p, st)
+            h, kept, _ = O.decode_step(ids[:, t], Wm, layers, p, st)
             n_kept += kept.sum()
             for l in range(3):
                 for b in range(3):
@@ -648,7 +648,7 @@ class TestDecode:
         ids = rng(61).integers(0, 30, size=(2, 8))
         _, st = O.sparse_prefill(ids[:, :7], Wm, layers, p, [7, 7, 7])
         st["thr"] = [[-np.inf] * 2 for _ in range(3)]
-        h, kept = O.decode_step(ids[:, 7], Wm, layers, p, st)
+        h, kept, _ = O.decode_step(ids[:, 7], Wm, layers, p, st)
         assert kept.all()
         x = np.asarray(Wm["embed"])[ids]
         for W in layers:
@@ -661,7 +661,7 @@ class TestDecode:
         ids = rng(71).integers(0, 30, size=(2, 6))
         _, st = O.sparse_prefill(ids[:, :5], Wm, layers, p, [2, 2, 2])
         st["thr"] = [[np.inf] * 2 for _ in range(3)]
-        h, kept = O.decode_step(ids[:, 5], Wm, layers, p, st)
+        h, kept, _ = O.decode_step(ids[:, 5], Wm, layers, p, st)
         assert not kept.any()
         assert h == pytest.approx(O.rms_norm(np.asarray(Wm["embed"])[ids[:, 5]], Wm["final_w"], p["norm_eps"]),
                                   rel=1e-14)
