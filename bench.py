@@ -176,15 +176,22 @@ def rank_seed(seed, rank):
 
 def device_model(A, shape, seed, device):
     """Random-init weights of the backbone shape in the benchmark recipe,
-    drawn on the device (the reference arm draws the same tensors)."""
+    drawn on the device (the reference arm draws the same tensors), with the
+    norm parameters folded into the projections (adadsf_fold_norms; exact
+    here, as the recipe's gains are 1 and biases 0) so that the layers run
+    with ADADSF_FLAG_FOLDED_NORMS."""
     td = torch.bfloat16 if shape.dtype == "bf16" else torch.float32
-    layers = [{k: v.to(td) for k, v in S.bench_layer_weights(shape, seed, l, device).items()}
-              for l in range(shape.n_layers)]
+    cfg = A.make_cfg(shape, A.FLAG_FOLDED_NORMS)
+    layers = []
+    for l in range(shape.n_layers):
+        w = {k: v.to(td) for k, v in S.bench_layer_weights(shape, seed, l, device).items()}
+        A.adadsf_fold_norms(cfg, w)
+        layers.append(w)
     extra = {"embed": S.bench_embed(shape, seed, device).to(td),
              "final_w": torch.ones(shape.d, device=device, dtype=td)}
     if shape.arch == S.NEOX:
         extra["final_b"] = torch.zeros(shape.d, device=device, dtype=td)
-    return A.DeviceModel(A.make_cfg(shape), layers, extra)
+    return A.DeviceModel(cfg, layers, extra)
 
 
 def shared_config(wl, t_target, world):
@@ -343,6 +350,12 @@ def run_ours(args, rank, world, local_rank):
                                "dense": all(k == T for k in Kt)}
         assert A.adadsf_sync_check(ws, stream) == A.OK, A.adadsf_last_error()
 
+        # ---- generation: prefill the batch into a kept-token cache, then
+        # decode steps (one token per sequence) replayed from a CUDA graph
+        decode = None
+        if args.decode_steps > 0:
+            decode = run_decode(A, model, shape, ids, K, B, T, args, stream, device, world)
+
         # ---- end to end through the public call, host buffers in and out
         ids_host = ids.cpu().pin_memory()
         out_host = torch.empty(hidden.shape, dtype=hidden.dtype, pin_memory=True)
@@ -472,6 +485,7 @@ def run_ours(args, rank, world, local_rank):
                                "steps": n_side},
         "retention_sweep": sweep,
         "hbm_path": hbm_path,
+        "decode": decode,
         "calibration": {"ms": calib_ms, "stats_kernel": stats_kernel, "batch": list(wl.calib)},
         "normalized_flops": A.adadsf_normalized_flops(model.cfg, T, K),
         "kernels": kernels,
@@ -484,6 +498,58 @@ def run_ours(args, rank, world, local_rank):
     if world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(model, shape, K, ids, budget_s=args.cpu_budget)
     print(json.dumps(out), flush=True)
+
+
+def run_decode(A, model, shape, ids, K, B, T, args, stream, device, world):
+    """Prefill of the evaluation batch into a kept-token cache at the plan's
+    K_l, then args.decode_steps decode steps (one new token per sequence),
+    captured once in a CUDA graph and replayed; per step the algorithmic HBM
+    bytes are every layer's weights (routers included) plus the cached keys
+    and values the step's attention reads."""
+    L, n = shape.n_layers, args.decode_steps
+    C_max = T + n + 8
+    cache = A.kv_cache(model.cfg, B, C_max, device)
+    hid = torch.empty((B, T, shape.d), dtype=torch.bfloat16, device=device)
+    pws = A.workspace(A.adadsf_model_workspace_size(model.cfg, B, T, K, False), device)
+    A.adadsf_prefill(model, ids, K, hid, cache, C_max, ws=pws, stream=stream)
+    del hid, pws
+    dws = A.workspace(A.adadsf_decode_workspace_size(model.cfg, B, C_max), device)
+    new_ids = S.counter_ids(rank_seed(3, 0), n + 1, B, shape.vocab, device)
+    tok = torch.empty(B, dtype=torch.int32, device=device)
+    h = torch.empty((B, shape.d), dtype=torch.bfloat16, device=device)
+    kept = torch.zeros((L, B), dtype=torch.int32, device=device)
+    kept_sum = torch.zeros((L, B), dtype=torch.int64, device=device)
+    tok.copy_(new_ids[0])
+    A.adadsf_decode_step(model, tok, h, cache, C_max, kept_out=kept, ws=dws, stream=stream)   # outside the graph
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        A.adadsf_decode_step(model, tok, h, cache, C_max, kept_out=kept, ws=dws, stream=stream)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+    torch.cuda.synchronize()
+    for i, (e0, e1) in enumerate(ev):
+        tok.copy_(new_ids[i + 1])
+        e0.record(stream)
+        g.replay()
+        e1.record(stream)
+        kept_sum += kept
+    torch.cuda.synchronize()
+    assert A.adadsf_sync_check(dws, stream) == A.OK, A.adadsf_last_error()
+    ms = float(np.mean([e0.elapsed_time(e1) for e0, e1 in ev]))
+    es = 2 if shape.dtype == "bf16" else 4
+    w_bytes = sum(v.numel() for lw in model.layers for v in lw.values()) * es
+    # cached keys / values read by the timed steps: the prompt's kept tokens
+    # plus those kept during the steps (mean over the steps)
+    kv_tok = sum(K) * B + float(kept_sum.sum()) / 2
+    kv_bytes = kv_tok * 2 * shape.kv_dim * es
+    peaks, _ = load_peaks()
+    bytes_step = w_bytes + kv_bytes
+    gbs = bytes_step / (ms * 1e6)
+    return {"steps": n, "ms_per_step": ms, "value": B * world / (ms * 1e-3), "unit": "tokens/s",
+            "prompt": T, "kept_fraction": float(kept_sum.sum()) / (n * L * B),
+            "roofline": {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": gbs / peaks["hbm_gbs"], "bytes_per_step": bytes_step},
+            "how": f"prefill of the batch at this line's K_l into a kept-token cache, then {n} decode steps "
+                   "(one token per sequence) replayed from one CUDA graph, CUDA events per step"}
 
 
 def host_threads() -> int:
@@ -666,6 +732,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=20.0)
     ap.add_argument("--spin-up", type=float, default=1.5, help="seconds of untimed GPU work before measuring")
+    ap.add_argument("--decode-steps", type=int, default=32, help="decode steps timed after a prefill (0: none)")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
 

@@ -68,6 +68,13 @@ typedef enum { ADADSF_STATS_TOKEN = 0, ADADSF_STATS_FLAT = 1 } adadsf_stats_mode
  * K == T is exactly the dense layer. With it the router runs even when
  * K == T. */
 #define ADADSF_FLAG_GATE_SIGMOID 1u
+/* ADADSF_FLAG_FOLDED_NORMS: every layer's norm gains are 1 and (GPT-NeoX)
+ * norm biases 0, their values folded into the projections that read the
+ * normed rows (what adadsf_fold_norms leaves). The layers may then apply a
+ * norm's row scale inside those projections instead of a separate pass
+ * (bf16 Qwen: the post-attention RMSNorm). With unfolded weights the flag
+ * gives wrong results. */
+#define ADADSF_FLAG_FOLDED_NORMS 2u
 
 /* adadsf_alloc_ratios flags */
 #define ADADSF_ALLOC_RAW 1u      /* return Eq. 8 unclamped (ratios may exceed 1) */
@@ -198,6 +205,19 @@ adadsf_status adadsf_similarity(const double *acc_host, int L, int mode, double 
  * ---------------------------------------------------------------------- */
 adadsf_status adadsf_alloc_ratios(const double *s_host, int L, double t, double tau, double beta,
                                   int T, unsigned flags, double *r_out_host, int32_t *K_out_host);
+
+/* ------------------------------------------------------------------------
+ * Folds one layer's norm parameters into the projections that read the normed
+ * rows, IN PLACE (a reparameterisation; the layer computes the same function
+ * up to one bf16 rounding of the changed weights): for a norm n(x) g + b
+ * feeding W with bias c, W <- W diag(g) and c <- c + W b (GPT-NeoX: ln1 ->
+ * w_qkv / b_qkv, ln2 -> w_up / b_up; Qwen: ln1_w -> w_qkv, ln2_w -> w_gate
+ * and w_up), then g <- 1 and b <- 0. The tensors of `w` are modified (their
+ * pointers are const in the struct; they must be writable device memory).
+ * Afterwards the layer may run with ADADSF_FLAG_FOLDED_NORMS. Asynchronous
+ * on `stream`. No paper counterpart (an implementation device).
+ * ---------------------------------------------------------------------- */
+adadsf_status adadsf_fold_norms(const adadsf_model_cfg *cfg, const adadsf_layer_weights *w, void *stream);
 
 /* ------------------------------------------------------------------------
  * Sec. 4.1 (the normalized FLOPs of Tables 1-2): FLOPs of the depth-sparse

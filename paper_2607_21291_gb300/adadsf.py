@@ -25,6 +25,7 @@ STATS_TOKEN, STATS_FLAT = 0, 1
 LINEAR_SPLIT_WS_BYTES = 256 + 160 * 128 * 256 * 4   # ADADSF_LINEAR_SPLIT_WS_BYTES
 ALLOC_RAW, ALLOC_ROUND = 1, 2
 FLAG_GATE_SIGMOID = 1
+FLAG_FOLDED_NORMS = 2
 
 TORCH_DTYPE = {F32: torch.float32, BF16: torch.bfloat16}
 DTYPE_CODE = {torch.float32: F32, torch.bfloat16: BF16}
@@ -84,6 +85,7 @@ def lib() -> ctypes.CDLL:
             "adadsf_layer_stats_noalloc": (i32, [vp, vp, i64, i32, i32, i32, vp, vp]),
             "adadsf_similarity": (i32, [vp, i32, i32, vp]),
             "adadsf_normalized_flops": (i32, [pcfg, i32, vp, vp]),
+            "adadsf_fold_norms": (i32, [pcfg, plw, vp]),
             "adadsf_alloc_ratios": (i32, [vp, i32, f64, f64, f64, i32, u32, vp, vp]),
             "adadsf_router_scores": (i32, [pcfg, plw, vp, i64, vp, vp, sz, vp]),
             "adadsf_topk_select": (i32, [vp, i32, i32, i32, vp, vp, vp]),
@@ -230,6 +232,13 @@ def adadsf_similarity(acc, mode: int = STATS_TOKEN) -> np.ndarray:
     _check(lib().adadsf_similarity(a.ctypes.data_as(ctypes.c_void_p), L, int(mode),
                                    s.ctypes.data_as(ctypes.c_void_p)))
     return s
+
+
+def adadsf_fold_norms(cfg: ModelCfg, w: dict, stream=None):
+    """Folds the layer's norm parameters into its projections, modifying the
+    device tensors of w in place (then run with FLAG_FOLDED_NORMS)."""
+    lw = layer_struct(w)
+    _check(lib().adadsf_fold_norms(ctypes.byref(cfg), ctypes.byref(lw), _s(stream)))
 
 
 def adadsf_normalized_flops(cfg: ModelCfg, T: int, K: Sequence[int]) -> float:

@@ -96,12 +96,13 @@ adadsf_status check_cfg(const adadsf_model_cfg* c) {
     return fail(ADADSF_ERR_INVALID_ARG, "rotary_dim=%d must be even and <= head_dim", c->rotary_dim);
   if (!(c->norm_eps > 0.f) || !(c->rope_theta > 0.f))
     return fail(ADADSF_ERR_INVALID_ARG, "norm_eps and rope_theta must be positive");
-  if ((unsigned)c->flags & ~(unsigned)ADADSF_FLAG_GATE_SIGMOID)
+  if ((unsigned)c->flags & ~(unsigned)(ADADSF_FLAG_GATE_SIGMOID | ADADSF_FLAG_FOLDED_NORMS))
     return fail(ADADSF_ERR_UNSUPPORTED, "flags 0x%x has unknown bits", (unsigned)c->flags);
   return ADADSF_OK;
 }
 
 bool gated(const adadsf_model_cfg* c) { return ((unsigned)c->flags & ADADSF_FLAG_GATE_SIGMOID) != 0; }
+bool folded(const adadsf_model_cfg* c) { return ((unsigned)c->flags & ADADSF_FLAG_FOLDED_NORMS) != 0; }
 
 adadsf_status check_shape(int B, int T, int K) {
   if (B < 0 || T <= 0 || K < 0 || K > T)
@@ -206,7 +207,7 @@ struct Carver {
 };
 
 struct LayerSlots {
-  size_t scores, idx, rows, n1, n2, qkv, vt, attn, ao, act, split, rsel;
+  size_t scores, idx, rows, n1, n2, qkv, vt, attn, ao, act, split, rsel, sq;
 };
 
 void carve_layer(const adadsf_model_cfg* c, int B, int T, int K, Carver& cv, LayerSlots& s) {
@@ -229,6 +230,9 @@ void carve_layer(const adadsf_model_cfg* c, int B, int T, int K, Carver& cv, Lay
   // router partial tiles (tensor-core path; its counters sit in the
   // workspace's synchronisation area)
   s.rsel = c->dtype == ADADSF_BF16 ? cv.take(router_partial_bytes()) : 0;
+  // per-chunk sums of squares of h (Qwen, bf16, folded norms: the second
+  // RMSNorm applied in the gate / up epilogue)
+  s.sq = c->dtype == ADADSF_BF16 && c->arch == ADADSF_ARCH_QWEN ? cv.take(M * (c->d / 32) * 4) : 0;
 }
 
 size_t rope_bytes(const adadsf_model_cfg* c, int T) { return (size_t)T * (c->rotary_dim / 2) * 8; }
@@ -248,6 +252,8 @@ struct LayerBufs {
   float* split;   // null on the fp32 path
   int* sync;       // the workspace's synchronisation area
   float* rpart;    // router partial tiles, null on the fp32 path
+  float* sq = nullptr;        // [M][d/32] chunk sums of squares of h (folded second RMSNorm)
+  float4* cospart = nullptr;  // [B T][d/32] Eq. 4 partials from the down epilogue (dense, bf16)
 };
 
 adadsf_status run_linear(int dtype, const GemmArgs& g, const Dev& dev, const char* what) {
@@ -488,6 +494,11 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
     g.epi.out = x;
     g.epi.ld_out = d;
     if (gate) g.epi.gate_scores = lb.scores;   // x[row] + sigmoid(s) delta
+    if (lb.cospart) {
+      // Eq. 4 partials of (x_in, x_out) per chunk; the residual rows are x_in
+      g.epi.cos_out = lb.cospart;
+      g.epi.cos_ld = d / 32;
+    }
     TRY(launch(dev, ADADSF_KERNEL_GEMM_O_DOWN, true, 2.0 * M * d * ((double)q + F),
                ((double)M * (q + F) + (double)d * (q + F) + 2.0 * Md) * es,
                [&] { return run_linear(dt, g, dev, "output + mlp down projections + residual scatter"); }));
@@ -537,17 +548,31 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
     g.epi.out_mapped = false;
     g.epi.out = lb.ao;
     g.epi.ld_out = d;
+    // folded second RMSNorm (bf16): the O epilogue also leaves each h row's
+    // chunk sums of squares; the gate / up epilogue turns them into its rstd
+    const bool fold2 = tc && folded(c) && lb.sq;
+    if (fold2) {
+      g.epi.sq_out = lb.sq;
+      g.epi.sq_ld = d / 32;
+    }
     TRY(launch(dev, ADADSF_KERNEL_GEMM_O, tc, 2.0 * M * d * q,
                ((double)M * q + (double)d * q + 2.0 * Md) * es,
                [&] { return run_linear(dt, g, dev, "output projection + residual"); }));
-    // a4': RMS2(h)
-    TRY(launch(dev, ADADSF_KERNEL_NORM2, false, 0, 2.0 * Md * es,
-               CALL(gather_norm(dt, lb.ao, nullptr, M, d, true, w->ln2_w, nullptr, nullptr, nullptr,
-                                c->norm_eps, lb.n1, nullptr, dev),
-                    "post-attention norm")));
+    // a4': RMS2(h) (a pass of its own unless folded)
+    if (!fold2)
+      TRY(launch(dev, ADADSF_KERNEL_NORM2, false, 0, 2.0 * Md * es,
+                 CALL(gather_norm(dt, lb.ao, nullptr, M, d, true, w->ln2_w, nullptr, nullptr, nullptr,
+                                  c->norm_eps, lb.n1, nullptr, dev),
+                      "post-attention norm")));
     // a8: act = SiLU(h' W_gate^T) * (h' W_up^T)
-    GemmArgs u = linear_args(lb.n1, d, w->w_gate, M, F, d);
+    GemmArgs u = linear_args(fold2 ? lb.ao : lb.n1, d, w->w_gate, M, F, d);
     u.W2 = w->w_up;
+    if (fold2) {
+      u.epi.nrm_psum = lb.sq;
+      u.epi.nrm_nps = d / 32;
+      u.epi.nrm_d = d;
+      u.epi.nrm_eps = c->norm_eps;
+    }
     u.epi.act = ACT_SWIGLU;
     u.epi.out = lb.act;
     u.epi.ld_out = F;
@@ -570,6 +595,13 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
       dn.epi.gate_base = x;
       dn.epi.ld_gate_base = d;
     }
+    if (lb.cospart) {
+      // Eq. 4 partials of (x_in, x_out) per chunk, x_in read before it is overwritten
+      dn.epi.cos_out = lb.cospart;
+      dn.epi.cos_ld = d / 32;
+      dn.epi.cos_in = x;
+      dn.epi.ld_cos_in = d;
+    }
     TRY(launch(dev, ADADSF_KERNEL_GEMM_DOWN, tc, 2.0 * M * d * F,
                ((double)M * F + (double)d * F + (gate ? 3.0 : 2.0) * Md) * es,
                [&] { return run_linear(dt, dn, dev, "mlp down + residual scatter"); }));
@@ -588,7 +620,7 @@ size_t layer_ws_bytes(const adadsf_model_cfg* c, int B, int T, int K) {
 }
 
 struct ModelSlots {
-  size_t x, xin, partials, rope;
+  size_t x, xin, partials, cospart, rope;
   LayerSlots layer;
   size_t total;
 };
@@ -601,6 +633,9 @@ void carve_model(const adadsf_model_cfg* c, int B, int T, int Kmax, bool stats, 
   m.x = cv.take((size_t)B * T * c->d * es);
   m.xin = stats ? cv.take((size_t)B * T * c->d * es) : 0;
   m.partials = stats ? cv.take((size_t)stats_partials_count((int64_t)B * T) * 3 * 8) : 0;
+  // bf16: the Eq. 4 partials of dense layers come from the down epilogue, 16
+  // bytes per row and 32-column chunk
+  m.cospart = stats && c->dtype == ADADSF_BF16 ? cv.take((size_t)B * T * (c->d / 32) * 16) : 0;
   m.rope = cv.take(rope_bytes(c, T));
   carve_layer(c, B, T, Kmax, cv, m.layer);
   m.total = cv.cur;
@@ -731,12 +766,18 @@ adadsf_status model_forward_impl(const adadsf_model_cfg* cfg, const adadsf_model
   lb.split = m.layer.split ? at<float>(ws, m.layer.split) : nullptr;
   lb.sync = at<int>(ws, kErrBytes);
   lb.rpart = m.layer.rsel ? at<float>(ws, m.layer.rsel) : nullptr;
+  lb.sq = m.layer.sq ? at<float>(ws, m.layer.sq) : nullptr;
   const size_t xbytes = (size_t)B * T * cfg->d * es;
   int64_t idx_off = 0;
   for (int l = 0; l < cfg->n_layers; ++l) {
     const int K = K_host[l];
     lb.idx = idx_out_dev ? idx_out_dev + idx_off : at<int32_t>(ws, m.layer.idx);
-    if (stats_acc_dev)
+    // Eq. 4 of a dense bf16 layer: partials from its down-projection epilogue
+    // (x_in and x_out are both at hand there); otherwise a copy of the input
+    // and a statistics pass
+    const bool fused_stats = stats_acc_dev && m.cospart && K == T;
+    lb.cospart = fused_stats ? at<float4>(ws, m.cospart) : nullptr;
+    if (stats_acc_dev && !fused_stats)
       TRY(launch(dev, ADADSF_KERNEL_COPY, false, 0, 2.0 * xbytes_d,
                  CALL(cudaMemcpyAsync(at<char>(ws, m.xin), x, xbytes, cudaMemcpyDeviceToDevice, dev.stream),
                       "copy of the layer input")));
@@ -749,7 +790,12 @@ adadsf_status model_forward_impl(const adadsf_model_cfg* cfg, const adadsf_model
       sink.C_max = cache->C_max;
     }
     TRY(layer_impl(cfg, &w->layers[l], x, B, T, K, lb, idx_out_dev != nullptr, dev, cache ? &sink : nullptr));
-    if (stats_acc_dev)
+    if (fused_stats)
+      TRY(launch(dev, ADADSF_KERNEL_STATS, false, 0, 16.0 * B * T * (cfg->d / 32),
+                 CALL(cos_stats_chunks(at<float4>(ws, m.cospart), (int64_t)B * T, cfg->d / 32, ADADSF_STATS_TOKEN,
+                                       at<double>(ws, m.partials), stats_acc_dev + 2 * l, dev),
+                      "similarity statistics")));
+    else if (stats_acc_dev)
       TRY(launch(dev, ADADSF_KERNEL_STATS, false, 0, 2.0 * xbytes_d,
                  CALL(cos_stats(dt, at<char>(ws, m.xin), x, (int64_t)B * T, cfg->d, ADADSF_STATS_TOKEN,
                                 at<double>(ws, m.partials), stats_acc_dev + 2 * l, dev),
@@ -933,6 +979,25 @@ adadsf_status adadsf_similarity(const double* acc_host, int L, int mode, double*
     }
     if (!isfinite(s_out_host[l])) return fail(ADADSF_ERR_INVALID_ARG, "layer %d: similarity is not finite", l);
   }
+  return ADADSF_OK;
+}
+
+adadsf_status adadsf_fold_norms(const adadsf_model_cfg* cfg, const adadsf_layer_weights* w, void* stream) {
+  TRY(check_cfg(cfg));
+  TRY(check_layer_weights(cfg, w, false));
+  const bool neox = cfg->arch == ADADSF_ARCH_NEOX;
+  if (neox) {
+    NEED_PTR(w->b_qkv, "b_qkv");
+    NEED_PTR(w->b_up, "b_up");
+  }
+  Dev dev;
+  TRY(device_info(&dev, stream, nullptr));
+  const int qkv = (cfg->n_heads + 2 * cfg->n_kv_heads) * cfg->head_dim;
+  auto mut = [](const void* p) { return const_cast<void*>(p); };
+  CUDA_TRY(fold_layer_norms(cfg->dtype, neox, cfg->d, qkv, cfg->ffn, mut(w->w_qkv), mut(w->b_qkv), mut(w->w_up),
+                            mut(w->b_up), mut(w->w_gate), mut(w->ln1_w), mut(w->ln1_b), mut(w->ln2_w),
+                            mut(w->ln2_b), dev),
+           "norm folding");
   return ADADSF_OK;
 }
 
@@ -1156,6 +1221,7 @@ adadsf_status adadsf_sparse_layer_forward(const adadsf_model_cfg* cfg, const ada
   lb.split = s.split ? at<float>(ws, s.split) : nullptr;
   lb.sync = at<int>(ws, kErrBytes);
   lb.rpart = s.rsel ? at<float>(ws, s.rsel) : nullptr;
+  lb.sq = s.sq ? at<float>(ws, s.sq) : nullptr;
   if (cfg->rotary_dim > 0)
     TRY(launch(dev, ADADSF_KERNEL_ROPE_TABLE, false, 0, rope_bytes(cfg, T),
                CALL(rope_table(at<float2>(ws, rope_off), T, cfg->rotary_dim, cfg->rope_theta, dev),
@@ -1254,6 +1320,7 @@ adadsf_status adadsf_decode_step(const adadsf_model_cfg* cfg, const adadsf_model
   lb.split = ds.layer.split ? at<float>(ws, ds.layer.split) : nullptr;
   lb.sync = at<int>(ws, kErrBytes);
   lb.rpart = ds.layer.rsel ? at<float>(ws, ds.layer.rsel) : nullptr;
+  lb.sq = ds.layer.sq ? at<float>(ws, ds.layer.sq) : nullptr;
   for (int l = 0; l < cfg->n_layers; ++l) {
     DecodeCtx dc;
     dc.thr = cv.thr + (int64_t)l * B;

@@ -106,6 +106,12 @@ struct GemmDev {
   // gbase + g (v + add - gbase) (add packed, gbase gathered)
   const float* gate;
   const bf16* gbase; int64_t ld_gbase;
+  // folded RMSNorm of the A rows (see Epilogue::nrm_psum)
+  const float* nrm_psum; int nrm_nps; float nrm_inv_d, nrm_eps;
+  // per-chunk sums of squares / Eq. 4 partials of the stored rows
+  float* sq_out; int sq_ld;
+  float4* cos_out; int cos_ld;
+  const bf16* cin; int64_t ld_cin;
   int* err;
   unsigned long long timeout_ns;
 };
@@ -283,7 +289,8 @@ __device__ __forceinline__ void store_chunk_rows(uint32_t stg, int lane, const u
 template <bool RES>
 __device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, const uint4* res,
                                                 float g, const uint4* gb, int64_t orow, int n0,
-                                                bool valid, uint32_t stg, int lane) {
+                                                bool valid, uint32_t stg, int lane, int64_t m,
+                                                const uint4* xin) {
   if (RES && p.add) {
     if (!p.gate) {
 #pragma unroll
@@ -321,6 +328,26 @@ __device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, cons
   uint4 pk[4];
 #pragma unroll
   for (int i = 0; i < 4; ++i) pk[i] = pack16(v + 8 * i, bf16());
+  if (RES && valid && (p.sq_out || p.cos_out)) {
+    // statistics of the stored (rounded) chunk for the next norm / Eq. 4
+    float sq = 0.f, dot = 0.f, nx = 0.f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      float o[8], a[8];
+      unpack16(pk[i], o, bf16());
+      if (p.cos_out) unpack16(xin[i], a, bf16());
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        sq = fmaf(o[j], o[j], sq);
+        if (p.cos_out) {
+          dot = fmaf(a[j], o[j], dot);
+          nx = fmaf(a[j], a[j], nx);
+        }
+      }
+    }
+    if (p.sq_out) p.sq_out[m * p.sq_ld + (n0 >> 5)] = sq;
+    if (p.cos_out) p.cos_out[m * p.cos_ld + (n0 >> 5)] = make_float4(dot, nx, sq, 0.f);
+  }
   store_chunk_rows(stg, lane, pk, valid ? p.out + orow * p.ld_out + n0 : nullptr);
 }
 
@@ -451,6 +478,15 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
   const int64_t orow = p.out_mapped ? arow : (int64_t)m;
   float gate = 1.f;
   if (!ROPE && p.gate && mvalid) gate = 1.f / (1.f + expf(-p.gate[arow]));
+  // folded RMSNorm of this A row: its rstd from the chunk sums of squares
+  float rs = 1.f;
+  if (p.nrm_psum && mvalid) {
+    const float* ps = p.nrm_psum + (int64_t)m * p.nrm_nps;
+    float sum = 0.f;
+#pragma unroll 4
+    for (int i = 0; i < p.nrm_nps; ++i) sum += ps[i];
+    rs = 1.f / sqrtf(sum * p.nrm_inv_d + p.nrm_eps);
+  }
   const float2* tab_row = nullptr;
   if (rope && mvalid)
     tab_row = p.rope_tab + (int64_t)(p.rope_pos ? p.rope_pos[m] : m % p.rope_T) * p.rope_half;
@@ -488,6 +524,10 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
         v[4 * j + 3] += f.w;
       }
     }
+    if (p.nrm_psum) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] *= rs;
+    }
     if (has_consts) add_consts32(sc, c * 32, v);
     if (!DUAL && p.vt && n0 >= p.vt_col0 && mvalid) {
       // value columns: also store this row's 32 features transposed
@@ -500,7 +540,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
     }
     if (DUAL) {
 #pragma unroll
-      for (int j = 0; j < 32; ++j) v[j] = silu_f(v[j]) * __uint_as_float(r2[j]);
+      for (int j = 0; j < 32; ++j) v[j] = silu_f(v[j]) * (rs * __uint_as_float(r2[j]));
     } else if (p.act == ACT_GELU) {
 #pragma unroll
       for (int j = 0; j < 32; j += 2) {
@@ -537,7 +577,14 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
 #pragma unroll
       for (int i = 0; i < 4; ++i) gb[i] = src[i];
     }
-    epi_chunk_store<!ROPE>(p, v, res, gate, gb, orow, n0, mvalid, stg, lane);
+    // the layer input of this chunk for the Eq. 4 partials
+    uint4 xi[4] = {res[0], res[1], res[2], res[3]};
+    if (!ROPE && p.cin && mvalid) {
+      const uint4* src = reinterpret_cast<const uint4*>(p.cin + arow * p.ld_cin + n0);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) xi[i] = src[i];
+    }
+    epi_chunk_store<!ROPE>(p, v, res, gate, gb, orow, n0, mvalid, stg, lane, m, xi);
   }
 }
 
@@ -1269,6 +1316,24 @@ bool make_dev(const GemmArgs& a, const Dev& dev, GemmDev& p) {
   p.rows = a.epi.rows;
   p.out_mapped = a.epi.out_mapped ? 1 : 0;
   p.out = static_cast<bf16*>(a.epi.out); p.ld_out = a.epi.ld_out;
+  if (a.epi.nrm_psum) {
+    if (a.epi.rope_tab || a.epi.nrm_d <= 0) return false;
+    p.nrm_psum = a.epi.nrm_psum;
+    p.nrm_nps = a.epi.nrm_nps;
+    p.nrm_inv_d = 1.f / (float)a.epi.nrm_d;
+    p.nrm_eps = a.epi.nrm_eps;
+  }
+  if (a.epi.sq_out || a.epi.cos_out) {
+    // statistics of stored rows: plain or residual outputs, no rotary tiles
+    if (a.epi.rope_tab || a.N % 32 != 0) return false;
+    if (a.epi.cos_out && !a.epi.cos_in && !a.epi.add_rows) return false;
+    p.sq_out = a.epi.sq_out;
+    p.sq_ld = a.epi.sq_ld;
+    p.cos_out = a.epi.cos_out;
+    p.cos_ld = a.epi.cos_ld;
+    p.cin = static_cast<const bf16*>(a.epi.cos_in);
+    p.ld_cin = a.epi.ld_cos_in;
+  }
   if (a.epi.gate_scores) {
     // gated residual: x gathered (out = x + g v), or h packed with x as the base
     if (a.epi.rope_tab) return false;

@@ -54,6 +54,24 @@ struct Epilogue {
   const float* gate_scores = nullptr;
   const void* gate_base = nullptr;
   int64_t ld_gate_base = 0;
+  // RMSNorm of the A rows folded into the projection (its gain already in the
+  // weights; bf16 tensor-core path): acc *= rstd[m] before anything else,
+  // rstd = 1 / sqrt(sum_j nrm_psum[m * nrm_nps + j] / nrm_d + nrm_eps); for
+  // ACT_SWIGLU both accumulators are scaled.
+  const float* nrm_psum = nullptr;
+  int nrm_nps = 0, nrm_d = 0;
+  float nrm_eps = 0.f;
+  // Sum of squares of each stored 32-column chunk (of the bf16 values):
+  // sq_out[m * sq_ld + n / 32] (bf16 path; the next RMSNorm's statistics).
+  float* sq_out = nullptr;
+  int sq_ld = 0;
+  // Eq. 4 partials of each stored 32-column chunk (bf16 path), as float4
+  // {x_in . out, |x_in|^2, |out|^2, 0} at cos_out[m * cos_ld + n / 32]; x_in
+  // = cos_in[row(m)] when given, else the gathered residual add_rows.
+  float4* cos_out = nullptr;
+  int cos_ld = 0;
+  const void* cos_in = nullptr;
+  int64_t ld_cos_in = 0;
 };
 
 // acc = A . W^T (+ A2 . Wk2^T when K2 > 0: a second K source, bf16
@@ -148,6 +166,12 @@ cudaError_t iota_positions(int32_t* idx, int B, int K, const Dev& dev);
 cudaError_t cos_stats(int dtype, const void* a, const void* b, int64_t n_rows, int d, int mode,
                       double* partials, double* acc, const Dev& dev);
 cudaError_t bounded_wait_selftest(int timeout_us, const Dev& dev);
+// Eq. 4 sums from per-32-column-chunk partials {a.b, |a|^2, |b|^2} ([n_rows][nch]).
+cudaError_t cos_stats_chunks(const float4* parts, int64_t n_rows, int nch, int mode, double* partials,
+                             double* acc, const Dev& dev);
+// fold.cu -- norm gains (and GPT-NeoX norm biases) folded into the projections, in place.
+cudaError_t fold_layer_norms(int dtype, bool neox, int d, int qkv, int F, void* w_qkv, void* b_qkv, void* w_up,
+                             void* b_up, void* w_gate, void* g1, void* b1, void* g2, void* b2, const Dev& dev);
 // Workspace-free variant of cos_stats: partial sums in a fixed device array.
 int stats_static_capacity();
 cudaError_t cos_stats_static(int dtype, const void* a, const void* b, int64_t n_rows, int d,

@@ -493,6 +493,45 @@ __global__ void __launch_bounds__(kStatThreads) cos_rows_kernel(const T* a, cons
   }
 }
 
+// Eq. 4 from per-chunk partials {a.b, |a|^2, |b|^2} ([n_rows][nch] float4,
+// written by a projection epilogue): one warp per row sums its chunks (fp32,
+// fixed lane order), then the same per-block fixed-order fp64 sums as
+// cos_rows_kernel.
+__global__ void __launch_bounds__(kStatThreads) cos_chunks_kernel(const float4* parts, int64_t n_rows,
+                                                                  int nch, int mode, double* partials) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ double red[kStatThreads / 32][3];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int64_t nwarps = (int64_t)gridDim.x * (kStatThreads / 32);
+  double acc0 = 0, acc1 = 0, acc2 = 0;
+  for (int64_t r = (int64_t)blockIdx.x * (kStatThreads / 32) + w; r < n_rows; r += nwarps) {
+    float dot = 0.f, na = 0.f, nb = 0.f;
+    for (int c = lane; c < nch; c += 32) {
+      const float4 f = parts[r * nch + c];
+      dot += f.x;
+      na += f.y;
+      nb += f.z;
+    }
+    dot = warp_sum(dot);
+    na = warp_sum(na);
+    nb = warp_sum(nb);
+    if (mode == 0) {
+      const double den = fmax(sqrt((double)na), 1e-8) * fmax(sqrt((double)nb), 1e-8);
+      acc0 += (double)dot / den;
+    } else {
+      acc0 += dot; acc1 += na; acc2 += nb;
+    }
+  }
+  if (lane == 0) { red[w][0] = acc0; red[w][1] = acc1; red[w][2] = acc2; }
+  __syncthreads();
+  if (threadIdx.x < 3) {
+    double s = 0;
+    for (int i = 0; i < kStatThreads / 32; ++i) s += red[i][threadIdx.x];
+    partials[(int64_t)blockIdx.x * 3 + threadIdx.x] = s;
+  }
+}
+
 // Fixed-order sum of the per-block partials, added to acc.
 __global__ void cos_finish_kernel(const double* partials, int nblocks, int64_t n_rows, int mode,
                                   double* acc) {
@@ -757,6 +796,16 @@ cudaError_t cos_stats(int dtype, const void* a, const void* b, int64_t n_rows, i
   if (e != cudaSuccess) return e;
   return launch_pdl(cos_finish_kernel, dim3(1), dim3(256), 0, dev.stream, partials, nb, n_rows, mode,
                     acc);
+}
+
+cudaError_t cos_stats_chunks(const float4* parts, int64_t n_rows, int nch, int mode, double* partials,
+                             double* acc, const Dev& dev) {
+  if (n_rows <= 0) return cudaSuccess;
+  const int nb = stats_partials_count(n_rows);
+  cudaError_t e = launch_pdl(cos_chunks_kernel, dim3(nb), dim3(kStatThreads), 0, dev.stream, parts, n_rows, nch,
+                             mode, partials);
+  if (e != cudaSuccess) return e;
+  return launch_pdl(cos_finish_kernel, dim3(1), dim3(256), 0, dev.stream, partials, nb, n_rows, mode, acc);
 }
 
 int stats_static_capacity() { return kStatMaxBlocks; }

@@ -220,3 +220,67 @@ def test_model_qwen_end_to_end(A):
     extra = H.f64(H.host_extra(shape, 8))
     ref, _, _ = O.sparse_model_forward(ids, extra, hostL, O.params_of(shape), K, idx_force=kept)
     H.assert_close(H.to_np(hidden), ref, H.BF16_TOL, "qwen model")
+
+
+FOLD_CASES = [
+    # (shape, B, T, K): Qwen bf16 takes the folded second RMSNorm (no separate
+    # norm pass); GPT-NeoX and fp32 run their usual passes on folded weights
+    (QWEN_SMALL, 2, 150, 70),
+    (QWEN_SMALL, 4, 2048, 1024),
+    (QWEN_SMALL, 1, 96, 96),
+    (S.PYTHIA_160M, 2, 200, 77),
+    (S.PYTHIA_70M, 1, 128, 64),
+]
+
+
+@pytest.mark.parametrize("shape,B,T,K", FOLD_CASES)
+def test_folded_norms(A, shape, B, T, K):
+    """adadsf_fold_norms folds the norm gains (and GPT-NeoX norm biases) into
+    the projections in place; the layer run with FLAG_FOLDED_NORMS on the
+    folded weights matches the oracle on the original weights, and the norm
+    parameters end at 1 / 0."""
+    W = H.host_layer(shape, 31)
+    x = S.round_to(S.hidden(31, B, T, shape.d), shape.dtype)
+    td = H.tdtype(shape)
+    wd = A.to_device(W, td)
+    A.adadsf_fold_norms(A.make_cfg(shape.replace(n_layers=1)), wd)
+    assert torch.equal(wd["ln1_w"].float().cpu(), torch.ones(shape.d))
+    if shape.arch == S.NEOX:
+        assert torch.equal(wd["ln2_b"].float().cpu(), torch.zeros(shape.d))
+    xd = H.to_dev(x, td)
+    idx = torch.full((B, K), -1, dtype=torch.int32, device="cuda")
+    sc = torch.empty((B, T), dtype=torch.float32, device="cuda")
+    cfg = A.make_cfg(shape.replace(n_layers=1), A.FLAG_FOLDED_NORMS)
+    ws = A.workspace(A.adadsf_layer_workspace_size(cfg, B, T, K))
+    A.adadsf_sparse_layer_forward(cfg, wd, xd, K, idx, sc, ws)
+    assert A.adadsf_sync_check(ws) == A.OK
+    gi = idx.cpu().numpy()
+    W64 = H.f64(W)
+    x64 = x.astype(np.float64)
+    if K < T:
+        H.check_kept_sets(sc.cpu().numpy(), gi, O.router_scores(x64, W64), K)
+    ref, _, _ = O.sparse_layer_forward(x64, W64, O.params_of(shape), K, idx=gi)
+    H.assert_close(H.to_np(xd), ref, H.tol(shape), "folded layer")
+
+
+def test_model_qwen_calibration_statistics(A):
+    """The bf16 dense pass takes its Eq. 4 partials from the down-projection
+    epilogue: per-layer similarities against the oracle's, and two passes
+    agree bit for bit."""
+    shape = QWEN_SMALL.replace(n_layers=3, vocab=1000)
+    B, T, L = 2, 300, 3
+    model = build_model(A, shape, 8)
+    ids = S.token_ids(12, B, T, shape.vocab)
+    accs = []
+    for _ in range(2):
+        acc = torch.zeros(2 * L, dtype=torch.float64, device="cuda")
+        out = torch.empty((B, T, shape.d), dtype=torch.bfloat16, device="cuda")
+        A.adadsf_sparse_model_forward(model, torch.from_numpy(ids).cuda(), [T] * L, out, stats_acc=acc)
+        accs.append(acc.cpu().numpy())
+    assert np.array_equal(accs[0], accs[1])
+    assert accs[0][1::2].tolist() == [B * T] * L
+    hostL = [H.f64(H.host_layer(shape, 8, l)) for l in range(L)]
+    _, _, st = O.sparse_model_forward(ids, H.f64(H.host_extra(shape, 8)), hostL, O.params_of(shape), [T] * L,
+                                      stats_mode="token")
+    s_ref = np.array([O.similarity(a) for a in st])
+    assert np.max(np.abs(A.adadsf_similarity(accs[0]) - s_ref)) < 5e-3
