@@ -174,18 +174,19 @@ def rank_seed(seed, rank):
     return seed + 7919 * rank
 
 
-def device_model(A, shape, seed, device):
+def device_model(A, shape, seed, device, fold=False):
     """Random-init weights of the backbone shape in the benchmark recipe,
-    drawn on the device (the reference arm draws the same tensors), with the
-    norm parameters folded into the projections (adadsf_fold_norms; exact
-    here, as the recipe's gains are 1 and biases 0) so that the layers run
-    with ADADSF_FLAG_FOLDED_NORMS."""
+    drawn on the device (the reference arm draws the same tensors). With
+    fold, the norm parameters are folded into the projections
+    (adadsf_fold_norms; exact here, as the recipe's gains are 1 and biases 0)
+    and the layers run with ADADSF_FLAG_FOLDED_NORMS."""
     td = torch.bfloat16 if shape.dtype == "bf16" else torch.float32
-    cfg = A.make_cfg(shape, A.FLAG_FOLDED_NORMS)
+    cfg = A.make_cfg(shape, A.FLAG_FOLDED_NORMS if fold else 0)
     layers = []
     for l in range(shape.n_layers):
         w = {k: v.to(td) for k, v in S.bench_layer_weights(shape, seed, l, device).items()}
-        A.adadsf_fold_norms(cfg, w)
+        if fold:
+            A.adadsf_fold_norms(cfg, w)
         layers.append(w)
     extra = {"embed": S.bench_embed(shape, seed, device).to(td),
              "final_w": torch.ones(shape.d, device=device, dtype=td)}
@@ -222,7 +223,7 @@ def run_ours(args, rank, world, local_rank):
     L = shape.n_layers
     t_target = retention_of(args, wl)
     stream = torch.cuda.Stream(device)
-    model = device_model(A, shape, WEIGHT_SEED, device)
+    model = device_model(A, shape, WEIGHT_SEED, device, fold=args.folded_norms)
     sampler = ClockSampler(gpu_id_for_smi(local_rank))
     n_rec = 4 + 12 * L
 
@@ -733,6 +734,8 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=20.0)
     ap.add_argument("--spin-up", type=float, default=1.5, help="seconds of untimed GPU work before measuring")
     ap.add_argument("--decode-steps", type=int, default=32, help="decode steps timed after a prefill (0: none)")
+    ap.add_argument("--folded-norms", action="store_true",
+                    help="fold the norms into the projections (ADADSF_FLAG_FOLDED_NORMS)")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
 

@@ -286,13 +286,17 @@ __device__ __forceinline__ void store_chunk_rows(uint32_t stg, int lane, const u
 
 // Store one 32-column chunk of output row orow (adding the residual `res`
 // if RES and the problem has one); rows with !valid store nothing. Whole warp.
-template <bool RES>
+// EXTRA: the instance for the rarer epilogue features (score gate, chunk
+// statistics for the next norm or Eq. 4); without it the plain residual path
+// compiles as lean as possible.
+template <bool RES, bool EXTRA>
 __device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, const uint4* res,
-                                                float g, const uint4* gb, int64_t orow, int n0,
-                                                bool valid, uint32_t stg, int lane, int64_t m,
-                                                const uint4* xin) {
+                                                int64_t arow, int64_t orow, int n0, bool valid,
+                                                uint32_t stg, int lane, int64_t m) {
   if (RES && p.add) {
-    if (!p.gate) {
+    // the score gate of this row (gated variant)
+    const float g = (EXTRA && p.gate && valid) ? 1.f / (1.f + expf(-p.gate[arow])) : 1.f;
+    if (!EXTRA || !p.gate) {
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         float f[8];
@@ -315,32 +319,34 @@ __device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, cons
       }
     } else {
       // gated, residual = h (packed), base = x: out = x + g (v + h - x)
+      const uint4* gsrc = reinterpret_cast<const uint4*>(p.gbase + arow * p.ld_gbase + n0);
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
         float f[8], b[8];
         unpack16(res[i], f, bf16());
-        unpack16(gb[i], b, bf16());
+        unpack16(valid ? gsrc[i] : make_uint4(0, 0, 0, 0), b, bf16());
 #pragma unroll
         for (int j = 0; j < 8; ++j) v[8 * i + j] = fmaf(g, (v[8 * i + j] + f[j]) - b[j], b[j]);
       }
     }
   }
-  uint4 pk[4];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) pk[i] = pack16(v + 8 * i, bf16());
-  if (RES && valid && (p.sq_out || p.cos_out)) {
-    // statistics of the stored (rounded) chunk for the next norm / Eq. 4
+  if (EXTRA && RES && valid && (p.sq_out || p.cos_out)) {
+    // statistics of the chunk for the next norm / Eq. 4, from the fp32
+    // values about to be stored (their bf16 rounding moves a sum of 32
+    // squares by ~2^-9 relative at most)
     float sq = 0.f, dot = 0.f, nx = 0.f;
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      float o[8], a[8];
-      unpack16(pk[i], o, bf16());
-      if (p.cos_out) unpack16(xin[i], a, bf16());
+    for (int j = 0; j < 32; ++j) sq = fmaf(v[j], v[j], sq);
+    if (p.cos_out) {
+      // the layer input of this chunk: cos_in rows, else the residual
+      const uint4* csrc = reinterpret_cast<const uint4*>(p.cin + arow * p.ld_cin + n0);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        sq = fmaf(o[j], o[j], sq);
-        if (p.cos_out) {
-          dot = fmaf(a[j], o[j], dot);
+      for (int i = 0; i < 4; ++i) {
+        float a[8];
+        unpack16(p.cin ? csrc[i] : res[i], a, bf16());
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          dot = fmaf(a[j], v[8 * i + j], dot);
           nx = fmaf(a[j], a[j], nx);
         }
       }
@@ -348,6 +354,9 @@ __device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, cons
     if (p.sq_out) p.sq_out[m * p.sq_ld + (n0 >> 5)] = sq;
     if (p.cos_out) p.cos_out[m * p.cos_ld + (n0 >> 5)] = make_float4(dot, nx, sq, 0.f);
   }
+  uint4 pk[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) pk[i] = pack16(v + 8 * i, bf16());
   store_chunk_rows(stg, lane, pk, valid ? p.out + orow * p.ld_out + n0 : nullptr);
 }
 
@@ -455,7 +464,36 @@ struct EpiPre {
   uint4 res[2][4];   // residual of the first two chunks this warp finalises
   int n;             // how many of them are valid
   bool nt;           // res holds rotary pairs instead
+  float rs;          // folded RMSNorm: the row's 1 / rms (1 without)
 };
+
+// The folded RMSNorm's scale of A row m from its chunk sums of squares
+// (vector loads when the row of sums is 16-byte aligned); before the
+// accumulator is ready.
+__device__ __forceinline__ float norm_scale(const GemmDev& p, int m) {
+  if (!p.nrm_psum || m >= p.M) return 1.f;
+  const float* ps = p.nrm_psum + (int64_t)m * p.nrm_nps;
+  float sum = 0.f;
+  if ((p.nrm_nps & 3) == 0) {
+    const float4* p4 = reinterpret_cast<const float4*>(ps);
+    const int n4 = p.nrm_nps >> 2;
+    float s0 = 0.f, s1 = 0.f;
+    int i = 0;
+    for (; i + 1 < n4; i += 2) {   // two vector loads in flight per step
+      const float4 f = p4[i], h = p4[i + 1];
+      s0 += (f.x + f.y) + (f.z + f.w);
+      s1 += (h.x + h.y) + (h.z + h.w);
+    }
+    if (i < n4) {
+      const float4 f = p4[i];
+      s0 += (f.x + f.y) + (f.z + f.w);
+    }
+    sum = s0 + s1;
+  } else {
+    for (int i = 0; i < p.nrm_nps; ++i) sum += ps[i];
+  }
+  return 1.f / sqrtf(sum * p.nrm_inv_d + p.nrm_eps);
+}
 
 // Epilogue of one accumulator tile for the calling thread's row m over the
 // chunks [c_lo, c_hi) of 32 TMEM columns -> constants / activation / rotary /
@@ -463,7 +501,7 @@ struct EpiPre {
 // per-column constants (has_consts), `pre` the prefetched residual chunks,
 // `red` the split-K partial to add first. ROPE: the instance for rotary
 // tiles (query / key / value projections, which have no residual).
-template <int BN, bool DUAL, bool ROPE>
+template <int BN, bool DUAL, bool ROPE, bool EXTRA>
 __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, int m, int nb, int bn,
                                               int c_lo, int c_hi, uint32_t sc, bool has_consts,
                                               const EpiPre& pre, const EpiRed& red, uint32_t stg,
@@ -476,17 +514,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
     if (arow < 0) mvalid = false;   // a row that bypasses the layer: nothing read or written
   }
   const int64_t orow = p.out_mapped ? arow : (int64_t)m;
-  float gate = 1.f;
-  if (!ROPE && p.gate && mvalid) gate = 1.f / (1.f + expf(-p.gate[arow]));
-  // folded RMSNorm of this A row: its rstd from the chunk sums of squares
-  float rs = 1.f;
-  if (p.nrm_psum && mvalid) {
-    const float* ps = p.nrm_psum + (int64_t)m * p.nrm_nps;
-    float sum = 0.f;
-#pragma unroll 4
-    for (int i = 0; i < p.nrm_nps; ++i) sum += ps[i];
-    rs = 1.f / sqrtf(sum * p.nrm_inv_d + p.nrm_eps);
-  }
+  const float rs = pre.rs;   // folded RMSNorm of this A row (1 without)
   const float2* tab_row = nullptr;
   if (rope && mvalid)
     tab_row = p.rope_tab + (int64_t)(p.rope_pos ? p.rope_pos[m] : m % p.rope_T) * p.rope_half;
@@ -524,7 +552,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
         v[4 * j + 3] += f.w;
       }
     }
-    if (p.nrm_psum) {
+    if (EXTRA && p.nrm_psum) {
 #pragma unroll
       for (int j = 0; j < 32; ++j) v[j] *= rs;
     }
@@ -540,7 +568,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
     }
     if (DUAL) {
 #pragma unroll
-      for (int j = 0; j < 32; ++j) v[j] = silu_f(v[j]) * (rs * __uint_as_float(r2[j]));
+      for (int j = 0; j < 32; ++j) v[j] = silu_f(v[j]) * ((EXTRA ? rs : 1.f) * __uint_as_float(r2[j]));
     } else if (p.act == ACT_GELU) {
 #pragma unroll
       for (int j = 0; j < 32; j += 2) {
@@ -570,21 +598,7 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
         default: break;
       }
     }
-    uint4 gb[4] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0),
-                   make_uint4(0, 0, 0, 0)};
-    if (!ROPE && p.gbase && mvalid) {
-      const uint4* src = reinterpret_cast<const uint4*>(p.gbase + arow * p.ld_gbase + n0);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) gb[i] = src[i];
-    }
-    // the layer input of this chunk for the Eq. 4 partials
-    uint4 xi[4] = {res[0], res[1], res[2], res[3]};
-    if (!ROPE && p.cin && mvalid) {
-      const uint4* src = reinterpret_cast<const uint4*>(p.cin + arow * p.ld_cin + n0);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) xi[i] = src[i];
-    }
-    epi_chunk_store<!ROPE>(p, v, res, gate, gb, orow, n0, mvalid, stg, lane, m, xi);
+    epi_chunk_store<!ROPE, EXTRA>(p, v, res, arow, orow, n0, mvalid, stg, lane, m);
   }
 }
 
@@ -609,7 +623,7 @@ __device__ __forceinline__ void prefetch_res(const GemmDev& p, int m, int nb, in
 // The epilogue warps' part of a tile once its coordinates are known: stage
 // constants, prefetch residuals, wait for the accumulator (bounded), run the
 // epilogue. Returns false if the wait gave up.
-template <int BN, bool DUAL>
+template <int BN, bool DUAL, bool EXTRA>
 __device__ __forceinline__ bool epilogue_role(const GemmDev& P, int m, int nb, int half,
                                               uint32_t tacc, uint32_t sc, uint32_t tfull,
                                               uint32_t parity, volatile int* abort_flag,
@@ -623,6 +637,7 @@ __device__ __forceinline__ bool epilogue_role(const GemmDev& P, int m, int nb, i
   EpiPre pre;
   pre.n = 0;
   pre.nt = false;
+  pre.rs = (EXTRA && P.nrm_psum) ? norm_scale(P, m) : 1.f;
   if (!P.rope_tab) {
     prefetch_res(P, m, nb, bn, c_lo, c_hi, pre);
   } else if (!DUAL && P.rope_half >= 32 && m < P.M) {
@@ -644,13 +659,13 @@ __device__ __forceinline__ bool epilogue_role(const GemmDev& P, int m, int nb, i
   tc_fence_after();
   const EpiRed none = {nullptr, 0, 0, 0};
   if (!DUAL && P.rope_tab)
-    epilogue_tile<BN, DUAL, true>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none, stg, lane);
+    epilogue_tile<BN, DUAL, true, false>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none, stg, lane);
   else
-    epilogue_tile<BN, DUAL, false>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none, stg, lane);
+    epilogue_tile<BN, DUAL, false, EXTRA>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none, stg, lane);
   return true;
 }
 
-template <int BN, bool DUAL>
+template <int BN, bool DUAL, bool EXTRA>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmB2,
@@ -825,7 +840,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int acc = it & 1;
       const uint32_t sc = sconst + 4u * kConstFloats * ((warp - 2) * 2 + acc);
       const uint32_t tacc = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C::ACC_COLS;
-      if (!epilogue_role<BN, DUAL>(P, ti.mb * BM + row_in_tile, ti.nb, half, tacc, sc,
+      if (!epilogue_role<BN, DUAL, EXTRA>(P, ti.mb * BM + row_in_tile, ti.nb, half, tacc, sc,
                                            tfull0 + 8 * acc, (it >> 1) & 1, abort_flag, lane,
                                            sconst + C::CONST_BYTES + kStgBytes * (warp - 2)))
         break;
@@ -855,7 +870,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // orders the writes before the reads, and each CTA adds the other CTAs'
 // slots in rank order (a fixed order: the sum does not depend on timing) to
 // its own columns before the usual epilogue.
-template <int BN>
+template <int BN, bool EXTRA>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_tc_sk_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmB2,
@@ -927,6 +942,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const bool has_consts = p.bias || p.bias2;
   EpiPre pre;
   pre.n = 0;
+  pre.nt = false;
+  pre.rs = 1.f;
   int ok = 0;
 
   if (warp == 0) {
@@ -1015,7 +1032,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                                __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3])));
         }
       }
-      if (h_lo < h_hi) prefetch_res(p, m, ti.nb, BN, c_lo, c_hi, pre);
+      if (h_lo < h_hi) {
+        prefetch_res(p, m, ti.nb, BN, c_lo, c_hi, pre);
+        if (EXTRA && p.nrm_psum) pre.rs = norm_scale(p, m);
+      }
     }
   }
 
@@ -1027,12 +1047,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp >= 2 && ok && h_lo < h_hi) {
     // ------------------------------------------------------------ epilogue, part 2
     const EpiRed red = {p.scratch + (size_t)tile * S * BM * BN, S, rank, BN};
+    const uint32_t stg = sconst + C::CONST_BYTES + kStgBytes * (warp - 2);
     if (p.rope_tab)   // rotary halves of at most 16 features (one chunk)
-      epilogue_tile<BN, false, true>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre, red,
-                                     sconst + C::CONST_BYTES + kStgBytes * (warp - 2), lane);
+      epilogue_tile<BN, false, true, false>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre, red, stg,
+                                            lane);
     else
-      epilogue_tile<BN, false, false>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre,
-                                      red, sconst + C::CONST_BYTES + kStgBytes * (warp - 2), lane);
+      epilogue_tile<BN, false, false, EXTRA>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre, red, stg,
+                                             lane);
   }
 
   __syncwarp();
@@ -1054,7 +1075,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // of both CTAs; both CTAs' epilogue warps release the accumulator on the even
 // CTA's empty-accumulator barrier. Two K sources and grouped problems work
 // as in the one-CTA kernel (not with DUAL).
-template <int BN, bool DUAL>
+template <int BN, bool DUAL, bool EXTRA>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __grid_constant__ CUtensorMap tmA2, const __grid_constant__ CUtensorMap tmB2,
@@ -1232,7 +1253,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int acc = it & 1;
       const uint32_t sc = sconst + 4u * kConstFloats * ((warp - 2) * 2 + acc);
       const uint32_t tacc = tmem_base + ((uint32_t)(quarter * 32) << 16) + acc * C::ACC_COLS;
-      if (!epilogue_role<BN, DUAL>(P, ti.mb * 2 * BM + (int)rank * BM + row_in_tile, ti.nb,
+      if (!epilogue_role<BN, DUAL, EXTRA>(P, ti.mb * 2 * BM + (int)rank * BM + row_in_tile, ti.nb,
                                           half, tacc, sc, tfull0 + 8 * acc, (it >> 1) & 1,
                                           abort_flag, lane, sconst + C::CONST_BYTES + kStgBytes * (warp - 2)))
         break;
@@ -1407,14 +1428,19 @@ cudaError_t prepare(const GemmArgs& a, const GemmArgs* b, uint32_t a_rows, int b
   return cudaSuccess;
 }
 
-template <int BN, bool DUAL>
-cudaError_t launch(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
+// Whether a launch needs the epilogue instance with the rarer features.
+bool extra_args(const GemmArgs& a) {
+  return a.epi.gate_scores || a.epi.sq_out || a.epi.cos_out || a.epi.nrm_psum;
+}
+
+template <int BN, bool DUAL, bool EXTRA>
+cudaError_t launch_x(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
   using C = TileCfg<BN, DUAL>;
   static int attr_done[64] = {0};
   int device = 0;
   cudaGetDevice(&device);
   if (device < 64 && !attr_done[device]) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, DUAL>,
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, DUAL, EXTRA>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
     if (e != cudaSuccess) return e;
     attr_done[device] = 1;
@@ -1426,18 +1452,24 @@ cudaError_t launch(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
   int64_t num_tiles = ((a.M + BM - 1) / BM) * ((a.N + p.bn - 1) / p.bn);
   if (b) num_tiles += ((b->M + BM - 1) / BM) * ((b->N + p2.bn - 1) / p2.bn);
   const int grid = (int)(num_tiles < dev.num_sms ? num_tiles : dev.num_sms);
-  return launch_pdl(gemm_tc_kernel<BN, DUAL>, dim3(grid), dim3(kThreads), C::SMEM_BYTES,
+  return launch_pdl(gemm_tc_kernel<BN, DUAL, EXTRA>, dim3(grid), dim3(kThreads), C::SMEM_BYTES,
                     dev.stream, tm[0], tm[1], tm[2], tm[3], p, p2);
 }
 
 template <int BN, bool DUAL>
-cudaError_t launch_pair(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
+cudaError_t launch(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
+  return (extra_args(a) || (b && extra_args(*b))) ? launch_x<BN, DUAL, true>(a, b, dev)
+                                                  : launch_x<BN, DUAL, false>(a, b, dev);
+}
+
+template <int BN, bool DUAL, bool EXTRA>
+cudaError_t launch_pair_x(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
   using C = TileCfg<BN, DUAL, true>;
   static int attr_done[64] = {0};
   int device = 0;
   cudaGetDevice(&device);
   if (device < 64 && !attr_done[device]) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc2_kernel<BN, DUAL>,
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc2_kernel<BN, DUAL, EXTRA>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM_BYTES);
     if (e != cudaSuccess) return e;
     attr_done[device] = 1;
@@ -1451,7 +1483,7 @@ cudaError_t launch_pair(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = C::SMEM_BYTES;
     int n = 0;
-    cudaError_t e = cudaOccupancyMaxActiveClusters(&n, gemm_tc2_kernel<BN, DUAL>, &cfg);
+    cudaError_t e = cudaOccupancyMaxActiveClusters(&n, gemm_tc2_kernel<BN, DUAL, EXTRA>, &cfg);
     if (e != cudaSuccess || n <= 0) return e != cudaSuccess ? e : cudaErrorInvalidConfiguration;
     max_pairs[device] = n;
   }
@@ -1470,8 +1502,14 @@ cudaError_t launch_pair(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
   int64_t num_tiles = ((a.M + 2 * BM - 1) / (2 * BM)) * ((a.N + BN - 1) / BN);
   if (b) num_tiles += ((b->M + 2 * BM - 1) / (2 * BM)) * ((b->N + BN - 1) / BN);
   const int64_t pairs = num_tiles < cap ? num_tiles : cap;
-  return launch_pdl(gemm_tc2_kernel<BN, DUAL>, dim3((unsigned)(2 * pairs)), dim3(kThreads),
+  return launch_pdl(gemm_tc2_kernel<BN, DUAL, EXTRA>, dim3((unsigned)(2 * pairs)), dim3(kThreads),
                     C::SMEM_BYTES, dev.stream, tm[0], tm[1], tm[2], tm[3], p, p2);
+}
+
+template <int BN, bool DUAL>
+cudaError_t launch_pair(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
+  return (extra_args(a) || (b && extra_args(*b))) ? launch_pair_x<BN, DUAL, true>(a, b, dev)
+                                                  : launch_pair_x<BN, DUAL, false>(a, b, dev);
 }
 
 // Clusters of S CTAs of the split-K kernel that can be resident at once
@@ -1485,7 +1523,9 @@ int sk_max_clusters(int S, const Dev& dev) {
   cudaGetDevice(&device);
   if (device >= 64 || S < 2 || S > 4) return 0;
   if (!attr_done[device]) {
-    if (cudaFuncSetAttribute(gemm_tc_sk_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(gemm_tc_sk_kernel<BN, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             C::SMEM_BYTES) != cudaSuccess ||
+        cudaFuncSetAttribute(gemm_tc_sk_kernel<BN, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              C::SMEM_BYTES) != cudaSuccess)
       return 0;
     attr_done[device] = 1;
@@ -1503,7 +1543,7 @@ int sk_max_clusters(int S, const Dev& dev) {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_sk_kernel<BN>, &cfg) != cudaSuccess) n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc_sk_kernel<BN, false>, &cfg) != cudaSuccess) n = 0;
     cache[device][S] = n > 0 ? n : -1;
   }
   return cache[device][S] > 0 ? cache[device][S] : 0;
@@ -1532,7 +1572,10 @@ cudaError_t launch_sk(const GemmArgs& a, const Dev& dev, int S) {
   cudaError_t e = prepare<false>(a_full, nullptr, BM, BN, BN, dev, tm, p, p2);
   if (e != cudaSuccess) return e;
   const int64_t num_tiles = ((a.M + BM - 1) / BM) * ((a.N + BN - 1) / BN);
-  return launch_pdl_cluster(gemm_tc_sk_kernel<BN>, dim3((unsigned)(num_tiles * S)), dim3(kThreads),
+  if (extra_args(a))
+    return launch_pdl_cluster(gemm_tc_sk_kernel<BN, true>, dim3((unsigned)(num_tiles * S)), dim3(kThreads),
+                              C::SMEM_BYTES, dev.stream, S, tm[0], tm[1], tm[2], tm[3], p);
+  return launch_pdl_cluster(gemm_tc_sk_kernel<BN, false>, dim3((unsigned)(num_tiles * S)), dim3(kThreads),
                             C::SMEM_BYTES, dev.stream, S, tm[0], tm[1], tm[2], tm[3], p);
 }
 

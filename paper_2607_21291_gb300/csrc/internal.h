@@ -61,11 +61,12 @@ struct Epilogue {
   const float* nrm_psum = nullptr;
   int nrm_nps = 0, nrm_d = 0;
   float nrm_eps = 0.f;
-  // Sum of squares of each stored 32-column chunk (of the bf16 values):
-  // sq_out[m * sq_ld + n / 32] (bf16 path; the next RMSNorm's statistics).
+  // Sum of squares of each stored 32-column chunk (of the fp32 values before
+  // their bf16 rounding): sq_out[m * sq_ld + n / 32] (bf16 path; the next
+  // RMSNorm's statistics).
   float* sq_out = nullptr;
   int sq_ld = 0;
-  // Eq. 4 partials of each stored 32-column chunk (bf16 path), as float4
+  // Eq. 4 partials of each stored 32-column chunk (bf16 path; fp32 values), as float4
   // {x_in . out, |x_in|^2, |out|^2, 0} at cos_out[m * cos_ld + n / 32]; x_in
   // = cos_in[row(m)] when given, else the gathered residual add_rows.
   float4* cos_out = nullptr;

@@ -96,7 +96,10 @@ def case_layer(a, stream):
     for n in ("ln1_w", "ln2_w"):
         w[n] = torch.ones_like(w[n])
     x = torch.randn(B, T, shape.d, generator=g, device="cuda").to(dt)
-    cfg = A.make_cfg(shape)
+    flags = (A.FLAG_FOLDED_NORMS if a.fold else 0) | (A.FLAG_GATE_SIGMOID if a.gate else 0)
+    cfg = A.make_cfg(shape, flags)
+    if a.fold:
+        A.adadsf_fold_norms(cfg, w, stream)
     ws = A.workspace(A.adadsf_layer_workspace_size(cfg, B, T, K))
     fn = lambda: A.adadsf_sparse_layer_forward(cfg, w, x, K, ws=ws, stream=stream)
     per_tok = 2.0 * (shape.qkv_dim * shape.d + shape.d * shape.q_dim
@@ -173,6 +176,8 @@ def main():
     ap.add_argument("--iters", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--profile", action="store_true", help="also report the library's per-launch events")
+    ap.add_argument("--fold", action="store_true", help="layer: fold the norms (FLAG_FOLDED_NORMS)")
+    ap.add_argument("--gate", action="store_true", help="layer: the score-gated variant")
     ap.add_argument("--graph", type=int, default=0, help="also time R calls replayed from one CUDA graph")
     a = ap.parse_args()
     if a.case == "linear" and a.K is None:
