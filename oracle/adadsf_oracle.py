@@ -445,3 +445,79 @@ def decode_step(ids_new, Wm, layers, p, st, kept_force=None):
         x = x_next
     st["T"] = t + 1
     return final_norm(x, Wm, p), kept, scores
+
+
+# --------------------------------------------------------------------------
+# Sec. 3.5, Eqs. 9-11 -- feature-preserving alignment objective, and the
+# router's gradient through the score gate (Sec. 3.4: the score pathway is
+# kept differentiable)
+# --------------------------------------------------------------------------
+def softmax(z, axis=-1):
+    """exp(z - max) / sum exp(z - max) along `axis`."""
+    z = np.asarray(z, dtype=np.float64)
+    e = np.exp(z - z.max(axis=axis, keepdims=True))
+    return e / e.sum(axis=axis, keepdims=True)
+
+
+def hidden_alignment(h_sparse, h_dense):
+    """Eq. 9 for one layer, per token: || softmax(h_sparse) - softmax(h_dense) ||_2
+    with the softmax over the hidden features of the token. Returns the
+    per-token values (shape of the inputs without the last axis); the layer's
+    loss is their mean."""
+    return np.sqrt(((softmax(h_sparse) - softmax(h_dense)) ** 2).sum(axis=-1))
+
+
+def hidden_alignment_grad(h_sparse, h_dense):
+    """Gradient of each token's Eq. 9 value with respect to its h_sparse row
+    (by the chain rule through the norm and the softmax): with p =
+    softmax(h_sparse), q = softmax(h_dense), r = p - q, n = |r|,
+    d n / d h = p * (r / n - p . r / n); zero where n = 0."""
+    p = softmax(h_sparse)
+    r = p - softmax(h_dense)
+    n = np.sqrt((r * r).sum(axis=-1, keepdims=True))
+    safe = np.where(n > 0, n, 1.0)
+    u = r / safe
+    g = p * (u - (p * u).sum(axis=-1, keepdims=True))
+    return np.where(n > 0, g, 0.0)
+
+
+def output_alignment(h_sparse, h_dense, w_head):
+    """Eq. 10 per token: KL(P_dense || P_sparse) = sum_c P_dense(c) log(P_dense(c)
+    / P_sparse(c)), P = softmax of the logits h W_head^T over the classes.
+    Returns the per-token values; the loss is their mean."""
+    ls = np.asarray(h_sparse, dtype=np.float64) @ np.asarray(w_head, dtype=np.float64).T
+    ld = np.asarray(h_dense, dtype=np.float64) @ np.asarray(w_head, dtype=np.float64).T
+    lps = ls - ls.max(axis=-1, keepdims=True)
+    lps = lps - np.log(np.exp(lps).sum(axis=-1, keepdims=True))
+    lpd = ld - ld.max(axis=-1, keepdims=True)
+    lpd = lpd - np.log(np.exp(lpd).sum(axis=-1, keepdims=True))
+    return (np.exp(lpd) * (lpd - lps)).sum(axis=-1)
+
+
+def alignment_objective(l_align, l_hid_layers):
+    """Eq. 11: L = L_align + (1/L) sum_l L_hid^(l), from the per-token means."""
+    return float(l_align) + float(np.mean(l_hid_layers))
+
+
+def router_grad(x, W, rows, delta, grad_y):
+    """Gradient of a loss with respect to the router parameters of one gated
+    layer (kept rows y = x + sigmoid(s) delta, Sec. 3.4), given the loss's
+    gradient grad_y at the kept rows' outputs and the layer's ungated delta
+    there; x and the layer's other weights are held fixed, and the Top-K
+    choice itself carries no gradient. rows: the kept rows of x (n, d) as a
+    flat index; delta, grad_y: (n_kept, d). Chain rule:
+      ds = sigmoid'(s) (grad_y . delta),  s = w2 . SiLU(u) + b2,  u = W1 x + b1
+      dw2 = sum ds SiLU(u), db2 = sum ds, du = ds w2 SiLU'(u),
+      dW1 = sum du (x) x, db1 = sum du.
+    Returns a dict with router_w1, router_b1, router_w2, router_b2."""
+    xs = np.asarray(x, dtype=np.float64).reshape(-1, np.shape(x)[-1])[np.asarray(rows)]
+    u = xs @ W["router_w1"].T + W["router_b1"]
+    sg = 1.0 / (1.0 + np.exp(-u))
+    su = u * sg
+    s = su @ W["router_w2"] + W["router_b2"][0]
+    sig = sigmoid(s)
+    ds = sig * (1.0 - sig) * (np.asarray(grad_y, dtype=np.float64) * np.asarray(delta, dtype=np.float64)).sum(-1)
+    dsilu = sg * (1.0 + u * (1.0 - sg))
+    du = ds[:, None] * W["router_w2"][None, :] * dsilu
+    return {"router_w1": du.T @ xs, "router_b1": du.sum(0), "router_w2": (ds[:, None] * su).sum(0),
+            "router_b2": np.array([ds.sum()])}

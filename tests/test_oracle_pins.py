@@ -676,3 +676,99 @@ class TestDecode:
         assert O.decode_keep(0.71, 0.7) and not O.decode_keep(0.7, 0.7)
         assert not O.decode_keep(float("nan"), 0.7) and not O.decode_keep(float("nan"), -np.inf)
         assert O.kept_threshold(sc, []) == np.inf              # nothing kept: nothing will be
+
+
+# ---------------------------------------------------------------- Sec. 3.5, Eqs. 9-11; router gradient
+class TestAlignment:
+    def test_softmax_matches_scipy(self):
+        from scipy.special import softmax as sp_softmax
+        z = rng(80).normal(size=(5, 9)) * 4
+        assert O.softmax(z) == pytest.approx(sp_softmax(z, axis=-1), rel=1e-14)
+
+    def test_hidden_alignment_hand_value_and_limits(self):
+        """h_s = (0, 0) -> p = (1/2, 1/2); h_d = (ln 3, 0) -> q = (3/4, 1/4);
+        |p - q| = sqrt(2) / 4. Identical rows give 0; adding a constant to a
+        row changes nothing (the softmax is shift invariant)."""
+        hs = np.array([[0.0, 0.0]])
+        hd = np.array([[math.log(3.0), 0.0]])
+        assert O.hidden_alignment(hs, hd)[0] == pytest.approx(math.sqrt(2) / 4, rel=1e-15)
+        x = rng(81).normal(size=(4, 16))
+        assert O.hidden_alignment(x, x) == pytest.approx(np.zeros(4), abs=1e-15)
+        y = rng(82).normal(size=(4, 16))
+        assert O.hidden_alignment(x + 3.0, y - 1.5) == pytest.approx(O.hidden_alignment(x, y), rel=1e-12)
+
+    def test_hidden_alignment_grad_matches_finite_differences_and_autograd(self):
+        hs = rng(83).normal(size=(3, 7))
+        hd = rng(84).normal(size=(3, 7))
+        g = O.hidden_alignment_grad(hs, hd)
+        eps = 1e-6
+        fd = np.zeros_like(hs)
+        for i in range(hs.shape[0]):
+            for j in range(hs.shape[1]):
+                a, b = hs.copy(), hs.copy()
+                a[i, j] += eps
+                b[i, j] -= eps
+                fd[i, j] = (O.hidden_alignment(a, hd)[i] - O.hidden_alignment(b, hd)[i]) / (2 * eps)
+        assert g == pytest.approx(fd, rel=1e-6, abs=1e-9)
+        t = torch.tensor(hs, requires_grad=True)
+        loss = torch.linalg.vector_norm(torch.softmax(t, -1) - torch.softmax(torch.tensor(hd), -1), dim=-1).sum()
+        loss.backward()
+        assert g == pytest.approx(t.grad.numpy(), rel=1e-12, abs=1e-15)
+
+    def test_output_alignment(self):
+        """W_head = I: logits are the hidden rows. P_s = (1/2, 1/2), P_d = (3/4, 1/4):
+        KL = 3/4 ln(3/2) + 1/4 ln(1/2) = 0.13081203594113694. KL(P || P) = 0,
+        KL >= 0, and agreement with scipy.special.rel_entr."""
+        from scipy.special import rel_entr, softmax as sp_softmax
+        kl = O.output_alignment(np.array([[0.0, 0.0]]), np.array([[math.log(3.0), 0.0]]), np.eye(2))
+        assert kl[0] == pytest.approx(0.75 * math.log(1.5) + 0.25 * math.log(0.5), rel=1e-14)
+        assert kl[0] == pytest.approx(0.13081203594113694, rel=1e-14)
+        g = rng(85)
+        W = g.normal(size=(30, 8))
+        hs, hd = g.normal(size=(6, 8)), g.normal(size=(6, 8))
+        assert O.output_alignment(hs, hs, W) == pytest.approx(np.zeros(6), abs=1e-14)
+        got = O.output_alignment(hs, hd, W)
+        ref = rel_entr(sp_softmax(hd @ W.T, axis=-1), sp_softmax(hs @ W.T, axis=-1)).sum(-1)
+        assert got == pytest.approx(ref, rel=1e-12) and (got >= 0).all()
+
+    def test_objective(self):
+        assert O.alignment_objective(0.1, [0.2, 0.4]) == pytest.approx(0.4, rel=1e-15)
+
+    @pytest.mark.parametrize("arch", [O.NEOX, O.QWEN])
+    def test_router_grad_through_the_gated_layer(self, arch):
+        """L(theta) = sum over kept rows of grad_y . y, y the gated layer's
+        output with the kept set held fixed: its finite-difference gradient in
+        every router parameter equals router_grad (delta = the ungated layer's
+        delta); and torch autograd of the same expression agrees."""
+        p = dict(_params(arch, Hkv=2 if arch == O.QWEN else 4), gate="sigmoid")
+        W = _weights(p, 86)
+        x = rng(87).normal(size=(2, 9, 32))
+        idx = np.array([[0, 3, 4, 8], [1, 2, 6, 7]])
+        rows = (np.arange(2)[:, None] * 9 + idx).ravel()
+        G = rng(88).normal(size=(8, 32))
+        plain, _, _ = O.sparse_layer_forward(x, W, dict(p, gate="none"), 4, idx=idx)
+        delta = (plain - x).reshape(-1, 32)[rows]
+        got = O.router_grad(x, W, rows, delta, G)
+
+        def loss(Wr):
+            y, _, _ = O.sparse_layer_forward(x, Wr, p, 4, idx=idx)
+            return float((G * y.reshape(-1, 32)[rows]).sum())
+
+        eps = 1e-6
+        for name in ("router_w1", "router_b1", "router_w2", "router_b2"):
+            fd = np.zeros_like(W[name])
+            flat = fd.reshape(-1)
+            for k in range(flat.size):
+                a = {kk: vv.copy() for kk, vv in W.items()}
+                b = {kk: vv.copy() for kk, vv in W.items()}
+                a[name].reshape(-1)[k] += eps
+                b[name].reshape(-1)[k] -= eps
+                flat[k] = (loss(a) - loss(b)) / (2 * eps)
+            assert got[name] == pytest.approx(fd, rel=1e-5, abs=1e-8), name
+        # autograd of sum G . (x + sigmoid(s) delta) over the router parameters
+        tw = {k: torch.tensor(W[k], requires_grad=True) for k in ("router_w1", "router_b1", "router_w2", "router_b2")}
+        xs = torch.tensor(x.reshape(-1, 32)[rows])
+        s = torch.nn.functional.silu(xs @ tw["router_w1"].T + tw["router_b1"]) @ tw["router_w2"] + tw["router_b2"][0]
+        (torch.tensor(G) * (xs + torch.sigmoid(s)[:, None] * torch.tensor(delta))).sum().backward()
+        for k, t in tw.items():
+            assert got[k] == pytest.approx(t.grad.numpy(), rel=1e-12, abs=1e-14), k
