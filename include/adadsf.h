@@ -220,6 +220,52 @@ adadsf_status adadsf_alloc_ratios(const double *s_host, int L, double t, double 
 adadsf_status adadsf_fold_norms(const adadsf_model_cfg *cfg, const adadsf_layer_weights *w, void *stream);
 
 /* ------------------------------------------------------------------------
+ * Sec. 3.5: the feature-preserving alignment objective, on device.
+ * Eq. 9 (adadsf_align_hidden), per row r of n_rows rows of d features
+ * (dtype): n_r = || softmax(hs_r) - softmax(hd_r) ||_2, the softmax over the
+ * row's features; acc_dev[0] += sum_r n_r, acc_dev[1] += n_rows (a layer's
+ * L_hid is their ratio). grad_dev (NULL or fp32 [n_rows, d]) receives
+ * d n_r / d hs_r = p (r / n - p . r / n), p = softmax(hs_r), r = p -
+ * softmax(hd_r) (zero where n = 0); divide by the row count for the mean's
+ * gradient.
+ * Eq. 10 (adadsf_align_output): KL(P_dense || P_sparse) per row, P the
+ * softmax over n_classes of the logits h W_head^T (w_head_dev [n_classes, d],
+ * e.g. the tied embedding); acc_dev[0] += sum of the rows' KL, acc_dev[1] +=
+ * n_rows. Logits are fp32 (workspace: adadsf_align_workspace_size(n_rows,
+ * n_classes), 8 n_rows n_classes bytes of them: call on row chunks for large
+ * vocabularies). bf16 needs d and n_classes multiples of 64.
+ * Eq. 11 is L_align + (1/L) sum_l L_hid^(l) of those accumulators.
+ * Sums run in a fixed order (bit-reproducible).
+ * ---------------------------------------------------------------------- */
+size_t adadsf_align_workspace_size(int64_t n_rows, int n_classes);
+adadsf_status adadsf_align_hidden(const void *hs_dev, const void *hd_dev, int64_t n_rows, int d, int dtype,
+                                  double *acc_dev, float *grad_dev, void *ws, size_t ws_bytes, void *stream);
+adadsf_status adadsf_align_output(const void *hs_dev, const void *hd_dev, const void *w_head_dev,
+                                  int64_t n_rows, int d, int n_classes, int dtype, double *acc_dev,
+                                  void *ws, size_t ws_bytes, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Sec. 3.4 ("the router-score pathway is kept differentiable"): the gradient
+ * of a loss with respect to one layer's router parameters through the score
+ * gate of ADADSF_FLAG_GATE_SIGMOID, where a kept row is y = x + sigmoid(s)
+ * delta. The layer input and its other weights are held fixed and the Top-K
+ * choice carries no gradient. x_dev [B*T, d]: the layer input; y_plain_dev
+ * [B*T, d]: the UNGATED layer's output on the same kept set (delta =
+ * y_plain - x on kept rows); rows_dev [n_kept]: the kept rows (b*T +
+ * position); grad_y_dev fp32 [B*T, d]: dL/dy (only kept rows are read).
+ * grad_out_dev fp32 receives, contiguously, dL/dW1 [router_hidden, d],
+ * dL/db1 [router_hidden], dL/dw2 [router_hidden], dL/db2 [1]:
+ *   ds = sigmoid'(s) (dL/dy . delta), dw2 = sum ds SiLU(u), db2 = sum ds,
+ *   du = ds w2 SiLU'(u), dW1 = sum du x^T, db1 = sum du, u = W1 x + b1.
+ * ws: adadsf_router_backward_workspace_size(cfg, n_kept) bytes.
+ * ---------------------------------------------------------------------- */
+size_t adadsf_router_backward_workspace_size(const adadsf_model_cfg *cfg, int64_t n_kept);
+adadsf_status adadsf_router_backward(const adadsf_model_cfg *cfg, const adadsf_layer_weights *w,
+                                     const void *x_dev, const void *y_plain_dev, const int32_t *rows_dev,
+                                     int64_t n_kept, const float *grad_y_dev, float *grad_out_dev,
+                                     void *ws, size_t ws_bytes, void *stream);
+
+/* ------------------------------------------------------------------------
  * Sec. 4.1 (the normalized FLOPs of Tables 1-2): FLOPs of the depth-sparse
  * forward over those of the dense model, per sequence of T tokens. Host
  * only, pure. Counted per layer l: the router on all T tokens when
@@ -420,6 +466,7 @@ typedef enum {
   ADADSF_KERNEL_TOPK_GATHER_NORM, /* Top-K fused with the gather and norms of the kept rows */
   ADADSF_KERNEL_DECIDE,        /* decode: keep decision of each new token */
   ADADSF_KERNEL_KV_CACHE,      /* decode cache: fill (prefill), thresholds, append */
+  ADADSF_KERNEL_ALIGN,         /* alignment objective and router gradient (Eqs. 9-10) */
   ADADSF_KERNEL_COUNT
 } adadsf_kernel_kind;
 

@@ -86,6 +86,11 @@ def lib() -> ctypes.CDLL:
             "adadsf_similarity": (i32, [vp, i32, i32, vp]),
             "adadsf_normalized_flops": (i32, [pcfg, i32, vp, vp]),
             "adadsf_fold_norms": (i32, [pcfg, plw, vp]),
+            "adadsf_align_workspace_size": (sz, [i64, i32]),
+            "adadsf_align_hidden": (i32, [vp, vp, i64, i32, i32, vp, vp, vp, sz, vp]),
+            "adadsf_align_output": (i32, [vp, vp, vp, i64, i32, i32, i32, vp, vp, sz, vp]),
+            "adadsf_router_backward_workspace_size": (sz, [pcfg, i64]),
+            "adadsf_router_backward": (i32, [pcfg, plw, vp, vp, vp, i64, vp, vp, vp, sz, vp]),
             "adadsf_alloc_ratios": (i32, [vp, i32, f64, f64, f64, i32, u32, vp, vp]),
             "adadsf_router_scores": (i32, [pcfg, plw, vp, i64, vp, vp, sz, vp]),
             "adadsf_topk_select": (i32, [vp, i32, i32, i32, vp, vp, vp]),
@@ -239,6 +244,47 @@ def adadsf_fold_norms(cfg: ModelCfg, w: dict, stream=None):
     device tensors of w in place (then run with FLAG_FOLDED_NORMS)."""
     lw = layer_struct(w)
     _check(lib().adadsf_fold_norms(ctypes.byref(cfg), ctypes.byref(lw), _s(stream)))
+
+
+def adadsf_align_hidden(hs: torch.Tensor, hd: torch.Tensor, acc: torch.Tensor,
+                        grad: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None, stream=None):
+    """Eq. 9: adds {sum of per-row softmax distances, rows} to acc (fp64);
+    grad (fp32, hs's shape) receives each row's gradient."""
+    _dev(hs, "hs"); _dev(hd, "hd"); _dev(acc, "acc")
+    d = hs.shape[-1]
+    n = hs.numel() // d
+    if ws is None:
+        ws = workspace(lib().adadsf_align_workspace_size(n, 0), hs.device)
+    _check(lib().adadsf_align_hidden(_p(hs), _p(hd), n, d, DTYPE_CODE[hs.dtype], _p(acc), _p(grad), _p(ws),
+                                     ws.numel(), _s(stream)))
+
+
+def adadsf_align_output(hs: torch.Tensor, hd: torch.Tensor, w_head: torch.Tensor, acc: torch.Tensor,
+                        ws: Optional[torch.Tensor] = None, stream=None):
+    """Eq. 10: adds {sum of per-row KL(P_dense || P_sparse), rows} to acc (fp64)."""
+    _dev(hs, "hs"); _dev(hd, "hd"); _dev(w_head, "w_head"); _dev(acc, "acc")
+    n_cls, d = w_head.shape
+    n = hs.numel() // d
+    if ws is None:
+        ws = workspace(lib().adadsf_align_workspace_size(n, n_cls), hs.device)
+    _check(lib().adadsf_align_output(_p(hs), _p(hd), _p(w_head), n, d, n_cls, DTYPE_CODE[hs.dtype], _p(acc),
+                                     _p(ws), ws.numel(), _s(stream)))
+
+
+def adadsf_router_backward(cfg: ModelCfg, w: dict, x: torch.Tensor, y_plain: torch.Tensor, rows: torch.Tensor,
+                           grad_y: torch.Tensor, ws: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Router gradient through the score gate; returns fp32 [h*d + 2h + 1]
+    (dW1, db1, dw2, db2)."""
+    _dev(x, "x"); _dev(y_plain, "y_plain"); _dev(rows, "rows"); _dev(grad_y, "grad_y")
+    n = rows.numel()
+    h = cfg.router_hidden
+    out = torch.empty(h * cfg.d + 2 * h + 1, dtype=torch.float32, device=x.device)
+    if ws is None:
+        ws = workspace(lib().adadsf_router_backward_workspace_size(ctypes.byref(cfg), n), x.device)
+    lw = layer_struct(w)
+    _check(lib().adadsf_router_backward(ctypes.byref(cfg), ctypes.byref(lw), _p(x), _p(y_plain), _p(rows), n,
+                                        _p(grad_y), _p(out), _p(ws), ws.numel(), _s(stream)))
+    return out
 
 
 def adadsf_normalized_flops(cfg: ModelCfg, T: int, K: Sequence[int]) -> float:

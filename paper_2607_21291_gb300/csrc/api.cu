@@ -1001,6 +1001,118 @@ adadsf_status adadsf_fold_norms(const adadsf_model_cfg* cfg, const adadsf_layer_
   return ADADSF_OK;
 }
 
+size_t adadsf_align_workspace_size(int64_t n_rows, int n_classes) {
+  if (n_rows < 0 || n_classes < 0) return 0;
+  return kErrBytes + kSyncBytes + align256((size_t)train_row_blocks(n_rows) * 8) +
+         2 * align256((size_t)n_rows * n_classes * 4);
+}
+
+adadsf_status adadsf_align_hidden(const void* hs_dev, const void* hd_dev, int64_t n_rows, int d, int dtype,
+                                  double* acc_dev, float* grad_dev, void* ws, size_t ws_bytes, void* stream) {
+  if (dtype != ADADSF_F32 && dtype != ADADSF_BF16) return fail(ADADSF_ERR_INVALID_ARG, "dtype %d unknown", dtype);
+  if (n_rows < 0 || d <= 0) return fail(ADADSF_ERR_INVALID_ARG, "need n_rows >= 0 and d > 0");
+  if (!acc_dev || (reinterpret_cast<uintptr_t>(acc_dev) & 7u))
+    return fail(ADADSF_ERR_INVALID_ARG, "acc_dev is NULL or not 8-byte aligned");
+  TRY(check_ws(ws, ws_bytes, adadsf_align_workspace_size(n_rows, 0)));
+  if (n_rows == 0) return ADADSF_OK;
+  NEED_PTR(hs_dev, "hs_dev");
+  NEED_PTR(hd_dev, "hd_dev");
+  if (grad_dev && (reinterpret_cast<uintptr_t>(grad_dev) & 3u))
+    return fail(ADADSF_ERR_INVALID_ARG, "grad_dev misaligned");
+  Dev dev;
+  TRY(device_info(&dev, stream, ws));
+  return launch(dev, ADADSF_KERNEL_ALIGN, false, 0, (2.0 + (grad_dev ? 2.0 : 0.0)) * n_rows * d * elem_size(dtype),
+                CALL(align_hidden(dtype, hs_dev, hd_dev, n_rows, d, grad_dev, at<double>(ws, kErrBytes + kSyncBytes),
+                                  acc_dev, dev),
+                     "hidden-state alignment"));
+}
+
+adadsf_status adadsf_align_output(const void* hs_dev, const void* hd_dev, const void* w_head_dev, int64_t n_rows,
+                                  int d, int n_classes, int dtype, double* acc_dev, void* ws, size_t ws_bytes,
+                                  void* stream) {
+  if (dtype != ADADSF_F32 && dtype != ADADSF_BF16) return fail(ADADSF_ERR_INVALID_ARG, "dtype %d unknown", dtype);
+  if (n_rows < 0 || d <= 0 || n_classes <= 0) return fail(ADADSF_ERR_INVALID_ARG, "need n_rows >= 0, d, n_classes > 0");
+  if (dtype == ADADSF_BF16 ? (d % 64 || n_classes % 64) : (d % 4 || n_classes % 4))
+    return fail(ADADSF_ERR_UNSUPPORTED, "d and n_classes must be multiples of %d", dtype == ADADSF_BF16 ? 64 : 4);
+  if (n_rows > (int64_t)INT32_MAX) return fail(ADADSF_ERR_UNSUPPORTED, "n_rows too large");
+  if (!acc_dev || (reinterpret_cast<uintptr_t>(acc_dev) & 7u))
+    return fail(ADADSF_ERR_INVALID_ARG, "acc_dev is NULL or not 8-byte aligned");
+  TRY(check_ws(ws, ws_bytes, adadsf_align_workspace_size(n_rows, n_classes)));
+  if (n_rows == 0) return ADADSF_OK;
+  NEED_PTR(hs_dev, "hs_dev");
+  NEED_PTR(hd_dev, "hd_dev");
+  NEED_PTR(w_head_dev, "w_head_dev");
+  Dev dev;
+  TRY(device_info(&dev, stream, ws));
+  Carver cv;
+  cv.take(kErrBytes);
+  cv.take(kSyncBytes);
+  const size_t part = cv.take((size_t)train_row_blocks(n_rows) * 8);
+  const size_t ls = cv.take((size_t)n_rows * n_classes * 4);
+  const size_t ld = cv.take((size_t)n_rows * n_classes * 4);
+  // logits h W_head^T of both models, fp32
+  for (int k = 0; k < 2; ++k) {
+    GemmArgs g = linear_args(k == 0 ? hs_dev : hd_dev, d, w_head_dev, n_rows, n_classes, d);
+    float* lg = at<float>(ws, k == 0 ? ls : ld);
+    if (dtype == ADADSF_BF16) {
+      g.epi.out_f32 = lg;
+      g.epi.ld_out = n_classes;
+    } else {
+      g.epi.out = lg;
+      g.epi.ld_out = n_classes;
+    }
+    TRY(launch(dev, ADADSF_KERNEL_LINEAR, dtype == ADADSF_BF16, 2.0 * n_rows * n_classes * d,
+               ((double)n_rows * d + (double)n_classes * d) * elem_size(dtype) + 4.0 * n_rows * n_classes,
+               [&] { return run_linear(dtype, g, dev, "head logits"); }));
+  }
+  return launch(dev, ADADSF_KERNEL_ALIGN, false, 0, 8.0 * n_rows * n_classes,
+                CALL(kl_rows(at<float>(ws, ls), at<float>(ws, ld), n_rows, n_classes, at<double>(ws, part), acc_dev,
+                             dev),
+                     "output alignment"));
+}
+
+size_t adadsf_router_backward_workspace_size(const adadsf_model_cfg* cfg, int64_t n_kept) {
+  if (check_cfg(cfg) != ADADSF_OK || n_kept < 0) return 0;
+  const size_t h = cfg->router_hidden;
+  return kErrBytes + align256((size_t)n_kept * h * 4) * 2 + align256((size_t)n_kept * 4);
+}
+
+adadsf_status adadsf_router_backward(const adadsf_model_cfg* cfg, const adadsf_layer_weights* w, const void* x_dev,
+                                     const void* y_plain_dev, const int32_t* rows_dev, int64_t n_kept,
+                                     const float* grad_y_dev, float* grad_out_dev, void* ws, size_t ws_bytes,
+                                     void* stream) {
+  TRY(check_cfg(cfg));
+  if (!w) return fail(ADADSF_ERR_INVALID_ARG, "weights are NULL");
+  NEED_PTR(w->router_w1, "router_w1");
+  NEED_PTR(w->router_b1, "router_b1");
+  NEED_PTR(w->router_w2, "router_w2");
+  if (!w->router_b2) return fail(ADADSF_ERR_INVALID_ARG, "router_b2 is NULL");
+  if (cfg->router_hidden > 64) return fail(ADADSF_ERR_UNSUPPORTED, "router_hidden > 64");
+  if (n_kept < 0) return fail(ADADSF_ERR_INVALID_ARG, "n_kept < 0");
+  NEED_PTR(grad_out_dev, "grad_out_dev");
+  TRY(check_ws(ws, ws_bytes, adadsf_router_backward_workspace_size(cfg, n_kept)));
+  if (n_kept > 0) {
+    NEED_PTR(x_dev, "x_dev");
+    NEED_PTR(y_plain_dev, "y_plain_dev");
+    if (!rows_dev) return fail(ADADSF_ERR_INVALID_ARG, "rows_dev is NULL");
+    if (!grad_y_dev) return fail(ADADSF_ERR_INVALID_ARG, "grad_y_dev is NULL");
+  }
+  Dev dev;
+  TRY(device_info(&dev, stream, ws));
+  const int h = cfg->router_hidden, d = cfg->d;
+  Carver cv;
+  cv.take(kErrBytes);
+  float* du = at<float>(ws, cv.take((size_t)n_kept * h * 4));
+  float* su = at<float>(ws, cv.take((size_t)n_kept * h * 4));
+  float* ds = at<float>(ws, cv.take((size_t)n_kept * 4));
+  return launch(dev, ADADSF_KERNEL_ALIGN, false, 4.0 * n_kept * h * d,
+                (double)n_kept * d * (2.0 * elem_size(cfg->dtype) + 4.0),
+                CALL(router_backward(cfg->dtype, x_dev, y_plain_dev, rows_dev, n_kept, d, h, w->router_w1,
+                                     w->router_b1, w->router_w2, w->router_b2, grad_y_dev, du, su, ds, grad_out_dev,
+                                     dev),
+                     "router backward"));
+}
+
 adadsf_status adadsf_normalized_flops(const adadsf_model_cfg* cfg, int T, const int32_t* K_host,
                                       double* out_host) {
   TRY(check_cfg(cfg));
@@ -1411,7 +1523,7 @@ const char* adadsf_kernel_name(int kind) {
   static const char* names[ADADSF_KERNEL_COUNT] = {
       "embed", "router", "topk", "positions", "gather_norm", "gemm_qkv", "rope_table", "rope",
       "attention", "gemm_o", "norm2", "gemm_up", "gemm_down", "stats", "final_norm", "copy",
-      "linear", "selftest", "gemm_qkv_up", "gemm_o_down", "topk_gather_norm", "decide", "kv_cache"};
+      "linear", "selftest", "gemm_qkv_up", "gemm_o_down", "topk_gather_norm", "decide", "kv_cache", "align"};
   return (kind >= 0 && kind < ADADSF_KERNEL_COUNT) ? names[kind] : "unknown";
 }
 

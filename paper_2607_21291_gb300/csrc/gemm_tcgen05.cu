@@ -112,6 +112,7 @@ struct GemmDev {
   float* sq_out; int sq_ld;
   float4* cos_out; int cos_ld;
   const bf16* cin; int64_t ld_cin;
+  float* out_f32;            // fp32 output instead of out (see Epilogue::out_f32)
   int* err;
   unsigned long long timeout_ns;
 };
@@ -353,6 +354,15 @@ __device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, cons
     }
     if (p.sq_out) p.sq_out[m * p.sq_ld + (n0 >> 5)] = sq;
     if (p.cos_out) p.cos_out[m * p.cos_ld + (n0 >> 5)] = make_float4(dot, nx, sq, 0.f);
+  }
+  if (EXTRA && p.out_f32) {
+    // fp32 output row chunk (uniform branch for the warp)
+    if (valid) {
+      float4* dst = reinterpret_cast<float4*>(p.out_f32 + orow * p.ld_out + n0);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+    }
+    return;
   }
   uint4 pk[4];
 #pragma unroll
@@ -1355,6 +1365,10 @@ bool make_dev(const GemmArgs& a, const Dev& dev, GemmDev& p) {
     p.cin = static_cast<const bf16*>(a.epi.cos_in);
     p.ld_cin = a.epi.ld_cos_in;
   }
+  if (a.epi.out_f32) {
+    if (a.epi.rope_tab || a.epi.add_packed || a.epi.add_rows || a.epi.vt || a.N % 32 != 0) return false;
+    p.out_f32 = a.epi.out_f32;
+  }
   if (a.epi.gate_scores) {
     // gated residual: x gathered (out = x + g v), or h packed with x as the base
     if (a.epi.rope_tab) return false;
@@ -1430,7 +1444,7 @@ cudaError_t prepare(const GemmArgs& a, const GemmArgs* b, uint32_t a_rows, int b
 
 // Whether a launch needs the epilogue instance with the rarer features.
 bool extra_args(const GemmArgs& a) {
-  return a.epi.gate_scores || a.epi.sq_out || a.epi.cos_out || a.epi.nrm_psum;
+  return a.epi.gate_scores || a.epi.sq_out || a.epi.cos_out || a.epi.nrm_psum || a.epi.out_f32;
 }
 
 template <int BN, bool DUAL, bool EXTRA>

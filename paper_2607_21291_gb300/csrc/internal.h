@@ -73,6 +73,9 @@ struct Epilogue {
   int cos_ld = 0;
   const void* cos_in = nullptr;
   int64_t ld_cos_in = 0;
+  // fp32 output instead of `out` (bf16 path, no residual): out_f32[row][n],
+  // leading dimension ld_out (the logits of the output alignment, Eq. 10)
+  float* out_f32 = nullptr;
 };
 
 // acc = A . W^T (+ A2 . Wk2^T when K2 > 0: a second K source, bf16
@@ -118,6 +121,15 @@ cudaError_t gemm_bf16(const GemmArgs& a, const Dev& dev);
 // Two independent plain projections (no SwiGLU, router or second K source)
 // in one launch.
 cudaError_t gemm_bf16_grouped(const GemmArgs& a, const GemmArgs& b, const Dev& dev);
+// train.cu -- alignment objective (Eqs. 9-10) and the router gradient.
+int train_row_blocks(int64_t n);
+cudaError_t align_hidden(int dtype, const void* hs, const void* hd, int64_t n_rows, int d, float* grad,
+                         double* partials, double* acc, const Dev& dev);
+cudaError_t kl_rows(const float* ls, const float* ld, int64_t n_rows, int n_cls, double* partials, double* acc,
+                    const Dev& dev);
+cudaError_t router_backward(int dtype, const void* x, const void* y_plain, const int32_t* rows, int64_t M, int d,
+                            int h, const void* w1, const void* b1, const void* w2, const void* b2, const float* G,
+                            float* du, float* su, float* ds, float* grad, const Dev& dev);
 // gemm_simt.cu -- fp32 projections on CUDA cores.
 cudaError_t gemm_f32(const GemmArgs& a, const Dev& dev);
 

@@ -1,0 +1,105 @@
+"""GPU parity of the training-side pieces against the oracle, through the C
+ABI: the hidden-state alignment of Eq. 9 (value and gradient), the output
+alignment of Eq. 10 (KL over the classes of an LM head), and the router's
+gradient through the score gate (Sec. 3.4, differentiable score pathway)."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import adadsf_oracle as O
+from paper_2607_21291_gb300 import synth as S
+from tests import helpers as H
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def A():
+    from paper_2607_21291_gb300 import adadsf
+    adadsf.lib()
+    return adadsf
+
+
+@pytest.mark.parametrize("n,d,dtype", [(1, 64, "f32"), (3001, 1024, "bf16"), (777, 512, "f32"), (40, 3584, "bf16")])
+def test_align_hidden(A, n, d, dtype):
+    g = np.random.default_rng(n + d)
+    hs = S.round_to(g.standard_normal((n, d)).astype(np.float32) * 2, dtype)
+    hd = S.round_to((hs + 0.5 * g.standard_normal((n, d))).astype(np.float32), dtype)
+    td = torch.bfloat16 if dtype == "bf16" else torch.float32
+    acc = torch.zeros(2, dtype=torch.float64, device="cuda")
+    grad = torch.empty((n, d), dtype=torch.float32, device="cuda")
+    A.adadsf_align_hidden(H.to_dev(hs, td), H.to_dev(hd, td), acc, grad)
+    got = acc.cpu().numpy()
+    ref = O.hidden_alignment(hs.astype(np.float64), hd.astype(np.float64))
+    assert got[1] == n
+    assert got[0] == pytest.approx(ref.sum(), rel=1e-4)
+    H.assert_close(grad.cpu().numpy(), O.hidden_alignment_grad(hs.astype(np.float64), hd.astype(np.float64)),
+                   1e-3, "grad")
+    again = torch.zeros(2, dtype=torch.float64, device="cuda")
+    A.adadsf_align_hidden(H.to_dev(hs, td), H.to_dev(hd, td), again)
+    assert again.cpu().numpy().tolist() == got.tolist()        # fixed summation order
+
+
+@pytest.mark.parametrize("n,d,V,dtype", [(64, 1024, 2048, "bf16"), (5, 64, 128, "bf16"), (33, 512, 1000, "f32"),
+                                         (300, 768, 6272, "bf16")])
+def test_align_output(A, n, d, V, dtype):
+    g = np.random.default_rng(n * V + d)
+    hs = S.round_to(g.standard_normal((n, d)).astype(np.float32), dtype)
+    hd = S.round_to((hs + 0.3 * g.standard_normal((n, d))).astype(np.float32), dtype)
+    W = S.round_to((g.standard_normal((V, d)) * 0.05).astype(np.float32), dtype)
+    td = torch.bfloat16 if dtype == "bf16" else torch.float32
+    acc = torch.zeros(2, dtype=torch.float64, device="cuda")
+    A.adadsf_align_output(H.to_dev(hs, td), H.to_dev(hd, td), H.to_dev(W, td), acc)
+    got = acc.cpu().numpy()
+    ref = O.output_alignment(hs.astype(np.float64), hd.astype(np.float64), W.astype(np.float64))
+    assert got[1] == n
+    assert got[0] == pytest.approx(ref.sum(), rel=2e-3)
+    same = torch.zeros(2, dtype=torch.float64, device="cuda")
+    A.adadsf_align_output(H.to_dev(hs, td), H.to_dev(hs, td), H.to_dev(W, td), same)
+    assert abs(same.cpu().numpy()[0]) < 1e-5 * n                # KL(P || P) = 0
+
+
+QWEN_SMALL = S.QWEN25_1_5B.replace(d=1024, n_heads=8, n_kv_heads=2, ffn=1536, n_layers=1)
+
+
+@pytest.mark.parametrize("shape,B,T,K", [(QWEN_SMALL, 2, 150, 70), (S.PYTHIA_160M.replace(n_layers=1), 3, 100, 37),
+                                         (S.PYTHIA_70M.replace(n_layers=1), 1, 128, 64),
+                                         (QWEN_SMALL, 2, 2048, 1500)])
+def test_router_backward(A, shape, B, T, K):
+    """The gated layer on the GPU, the ungated one on the same kept set (its
+    delta), an upstream gradient G; the router gradient matches the oracle's
+    chain rule on the same delta, and the gated layer still matches the
+    oracle's gated layer."""
+    td = H.tdtype(shape)
+    W = H.host_layer(shape, 41)
+    x = S.round_to(S.hidden(41, B, T, shape.d), shape.dtype)
+    wd = A.to_device(W, td)
+    outs = {}
+    for flags in (A.FLAG_GATE_SIGMOID, 0):
+        cfg = A.make_cfg(shape, flags)
+        xd = H.to_dev(x, td)
+        idx = torch.empty((B, K), dtype=torch.int32, device="cuda")
+        ws = A.workspace(A.adadsf_layer_workspace_size(cfg, B, T, K))
+        A.adadsf_sparse_layer_forward(cfg, wd, xd, K, idx, None, ws)
+        assert A.adadsf_sync_check(ws) == A.OK
+        outs[flags] = (xd, idx)
+    (yg, idx_g), (yp, idx_p) = outs[A.FLAG_GATE_SIGMOID], outs[0]
+    assert torch.equal(idx_g, idx_p)
+    gi = idx_g.cpu().numpy()
+    rows = (np.arange(B)[:, None] * T + gi).reshape(-1)
+    G = np.random.default_rng(B * T + K).standard_normal((B * T, shape.d)).astype(np.float32)
+    grad = A.adadsf_router_backward(A.make_cfg(shape, A.FLAG_GATE_SIGMOID), wd, H.to_dev(x, td), yp,
+                                    torch.from_numpy(rows.astype(np.int32)).cuda(), H.to_dev(G, torch.float32))
+    x64 = x.astype(np.float64)
+    delta = (H.to_np(yp).reshape(-1, shape.d) - x64.reshape(-1, shape.d))[rows]
+    ref = O.router_grad(x64, H.f64(W), rows, delta, G.astype(np.float64)[rows])
+    h, d = shape.router_hidden, shape.d
+    g = grad.cpu().numpy().astype(np.float64)
+    parts = {"router_w1": g[:h * d].reshape(h, d), "router_b1": g[h * d:h * d + h],
+             "router_w2": g[h * d + h:h * d + 2 * h], "router_b2": g[h * d + 2 * h:]}
+    tol = 2e-3 if shape.dtype == "bf16" else 1e-4
+    for k, v in parts.items():
+        H.assert_close(v, ref[k], tol, k)
+    # and the gated forward itself follows the oracle's gated layer
+    refg, _, _ = O.sparse_layer_forward(x64, H.f64(W), dict(O.params_of(shape), gate="sigmoid"), K, idx=gi)
+    H.assert_close(H.to_np(yg), refg, H.tol(shape), "gated layer")
