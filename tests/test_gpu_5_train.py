@@ -103,3 +103,22 @@ def test_router_backward(A, shape, B, T, K):
     # and the gated forward itself follows the oracle's gated layer
     refg, _, _ = O.sparse_layer_forward(x64, H.f64(W), dict(O.params_of(shape), gate="sigmoid"), K, idx=gi)
     H.assert_close(H.to_np(yg), refg, H.tol(shape), "gated layer")
+
+
+@pytest.mark.parametrize("shape,lr", [(S.PYTHIA_70M.replace(n_layers=1), 3000.0),
+                                      (QWEN_SMALL.replace(dtype="f32"), 3000.0)])
+def test_router_alignment_descends(A, shape, lr):
+    """Plain SGD on the router through the gated layer (paper_2607_21291_gb300.align)
+    lowers the layer's Eq. 9 loss against the dense layer's output: the
+    gradient points downhill."""
+    from paper_2607_21291_gb300 import align
+    B, T, K = 2, 96, 48
+    td = H.tdtype(shape)
+    w = A.to_device(H.host_layer(shape, 51), td)
+    x = H.to_dev(S.round_to(S.hidden(51, B, T, shape.d), shape.dtype), td)
+    cfg = A.make_cfg(shape)
+    h_dense = x.clone()
+    A.adadsf_sparse_layer_forward(cfg, w, h_dense, T)          # the dense layer
+    losses = [align.router_alignment_step(cfg, w, x, h_dense, K, lr) for _ in range(6)]
+    assert all(b <= a * (1 + 1e-6) for a, b in zip(losses, losses[1:])), losses
+    assert losses[-1] < losses[0] * 0.999, losses
