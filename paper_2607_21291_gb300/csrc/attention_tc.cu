@@ -1,10 +1,14 @@
 // Eq. 1 among the kept tokens on the 5th-generation tensor cores (bf16).
 //
-// One CTA per (pair of 128-query blocks, query head, sequence): the two
-// query tiles share every K / V tile the CTA loads, which halves the K / V
-// traffic per flop, and their softmax work alternates with the other tile's
-// matrix products. When pairs would leave SMs idle (few, short sequences),
-// one CTA per query block instead. Keys arrive in blocks of 128; attention is causal in
+// Work items are (pair of 128-query blocks, query head, sequence): the two
+// query tiles share every K / V tile loaded, which halves the K / V traffic
+// per flop, and their softmax work alternates with the other tile's matrix
+// products. When pairs would leave SMs idle (few, short sequences), one
+// query block per item instead. The kernel is persistent: one CTA per SM
+// walks its share of the items (longest causal rows first), the K / V rings
+// and every barrier phase running on across items, so one item's output
+// epilogue overlaps the next item's Q load and first scores, and the CTA's
+// set-up (barriers, TMEM) is paid once. Keys arrive in blocks of 128; attention is causal in
 // packed order (kept positions ascend, so this is the original causal mask
 // restricted to the kept set, Sec. 3.4).
 //   warp 0     TMA, lane 0: both Q tiles once, then the K tile of each key
@@ -63,7 +67,7 @@ struct AttnCfg {
   static constexpr int V_SLAB = HD * 128;          // HD feature rows x 64 keys
   static constexpr int V_BYTES = 2 * V_SLAB;       // 128 keys
   static constexpr int DATA = 2 * Q_BYTES + KST * K_BYTES + VST * V_BYTES;
-  static constexpr int NBARS = 1 + 2 * KST + 2 * VST + 7;
+  static constexpr int NBARS = 1 + 2 * KST + 2 * VST + 10;
   // barriers, TMEM address, abort flag; then the softmax pairs' exchange
   // area: [tile][quarter][half][lane] floats
   static constexpr int XCHG = 2 * 4 * 2 * 32 * 4;
@@ -99,14 +103,34 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
 
 struct AttnDev {
   int K;                 // kept tokens per sequence
-  int pair;              // 1: two query blocks per CTA, 0: one
-  int Hq, Hkv, q_dim;
+  int pair;              // 1: two query blocks per work item, 0: one
+  int B, Hq, Hkv, q_dim;
   float scale_log2;      // log2(e) / sqrt(hd)
   bf16* out;
   int64_t ld_out;
   int* err;
   unsigned long long timeout_ns;
 };
+
+// Work item w of the persistent schedule: query head h, sequence b and
+// query-block group z (z = 0 holds each (head, sequence)'s longest causal
+// rows). Items are numbered h fastest, then b, then z, so the longest rows of
+// every head and sequence come first; CTA c takes items c, c + G, c + 2G, ...
+struct AttnItem {
+  int h, b, qb0, two, n_kv, g, row0;
+};
+__device__ __forceinline__ AttnItem attn_item(const AttnDev& p, int w, int nqb) {
+  AttnItem it;
+  it.h = w % p.Hq;
+  it.b = (w / p.Hq) % p.B;
+  const int z = w / (p.Hq * p.B);
+  it.qb0 = p.pair ? 2 * ((nqb + 1) / 2 - 1 - z) : nqb - 1 - z;
+  it.two = (p.pair && it.qb0 + 1 < nqb) ? 1 : 0;   // tile 1 holds query block qb0 + 1
+  it.n_kv = it.two ? it.qb0 + 2 : it.qb0 + 1;        // tile 0 takes blocks 0..qb0, tile 1 all
+  it.g = it.h / (p.Hq / p.Hkv);
+  it.row0 = it.b * p.K;
+  return it;
+}
 
 template <int HD>
 __global__ void __launch_bounds__(kAttnThreads, 1)
@@ -135,6 +159,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const uint32_t p_full0 = s_full0 + 16;           // [2] per tile: P_t written (8 warps)
   const uint32_t o_done0 = p_full0 + 16;           // [2] per tile: P_t V of the block done
   const uint32_t drain = o_done0 + 16;
+  const uint32_t q_empty = drain + 8;              // the item's S products have read Q
+  const uint32_t o_free0 = q_empty + 8;            // [2] per tile: O_t read out (8 warps)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + C::NBARS);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   // softmax pairs' exchange: [tile][quarter][half][lane]
@@ -143,19 +169,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int nqb = (p.K + kQB - 1) / kQB;
-  // Block (h, b, z): blocks are dispatched in linear order (x fastest), so
-  // every head and sequence starts its longest rows (z = 0) before any
-  // shorter ones and the last wave holds the short ones.
-  const int qb0 = p.pair ? 2 * ((nqb + 1) / 2 - 1 - (int)blockIdx.z) : nqb - 1 - (int)blockIdx.z;
-  const bool two = p.pair && qb0 + 1 < nqb;     // tile 1 holds query block qb0 + 1
-  const int n_kv = two ? qb0 + 2 : qb0 + 1;     // tile 0 takes blocks 0..qb0, tile 1 all
-  const int h = blockIdx.x, b = blockIdx.y;
-  const int g = h / (p.Hq / p.Hkv);
-  const int row0 = b * p.K;
+  const int n_items = p.Hq * p.B * (p.pair ? (nqb + 1) / 2 : nqb);
 
   pdl_trigger();
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
+    mbar_init(q_empty, 1);
     for (int i = 0; i < KST; ++i) {
       mbar_init(k_full0 + 8 * i, 1);
       mbar_init(k_empty0 + 8 * i, 1);
@@ -168,6 +187,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       mbar_init(s_full0 + 8 * t, 1);
       mbar_init(p_full0 + 8 * t, 8);
       mbar_init(o_done0 + 8 * t, 1);
+      mbar_init(o_free0 + 8 * t, 8);
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -187,41 +207,51 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producers
-    // lane 0: both Q tiles once, then the K ring; lane 1: the V^T ring
+    // lane 0: each item's Q tiles (once the previous item's scores are done
+    // with Q), then its K blocks into the ring; lane 1: the V^T ring. Ring
+    // positions run on across items.
     if (lane < 2) {
       const bool kprod = lane == 0;
       const int NST = kprod ? KST : VST;
       pdl_wait();
-      if (kprod) {
-        mbar_arrive_expect_tx(q_full, (two ? 2 : 1) * C::Q_BYTES);
-        for (int t = 0; t < (two ? 2 : 1); ++t)
-          for (int s = 0; s < C::HS; ++s)
-            tma_load_2d(sQ + t * C::Q_BYTES + s * C::SLAB, &tmQK, h * HD + s * 64,
-                        row0 + (qb0 + t) * kQB, q_full);
-      }
       const uint32_t full0 = kprod ? k_full0 : v_full0;
       const uint32_t empty0 = kprod ? k_empty0 : v_empty0;
-      int issued = 0;
-      for (int j = 0; j < n_kv; ++j) {
-        const int st = j % NST;
-        if (!mbar_wait_bounded(empty0 + 8 * st, ((j / NST) & 1) ^ 1, abort_flag, p.err, p.timeout_ns))
-          break;
-        const uint32_t fb = full0 + 8 * st;
+      int issued = 0;   // ring position (copies issued)
+      int it = 0;       // items of this CTA
+      bool ok = true;
+      for (int w = blockIdx.x; ok && w < n_items; w += gridDim.x, ++it) {
+        const AttnItem I = attn_item(p, w, nqb);
         if (kprod) {
-          mbar_arrive_expect_tx(fb, C::K_BYTES);
-          for (int s = 0; s < C::HS; ++s)
-            tma_load_2d(sK0 + st * C::K_BYTES + s * C::SLAB, &tmQK, p.q_dim + g * HD + s * 64,
-                        row0 + j * kKB, fb);
-        } else {
-          mbar_arrive_expect_tx(fb, C::V_BYTES);
-          for (int ks = 0; ks < 2; ++ks)
-            tma_load_2d(sV0 + st * C::V_BYTES + ks * C::V_SLAB, &tmVt, j * kKB + ks * 64,
-                        (b * p.Hkv + g) * HD, fb);
+          if (it > 0 && !mbar_wait_bounded(q_empty, (it - 1) & 1, abort_flag, p.err, p.timeout_ns)) break;
+          mbar_arrive_expect_tx(q_full, (I.two ? 2 : 1) * C::Q_BYTES);
+          for (int t = 0; t < (I.two ? 2 : 1); ++t)
+            for (int s = 0; s < C::HS; ++s)
+              tma_load_2d(sQ + t * C::Q_BYTES + s * C::SLAB, &tmQK, I.h * HD + s * 64,
+                          I.row0 + (I.qb0 + t) * kQB, q_full);
         }
-        ++issued;
+        for (int j = 0; j < I.n_kv; ++j) {
+          const int st = issued % NST;
+          if (!mbar_wait_bounded(empty0 + 8 * st, ((issued / NST) & 1) ^ 1, abort_flag, p.err, p.timeout_ns)) {
+            ok = false;
+            break;
+          }
+          const uint32_t fb = full0 + 8 * st;
+          if (kprod) {
+            mbar_arrive_expect_tx(fb, C::K_BYTES);
+            for (int s = 0; s < C::HS; ++s)
+              tma_load_2d(sK0 + st * C::K_BYTES + s * C::SLAB, &tmQK, p.q_dim + I.g * HD + s * 64,
+                          I.row0 + j * kKB, fb);
+          } else {
+            mbar_arrive_expect_tx(fb, C::V_BYTES);
+            for (int ks = 0; ks < 2; ++ks)
+              tma_load_2d(sV0 + st * C::V_BYTES + ks * C::V_SLAB, &tmVt, j * kKB + ks * 64,
+                          (I.b * p.Hkv + I.g) * HD, fb);
+          }
+          ++issued;
+        }
       }
-      // drain: the copies issued last into each stage have landed
-      if (kprod) mbar_wait_drain(q_full, 0, p.timeout_ns);
+      // drain: the copies issued last into each stage (and the last Q) have landed
+      if (kprod && it > 0) mbar_wait_drain(q_full, (it - 1) & 1, p.timeout_ns);
       for (int st = 0; st < NST && st < issued; ++st) {
         const int last = st + ((issued - 1 - st) / NST) * NST;
         mbar_wait_drain(full0 + 8 * st, (uint32_t)((last / NST) & 1), p.timeout_ns);
@@ -232,9 +262,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     if (lane == 0) {
       constexpr uint32_t idesc_s = idesc_bf16_f32(kQB, kKB);
       constexpr uint32_t idesc_o = idesc_bf16_f32(kQB, HD);
-      // S_t(j) = Q_t K(j)^T into TMEM S_t
-      auto issue_s = [&](int t, int j) {
-        const uint32_t kst = sK0 + (j % KST) * C::K_BYTES;
+      // S_t(j) = Q_t K(j)^T into TMEM S_t, K block in ring slot kslot
+      auto issue_s = [&](int t, int kslot) {
+        const uint32_t kst = sK0 + kslot * C::K_BYTES;
         const uint32_t qt = sQ + t * C::Q_BYTES;
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk) {
@@ -244,47 +274,73 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
         }
         tc_commit(s_full0 + 8 * t);
       };
-      // O_t += P_t(j) V(j), P_t read from TMEM
-      auto issue_pv = [&](int t, int j) {
-        const uint32_t vst = sV0 + (j % VST) * C::V_BYTES;
+      // O_t (+)= P_t V, P_t read from TMEM, V^T block in ring slot vslot
+      auto issue_pv = [&](int t, int vslot, bool acc) {
+        const uint32_t vst = sV0 + vslot * C::V_BYTES;
 #pragma unroll
         for (int kk = 0; kk < kKB / 16; ++kk)   // keys 16 kk.. of P_t: columns 64 (kk / 4) + 8 (kk % 4)
           tc_mma_f16_ta(tmem_base + C::TO + t * HD, tmem_base + C::TS + t * kKB + (kk >> 2) * 64 + (kk & 3) * 8,
                         smem_desc_sw128(vst + (kk >> 2) * C::V_SLAB + (kk & 3) * 32), idesc_o,
-                        (j > 0 || kk > 0) ? 1u : 0u);
+                        (acc || kk > 0) ? 1u : 0u);
         tc_commit(o_done0 + 8 * t);
       };
       auto wait = [&](uint32_t bar, uint32_t parity) {
         return mbar_wait_bounded(bar, parity, abort_flag, p.err, p.timeout_ns);
       };
-      const int last0 = qb0;   // tile 0's last key block
-      bool ok = wait(q_full, 0) && wait(k_full0, 0);
-      if (ok) {
+      int kc = 0, vc = 0;          // ring positions of the K and V^T blocks
+      int pc[2] = {0, 0};          // P_t blocks consumed per tile
+      int oc[2] = {0, 0};          // items finished per tile (their O read out)
+      bool ok = true;
+      int it = 0;
+      for (int w = blockIdx.x; ok && w < n_items; w += gridDim.x, ++it) {
+        const AttnItem I = attn_item(p, w, nqb);
+        const int last0 = I.qb0;   // tile 0's last key block
+        ok = wait(q_full, it & 1) && wait(k_full0 + 8 * (kc % KST), (kc / KST) & 1);
+        if (!ok) break;
         tc_fence_after();
-        issue_s(0, 0);
-        if (two) issue_s(1, 0);
-        tc_commit(k_empty0);
-      }
-      for (int j = 0; ok && j < n_kv; ++j) {
-        const bool has0 = j <= last0;
-        const bool next = j + 1 < n_kv;
-        if (!wait(v_full0 + 8 * (j % VST), (j / VST) & 1)) { ok = false; break; }
-        if (has0) {
-          if (!wait(p_full0, j & 1)) { ok = false; break; }
+        // S_t(0) may overwrite the previous item's P_t: its P V was issued
+        // before, and one thread's tcgen05 operations run in order
+        issue_s(0, kc % KST);
+        if (I.two) issue_s(1, kc % KST);
+        tc_commit(k_empty0 + 8 * (kc % KST));
+        for (int j = 0; j < I.n_kv; ++j) {
+          const bool has0 = j <= last0;
+          const bool next = j + 1 < I.n_kv;
+          const int vslot = vc % VST;
+          const int knext = (kc + 1) % KST;
+          if (!wait(v_full0 + 8 * vslot, (vc / VST) & 1)) { ok = false; break; }
+          if (has0) {
+            if (!wait(p_full0, pc[0] & 1)) { ok = false; break; }
+            ++pc[0];
+            // the first P V of an item overwrites O_0: the previous item's
+            // epilogue must have read it out
+            if (j == 0 && oc[0] > 0 && !wait(o_free0, (oc[0] - 1) & 1)) { ok = false; break; }
+            tc_fence_after();
+            issue_pv(0, vslot, j > 0);
+          }
+          if (next && !wait(k_full0 + 8 * knext, ((kc + 1) / KST) & 1)) { ok = false; break; }
           tc_fence_after();
-          issue_pv(0, j);
+          if (next && j + 1 <= last0) issue_s(0, knext);
+          if (I.two) {
+            if (!wait(p_full0 + 8, pc[1] & 1)) { ok = false; break; }
+            ++pc[1];
+            if (j == 0 && oc[1] > 0 && !wait(o_free0 + 8, (oc[1] - 1) & 1)) { ok = false; break; }
+            tc_fence_after();
+            issue_pv(1, vslot, j > 0);
+            if (next) issue_s(1, knext);
+          }
+          tc_commit(v_empty0 + 8 * vslot);            // V(j) read by both tiles
+          ++vc;
+          if (next) {
+            tc_commit(k_empty0 + 8 * knext);          // K(j+1) read by both tiles
+            ++kc;
+          }
         }
-        if (next && !wait(k_full0 + 8 * ((j + 1) % KST), ((j + 1) / KST) & 1)) { ok = false; break; }
-        tc_fence_after();
-        if (next && j + 1 <= last0) issue_s(0, j + 1);
-        if (two) {
-          if (!wait(p_full0 + 8, j & 1)) { ok = false; break; }
-          tc_fence_after();
-          issue_pv(1, j);
-          if (next) issue_s(1, j + 1);
-        }
-        tc_commit(v_empty0 + 8 * (j % VST));            // V(j) read by both tiles
-        if (next) tc_commit(k_empty0 + 8 * ((j + 1) % KST));   // K(j+1) read by both tiles
+        if (!ok) break;
+        ++kc;                                  // past the item's last K block
+        for (int t = 0; t < 2; ++t)
+          if (t == 0 || I.two) ++oc[t];
+        tc_commit(q_empty);                    // the item's scores are done with Q
       }
       tc_commit(drain);
       mbar_wait_drain(drain, 0, p.timeout_ns);
@@ -296,12 +352,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
     const int half = ((warp - 2) >> 2) & 1;        // key columns [64 half, 64 half + 64)
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;             // query row in the tile = TMEM lane
-    const int qbt = qb0 + t;
-    const int qi = qbt * kQB + r;                  // query index in the sequence
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
     const uint32_t tS = tmem_base + C::TS + t * kKB + lane_off;
     const uint32_t tO = tmem_base + C::TO + t * HD + lane_off + half * (HD / 2);
-    const bool active = t == 0 || two;
     const int bar_id = 1 + t * 4 + quarter;        // named barrier of the warp pair
     volatile float* xq = xchg + (t * 4 + quarter) * 64;
     // partner's value (same rows, other half of the columns); the second
@@ -313,11 +366,19 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       named_bar_sync(bar_id, 64);
       return theirs;
     };
+    int sc = 0;    // S_t blocks consumed (the s_full phase)
+    int pvc = 0;   // P_t V products of earlier items (the o_done phase)
+    bool ok = true;
+    for (int wi = blockIdx.x; ok && wi < n_items; wi += gridDim.x) {
+    const AttnItem I = attn_item(p, wi, nqb);
+    if (t == 1 && !I.two) continue;                // this item has one query tile
+    const int qbt = I.qb0 + t;
+    const int qi = qbt * kQB + r;                  // query index in the sequence
     float m_used = -INFINITY, l = 0.f;
-    bool ok = active;
     for (int j = 0; ok && j <= qbt; ++j) {
       int w = 0;
-      if (lane == 0) w = mbar_wait_bounded(s_full0 + 8 * t, j & 1, abort_flag, p.err, p.timeout_ns);
+      if (lane == 0) w = mbar_wait_bounded(s_full0 + 8 * t, sc & 1, abort_flag, p.err, p.timeout_ns);
+      ++sc;
       w = __shfl_sync(0xffffffffu, w, 0);
       tc_fence_after();
       const uint32_t tSh = tS + half * 64;         // this half's 64 score columns
@@ -399,17 +460,19 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
       if (lane == 0) mbar_arrive(p_full0 + 8 * t);
     }
     // epilogue: O_t / l (both halves' sums) once the tile's last P V is done
-    if (active) {
+    {
       const float l_all = l + exchange(l);
       if (ok) {
         int w = 0;
-        if (lane == 0) w = mbar_wait_bounded(o_done0 + 8 * t, qbt & 1, abort_flag, p.err, p.timeout_ns);
+        if (lane == 0)
+          w = mbar_wait_bounded(o_done0 + 8 * t, (pvc + qbt) & 1, abort_flag, p.err, p.timeout_ns);
         ok = __shfl_sync(0xffffffffu, w, 0) != 0;
       }
+      pvc += qbt + 1;
       if (ok) {
         tc_fence_after();
         const float inv = 1.f / l_all;
-        bf16* dst = p.out + (int64_t)(row0 + qi) * p.ld_out + (int64_t)h * HD + half * (HD / 2);
+        bf16* dst = p.out + (int64_t)(I.row0 + qi) * p.ld_out + (int64_t)I.h * HD + half * (HD / 2);
 #pragma unroll 1
         for (int c = 0; c < HD / 64; ++c) {
           uint32_t o[32];
@@ -424,7 +487,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1)
           }
         }
       }
+      // O_t is read out: the next item's first P V may overwrite it
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(o_free0 + 8 * t);
     }
+    }   // items
   }
 
   // Reconverge each warp first: in the producer and MMA warps only lane 0
@@ -516,6 +584,7 @@ cudaError_t launch_attn(const void* qkv, int64_t ld_qkv, const void* vt, int pad
     return cudaErrorInvalidValue;
   AttnDev p;
   p.K = K;
+  p.B = B;
   p.Hq = Hq;
   p.Hkv = Hkv;
   p.q_dim = Hq * HD;
@@ -526,8 +595,12 @@ cudaError_t launch_attn(const void* qkv, int64_t ld_qkv, const void* vt, int pad
   p.timeout_ns = kWaitTimeoutNs;
   const int nqb = (K + kQB - 1) / kQB;
   p.pair = (int64_t)((nqb + 1) / 2) * Hq * B >= dev.num_sms ? 1 : 0;
-  dim3 grid(Hq, B, p.pair ? (nqb + 1) / 2 : nqb);
-  return launch_pdl(attn_tc_kernel<HD>, grid, dim3(kAttnThreads), C::SMEM, dev.stream, tq, tv, p);
+  // persistent: one CTA per SM (TMEM is allocated in full) over the work
+  // items, each CTA taking every G-th item of the longest-first order
+  const int64_t items = (int64_t)Hq * B * (p.pair ? (nqb + 1) / 2 : nqb);
+  if (items > INT32_MAX) return cudaErrorInvalidValue;
+  const int64_t grid = items < dev.num_sms ? items : dev.num_sms;
+  return launch_pdl(attn_tc_kernel<HD>, dim3((unsigned)grid), dim3(kAttnThreads), C::SMEM, dev.stream, tq, tv, p);
 }
 
 }  // namespace
