@@ -539,6 +539,19 @@ def run_decode(A, model, shape, ids, K, B, T, args, stream, device, world):
     torch.cuda.synchronize()
     assert A.adadsf_sync_check(dws, stream) == A.OK, A.adadsf_last_error()
     ms = float(np.mean([e0.elapsed_time(e1) for e0, e1 in ev]))
+    # one more step, eager under the library's per-launch events: where a
+    # decode step's time goes
+    tok.copy_(new_ids[0])
+    torch.cuda.synchronize()
+    A.adadsf_profile_begin(64 * L + 16)
+    A.adadsf_decode_step(model, tok, h, cache, C_max, kept_out=kept, ws=dws, stream=stream)
+    recs = A.adadsf_profile_end(64 * L + 16)
+    prof = {}
+    for name, _, kms, _, by in recs:
+        a_ = prof.setdefault(name, {"launches": 0, "ms": 0.0, "bytes": 0.0})
+        a_["launches"] += 1
+        a_["ms"] += kms
+        a_["bytes"] += by
     es = 2 if shape.dtype == "bf16" else 4
     w_bytes = sum(v.numel() for lw in model.layers for v in lw.values()) * es
     # cached keys / values read by the timed steps: the prompt's kept tokens
@@ -552,8 +565,12 @@ def run_decode(A, model, shape, ids, K, B, T, args, stream, device, world):
             "prompt": T, "kept_fraction": float(kept_sum.sum()) / (n * L * B),
             "roofline": {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                          "frac": gbs / peaks["hbm_gbs"], "bytes_per_step": bytes_step},
+            "kernels_eager": {k: {"launches": v["launches"], "ms": v["ms"],
+                                  "gbs": v["bytes"] / (v["ms"] * 1e6) if v["ms"] > 0 else None}
+                              for k, v in sorted(prof.items(), key=lambda kv: -kv[1]["ms"])},
             "how": f"prefill of the batch at this line's K_l into a kept-token cache, then {n} decode steps "
-                   "(one token per sequence) replayed from one CUDA graph, CUDA events per step"}
+                   "(one token per sequence) replayed from one CUDA graph, CUDA events per step; "
+                   "kernels_eager: one more step run eagerly with events around every launch"}
 
 
 def host_threads() -> int:
