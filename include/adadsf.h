@@ -418,7 +418,8 @@ adadsf_status adadsf_sparse_model_forward(const adadsf_model_cfg *cfg, const ada
  * cache is full, sets the device error word (adadsf_sync_check reports
  * ADADSF_ERR_INVALID_ARG) and appends nothing. Prefill needs T < C_max and
  * the workspace of adadsf_model_workspace_size(cfg, B, T, K_host, 0); a
- * decode step adadsf_decode_workspace_size(cfg, B, C_max).
+ * decode step adadsf_decode_workspace_size(cfg, B, C_max), and at most 16
+ * query heads per key/value head (else ADADSF_ERR_UNSUPPORTED).
  * ---------------------------------------------------------------------- */
 size_t adadsf_kv_cache_size(const adadsf_model_cfg *cfg, int B, int C_max);
 adadsf_status adadsf_prefill(const adadsf_model_cfg *cfg, const adadsf_model_weights *w,

@@ -444,18 +444,19 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
                                c->rotary_dim, pos, T, lb.rope, dev),
                     "rotary")));
   if (dec) {
-    // a6 (decode): the new token against the layer's cached kept tokens and
-    // itself; then the kept tokens' keys and values join the cache
-    TRY(launch(dev, ADADSF_KERNEL_ATTENTION, false, 0,
-               (double)B * (q + 2.0 * kv) * es + 2.0 * B * kv * es * dec->C_max,
-               CALL(decode_attention(dt, lb.qkv, qkv_dim, c->n_heads, c->n_kv_heads, c->head_dim, dec->kc,
-                                     dec->vc, dec->lens, dec->C_max, B, dec->part_o, dec->part_ml, lb.attn, q,
-                                     dev),
-                    "decode attention")));
+    // a6 (decode): the kept new tokens' keys and values join the cache, then
+    // each new token attends to its layer's cached kept tokens (itself
+    // included when kept)
     TRY(launch(dev, ADADSF_KERNEL_KV_CACHE, false, 0, 4.0 * B * kv * es,
                CALL(kv_append(dt, lb.qkv, qkv_dim, q, kv, c->head_dim, B, dec->rows, dec->lens, dec->C_max,
                               dec->kc, dec->vc, dev),
                     "cache append")));
+    TRY(launch(dev, ADADSF_KERNEL_ATTENTION, false, 0,
+               (double)B * 2.0 * q * es + 2.0 * B * kv * es * dec->C_max,
+               CALL(decode_attention(dt, lb.qkv, qkv_dim, c->n_heads, c->n_kv_heads, c->head_dim, dec->kc,
+                                     dec->vc, dec->lens, dec->C_max, B, dec->part_o, dec->part_ml, lb.attn, q,
+                                     dev),
+                    "decode attention")));
   } else {
     // a6: causal attention among the kept tokens.
     TRY(launch(dev, ADADSF_KERNEL_ATTENTION, tc, 2.0 * B * c->n_heads * c->head_dim * (double)K * (K + 1),
@@ -1391,6 +1392,9 @@ adadsf_status adadsf_decode_step(const adadsf_model_cfg* cfg, const adadsf_model
                                  int B, void* hidden_out_dev, int32_t* kept_out_dev, void* cache_dev,
                                  size_t cache_bytes, int C_max, void* ws, size_t ws_bytes, void* stream) {
   TRY(check_cfg(cfg));
+  if (cfg->n_heads / cfg->n_kv_heads > 16)
+    return fail(ADADSF_ERR_UNSUPPORTED, "decode takes at most 16 query heads per key/value head, not %d",
+                cfg->n_heads / cfg->n_kv_heads);
   if (!w || !w->layers) return fail(ADADSF_ERR_INVALID_ARG, "model weights or layer array is NULL");
   if (B <= 0) return fail(ADADSF_ERR_INVALID_ARG, "B=%d must be positive", B);
   for (int l = 0; l < cfg->n_layers; ++l) TRY(check_layer_weights(cfg, &w->layers[l], true));

@@ -23,8 +23,12 @@
 namespace adadsf {
 namespace {
 
-constexpr int kDecThreads = 128;        // 4 warps per attention CTA
+constexpr int kDecThreads = 128;        // 4 warps per fp32 attention CTA
 constexpr int kMaxGroup = 16;           // query heads per key/value head
+constexpr int kDecTK = 64;              // keys per tile (split granularity, ring stage)
+constexpr int kDecStages = 3;           // ring stages of the bf16 kernel
+constexpr int kDecWarps = 4;            // consumer warps of the bf16 kernel, 16 keys of a tile each
+constexpr int kDecTcThreads = 32 * (kDecWarps + 1);
 
 // ---------------------------------------------------------------- prefill -> cache
 // K and V of the kept (packed) rows m = b K + j of one layer into the cache:
@@ -108,33 +112,38 @@ __global__ void decode_decide_kernel(const float* scores, const float* thr, cons
   if (kept_out) kept_out[b] = keep ? 1 : 0;
 }
 
-// Attention of the new token of sequence b, query heads g0 .. g0 + G - 1 of
-// key/value head h, over keys [lo, hi) of the n = lens[b] + 1 keys: the
-// cached kept tokens, then the token itself (from qkv). One CTA per (split,
-// kv head, sequence); each warp takes every 4th key with an online softmax
-// per query head; the CTA's partial (max, sum, output) per head goes to
-// part_ml / part_o for the combine step.
-template <typename T>
+// Attention of the new token of sequence b, query heads h G .. h G + G - 1
+// (G = Hq / Hkv) of key/value head h, over split s of the n = lens[b] cached
+// keys (the token's own key is already appended). The splits cover [0, n) in
+// whole tiles of kDecTK keys; a split's partial (row max in log2 units, sum,
+// unnormalised output) per query head goes to part_ml / part_o for the
+// combine step. Scores carry log2(e) / sqrt(hd), so the softmax runs on exp2.
+__device__ __forceinline__ void dec_split_range(int n, int nsplit, int s, int& lo, int& hi) {
+  const int per = ((n + nsplit - 1) / nsplit + kDecTK - 1) / kDecTK * kDecTK;
+  lo = min(n, s * per);
+  hi = min(n, lo + per);
+}
+
+// fp32 storage: CUDA cores, each warp of the CTA takes every 4th key with an
+// online softmax per query head.
 __global__ void __launch_bounds__(kDecThreads)
-    decode_attn_kernel(const T* qkv, int64_t ld, int q, int kvw, int Hq, int Hkv, int hd,
-                       const T* kc, const T* vc, const int32_t* lens, int C_max, int nsplit,
-                       float scale, float* part_o, float2* part_ml) {
+    decode_attn_f32_kernel(const float* qkv, int64_t ld, int Hq, int Hkv, int hd, const float* kc,
+                           const float* vc, const int32_t* lens, int C_max, int nsplit, float scale_log2,
+                           float* part_o, float2* part_ml) {
   pdl_trigger();
   pdl_wait();
   const int s = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int G = Hq / Hkv;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int per = hd / 32;                        // features per lane (2 or 4)
-  int len = lens[b];
-  if (len < 0) len = 0;
-  if (len > C_max) len = C_max;
-  const int n = len + 1;
-  const int lo = (int)((int64_t)s * n / nsplit), hi = (int)((int64_t)(s + 1) * n / nsplit);
-  const T* qrow = qkv + (int64_t)b * ld;
+  int n = lens[b];
+  n = n < 0 ? 0 : (n > C_max ? C_max : n);
+  int lo, hi;
+  dec_split_range(n, nsplit, s, lo, hi);
+  const float* qrow = qkv + (int64_t)b * ld;
   float qv[kMaxGroup][4];
   for (int g = 0; g < G; ++g)
-    for (int i = 0; i < per; ++i)
-      qv[g][i] = Elem<T>::to_f(qrow[(h * G + g) * hd + lane * per + i]) * scale;
+    for (int i = 0; i < per; ++i) qv[g][i] = qrow[(h * G + g) * hd + lane * per + i] * scale_log2;
   float mx[kMaxGroup], sm[kMaxGroup], acc[kMaxGroup][4];
   for (int g = 0; g < G; ++g) {
     mx[g] = -INFINITY;
@@ -143,20 +152,20 @@ __global__ void __launch_bounds__(kDecThreads)
   }
   const int64_t base = ((int64_t)b * Hkv + h) * C_max;
   for (int j = lo + warp; j < hi; j += 4) {
-    const T* kr = j < len ? kc + (base + j) * hd : qrow + q + h * hd;
-    const T* vr = j < len ? vc + (base + j) * hd : qrow + q + kvw + h * hd;
+    const float* kr = kc + (base + j) * hd;
+    const float* vr = vc + (base + j) * hd;
     float kf[4], vf[4];
     for (int i = 0; i < per; ++i) {
-      kf[i] = Elem<T>::to_f(kr[lane * per + i]);
-      vf[i] = Elem<T>::to_f(vr[lane * per + i]);
+      kf[i] = kr[lane * per + i];
+      vf[i] = vr[lane * per + i];
     }
     for (int g = 0; g < G; ++g) {
       float dot = 0.f;
       for (int i = 0; i < per; ++i) dot = fmaf(qv[g][i], kf[i], dot);
       dot = warp_sum(dot);
       const float mnew = fmaxf(mx[g], dot);
-      const float corr = expf(mx[g] - mnew);
-      const float pj = expf(dot - mnew);
+      const float corr = exp2f(mx[g] - mnew);
+      const float pj = exp2f(dot - mnew);
       sm[g] = sm[g] * corr + pj;
       for (int i = 0; i < per; ++i) acc[g][i] = fmaf(acc[g][i], corr, pj * vf[i]);
       mx[g] = mnew;
@@ -180,7 +189,7 @@ __global__ void __launch_bounds__(kDecThreads)
     float l = 0.f, o = 0.f;
     if (m > -INFINITY) {
       for (int w = 0; w < 4; ++w) {
-        const float c = expf(s_ml[w][g][0] - m);
+        const float c = exp2f(s_ml[w][g][0] - m);
         l += s_ml[w][g][1] * c;
         o += s_o[w][g][e] * c;
       }
@@ -191,7 +200,248 @@ __global__ void __launch_bounds__(kDecThreads)
   }
 }
 
-// out[b][head] = sum_s e^(m_s - m) o_s / sum_s e^(m_s - m) l_s over the splits.
+// bf16 storage: tensor cores (warp-level mma.sync m16n8k16, bf16 in, fp32
+// accumulate). The G query heads of the group are the 16 rows of the A
+// operand (rows >= G are zero), so one key tile costs the same whatever G.
+// Warp 4 streams the key/value tiles of the split through a ring of
+// kDecStages stages with 2-D TMA copies (128-byte swizzle, 64 features per
+// box); warps 0..3 each take 16 keys of a tile:
+//   S (16 x 16)  = Q (16 x HD) . K^T           (ldmatrix from the swizzled tile)
+//   online softmax per row (exp2; the 4 lanes of a quad share a row)
+//   O (16 x HD) += P (16 x 16, bf16) . V (16 x HD)   (ldmatrix.trans)
+// and the four warps' (max, sum, O) merge in shared memory at the end.
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t (&r)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+// D += A . B for one m16n8k16 tile (A row-major 16 x 16, B column-major 16 x 8).
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                               uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+// Byte offset of (row, col) in a ring tile: boxes of 64 features (128 bytes)
+// side by side, each kDecTK rows of 128 bytes with the 16-byte chunks of a
+// row permuted by XOR with (row mod 8), as the TMA 128-byte swizzle writes them.
+__device__ __forceinline__ uint32_t dec_swz(int row, int col) {
+  return (uint32_t)((col >> 6) * (kDecTK * 128) + row * 128 + ((((col & 63) >> 3) ^ (row & 7)) << 4));
+}
+__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
+
+template <int HD>
+struct DecTc {
+  static constexpr int TILE = HD / 64 * kDecTK * 128;     // K (or V) of one stage, bytes
+  static constexpr int STAGE = 2 * TILE;
+  static constexpr int RING = kDecStages * STAGE;
+  static constexpr int OLD = HD + 8;                      // merge row stride (floats), padded
+  static constexpr int MERGE = kDecWarps * 16 * (OLD + 2) * 4;
+  static_assert(MERGE <= RING, "the merge area reuses the ring");
+  static constexpr int SMEM = RING + 1024;                // + alignment slack
+};
+
+template <int HD>
+__global__ void __launch_bounds__(kDecTcThreads)
+    decode_attn_tc_kernel(const __grid_constant__ CUtensorMap tk, const __grid_constant__ CUtensorMap tv,
+                          const bf16* qkv, int64_t ld, int Hq, int Hkv, const int32_t* lens, int C_max,
+                          int nsplit, float scale_log2, float* part_o, float2* part_ml, int* err,
+                          unsigned long long timeout_ns) {
+  using C = DecTc<HD>;
+  extern __shared__ __align__(1024) uint8_t dsm[];
+  __shared__ __align__(8) uint64_t bars[2 * kDecStages];
+  __shared__ int abort_s;
+  const uint32_t ring = (smem_u32(dsm) + 1023u) & ~1023u;
+  uint8_t* ring_p = dsm + (ring - smem_u32(dsm));
+  const uint32_t full0 = smem_u32(&bars[0]), empty0 = smem_u32(&bars[kDecStages]);
+  volatile int* abort_flag = &abort_s;
+  const int s = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int G = Hq / Hkv;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kDecStages; ++i) {
+      mbar_init(full0 + 8 * i, 1);
+      mbar_init(empty0 + 8 * i, kDecWarps);
+    }
+    abort_s = 0;
+    fence_barrier_init();
+  }
+  if (warp == kDecWarps && lane == 0) {
+    tma_prefetch_desc(&tk);
+    tma_prefetch_desc(&tv);
+  }
+  __syncthreads();
+  pdl_trigger();
+  pdl_wait();
+  int n = lens[b];
+  n = n < 0 ? 0 : (n > C_max ? C_max : n);
+  int lo, hi;
+  dec_split_range(n, nsplit, s, lo, hi);
+  const int ntiles = (hi - lo + kDecTK - 1) / kDecTK;
+  const int row0 = (b * Hkv + h) * C_max + lo;            // first key's row in the layer's cache
+
+  const int gid = lane >> 2, tig = lane & 3;
+  float o[HD / 8][4];
+  float m_r[2] = {-INFINITY, -INFINITY}, l_r[2] = {0.f, 0.f};   // rows gid, gid + 8
+#pragma unroll
+  for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+
+  if (warp == kDecWarps) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int t = 0;
+      for (; t < ntiles; ++t) {
+        const int st = t % kDecStages;
+        if (!mbar_wait_bounded(empty0 + 8 * st, ((t / kDecStages) & 1) ^ 1, abort_flag, err, timeout_ns)) break;
+        const uint32_t fb = full0 + 8 * st;
+        mbar_arrive_expect_tx(fb, C::STAGE);
+        const uint32_t dk = ring + st * C::STAGE;
+#pragma unroll
+        for (int x = 0; x < HD / 64; ++x) {
+          tma_load_2d(dk + x * kDecTK * 128, &tk, x * 64, row0 + t * kDecTK, fb);
+          tma_load_2d(dk + C::TILE + x * kDecTK * 128, &tv, x * 64, row0 + t * kDecTK, fb);
+        }
+      }
+      // drain: the copies issued last into each stage have landed
+      for (int st = 0; st < kDecStages && st < t; ++st) {
+        const int last = st + ((t - 1 - st) / kDecStages) * kDecStages;
+        mbar_wait_drain(full0 + 8 * st, (uint32_t)((last / kDecStages) & 1), timeout_ns);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ consumers
+    // Q of the group as A fragments (rows g >= G zero), once
+    uint32_t qa[HD / 16][4];
+    const bf16* qrow = qkv + (int64_t)b * ld + (int64_t)h * G * HD;
+    const bool r0 = gid < G, r1 = gid + 8 < G;
+#pragma unroll
+    for (int ks = 0; ks < HD / 16; ++ks) {
+      const int c = ks * 16 + tig * 2;
+      qa[ks][0] = r0 ? *reinterpret_cast<const uint32_t*>(qrow + gid * HD + c) : 0u;
+      qa[ks][1] = r1 ? *reinterpret_cast<const uint32_t*>(qrow + (gid + 8) * HD + c) : 0u;
+      qa[ks][2] = r0 ? *reinterpret_cast<const uint32_t*>(qrow + gid * HD + c + 8) : 0u;
+      qa[ks][3] = r1 ? *reinterpret_cast<const uint32_t*>(qrow + (gid + 8) * HD + c + 8) : 0u;
+    }
+    const int mi = lane >> 3, mr = lane & 7;   // ldmatrix: this lane's matrix and row
+    for (int t = 0; t < ntiles; ++t) {
+      const int st = t % kDecStages;
+      const bool ok = mbar_wait_bounded(full0 + 8 * st, (t / kDecStages) & 1, abort_flag, err, timeout_ns);
+      if (!__all_sync(0xffffffffu, ok)) break;
+      const uint32_t kt = ring + st * C::STAGE, vt = kt + C::TILE;
+      const int kw = warp * 16;                             // this warp's keys within the tile
+      float sc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+#pragma unroll
+      for (int ks = 0; ks < HD / 16; ++ks) {
+        uint32_t kb[4];
+        ldsm_x4(kt + dec_swz(kw + (mi >> 1) * 8 + mr, ks * 16 + (mi & 1) * 8), kb);
+        mma_bf16_16816(sc[0], qa[ks], kb[0], kb[1]);
+        mma_bf16_16816(sc[1], qa[ks], kb[2], kb[3]);
+      }
+      // online softmax over the warp's 16 keys; key j0 + 8 nt + 2 tig + e
+      const int j0 = lo + t * kDecTK + kw;
+      float tmax[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const bool valid = j0 + nt * 8 + tig * 2 + (e & 1) < hi;
+          sc[nt][e] = valid ? sc[nt][e] * scale_log2 : -INFINITY;
+          tmax[e >> 1] = fmaxf(tmax[e >> 1], sc[nt][e]);
+        }
+      float corr[2], base[2];
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        tmax[r] = fmaxf(tmax[r], __shfl_xor_sync(0xffffffffu, tmax[r], 1));
+        tmax[r] = fmaxf(tmax[r], __shfl_xor_sync(0xffffffffu, tmax[r], 2));
+        const float mn = fmaxf(m_r[r], tmax[r]);
+        base[r] = mn == -INFINITY ? 0.f : mn;
+        corr[r] = exp2f(m_r[r] - base[r]);
+        m_r[r] = mn;
+      }
+      uint32_t pa[4];
+      float psum[2] = {0.f, 0.f};
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const uint32_t pk = pack_bf16x2(exp2f(sc[nt][2 * r] - base[r]), exp2f(sc[nt][2 * r + 1] - base[r]));
+          pa[nt * 2 + r] = pk;
+          psum[r] += bf16_lo(pk) + bf16_hi(pk);
+        }
+#pragma unroll
+      for (int r = 0; r < 2; ++r) l_r[r] = l_r[r] * corr[r] + psum[r];
+#pragma unroll
+      for (int i = 0; i < HD / 8; ++i) {
+        o[i][0] *= corr[0];
+        o[i][1] *= corr[0];
+        o[i][2] *= corr[1];
+        o[i][3] *= corr[1];
+      }
+#pragma unroll
+      for (int np = 0; np < HD / 16; ++np) {
+        uint32_t vb[4];
+        ldsm_x4_t(vt + dec_swz(kw + (mi & 1) * 8 + mr, np * 16 + (mi >> 1) * 8), vb);
+        mma_bf16_16816(o[2 * np], pa, vb[0], vb[1]);
+        mma_bf16_16816(o[2 * np + 1], pa, vb[2], vb[3]);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(empty0 + 8 * st);
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      l_r[r] += __shfl_xor_sync(0xffffffffu, l_r[r], 1);
+      l_r[r] += __shfl_xor_sync(0xffffffffu, l_r[r], 2);
+    }
+  }
+  __syncthreads();   // the ring is drained and read: its memory takes the merge
+  float* mo = reinterpret_cast<float*>(ring_p);                     // [warp][16][OLD]
+  float* mml = mo + kDecWarps * 16 * C::OLD;                        // [warp][16][2]
+  if (warp < kDecWarps) {
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const int row = gid + 8 * r;
+      if (row < G) {
+        float* dst = mo + (warp * 16 + row) * C::OLD + tig * 2;
+#pragma unroll
+        for (int i = 0; i < HD / 8; ++i) *reinterpret_cast<float2*>(dst + i * 8) = make_float2(o[i][2 * r], o[i][2 * r + 1]);
+        if (tig == 0) {
+          mml[(warp * 16 + row) * 2] = m_r[r];
+          mml[(warp * 16 + row) * 2 + 1] = l_r[r];
+        }
+      }
+    }
+  }
+  __syncthreads();
+  for (int k = threadIdx.x; k < G * HD; k += kDecTcThreads) {
+    const int g = k / HD, e = k % HD;
+    float m = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < kDecWarps; ++w) m = fmaxf(m, mml[(w * 16 + g) * 2]);
+    float l = 0.f, ov = 0.f;
+    if (m > -INFINITY) {
+#pragma unroll
+      for (int w = 0; w < kDecWarps; ++w) {
+        const float c = exp2f(mml[(w * 16 + g) * 2] - m);
+        l += mml[(w * 16 + g) * 2 + 1] * c;
+        ov += mo[(w * 16 + g) * C::OLD + e] * c;
+      }
+    }
+    const int64_t slot = ((int64_t)b * Hq + h * G + g) * nsplit + s;
+    part_o[slot * HD + e] = ov;
+    if (e == 0) part_ml[slot] = make_float2(m, l);
+  }
+}
+
+// out[b][head] = sum_s 2^(m_s - m) o_s / sum_s 2^(m_s - m) l_s over the
+// splits; a head with no key at all (an empty cache) gets zeros.
 template <typename T>
 __global__ void decode_combine_kernel(const float* part_o, const float2* part_ml, int Hq, int hd,
                                       int nsplit, T* out, int64_t ld_out) {
@@ -206,15 +456,16 @@ __global__ void decode_combine_kernel(const float* part_o, const float2* part_ml
     for (int s = 0; s < nsplit; ++s) {
       const float2 ml = part_ml[slot0 + s];
       if (ml.x == -INFINITY) continue;
-      const float c = expf(ml.x - m);
+      const float c = exp2f(ml.x - m);
       l += ml.y * c;
       o += part_o[(slot0 + s) * hd + e] * c;
     }
-    out[(int64_t)b * ld_out + hq * hd + e] = Elem<T>::from_f(o / l);
+    out[(int64_t)b * ld_out + hq * hd + e] = Elem<T>::from_f(l > 0.f ? o / l : 0.f);
   }
 }
 
-// The kept new tokens' keys and values join the layer's cache.
+// The kept new tokens' keys and values join the layer's cache (before the
+// step's attention, which then reads every key from the cache).
 template <typename T>
 __global__ void kv_append_kernel(const T* qkv, int64_t ld, int q, int kvw, int hd, int B,
                                  const int32_t* rows, int32_t* lens, int C_max, T* kc, T* vc,
@@ -249,9 +500,9 @@ __global__ void decode_advance_kernel(int32_t* hdr) {
 
 // ---------------------------------------------------------------- host side
 int decode_splits(int B, int Hkv, int C_max, int num_sms) {
-  const int units = B * Hkv;
-  int s = (2 * num_sms + units - 1) / units;
-  const int max_s = (C_max + 63) / 64;             // at least 64 keys a split
+  // two CTAs of the bf16 kernel per SM in one wave, at least one tile a split
+  int s = 2 * num_sms / (B * Hkv);
+  const int max_s = (C_max + kDecTK - 1) / kDecTK;
   if (s > max_s) s = max_s;
   if (s > 64) s = 64;
   return s < 1 ? 1 : s;
@@ -286,24 +537,47 @@ cudaError_t decode_decide(const float* scores, const float* thr, const int32_t* 
                     C_max, rows, pos, kept_out, dev.err);
 }
 
+template <int HD>
+static cudaError_t launch_decode_tc(const CUtensorMap& tk, const CUtensorMap& tv, const bf16* qkv, int64_t ld,
+                                    int Hq, int Hkv, const int32_t* lens, int C_max, int B, int ns,
+                                    float scale_log2, float* part_o, float2* part_ml, const Dev& dev) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(decode_attn_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         DecTc<HD>::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  return launch_pdl(decode_attn_tc_kernel<HD>, dim3(ns, Hkv, B), dim3(kDecTcThreads), (size_t)DecTc<HD>::SMEM,
+                    dev.stream, tk, tv, qkv, ld, Hq, Hkv, lens, C_max, ns, scale_log2, part_o, part_ml, dev.err,
+                    kWaitTimeoutNs);
+}
+
 cudaError_t decode_attention(int dtype, const void* qkv, int64_t ld, int Hq, int Hkv, int hd, const void* kc,
                              const void* vc, const int32_t* lens, int C_max, int B, float* part_o,
                              float2* part_ml, void* out, int64_t ld_out, const Dev& dev) {
   if (B <= 0) return cudaSuccess;
   if (Hq % Hkv != 0 || Hq / Hkv > kMaxGroup || (hd != 64 && hd != 128)) return cudaErrorInvalidValue;
-  const int q = Hq * hd, kvw = Hkv * hd;
   const int ns = decode_splits(B, Hkv, C_max, dev.num_sms);
-  const float scale = 1.f / sqrtf((float)hd);
-  const dim3 grid(ns, Hkv, B);
+  const float scale_log2 = 1.4426950408889634f / sqrtf((float)hd);   // log2(e) / sqrt(hd)
   cudaError_t e;
-  if (dtype == kBF16)
-    e = launch_pdl(decode_attn_kernel<bf16>, grid, dim3(kDecThreads), 0, dev.stream,
-                   static_cast<const bf16*>(qkv), ld, q, kvw, Hq, Hkv, hd, static_cast<const bf16*>(kc),
-                   static_cast<const bf16*>(vc), lens, C_max, ns, scale, part_o, part_ml);
-  else
-    e = launch_pdl(decode_attn_kernel<float>, grid, dim3(kDecThreads), 0, dev.stream,
-                   static_cast<const float*>(qkv), ld, q, kvw, Hq, Hkv, hd, static_cast<const float*>(kc),
-                   static_cast<const float*>(vc), lens, C_max, ns, scale, part_o, part_ml);
+  if (dtype == kBF16) {
+    // the layer's keys (values) as one [B Hkv C_max, hd] matrix; a tile's
+    // first row must fit the copy's 32-bit coordinate
+    const int64_t rows = (int64_t)B * Hkv * C_max;
+    if (rows + kDecTK > INT32_MAX) return cudaErrorInvalidValue;
+    CUtensorMap tk, tv;
+    if (!make_tmap_bf16(&tk, kc, (uint64_t)rows, (uint64_t)hd, (uint64_t)hd, 64, kDecTK) ||
+        !make_tmap_bf16(&tv, vc, (uint64_t)rows, (uint64_t)hd, (uint64_t)hd, 64, kDecTK))
+      return cudaErrorInvalidValue;
+    const bf16* q = static_cast<const bf16*>(qkv);
+    e = hd == 128 ? launch_decode_tc<128>(tk, tv, q, ld, Hq, Hkv, lens, C_max, B, ns, scale_log2, part_o, part_ml, dev)
+                  : launch_decode_tc<64>(tk, tv, q, ld, Hq, Hkv, lens, C_max, B, ns, scale_log2, part_o, part_ml, dev);
+  } else {
+    e = launch_pdl(decode_attn_f32_kernel, dim3(ns, Hkv, B), dim3(kDecThreads), 0, dev.stream,
+                   static_cast<const float*>(qkv), ld, Hq, Hkv, hd, static_cast<const float*>(kc),
+                   static_cast<const float*>(vc), lens, C_max, ns, scale_log2, part_o, part_ml);
+  }
   if (e != cudaSuccess) return e;
   if (dtype == kBF16)
     return launch_pdl(decode_combine_kernel<bf16>, dim3(Hq, B), dim3(128), 0, dev.stream, part_o, part_ml, Hq,

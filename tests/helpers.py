@@ -18,6 +18,11 @@ F32_TOL = 1e-4      # same, fp32 storage
 # 3-4% of rms (tests/test_precision_cpu.py). 5e-2 bounds that with margin;
 # fp32 storage keeps F32_TOL element-wise.
 BF16_ELEM_TOL = 5e-2
+# The same bound for a two-layer model at the Qwen2.5-7B attention geometry
+# (28 query heads on 4 key/value heads, 700-token prompt) through the final
+# norm: the fp64 emulation of the same storage points gives 6.6e-2 there
+# (tests/test_precision_cpu.py), so its tests take 1e-1.
+BF16_DEEP_ELEM_TOL = 1e-1
 
 
 def tdtype(shape):

@@ -28,13 +28,22 @@ def A():
 QWEN_SMALL = S.QWEN25_1_5B.replace(d=1024, n_heads=8, n_kv_heads=2, ffn=1536, n_layers=3, vocab=500)
 NEOX_SMALL = S.PYTHIA_160M.replace(n_layers=3, vocab=500)
 NEOX_F32 = S.PYTHIA_70M.replace(n_layers=2, vocab=500)
+# the Qwen2.5-7B attention geometry (28 query heads on 4 key/value heads,
+# head_dim 128) with a narrow MLP: caches of several hundred keys spread over
+# several splits, some of them empty
+QWEN7_ATTN = S.QWEN25_7B.replace(ffn=2048, n_layers=2, vocab=500)
+# 16 query heads on one key/value head, head_dim 64: every row of the tensor
+# core tile is a real head
+QWEN_G16 = QWEN_SMALL.replace(n_heads=16, n_kv_heads=1, head_dim=64, rotary_dim=64, n_layers=2)
 
 CASES = [
-    # (shape, B, T0, K per layer, steps, C_max, gated)
-    (NEOX_SMALL, 3, 64, [64, 20, 40], 5, 80, False),
-    (QWEN_SMALL, 2, 100, [50, 100, 0], 4, 128, False),
-    (QWEN_SMALL, 2, 96, [48, 30, 96], 3, 100, True),
-    (NEOX_F32, 2, 40, [20, 40], 4, 48, False),
+    # (shape, B, T0, K per layer, steps, C_max, gated, element-wise tolerance)
+    (NEOX_SMALL, 3, 64, [64, 20, 40], 5, 80, False, None),
+    (QWEN_SMALL, 2, 100, [50, 100, 0], 4, 128, False, None),
+    (QWEN_SMALL, 2, 96, [48, 30, 96], 3, 100, True, None),
+    (NEOX_F32, 2, 40, [20, 40], 4, 48, False, None),
+    (QWEN7_ATTN, 2, 700, [350, 700], 3, 720, False, H.BF16_DEEP_ELEM_TOL),
+    (QWEN_G16, 3, 200, [131, 64], 3, 216, True, None),
 ]
 
 
@@ -47,8 +56,8 @@ def _cache_counts(A, cache, L, B):
     return lens, thr
 
 
-@pytest.mark.parametrize("shape,B,T0,K,steps,C_max,gated", CASES)
-def test_prefill_then_decode(A, shape, B, T0, K, steps, C_max, gated):
+@pytest.mark.parametrize("shape,B,T0,K,steps,C_max,gated,etol", CASES)
+def test_prefill_then_decode(A, shape, B, T0, K, steps, C_max, gated, etol):
     L = shape.n_layers
     td = H.tdtype(shape)
     flags = A.FLAG_GATE_SIGMOID if gated else 0
@@ -71,7 +80,7 @@ def test_prefill_then_decode(A, shape, B, T0, K, steps, C_max, gated):
     W64 = [H.f64(w) for w in hostL]
     E64 = H.f64(extra)
     ref, st = O.sparse_prefill(ids[:, :T0], E64, W64, p, K, idx_force=kept_sets)
-    H.assert_close(H.to_np(hidden), ref, H.tol(shape), "prefill")
+    H.assert_close(H.to_np(hidden), ref, H.tol(shape), "prefill", etol)
     lens, thr = _cache_counts(A, cache, L, B)
     assert lens.tolist() == [[k] * B for k in K]
     thr_ref = np.array(st["thr"])
@@ -93,7 +102,7 @@ def test_prefill_then_decode(A, shape, B, T0, K, steps, C_max, gated):
         margin = np.abs(sref - thr_ref) > 1e-3 * np.maximum(1.0, np.abs(thr_ref))
         assert (kg[margin] == kown[margin]).all(), (step, kg, kown)
         n_checked += int(margin.sum())
-        H.assert_close(H.to_np(h), href, H.tol(shape), f"decode step {step}")
+        H.assert_close(H.to_np(h), href, H.tol(shape), f"decode step {step}", etol)
         counts += kg
         lens, _ = _cache_counts(A, cache, L, B)
         assert (lens == counts).all()
@@ -145,3 +154,41 @@ def test_decode_step_in_a_cuda_graph(A):
         assert A.adadsf_sync_check(dws) == A.OK
         outs.append(torch.stack(res))
     assert torch.equal(outs[0], outs[1])
+
+
+def test_decode_at_bench_geometry(A):
+    """A decode step at the geometry the throughput measurement replays
+    (16 sequences, a 4096-token prompt, the Qwen2.5-7B attention shape, half
+    the prompt kept, the same cache length and split count), one layer with a
+    narrow MLP. Sequences are independent, so the oracle runs on a sample of
+    two of them, with the GPU's kept sets and decisions."""
+    shape = QWEN7_ATTN.replace(n_layers=1)
+    B, T0, steps = 16, 4096, 2
+    C_max, K = T0 + 32 + 8, [2048]
+    td = H.tdtype(shape)
+    hostL = [H.host_layer(shape, 31, 0)]
+    extra = H.host_extra(shape, 31)
+    model = A.DeviceModel(A.make_cfg(shape), [A.to_device(w, td) for w in hostL], A.to_device(extra, td))
+    ids = S.token_ids(32, B, T0 + steps, shape.vocab)
+    ids_d = torch.from_numpy(ids).cuda()
+    cache = A.kv_cache(model.cfg, B, C_max)
+    idx = torch.full((B * K[0],), -1, dtype=torch.int32, device="cuda")
+    ws = A.workspace(A.adadsf_model_workspace_size(model.cfg, B, T0, K, False))
+    A.adadsf_prefill(model, ids_d[:, :T0].contiguous(), K, torch.empty((B, T0, shape.d), dtype=td, device="cuda"),
+                     cache, C_max, idx_out=idx, ws=ws)
+    assert A.adadsf_sync_check(ws) == A.OK
+    del ws
+    sample = [0, B - 1]
+    kept_set = idx.cpu().numpy().reshape(B, K[0])[sample]
+    W64, E64 = [H.f64(hostL[0])], H.f64(extra)
+    p = O.params_of(shape)
+    _, st = O.sparse_prefill(ids[sample, :T0], E64, W64, p, K, idx_force=[kept_set])
+    dws = A.workspace(A.adadsf_decode_workspace_size(model.cfg, B, C_max))
+    for step in range(steps):
+        h = torch.empty((B, shape.d), dtype=td, device="cuda")
+        kept = torch.full((1, B), -1, dtype=torch.int32, device="cuda")
+        A.adadsf_decode_step(model, ids_d[:, T0 + step].contiguous(), h, cache, C_max, kept_out=kept, ws=dws)
+        assert A.adadsf_sync_check(dws) == A.OK
+        kg = kept.cpu().numpy().astype(bool)[:, sample]
+        href, _, _ = O.decode_step(ids[sample, T0 + step], E64, W64, p, st, kept_force=kg)
+        H.assert_close(H.to_np(h)[sample], href, H.tol(shape), f"decode step {step}", H.BF16_DEEP_ELEM_TOL)

@@ -8,7 +8,10 @@ fp64 with exactly those tensors rounded to bf16, on a shortened sequence, and
 measures the error against the plain fp64 oracle. The per-tensor error stays
 far inside the 2e-2 tolerance, while the largest element-wise error (each
 element against max(|r|, rms(r))) lands at a few percent: bf16 storage alone
-puts it above 2e-2 and below the 5e-2 element-wise bound the GPU tests use."""
+puts it above 2e-2 and below the 5e-2 element-wise bound the GPU tests use.
+A two-layer model at the Qwen2.5-7B attention geometry with a 700-token
+prompt, through the final norm, lands at 6.6e-2 element-wise: the bound its
+GPU tests take is 1e-1."""
 import numpy as np
 
 from oracle import adadsf_oracle as O
@@ -51,3 +54,27 @@ def test_bf16_storage_error_at_qwen7b_layer_shape():
     assert H.max_rel(got, kept) < H.BF16_TOL / 2
     assert 1e-3 < H.rel_rms(got, kept) < 1e-2
     assert H.BF16_TOL < H.elem_rel(got, kept) < H.BF16_ELEM_TOL
+
+
+def test_bf16_storage_error_two_layer_model_at_qwen7b_attention_shape():
+    """The two-layer case of the decode tests (seeds, prompt and kept counts
+    as there): embedding, two sparse layers with bf16 storage, the final norm
+    rounded to bf16, against the fp64 oracle model."""
+    shape = S.QWEN25_7B.replace(ffn=2048, n_layers=2, vocab=500)
+    B, T0, K = 2, 700, [350, 700]
+    W = [H.f64(H.host_layer(shape, 13, l)) for l in range(2)]
+    E = H.f64(H.host_extra(shape, 13))
+    ids = S.token_ids(14, B, T0 + 3, shape.vocab)[:, :T0]
+    p = O.params_of(shape)
+    ref = O.sparse_model_forward(ids, E, W, p, K)
+    ref = ref[0] if isinstance(ref, tuple) else ref
+    x = E["embed"][ids]
+    for l in range(2):
+        nxt = x.copy()
+        for b in range(B):
+            sel = O.topk_keep(O.router_scores(x[b], W[l]), K[l])
+            nxt[b, sel] = _layer_with_bf16_storage(x[b, sel], sel, W[l], p)
+        x = nxt
+    got = _r16(O.final_norm(x, E, p))
+    assert H.max_rel(got, ref) < H.BF16_TOL
+    assert H.BF16_ELEM_TOL < H.elem_rel(got, ref) < H.BF16_DEEP_ELEM_TOL
