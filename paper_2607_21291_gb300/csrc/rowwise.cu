@@ -188,10 +188,32 @@ constexpr int kRowSlots = 16;                      // ring slots (two rows per c
 static_assert(kRowSlots % kRowWarps == 0, "a slot is always consumed by the same warp");
 constexpr int kMaxRowBytes = 8192;   // d <= 4096 (bf16) or 2048 (fp32)
 
+// A 16-byte vector as V / 2 pairs of floats, and back (round to nearest even).
+__device__ __forceinline__ void unpack_pairs(const uint4& u, float2* p, bf16) {
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) p[i] = make_float2(__uint_as_float(w[i] << 16), __uint_as_float(w[i] & 0xffff0000u));
+}
+__device__ __forceinline__ void unpack_pairs(const uint4& u, float2* p, float) {
+  p[0] = make_float2(__uint_as_float(u.x), __uint_as_float(u.y));
+  p[1] = make_float2(__uint_as_float(u.z), __uint_as_float(u.w));
+}
+__device__ __forceinline__ uint4 pack_pairs(const float2* p, bf16) {
+  return make_uint4(pack_bf16x2(p[0].x, p[0].y), pack_bf16x2(p[1].x, p[1].y), pack_bf16x2(p[2].x, p[2].y),
+                    pack_bf16x2(p[3].x, p[3].y));
+}
+__device__ __forceinline__ uint4 pack_pairs(const float2* p, float) {
+  return make_uint4(__float_as_uint(p[0].x), __float_as_uint(p[0].y), __float_as_uint(p[1].x),
+                    __float_as_uint(p[1].y));
+}
+
 // out1[m] = norm(x[row(m)]; g1, b1), out2[m] = norm(x[row(m)]; g2, b2) for the
 // block's contiguous share of m. Shared memory: the staged parameters
 // ([4][d]), then the ring (kRowSlots rows of d), then 2 kRowSlots mbarriers.
-template <typename T, bool RMS>
+// NCH: the 16-byte vectors of a row per lane, ceil(d / (32 V)) rounded up to
+// a compiled bucket: a consumer warp holds its row in registers (one shared-
+// memory read of the slot) and works on pairs of floats.
+template <typename T, bool RMS, int NCH>
 __global__ void __launch_bounds__(kRowThreads)
     gather_norm_tma_kernel(const T* x, const int32_t* rows, int64_t M, int d, const T* g1,
                            const T* b1, const T* g2, const T* b2, float eps, T* out1, T* out2,
@@ -259,7 +281,9 @@ __global__ void __launch_bounds__(kRowThreads)
       }
   } else {
     // ------------------------------------------------------------ consumers
+    constexpr int P = V / 2;                    // float pairs per vector
     const int nv = d / V;
+    const float inv_d = 1.f / (float)d;
     for (int64_t j = warp; j < n; j += kRowWarps) {
       const int s = (int)(j % kRowSlots);
       int ok = 0;
@@ -267,47 +291,70 @@ __global__ void __launch_bounds__(kRowThreads)
         ok = mbar_wait_bounded(full0 + 8 * s, (uint32_t)((j / kRowSlots) & 1), abort_v, err, timeout_ns);
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
-      const T* xr = reinterpret_cast<const T*>(ring + (size_t)s * row_bytes);
-      float sum = 0.f;
-      for (int ci = lane; ci < nv; ci += 32) {
-        float f[V];
-        load_vec(xr + ci * V, f);
+      const uint4* xr = reinterpret_cast<const uint4*>(ring + (size_t)s * row_bytes);
+      uint4 raw[NCH];
 #pragma unroll
-        for (int k = 0; k < V; ++k) sum += RMS ? f[k] * f[k] : f[k];
+      for (int c = 0; c < NCH; ++c)
+        if (c * 32 + lane < nv) raw[c] = xr[c * 32 + lane];
+      // statistics over pairs (two partial sums), then over the warp
+      float2 acc = make_float2(0.f, 0.f);
+#pragma unroll
+      for (int c = 0; c < NCH; ++c) {
+        if (c * 32 + lane < nv) {
+          float2 f[P];
+          unpack_pairs(raw[c], f, T());
+#pragma unroll
+          for (int k = 0; k < P; ++k) acc = RMS ? __ffma2_rn(f[k], f[k], acc) : __fadd2_rn(acc, f[k]);
+        }
       }
+      // every value of the slot has been used: it may be refilled
+      __syncwarp();
+      if (lane == 0) mbar_arrive(empty0 + 8 * s);
       float mean = 0.f, rstd;
       if (RMS) {
-        rstd = 1.f / sqrtf(warp_sum(sum) / d + eps);
+        rstd = 1.f / sqrtf(warp_sum(acc.x + acc.y) * inv_d + eps);
       } else {
-        mean = warp_sum(sum) / d;
-        float q = 0.f;
-        for (int ci = lane; ci < nv; ci += 32) {
-          float f[V];
-          load_vec(xr + ci * V, f);
+        mean = warp_sum(acc.x + acc.y) * inv_d;
+        const float2 negm = make_float2(-mean, -mean);
+        float2 q = make_float2(0.f, 0.f);
 #pragma unroll
-          for (int k = 0; k < V; ++k) q += (f[k] - mean) * (f[k] - mean);
+        for (int c = 0; c < NCH; ++c) {
+          if (c * 32 + lane < nv) {
+            float2 f[P];
+            unpack_pairs(raw[c], f, T());
+#pragma unroll
+            for (int k = 0; k < P; ++k) {
+              const float2 t = __fadd2_rn(f[k], negm);
+              q = __ffma2_rn(t, t, q);
+            }
+          }
         }
-        rstd = 1.f / sqrtf(warp_sum(q) / d + eps);
+        rstd = 1.f / sqrtf(warp_sum(q.x + q.y) * inv_d + eps);
       }
+      const float2 negm = make_float2(-mean, -mean), rs = make_float2(rstd, rstd);
       const int64_t m = lo + j;
-      for (int ci = lane; ci < nv; ci += 32) {
-        float f[V], g[V], bb[V], o[V];
-        load_vec(xr + ci * V, f);
-        load_vec(sp + ci * V, g);
-        if (!RMS) load_vec(sp + d + ci * V, bb);
 #pragma unroll
-        for (int k = 0; k < V; ++k) o[k] = (f[k] - mean) * rstd * g[k] + (RMS ? 0.f : bb[k]);
-        store_vec(out1 + m * d + ci * V, o);
-        if (out2) {
-          load_vec(sp + 2 * d + ci * V, g);
-          if (!RMS) load_vec(sp + 3 * d + ci * V, bb);
+      for (int c = 0; c < NCH; ++c) {
+        const int ci = c * 32 + lane;
+        if (ci < nv) {
+          float2 f[P], g[P], bb[P], o[P];
+          unpack_pairs(raw[c], f, T());
 #pragma unroll
-          for (int k = 0; k < V; ++k) o[k] = (f[k] - mean) * rstd * g[k] + (RMS ? 0.f : bb[k]);
-          store_vec(out2 + m * d + ci * V, o);
+          for (int k = 0; k < P; ++k) f[k] = __fmul2_rn(RMS ? f[k] : __fadd2_rn(f[k], negm), rs);
+          unpack_pairs(reinterpret_cast<const uint4*>(sp)[ci], g, T());
+          if (!RMS) unpack_pairs(reinterpret_cast<const uint4*>(sp + d)[ci], bb, T());
+#pragma unroll
+          for (int k = 0; k < P; ++k) o[k] = RMS ? __fmul2_rn(f[k], g[k]) : __ffma2_rn(f[k], g[k], bb[k]);
+          reinterpret_cast<uint4*>(out1 + m * d)[ci] = pack_pairs(o, T());
+          if (out2) {
+            unpack_pairs(reinterpret_cast<const uint4*>(sp + 2 * d)[ci], g, T());
+            if (!RMS) unpack_pairs(reinterpret_cast<const uint4*>(sp + 3 * d)[ci], bb, T());
+#pragma unroll
+            for (int k = 0; k < P; ++k) o[k] = RMS ? __fmul2_rn(f[k], g[k]) : __ffma2_rn(f[k], g[k], bb[k]);
+            reinterpret_cast<uint4*>(out2 + m * d)[ci] = pack_pairs(o, T());
+          }
         }
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(empty0 + 8 * s);   // the slot may be refilled
     }
   }
 }
@@ -634,17 +681,17 @@ cudaError_t with_nch(int d, F f) {
   }
 }
 
-template <typename T, bool RMS>
-cudaError_t gather_norm_t(const void* x, const int32_t* rows, int64_t M, int d, const void* g1,
-                          const void* b1, const void* g2, const void* b2, float eps, void* out1,
-                          void* out2, const Dev& dev) {
+template <typename T, bool RMS, int NCH>
+cudaError_t gather_norm_launch(const void* x, const int32_t* rows, int64_t M, int d, const void* g1,
+                               const void* b1, const void* g2, const void* b2, float eps, void* out1,
+                               void* out2, const Dev& dev) {
   const size_t row_bytes = (size_t)d * sizeof(T);
   const size_t smem = 4 * row_bytes + kRowSlots * row_bytes + 2 * kRowSlots * 8;
   static int attr_done[64] = {0};
   int device = 0;
   cudaGetDevice(&device);
   if (device < 64 && !attr_done[device]) {
-    cudaError_t e = cudaFuncSetAttribute(gather_norm_tma_kernel<T, RMS>,
+    cudaError_t e = cudaFuncSetAttribute(gather_norm_tma_kernel<T, RMS, NCH>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (4 + kRowSlots) * kMaxRowBytes + 2 * kRowSlots * 8);
     if (e != cudaSuccess) return e;
@@ -655,11 +702,20 @@ cudaError_t gather_norm_t(const void* x, const int32_t* rows, int64_t M, int d, 
   const int64_t fit = std::max<int64_t>(1, std::min<int64_t>(2, 232448 / (int64_t)(smem + 1024)));
   const int64_t grid = std::max<int64_t>(1, std::min<int64_t>((M + kRowWarps - 1) / kRowWarps,
                                                              fit * dev.num_sms));
-  return launch_pdl(gather_norm_tma_kernel<T, RMS>, dim3((unsigned)grid), dim3(kRowThreads), smem,
+  return launch_pdl(gather_norm_tma_kernel<T, RMS, NCH>, dim3((unsigned)grid), dim3(kRowThreads), smem,
                     dev.stream, static_cast<const T*>(x), rows, M, d, static_cast<const T*>(g1),
                     static_cast<const T*>(b1), static_cast<const T*>(g2),
                     static_cast<const T*>(b2), eps, static_cast<T*>(out1), static_cast<T*>(out2),
                     dev.err, kWaitTimeoutNs);
+}
+
+template <typename T, bool RMS>
+cudaError_t gather_norm_t(const void* x, const int32_t* rows, int64_t M, int d, const void* g1,
+                          const void* b1, const void* g2, const void* b2, float eps, void* out1,
+                          void* out2, const Dev& dev) {
+  return with_nch<T>(d, [&](auto nch) {
+    return gather_norm_launch<T, RMS, decltype(nch)::value>(x, rows, M, d, g1, b1, g2, b2, eps, out1, out2, dev);
+  });
 }
 
 cudaError_t gather_norm(int dtype, const void* x, const int32_t* rows, int64_t M, int d,
