@@ -395,7 +395,10 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
   // for GPT-NeoX (parallel residual) the MLP up projection of the second
   // norm shares the launch (a8).
   const int half = c->rotary_dim / 2;
-  const bool fuse_rope = tc && (half == 4 || half == 8 || half == 16 || (half > 0 && half % 32 == 0));
+  // (not in a decode step: with a few rows the projection runs split along K,
+  // which rotary tiles of halves above 16 features rule out; a separate pass
+  // rotates the few rows instead)
+  const bool fuse_rope = tc && !dec && (half == 4 || half == 8 || half == 16 || (half > 0 && half % 32 == 0));
   const bool neox_tc = neox && tc;
   {
     GemmArgs g = linear_args(lb.n1, d, w->w_qkv, M, qkv_dim, d);
