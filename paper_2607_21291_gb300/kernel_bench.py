@@ -3,6 +3,7 @@
   python -m paper_2607_21291_gb300.kernel_bench linear --M 8192 --N 8192 --K 2048
   python -m paper_2607_21291_gb300.kernel_bench layer --workload c3 --B 2
   python -m paper_2607_21291_gb300.kernel_bench attention --workload c5 --B 1 --K 2048
+  python -m paper_2607_21291_gb300.kernel_bench decode --workload c5 --B 16 --layers 2
 
 Each case runs `--warmup` untimed calls, then `--iters` calls each bracketed by
 CUDA events on the launching stream (L2 flushed between calls by a 256 MiB
@@ -149,6 +150,49 @@ def case_router(a, stream):
     return fn, flops, x.numel() * x.element_size(), ws
 
 
+def case_decode(a, stream):
+    """Decode steps (adadsf_decode_step) of a model of the workload's layer
+    shape with --layers layers and a small vocabulary, after a prefill of B
+    sequences of T tokens at K kept per layer; gbs counts the step's weights
+    and the cached keys and values at K per layer."""
+    wl = S.WORKLOADS[a.workload]
+    shape = wl.shape.replace(n_layers=a.layers, vocab=1024)
+    B = a.B or wl.B
+    T = a.T or wl.T
+    K = a.K if a.K is not None else T // 2
+    dt = torch.bfloat16 if shape.dtype == "bf16" else torch.float32
+    g = torch.Generator(device="cuda").manual_seed(0)
+    layers = []
+    for _ in range(shape.n_layers):
+        w = {n: (0.02 * torch.randn(shp, generator=g, device="cuda")).to(dt)
+             for n, shp in S.layer_weight_shapes(shape).items()}
+        for n in ("ln1_w", "ln2_w"):
+            w[n] = torch.ones_like(w[n])
+        layers.append(w)
+    extra = {"embed": (0.02 * torch.randn(shape.vocab, shape.d, generator=g, device="cuda")).to(dt),
+             "final_w": torch.ones(shape.d, device="cuda", dtype=dt)}
+    if shape.arch == S.NEOX:
+        extra["final_b"] = torch.zeros(shape.d, device="cuda", dtype=dt)
+    model = A.DeviceModel(A.make_cfg(shape), layers, extra)
+    Ks = [K] * shape.n_layers
+    steps = (a.warmup + a.iters + 4) * (1 + a.graph)   # every call advances the position
+    C_max = T + steps + 8
+    cache = A.kv_cache(model.cfg, B, C_max)
+    ids = torch.randint(0, shape.vocab, (B, T), generator=g, device="cuda", dtype=torch.int32)
+    hid = torch.empty((B, T, shape.d), dtype=dt, device="cuda")
+    pws = A.workspace(A.adadsf_model_workspace_size(model.cfg, B, T, Ks, False))
+    A.adadsf_prefill(model, ids, Ks, hid, cache, C_max, ws=pws, stream=stream)
+    del hid, pws
+    ws = A.workspace(A.adadsf_decode_workspace_size(model.cfg, B, C_max))
+    tok = torch.randint(0, shape.vocab, (B,), generator=g, device="cuda", dtype=torch.int32)
+    h = torch.empty((B, shape.d), dtype=dt, device="cuda")
+    fn = lambda: A.adadsf_decode_step(model, tok, h, cache, C_max, ws=ws, stream=stream)
+    es = 2 if dt == torch.bfloat16 else 4
+    w_bytes = sum(v.numel() for w in layers for v in w.values()) * es
+    kv_bytes = shape.n_layers * B * K * 2 * shape.kv_dim * es
+    return fn, 0.0, w_bytes + kv_bytes, ws
+
+
 def case_topk(a, stream):
     wl = S.WORKLOADS[a.workload]
     B = a.B or wl.B
@@ -164,7 +208,7 @@ def case_topk(a, stream):
 
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
-    ap.add_argument("case", choices=("linear", "layer", "attention", "router", "router_select", "topk"))
+    ap.add_argument("case", choices=("linear", "layer", "attention", "router", "router_select", "topk", "decode"))
     ap.add_argument("--M", type=int, default=8192)
     ap.add_argument("--N", type=int, default=8192)
     ap.add_argument("--K", type=int, default=None)
@@ -179,6 +223,7 @@ def main():
     ap.add_argument("--fold", action="store_true", help="layer: fold the norms (FLAG_FOLDED_NORMS)")
     ap.add_argument("--gate", action="store_true", help="layer: the score-gated variant")
     ap.add_argument("--graph", type=int, default=0, help="also time R calls replayed from one CUDA graph")
+    ap.add_argument("--layers", type=int, default=2, help="decode: layers of the model")
     a = ap.parse_args()
     if a.case == "linear" and a.K is None:
         a.K = 2048
@@ -187,7 +232,7 @@ def main():
     with torch.cuda.stream(stream):
         fn, flops, nbytes, ws = {"linear": case_linear, "layer": case_layer, "attention": case_attention,
                             "router": case_router, "router_select": case_router,
-                            "topk": case_topk}[a.case](a, stream)
+                            "topk": case_topk, "decode": case_decode}[a.case](a, stream)
         ms = _time(fn, a.iters, a.warmup, stream)
         out = {"case": a.case, "ms": ms}
         if flops:
