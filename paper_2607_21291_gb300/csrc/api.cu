@@ -440,20 +440,21 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
                  [&] { return run_linear(dt, g, dev, "qkv projection"); }));
     }
   }
-  if (c->rotary_dim > 0 && !fuse_rope)
+  if (c->rotary_dim > 0 && !fuse_rope && !dec)
     TRY(launch(dev, ADADSF_KERNEL_ROPE, false, 0,
                2.0 * M * (c->n_heads + c->n_kv_heads) * c->rotary_dim * es,
                CALL(rope_apply(dt, lb.qkv, M, qkv_dim, c->n_heads, c->n_kv_heads, c->head_dim,
                                c->rotary_dim, pos, T, lb.rope, dev),
                     "rotary")));
   if (dec) {
-    // a6 (decode): the kept new tokens' keys and values join the cache, then
-    // each new token attends to its layer's cached kept tokens (itself
-    // included when kept)
-    TRY(launch(dev, ADADSF_KERNEL_KV_CACHE, false, 0, 4.0 * B * kv * es,
-               CALL(kv_append(dt, lb.qkv, qkv_dim, q, kv, c->head_dim, B, dec->rows, dec->lens, dec->C_max,
-                              dec->kc, dec->vc, dev),
-                    "cache append")));
+    // a5' + a6 (decode): rotary of the new rows fused with the cache append
+    // (a kept token's rotated key and value join the cache), then each new
+    // token attends to its layer's cached kept tokens (itself included when kept)
+    TRY(launch(dev, ADADSF_KERNEL_KV_CACHE, false, 0,
+               2.0 * M * (c->n_heads + c->n_kv_heads) * c->rotary_dim * es + 4.0 * B * kv * es,
+               CALL(rope_append(dt, lb.qkv, qkv_dim, c->n_heads, c->n_kv_heads, c->head_dim, c->rotary_dim, B,
+                                dec->rows, dec->pos, lb.rope, dec->lens, dec->C_max, dec->kc, dec->vc, dev),
+                    "rotary + cache append")));
     TRY(launch(dev, ADADSF_KERNEL_ATTENTION, false, 0,
                (double)B * 2.0 * q * es + 2.0 * B * kv * es * dec->C_max,
                CALL(decode_attention(dt, lb.qkv, qkv_dim, c->n_heads, c->n_kv_heads, c->head_dim, dec->kc,

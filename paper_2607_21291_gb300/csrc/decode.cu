@@ -29,6 +29,7 @@ constexpr int kDecTK = 64;              // keys per tile (split granularity, rin
 constexpr int kDecStages = 3;           // ring stages of the bf16 kernel
 constexpr int kDecWarps = 4;            // consumer warps of the bf16 kernel, 16 keys of a tile each
 constexpr int kDecTcThreads = 32 * (kDecWarps + 1);
+constexpr int kRopeThreads = 1024;       // rotary + cache append: threads per sequence
 
 // ---------------------------------------------------------------- prefill -> cache
 // K and V of the kept (packed) rows m = b K + j of one layer into the cache:
@@ -464,30 +465,55 @@ __global__ void decode_combine_kernel(const float* part_o, const float2* part_ml
   }
 }
 
-// The kept new tokens' keys and values join the layer's cache (before the
-// step's attention, which then reads every key from the cache).
+// Rotary embedding of the new tokens' query and key heads at their positions
+// (feature i < half pairs with i + half, as in the prefill), fused with the
+// cache append: a kept token's rotated key and its value join the layer's
+// cache at lens[b], then lens[b] += 1. One block per sequence b, wide enough
+// that each thread has one or two pairs (the launch is latency bound).
 template <typename T>
-__global__ void kv_append_kernel(const T* qkv, int64_t ld, int q, int kvw, int hd, int B,
-                                 const int32_t* rows, int32_t* lens, int C_max, T* kc, T* vc,
-                                 int* err) {
+__global__ void __launch_bounds__(kRopeThreads) rope_append_kernel(T* qkv, int64_t ld, int Hq, int Hkv, int hd, int half,
+                                   const int32_t* pos, const float2* tab, const int32_t* rows,
+                                   int32_t* lens, int C_max, T* kc, T* vc, int* err) {
   pdl_trigger();
   pdl_wait();
   const int b = blockIdx.x;
-  if (rows[b] < 0) return;
+  T* row = qkv + (int64_t)b * ld;
+  const int q = Hq * hd, kvw = Hkv * hd;
+  bool append = rows[b] >= 0;
   const int len = lens[b];
-  if (len < 0 || len >= C_max) {
+  if (append && (len < 0 || len >= C_max)) {
     if (threadIdx.x == 0) set_device_error(err, DEVERR_INDEX);
-    return;
+    append = false;
   }
-  const int Hkv = kvw / hd;
-  for (int c = threadIdx.x; c < kvw; c += blockDim.x) {
-    const int h = c / hd, e = c % hd;
-    const int64_t dst = (((int64_t)b * Hkv + h) * C_max + len) * hd + e;
-    kc[dst] = qkv[(int64_t)b * ld + q + c];
-    vc[dst] = qkv[(int64_t)b * ld + q + kvw + c];
+  const float2* tab_row = tab + (int64_t)pos[b] * half;
+  // rotated pairs of every query and key head
+  for (int k = threadIdx.x; k < (Hq + Hkv) * half; k += blockDim.x) {
+    const int h = k / half, i = k % half;
+    T* base = row + (int64_t)h * hd;
+    const float2 cs = tab_row[i];
+    const float a = Elem<T>::to_f(base[i]);
+    const float c = Elem<T>::to_f(base[i + half]);
+    const T ra = Elem<T>::from_f(a * cs.x - c * cs.y);
+    const T rc = Elem<T>::from_f(c * cs.x + a * cs.y);
+    base[i] = ra;
+    base[i + half] = rc;
+    if (append && h >= Hq) {
+      const int64_t dst = (((int64_t)b * Hkv + (h - Hq)) * C_max + len) * hd;
+      kc[dst + i] = ra;
+      kc[dst + i + half] = rc;
+    }
+  }
+  if (append) {
+    // key features past the rotary pairs, and the values
+    for (int c = threadIdx.x; c < kvw; c += blockDim.x) {
+      const int h = c / hd, e = c % hd;
+      const int64_t dst = (((int64_t)b * Hkv + h) * C_max + len) * hd + e;
+      if (e >= 2 * half) kc[dst] = row[q + c];
+      vc[dst] = row[q + kvw + c];
+    }
   }
   __syncthreads();
-  if (threadIdx.x == 0) lens[b] = len + 1;
+  if (threadIdx.x == 0 && append) lens[b] = len + 1;
 }
 
 __global__ void decode_advance_kernel(int32_t* hdr) {
@@ -586,15 +612,17 @@ cudaError_t decode_attention(int dtype, const void* qkv, int64_t ld, int Hq, int
                     ns, static_cast<float*>(out), ld_out);
 }
 
-cudaError_t kv_append(int dtype, const void* qkv, int64_t ld, int q, int kvw, int hd, int B, const int32_t* rows,
-                      int32_t* lens, int C_max, void* kc, void* vc, const Dev& dev) {
+cudaError_t rope_append(int dtype, void* qkv, int64_t ld, int Hq, int Hkv, int hd, int rotary_dim, int B,
+                        const int32_t* rows, const int32_t* pos, const float2* tab, int32_t* lens, int C_max,
+                        void* kc, void* vc, const Dev& dev) {
   if (B <= 0) return cudaSuccess;
+  const int half = rotary_dim / 2;
   if (dtype == kBF16)
-    return launch_pdl(kv_append_kernel<bf16>, dim3(B), dim3(256), 0, dev.stream, static_cast<const bf16*>(qkv),
-                      ld, q, kvw, hd, B, rows, lens, C_max, static_cast<bf16*>(kc), static_cast<bf16*>(vc),
+    return launch_pdl(rope_append_kernel<bf16>, dim3(B), dim3(kRopeThreads), 0, dev.stream, static_cast<bf16*>(qkv), ld, Hq,
+                      Hkv, hd, half, pos, tab, rows, lens, C_max, static_cast<bf16*>(kc), static_cast<bf16*>(vc),
                       dev.err);
-  return launch_pdl(kv_append_kernel<float>, dim3(B), dim3(256), 0, dev.stream, static_cast<const float*>(qkv),
-                    ld, q, kvw, hd, B, rows, lens, C_max, static_cast<float*>(kc), static_cast<float*>(vc),
+  return launch_pdl(rope_append_kernel<float>, dim3(B), dim3(kRopeThreads), 0, dev.stream, static_cast<float*>(qkv), ld, Hq,
+                    Hkv, hd, half, pos, tab, rows, lens, C_max, static_cast<float*>(kc), static_cast<float*>(vc),
                     dev.err);
 }
 

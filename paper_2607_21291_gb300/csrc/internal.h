@@ -202,8 +202,10 @@ cudaError_t decode_decide(const float* scores, const float* thr, const int32_t* 
 cudaError_t decode_attention(int dtype, const void* qkv, int64_t ld, int Hq, int Hkv, int hd, const void* kc,
                              const void* vc, const int32_t* lens, int C_max, int B, float* part_o,
                              float2* part_ml, void* out, int64_t ld_out, const Dev& dev);
-cudaError_t kv_append(int dtype, const void* qkv, int64_t ld, int q, int kvw, int hd, int B, const int32_t* rows,
-                      int32_t* lens, int C_max, void* kc, void* vc, const Dev& dev);
+// Rotary embedding of the decode rows fused with the cache append (rotary_dim 0: append only).
+cudaError_t rope_append(int dtype, void* qkv, int64_t ld, int Hq, int Hkv, int hd, int rotary_dim, int B,
+                        const int32_t* rows, const int32_t* pos, const float2* tab, int32_t* lens, int C_max,
+                        void* kc, void* vc, const Dev& dev);
 cudaError_t decode_advance(int32_t* hdr, const Dev& dev);
 
 }  // namespace adadsf

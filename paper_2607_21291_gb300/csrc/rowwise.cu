@@ -175,6 +175,29 @@ __device__ __forceinline__ void norm_share(int64_t lo, int64_t hi, const T* x, i
   }
 }
 
+// ---------------------------------------------------------------- few rows
+// Gather + norm of a few rows (a decode step's one row per sequence): four
+// warps per block, one row per warp, the row in registers; the parameters
+// are staged before waiting for the previous kernel (they do not depend on it).
+constexpr int kFewRowWarps = 4;
+constexpr int64_t kFewRowsMax = 512;   // larger counts stream through gather_norm_tma_kernel
+
+template <typename T, bool RMS, int NCH>
+__global__ void __launch_bounds__(32 * kFewRowWarps)
+    norm_few_rows_kernel(const T* x, const int32_t* rows, int64_t M, int d, const T* g1, const T* b1,
+                         const T* g2, const T* b2, float eps, T* out1, T* out2) {
+  pdl_trigger();
+  extern __shared__ __align__(16) uint8_t smem_few[];
+  T* sp = reinterpret_cast<T*>(smem_few);
+  stage_norm_params(g1, RMS ? nullptr : b1, out2 ? g2 : nullptr, (RMS || !out2) ? nullptr : b2, d, sp);
+  pdl_wait();
+  const int64_t lo = (int64_t)blockIdx.x * kFewRowWarps;
+  const int64_t hi = lo + kFewRowWarps < M ? lo + kFewRowWarps : M;
+  norm_share<T, RMS, NCH>(
+      lo, hi, x, d, sp, eps, out1, out2, [&](int64_t i) { return rows ? (int64_t)rows[i] : i; },
+      [&](int64_t i) { return i; });
+}
+
 // ---------------------------------------------------------------- TMA-staged gather + norm
 // For large row counts (HBM bound): one warp streams whole source rows into a
 // shared-memory ring with one bulk copy each (cp.async.bulk, completion on the
@@ -714,7 +737,13 @@ cudaError_t gather_norm_t(const void* x, const int32_t* rows, int64_t M, int d, 
                           const void* b1, const void* g2, const void* b2, float eps, void* out1,
                           void* out2, const Dev& dev) {
   return with_nch<T>(d, [&](auto nch) {
-    return gather_norm_launch<T, RMS, decltype(nch)::value>(x, rows, M, d, g1, b1, g2, b2, eps, out1, out2, dev);
+    constexpr int NCH = decltype(nch)::value;
+    if (M <= kFewRowsMax)
+      return launch_pdl(norm_few_rows_kernel<T, RMS, NCH>, dim3((unsigned)((M + kFewRowWarps - 1) / kFewRowWarps)),
+                        dim3(32 * kFewRowWarps), 4 * (size_t)d * sizeof(T), dev.stream, static_cast<const T*>(x), rows,
+                        M, d, static_cast<const T*>(g1), static_cast<const T*>(b1), static_cast<const T*>(g2),
+                        static_cast<const T*>(b2), eps, static_cast<T*>(out1), static_cast<T*>(out2));
+    return gather_norm_launch<T, RMS, NCH>(x, rows, M, d, g1, b1, g2, b2, eps, out1, out2, dev);
   });
 }
 
