@@ -60,9 +60,9 @@ typedef enum { ADADSF_ARCH_NEOX = 0, ADADSF_ARCH_QWEN = 1 } adadsf_arch;
 typedef enum { ADADSF_STATS_TOKEN = 0, ADADSF_STATS_FLAT = 1 } adadsf_stats_mode;
 
 /* adadsf_model_cfg.flags.
- * ADADSF_FLAG_GATE_SIGMOID: the score-gated variant of Sec. 3.4 ("the
- * router-score pathway is kept differentiable"), in the Mixture-of-Depths
- * form: a kept row becomes x + sigmoid(s) * delta, s its router score, delta
+ * ADADSF_FLAG_GATE_SIGMOID: the score-gated variant of Sec. 3.4 (where the
+ * router scores stay on the differentiable path in training), in the
+ * Mixture-of-Depths form: a kept row becomes x + sigmoid(s) * delta, s its router score, delta
  * the layer's whole residual update (inside the layer nothing changes).
  * Without it (default) scores only select and kept rows get x + delta, so
  * K == T is exactly the dense layer. With it the router runs even when
@@ -245,7 +245,7 @@ adadsf_status adadsf_align_output(const void *hs_dev, const void *hd_dev, const 
                                   void *ws, size_t ws_bytes, void *stream);
 
 /* ------------------------------------------------------------------------
- * Sec. 3.4 ("the router-score pathway is kept differentiable"): the gradient
+ * Sec. 3.4 (router scores on the differentiable path): the gradient
  * of a loss with respect to one layer's router parameters through the score
  * gate of ADADSF_FLAG_GATE_SIGMOID, where a kept row is y = x + sigmoid(s)
  * delta. The layer input and its other weights are held fixed and the Top-K
@@ -465,7 +465,7 @@ typedef enum {
   ADADSF_KERNEL_GEMM_QKV_UP,   /* GPT-NeoX, bf16: QKV and MLP-up projections in one launch */
   ADADSF_KERNEL_GEMM_O_DOWN,   /* GPT-NeoX, bf16: output + MLP-down projections, one accumulator */
   ADADSF_KERNEL_TOPK_GATHER_NORM, /* Top-K fused with the gather and norms of the kept rows */
-  ADADSF_KERNEL_DECIDE,        /* decode: keep decision of each new token */
+  ADADSF_KERNEL_DECIDE,        /* decode keep decision: runs inside the norm launch (ADADSF_KERNEL_GATHER_NORM); no launch records this kind */
   ADADSF_KERNEL_KV_CACHE,      /* decode cache: fill (prefill), thresholds, append */
   ADADSF_KERNEL_ALIGN,         /* alignment objective and router gradient (Eqs. 9-10) */
   ADADSF_KERNEL_COUNT

@@ -449,8 +449,8 @@ def decode_step(ids_new, Wm, layers, p, st, kept_force=None):
 
 # --------------------------------------------------------------------------
 # Sec. 3.5, Eqs. 9-11 -- feature-preserving alignment objective, and the
-# router's gradient through the score gate (Sec. 3.4: the score pathway is
-# kept differentiable)
+# router's gradient through the score gate (Sec. 3.4: router scores on the
+# differentiable path)
 # --------------------------------------------------------------------------
 def softmax(z, axis=-1):
     """exp(z - max) / sum exp(z - max) along `axis`."""

@@ -1,7 +1,7 @@
 """Feature-preserving alignment of one sparse layer's router (Sec. 3.5), on
 synthetic data: the layer-local form of Eq. 9 with the router trained
-through the score gate of the gated variant (Sec. 3.4, "the router-score
-pathway is kept differentiable"). Every step of the method runs in the
+through the score gate of the gated variant (Sec. 3.4: the router scores
+stay on the differentiable path in training). Every step of the method runs in the
 library's kernels (the gated and ungated layer forwards, the Eq. 9 value and
 gradient, the router's parameter gradient); this module only sequences the
 calls and applies the plain SGD update to the router tensors.

@@ -344,17 +344,14 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
                     "router")));
   }
   if (dec) {
-    // decode: keep decision of each new token, then the norms of all B rows
+    // decode: keep decision of each new token and the norms of all B rows
     // (a bypassing token's block output is computed and dropped: the
     // projections stream their weights once either way)
-    TRY(launch(dev, ADADSF_KERNEL_DECIDE, false, 0, 16.0 * B,
-               CALL(decode_decide(lb.scores, dec->thr, dec->hdr, B, dec->C_max, dec->rows, dec->pos,
-                                  dec->kept_out, dev),
-                    "keep decision")));
-    TRY(launch(dev, ADADSF_KERNEL_GATHER_NORM, false, 0, Md * es * (neox ? 3 : 2),
-               CALL(gather_norm(dt, x, nullptr, M, d, !neox, w->ln1_w, w->ln1_b, w->ln2_w,
-                                w->ln2_b, c->norm_eps, lb.n1, neox ? lb.n2 : nullptr, dev),
-                    "norm")));
+    TRY(launch(dev, ADADSF_KERNEL_GATHER_NORM, false, 0, Md * es * (neox ? 3 : 2) + 16.0 * B,
+               CALL(decide_norm(dt, x, B, d, !neox, w->ln1_w, w->ln1_b, w->ln2_w, w->ln2_b, c->norm_eps, lb.n1,
+                                neox ? lb.n2 : nullptr, lb.scores, dec->thr, dec->hdr, dec->C_max, dec->rows,
+                                dec->pos, dec->kept_out, dev),
+                    "keep decision + norm")));
     rows = dec->rows;
     pos = dec->pos;
   } else if (!dense) {

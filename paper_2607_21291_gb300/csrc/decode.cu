@@ -91,28 +91,6 @@ __global__ void cache_header_kernel(int32_t* hdr, int T, int C_max, int L, int B
 }
 
 // ---------------------------------------------------------------- decode step
-// Keep decision of the new token of every sequence at one layer, its
-// position, and the packed-row map of the projections (rows[b] = b if kept,
-// -1 if it bypasses the layer: the residual scatter then skips it).
-__global__ void decode_decide_kernel(const float* scores, const float* thr, const int32_t* hdr, int B,
-                                     int C_max, int32_t* rows, int32_t* pos, int32_t* kept_out, int* err) {
-  pdl_trigger();
-  pdl_wait();
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b >= B) return;
-  int t = hdr[0];
-  // a cache not filled by a prefill of this shape, or no room left for the
-  // position in its rotary table: flag it and stay in bounds
-  if (hdr[1] != C_max || t < 0 || t >= C_max) {
-    set_device_error(err, DEVERR_INDEX);
-    t = t < 0 ? 0 : (t >= C_max ? C_max - 1 : t);
-  }
-  const bool keep = scores[b] > thr[b];   // a tie loses, NaN never wins
-  rows[b] = keep ? b : -1;
-  pos[b] = t;
-  if (kept_out) kept_out[b] = keep ? 1 : 0;
-}
-
 // Attention of the new token of sequence b, query heads h G .. h G + G - 1
 // (G = Hq / Hkv) of key/value head h, over split s of the n = lens[b] cached
 // keys (the token's own key is already appended). The splits cover [0, n) in
@@ -555,12 +533,6 @@ cudaError_t kv_threshold(const float* scores, const int32_t* idx, int B, int T, 
 
 cudaError_t cache_header(int32_t* hdr, int T, int C_max, int L, int B, const Dev& dev) {
   return launch_pdl(cache_header_kernel, dim3(1), dim3(32), 0, dev.stream, hdr, T, C_max, L, B);
-}
-
-cudaError_t decode_decide(const float* scores, const float* thr, const int32_t* hdr, int B, int C_max,
-                          int32_t* rows, int32_t* pos, int32_t* kept_out, const Dev& dev) {
-  return launch_pdl(decode_decide_kernel, dim3((B + 127) / 128), dim3(128), 0, dev.stream, scores, thr, hdr, B,
-                    C_max, rows, pos, kept_out, dev.err);
 }
 
 template <int HD>

@@ -198,6 +198,41 @@ __global__ void __launch_bounds__(32 * kFewRowWarps)
       [&](int64_t i) { return i; });
 }
 
+// A decode step's first pass: the norm(s) of the B new rows (one per
+// sequence) as above, and each row's keep decision at this layer (lane 0 of
+// its warp): kept iff its router score is above the layer's threshold (a tie
+// loses, NaN never wins); rows[b] = b if kept, else -1 (the residual scatter
+// skips it); pos[b] = the current position from the cache header. A cache
+// not filled by a prefill of this shape, or a position past its rotary
+// table, raises DEVERR_INDEX and the position is clamped into range.
+template <typename T, bool RMS, int NCH>
+__global__ void __launch_bounds__(32 * kFewRowWarps)
+    decide_norm_kernel(const T* x, int B, int d, const T* g1, const T* b1, const T* g2, const T* b2, float eps,
+                       T* out1, T* out2, const float* scores, const float* thr, const int32_t* hdr, int C_max,
+                       int32_t* rows, int32_t* pos, int32_t* kept_out, int* err) {
+  pdl_trigger();
+  extern __shared__ __align__(16) uint8_t smem_dn[];
+  T* sp = reinterpret_cast<T*>(smem_dn);
+  stage_norm_params(g1, RMS ? nullptr : b1, out2 ? g2 : nullptr, (RMS || !out2) ? nullptr : b2, d, sp);
+  pdl_wait();
+  const int64_t lo = (int64_t)blockIdx.x * kFewRowWarps;
+  const int64_t hi = lo + kFewRowWarps < B ? lo + kFewRowWarps : B;
+  const int b = (int)lo + (int)(threadIdx.x >> 5);
+  if (b < hi && (threadIdx.x & 31) == 0) {
+    int t = hdr[0];
+    if (hdr[1] != C_max || t < 0 || t >= C_max) {
+      set_device_error(err, DEVERR_INDEX);
+      t = t < 0 ? 0 : (t >= C_max ? C_max - 1 : t);
+    }
+    const bool keep = scores[b] > thr[b];
+    rows[b] = keep ? b : -1;
+    pos[b] = t;
+    if (kept_out) kept_out[b] = keep ? 1 : 0;
+  }
+  norm_share<T, RMS, NCH>(lo, hi, x, d, sp, eps, out1, out2, [](int64_t i) { return i; },
+                          [](int64_t i) { return i; });
+}
+
 // ---------------------------------------------------------------- TMA-staged gather + norm
 // For large row counts (HBM bound): one warp streams whole source rows into a
 // shared-memory ring with one bulk copy each (cp.async.bulk, completion on the
@@ -745,6 +780,37 @@ cudaError_t gather_norm_t(const void* x, const int32_t* rows, int64_t M, int d, 
                         static_cast<const T*>(b2), eps, static_cast<T*>(out1), static_cast<T*>(out2));
     return gather_norm_launch<T, RMS, NCH>(x, rows, M, d, g1, b1, g2, b2, eps, out1, out2, dev);
   });
+}
+
+template <typename T, bool RMS>
+cudaError_t decide_norm_t(const void* x, int B, int d, const void* g1, const void* b1, const void* g2,
+                          const void* b2, float eps, void* out1, void* out2, const float* scores, const float* thr,
+                          const int32_t* hdr, int C_max, int32_t* rows, int32_t* pos, int32_t* kept_out,
+                          const Dev& dev) {
+  return with_nch<T>(d, [&](auto nch) {
+    return launch_pdl(decide_norm_kernel<T, RMS, decltype(nch)::value>,
+                      dim3((unsigned)((B + kFewRowWarps - 1) / kFewRowWarps)), dim3(32 * kFewRowWarps),
+                      4 * (size_t)d * sizeof(T), dev.stream, static_cast<const T*>(x), B, d,
+                      static_cast<const T*>(g1), static_cast<const T*>(b1), static_cast<const T*>(g2),
+                      static_cast<const T*>(b2), eps, static_cast<T*>(out1), static_cast<T*>(out2), scores, thr,
+                      hdr, C_max, rows, pos, kept_out, dev.err);
+  });
+}
+
+cudaError_t decide_norm(int dtype, const void* x, int B, int d, bool is_rms, const void* g1, const void* b1,
+                        const void* g2, const void* b2, float eps, void* out1, void* out2, const float* scores,
+                        const float* thr, const int32_t* hdr, int C_max, int32_t* rows, int32_t* pos,
+                        int32_t* kept_out, const Dev& dev) {
+  if (B <= 0) return cudaSuccess;
+  if (dtype == kBF16)
+    return is_rms ? decide_norm_t<bf16, true>(x, B, d, g1, b1, g2, b2, eps, out1, out2, scores, thr, hdr, C_max,
+                                               rows, pos, kept_out, dev)
+                  : decide_norm_t<bf16, false>(x, B, d, g1, b1, g2, b2, eps, out1, out2, scores, thr, hdr, C_max,
+                                                rows, pos, kept_out, dev);
+  return is_rms ? decide_norm_t<float, true>(x, B, d, g1, b1, g2, b2, eps, out1, out2, scores, thr, hdr, C_max,
+                                              rows, pos, kept_out, dev)
+                : decide_norm_t<float, false>(x, B, d, g1, b1, g2, b2, eps, out1, out2, scores, thr, hdr, C_max,
+                                               rows, pos, kept_out, dev);
 }
 
 cudaError_t gather_norm(int dtype, const void* x, const int32_t* rows, int64_t M, int d,
