@@ -38,6 +38,7 @@
 // Every barrier wait is bounded in time; on give-up the CTA records
 // DEVERR_TIMEOUT, drains its in-flight copies and MMAs, frees TMEM and exits.
 #include <cuda.h>
+#include <cmath>
 #include <cudaTypedefs.h>
 
 #include <algorithm>
@@ -1606,13 +1607,19 @@ cudaError_t gemm_plain(const GemmArgs& a, const Dev& dev) {
   const int64_t t128 = mb128 * ((a.N + 127) / 128), t256 = mb128 * ((a.N + 255) / 256);
   const int64_t tpair = mb256 * ((a.N + 255) / 256);
   const int64_t sms = dev.num_sms;
-  constexpr int64_t kChunk = 2;      // 2 x (k-block cost) per epilogue chunk of 32 columns
-  constexpr int64_t kExchange = 4;   // partial-tile exchange through distributed shared memory
-  auto rounds = [](int64_t tiles, int64_t slots) { return (tiles + slots - 1) / slots; };
-  const int64_t cost_pair = rounds(tpair, sms / 2) * num_kb + 4 * kChunk;
-  const int64_t cost256 = rounds(t256, sms) * num_kb + 4 * kChunk;
-  const int64_t cost128 = rounds(t128, sms) * num_kb + 2 * kChunk;
-  int64_t best = cost_pair;
+  constexpr double kChunk = 2;      // 2 x (k-block cost) per epilogue chunk of 32 columns
+  constexpr double kExchange = 4;   // partial-tile exchange through distributed shared memory
+  // A k-block of a 256-column tile is the unit. With a single block of at most
+  // 128 rows (a decode step's few rows) the product streams its weights and a
+  // k-block costs in proportion to the weight rows it reads: narrower tiles,
+  // on more CTAs, go faster.
+  const bool stream_w = a.M <= BM;
+  auto kb = [&](int bn) { return stream_w ? (double)num_kb * bn / 256.0 : (double)num_kb; };
+  auto rounds = [](int64_t tiles, int64_t slots) { return (double)((tiles + slots - 1) / slots); };
+  const double cost_pair = rounds(tpair, sms / 2) * num_kb + 4 * kChunk;
+  const double cost256 = rounds(t256, sms) * kb(256) + 4 * kChunk;
+  const double cost128 = rounds(t128, sms) * kb(128) + 2 * kChunk;
+  double best = cost_pair;
   int pick = 0;   // 0 pair, 1 one-CTA 256, 2 one-CTA 128, 3 split 256, 4 split 128
   if (cost256 < best) { best = cost256; pick = 1; }
   if (cost128 < best) { best = cost128; pick = 2; }
@@ -1628,13 +1635,13 @@ cudaError_t gemm_plain(const GemmArgs& a, const Dev& dev) {
   if (can_split) {
     for (int S = 2; S <= 4; S += 2) {
       if (S > num_kb || (force && force != S)) continue;
-      const int64_t k = (num_kb + S - 1) / S + kExchange;
+      const double k256 = std::ceil(kb(256) / S) + kExchange, k128 = std::ceil(kb(128) / S) + kExchange;
       if (fits(t256, S, 256) && t256 <= sk_max_clusters<256>(S, dev)) {
-        const int64_t c = k + kChunk * ((256 / S / 32 + 1) / 2);
+        const double c = k256 + kChunk * ((256 / S / 32 + 1) / 2);
         if (c < best || force) { best = c; pick = 3; split_s = S; }
       }
       if (fits(t128, S, 128) && t128 <= sk_max_clusters<128>(S, dev)) {
-        const int64_t c = k + kChunk * ((128 / S / 32 + 1) / 2);
+        const double c = k128 + kChunk * ((128 / S / 32 + 1) / 2);
         if (c < best || (force && pick != 3)) { best = c; pick = 4; split_s = S; }
       }
     }
