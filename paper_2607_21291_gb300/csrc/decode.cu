@@ -557,6 +557,7 @@ cudaError_t decode_attention(int dtype, const void* qkv, int64_t ld, int Hq, int
   if (B <= 0) return cudaSuccess;
   if (Hq % Hkv != 0 || Hq / Hkv > kMaxGroup || (hd != 64 && hd != 128)) return cudaErrorInvalidValue;
   const int ns = decode_splits(B, Hkv, C_max, dev.num_sms);
+  if ((int64_t)ns * (C_max + kDecTK) > INT32_MAX) return cudaErrorInvalidValue;   // split bounds stay in int
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)hd);   // log2(e) / sqrt(hd)
   cudaError_t e;
   if (dtype == kBF16) {
