@@ -12,8 +12,10 @@
  *    error word, which must start at zero).
  *  - Device pointers must be 16-byte aligned; the workspace 256-byte aligned.
  *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
- *    stream). Every device entry point only enqueues work on that stream and
- *    returns without synchronising; results are ready once the stream is.
+ *    stream). Every device entry point only enqueues work on that stream
+ *    (adadsf_decode_step also on a stream of its own that it joins back into
+ *    it) and returns without synchronising; results are ready once the
+ *    stream is.
  *  - Tensors are dense row-major. Weights are [out_features, in_features]
  *    (the torch.nn.Linear layout); the fused QKV weight stacks the query
  *    rows, then the key rows, then the value rows.
@@ -420,6 +422,13 @@ adadsf_status adadsf_sparse_model_forward(const adadsf_model_cfg *cfg, const ada
  * the workspace of adadsf_model_workspace_size(cfg, B, T, K_host, 0); a
  * decode step adadsf_decode_workspace_size(cfg, B, C_max), and at most 16
  * query heads per key/value head (else ADADSF_ERR_UNSUPPORTED).
+ * A decode step runs each layer's router and keep decision on a second
+ * stream owned by the library, beside the norm and QKV projection on
+ * `stream`. Events fork that stream from `stream` and join it back before
+ * the layer's cache append, so the step is complete when `stream` is, and a
+ * graph captured from `stream` contains it. The second stream is made on
+ * the first decode step of the device. A step captured before any uncaptured
+ * step on the device runs on `stream` alone, with the same results.
  * ---------------------------------------------------------------------- */
 size_t adadsf_kv_cache_size(const adadsf_model_cfg *cfg, int B, int C_max);
 adadsf_status adadsf_prefill(const adadsf_model_cfg *cfg, const adadsf_model_weights *w,
@@ -465,7 +474,7 @@ typedef enum {
   ADADSF_KERNEL_GEMM_QKV_UP,   /* GPT-NeoX, bf16: QKV and MLP-up projections in one launch */
   ADADSF_KERNEL_GEMM_O_DOWN,   /* GPT-NeoX, bf16: output + MLP-down projections, one accumulator */
   ADADSF_KERNEL_TOPK_GATHER_NORM, /* Top-K fused with the gather and norms of the kept rows */
-  ADADSF_KERNEL_DECIDE,        /* decode keep decision: runs inside the norm launch (ADADSF_KERNEL_GATHER_NORM); no launch records this kind */
+  ADADSF_KERNEL_DECIDE,        /* decode: keep decision of each new token (inside the norm launch when the step runs on one stream) */
   ADADSF_KERNEL_KV_CACHE,      /* decode cache: fill (prefill), thresholds, append */
   ADADSF_KERNEL_ALIGN,         /* alignment objective and router gradient (Eqs. 9-10) */
   ADADSF_KERNEL_COUNT

@@ -6,6 +6,7 @@
 #include <stdarg.h>
 #include <stdio.h>
 
+#include <map>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -297,7 +298,44 @@ struct DecodeCtx {
   float* part_o;         // split-attention partials
   float2* part_ml;
   int32_t* kept_out;     // [B] or null
+  // A second stream for the router and the keep decision, which need only
+  // the layer input, so they run beside the norm and the QKV projection;
+  // joined before the cache append (null: everything on one stream).
+  cudaStream_t side = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
 };
+
+// The second stream and the two events of a decode step on `device`, made
+// once (not while the caller's stream is being captured into a graph: the
+// step then runs on one stream). False when they are not available.
+bool decode_side_stream(cudaStream_t main, cudaStream_t* side, cudaEvent_t* fork, cudaEvent_t* join) {
+  struct Side {
+    cudaStream_t s = nullptr;
+    cudaEvent_t f = nullptr, j = nullptr;
+  };
+  static std::mutex mu;
+  static std::map<int, Side> by_device;
+  int device = 0;
+  if (cudaGetDevice(&device) != cudaSuccess) return false;
+  std::lock_guard<std::mutex> lk(mu);
+  auto it = by_device.find(device);
+  if (it == by_device.end()) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(main, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) return false;
+    Side sd;
+    if (cudaStreamCreateWithFlags(&sd.s, cudaStreamNonBlocking) != cudaSuccess) return false;
+    if (cudaEventCreateWithFlags(&sd.f, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&sd.j, cudaEventDisableTiming) != cudaSuccess) {
+      cudaGetLastError();
+      return false;
+    }
+    it = by_device.emplace(device, sd).first;
+  }
+  *side = it->second.s;
+  *fork = it->second.f;
+  *join = it->second.j;
+  return true;
+}
 
 // Sec. 3.4: router -> Top-K -> gather + norm -> block on the packed rows ->
 // residual delta scattered back into x. K == T skips router and Top-K.
@@ -327,31 +365,52 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
   const int32_t* rows = nullptr;
   const int32_t* pos = nullptr;
 
+  // decode on two streams: the router and the keep decision on the side
+  // stream (from the layer input x), the norm and QKV on the main one
+  const bool forked = dec && dec->side;
+  Dev sdev = dev;
+  if (forked) {
+    sdev.stream = dec->side;
+    CUDA_TRY(cudaEventRecord(dec->fork, dev.stream), "fork the router stream");
+    CUDA_TRY(cudaStreamWaitEvent(dec->side, dec->fork, 0), "fork the router stream");
+  }
   if (!dense || gate || sink) {
     const double rf = 2.0 * BT * c->router_hidden * d;
     const double rb = (double)BT * d * es + (double)c->router_hidden * d * es + BT * 4.0;
     // a2: router scores of every token (bf16: tensor cores, tiles split
     // along d when there are few of them); the gated variant also needs
     // them when every token is kept
-    TRY(launch(dev, ADADSF_KERNEL_ROUTER, false, rf, rb,
+    TRY(launch(sdev, ADADSF_KERNEL_ROUTER, false, rf, rb,
                CALL(tc ? router_tc(x, BT, d, w->router_w1, w->router_b1, w->router_w2, w->router_b2,
-                                   lb.scores, lb.sync, lb.rpart, dev)
+                                   lb.scores, lb.sync, lb.rpart, sdev)
                        : router_f32(static_cast<const float*>(x), BT, d, c->router_hidden,
                                     static_cast<const float*>(w->router_w1),
                                     static_cast<const float*>(w->router_b1),
                                     static_cast<const float*>(w->router_w2),
-                                    static_cast<const float*>(w->router_b2), lb.scores, dev),
+                                    static_cast<const float*>(w->router_b2), lb.scores, sdev),
                     "router")));
   }
   if (dec) {
     // decode: keep decision of each new token and the norms of all B rows
     // (a bypassing token's block output is computed and dropped: the
     // projections stream their weights once either way)
-    TRY(launch(dev, ADADSF_KERNEL_GATHER_NORM, false, 0, Md * es * (neox ? 3 : 2) + 16.0 * B,
-               CALL(decide_norm(dt, x, B, d, !neox, w->ln1_w, w->ln1_b, w->ln2_w, w->ln2_b, c->norm_eps, lb.n1,
-                                neox ? lb.n2 : nullptr, lb.scores, dec->thr, dec->hdr, dec->C_max, dec->rows,
-                                dec->pos, dec->kept_out, dev),
-                    "keep decision + norm")));
+    if (forked) {
+      TRY(launch(sdev, ADADSF_KERNEL_DECIDE, false, 0, 16.0 * B,
+                 CALL(decode_decide(lb.scores, dec->thr, dec->hdr, B, dec->C_max, dec->rows, dec->pos,
+                                    dec->kept_out, sdev),
+                      "keep decision")));
+      CUDA_TRY(cudaEventRecord(dec->join, dec->side), "join the router stream");
+      TRY(launch(dev, ADADSF_KERNEL_GATHER_NORM, false, 0, Md * es * (neox ? 3 : 2),
+                 CALL(gather_norm(dt, x, nullptr, M, d, !neox, w->ln1_w, w->ln1_b, w->ln2_w, w->ln2_b,
+                                  c->norm_eps, lb.n1, neox ? lb.n2 : nullptr, dev),
+                      "norm")));
+    } else {
+      TRY(launch(dev, ADADSF_KERNEL_GATHER_NORM, false, 0, Md * es * (neox ? 3 : 2) + 16.0 * B,
+                 CALL(decide_norm(dt, x, B, d, !neox, w->ln1_w, w->ln1_b, w->ln2_w, w->ln2_b, c->norm_eps,
+                                  lb.n1, neox ? lb.n2 : nullptr, lb.scores, dec->thr, dec->hdr, dec->C_max,
+                                  dec->rows, dec->pos, dec->kept_out, dev),
+                      "keep decision + norm")));
+    }
     rows = dec->rows;
     pos = dec->pos;
   } else if (!dense) {
@@ -444,6 +503,7 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
                                c->rotary_dim, pos, T, lb.rope, dev),
                     "rotary")));
   if (dec) {
+    if (forked) CUDA_TRY(cudaStreamWaitEvent(dev.stream, dec->join, 0), "join the router stream");
     // a5' + a6 (decode): rotary of the new rows fused with the cache append
     // (a kept token's rotated key and value join the cache), then each new
     // token attends to its layer's cached kept tokens (itself included when kept)
@@ -1438,6 +1498,9 @@ adadsf_status adadsf_decode_step(const adadsf_model_cfg* cfg, const adadsf_model
   lb.sync = at<int>(ws, kErrBytes);
   lb.rpart = ds.layer.rsel ? at<float>(ws, ds.layer.rsel) : nullptr;
   lb.sq = ds.layer.sq ? at<float>(ws, ds.layer.sq) : nullptr;
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  const bool has_side = decode_side_stream(dev.stream, &side, &ev_fork, &ev_join);
   for (int l = 0; l < cfg->n_layers; ++l) {
     DecodeCtx dc;
     dc.thr = cv.thr + (int64_t)l * B;
@@ -1451,6 +1514,11 @@ adadsf_status adadsf_decode_step(const adadsf_model_cfg* cfg, const adadsf_model
     dc.part_o = at<float>(ws, ds.part_o);
     dc.part_ml = at<float2>(ws, ds.part_ml);
     dc.kept_out = kept_out_dev ? kept_out_dev + (int64_t)l * B : nullptr;
+    if (has_side) {
+      dc.side = side;
+      dc.fork = ev_fork;
+      dc.join = ev_join;
+    }
     TRY(layer_impl(cfg, &w->layers[l], x, B, 1, 1, lb, false, dev, nullptr, &dc));
   }
   TRY(launch(dev, ADADSF_KERNEL_FINAL_NORM, false, 0, 2.0 * B * cfg->d * es,

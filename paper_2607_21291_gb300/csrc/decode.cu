@@ -91,6 +91,30 @@ __global__ void cache_header_kernel(int32_t* hdr, int T, int C_max, int L, int B
 }
 
 // ---------------------------------------------------------------- decode step
+// Keep decision of the new token of every sequence at one layer, its
+// position, and the packed-row map of the projections (rows[b] = b if kept,
+// -1 if it bypasses the layer: the residual scatter then skips it). A tie
+// loses and NaN never wins. A cache not filled by a prefill of this shape, or
+// no room left in its rotary table, raises DEVERR_INDEX and the position is
+// clamped into range. (The same rule runs inside decide_norm_kernel when the
+// router is not forked onto a stream of its own.)
+__global__ void decode_decide_kernel(const float* scores, const float* thr, const int32_t* hdr, int B,
+                                     int C_max, int32_t* rows, int32_t* pos, int32_t* kept_out, int* err) {
+  pdl_trigger();
+  pdl_wait();
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  int t = hdr[0];
+  if (hdr[1] != C_max || t < 0 || t >= C_max) {
+    set_device_error(err, DEVERR_INDEX);
+    t = t < 0 ? 0 : (t >= C_max ? C_max - 1 : t);
+  }
+  const bool keep = scores[b] > thr[b];
+  rows[b] = keep ? b : -1;
+  pos[b] = t;
+  if (kept_out) kept_out[b] = keep ? 1 : 0;
+}
+
 // Attention of the new token of sequence b, query heads h G .. h G + G - 1
 // (G = Hq / Hkv) of key/value head h, over split s of the n = lens[b] cached
 // keys (the token's own key is already appended). The splits cover [0, n) in
@@ -549,6 +573,12 @@ static cudaError_t launch_decode_tc(const CUtensorMap& tk, const CUtensorMap& tv
   return launch_pdl(decode_attn_tc_kernel<HD>, dim3(ns, Hkv, B), dim3(kDecTcThreads), (size_t)DecTc<HD>::SMEM,
                     dev.stream, tk, tv, qkv, ld, Hq, Hkv, lens, C_max, ns, scale_log2, part_o, part_ml, dev.err,
                     kWaitTimeoutNs);
+}
+
+cudaError_t decode_decide(const float* scores, const float* thr, const int32_t* hdr, int B, int C_max,
+                          int32_t* rows, int32_t* pos, int32_t* kept_out, const Dev& dev) {
+  return launch_pdl(decode_decide_kernel, dim3((B + 127) / 128), dim3(128), 0, dev.stream, scores, thr, hdr, B,
+                    C_max, rows, pos, kept_out, dev.err);
 }
 
 cudaError_t decode_attention(int dtype, const void* qkv, int64_t ld, int Hq, int Hkv, int hd, const void* kc,

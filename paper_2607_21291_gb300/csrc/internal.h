@@ -197,6 +197,9 @@ cudaError_t kv_fill(int dtype, const void* qkv, int64_t ld, int q, int kvw, int 
 cudaError_t kv_threshold(const float* scores, const int32_t* idx, int B, int T, int K, int32_t* lens,
                          float* thr, const Dev& dev);
 cudaError_t cache_header(int32_t* hdr, int T, int C_max, int L, int B, const Dev& dev);
+// Keep decision of each new token (one per sequence) at one layer (decode.cu).
+cudaError_t decode_decide(const float* scores, const float* thr, const int32_t* hdr, int B, int C_max,
+                          int32_t* rows, int32_t* pos, int32_t* kept_out, const Dev& dev);
 // Keep decision of each new token (one per sequence) at one layer, fused with
 // the norm(s) of the B new rows (rowwise.cu).
 cudaError_t decide_norm(int dtype, const void* x, int B, int d, bool is_rms, const void* g1, const void* b1,
