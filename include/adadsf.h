@@ -427,8 +427,9 @@ adadsf_status adadsf_sparse_model_forward(const adadsf_model_cfg *cfg, const ada
  * `stream`. Events fork that stream from `stream` and join it back before
  * the layer's cache append, so the step is complete when `stream` is, and a
  * graph captured from `stream` contains it. The second stream is made on
- * the first decode step of the device. A step captured before any uncaptured
- * step on the device runs on `stream` alone, with the same results.
+ * the first decode step enqueued on `stream`; a step captured before any
+ * uncaptured step on that stream runs on `stream` alone, with the same
+ * results.
  * ---------------------------------------------------------------------- */
 size_t adadsf_kv_cache_size(const adadsf_model_cfg *cfg, int B, int C_max);
 adadsf_status adadsf_prefill(const adadsf_model_cfg *cfg, const adadsf_model_weights *w,

@@ -9,6 +9,7 @@
 #include <map>
 #include <mutex>
 #include <string>
+#include <utility>
 #include <vector>
 
 #include "adadsf.h"
@@ -305,21 +306,25 @@ struct DecodeCtx {
   cudaEvent_t fork = nullptr, join = nullptr;
 };
 
-// The second stream and the two events of a decode step on `device`, made
-// once (not while the caller's stream is being captured into a graph: the
-// step then runs on one stream). False when they are not available.
+// The second stream and the two events of decode steps on the caller's
+// stream `main` (of the current device), made once per such stream (not
+// while `main` is being captured into a graph: the step then runs on one
+// stream). Keyed by the caller's stream, so that steps enqueued on different
+// streams from different host threads never share the fork and join events.
+// False when they are not available.
 bool decode_side_stream(cudaStream_t main, cudaStream_t* side, cudaEvent_t* fork, cudaEvent_t* join) {
   struct Side {
     cudaStream_t s = nullptr;
     cudaEvent_t f = nullptr, j = nullptr;
   };
   static std::mutex mu;
-  static std::map<int, Side> by_device;
+  static std::map<std::pair<int, cudaStream_t>, Side> by_stream;
   int device = 0;
   if (cudaGetDevice(&device) != cudaSuccess) return false;
   std::lock_guard<std::mutex> lk(mu);
-  auto it = by_device.find(device);
-  if (it == by_device.end()) {
+  const auto key = std::make_pair(device, main);
+  auto it = by_stream.find(key);
+  if (it == by_stream.end()) {
     cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
     if (cudaStreamIsCapturing(main, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) return false;
     Side sd;
@@ -329,7 +334,7 @@ bool decode_side_stream(cudaStream_t main, cudaStream_t* side, cudaEvent_t* fork
       cudaGetLastError();
       return false;
     }
-    it = by_device.emplace(device, sd).first;
+    it = by_stream.emplace(key, sd).first;
   }
   *side = it->second.s;
   *fork = it->second.f;
