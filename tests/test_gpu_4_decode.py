@@ -192,3 +192,90 @@ def test_decode_at_bench_geometry(A):
         kg = kept.cpu().numpy().astype(bool)[:, sample]
         href, _, _ = O.decode_step(ids[sample, T0 + step], E64, W64, p, st, kept_force=kg)
         H.assert_close(H.to_np(h)[sample], href, H.tol(shape), f"decode step {step}", H.BF16_DEEP_ELEM_TOL)
+
+
+def _small_model(A, shape, seed):
+    td = H.tdtype(shape)
+    hostL = [H.host_layer(shape, seed, l) for l in range(shape.n_layers)]
+    return A.DeviceModel(A.make_cfg(shape), [A.to_device(w, td) for w in hostL],
+                         A.to_device(H.host_extra(shape, seed), td)), td
+
+
+def _decode_run(A, model, td, ids, B, T0, K, C_max, steps, stream, capture_first=False):
+    """Prefill then `steps` decode steps on `stream`; with capture_first the
+    steps are replayed from a graph captured before any eager step on this
+    stream (the step then runs on the caller's stream alone)."""
+    d = model.cfg.d
+    cache = A.kv_cache(model.cfg, B, C_max)
+    dws = A.workspace(A.adadsf_decode_workspace_size(model.cfg, B, C_max))
+    tok = torch.empty(B, dtype=torch.int32, device="cuda")
+    h = torch.empty((B, d), dtype=td, device="cuda")
+    out = []
+    with torch.cuda.stream(stream):
+        A.adadsf_prefill(model, ids[:, :T0].contiguous(), K, torch.empty((B, T0, d), dtype=td, device="cuda"),
+                         cache, C_max, stream=stream)
+        if capture_first:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                A.adadsf_decode_step(model, tok, h, cache, C_max, ws=dws, stream=stream)
+            for t in range(steps):
+                tok.copy_(ids[:, T0 + t])
+                g.replay()
+                out.append(h.clone())
+        else:
+            for t in range(steps):
+                tok.copy_(ids[:, T0 + t])
+                A.adadsf_decode_step(model, tok, h, cache, C_max, ws=dws, stream=stream)
+                out.append(h.clone())
+    torch.cuda.synchronize()
+    assert A.adadsf_sync_check(dws) == A.OK
+    return torch.stack(out)
+
+
+def test_decode_captured_before_any_eager_step(A):
+    """A step captured into a graph before any uncaptured step on its stream
+    runs on that stream alone (keep decision inside the norm launch); its
+    outputs equal those of eager steps, which fork the router onto a second
+    stream."""
+    shape = QWEN_SMALL
+    model, td = _small_model(A, shape, 61)
+    B, T0, C_max, K = 2, 96, 112, [48, 30, 96]
+    ids = torch.from_numpy(S.token_ids(62, B, T0 + 4, shape.vocab)).cuda()
+    eager = _decode_run(A, model, td, ids, B, T0, K, C_max, 4, torch.cuda.Stream())
+    graph = _decode_run(A, model, td, ids, B, T0, K, C_max, 4, torch.cuda.Stream(), capture_first=True)
+    assert torch.equal(eager, graph)
+
+
+def test_decode_on_two_streams_interleaved(A):
+    """Two models decode on two streams with their steps enqueued in turn:
+    each gets the outputs it gets alone (each caller stream has its own
+    second stream and fork / join events)."""
+    shape = NEOX_SMALL
+    (m1, td), (m2, _) = _small_model(A, shape, 71), _small_model(A, shape, 72)
+    B, T0, C_max, K, steps = 2, 64, 80, [40, 64, 20], 4
+    ids1 = torch.from_numpy(S.token_ids(73, B, T0 + steps, shape.vocab)).cuda()
+    ids2 = torch.from_numpy(S.token_ids(74, B, T0 + steps, shape.vocab)).cuda()
+    alone1 = _decode_run(A, m1, td, ids1, B, T0, K, C_max, steps, torch.cuda.Stream())
+    alone2 = _decode_run(A, m2, td, ids2, B, T0, K, C_max, steps, torch.cuda.Stream())
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    caches, wss, toks, hs, outs = [], [], [], [], [[], []]
+    for m, ids, s in ((m1, ids1, s1), (m2, ids2, s2)):
+        cache = A.kv_cache(m.cfg, B, C_max)
+        with torch.cuda.stream(s):
+            A.adadsf_prefill(m, ids[:, :T0].contiguous(), K, torch.empty((B, T0, shape.d), dtype=td, device="cuda"),
+                             cache, C_max, stream=s)
+        caches.append(cache)
+        wss.append(A.workspace(A.adadsf_decode_workspace_size(m.cfg, B, C_max)))
+        toks.append(torch.empty(B, dtype=torch.int32, device="cuda"))
+        hs.append(torch.empty((B, shape.d), dtype=td, device="cuda"))
+    torch.cuda.synchronize()
+    for t in range(steps):
+        for i, (m, ids, s) in enumerate(((m1, ids1, s1), (m2, ids2, s2))):
+            with torch.cuda.stream(s):
+                toks[i].copy_(ids[:, T0 + t])
+                A.adadsf_decode_step(m, toks[i], hs[i], caches[i], C_max, ws=wss[i], stream=s)
+                outs[i].append(hs[i].clone())
+    torch.cuda.synchronize()
+    assert A.adadsf_sync_check(wss[0]) == A.OK and A.adadsf_sync_check(wss[1]) == A.OK
+    assert torch.equal(torch.stack(outs[0]), alone1)
+    assert torch.equal(torch.stack(outs[1]), alone2)
