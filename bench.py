@@ -505,6 +505,7 @@ def run_ours(args, rank, world, local_rank):
                        "copied out every step (the copy out of step i on a second stream under step i+1); "
                        "one event pair around all steps, L2 flush between steps inside it"},
         "gpu_launches": launches_per_step * args.steps,
+        "folded_norms": bool(args.folded_norms),
         "clocks": clocks,
         "dense_same_kernels": {"ms_per_step": dense, "value": tokens / (dense * 1e-3), "unit": "tokens/s",
                                "steps": n_side},
@@ -776,7 +777,9 @@ def main():
     ap.add_argument("--spin-up", type=float, default=1.5, help="seconds of untimed GPU work before measuring")
     ap.add_argument("--decode-steps", type=int, default=32, help="decode steps timed after a prefill (0: none)")
     ap.add_argument("--folded-norms", action="store_true",
-                    help="fold the norms into the projections (ADADSF_FLAG_FOLDED_NORMS)")
+                    help="fold the norm gains into the projections (ADADSF_FLAG_FOLDED_NORMS; exact for the "
+                         "benchmark models, whose gains are 1): a decode step's post-attention RMSNorm then "
+                         "runs inside its projections")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
 

@@ -74,8 +74,8 @@ typedef enum { ADADSF_STATS_TOKEN = 0, ADADSF_STATS_FLAT = 1 } adadsf_stats_mode
  * norm biases 0, their values folded into the projections that read the
  * normed rows (what adadsf_fold_norms leaves). The layers may then apply a
  * norm's row scale inside those projections instead of a separate pass
- * (bf16 Qwen: the post-attention RMSNorm). With unfolded weights the flag
- * gives wrong results. */
+ * (bf16 Qwen: the post-attention RMSNorm of at most 128 rows, as in a decode
+ * step). With unfolded weights the flag gives wrong results. */
 #define ADADSF_FLAG_FOLDED_NORMS 2u
 
 /* adadsf_alloc_ratios flags */

@@ -615,9 +615,13 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
     g.epi.out_mapped = false;
     g.epi.out = lb.ao;
     g.epi.ld_out = d;
-    // folded second RMSNorm (bf16): the O epilogue also leaves each h row's
-    // chunk sums of squares; the gate / up epilogue turns them into its rstd
-    const bool fold2 = tc && folded(c) && lb.sq;
+    // folded second RMSNorm (bf16), for few rows (a decode step): the O
+    // epilogue also leaves each h row's chunk sums of squares and the gate /
+    // up epilogue turns them into its rstd, in place of a norm launch. With
+    // many rows the two epilogues' extra work costs more than the pass it
+    // saves (measured at the Qwen2.5-7B shape), so the pass runs with the
+    // folded unit gains.
+    const bool fold2 = tc && folded(c) && lb.sq && M <= 128;
     if (fold2) {
       g.epi.sq_out = lb.sq;
       g.epi.sq_ld = d / 32;

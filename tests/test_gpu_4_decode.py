@@ -58,12 +58,28 @@ def _cache_counts(A, cache, L, B):
 
 @pytest.mark.parametrize("shape,B,T0,K,steps,C_max,gated,etol", CASES)
 def test_prefill_then_decode(A, shape, B, T0, K, steps, C_max, gated, etol):
+    _prefill_then_decode(A, shape, B, T0, K, steps, C_max, gated, etol)
+
+
+@pytest.mark.parametrize("gated", [False, True])
+def test_prefill_then_decode_folded_norms(A, gated):
+    """The same check on weights with the norm gains folded in
+    (adadsf_fold_norms, FLAG_FOLDED_NORMS): the decode step's post-attention
+    RMSNorm then runs inside the output and gate / up projections."""
+    _prefill_then_decode(A, QWEN_SMALL, 2, 96, [48, 30, 96], 3, 100, gated, None, folded=True)
+
+
+def _prefill_then_decode(A, shape, B, T0, K, steps, C_max, gated, etol, folded=False):
     L = shape.n_layers
     td = H.tdtype(shape)
-    flags = A.FLAG_GATE_SIGMOID if gated else 0
+    flags = (A.FLAG_GATE_SIGMOID if gated else 0) | (A.FLAG_FOLDED_NORMS if folded else 0)
     hostL = [H.host_layer(shape, 13, l) for l in range(L)]
     extra = H.host_extra(shape, 13)
-    model = A.DeviceModel(A.make_cfg(shape, flags), [A.to_device(w, td) for w in hostL], A.to_device(extra, td))
+    layers = [A.to_device(w, td) for w in hostL]
+    if folded:
+        for w in layers:
+            A.adadsf_fold_norms(A.make_cfg(shape.replace(n_layers=1)), w)
+    model = A.DeviceModel(A.make_cfg(shape, flags), layers, A.to_device(extra, td))
     ids = S.token_ids(14, B, T0 + steps, shape.vocab)
     ids_d = torch.from_numpy(ids).cuda()
     cache = A.kv_cache(model.cfg, B, C_max)
