@@ -95,6 +95,7 @@ struct GemmDev {
   int add_gathered;
   const int32_t* rows;
   int out_mapped;
+  int a_box_rows;            // A rows a stage loads: 128, or fewer for a single block of fewer rows
   bf16* out; int64_t ld_out;
   // rotary embedding fused into the QKV epilogue (rope_tab == nullptr: off)
   const float2* rope_tab;    // [T][rope_half] (cos, sin)
@@ -740,7 +741,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t phase = 0;
       int64_t issued = 0;
       // bytes per stage: the A tile and this problem's weight tile(s)
-      auto stage_tx = [](int bn) { return (uint32_t)(C::A_BYTES + bn * BK * 2 * C::NUM_B); };
+      auto stage_tx = [&](int bn) { return (uint32_t)(p.a_box_rows * BK * 2 + bn * BK * 2 * C::NUM_B); };
       // The weights do not depend on the previous kernel: the first tile's
       // weight tiles are requested before waiting for it.
       int pre = 0;
@@ -960,7 +961,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
-      constexpr uint32_t tx = C::STAGE_BYTES;
+      const uint32_t tx = (uint32_t)(p.a_box_rows * BK * 2 + C::B_BYTES);
       const int npre = nkb < C::STAGES ? nkb : C::STAGES;
       for (int i = 0; i < npre; ++i) {   // weights first: independent of the previous kernel
         const KbSrc src = kb_source(ti, kb0 + i, &tmA, &tmB, &tmA2, &tmB2);
@@ -1424,8 +1425,10 @@ cudaError_t prepare(const GemmArgs& a, const GemmArgs* b, uint32_t a_rows, int b
     return cudaErrorInvalidValue;
   if (!make_dev(a, dev, p)) return cudaErrorInvalidValue;
   p.bn = width(a);
+  p.a_box_rows = (int)a_rows;
   p2 = GemmDev{};
   p2.bn = bn;
+  p2.a_box_rows = (int)a_rows;
   if (!problem_maps(a, a_rows, rows(a), tm[0], tm[1], &tm[2], &tm[3])) return cudaErrorInvalidValue;
   if (DUAL) {
     if (p.bn != bn || !make_tmap(&tm[3], a.W2, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, b_rows))
@@ -1434,6 +1437,7 @@ cudaError_t prepare(const GemmArgs& a, const GemmArgs* b, uint32_t a_rows, int b
   } else if (b) {
     if (a.K2 > 0 || b->K2 > 0 || !make_dev(*b, dev, p2)) return cudaErrorInvalidValue;
     p2.bn = width(*b);
+    p2.a_box_rows = (int)a_rows;
     if (!problem_maps(*b, a_rows, rows(*b), tm[2], tm[3], nullptr, nullptr))
       return cudaErrorInvalidValue;
   } else if (a.K2 == 0) {
@@ -1441,6 +1445,15 @@ cudaError_t prepare(const GemmArgs& a, const GemmArgs* b, uint32_t a_rows, int b
     tm[3] = tm[1];
   }
   return cudaSuccess;
+}
+
+// A rows a stage of the one-CTA kernels loads. A single block of fewer than
+// 128 rows (a decode step's few rows) loads only those, rounded up to 8:
+// the rows past them stay as they are in shared memory, and the
+// accumulator rows they give are never stored.
+uint32_t a_box_rows(const GemmArgs& a, const GemmArgs* b) {
+  const int64_t m = b ? std::max(a.M, b->M) : a.M;
+  return m < BM ? (uint32_t)((m + 7) / 8 * 8) : (uint32_t)BM;
 }
 
 // Whether a launch needs the epilogue instance with the rarer features.
@@ -1462,7 +1475,7 @@ cudaError_t launch_x(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
   }
   CUtensorMap tm[4];
   GemmDev p, p2;
-  cudaError_t e = prepare<DUAL>(a, b, BM, BN, BN, dev, tm, p, p2);
+  cudaError_t e = prepare<DUAL>(a, b, a_box_rows(a, b), BN, BN, dev, tm, p, p2);
   if (e != cudaSuccess) return e;
   int64_t num_tiles = ((a.M + BM - 1) / BM) * ((a.N + p.bn - 1) / p.bn);
   if (b) num_tiles += ((b->M + BM - 1) / BM) * ((b->N + p2.bn - 1) / p2.bn);
@@ -1584,7 +1597,7 @@ cudaError_t launch_sk(const GemmArgs& a, const Dev& dev, int S) {
   GemmDev p, p2;
   GemmArgs a_full = a;
   a_full.tile_n = 0;
-  cudaError_t e = prepare<false>(a_full, nullptr, BM, BN, BN, dev, tm, p, p2);
+  cudaError_t e = prepare<false>(a_full, nullptr, a_box_rows(a, nullptr), BN, BN, dev, tm, p, p2);
   if (e != cudaSuccess) return e;
   const int64_t num_tiles = ((a.M + BM - 1) / BM) * ((a.N + BN - 1) / BN);
   if (extra_args(a))
