@@ -108,7 +108,10 @@ def test_linear_bf16(A, M, N, Kd, act):
 @pytest.mark.parametrize("M,N,Kd,act", [(1, 64, 3072, 0), (300, 768, 3072, 1), (1384, 768, 3072, 0),
                                         (128, 256, 2048, 0), (777, 2304, 768, 1), (1000, 384, 1024, 0),
                                         (1024, 768, 768, 1), (1024, 768, 3072, 0), (333, 640, 960, 1),
-                                        (129, 128, 192, 0)])
+                                        (129, 128, 192, 0),
+                                        # fewer than 128 rows: a stage loads only them, rounded up to 8
+                                        (5, 512, 3584, 0), (13, 4608, 3584, 1), (16, 3584, 18944, 0),
+                                        (17, 1024, 2048, 1), (100, 640, 1536, 0)])
 def test_linear_bf16_small_m(A, M, N, Kd, act):
     """Small-M projections of the sparse layers: one wave of tiles, long K
     (with room for scratch most of these run split along K over clusters of 2
