@@ -174,14 +174,16 @@ def rank_seed(seed, rank):
     return seed + 7919 * rank
 
 
-def device_model(A, shape, seed, device, fold=False):
+def device_model(A, shape, seed, device, fold=False, gathered=False):
     """Random-init weights of the backbone shape in the benchmark recipe,
     drawn on the device (the reference arm draws the same tensors). With
     fold, the norm parameters are folded into the projections
     (adadsf_fold_norms; exact here, as the recipe's gains are 1 and biases 0)
-    and the layers run with ADADSF_FLAG_FOLDED_NORMS."""
+    and the layers run with ADADSF_FLAG_FOLDED_NORMS (and, with gathered,
+    ADADSF_FLAG_GATHERED_QKV)."""
     td = torch.bfloat16 if shape.dtype == "bf16" else torch.float32
-    cfg = A.make_cfg(shape, A.FLAG_FOLDED_NORMS if fold else 0)
+    flags = (A.FLAG_FOLDED_NORMS | (A.FLAG_GATHERED_QKV if gathered else 0)) if fold else 0
+    cfg = A.make_cfg(shape, flags)
     layers = []
     for l in range(shape.n_layers):
         w = {k: v.to(td) for k, v in S.bench_layer_weights(shape, seed, l, device).items()}
@@ -223,7 +225,8 @@ def run_ours(args, rank, world, local_rank):
     L = shape.n_layers
     t_target = retention_of(args, wl)
     stream = torch.cuda.Stream(device)
-    model = device_model(A, shape, WEIGHT_SEED, device, fold=args.folded_norms)
+    model = device_model(A, shape, WEIGHT_SEED, device, fold=args.folded_norms or args.gathered_qkv,
+                         gathered=args.gathered_qkv)
     sampler = ClockSampler(gpu_id_for_smi(local_rank))
     n_rec = 4 + 12 * L
 
@@ -505,7 +508,8 @@ def run_ours(args, rank, world, local_rank):
                        "copied out every step (the copy out of step i on a second stream under step i+1); "
                        "one event pair around all steps, L2 flush between steps inside it"},
         "gpu_launches": launches_per_step * args.steps,
-        "folded_norms": bool(args.folded_norms),
+        "folded_norms": bool(args.folded_norms or args.gathered_qkv),
+        "gathered_qkv": bool(args.gathered_qkv),
         "clocks": clocks,
         "dense_same_kernels": {"ms_per_step": dense, "value": tokens / (dense * 1e-3), "unit": "tokens/s",
                                "steps": n_side},
@@ -780,6 +784,9 @@ def main():
                     help="fold the norm gains into the projections (ADADSF_FLAG_FOLDED_NORMS; exact for the "
                          "benchmark models, whose gains are 1): a decode step's post-attention RMSNorm then "
                          "runs inside its projections")
+    ap.add_argument("--gathered-qkv", action="store_true",
+                    help="with folded norms, the first RMSNorm inside the QKV projection, whose loads gather the "
+                         "kept rows of x (ADADSF_FLAG_GATHERED_QKV)")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
 

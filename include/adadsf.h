@@ -77,6 +77,16 @@ typedef enum { ADADSF_STATS_TOKEN = 0, ADADSF_STATS_FLAT = 1 } adadsf_stats_mode
  * (bf16 Qwen: the post-attention RMSNorm of at most 128 rows, as in a decode
  * step). With unfolded weights the flag gives wrong results. */
 #define ADADSF_FLAG_FOLDED_NORMS 2u
+/* ADADSF_FLAG_GATHERED_QKV (with ADADSF_FLAG_FOLDED_NORMS; bf16 Qwen layers
+ * that keep K < T tokens of more than 32 rows per SM): the first RMSNorm runs
+ * inside the QKV projection. The router also sums the squares of every token
+ * row it reads, the projection loads the kept rows of x by row-gather copies
+ * (four rows per copy) instead of reading a gathered, normed copy, and its
+ * epilogue scales each row by 1 / rms. Exact up to rounding; off by default
+ * because the row gathers feed the tensor cores more slowly than the separate
+ * gather + norm pass costs (at the Qwen2.5-7B shape the QKV projection takes
+ * 3.7x its time). Ignored without ADADSF_FLAG_FOLDED_NORMS. */
+#define ADADSF_FLAG_GATHERED_QKV 4u
 
 /* adadsf_alloc_ratios flags */
 #define ADADSF_ALLOC_RAW 1u      /* return Eq. 8 unclamped (ratios may exceed 1) */

@@ -26,6 +26,7 @@ LINEAR_SPLIT_WS_BYTES = 256 + 160 * 128 * 256 * 4   # ADADSF_LINEAR_SPLIT_WS_BYT
 ALLOC_RAW, ALLOC_ROUND = 1, 2
 FLAG_GATE_SIGMOID = 1
 FLAG_FOLDED_NORMS = 2
+FLAG_GATHERED_QKV = 4
 
 TORCH_DTYPE = {F32: torch.float32, BF16: torch.bfloat16}
 DTYPE_CODE = {torch.float32: F32, torch.bfloat16: BF16}

@@ -98,13 +98,16 @@ adadsf_status check_cfg(const adadsf_model_cfg* c) {
     return fail(ADADSF_ERR_INVALID_ARG, "rotary_dim=%d must be even and <= head_dim", c->rotary_dim);
   if (!(c->norm_eps > 0.f) || !(c->rope_theta > 0.f))
     return fail(ADADSF_ERR_INVALID_ARG, "norm_eps and rope_theta must be positive");
-  if ((unsigned)c->flags & ~(unsigned)(ADADSF_FLAG_GATE_SIGMOID | ADADSF_FLAG_FOLDED_NORMS))
+  if ((unsigned)c->flags & ~(unsigned)(ADADSF_FLAG_GATE_SIGMOID | ADADSF_FLAG_FOLDED_NORMS | ADADSF_FLAG_GATHERED_QKV))
     return fail(ADADSF_ERR_UNSUPPORTED, "flags 0x%x has unknown bits", (unsigned)c->flags);
   return ADADSF_OK;
 }
 
 bool gated(const adadsf_model_cfg* c) { return ((unsigned)c->flags & ADADSF_FLAG_GATE_SIGMOID) != 0; }
 bool folded(const adadsf_model_cfg* c) { return ((unsigned)c->flags & ADADSF_FLAG_FOLDED_NORMS) != 0; }
+bool gathered_qkv(const adadsf_model_cfg* c) {
+  return folded(c) && ((unsigned)c->flags & ADADSF_FLAG_GATHERED_QKV) != 0;
+}
 
 adadsf_status check_shape(int B, int T, int K) {
   if (B < 0 || T <= 0 || K < 0 || K > T)
@@ -209,7 +212,7 @@ struct Carver {
 };
 
 struct LayerSlots {
-  size_t scores, idx, rows, n1, n2, qkv, vt, attn, ao, act, split, rsel, sq;
+  size_t scores, idx, rows, n1, n2, qkv, vt, attn, ao, act, split, rsel, sq, tsq;
 };
 
 void carve_layer(const adadsf_model_cfg* c, int B, int T, int K, Carver& cv, LayerSlots& s) {
@@ -235,6 +238,9 @@ void carve_layer(const adadsf_model_cfg* c, int B, int T, int K, Carver& cv, Lay
   // per-chunk sums of squares of h (Qwen, bf16, folded norms: the second
   // RMSNorm applied in the gate / up epilogue)
   s.sq = c->dtype == ADADSF_BF16 && c->arch == ADADSF_ARCH_QWEN ? cv.take(M * (c->d / 32) * 4) : 0;
+  // every token's sum of squares from the router (Qwen, bf16, folded norms:
+  // the first RMSNorm applied in the QKV epilogue)
+  s.tsq = c->dtype == ADADSF_BF16 && c->arch == ADADSF_ARCH_QWEN && gathered_qkv(c) ? cv.take((size_t)B * T * 4) : 0;
 }
 
 size_t rope_bytes(const adadsf_model_cfg* c, int T) { return (size_t)T * (c->rotary_dim / 2) * 8; }
@@ -255,6 +261,7 @@ struct LayerBufs {
   int* sync;       // the workspace's synchronisation area
   float* rpart;    // router partial tiles, null on the fp32 path
   float* sq = nullptr;        // [M][d/32] chunk sums of squares of h (folded second RMSNorm)
+  float* tsq = nullptr;       // [B T] sums of squares of the layer input rows (folded first RMSNorm)
   float4* cospart = nullptr;  // [B T][d/32] Eq. 4 partials from the down epilogue (dense, bf16)
 };
 
@@ -379,6 +386,11 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
     CUDA_TRY(cudaEventRecord(dec->fork, dev.stream), "fork the router stream");
     CUDA_TRY(cudaStreamWaitEvent(dec->side, dec->fork, 0), "fork the router stream");
   }
+  // a4 inside the QKV projection (opt-in; bf16 Qwen layers with folded gains
+  // that take the Top-K path): the router also leaves each token's sum of
+  // squares, the projection loads the kept rows of x by row gathers, and its
+  // epilogue scales each row by 1 / rms before the bias and rotary.
+  const bool fuse1 = tc && !dec && !dense && !neox && gathered_qkv(c) && lb.tsq && M > 32LL * dev.num_sms;
   if (!dense || gate || sink) {
     const double rf = 2.0 * BT * c->router_hidden * d;
     const double rb = (double)BT * d * es + (double)c->router_hidden * d * es + BT * 4.0;
@@ -387,7 +399,7 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
     // them when every token is kept
     TRY(launch(sdev, ADADSF_KERNEL_ROUTER, false, rf, rb,
                CALL(tc ? router_tc(x, BT, d, w->router_w1, w->router_b1, w->router_w2, w->router_b2,
-                                   lb.scores, lb.sync, lb.rpart, sdev)
+                                   lb.scores, fuse1 ? lb.tsq : nullptr, lb.sync, lb.rpart, sdev)
                        : router_f32(static_cast<const float*>(x), BT, d, c->router_hidden,
                                     static_cast<const float*>(w->router_w1),
                                     static_cast<const float*>(w->router_b1),
@@ -434,10 +446,11 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
       TRY(launch(dev, ADADSF_KERNEL_TOPK, false, 0, BT * 4.0 + M * 8.0,
                  CALL(topk(lb.scores, B, T, K, lb.idx, lb.rows, dev), "top-k")));
       // a4: gather the kept rows and normalise them (NeoX: LN1 and LN2)
-      TRY(launch(dev, ADADSF_KERNEL_GATHER_NORM, false, 0, Md * es * (neox ? 3 : 2),
-                 CALL(gather_norm(dt, x, lb.rows, M, d, !neox, w->ln1_w, w->ln1_b, w->ln2_w,
-                                  w->ln2_b, c->norm_eps, lb.n1, neox ? lb.n2 : nullptr, dev),
-                      "gather+norm")));
+      if (!fuse1)
+        TRY(launch(dev, ADADSF_KERNEL_GATHER_NORM, false, 0, Md * es * (neox ? 3 : 2),
+                   CALL(gather_norm(dt, x, lb.rows, M, d, !neox, w->ln1_w, w->ln1_b, w->ln2_w,
+                                    w->ln2_b, c->norm_eps, lb.n1, neox ? lb.n2 : nullptr, dev),
+                        "gather+norm")));
     }
     rows = lb.rows;
     pos = lb.idx;
@@ -462,9 +475,18 @@ adadsf_status layer_impl(const adadsf_model_cfg* c, const adadsf_layer_weights* 
   const bool fuse_rope = tc && !dec && (half == 4 || half == 8 || half == 16 || (half > 0 && half % 32 == 0));
   const bool neox_tc = neox && tc;
   {
-    GemmArgs g = linear_args(lb.n1, d, w->w_qkv, M, qkv_dim, d);
+    GemmArgs g = linear_args(fuse1 ? x : lb.n1, d, w->w_qkv, M, qkv_dim, d);
     g.scratch = lb.split;
     g.scratch_bytes = lb.split ? gemm_split_scratch_bytes() : 0;
+    if (fuse1) {
+      g.a_gather = lb.rows;
+      g.a_gather_rows = BT;
+      g.epi.nrm_psum = lb.tsq;
+      g.epi.nrm_rows = lb.rows;
+      g.epi.nrm_nps = 1;
+      g.epi.nrm_d = d;
+      g.epi.nrm_eps = c->norm_eps;
+    }
     g.epi.bias = w->b_qkv;
     g.epi.out = lb.qkv;
     g.epi.ld_out = qkv_dim;
@@ -838,6 +860,7 @@ adadsf_status model_forward_impl(const adadsf_model_cfg* cfg, const adadsf_model
   lb.sync = at<int>(ws, kErrBytes);
   lb.rpart = m.layer.rsel ? at<float>(ws, m.layer.rsel) : nullptr;
   lb.sq = m.layer.sq ? at<float>(ws, m.layer.sq) : nullptr;
+  lb.tsq = m.layer.tsq ? at<float>(ws, m.layer.tsq) : nullptr;
   const size_t xbytes = (size_t)B * T * cfg->d * es;
   int64_t idx_off = 0;
   for (int l = 0; l < cfg->n_layers; ++l) {
@@ -1229,7 +1252,7 @@ adadsf_status adadsf_router_scores(const adadsf_model_cfg* cfg, const adadsf_lay
     // for 128-token tiles split along d
     const bool split = ws_bytes >= kErrBytes + kSyncBytes + router_partial_bytes();
     CUDA_TRY(router_tc(x_dev, n_rows, cfg->d, w->router_w1, w->router_b1, w->router_w2, w->router_b2,
-                       scores_dev, split ? at<int>(ws, kErrBytes) : nullptr,
+                       scores_dev, nullptr, split ? at<int>(ws, kErrBytes) : nullptr,
                        split ? at<float>(ws, kErrBytes + kSyncBytes) : nullptr, dev),
              "router");
     return ADADSF_OK;
@@ -1285,7 +1308,7 @@ adadsf_status adadsf_router_select(const adadsf_model_cfg* cfg, const adadsf_lay
   const int64_t BT = (int64_t)B * T;
   if (cfg->dtype == ADADSF_BF16)
     CUDA_TRY(router_tc(x_dev, BT, cfg->d, w->router_w1, w->router_b1, w->router_w2, w->router_b2,
-                       scores_dev, at<int>(ws, kErrBytes), at<float>(ws, kErrBytes + kSyncBytes), dev),
+                       scores_dev, nullptr, at<int>(ws, kErrBytes), at<float>(ws, kErrBytes + kSyncBytes), dev),
              "router");
   else
     CUDA_TRY(router_f32(static_cast<const float*>(x_dev), BT, cfg->d, cfg->router_hidden,
@@ -1405,6 +1428,7 @@ adadsf_status adadsf_sparse_layer_forward(const adadsf_model_cfg* cfg, const ada
   lb.sync = at<int>(ws, kErrBytes);
   lb.rpart = s.rsel ? at<float>(ws, s.rsel) : nullptr;
   lb.sq = s.sq ? at<float>(ws, s.sq) : nullptr;
+  lb.tsq = s.tsq ? at<float>(ws, s.tsq) : nullptr;
   if (cfg->rotary_dim > 0)
     TRY(launch(dev, ADADSF_KERNEL_ROPE_TABLE, false, 0, rope_bytes(cfg, T),
                CALL(rope_table(at<float2>(ws, rope_off), T, cfg->rotary_dim, cfg->rope_theta, dev),
@@ -1507,6 +1531,7 @@ adadsf_status adadsf_decode_step(const adadsf_model_cfg* cfg, const adadsf_model
   lb.sync = at<int>(ws, kErrBytes);
   lb.rpart = ds.layer.rsel ? at<float>(ws, ds.layer.rsel) : nullptr;
   lb.sq = ds.layer.sq ? at<float>(ws, ds.layer.sq) : nullptr;
+  lb.tsq = ds.layer.tsq ? at<float>(ws, ds.layer.tsq) : nullptr;
   cudaStream_t side = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   const bool has_side = decode_side_stream(dev.stream, &side, &ev_fork, &ev_join);

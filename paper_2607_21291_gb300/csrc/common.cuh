@@ -321,6 +321,18 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const void* tmap,
       "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(cluster_bar)
       : "memory");
 }
+// Row gather (tile::gather4): the box (c0, r0..r3) of a tensor map whose box is
+// one row high brings 4 rows, in that order, to consecutive box-sized lines at
+// dst (the swizzle follows the shared-memory address); completion counted on
+// `cluster_bar`, an mbarrier of either CTA of the pair.
+__device__ __forceinline__ void tma_gather4_pair(uint32_t dst, const void* tmap, int c0, int r0, int r1,
+                                                 int r2, int r3, uint32_t cluster_bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(r0), "r"(r1), "r"(r2), "r"(r3), "r"(cluster_bar)
+      : "memory");
+}
 // Bulk copy of `bytes` (multiple of 16, both addresses 16-byte aligned) from
 // global memory into this CTA's shared memory; completion is counted as
 // transaction bytes on `bar`.

@@ -99,7 +99,7 @@ __global__ void __launch_bounds__(256) gemm_f32_kernel(const SimtDev p) {
 
 cudaError_t gemm_f32(const GemmArgs& a, const Dev& dev) {
   if (a.M <= 0) return cudaSuccess;
-  if (a.K2 > 0 || a.epi.bias2) return cudaErrorInvalidValue;
+  if (a.K2 > 0 || a.epi.bias2 || a.a_gather || a.epi.nrm_psum) return cudaErrorInvalidValue;
   SimtDev p;
   p.A = static_cast<const float*>(a.A); p.lda = a.lda;
   p.W = static_cast<const float*>(a.W); p.W2 = static_cast<const float*>(a.W2); p.ldw = a.ldw;

@@ -109,7 +109,8 @@ struct GemmDev {
   const float* gate;
   const bf16* gbase; int64_t ld_gbase;
   // folded RMSNorm of the A rows (see Epilogue::nrm_psum)
-  const float* nrm_psum; int nrm_nps; float nrm_inv_d, nrm_eps;
+  const float* nrm_psum; const int32_t* nrm_rows; int nrm_nps; float nrm_inv_d, nrm_eps;
+  const int32_t* a_gather;   // A rows by index (gemm_tc2_kernel; see GemmArgs::a_gather)
   // per-chunk sums of squares / Eq. 4 partials of the stored rows
   float* sq_out; int sq_ld;
   float4* cos_out; int cos_ld;
@@ -377,12 +378,14 @@ __device__ __forceinline__ void epi_chunk_store(const GemmDev& p, float* v, cons
 // b' = b cos + a sin. The row's (cos, sin) pairs are loaded 16 at a time (the
 // first 16 of the tile may have been prefetched before the accumulator was
 // ready: tpre), the accumulator 8 columns at a time. These are query / key
-// columns: no activation, residual or transposed copy.
+// columns: no activation, residual or transposed copy. SCALE: the
+// accumulator is first multiplied by rs (the row's folded RMSNorm).
+template <bool SCALE>
 __device__ __forceinline__ void rope_pair(const GemmDev& p, uint32_t tacc, int c, int c2, int bn,
                                           int nb, uint32_t sc, bool has_consts,
                                           const float2* tab_row, bool mvalid, int64_t orow,
                                           const uint4 (&tpre)[2][4], bool use_pre, uint32_t stg,
-                                          int lane) {
+                                          int lane, float rs) {
   const int n0 = nb * bn + c * 32, n2 = nb * bn + c2 * 32;
   const int i0 = n0 % p.rope_hd;
   uint4 pa[4], pb[4];   // the two chunks, bf16
@@ -414,6 +417,10 @@ __device__ __forceinline__ void rope_pair(const GemmDev& p, uint32_t tacc, int c
       for (int j = 0; j < 8; ++j) {
         a[j] = __uint_as_float(ra[j]);
         b[j] = __uint_as_float(rb[j]);
+        if (SCALE) {
+          a[j] *= rs;
+          b[j] *= rs;
+        }
       }
       if (has_consts) {
         float f[4];
@@ -484,7 +491,7 @@ struct EpiPre {
 // accumulator is ready.
 __device__ __forceinline__ float norm_scale(const GemmDev& p, int m) {
   if (!p.nrm_psum || m >= p.M) return 1.f;
-  const float* ps = p.nrm_psum + (int64_t)m * p.nrm_nps;
+  const float* ps = p.nrm_psum + (int64_t)(p.nrm_rows ? p.nrm_rows[m] : m) * p.nrm_nps;
   float sum = 0.f;
   if ((p.nrm_nps & 3) == 0) {
     const float4* p4 = reinterpret_cast<const float4*>(ps);
@@ -539,8 +546,8 @@ __device__ __forceinline__ void epilogue_tile(const GemmDev& p, uint32_t tacc, i
     const bool rot = rope && n0 < p.rope_cols;
     if (rot && p.rope_half >= 32) {
       if ((n0 % p.rope_hd) < p.rope_half && n0 < p.N)   // else done with its partner
-        rope_pair(p, tacc, c, c + p.rope_half / 32, bn, nb, sc, has_consts, tab_row, mvalid, orow,
-                  pre.res, c == c_lo && pre.nt, stg, lane);
+        rope_pair<EXTRA>(p, tacc, c, c + p.rope_half / 32, bn, nb, sc, has_consts, tab_row, mvalid, orow,
+                         pre.res, c == c_lo && pre.nt, stg, lane, rs);
       continue;
     }
     uint32_t r[32];
@@ -671,7 +678,7 @@ __device__ __forceinline__ bool epilogue_role(const GemmDev& P, int m, int nb, i
   tc_fence_after();
   const EpiRed none = {nullptr, 0, 0, 0};
   if (!DUAL && P.rope_tab)
-    epilogue_tile<BN, DUAL, true, false>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none, stg, lane);
+    epilogue_tile<BN, DUAL, true, EXTRA>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none, stg, lane);
   else
     epilogue_tile<BN, DUAL, false, EXTRA>(P, tacc, m, nb, bn, c_lo, c_hi, sc, has_consts, pre, none, stg, lane);
   return true;
@@ -1061,7 +1068,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const EpiRed red = {p.scratch + (size_t)tile * S * BM * BN, S, rank, BN};
     const uint32_t stg = sconst + C::CONST_BYTES + kStgBytes * (warp - 2);
     if (p.rope_tab)   // rotary halves of at most 16 features (one chunk)
-      epilogue_tile<BN, false, true, false>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre, red, stg,
+      epilogue_tile<BN, false, true, EXTRA>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre, red, stg,
                                             lane);
     else
       epilogue_tile<BN, false, false, EXTRA>(p, tacc, m, ti.nb, BN, c_lo, c_hi, sc, has_consts, pre, red, stg,
@@ -1154,7 +1161,67 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const uint32_t full_lead = map_to_cta(full0, 0);
   const uint32_t tempty_lead = map_to_cta(tempty0, 0);
 
-  if (warp == 0) {
+  if (warp == 0 && p.a_gather) {
+    // ------------------------------------------------------------ TMA producer, gathered A
+    // (one problem, one K source). Lane l brings rows 4l .. 4l + 3 of the
+    // CTA's 128-row block, row r of the block being row a_gather[r] of A, by
+    // one row gather per k-block; lane 0 waits for the stage and loads the
+    // weight tile. Rows past M repeat the last one (never stored).
+    int stage = 0;
+    uint32_t phase = 0;
+    int64_t issued = 0;
+    constexpr uint32_t tx = 2 * C::STAGE_BYTES;
+    int pre = 0;
+    if (pair < num_tiles) {
+      const TileInfo ti = tile_info(pair, p, p2, tiles0, 2 * BM);
+      pre = ti.nkb < C::STAGES ? ti.nkb : C::STAGES;
+      if (lane == 0) {
+        for (int kb = 0; kb < pre; ++kb) {
+          if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * kb, tx);
+          tma_load_2d_pair(sB + kb * C::B_BYTES, &tmB, kb * BK, ti.nb * BN + brow_off, full_lead + 8 * kb);
+        }
+      }
+    }
+    pdl_wait();
+    bool first = true;
+    for (int t = pair; t < num_tiles; t += num_pairs) {
+      const TileInfo ti = tile_info(t, p, p2, tiles0, 2 * BM);
+      const int m0 = ti.mb * 2 * BM + (int)rank * BM + 4 * lane;
+      int g[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) g[j] = __ldg(p.a_gather + min(m0 + j, p.M - 1));
+      const int brow0 = ti.nb * BN + brow_off;
+      bool ok = true;
+      for (int kb = 0; kb < ti.nkb; ++kb) {
+        const uint32_t fb = full_lead + 8 * stage;
+        if (!(first && kb < pre)) {
+          int w = 1;
+          if (lane == 0) {
+            w = mbar_wait_bounded(empty0 + 8 * stage, phase ^ 1, abort_flag, p.err, p.timeout_ns);
+            if (w) {
+              if (rank == 0) mbar_arrive_expect_tx(full0 + 8 * stage, tx);
+              tma_load_2d_pair(sB + stage * C::B_BYTES, &tmB, kb * BK, brow0, fb);
+            }
+          }
+          ok = __shfl_sync(0xffffffffu, w, 0) != 0;
+          if (!ok) break;
+        }
+        tma_gather4_pair(sA + stage * C::A_BYTES + lane * 4 * BK * 2, &tmA, kb * BK, g[0], g[1], g[2], g[3], fb);
+        ++issued;
+        if (++stage == C::STAGES) { stage = 0; phase ^= 1; }
+      }
+      first = false;
+      if (!ok) break;
+    }
+    // Drain (even CTA, whose full barriers count both CTAs' copies).
+    if (lane == 0 && rank == 0) {
+      for (int s = 0; s < C::STAGES; ++s) {
+        if (issued <= s) break;
+        const int64_t last = s + ((issued - 1 - s) / C::STAGES) * C::STAGES;
+        mbar_wait_drain(full0 + 8 * s, (uint32_t)((last / C::STAGES) & 1), p.timeout_ns);
+      }
+    }
+  } else if (warp == 0) {
     // ------------------------------------------------------------ TMA producer (both CTAs)
     if (lane == 0) {
       int stage = 0;
@@ -1347,11 +1414,13 @@ bool make_dev(const GemmArgs& a, const Dev& dev, GemmDev& p) {
     p.add_gathered = a.epi.rows ? 1 : 0;
   }
   p.rows = a.epi.rows;
+  p.a_gather = a.a_gather;
   p.out_mapped = a.epi.out_mapped ? 1 : 0;
   p.out = static_cast<bf16*>(a.epi.out); p.ld_out = a.epi.ld_out;
   if (a.epi.nrm_psum) {
-    if (a.epi.rope_tab || a.epi.nrm_d <= 0) return false;
+    if (a.epi.nrm_d <= 0 || a.epi.nrm_nps <= 0) return false;
     p.nrm_psum = a.epi.nrm_psum;
+    p.nrm_rows = a.epi.nrm_rows;
     p.nrm_nps = a.epi.nrm_nps;
     p.nrm_inv_d = 1.f / (float)a.epi.nrm_d;
     p.nrm_eps = a.epi.nrm_eps;
@@ -1400,7 +1469,9 @@ bool make_dev(const GemmArgs& a, const Dev& dev, GemmDev& p) {
 // Tensor maps of one problem: (A, W) and, for two K sources, (A2, W2).
 bool problem_maps(const GemmArgs& a, uint32_t a_rows, uint32_t b_rows, CUtensorMap& ta,
                   CUtensorMap& tb, CUtensorMap* ta2, CUtensorMap* tb2) {
-  if (!make_tmap(&ta, a.A, (uint64_t)a.M, (uint64_t)a.K, (uint64_t)a.lda, a_rows) ||
+  // gathered A: all of A's rows, boxes one row high (four per gather)
+  if (!(a.a_gather ? make_tmap(&ta, a.A, (uint64_t)a.a_gather_rows, (uint64_t)a.K, (uint64_t)a.lda, 1)
+                   : make_tmap(&ta, a.A, (uint64_t)a.M, (uint64_t)a.K, (uint64_t)a.lda, a_rows)) ||
       !make_tmap(&tb, a.W, (uint64_t)a.N, (uint64_t)a.K, (uint64_t)a.ldw, b_rows))
     return false;
   if (a.K2 > 0) {
@@ -1464,6 +1535,7 @@ bool extra_args(const GemmArgs& a) {
 template <int BN, bool DUAL, bool EXTRA>
 cudaError_t launch_x(const GemmArgs& a, const GemmArgs* b, const Dev& dev) {
   using C = TileCfg<BN, DUAL>;
+  if (a.a_gather || (b && b->a_gather)) return cudaErrorInvalidValue;
   static int attr_done[64] = {0};
   int device = 0;
   cudaGetDevice(&device);
@@ -1593,6 +1665,7 @@ int split_override() {
 template <int BN>
 cudaError_t launch_sk(const GemmArgs& a, const Dev& dev, int S) {
   using C = TileCfg<BN, false>;
+  if (a.a_gather) return cudaErrorInvalidValue;
   CUtensorMap tm[4];
   GemmDev p, p2;
   GemmArgs a_full = a;
@@ -1615,6 +1688,8 @@ cudaError_t launch_sk(const GemmArgs& a, const Dev& dev, int S) {
 // the exchange of partial tiles through the L2 (needs a.scratch). CTA pairs (256-row tiles) move half of the
 // weight bytes per SM, the tie-breaker for large M.
 cudaError_t gemm_plain(const GemmArgs& a, const Dev& dev) {
+  // gathered A rows: CTA pairs (the only kernel that gathers)
+  if (a.a_gather) return a.K2 > 0 ? cudaErrorInvalidValue : launch_pair<256, false>(a, nullptr, dev);
   const int num_kb = (a.K + (a.K2 > 0 ? a.K2 : 0) + BK - 1) / BK;
   const int64_t mb128 = (a.M + BM - 1) / BM, mb256 = (a.M + 2 * BM - 1) / (2 * BM);
   const int64_t t128 = mb128 * ((a.N + 127) / 128), t256 = mb128 * ((a.N + 255) / 256);
@@ -1676,6 +1751,7 @@ size_t gemm_split_scratch_bytes() { return (size_t)160 * BM * 256 * 4; }
 
 cudaError_t gemm_bf16(const GemmArgs& a, const Dev& dev) {
   if (a.M <= 0) return cudaSuccess;
+  if (a.a_gather && (a.epi.act == ACT_SWIGLU || a.a_gather_rows <= 0)) return cudaErrorInvalidValue;
   // SwiGLU: 256 x 128 gate/up tiles on CTA pairs when that still gives every
   // pair of SMs at least two tiles.
   if (a.epi.act == ACT_SWIGLU) {
@@ -1688,6 +1764,7 @@ cudaError_t gemm_bf16(const GemmArgs& a, const Dev& dev) {
 }
 
 cudaError_t gemm_bf16_grouped(const GemmArgs& a, const GemmArgs& b, const Dev& dev) {
+  if (a.a_gather || b.a_gather) return cudaErrorInvalidValue;
   if (a.M <= 0 && b.M <= 0) return cudaSuccess;
   if (a.M <= 0) return gemm_bf16(b, dev);
   if (b.M <= 0) return gemm_bf16(a, dev);

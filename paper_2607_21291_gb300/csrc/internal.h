@@ -58,7 +58,9 @@ struct Epilogue {
   // weights; bf16 tensor-core path): acc *= rstd[m] before anything else,
   // rstd = 1 / sqrt(sum_j nrm_psum[m * nrm_nps + j] / nrm_d + nrm_eps); for
   // ACT_SWIGLU both accumulators are scaled.
+  // nrm_rows (or null): the sums of row m are at nrm_psum[nrm_rows[m] * nrm_nps]
   const float* nrm_psum = nullptr;
+  const int32_t* nrm_rows = nullptr;
   int nrm_nps = 0, nrm_d = 0;
   float nrm_eps = 0.f;
   // Sum of squares of each stored 32-column chunk (of the fp32 values before
@@ -87,6 +89,10 @@ struct GemmArgs {
   const void* A2 = nullptr;  int64_t lda2 = 0;    // [M, K2]
   const void* Wk2 = nullptr; int64_t ldwk2 = 0;   // [N, K2]
   int64_t M = 0; int N = 0; int K = 0; int K2 = 0;
+  // Gathered A (bf16, one K source, no second problem): row m of the product
+  // is row a_gather[m] of A, which has a_gather_rows rows (all in range)
+  const int32_t* a_gather = nullptr;
+  int64_t a_gather_rows = 0;
   Epilogue epi;
   // fp32 scratch for splitting small-M products along K (bf16 path); the
   // split is used only when it fits (gemm_split_scratch_bytes covers every case)
@@ -164,10 +170,11 @@ cudaError_t topk(const float* scores, int B, int T, int K, int32_t* idx, int32_t
 // for r < rows. sync: the workspace's synchronisation area (kSyncBytes, zero
 // before the call and left at zero) and partials: router_partial_bytes() of
 // fp32 scratch, both needed to split 128-token tiles along d (either null:
-// no split).
+// no split). tsq (or null): tsq[r] = sum of x[r][j]^2 over j < d, fp32, from
+// the same loads (the first RMSNorm's statistic of every token).
 size_t router_partial_bytes();
 cudaError_t router_tc(const void* x, int64_t rows, int d, const void* w1, const void* b1, const void* w2,
-                      const void* b2, float* scores, int* sync, float* partials, const Dev& dev);
+                      const void* b2, float* scores, float* tsq, int* sync, float* partials, const Dev& dev);
 // Top-K of each sequence's scores fused with gather_norm of the kept rows
 // (out rows b K + i, i-th kept position ascending); also writes idx / rows.
 cudaError_t select_gather_norm(int dtype, const float* scores, int B, int T, int K, const void* x,

@@ -56,7 +56,11 @@ constexpr int kROffBar = kRRing;
 constexpr int kROffMisc = kROffBar + 256;
 constexpr int kROffConst = kROffMisc + 128;
 constexpr int kROffXchg = kROffConst + 2 * kRN * 4;
-constexpr int kRSmem = 1024 + kROffXchg + 2 * kRM * 4;   // with the alignment slack
+constexpr int kROffXsq = kROffXchg + 2 * kRM * 4;
+constexpr int kRSmem = 1024 + kROffXsq + 2 * kRM * 4;   // with the alignment slack
+// One CTA's partial of a split tile: the hidden-unit tile, then the sums of
+// squares of the token rows over its k-blocks (one row of 128 per half).
+constexpr int kRSlot = kRTile + 2 * kRM;
 static_assert((2 * kRStages + 5) * 8 <= 256, "barrier area");
 static_assert(kRMaxCtas * 4 <= (int)kSyncBytes, "tile counters");
 
@@ -69,7 +73,8 @@ struct RouterDev {
   const bf16* w2;
   const bf16* b2;
   float* scores;
-  float* partials;       // [G][2][kRTile]
+  float* tsq;            // [rows] sum of squares of each token row of X, or null
+  float* partials;       // [G][2][kRSlot]
   int* tile_cnt;         // [G]: split tile counted at its first CTA
   int* err;
   unsigned long long timeout_ns;
@@ -109,6 +114,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
   volatile int* ok_flags = misc + 4;   // [2][kREpiWarps]
   float* cst = reinterpret_cast<float*>(smem + kROffConst);   // b1[64], w2[64]
   float* xchg = reinterpret_cast<float*>(smem + kROffXchg);   // [2][128]
+  float* xsq = reinterpret_cast<float*>(smem + kROffXsq);     // [2][128]
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -119,7 +125,8 @@ __global__ void __launch_bounds__(kRThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < kRStages; ++s) {
       mbar_init(full0 + 8 * s, 1);
-      mbar_init(empty0 + 8 * s, 1);
+      // freed by the MMA commit and, with row statistics, each epilogue warp
+      mbar_init(empty0 + 8 * s, p.tsq ? 1 + kREpiWarps : 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(tfull0 + 8 * a, 1);
@@ -234,12 +241,48 @@ __global__ void __launch_bounds__(kRThreads, 1)
     esync();
     int it = 0, seg = 0;
     int64_t u = u0;
+    // row statistics: the ring stage and phase of the next unit
+    int sstage = 0;
+    uint32_t sphase = 0;
+    bool sok = true;
     while (u < u1) {
       const int64_t tile = u / p.nkb;
       const int64_t tstart = tile * p.nkb, tend = tstart + p.nkb;
       const int64_t uend = min(u1, tend);
       const bool whole = u == tstart && uend == tend;
       const int acc = it & 1;
+      // Sum of squares of token row r over this segment's k-blocks: the
+      // thread reads its half of the row's 128-byte swizzled line (16-byte
+      // chunk c sits at c ^ (r % 8)) from each stage, then frees the stage
+      // with its warp.
+      float sq0 = 0.f, sq1 = 0.f;
+      if (p.tsq) {
+        for (int64_t v = u; v < uend; ++v) {
+          if (sok) {
+            int sw = 1;
+            if (lane == 0) sw = mbar_wait_bounded(full0 + 8 * sstage, sphase, abort_flag, p.err, p.timeout_ns);
+            sok = __shfl_sync(0xffffffffu, sw, 0) != 0;
+          }
+          if (sok) {
+            const uint4* line = reinterpret_cast<const uint4*>(smem + sstage * kRA + r * 128);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const uint4 q = line[(4 * half + i) ^ (r & 7)];
+              const uint32_t wv[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+              for (int j = 0; j < 4; ++j) {
+                const float lo = __uint_as_float(wv[j] << 16), hi = __uint_as_float(wv[j] & 0xffff0000u);
+                sq0 = fmaf(lo, lo, sq0);
+                sq1 = fmaf(hi, hi, sq1);
+              }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(empty0 + 8 * sstage);
+          }
+          if (++sstage == kRStages) { sstage = 0; sphase ^= 1; }
+        }
+      }
+      const float sq = sq0 + sq1;
       int w = 1;
       if (lane == 0) w = mbar_wait_bounded(tfull0 + 8 * acc, (it >> 1) & 1, abort_flag, p.err, p.timeout_ns);
       w = __shfl_sync(0xffffffffu, w, 0);
@@ -263,11 +306,12 @@ __global__ void __launch_bounds__(kRThreads, 1)
       bool fin = whole;
       if (!whole) {
         // partial tile: slot 0 holds a CTA's first segment, slot 1 its last
-        float* mine = p.partials + ((size_t)blockIdx.x * 2 + (seg == 0 ? 0 : 1)) * kRTile;
+        float* mine = p.partials + ((size_t)blockIdx.x * 2 + (seg == 0 ? 0 : 1)) * kRSlot;
 #pragma unroll
         for (int j = 0; j < 8; ++j)
           __stcg(reinterpret_cast<float4*>(mine + partial_at(r, half * 32 + 4 * j)),
                  make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]));
+        if (p.tsq) __stcg(mine + kRTile + half * kRM + r, sq);
         esync();
         const int c_lo = unit_owner(tstart, p), c_hi = unit_owner(tend - 1, p);
         if (etid == 0) {
@@ -292,7 +336,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
               for (int j = 0; j < 32; ++j) s[j] += v[j];
             } else {
               const int slot = unit_start(c, p) / p.nkb == tile ? 0 : 1;
-              const float* src = p.partials + ((size_t)c * 2 + slot) * kRTile;
+              const float* src = p.partials + ((size_t)c * 2 + slot) * kRSlot;
 #pragma unroll
               for (int j = 0; j < 8; ++j) {
                 const float4 f = __ldcg(reinterpret_cast<const float4*>(src + partial_at(r, half * 32 + 4 * j)));
@@ -315,10 +359,29 @@ __global__ void __launch_bounds__(kRThreads, 1)
           part[j & 3] += cst[kRN + half * 32 + j] * silu_r(v[j] + cst[half * 32 + j]);
         const float mine = (part[0] + part[1]) + (part[2] + part[3]);
         float* xb = xchg + acc * kRM;
-        if (half == 1) xb[r] = mine;
+        if (half == 1) {
+          xb[r] = mine;
+          if (p.tsq && whole) xsq[acc * kRM + r] = sq;
+        }
         esync();
         const int64_t row = tile * kRM + r;
-        if (half == 0 && row < p.rows) p.scores[row] = (mine + xb[r]) + b2;
+        if (half == 0 && row < p.rows) {
+          p.scores[row] = (mine + xb[r]) + b2;
+          if (p.tsq) {
+            float t = 0.f;
+            if (whole) {
+              t = sq + xsq[acc * kRM + r];
+            } else {
+              // every contributing CTA's two half-row sums, in CTA order
+              for (int c = unit_owner(tstart, p); c <= unit_owner(tend - 1, p); ++c) {
+                const int slot = unit_start(c, p) / p.nkb == tile ? 0 : 1;
+                const float* src = p.partials + ((size_t)c * 2 + slot) * kRSlot + kRTile;
+                t += __ldcg(src + r) + __ldcg(src + kRM + r);
+              }
+            }
+            p.tsq[row] = t;
+          }
+        }
       }
       u = uend;
       ++seg;
@@ -407,10 +470,10 @@ int router_ctas(int64_t n_tiles, int nkb, int sms, bool split) {
 
 }  // namespace
 
-size_t router_partial_bytes() { return (size_t)kRMaxCtas * 2 * kRTile * 4; }
+size_t router_partial_bytes() { return (size_t)kRMaxCtas * 2 * kRSlot * 4; }
 
 cudaError_t router_tc(const void* x, int64_t rows, int d, const void* w1, const void* b1, const void* w2,
-                      const void* b2, float* scores, int* sync, float* partials, const Dev& dev) {
+                      const void* b2, float* scores, float* tsq, int* sync, float* partials, const Dev& dev) {
   if (rows <= 0) return cudaSuccess;
   if (d % kRK != 0 || d <= 0) return cudaErrorInvalidValue;
   const int64_t n_tiles = (rows + kRM - 1) / kRM;
@@ -424,6 +487,7 @@ cudaError_t router_tc(const void* x, int64_t rows, int d, const void* w1, const 
   p.w2 = static_cast<const bf16*>(w2);
   p.b2 = static_cast<const bf16*>(b2);
   p.scores = scores;
+  p.tsq = tsq;
   p.tile_cnt = sync;
   p.partials = partials;
   p.err = dev.err;

@@ -68,6 +68,15 @@ def assert_close(got, ref, tol, what="", elem_tol=None):
     return m, e
 
 
+def row_spread(x, seed, sigma=0.5):
+    """x with each token row scaled by exp(sigma z), z ~ N(0, 1) drawn per row.
+    Rows of N(0, 1) draws all have an rms near 1, so a norm scale that is
+    dropped, or taken from another row, changes them by only ~2 %; with the
+    spread it changes them by tens of percent."""
+    z = S.normal(seed, ("row_spread",), x.shape[:-1] + (1,))
+    return (x * np.exp(np.float32(sigma) * z)).astype(np.float32)
+
+
 def host_layer(shape, seed, layer=0, gain_std=0.1):
     """Seeded layer weights rounded to the storage dtype (float32 arrays)."""
     return {k: S.round_to(v, shape.dtype) for k, v in S.layer_weights(shape, seed, layer, gain_std).items()}

@@ -43,7 +43,7 @@ LAYER_CASES = [
 def run_layer(A, shape, B, T, K, seed=5, x=None, flags=0):
     W = H.host_layer(shape, seed)
     if x is None:
-        x = S.round_to(S.hidden(seed, B, T, shape.d), shape.dtype)
+        x = S.round_to(H.row_spread(S.hidden(seed, B, T, shape.d), seed), shape.dtype)
     td = H.tdtype(shape)
     xd = H.to_dev(x, td)
     idx = torch.full((B, max(K, 1)), -1, dtype=torch.int32, device="cuda")
@@ -231,17 +231,33 @@ FOLD_CASES = [
     (QWEN_SMALL, 1, 96, 96),
     (S.PYTHIA_160M, 2, 200, 77),
     (S.PYTHIA_70M, 1, 128, 64),
+    # Qwen bf16 above 32 kept rows per SM: with FLAG_GATHERED_QKV the first
+    # RMSNorm runs inside the QKV projection (router sums of squares, kept rows
+    # gathered from x); both settings are run
+    (QWEN_SMALL, 3, 3000, 1728),   # M = 5184: the last CTA pair's odd CTA has no row
+    (QWEN_SMALL, 2, 4096, 2500),   # M = 5000: its odd CTA has 8 rows
+    (QWEN_SMALL, 6, 4096, 1000),   # 192 router tiles: whole tiles in two waves
+    (QWEN_SMALL, 1, 16384, 5000),  # one long sequence
 ]
 
 
+def _kinds(A, run):
+    A.adadsf_profile_begin(4096)
+    run()
+    return {r[0] for r in A.adadsf_profile_end(4096)}
+
+
+@pytest.mark.parametrize("gathered", [False, True])
 @pytest.mark.parametrize("shape,B,T,K", FOLD_CASES)
-def test_folded_norms(A, shape, B, T, K):
+def test_folded_norms(A, shape, B, T, K, gathered):
     """adadsf_fold_norms folds the norm gains (and GPT-NeoX norm biases) into
     the projections in place; the layer run with FLAG_FOLDED_NORMS on the
     folded weights matches the oracle on the original weights, and the norm
-    parameters end at 1 / 0."""
+    parameters end at 1 / 0. With FLAG_GATHERED_QKV, the layers that qualify
+    run no gather + norm launch. Token rows carry a spread of scales, so that
+    a row norm dropped or taken from another row shows."""
     W = H.host_layer(shape, 31)
-    x = S.round_to(S.hidden(31, B, T, shape.d), shape.dtype)
+    x = S.round_to(H.row_spread(S.hidden(31, B, T, shape.d), 31), shape.dtype)
     td = H.tdtype(shape)
     wd = A.to_device(W, td)
     A.adadsf_fold_norms(A.make_cfg(shape.replace(n_layers=1)), wd)
@@ -251,10 +267,14 @@ def test_folded_norms(A, shape, B, T, K):
     xd = H.to_dev(x, td)
     idx = torch.full((B, K), -1, dtype=torch.int32, device="cuda")
     sc = torch.empty((B, T), dtype=torch.float32, device="cuda")
-    cfg = A.make_cfg(shape.replace(n_layers=1), A.FLAG_FOLDED_NORMS)
+    flags = A.FLAG_FOLDED_NORMS | (A.FLAG_GATHERED_QKV if gathered else 0)
+    cfg = A.make_cfg(shape.replace(n_layers=1), flags)
     ws = A.workspace(A.adadsf_layer_workspace_size(cfg, B, T, K))
-    A.adadsf_sparse_layer_forward(cfg, wd, xd, K, idx, sc, ws)
+    kinds = _kinds(A, lambda: A.adadsf_sparse_layer_forward(cfg, wd, xd, K, idx, sc, ws))
     assert A.adadsf_sync_check(ws) == A.OK
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    fused = gathered and shape.arch == S.QWEN and shape.dtype == "bf16" and K < T and B * K > 32 * sms
+    assert bool(kinds & {"gather_norm", "topk_gather_norm"}) != fused, kinds
     gi = idx.cpu().numpy()
     W64 = H.f64(W)
     x64 = x.astype(np.float64)

@@ -95,3 +95,48 @@ def test_fullsize_layer(A, key, layer, r):
             H.check_kept_sets(gs[b:b + 1], gi[b:b + 1], O.router_scores(xb, W64), K)
         ref, _, _ = O.sparse_layer_forward(xb, W64, p, K, idx=gi[b:b + 1])
         H.assert_close(got[b:b + 1], ref, H.BF16_TOL, f"{key} layer {layer} K {K} seq {b}")
+
+
+FOLDED_CASES = [("c4", _mid("c4"), 0.5), ("c5", 0, 0.5), ("c5", _mid("c5"), 0.75), ("c5", _last("c5"), 0.25)]
+
+
+@pytest.mark.parametrize("key,layer,r", FOLDED_CASES)
+def test_fullsize_layer_gathered_qkv(A, key, layer, r):
+    """Qwen shapes with folded norm gains and FLAG_GATHERED_QKV at full size:
+    the first RMSNorm runs inside the QKV projection (the router's per-token sums of squares, the
+    kept rows gathered from x by the projection's loads), so no gather + norm
+    launch remains; sampled sequences against the oracle on the unfolded
+    weights, skipped rows bit-identical. Token rows carry a spread of scales,
+    so that a row norm dropped or taken from another row shows."""
+    wl = S.WORKLOADS[key]
+    shape, B, T = wl.shape, wl.B, wl.T
+    K = int(np.floor(r * T))
+    td = H.tdtype(shape)
+    W = _weights(key, layer)
+    x = S.round_to(H.row_spread(S.hidden(11 + layer, B, T, shape.d), 11 + layer), shape.dtype)
+    xd = H.to_dev(x, td)
+    x0 = xd.clone()
+    wd = A.to_device(W, td)
+    A.adadsf_fold_norms(A.make_cfg(shape.replace(n_layers=1)), wd)
+    idx = torch.empty((B, K), dtype=torch.int32, device="cuda")
+    sc = torch.empty((B, T), dtype=torch.float32, device="cuda")
+    cfg = A.make_cfg(shape, A.FLAG_FOLDED_NORMS | A.FLAG_GATHERED_QKV)
+    ws = A.workspace(A.adadsf_layer_workspace_size(cfg, B, T, K))
+    A.adadsf_profile_begin(256)
+    A.adadsf_sparse_layer_forward(cfg, wd, xd, K, idx, sc, ws)
+    kinds = {rec[0] for rec in A.adadsf_profile_end(256)}
+    assert A.adadsf_sync_check(ws) == A.OK
+    assert not kinds & {"gather_norm", "topk_gather_norm"}, kinds
+    keep = torch.zeros((B, T), dtype=torch.bool, device="cuda")
+    keep.scatter_(1, idx.long(), True)
+    assert torch.equal(xd[~keep], x0[~keep])
+    gi = idx.cpu().numpy()
+    gs = sc.cpu().numpy()
+    W64 = H.f64(W)
+    p = O.params_of(shape)
+    got = xd.float().cpu().numpy()
+    for b in (0, B - 1):
+        xb = x[b:b + 1].astype(np.float64)
+        H.check_kept_sets(gs[b:b + 1], gi[b:b + 1], O.router_scores(xb, W64), K)
+        ref, _, _ = O.sparse_layer_forward(xb, W64, p, K, idx=gi[b:b + 1])
+        H.assert_close(got[b:b + 1], ref, H.BF16_TOL, f"{key} folded layer {layer} K {K} seq {b}")
