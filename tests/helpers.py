@@ -47,7 +47,7 @@ def rel_rms(got, ref):
 
 def elem_rel(got, ref):
     """Largest element-wise error, each element's |g - r| over max(|r|, rms(r)):
-    an error is judged against its own element unless that element is smaller
+    an error is measured against its own element unless that element is smaller
     than the tensor's rms (the floor keeps near-zero elements from dividing
     by ~0)."""
     got = np.asarray(got, dtype=np.float64)
