@@ -119,6 +119,23 @@ def test_workspace_sizes(A):
     assert "head_dim" in A.adadsf_last_error()
 
 
+def test_flags_and_their_workspace(A):
+    """FLAG_GATHERED_QKV is accepted with or without FLAG_FOLDED_NORMS; it
+    adds exactly one fp32 sum of squares per token (B T floats, 256-byte
+    aligned) to a bf16 Qwen layer's workspace, and only together with
+    FLAG_FOLDED_NORMS (alone it is ignored); unknown flag bits are refused."""
+    B, T, K = 4, 1000, 500
+    for shape, grows in ((S.QWEN25_1_5B, True), (S.PYTHIA_160M, False)):
+        sizes = {f: A.adadsf_layer_workspace_size(A.make_cfg(shape, f), B, T, K)
+                 for f in (0, A.FLAG_FOLDED_NORMS, A.FLAG_GATHERED_QKV,
+                           A.FLAG_FOLDED_NORMS | A.FLAG_GATHERED_QKV)}
+        assert sizes[A.FLAG_FOLDED_NORMS] == sizes[0] == sizes[A.FLAG_GATHERED_QKV]
+        extra = sizes[A.FLAG_FOLDED_NORMS | A.FLAG_GATHERED_QKV] - sizes[0]
+        assert extra == ((B * T * 4 + 255) // 256 * 256 if grows else 0)
+    with pytest.raises(A.AdadsfError):
+        A.adadsf_layer_workspace_size(A.make_cfg(S.QWEN25_1_5B, 8), B, T, K)
+
+
 def test_argument_errors_precede_launch(A):
     lib = A.lib()
     cfg = A.make_cfg(S.PYTHIA_160M)
