@@ -97,9 +97,11 @@ def case_layer(a, stream):
     for n in ("ln1_w", "ln2_w"):
         w[n] = torch.ones_like(w[n])
     x = torch.randn(B, T, shape.d, generator=g, device="cuda").to(dt)
-    flags = (A.FLAG_FOLDED_NORMS if a.fold else 0) | (A.FLAG_GATE_SIGMOID if a.gate else 0)
+    fold = a.fold or a.gathered
+    flags = ((A.FLAG_FOLDED_NORMS if fold else 0) | (A.FLAG_GATE_SIGMOID if a.gate else 0)
+             | (A.FLAG_GATHERED_QKV if a.gathered else 0))
     cfg = A.make_cfg(shape, flags)
-    if a.fold:
+    if fold:
         A.adadsf_fold_norms(cfg, w, stream)
     ws = A.workspace(A.adadsf_layer_workspace_size(cfg, B, T, K))
     fn = lambda: A.adadsf_sparse_layer_forward(cfg, w, x, K, ws=ws, stream=stream)
@@ -222,6 +224,8 @@ def main():
     ap.add_argument("--profile", action="store_true", help="also report the library's per-launch events")
     ap.add_argument("--fold", action="store_true", help="layer: fold the norms (FLAG_FOLDED_NORMS)")
     ap.add_argument("--gate", action="store_true", help="layer: the score-gated variant")
+    ap.add_argument("--gathered", action="store_true",
+                    help="layer: folded norms and the first RMSNorm inside the QKV projection (FLAG_GATHERED_QKV)")
     ap.add_argument("--graph", type=int, default=0, help="also time R calls replayed from one CUDA graph")
     ap.add_argument("--layers", type=int, default=2, help="decode: layers of the model")
     a = ap.parse_args()
