@@ -23,7 +23,10 @@
 //   warp 1      TMEM (two 64-column accumulators); one thread issues the MMAs
 //   warps 2-9   two per TMEM lane quarter, 32 hidden units each: partial
 //               tiles and the score epilogue (a group of 256 threads on a
-//               named barrier)
+//               named barrier); on request also every token row's sum of
+//               squares (the first RMSNorm's statistic), read from each
+//               stage's token tile before the stage is freed, split tiles'
+//               row sums travelling with their partial tiles
 // Every barrier wait is bounded in time (device error word on give-up).
 #include <algorithm>
 #include <cstdlib>
@@ -262,6 +265,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
             int sw = 1;
             if (lane == 0) sw = mbar_wait_bounded(full0 + 8 * sstage, sphase, abort_flag, p.err, p.timeout_ns);
             sok = __shfl_sync(0xffffffffu, sw, 0) != 0;
+            __syncwarp();   // the other lanes' reads follow lane 0's observation of the stage
           }
           if (sok) {
             const uint4* line = reinterpret_cast<const uint4*>(smem + sstage * kRA + r * 128);
